@@ -1,0 +1,436 @@
+"""Pins of the oracle to facts the paper and the mathematics fix.
+
+Each pin_* function takes an `oracle.Oracle` and raises AssertionError when
+the oracle disagrees with something that does NOT come from re-running the
+oracle's own formula: closed forms, polynomials the quintic Hermite basis
+must reproduce exactly, the Hermite remainder bound on sin(), finite
+differences, symmetries of the descriptor (Sec. II: translation, rotation and
+permutation symmetry), brute-force hand cases, and library matmuls.
+test_oracle_pins.py runs them on the real oracle; test_oracle_mutants.py
+runs them on oracle builds with planted mistakes and expects a failure.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+import workloads as W
+
+
+def _rel(x, ref):
+    x, ref = np.asarray(x, dtype=np.float64), np.asarray(ref, dtype=np.float64)
+    scale = np.max(np.abs(ref))
+    return float(np.max(np.abs(x - ref)) / (scale if scale > 0 else 1.0))
+
+
+def _poly_nodes(o, info, coef):
+    """Node values of p(x) = sum_k coef[k] x^k, its first and second derivative (numpy polyval)."""
+    xs = np.array([o.node_x(info, l) for l in range(info.nint + 1)])
+    P = np.polynomial.Polynomial(coef)
+    return xs, P(xs), P.deriv(1)(xs), P.deriv(2)(xs), P
+
+
+# --------------------------------------------------------------- embedding net
+
+def pin_net_skip_wiring(o):
+    """All weights 0: every layer outputs tanh(bias) plus its skip, so values are hand-computable.
+
+    widths 1-2-4 (both layers double: u = tanh(b) + (v, v)), 1-3-3 (equal: u = tanh(b) + v),
+    1-3-5 (no skip).  d/dx of each output is the number of x's it carries; d2 = 0.
+    """
+    x = 0.37
+    # 1 -> 2 -> 4
+    b1 = np.array([0.2, -0.7])
+    b2 = np.array([0.1, 0.3, -0.4, 0.9])
+    params = np.concatenate([np.zeros(2), b1, np.zeros(8), b2])
+    y, dy, d2y = o.net_eval(params, [1, 2, 4], x)
+    u1 = np.tanh(b1) + x
+    exp = np.tanh(b2) + np.concatenate([u1, u1])
+    assert _rel(y, exp) < 1e-15, ("1-2-4", y, exp)
+    assert np.allclose(dy, 1.0, rtol=0, atol=1e-15) and np.allclose(d2y, 0.0, atol=1e-15)
+    # 1 -> 3 -> 3
+    b1 = np.array([0.5, -0.25, 1.5])
+    b2 = np.array([-1.0, 0.75, 0.05])
+    params = np.concatenate([np.zeros(3), b1, np.zeros(9), b2])
+    y, dy, d2y = o.net_eval(params, [1, 3, 3], x)
+    exp = np.tanh(b2) + np.tanh(b1)  # first layer 1->3: no skip; second 3->3: skip
+    assert _rel(y, exp) < 1e-15, ("1-3-3", y, exp)
+    assert np.allclose(dy, 0.0, atol=1e-15)
+    # 1 -> 3 -> 5 : no skip anywhere, constant output
+    b2 = np.array([0.1, 0.2, 0.3, 0.4, 0.5])
+    params = np.concatenate([np.zeros(3), b1, np.zeros(15), b2])
+    y, dy, _ = o.net_eval(params, [1, 3, 5], x)
+    assert _rel(y, np.tanh(b2)) < 1e-15 and np.allclose(dy, 0.0, atol=1e-15)
+
+
+def pin_net_single_neuron(o):
+    """One tanh neuron: G(x) = tanh(w x + b); values against math.tanh, derivatives against FD of math.tanh."""
+    w, b = 1.7, -0.3
+    for x in (-0.8, 0.0, 0.45, 1.3):
+        y, dy, d2y = o.net_eval(np.array([w, b]), [1, 1], x)
+        # widths 1->1 keep the width: u = tanh(z) + x
+        assert abs(y[0] - (math.tanh(w * x + b) + x)) < 1e-15
+        h = 1e-4
+        f = lambda z: math.tanh(w * z + b) + z  # noqa: E731
+        fd1 = (f(x + h) - f(x - h)) / (2 * h)
+        fd2 = (f(x + h) - 2 * f(x) + f(x - h)) / (h * h)
+        assert abs(dy[0] - fd1) < 1e-7, (dy[0], fd1)
+        assert abs(d2y[0] - fd2) < 1e-5, (d2y[0], fd2)
+
+
+def pin_net_derivatives_fd(o):
+    """Forward-mode G', G'' of a random 1-8-16-32 net against central differences of G and G'."""
+    params = W.net_params(11, [1, 8, 16, 32], 1)[0]
+    h = 1e-5
+    for x in (0.05, 0.4, 0.93):
+        y, dy, d2y = o.net_eval(params, [1, 8, 16, 32], x)
+        yp, dyp, _ = o.net_eval(params, [1, 8, 16, 32], x + h)
+        ym, dym, _ = o.net_eval(params, [1, 8, 16, 32], x - h)
+        assert _rel(dy, (yp - ym) / (2 * h)) < 1e-8
+        assert _rel(d2y, (dyp - dym) / (2 * h)) < 1e-8
+
+
+# ----------------------------------------------------------------- table range
+
+def pin_table_info(o):
+    """Range rules on hand cases: lower/upper snapped outward to the steps, coarse segment to 5x upper."""
+    info = o.table_info(0.0, 1.05)
+    assert (info.lower, info.n0, info.n1) == (0.0, 110, 44)
+    assert abs(info.upper - 1.1) < 1e-15 and abs(info.upper_ext - 5.5) < 1e-14
+    info = o.table_info(-0.237, 0.42)
+    assert abs(info.lower + 0.24) < 1e-15 and abs(info.upper - 0.5) < 1e-15 and info.n0 == 74 and info.n1 == 20
+    # node positions
+    assert o.node_x(info, 0) == info.lower and o.node_x(info, info.n0) == info.upper
+    assert abs(o.node_x(info, 3) - (info.lower + 0.03)) < 1e-15
+    assert abs(o.node_x(info, info.n0 + 2) - (info.upper + 0.2)) < 1e-15
+    assert abs(o.node_x(info, info.nint) - info.upper_ext) < 1e-14
+
+
+def pin_locate(o):
+    """Interval search on hand cases, both segments, both clamps and NaN."""
+    info = o.table_info(0.0, 1.05)  # [0, 1.1) step 0.01, [1.1, 5.5) step 0.1
+    l, t, c = o.locate(info, 0.035)
+    assert (l, c) == (3, False) and abs(t - 0.005) < 1e-15
+    l, t, c = o.locate(info, 0.0)
+    assert (l, c) == (0, False) and t == 0.0
+    l, t, c = o.locate(info, 1.099)
+    assert (l, c) == (109, False) and abs(t - 0.009) < 1e-14
+    l, t, c = o.locate(info, 1.1)
+    assert (l, c) == (110, False) and abs(t) < 1e-15
+    l, t, c = o.locate(info, 2.35)
+    assert (l, c) == (122, False) and abs(t - 0.05) < 1e-14
+    l, t, c = o.locate(info, -0.5)
+    assert (l, t, c) == (0, 0.0, True)
+    l, t, c = o.locate(info, 5.5)
+    assert (l, c) == (153, True) and abs(t - 0.1) < 1e-15
+    l, t, c = o.locate(info, 1e9)
+    assert (l, c) == (153, True)
+    l, t, c = o.locate(info, float("nan"))
+    assert l == 0 and math.isnan(t) and not c
+
+
+# ----------------------------------------------------------------------- table
+
+def pin_table_nodes(o):
+    """Table reproduces y, y', y'' at both ends of every interval (<= 1e-12 relative, max-norm per channel).
+
+    At t = 0 this is exact by construction (f = y, e = y', 2d = y''); at t = Dt it
+    holds only when a, b, c follow the closed forms.  Continuity C2 across
+    intervals follows.
+    """
+    params = W.net_params(21, [1, 25, 50, 100], 1)[0]
+    for step in (0.01, 0.001):
+        info = o.table_info(0.0, 0.45, step, 0.1, 5.0)
+        y, dy, d2y = o.nodes(params, [1, 25, 50, 100], info)
+        tab = o.table_build(y, dy, d2y, info)
+        ref = (y, dy, d2y)
+        for l in list(range(0, info.n0, max(1, info.n0 // 40))) + [info.n0 - 1, info.n0, info.nint - 1]:
+            Dt = info.stride0 if l < info.n0 else info.stride1
+            for order in range(3):
+                v0 = o.poly_eval(tab, l, 0.0, order)
+                v1 = o.poly_eval(tab, l, Dt, order)
+                scale = np.maximum(np.abs(ref[order]).max(axis=0), 1e-300)
+                e0 = np.max(np.abs(v0 - ref[order][l]) / scale)
+                e1 = np.max(np.abs(v1 - ref[order][l + 1]) / scale)
+                assert e0 < 1e-15, (step, l, order, e0)
+                assert e1 < 1e-12, (step, l, order, e1)
+
+
+def pin_table_quintic_exact(o):
+    """A degree-5 polynomial is its own quintic Hermite interpolant: reproduced to rounding everywhere."""
+    rng = np.random.default_rng(5)
+    info = o.table_info(0.0, 0.95, 0.05, 0.1, 3.0)
+    for deg in (0, 1, 3, 5):
+        coef = rng.normal(size=deg + 1)
+        xs, y, dy, d2y, P = _poly_nodes(o, info, coef)
+        tab = o.table_build(y[:, None], dy[:, None], d2y[:, None], info)
+        for l in range(info.nint):
+            Dt = info.stride0 if l < info.n0 else info.stride1
+            for frac in (0.13, 0.5, 0.87):
+                t = frac * Dt
+                v = o.poly_eval(tab, l, t, 0)[0]
+                ref = P(xs[l] + t)
+                assert abs(v - ref) <= 1e-12 * max(1.0, abs(ref)), (deg, l, frac, v, ref)
+                d1 = o.poly_eval(tab, l, t, 1)[0]
+                assert abs(d1 - P.deriv(1)(xs[l] + t)) <= 1e-10 * max(1.0, abs(P.deriv(1)(xs[l] + t)))
+
+
+def pin_table_sin_bound(o):
+    """sin(w x + p): midpoint error within the Hermite remainder bound w^6 Dt^6 / 46080, and order 6.
+
+    f - p = f^(6)(xi)/6! t^3 (t - Dt)^3, largest at t = Dt/2; |f^(6)| <= w^6.
+    Halving Dt divides the error by about 2^6 = 64.
+    """
+    om, ph = 10.0, 0.3
+    errs = []
+    for step in (0.1, 0.05):
+        info = o.table_info(0.0, 1.0, step, step * 10, 5.0)
+        xs = np.array([o.node_x(info, l) for l in range(info.nint + 1)])
+        tab = o.table_build(np.sin(om * xs + ph)[:, None], (om * np.cos(om * xs + ph))[:, None],
+                            (-om * om * np.sin(om * xs + ph))[:, None], info)
+        e = max(abs(o.poly_eval(tab, l, step / 2, 0)[0] - math.sin(om * (xs[l] + step / 2) + ph))
+                for l in range(info.n0))
+        bound = om ** 6 * step ** 6 / 46080.0
+        assert e <= bound * (1 + 1e-6) + 1e-15, (step, e, bound)
+        assert e >= 0.5 * bound, (step, e, bound)  # the bound is attained at the midpoint (sanity)
+        errs.append(e)
+    ratio = errs[0] / errs[1]
+    assert 55.0 < ratio < 70.0, ratio
+
+
+def pin_compressed_vs_net(o):
+    """Table of a real net vs the net itself: error falls ~64x when Dt halves (Sec. III: accuracy vs step)."""
+    params = W.net_params(31, [1, 8, 16, 32], 1)[0]
+    widths = [1, 8, 16, 32]
+    errs = []
+    for step in (0.08, 0.04):
+        info = o.table_info(0.0, 0.8, step, 0.4, 2.0)
+        tab = o.tables(params, widths, info)[0]
+        mids = []
+        for l in range(info.n0):
+            x = o.node_x(info, l) + step / 2
+            g = o.poly_eval(tab, l, step / 2, 0)
+            y, _, _ = o.net_eval(params, widths, x)
+            mids.append(np.max(np.abs(g - y)))
+        errs.append(max(mids))
+    ratio = errs[0] / errs[1]
+    assert 40.0 < ratio < 90.0, (errs, ratio)
+
+
+# ------------------------------------------------------------------- forward
+
+def _poly_table(o, info, coefs):
+    """Table [M][...] whose channel m tabulates polynomial coefs[m] (exact for degree <= 5)."""
+    cols = [_poly_nodes(o, info, c) for c in coefs]
+    y = np.stack([c[1] for c in cols], axis=1)
+    dy = np.stack([c[2] for c in cols], axis=1)
+    d2y = np.stack([c[3] for c in cols], axis=1)
+    return o.table_build(y, dy, d2y, info), [c[4] for c in cols]
+
+
+def pin_fwd_brute_force(o):
+    """One atom, one real neighbour, two padding rows, M = 1, table of p(x) = 1 + 2x - x^3:
+    T[k] = R~[k] p(s) / N_c with N_c = 3, by hand."""
+    info = o.table_info(0.0, 0.9, 0.01, 0.1, 5.0)
+    tab, polys = _poly_table(o, info, [[1.0, 2.0, 0.0, -1.0]])
+    s0 = 0.4321
+    s = np.array([[s0, 0.0, 0.0]])
+    Rt = np.zeros((1, 3, 4))
+    Rt[0, 0] = [s0, 0.3, -0.2, 0.1]
+    T = o.fwd(tab[None], info, s, Rt, np.array([[1]], np.int32), None, np.array([3], np.int32))
+    p = 1 + 2 * s0 - s0 ** 3
+    exp = np.array([s0, 0.3, -0.2, 0.1]) * p / 3.0
+    assert _rel(T[0, :, 0], exp) < 1e-14, (T[0, :, 0], exp)
+
+
+def pin_fwd_constant_G(o):
+    """G == c (constant tables, two types): T[k][m] = c_m * sum over valid rows of R~[k] / N_c."""
+    w = W.tiny(seed=7, nloc=5, nreal=6, sel=9, widths=(1, 4))
+    info = o.table_info(w.s_min, w.s_max)
+    consts = [0.5, -1.25, 2.0, 3.5]
+    tab, _ = _poly_table(o, info, [[c] for c in consts])
+    T = o.fwd(tab[None], info, w.s, w.Rt, w.nvalid, None, w.sel)
+    sumR = np.array([w.Rt[i, :w.nvalid[i, 0]].sum(axis=0) for i in range(w.nloc)])
+    exp = sumR[:, :, None] * np.array(consts)[None, None, :] / w.nnei
+    assert _rel(T, exp) < 1e-14
+
+
+def _small_water(nmol=40):
+    return W.water(seed=13, nmol=nmol, widths=(1, 4, 8, 16), M2=4, sel=(20, 40), rc=4.0, rcs=0.5)
+
+
+def pin_fwd_vs_explicit_G(o):
+    """Fused T equals forming the whole G (every row, padding included) then R~^T G / N_c by matmul.
+
+    Fig. 1(b) against Fig. 1(c): the skip of padded rows changes nothing because their R~ rows are 0.
+    """
+    w = _small_water()
+    info = o.table_info(w.s_min, w.s_max)
+    tabs = o.tables(w.params, w.widths, info)
+    T = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    G = o.embed_rows(tabs, info, w.s, w.atype, w.sel)
+    T2 = np.stack([w.Rt[i].T @ G[i] for i in range(w.nloc)]) / w.nnei
+    assert _rel(T, T2) < 1e-13, _rel(T, T2)
+
+
+def pin_fwd_padding(o):
+    """Skipped padding = processed padding (nvalid = sel on the same zero rows); more zero rows only rescale."""
+    w = _small_water(24)
+    info = o.table_info(w.s_min, w.s_max)
+    tabs = o.tables(w.params, w.widths, info)
+    T = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    full = np.broadcast_to(w.sel, w.nvalid.shape).astype(np.int32)
+    Tf = o.fwd(tabs, info, w.s, w.Rt, full, w.atype, w.sel)
+    assert _rel(Tf, T) < 1e-14
+    # add 5 zero rows to each segment: N_c grows by 10, T * N_c unchanged
+    sel2 = w.sel + 5
+    s2 = np.zeros((w.nloc, int(sel2.sum())))
+    R2 = np.zeros((w.nloc, int(sel2.sum()), 4))
+    s2[:, :w.sel[0]] = w.s[:, :w.sel[0]]
+    s2[:, sel2[0]:sel2[0] + w.sel[1]] = w.s[:, w.sel[0]:]
+    R2[:, :w.sel[0]] = w.Rt[:, :w.sel[0]]
+    R2[:, sel2[0]:sel2[0] + w.sel[1]] = w.Rt[:, w.sel[0]:]
+    T2 = o.fwd(tabs, info, s2, R2, w.nvalid, w.atype, sel2)
+    assert _rel(T2 * sel2.sum(), T * w.nnei) < 1e-14
+
+
+def pin_fwd_symmetries(o):
+    """Permuting valid neighbours of one type leaves T unchanged; rotating (x,y,z) rotates T's last 3 rows."""
+    w = _small_water(24)
+    info = o.table_info(w.s_min, w.s_max)
+    tabs = o.tables(w.params, w.widths, info)
+    T = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    rng = np.random.default_rng(3)
+    s2, R2 = w.s.copy(), w.Rt.copy()
+    for i in range(w.nloc):
+        off = 0
+        for b in range(w.ntypes):
+            nv = w.nvalid[i, b]
+            perm = off + rng.permutation(nv)
+            s2[i, off:off + nv] = w.s[i, perm]
+            R2[i, off:off + nv] = w.Rt[i, perm]
+            off += w.sel[b]
+    Tp = o.fwd(tabs, info, s2, R2, w.nvalid, w.atype, w.sel)
+    assert _rel(Tp, T) < 1e-13
+    Q, _ = np.linalg.qr(rng.normal(size=(3, 3)))
+    R3 = w.Rt.copy()
+    R3[..., 1:] = w.Rt[..., 1:] @ Q.T
+    Tr = o.fwd(tabs, info, w.s, R3, w.nvalid, w.atype, w.sel)
+    assert _rel(Tr[:, 0], T[:, 0]) < 1e-13
+    assert _rel(Tr[:, 1:], np.einsum("ab,nbm->nam", Q, T[:, 1:])) < 1e-13
+
+
+# ---------------------------------------------------------------------- grad
+
+def pin_grad_fd(o):
+    """dE/ds against central differences of L = <dT, T(s)>; dE/dR~ against the exact linear change."""
+    w = _small_water(24)
+    info = o.table_info(w.s_min, w.s_max)
+    tabs = o.tables(w.params, w.widths, info)
+    ds, dRt = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, w.dT)
+    def L(s, R, i):  # <dT_i, T_i>: only atom i depends on its own rows
+        return float(np.sum(w.dT[i] * o.fwd(tabs, info, s, R, w.nvalid, w.atype, w.sel, atoms=[i])[0]))
+    rng = np.random.default_rng(8)
+    h = 1e-6
+    checked = 0
+    for _ in range(12):
+        i = int(rng.integers(w.nloc))
+        b = int(rng.integers(w.ntypes))
+        if w.nvalid[i, b] == 0:
+            continue
+        r = int(w.sel[:b].sum()) + int(rng.integers(w.nvalid[i, b]))
+        sp, sm = w.s.copy(), w.s.copy()
+        sp[i, r] += h
+        sm[i, r] -= h
+        fd = (L(sp, w.Rt, i) - L(sm, w.Rt, i)) / (2 * h)
+        # tolerance: relative 1e-8 plus the rounding noise of L divided by the step
+        Ti = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, atoms=[i])[0]
+        noise = 50 * np.finfo(float).eps * float(np.sum(np.abs(w.dT[i] * Ti))) / h
+        assert abs(ds[i, r] - fd) <= 1e-8 * abs(fd) + noise, (i, r, ds[i, r], fd, noise)
+        k = int(rng.integers(4))
+        Rp = w.Rt.copy()
+        Rp[i, r, k] += 0.5
+        lin = (L(w.s, Rp, i) - L(w.s, w.Rt, i)) / 0.5
+        assert abs(dRt[i, r, k] - lin) <= 1e-10 * max(1.0, abs(lin)), (dRt[i, r, k], lin)
+        checked += 1
+    assert checked >= 6
+
+
+def pin_grad_identities(o):
+    """<dR~, R~> = <dT, T> (T is linear in R~); grad is linear in dT; padding rows get 0; clamped s get ds = 0."""
+    w = _small_water(24)
+    info = o.table_info(w.s_min, w.s_max)
+    tabs = o.tables(w.params, w.widths, info)
+    T = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    ds, dRt = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, w.dT)
+    lhs, rhs = float(np.sum(dRt * w.Rt)), float(np.sum(w.dT * T))
+    assert abs(lhs - rhs) <= 1e-12 * max(1.0, abs(rhs))
+    ds2, dR2 = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, 2.0 * w.dT + 0.5 * w.dT[::-1])
+    ds3, dR3 = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, w.dT[::-1])
+    assert _rel(ds2, 2.0 * ds + 0.5 * ds3) < 1e-13 and _rel(dR2, 2.0 * dRt + 0.5 * dR3) < 1e-13
+    mask = np.zeros(w.s.shape, bool)
+    off = 0
+    for b in range(w.ntypes):
+        mask[:, off:off + w.sel[b]] = np.arange(w.sel[b])[None, :] < w.nvalid[:, b:b + 1]
+        off += w.sel[b]
+    assert np.all(ds[~mask] == 0.0) and np.all(dRt[~mask] == 0.0)
+    assert np.any(ds[mask] != 0.0)
+    # push a few valid rows beyond upper_ext and below lower: their ds is exactly 0, dR~ is not
+    s2 = w.s.copy()
+    rows = np.argwhere(mask)[:6]
+    for q, (i, r) in enumerate(rows):
+        s2[i, r] = info.upper_ext + 1.0 if q % 2 == 0 else info.lower - 1.0
+    ds4, dR4 = o.grad(tabs, info, s2, w.Rt, w.nvalid, w.atype, w.sel, w.dT)
+    for i, r in rows:
+        assert ds4[i, r] == 0.0 and np.any(dR4[i, r] != 0.0)
+
+
+def pin_grad_brute_force(o):
+    """One atom, two real rows and one padding row, M = 2 channels tabulating random quintics on a
+    coarse step (Dt = 0.1, where the t^4, t^5 terms matter): by hand,
+    dE/dR~[j][k] = (1/3) sum_m dT[k][m] p_m(s_j),  dE/ds[j] = (1/3) sum_m (sum_k dT[k][m] R~[j][k]) p_m'(s_j)."""
+    rng = np.random.default_rng(12)
+    info = o.table_info(0.0, 0.95, 0.1, 0.5, 3.0)
+    coefs = [rng.normal(size=6) * 3.0, rng.normal(size=6) * 3.0]
+    tab, polys = _poly_table(o, info, coefs)
+    s = np.array([[0.537, 0.164, 0.0]])
+    Rt = np.zeros((1, 3, 4))
+    Rt[0, 0] = [0.537, 0.2, -0.4, 0.3]
+    Rt[0, 1] = [0.164, -0.1, 0.05, 0.12]
+    dT = rng.normal(size=(1, 4, 2))
+    ds, dRt = o.grad(tab[None], info, s, Rt, np.array([[2]], np.int32), None, np.array([3], np.int32), dT)
+    for j in range(2):
+        p = np.array([P(s[0, j]) for P in polys])
+        dp = np.array([P.deriv(1)(s[0, j]) for P in polys])
+        exp_dR = dT[0] @ p / 3.0
+        exp_ds = float(np.sum((dT[0].T @ Rt[0, j]) * dp)) / 3.0
+        assert _rel(dRt[0, j], exp_dR) < 1e-12, (dRt[0, j], exp_dR)
+        assert abs(ds[0, j] - exp_ds) <= 1e-12 * max(1.0, abs(exp_ds)), (ds[0, j], exp_ds)
+    assert ds[0, 2] == 0.0 and np.all(dRt[0, 2] == 0.0)
+
+
+# ----------------------------------------------------------------- descriptor
+
+def pin_descriptor(o):
+    """D = S (S^<)^T against a library matmul; invariant under rotations and same-type permutations."""
+    w = _small_water(24)
+    info = o.table_info(w.s_min, w.s_max)
+    tabs = o.tables(w.params, w.widths, info)
+    T = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    D = o.descriptor(T, w.M2)
+    ref = np.stack([(T[i].T @ T[i])[:, :w.M2] for i in range(w.nloc)])
+    assert _rel(D, ref) < 1e-14
+    assert _rel(D[:, :w.M2, :], np.transpose(D[:, :w.M2, :], (0, 2, 1))) < 1e-15
+    rng = np.random.default_rng(4)
+    Q, _ = np.linalg.qr(rng.normal(size=(3, 3)))
+    R3 = w.Rt.copy()
+    R3[..., 1:] = w.Rt[..., 1:] @ Q.T
+    D3 = o.descriptor(o.fwd(tabs, info, w.s, R3, w.nvalid, w.atype, w.sel), w.M2)
+    assert _rel(D3, D) < 1e-13
+
+
+ALL_PINS = [pin_net_skip_wiring, pin_net_single_neuron, pin_net_derivatives_fd, pin_table_info, pin_locate,
+            pin_table_nodes, pin_table_quintic_exact, pin_table_sin_bound, pin_compressed_vs_net,
+            pin_fwd_brute_force, pin_fwd_constant_G, pin_fwd_vs_explicit_G, pin_fwd_padding, pin_fwd_symmetries,
+            pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor]

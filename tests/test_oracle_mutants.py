@@ -1,0 +1,63 @@
+"""Plant plausible mistakes in copies of the oracle and check that a pin catches each one (CPU only).
+
+Each mutant is the oracle source with one textual change (a dropped term, a
+wrong sign, a swapped index, a transposed operand), compiled into a
+temporary library.  The real oracle source is never modified.
+"""
+import os
+
+import pytest
+
+import oracle
+import oracle_pins
+
+MUTANTS = [
+    ("a: sign of the y' term", "- 6.0L * (p1 + p0) * Dt", "+ 6.0L * (p1 + p0) * Dt"),
+    ("b: swapped y' weights", "(14.0L * p1 + 16.0L * p0)", "(16.0L * p1 + 14.0L * p0)"),
+    ("c: sign of y''_{l+1}", "(3.0L * q0 - q1)", "(3.0L * q0 + q1)"),
+    ("d = y'' instead of y''/2", "out[3] = (double)(q0 / 2.0L);", "out[3] = (double)(q0);"),
+    ("h = y1 + y0", "ld h = y1 - y0;", "ld h = y1 + y0;"),
+    ("coarse segment uses the fine step", "ld Dt = (ld)(l < in->n0 ? in->stride0 : in->stride1);",
+     "ld Dt = (ld)(in->stride0);"),
+    ("net: interleaved instead of concatenated skip", "u[o] = h + v[o % a];", "u[o] = h + v[o / 2];"),
+    ("net: sign of tanh''", "ld h2 = sech2 * z2 - 2.0L * h * sech2 * z1 * z1;",
+     "ld h2 = sech2 * z2 + 2.0L * h * sech2 * z1 * z1;"),
+    ("net: skip missing on equal width", "u[o] = h + v[o];", "u[o] = h;"),
+    ("range: floor instead of ceil", "out->upper = stride1 * ceil(s_max / stride1);",
+     "out->upper = stride1 * floor(s_max / stride1);"),
+    ("node: coarse nodes at fine step", "return in->upper + (double)(l - in->n0) * in->stride1;",
+     "return in->upper + (double)(l - in->n0) * in->stride0;"),
+    ("locate: ceil instead of floor", "k = (int32_t)floor((x - in->lower) / in->stride0);",
+     "k = (int32_t)ceil((x - in->lower) / in->stride0);"),
+    ("poly: a and b swapped", "return c[0] * t5 + c[1] * t4", "return c[1] * t5 + c[0] * t4"),
+    ("fwd: wrong R~ column", "Ti[k * M + m] += Rt[row * 4 + k] * g;", "Ti[k * M + m] += Rt[row * 4 + (k ^ 1)] * g;"),
+    ("fwd: 1/N_c dropped", "Ti[q] = Ti[q] / (double)nnei;", "Ti[q] = Ti[q];"),
+    ("fwd: type-segment offset dropped", "int64_t row = i * nnei + off[beta] + j;", "int64_t row = i * nnei + j;"),
+    ("grad: g' with 4a t^4", "return 5.0 * c[0] * t4 + 4.0 * c[1] * t3", "return 4.0 * c[0] * t4 + 4.0 * c[1] * t3"),
+    ("grad: ds uses g instead of g'", "dsum += rm * dg;", "dsum += rm * g;"),
+    ("grad: r_m from one R~ column", "rm += dTi[k * M + m] * Rt[row * 4 + k];", "rm += dTi[k * M + m] * Rt[row * 4 + 0];"),
+    ("grad: dR~ uses g'", "dr[k] += dTi[k * M + m] * g;", "dr[k] += dTi[k * M + m] * dg;"),
+    ("grad: padding rows processed",
+     "for (int j = 0; j < nvalid[i * ntypes + beta]; ++j) {\n        int r = off[beta] + j;",
+     "for (int j = 0; j < sel[beta]; ++j) {\n        int r = off[beta] + j;"),
+    ("grad: clamp ignored", "double dg = clamped ? 0.0 : poly_dg(c, t);", "double dg = poly_dg(c, t);"),
+    ("descriptor: wrong k on S^<", "v += Ta[k * M + m] * Ta[k * M + q];", "v += Ta[k * M + m] * Ta[((k + 1) % 4) * M + q];"),
+]
+
+
+@pytest.mark.parametrize("desc,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_mutant_is_caught(desc, old, new, tmp_path):
+    src = open(oracle._SRC).read()
+    assert src.count(old) == 1, f"mutation site not unique or missing: {old!r}"
+    msrc = tmp_path / "mutant.c"
+    msrc.write_text(src.replace(old, new))
+    lib = oracle.build(force=True, src=str(msrc), out=str(tmp_path / "libmutant.so"))
+    o = oracle.Oracle(lib)
+    failures = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(o)
+        except Exception as exc:  # noqa: BLE001 - any failure counts as "caught"
+            failures.append((pin.__name__, type(exc).__name__))
+    assert failures, f"no pin caught the mutant: {desc}"
+    os.remove(lib)
