@@ -1,0 +1,398 @@
+"""Benchmark of the DP Compress tabulate-fusion hot path on GB300.
+
+One step = one pass of the whole hot path over one synthetic batch:
+fused forward T = R~^T G / N_c (dp_tabulate_fusion_fwd), descriptor
+D = S S<^T (dp_descriptor_contract) and the backward from a given dE/dT
+(dp_tabulate_fusion_grad).  The table build (compression) is setup and is
+not timed.  Metric: valid neighbour x channel evaluations per second for
+fwd + grad (each valid (atom, neighbour, channel) triple counts once).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload cu85] [--dtype f64]
+  python bench.py --impl reference ...   # the oracle on the host cores (bounded sample)
+
+N > 1 runs under torch.distributed.run, one rank per GPU; every rank works on
+its own seeded instance of the workload (weak scaling, no collective on the
+data path); the reported time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "tabulate-fusion fwd+grad neighbour·channel evals/s (fp64) and % of roofline"
+UNIT = "evals/s"
+NSM = 152
+SM_MAX_MHZ = 2070.0
+# FP64 / FP32 FMA lanes per SM per clock: GB300 is specified at 1.25 TFLOP/s FP64
+# (2 lanes/clk/SM at 2.07 GHz over 152 SMs) and 128 FP32 lanes/clk/SM.
+FMA_LANES = {"f64": 2, "f32": 128}
+# algorithmic FMAs per valid neighbour x channel
+FMA_PER_EVAL = {"fwd": 9, "grad": 18}
+DESC_FMA_PER_ATOM = lambda M1, M2: 4 * M1 * M2  # noqa: E731
+
+
+def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
+    return NSM * FMA_LANES[dtype] * 2 * mhz * 1e6 / 1e12
+
+
+def workload_label(w) -> str:
+    d = w.describe()
+    return (f"{w.name}: nloc={w.nloc}, sel={d['sel']}, M1={w.M1}, M2={w.M2}, "
+            f"mean valid neighbours={d['mean_valid_neighbours']}")
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu: str):
+        self.idx = gpu
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.idx), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=5)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm), "sm_mhz_min": min(sm)}
+
+
+# --------------------------------------------------------------- native arm
+def run_native(args, rank, world, local_rank):
+    import torch
+
+    import paper_2107_02103_gb300 as dpc
+    import workloads as W
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    dtype = torch.float64 if args.dtype == "f64" else torch.float32
+    npdt = np.float64 if args.dtype == "f64" else np.float32
+    kw = {}
+    if args.workload == "alcumg":
+        kw["pad"] = args.pad
+    w = W.make(args.workload, seed=args.seed + 7919 * rank, **kw)
+    info = dpc.dp_table_info_make(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    model = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, dtype)
+    sel = [int(x) for x in w.sel]
+
+    host = {"s": np.ascontiguousarray(w.s.astype(npdt)), "Rt": np.ascontiguousarray(w.Rt.astype(npdt)),
+            "nvalid": w.nvalid, "atype": w.atype, "dT": np.ascontiguousarray(w.dT.astype(npdt))}
+    d = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
+    T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
+    D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
+    ds = torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev)
+    dRt = torch.empty((w.nloc, w.nnei, 4), dtype=dtype, device=dev)
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 256 MiB > 126 MiB L2
+    stream = torch.cuda.current_stream(dev)
+
+    def step(ev=None):
+        if ev:
+            ev[0].record(stream)
+        dpc.dp_tabulate_fusion_fwd(model.table, info, d["s"], d["Rt"], d["nvalid"], d["atype"], sel, out=T)
+        if ev:
+            ev[1].record(stream)
+        dpc.dp_descriptor_contract(T, w.M2, out=D)
+        if ev:
+            ev[2].record(stream)
+        dpc.dp_tabulate_fusion_grad(model.table, info, d["s"], d["Rt"], d["nvalid"], d["atype"], sel, d["dT"],
+                                    out=(ds, dRt))
+        if ev:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize(dev)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
+    clocks = ClockSampler(vis[local_rank] if local_rank < len(vis) else str(local_rank))
+    barrier()
+    torch.cuda.synchronize(dev)
+    if rank == 0:
+        clocks.start()
+    t_wall0 = time.perf_counter()
+    for k in range(args.steps):
+        flush.zero_()  # evict the previous step's data from L2 (outside the timed events)
+        step(evs[k])
+    torch.cuda.synchronize(dev)
+    t_wall = time.perf_counter() - t_wall0
+    barrier()
+    clk = clocks.stop() if rank == 0 else None
+
+    step_ms = [e[0].elapsed_time(e[3]) for e in evs]
+    k_ms = {"fwd": [e[0].elapsed_time(e[1]) for e in evs], "descriptor": [e[1].elapsed_time(e[2]) for e in evs],
+            "grad": [e[2].elapsed_time(e[3]) for e in evs]}
+    total_s = sum(step_ms) / 1e3
+    if world > 1:
+        t = torch.tensor([total_s], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_s = float(t.item())
+        ev_all = torch.tensor([float(w.evals)], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(ev_all)
+        evals_all = float(ev_all.item())
+    else:
+        evals_all = float(w.evals)
+    value = evals_all * args.steps / total_s
+
+    # ---- end to end through the public API: pinned host inputs -> device -> path -> host results
+    e2e = None if args.no_e2e else measure_e2e(args, host, d, dict(T=T, D=D, ds=ds, dRt=dRt), step, stream, dev,
+                                                world, barrier, evals_all)
+    if rank != 0:
+        return None
+    return report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall)
+
+
+def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_all):
+    import torch
+    pin = {k: torch.from_numpy(v).pin_memory() for k, v in host.items()}
+    outs_h = {k: torch.empty(t.shape, dtype=t.dtype).pin_memory() for k, t in outs.items()}
+    h2d = sum(v.numel() * v.element_size() for v in pin.values())
+    d2h = sum(v.numel() * v.element_size() for v in outs_h.values())
+
+    def e2e_step():
+        for k, v in pin.items():
+            d[k].copy_(v, non_blocking=True)
+        step()
+        for k, t in outs.items():
+            outs_h[k].copy_(t, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_s = e0.elapsed_time(e1) / 1e3
+    if world > 1:
+        t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    barrier()
+    return {"value": evals_all * args.steps / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h}
+
+
+def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall):
+    value = evals_all * args.steps / total_s
+    # ---- roofline of the dominant kernel (FMA pipe of the path's dtype)
+    mean = {k: sum(v) / len(v) for k, v in k_ms.items()}
+    flops = {"fwd": 2.0 * FMA_PER_EVAL["fwd"] * w.evals, "grad": 2.0 * FMA_PER_EVAL["grad"] * w.evals,
+             "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
+    pk = peak_tflops(args.dtype)
+    kernels = {k: {"ms": round(mean[k], 4), "share": round(mean[k] / sum(mean.values()), 4),
+                   "tflops": round(flops[k] / (mean[k] * 1e-3) / 1e12, 4),
+                   "frac": round(flops[k] / (mean[k] * 1e-3) / 1e12 / pk, 4)} for k in mean}
+    dom = max(mean, key=mean.get)
+    achieved = flops[dom] / (mean[dom] * 1e-3) / 1e12
+    path_tflops = (flops["fwd"] + flops["grad"]) / ((mean["fwd"] + mean["grad"]) * 1e-3) / 1e12
+    roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
+                "frac": round(achieved / pk, 4), "traffic": None, "kernel": f"dp_tabulate_fusion_{dom}",
+                "peak_basis": (f"FP{64 if args.dtype == 'f64' else 32} FMA pipe: {NSM} SMs x "
+                               f"{FMA_LANES[args.dtype]} lanes/clk x 2 flop x {SM_MAX_MHZ:.0f} MHz"),
+                "fwd_grad_frac": round(path_tflops / pk, 4)}
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": sum(step_ms) / len(step_ms), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": args.dtype, "data": "synthetic",
+        "config": {"workload": workload_label(w), "parallelism": f"replicas x{world} (independent seeded instances)",
+                   "step": "fwd + descriptor + grad", "l2": "flushed between steps (256 MiB write)",
+                   "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4)},
+        "atoms_per_s": w.nloc * world * args.steps / total_s,
+        "roofline": roofline,
+        "kernels": kernels,
+        "e2e": e2e,
+        "gpu_launches": 3 * args.steps * world,
+        "clocks": clk,
+        "wall_s_timed_region": round(t_wall, 4),
+    }
+    if world == 1 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(w, args.dtype, args.cpu_seconds)
+    return out
+
+
+# ------------------------------------------------------------- oracle timing
+def _oracle_pass(o, tabs, info, w, atoms, r):
+    s, Rt, dT = r(w.s), r(w.Rt), r(w.dT)
+    T = o.fwd(tabs, info, s, Rt, w.nvalid, w.atype, w.sel, atoms=atoms)
+    o.descriptor(T, w.M2)
+    o.grad(tabs, info, s, Rt, w.nvalid, w.atype, w.sel, dT, atoms=atoms)
+
+
+def _oracle_setup(w, dtype):
+    import oracle
+    o = oracle.default()
+    info = o.table_info(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    tabs = o.tables(w.params, w.widths, info)
+    r = (lambda a: a)
+    if dtype == "f32":
+        tabs = tabs.astype(np.float32).astype(np.float64)
+        r = lambda a: a.astype(np.float32).astype(np.float64)  # noqa: E731
+    return o, info, tabs, r
+
+
+def _cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def _calibrate(o, info, tabs, w, r, target_s):
+    """Atoms per oracle pass so one pass takes about target_s seconds."""
+    n = min(w.nloc, 64)
+    t0 = time.perf_counter()
+    _oracle_pass(o, tabs, info, w, np.arange(n), r)
+    dt = max(time.perf_counter() - t0, 1e-4)
+    return int(max(1, min(w.nloc, n * target_s / dt)))
+
+
+def cpu_baseline(w, dtype, target_s):
+    """The oracle, as it stands, on all host cores: repeated passes over (a prefix of) the same workload
+    until about target_s seconds of CPU work have run."""
+    o, info, tabs, r = _oracle_setup(w, dtype)
+    n = _calibrate(o, info, tabs, w, r, target_s)
+    atoms = np.arange(n)
+    ev = int(w.nvalid[:n].astype(np.int64).sum()) * w.M1
+    reps, t0 = 0, time.perf_counter()
+    while True:
+        _oracle_pass(o, tabs, info, w, atoms, r)
+        reps += 1
+        dt = time.perf_counter() - t0
+        if dt >= target_s:
+            break
+    return {"value": reps * ev / dt, "unit": UNIT, "cores": _cores(), "kind": "oracle",
+            "sample": (f"{reps} pass(es) of fwd + descriptor + grad over the first {n} of {w.nloc} atoms of "
+                       f"{w.name} ({reps * ev} evals in {dt:.1f} s)")}
+
+
+def run_reference(args, rank, world):
+    """Reference arm: the oracle on the host cores, one bounded sample of the workload per step."""
+    if rank != 0:
+        return None
+    import workloads as W
+    kw = {"pad": args.pad} if args.workload == "alcumg" else {}
+    w = W.make(args.workload, seed=args.seed, **kw)
+    o, info, tabs, r = _oracle_setup(w, args.dtype)
+    per_step = max(0.5, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
+    n = _calibrate(o, info, tabs, w, r, per_step)
+    atoms = np.arange(n)
+    for _ in range(args.warmup):
+        _oracle_pass(o, tabs, info, w, atoms, r)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        _oracle_pass(o, tabs, info, w, atoms, r)
+    dt = time.perf_counter() - t0
+    ev = int(w.nvalid[:n].astype(np.int64).sum()) * w.M1
+    value = ev * args.steps / dt
+    sample = f"first {n} of {w.nloc} atoms of {w.name} per step (fwd + descriptor + grad, {ev} evals)"
+    return {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": args.dtype, "data": "synthetic", "impl": "reference",
+            "config": {"workload": workload_label(w), "parallelism": "host cores (oracle)",
+                       "step": "fwd + descriptor + grad on a bounded atom sample"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": _cores(), "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "gpu_launches": 0}
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--workload", default="cu85", choices=["tiny", "cu85", "cugeo", "water", "alcumg", "water_large"])
+    ap.add_argument("--pad", type=float, default=0.3, help="alcumg padding fraction")
+    ap.add_argument("--dtype", choices=["f64", "f32"], default="f64")
+    ap.add_argument("--seed", type=int, default=2)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if world != args.gpus:
+        print(f"warning: --gpus {args.gpus} but WORLD_SIZE={world}", file=sys.stderr)
+    if args.impl == "reference":
+        out = run_reference(args, rank, world)
+    else:
+        if world > 1:
+            import torch
+            torch.cuda.set_device(local_rank)
+            torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+        out = run_native(args, rank, world, local_rank)
+        if world > 1:
+            import torch
+            torch.distributed.destroy_process_group()
+    if out is not None:
+        print(json.dumps(out), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,193 @@
+/*
+ * dp_compress.h -- C ABI of the GB300 (sm_103a) DP Compress tabulate-fusion library.
+ *
+ * The library implements the compressed single-atom workflow of DP Compress
+ * (Lu et al., arXiv 2107.02103, Sec. II "Methods"): the embedding net G(s) is
+ * replaced by piecewise fifth-order polynomials on a uniform grid, and the
+ * product S_i = G_i^T R~_i (here T_i = S_i^T / N_c, 4 x M) is formed in one
+ * fused pass that never stores G_i and skips padded neighbour rows.
+ *
+ * Conventions shared by every entry point
+ *   - Every pointer argument to a *_f64 / *_f32 compute call is DEVICE memory
+ *     allocated and owned by the caller, unless marked "host".  The library
+ *     allocates nothing and keeps no pointer after returning.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream).  Calls only ENQUEUE work on it; they never synchronise.  A
+ *     non-zero status means nothing was enqueued, except DP_ERR_CUDA from a
+ *     failed launch.  Faults during execution surface at the caller's next
+ *     synchronisation on that stream.
+ *   - Outputs are fully overwritten (padding rows included); nothing needs to
+ *     be zeroed beforehand.  Inputs and outputs must not overlap.
+ *   - Arrays are C-contiguous (row-major) in the layouts given per argument.
+ *     Device pointers must be 16-byte aligned (any cudaMalloc / torch
+ *     allocation is).
+ *   - Return value: DP_OK (0) or a negative dp_status; dp_last_error()
+ *     then describes the failure (per calling thread).
+ *
+ * Notation: nloc atoms, ntypes atom types, sel[b] rows reserved for
+ * neighbours of type b, nnei = N_c = sum_b sel[b] rows per atom; rows of
+ * type b occupy [off_b, off_b + sel[b]) with off_b = sum_{c<b} sel[c]; the
+ * first nvalid[i][b] of them are real neighbours, the rest are zero padding
+ * (Sec. II: neighbours sorted by type, then distance; missing rows are 0).
+ * M1 = M embedding channels, M2 = M' < M leading channels of the descriptor.
+ * A type pair (alpha, beta) = (centre type, neighbour type) has its own table
+ * at index alpha * ntypes + beta.
+ */
+#ifndef DP_COMPRESS_H
+#define DP_COMPRESS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DP_MAX_TYPES 8     /* ntypes <= DP_MAX_TYPES                         */
+#define DP_MAX_M1 256      /* fused forward supports M1 <= DP_MAX_M1          */
+#define DP_MAX_WIDTH 1024  /* embedding-net layer width limit                */
+#define DP_MAX_LAYERS 8    /* embedding-net depth limit                      */
+
+/*
+ * Table range (Sec. II: the domain of the embedding input is cut into equal
+ * intervals; its bounds come from a scan of the data, the upper bound
+ * covering the largest value).  Fine segment [lower, upper) with step
+ * stride0, coarse extrapolation segment [upper, upper_ext) with step stride1.
+ * Derived: n0 = (upper - lower) / stride0 and n1 = (upper_ext - upper) /
+ * stride1, both integral within 1e-9; nint = n0 + n1 intervals; nodes
+ * x_l = lower + l*stride0 (l < n0), x_n0 = upper, x_{n0+k} = upper + k*stride1.
+ */
+typedef struct dp_table_info {
+  double lower;
+  double upper;
+  double upper_ext;
+  double stride0;
+  double stride1;
+} dp_table_info;
+
+typedef enum dp_status {
+  DP_OK = 0,
+  DP_ERR_NULL = -1,        /* a required pointer is NULL                        */
+  DP_ERR_SHAPE = -2,       /* a size is negative, inconsistent or too large     */
+  DP_ERR_TABLE_INFO = -3,  /* table range not positive / not integral in steps  */
+  DP_ERR_CUDA = -4,        /* a CUDA launch failed (message has the CUDA error) */
+  DP_ERR_UNSUPPORTED = -5  /* outside the limits above (M1, ntypes, width)      */
+} dp_status;
+
+/* Message for the last non-OK status returned on the calling thread ("" if none).
+   The string stays valid until the next library call on that thread. */
+const char *dp_last_error(void);
+
+/*
+ * Host-only.  Table range from the data range [s_min, s_max] (Sec. II, the
+ * range is set by scanning the data; the upper bound covers its maximum):
+ *   lower = 0 if s_min >= 0 else stride0 * floor(s_min / stride0)
+ *   upper = stride1 * ceil(s_max / stride1),  upper_ext = ext * upper.
+ * Requires stride0 > 0, stride1 > 0, stride1/stride0 integral, ext >= 1,
+ * s_max > 0, s_min <= s_max.  Writes *out (host).  DP_ERR_TABLE_INFO otherwise.
+ */
+int dp_table_info_make(double s_min, double s_max, double stride0, double stride1, double ext,
+                       dp_table_info *out);
+
+/* Host-only.  Validates *info and writes n0, n1 (host) -- see dp_table_info. */
+int dp_table_info_sizes(const dp_table_info *info, int32_t *n0, int32_t *n1);
+
+/*
+ * Embedding net at the table nodes (Sec. II: the value y_l = G_m(x_l) and the
+ * derivatives y'_l, y''_l at every interpolation point, which the paper notes
+ * can be evaluated efficiently).  Net of `nlayer` layers with widths
+ * widths[0..nlayer] (host array, widths[0] == 1, widths[nlayer] == M1): layer
+ * l maps v (width a) to u (width b) by z = v W_l + b_l, h = tanh(z) and
+ *   u = h + v (b == a),  u = h + (v, v) (b == 2a),  u = h (otherwise).
+ *   params  [npair][P] f64, per pair and layer W_l [a][b] row-major then b_l [b],
+ *           P = sum_l (a_l b_l + b_l).
+ *   y, dy, d2y  [npair][nint + 1][M1] f64 outputs: G, dG/dx, d2G/dx2 at x_l.
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (npair < 1, widths[0] != 1),
+ * DP_ERR_UNSUPPORTED (nlayer > DP_MAX_LAYERS, width > DP_MAX_WIDTH),
+ * DP_ERR_TABLE_INFO, DP_ERR_CUDA.
+ */
+int dp_embedding_net_nodes_f64(const double *params, const int32_t *widths, int nlayer, int npair,
+                               const dp_table_info *info, double *y, double *dy, double *d2y, void *stream);
+
+/*
+ * Quintic Hermite table (Sec. II: on interval l, g_m^l(t) = a t^5 + b t^4 +
+ * c t^3 + d t^2 + e t + f with t = x - x_l, and the closed forms of a..f
+ * from (y, y', y'') at x_l and x_{l+1}, h = y_{l+1} - y_l, Dt = x_{l+1} - x_l).
+ * The brackets of a, b, c are evaluated in double-double arithmetic (they
+ * cancel to O(Dt^5) relative) and rounded once.
+ *   y, dy, d2y  [npair][nint + 1][M1] f64 node values (device).
+ *   table       [npair][nint][M1][6] (a, b, c, d, e, f), f64 or rounded to f32.
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (npair < 1, M1 < 1), DP_ERR_TABLE_INFO,
+ * DP_ERR_CUDA.
+ */
+int dp_table_build_f64(const double *y, const double *dy, const double *d2y, int npair, int M1,
+                       const dp_table_info *info, double *table, void *stream);
+int dp_table_build_f32(const double *y, const double *dy, const double *d2y, int npair, int M1,
+                       const dp_table_info *info, float *table, void *stream);
+
+/*
+ * Fused tabulated embedding + contraction, forward (Sec. II, kernel fusion:
+ * the column of G_i^T for neighbour j is evaluated from the table in
+ * registers and immediately multiplied into R~_i, only for valid j):
+ *   T[i][k][m] = (1/nnei) * sum_b sum_{j < nvalid[i][b]} R~[i][off_b + j][k] * g_m(s[i][off_b + j])
+ * with g_m the table of pair (atype[i], b).  Interval search: s in [lower,
+ * upper) uses l = floor((s - lower)/stride0), s in [upper, upper_ext) uses
+ * n0 + floor((s - upper)/stride1); s < lower evaluates the first node, s >=
+ * upper_ext the last node; NaN s gives NaN in that atom's T.
+ *   table   [npair][nint][M1][6] (from dp_table_build_*), npair = ntypes^2
+ *   s       [nloc][nnei]      embedding input per row
+ *   Rt      [nloc][nnei][4]   environment-matrix rows
+ *   nvalid  [nloc][ntypes] int32, real rows per type segment; entries are
+ *           clamped into [0, sel[b]] (rows beyond are never read);
+ *           NULL = every row valid
+ *   atype   [nloc] int32 centre type, clamped into [0, ntypes); NULL = type 0
+ *   sel     [ntypes] int32 HOST array; nnei must equal sum(sel)
+ *   T       [nloc][4][M1] output
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (nloc < 0, nnei < 1, sum(sel) != nnei,
+ * M1 < 1, table larger than 2^31 elements), DP_ERR_UNSUPPORTED (ntypes >
+ * DP_MAX_TYPES, M1 > DP_MAX_M1), DP_ERR_TABLE_INFO, DP_ERR_CUDA.  nloc == 0
+ * enqueues nothing, reads no device pointer (they may be NULL) and returns
+ * DP_OK once the sizes and the table info are valid.
+ */
+int dp_tabulate_fusion_fwd_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+                               const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                               const int32_t *sel, int M1, double *T, void *stream);
+int dp_tabulate_fusion_fwd_f32(const float *table, const dp_table_info *info, const float *s, const float *Rt,
+                               const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                               const int32_t *sel, int M1, float *T, void *stream);
+
+/*
+ * Backward of the fused forward (Sec. II: the compressed model serves both
+ * the forward and the backward propagation, which yields forces and virials).
+ * Given dT = dE/dT_i:
+ *   dRt[i][row][k] = (1/nnei) * sum_m dT[i][k][m] * g_m(s_row)
+ *   ds[i][row]     = (1/nnei) * sum_m (sum_k dT[i][k][m] * R~[i][row][k]) * g'_m(s_row)
+ * for valid rows; g' = 0 where s was clamped to an end node; padding rows
+ * get ds = 0 and dRt = 0.  When s is the first column of R~ the total
+ * derivative for that column is ds + dRt[..][0].
+ *   dT   [nloc][4][M1] input;  ds [nloc][nnei], dRt [nloc][nnei][4] outputs.
+ *   Other arguments, limits and errors as dp_tabulate_fusion_fwd_*.
+ */
+int dp_tabulate_fusion_grad_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+                                const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                const int32_t *sel, int M1, const double *dT, double *ds, double *dRt,
+                                void *stream);
+int dp_tabulate_fusion_grad_f32(const float *table, const dp_table_info *info, const float *s, const float *Rt,
+                                const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                const int32_t *sel, int M1, const float *dT, float *ds, float *dRt, void *stream);
+
+/*
+ * Descriptor (Sec. II): with S_i = T_i^T (M1 x 4) and S_i^< its first M2
+ * rows, D_i = S_i (S_i^<)^T, i.e. D[i][m][n] = sum_k T[i][k][m] * T[i][k][n].
+ *   T [nloc][4][M1] input,  D [nloc][M1][M2] output.
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (nloc < 0, M1 < 1, M2 < 1, M2 > M1),
+ * DP_ERR_UNSUPPORTED (M1 > 4096), DP_ERR_CUDA.  nloc == 0 returns DP_OK
+ * without reading T or D.
+ */
+int dp_descriptor_contract_f64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream);
+int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, float *D, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DP_COMPRESS_H */

@@ -1,0 +1,239 @@
+"""GB300 (sm_103a) DP Compress tabulate-fusion library: thin Python binding.
+
+Every function here has the name of a C entry point in include/dp_compress.h
+and only marshals arguments: it checks torch tensors (device, dtype,
+contiguity, shape), passes their data pointers and the current CUDA stream,
+and raises on a non-OK status.  All arithmetic runs in the CUDA kernels of
+libdpcompress.so; there is no CPU fallback -- importing this package fails
+if the library has not been built (see build.py).
+
+Calls are asynchronous on torch.cuda.current_stream() like any CUDA op.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libdpcompress.so")
+
+if not os.path.exists(LIB_PATH):
+    raise ImportError(f"{LIB_PATH} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'` "
+                      "(or paper_2107_02103_gb300/build.py); this package has no CPU fallback")
+
+_lib = ctypes.CDLL(LIB_PATH)
+
+DP_OK, DP_ERR_NULL, DP_ERR_SHAPE, DP_ERR_TABLE_INFO, DP_ERR_CUDA, DP_ERR_UNSUPPORTED = 0, -1, -2, -3, -4, -5
+DP_MAX_TYPES, DP_MAX_M1, DP_MAX_WIDTH, DP_MAX_LAYERS = 8, 256, 1024, 8
+
+
+class dp_table_info(ctypes.Structure):
+    """Table range (mirror of the C struct): fine [lower, upper) step stride0, coarse [upper, upper_ext) step stride1."""
+    _fields_ = [("lower", ctypes.c_double), ("upper", ctypes.c_double), ("upper_ext", ctypes.c_double),
+                ("stride0", ctypes.c_double), ("stride1", ctypes.c_double)]
+
+    def __repr__(self):
+        return (f"dp_table_info(lower={self.lower!r}, upper={self.upper!r}, upper_ext={self.upper_ext!r}, "
+                f"stride0={self.stride0!r}, stride1={self.stride1!r})")
+
+
+class DPError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"[{code}] {msg}")
+        self.code = code
+
+
+_P = ctypes.c_void_p
+_I32, _I64, _D = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+_INFO = ctypes.POINTER(dp_table_info)
+_SIGS = {
+    "dp_last_error": ([], ctypes.c_char_p),
+    "dp_table_info_make": ([_D, _D, _D, _D, _D, _INFO], ctypes.c_int),
+    "dp_table_info_sizes": ([_INFO, ctypes.POINTER(_I32), ctypes.POINTER(_I32)], ctypes.c_int),
+    "dp_embedding_net_nodes_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _INFO, _P, _P, _P, _P], ctypes.c_int),
+    "dp_table_build_f64": ([_P, _P, _P, ctypes.c_int, ctypes.c_int, _INFO, _P, _P], ctypes.c_int),
+    "dp_table_build_f32": ([_P, _P, _P, ctypes.c_int, ctypes.c_int, _INFO, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
+                                    _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
+                                    _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
+                                     _P, _P, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
+                                     _P, _P, _P, _P], ctypes.c_int),
+    "dp_descriptor_contract_f64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_descriptor_contract_f32": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+}
+for _name, (_args, _res) in _SIGS.items():
+    _fn = getattr(_lib, _name)
+    _fn.argtypes = _args
+    _fn.restype = _res
+
+
+def dp_last_error() -> str:
+    return _lib.dp_last_error().decode()
+
+
+def _check(rc: int):
+    if rc != DP_OK:
+        raise DPError(rc, dp_last_error())
+
+
+def _stream(t: torch.Tensor):
+    return ctypes.c_void_p(torch.cuda.current_stream(t.device).cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _dev(t: torch.Tensor, name: str, dtype=None, shape=None):
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t
+
+
+def _suffix(dtype) -> str:
+    if dtype == torch.float64:
+        return "f64"
+    if dtype == torch.float32:
+        return "f32"
+    raise TypeError(f"unsupported dtype {dtype}")
+
+
+def dp_table_info_make(s_min: float, s_max: float, stride0: float = 0.01, stride1: float = 0.1,
+                       ext: float = 5.0) -> dp_table_info:
+    info = dp_table_info()
+    _check(_lib.dp_table_info_make(float(s_min), float(s_max), float(stride0), float(stride1), float(ext),
+                                   ctypes.byref(info)))
+    return info
+
+
+def dp_table_info_sizes(info: dp_table_info) -> tuple[int, int]:
+    n0, n1 = _I32(), _I32()
+    _check(_lib.dp_table_info_sizes(ctypes.byref(info), ctypes.byref(n0), ctypes.byref(n1)))
+    return int(n0.value), int(n1.value)
+
+
+def dp_embedding_net_nodes(params: torch.Tensor, widths, info: dp_table_info, out=None):
+    """y, dy, d2y [npair][nint+1][M1] (f64) of the embedding net at the table nodes."""
+    params = _dev(params, "params", torch.float64)
+    w = (ctypes.c_int32 * len(widths))(*[int(x) for x in widths])
+    n0, n1 = dp_table_info_sizes(info)
+    npair, M1 = int(params.shape[0]), int(widths[-1])
+    shape = (npair, n0 + n1 + 1, M1)
+    if out is None:
+        out = tuple(torch.empty(shape, dtype=torch.float64, device=params.device) for _ in range(3))
+    y, dy, d2y = (_dev(o, "out", torch.float64, shape) for o in out)
+    _check(_lib.dp_embedding_net_nodes_f64(_ptr(params), w, len(widths) - 1, npair, ctypes.byref(info), _ptr(y),
+                                           _ptr(dy), _ptr(d2y), _stream(params)))
+    return y, dy, d2y
+
+
+def dp_table_build(y, dy, d2y, info: dp_table_info, dtype=torch.float64, out=None) -> torch.Tensor:
+    """Quintic coefficient table [npair][nint][M1][6] in `dtype` from f64 node values."""
+    y = _dev(y, "y", torch.float64)
+    npair, nn, M1 = (int(x) for x in y.shape)
+    dy = _dev(dy, "dy", torch.float64, y.shape)
+    d2y = _dev(d2y, "d2y", torch.float64, y.shape)
+    shape = (npair, nn - 1, M1, 6)
+    table = torch.empty(shape, dtype=dtype, device=y.device) if out is None else _dev(out, "out", dtype, shape)
+    fn = getattr(_lib, f"dp_table_build_{_suffix(dtype)}")
+    _check(fn(_ptr(y), _ptr(dy), _ptr(d2y), npair, M1, ctypes.byref(info), _ptr(table), _stream(y)))
+    return table
+
+
+def _sel_arr(sel):
+    sel = [int(x) for x in sel]
+    return (ctypes.c_int32 * len(sel))(*sel), len(sel), sum(sel)
+
+
+def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
+    dtype = table.dtype
+    table = _dev(table, "table", dtype)
+    s = _dev(s, "s", dtype)
+    nloc, nnei = (int(x) for x in s.shape)
+    Rt = _dev(Rt, "Rt", dtype, (nloc, nnei, 4))
+    selc, ntypes, nsum = _sel_arr(sel)
+    if nsum != nnei:
+        raise ValueError(f"sum(sel) = {nsum} != nnei = {nnei}")
+    if nvalid is not None:
+        nvalid = _dev(nvalid, "nvalid", torch.int32, (nloc, ntypes))
+    if atype is not None:
+        atype = _dev(atype, "atype", torch.int32, (nloc,))
+    M1 = int(table.shape[-2])
+    return dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1
+
+
+def dp_tabulate_fusion_fwd(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None) -> torch.Tensor:
+    """T [nloc][4][M1] = (1/nnei) R~^T G with G from the table, valid rows only."""
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
+                                                                                      sel)
+    shape = (nloc, 4, M1)
+    T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
+    fn = getattr(_lib, f"dp_tabulate_fusion_fwd_{_suffix(dtype)}")
+    _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
+              selc, M1, _ptr(T), _stream(s)))
+    return T
+
+
+def dp_tabulate_fusion_grad(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None):
+    """(ds [nloc][nnei], dRt [nloc][nnei][4]) from dT = dE/dT [nloc][4][M1]."""
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
+                                                                                      sel)
+    dT = _dev(dT, "dT", dtype, (nloc, 4, M1))
+    if out is None:
+        ds = torch.empty((nloc, nnei), dtype=dtype, device=s.device)
+        dRt = torch.empty((nloc, nnei, 4), dtype=dtype, device=s.device)
+    else:
+        ds = _dev(out[0], "ds", dtype, (nloc, nnei))
+        dRt = _dev(out[1], "dRt", dtype, (nloc, nnei, 4))
+    fn = getattr(_lib, f"dp_tabulate_fusion_grad_{_suffix(dtype)}")
+    _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
+              selc, M1, _ptr(dT), _ptr(ds), _ptr(dRt), _stream(s)))
+    return ds, dRt
+
+
+def dp_descriptor_contract(T, M2: int, out=None) -> torch.Tensor:
+    """D [nloc][M1][M2] = S (S^<)^T with S = T^T."""
+    T = _dev(T, "T", None)
+    nloc, four, M1 = (int(x) for x in T.shape)
+    if four != 4:
+        raise ValueError("T must be [nloc][4][M1]")
+    shape = (nloc, M1, int(M2))
+    D = torch.empty(shape, dtype=T.dtype, device=T.device) if out is None else _dev(out, "out", T.dtype, shape)
+    fn = getattr(_lib, f"dp_descriptor_contract_{_suffix(T.dtype)}")
+    _check(fn(_ptr(T), nloc, M1, int(M2), _ptr(D), _stream(T)))
+    return D
+
+
+@dataclass
+class Model:
+    """A compressed embedding: table range and the tables of every type pair, resident on the device."""
+    info: dp_table_info
+    table: torch.Tensor
+    ntypes: int
+    M1: int
+
+    @classmethod
+    def compress(cls, params: torch.Tensor, widths, info: dp_table_info, dtype=torch.float64) -> "Model":
+        """Net nodes (dp_embedding_net_nodes) -> coefficients (dp_table_build), all on the GPU."""
+        y, dy, d2y = dp_embedding_net_nodes(params, widths, info)
+        table = dp_table_build(y, dy, d2y, info, dtype)
+        npair = int(params.shape[0])
+        ntypes = int(round(npair ** 0.5))
+        if ntypes * ntypes != npair:
+            raise ValueError("params must hold ntypes^2 pair rows")
+        return cls(info=info, table=table, ntypes=ntypes, M1=int(widths[-1]))
+
+
+EXPORTS = tuple(_SIGS)

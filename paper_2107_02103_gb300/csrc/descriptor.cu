@@ -1,0 +1,81 @@
+// Descriptor (Sec. II): S_i = T_i^T is M1 x 4, S_i^< its first M2 rows, and
+// D_i = S_i (S_i^<)^T is M1 x M2:  D[i][m][n] = sum_k T[i][k][m] T[i][k][n].
+//
+// One warp per atom.  T_i (4 x M1) is staged in shared memory; the M1 x M2
+// output tile is contiguous, so lane l computes elements l, l + 32, ... of it
+// in storage order: every FP64 instruction has 32 busy lanes (M1*M2 is a
+// multiple of 32 for the paper's shapes) and every store is coalesced.
+#include "dp_common.cuh"
+
+namespace dpc {
+
+namespace {
+
+constexpr int kDescWarps = 4;
+
+template <typename real>
+__global__ void __launch_bounds__(kDescWarps * 32)
+    descriptor_kernel(const real *__restrict__ T, int64_t nloc, int M1, int M2, real *__restrict__ D) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t i = (int64_t)blockIdx.x * kDescWarps + w;
+  if (i >= nloc) return;  // warp-uniform; no block-wide barrier below
+  real *Ts = reinterpret_cast<real *>(smem_raw) + (size_t)w * 4 * M1;
+  const real *__restrict__ Ti = T + i * 4 * M1;
+  for (int e = lane; e < 4 * M1; e += 32) Ts[e] = __ldg(Ti + e);
+  __syncwarp();
+  real *__restrict__ Di = D + i * (int64_t)M1 * M2;
+  const int total = M1 * M2;
+  int m = lane / M2, n = lane - m * M2;
+  const int dm = 32 / M2, dn = 32 - dm * M2;  // advance of (m, n) per 32 elements
+  for (int e = lane; e < total; e += 32) {
+    real v = Ts[m] * Ts[n];
+    v = fma(Ts[M1 + m], Ts[M1 + n], v);
+    v = fma(Ts[2 * M1 + m], Ts[2 * M1 + n], v);
+    v = fma(Ts[3 * M1 + m], Ts[3 * M1 + n], v);
+    Di[e] = v;
+    m += dm;
+    n += dn;
+    if (n >= M2) {
+      n -= M2;
+      ++m;
+    }
+  }
+}
+
+template <typename real>
+int descriptor(const real *T, int64_t nloc, int M1, int M2, real *D, void *stream) {
+  clear_error();
+  if (nloc < 0 || M1 < 1 || M2 < 1 || M2 > M1)
+    return set_error(DP_ERR_SHAPE, "need nloc >= 0 and 1 <= M2 <= M1 (nloc %lld, M1 %d, M2 %d)", (long long)nloc, M1,
+                     M2);
+  if (M1 > 4096) return set_error(DP_ERR_UNSUPPORTED, "M1 = %d > 4096", M1);
+  if (nloc == 0) return DP_OK;
+  if (!T || !D) return set_error(DP_ERR_NULL, "T or D is NULL");
+  const int64_t blocks = (nloc + kDescWarps - 1) / kDescWarps;
+  if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
+  const size_t smem = (size_t)kDescWarps * 4 * M1 * sizeof(real);
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(descriptor_kernel<real>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                               (int)smem);
+    if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_descriptor_contract: %s", cudaGetErrorString(e));
+  }
+  descriptor_kernel<real><<<(unsigned)blocks, kDescWarps * 32, smem, (cudaStream_t)stream>>>(T, nloc, M1, M2, D);
+  return launch_status("dp_descriptor_contract");
+}
+
+}  // namespace
+
+}  // namespace dpc
+
+extern "C" {
+
+int dp_descriptor_contract_f64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream) {
+  return dpc::descriptor<double>(T, nloc, M1, M2, D, stream);
+}
+
+int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, float *D, void *stream) {
+  return dpc::descriptor<float>(T, nloc, M1, M2, D, stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,124 @@
+// Internal declarations shared by the library's translation units: error
+// state, table geometry, the interval search, and small load helpers.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "dp_compress.h"
+
+namespace dpc {
+
+// ---------------------------------------------------------------- errors
+int set_error(int code, const char *fmt, ...);  // stores the message, returns code
+void clear_error();
+int launch_status(const char *what);  // DP_ERR_CUDA if the last launch failed
+
+// --------------------------------------------------------- table geometry
+// dp_table_info with its derived sizes and reciprocal steps.
+struct TableGeom {
+  double lower, upper, upper_ext, stride0, stride1, inv0, inv1;
+  int32_t n0, n1, nint;
+};
+
+int make_geom(const dp_table_info *info, TableGeom *g);  // validates; DP_ERR_TABLE_INFO / DP_ERR_NULL
+
+// Per-type row layout: sel[b] rows of type b starting at off[b].
+struct Segments {
+  int32_t ntypes, nnei;
+  int32_t sel[DP_MAX_TYPES];
+};
+int make_segments(int ntypes, const int32_t *sel, int nnei, Segments *out);
+
+// Node x_l of the grid (Sec. II, the interpolation points): fine nodes
+// lower + l*stride0, the junction node `upper`, coarse nodes upper + k*stride1.
+__host__ __device__ __forceinline__ double node_x(const TableGeom &g, int l) {
+  if (l < g.n0) return g.lower + (double)l * g.stride0;
+  if (l == g.n0) return g.upper;
+  return g.upper + (double)(l - g.n0) * g.stride1;
+}
+
+// Interval l of input s and local variable t = s - x_l (Sec. II: g_m^l is a
+// polynomial in the offset from the left node of its interval).
+//   lower <= s < upper      -> l = floor((s - lower)/stride0) kept in [0, n0)
+//   upper <= s < upper_ext  -> l = n0 + floor((s - upper)/stride1) kept in [n0, nint)
+//   s < lower               -> first node (l = 0, t = 0), clamped
+//   s >= upper_ext          -> last node (l = nint-1, t = its width), clamped
+//   s NaN                   -> l = 0, t = NaN (propagates into the results)
+// Clamped inputs see the end value of the table and a zero derivative.
+__device__ __forceinline__ int locate(const TableGeom &g, double s, double &t, bool &clamped) {
+  clamped = false;
+  if (s >= g.lower) {
+    if (s < g.upper) {
+      const int l = min((int)((s - g.lower) * g.inv0), g.n0 - 1);
+      t = s - node_x(g, l);
+      return l;
+    }
+    if (s < g.upper_ext) {
+      const int k = min((int)((s - g.upper) * g.inv1), g.n1 - 1);
+      t = s - node_x(g, g.n0 + k);
+      return g.n0 + k;
+    }
+    clamped = true;
+    t = g.n1 > 0 ? g.stride1 : g.stride0;
+    return g.nint - 1;
+  }
+  if (s < g.lower) {
+    clamped = true;
+    t = 0.0;
+    return 0;
+  }
+  t = s;  // NaN
+  return 0;
+}
+
+// ------------------------------------------------------- vector helpers
+template <typename real> struct Vec4;
+template <> struct Vec4<double> {
+  double x, y, z, w;
+};
+template <> struct Vec4<float> {
+  float x, y, z, w;
+};
+
+// Four consecutive values (an environment-matrix row, a dT column).
+__device__ __forceinline__ Vec4<double> ld4(const double *p) {
+  const double2 a = __ldg(reinterpret_cast<const double2 *>(p));
+  const double2 b = __ldg(reinterpret_cast<const double2 *>(p) + 1);
+  return {a.x, a.y, b.x, b.y};
+}
+__device__ __forceinline__ Vec4<float> ld4(const float *p) {
+  const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
+  return {a.x, a.y, a.z, a.w};
+}
+
+// The six coefficients (a, b, c, d, e, f) of one channel of one interval.
+__device__ __forceinline__ void ld6(const double *p, double c[6]) {
+  const double2 *q = reinterpret_cast<const double2 *>(p);
+  const double2 x = __ldg(q), y = __ldg(q + 1), z = __ldg(q + 2);
+  c[0] = x.x; c[1] = x.y; c[2] = y.x; c[3] = y.y; c[4] = z.x; c[5] = z.y;
+}
+__device__ __forceinline__ void ld6(const float *p, float c[6]) {
+  const float2 *q = reinterpret_cast<const float2 *>(p);
+  const float2 x = __ldg(q), y = __ldg(q + 1), z = __ldg(q + 2);
+  c[0] = x.x; c[1] = x.y; c[2] = y.x; c[3] = y.y; c[4] = z.x; c[5] = z.y;
+}
+
+__device__ __forceinline__ void st4(double *p, double a, double b, double c, double d) {
+  reinterpret_cast<double2 *>(p)[0] = make_double2(a, b);
+  reinterpret_cast<double2 *>(p)[1] = make_double2(c, d);
+}
+__device__ __forceinline__ void st4(float *p, float a, float b, float c, float d) {
+  *reinterpret_cast<float4 *>(p) = make_float4(a, b, c, d);
+}
+
+__device__ __forceinline__ int clampi(int x, int lo, int hi) { return min(max(x, lo), hi); }
+
+// Validation shared by the forward and gradient entry points.
+int check_fusion_args(const void *table, const dp_table_info *info, const void *s, const void *Rt, int64_t nloc,
+                      int nnei, int ntypes, const int32_t *sel, int M1, const void *out0, const void *out1,
+                      TableGeom *g, Segments *seg);
+
+}  // namespace dpc
