@@ -47,6 +47,23 @@ def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
     return NSM * FMA_LANES[dtype] * 2 * mhz * 1e6 / 1e12
 
 
+def rank_seed(seed: int, rank: int) -> int:
+    """Seed of rank's own instance of the workload (weak scaling: every rank does the full per-GPU work)."""
+    return seed + 7919 * rank
+
+
+def reduce_over_ranks(total_s: float, evals: float, world: int, device) -> tuple[float, float]:
+    """Max of the timed seconds and sum of the work over ranks (timing only; the data path has no collective)."""
+    if world == 1:
+        return total_s, evals
+    import torch
+    t = torch.tensor([total_s], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    e = torch.tensor([evals], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(e)
+    return float(t.item()), float(e.item())
+
+
 def workload_label(w) -> str:
     d = w.describe()
     return (f"{w.name}: nloc={w.nloc}, sel={d['sel']}, M1={w.M1}, M2={w.M2}, "
@@ -125,7 +142,7 @@ def run_native(args, rank, world, local_rank):
     kw = {}
     if args.workload == "alcumg":
         kw["pad"] = args.pad
-    w = W.make(args.workload, seed=args.seed + 7919 * rank, **kw)
+    w = W.make(args.workload, seed=rank_seed(args.seed, rank), **kw)
     info = dpc.dp_table_info_make(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
     model = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, dtype)
     sel = [int(x) for x in w.sel]
@@ -181,17 +198,7 @@ def run_native(args, rank, world, local_rank):
     step_ms = [e[0].elapsed_time(e[3]) for e in evs]
     k_ms = {"fwd": [e[0].elapsed_time(e[1]) for e in evs], "descriptor": [e[1].elapsed_time(e[2]) for e in evs],
             "grad": [e[2].elapsed_time(e[3]) for e in evs]}
-    total_s = sum(step_ms) / 1e3
-    if world > 1:
-        t = torch.tensor([total_s], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_s = float(t.item())
-        ev_all = torch.tensor([float(w.evals)], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(ev_all)
-        evals_all = float(ev_all.item())
-    else:
-        evals_all = float(w.evals)
-    value = evals_all * args.steps / total_s
+    total_s, evals_all = reduce_over_ranks(sum(step_ms) / 1e3, float(w.evals), world, dev)
 
     # ---- end to end through the public API: pinned host inputs -> device -> path -> host results
     e2e = None if args.no_e2e else measure_e2e(args, host, d, dict(T=T, D=D, ds=ds, dRt=dRt), step, stream, dev,
@@ -225,11 +232,7 @@ def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_al
         e2e_step()
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_s = e0.elapsed_time(e1) / 1e3
-    if world > 1:
-        t = torch.tensor([e2e_s], dtype=torch.float64, device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s, _ = reduce_over_ranks(e0.elapsed_time(e1) / 1e3, 0.0, world, dev)
     barrier()
     return {"value": evals_all * args.steps / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h}

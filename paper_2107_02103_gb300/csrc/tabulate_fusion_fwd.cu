@@ -5,20 +5,23 @@
 // through the per-type valid counts.
 //
 // GB300 design.  The FP64 pipe issues one warp instruction per 16 SM clocks
-// no matter how many lanes are active, so the mapping is chosen to keep every
-// lane of every FP64 instruction busy:
-//   * one warp per atom; the warp's 32 lanes are G = 32/CL groups of CL
-//     channel lanes; group g takes every G-th valid neighbour, lane c of the
-//     group owns channels c, c + CL, ..., c + (R-1) CL (R rounds).  For M1 =
-//     100, CL = 8 and R = 13 fill 104 slots for 100 channels (96 %), against
-//     78 % for one neighbour per warp instruction.
-//   * the interval search, the segment lookup and the R~ row load are done
-//     once per neighbour, spread over the lanes (lane l handles neighbour
-//     base + l) and handed to the groups through shared memory, so their
-//     FP64 work costs 1/32 of an instruction per neighbour;
-//   * the G partial T_i are summed with xor shuffles once per atom.
-// Coefficients are read through the read-only path (the tables are a few MB
-// and stay resident in the 126 MB L2).
+// however many lanes are active, so every FP64 instruction must have 32 busy
+// lanes.  With M1 = 32 Q + RR:
+//   * Q full rounds: all 32 lanes work on the same neighbour, lane l owning
+//     channels l, l + 32, ..., l + 32 (Q-1).  The interval's coefficient row
+//     is one contiguous 6*M1 block, so each round reads 32 x 48 B coalesced.
+//   * one packed round for the RR remaining channels: lane l serves channel
+//     32 Q + (l mod RR) of neighbour l / RR, so PK = 32 / RR neighbours share
+//     one instruction (M1 = 100: 4 remainder channels x 8 neighbours fill all
+//     32 lanes, so 100 channels cost exactly 100/32 instructions).
+//   * the interval search, the segment lookup and the R~ row load run once
+//     per neighbour, spread over the lanes (lane l handles neighbour base +
+//     l), and are handed over through shared memory: their FP64 work costs
+//     1/32 of an instruction per neighbour.
+//   * one warp per block and per atom keeps the work units small, so the
+//     block scheduler balances the SMs to within one atom.
+// The packed round's partial sums meet in a shuffle reduction over the PK
+// lanes of each remainder channel, once per atom.
 #include <utility>
 
 #include "dp_common.cuh"
@@ -27,7 +30,7 @@ namespace dpc {
 
 namespace {
 
-constexpr int kFwdWarps = 4;
+constexpr int kFwdWarps = 1;
 
 template <typename real>
 struct FwdParams {
@@ -40,6 +43,7 @@ struct FwdParams {
   TableGeom geom;
   int64_t nloc;
   int32_t nnei, ntypes, M1, pair_stride;  // pair_stride = nint * M1 * 6
+  int32_t RR, PK;                          // remainder channels, neighbours per packed round
   int32_t sel[DP_MAX_TYPES];
   real inv_nnei;
 };
@@ -51,15 +55,23 @@ struct alignas(16) Stage {
   int32_t off[32];  // element offset of the interval's coefficient row in the centre type's tables
 };
 
-template <typename real, int CL, int R>
+template <typename real>
+__device__ __forceinline__ real horner5(const real c[6], real t) {
+  // g = ((((a t + b) t + c) t + d) t + e) t + f
+  real g = fma(c[0], t, c[1]);
+  g = fma(g, t, c[2]);
+  g = fma(g, t, c[3]);
+  g = fma(g, t, c[4]);
+  return fma(g, t, c[5]);
+}
+
+template <typename real, int Q>
 __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<real> P) {
-  constexpr int G = 32 / CL;
   __shared__ Stage<real> stage[kFwdWarps];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t i = (int64_t)blockIdx.x * kFwdWarps + w;
   if (i >= P.nloc) return;  // warp-uniform
   Stage<real> &st = stage[w];
-  const int g = lane / CL, c = lane % CL;
 
   // valid rows per type segment (clamped into [0, sel]) and their total
   int nvb[DP_MAX_TYPES];
@@ -76,9 +88,15 @@ __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<rea
   const real *__restrict__ srow = P.s + i * P.nnei;
   const real *__restrict__ Rrow = P.Rt + i * P.nnei * 4;
 
-  real acc[R][4];
+  // packed-round role of this lane: neighbour slot and remainder channel
+  const int rslot = P.RR > 0 ? lane / P.RR : 0;
+  const int rch = P.RR > 0 ? lane - rslot * P.RR : 0;
+  const bool ractive = P.RR > 0 && rslot < P.PK;
+
+  real acc[Q > 0 ? Q : 1][4];
 #pragma unroll
-  for (int r = 0; r < R; ++r) acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = real(0);
+  for (int r = 0; r < (Q > 0 ? Q : 1); ++r) acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = real(0);
+  real racc0 = real(0), racc1 = real(0), racc2 = real(0), racc3 = real(0);
 
   for (int base = 0; base < nv; base += 32) {
     // stage: lane l prepares valid neighbour base + l
@@ -107,50 +125,69 @@ __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<rea
     }
     __syncwarp();
     const int cnt = min(32, nv - base);
-    for (int q = 0; q < cnt; q += G) {
-      const int u = q + g;
-      if (u < cnt) {
+    if (Q > 0) {
+      for (int u = 0; u < cnt; ++u) {  // uniform: every lane on neighbour u
         const real t = st.t[u];
         const real r0 = st.r[u][0], r1 = st.r[u][1], r2 = st.r[u][2], r3 = st.r[u][3];
-        const real *__restrict__ cp = tab + st.off[u] + c * 6;
+        const real *__restrict__ cp = tab + st.off[u] + lane * 6;
 #pragma unroll
-        for (int r = 0; r < R; ++r) {
-          if (r < R - 1 || c + r * CL < P.M1) {
-            real cf[6];
-            ld6(cp + r * CL * 6, cf);
-            // g = ((((a t + b) t + c) t + d) t + e) t + f
-            real gv = fma(cf[0], t, cf[1]);
-            gv = fma(gv, t, cf[2]);
-            gv = fma(gv, t, cf[3]);
-            gv = fma(gv, t, cf[4]);
-            gv = fma(gv, t, cf[5]);
-            acc[r][0] = fma(r0, gv, acc[r][0]);
-            acc[r][1] = fma(r1, gv, acc[r][1]);
-            acc[r][2] = fma(r2, gv, acc[r][2]);
-            acc[r][3] = fma(r3, gv, acc[r][3]);
-          }
+        for (int r = 0; r < Q; ++r) {
+          real cf[6];
+          ld6(cp + r * 32 * 6, cf);
+          const real g = horner5(cf, t);
+          acc[r][0] = fma(r0, g, acc[r][0]);
+          acc[r][1] = fma(r1, g, acc[r][1]);
+          acc[r][2] = fma(r2, g, acc[r][2]);
+          acc[r][3] = fma(r3, g, acc[r][3]);
+        }
+      }
+    }
+    if (P.RR > 0) {
+      for (int u0 = 0; u0 < cnt; u0 += P.PK) {  // packed round: PK neighbours x RR channels
+        const int u = u0 + rslot;
+        if (ractive && u < cnt) {
+          const real t = st.t[u];
+          real cf[6];
+          ld6(tab + st.off[u] + (Q * 32 + rch) * 6, cf);
+          const real g = horner5(cf, t);
+          racc0 = fma(st.r[u][0], g, racc0);
+          racc1 = fma(st.r[u][1], g, racc1);
+          racc2 = fma(st.r[u][2], g, racc2);
+          racc3 = fma(st.r[u][3], g, racc3);
         }
       }
     }
     __syncwarp();
   }
 
-  // sum the G groups' partial T_i
+  real *__restrict__ Ti = P.T + i * 4 * P.M1;
 #pragma unroll
-  for (int sh = CL; sh < 32; sh <<= 1)
-#pragma unroll
-    for (int r = 0; r < R; ++r)
-#pragma unroll
-      for (int k = 0; k < 4; ++k) acc[r][k] += __shfl_xor_sync(0xffffffffu, acc[r][k], sh);
-
-  if (g == 0) {
-    real *__restrict__ Ti = P.T + i * 4 * P.M1;
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int m = c + r * CL;
-      if (m < P.M1)
-#pragma unroll
-        for (int k = 0; k < 4; ++k) Ti[k * P.M1 + m] = acc[r][k] * P.inv_nnei;
+  for (int r = 0; r < Q; ++r) {
+    const int m = r * 32 + lane;
+    Ti[m] = acc[r][0] * P.inv_nnei;
+    Ti[P.M1 + m] = acc[r][1] * P.inv_nnei;
+    Ti[2 * P.M1 + m] = acc[r][2] * P.inv_nnei;
+    Ti[3 * P.M1 + m] = acc[r][3] * P.inv_nnei;
+  }
+  if (P.RR > 0) {
+    // lanes rch, rch + RR, ..., rch + (PK-1) RR hold partial sums of channel 32 Q + rch
+    for (int k = 1; k < P.PK; ++k) {
+      const int src = lane + k * P.RR;
+      const real x0 = __shfl_sync(0xffffffffu, racc0, src & 31), x1 = __shfl_sync(0xffffffffu, racc1, src & 31);
+      const real x2 = __shfl_sync(0xffffffffu, racc2, src & 31), x3 = __shfl_sync(0xffffffffu, racc3, src & 31);
+      if (lane < P.RR) {
+        racc0 += x0;
+        racc1 += x1;
+        racc2 += x2;
+        racc3 += x3;
+      }
+    }
+    if (lane < P.RR) {
+      const int m = Q * 32 + lane;
+      Ti[m] = racc0 * P.inv_nnei;
+      Ti[P.M1 + m] = racc1 * P.inv_nnei;
+      Ti[2 * P.M1 + m] = racc2 * P.inv_nnei;
+      Ti[3 * P.M1 + m] = racc3 * P.inv_nnei;
     }
   }
 }
@@ -158,26 +195,11 @@ __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<rea
 template <typename real>
 using FwdKernel = void (*)(const FwdParams<real>);
 
-template <typename real, int CL, int... Rs>
-FwdKernel<real> pick_fwd(int R, std::integer_sequence<int, Rs...>) {
+template <typename real, int... Qs>
+FwdKernel<real> pick_fwd(int Q, std::integer_sequence<int, Qs...>) {
   FwdKernel<real> k = nullptr;
-  ((R == Rs + 1 ? (k = &fwd_kernel<real, CL, Rs + 1>, 0) : 0), ...);
+  ((Q == Qs ? (k = &fwd_kernel<real, Qs>, 0) : 0), ...);
   return k;
-}
-
-// Channel-lane width CL and rounds R for M1: the pair with the fewest idle
-// lane slots (CL = 8 costs a small group reduction, so it must win by >1 %).
-void choose_fwd_shape(int M1, int *CL, int *R) {
-  const int r32 = (M1 + 31) / 32, r8 = (M1 + 7) / 8;
-  const double e32 = r32 <= 8 ? (double)M1 / (32.0 * r32) : -1.0;
-  const double e8 = r8 <= 16 ? (double)M1 / (8.0 * r8) - 0.01 : -1.0;
-  if (e8 > e32) {
-    *CL = 8;
-    *R = r8;
-  } else {
-    *CL = 32;
-    *R = r32;
-  }
 }
 
 template <typename real>
@@ -202,12 +224,12 @@ int fwd(const real *table, const dp_table_info *info, const real *s, const real 
   P.ntypes = ntypes;
   P.M1 = M1;
   P.pair_stride = g.nint * M1 * 6;
+  const int Q = M1 / 32;
+  P.RR = M1 - 32 * Q;
+  P.PK = P.RR > 0 ? 32 / P.RR : 1;
   for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
   P.inv_nnei = (real)(1.0 / (double)nnei);
-  int CL, R;
-  choose_fwd_shape(M1, &CL, &R);
-  FwdKernel<real> k = CL == 8 ? pick_fwd<real, 8>(R, std::make_integer_sequence<int, 16>{})
-                              : pick_fwd<real, 32>(R, std::make_integer_sequence<int, 8>{});
+  FwdKernel<real> k = pick_fwd<real>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
   if (!k) return set_error(DP_ERR_UNSUPPORTED, "no forward kernel for M1 = %d", M1);
   const int64_t blocks = (nloc + kFwdWarps - 1) / kFwdWarps;
   if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
