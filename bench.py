@@ -43,6 +43,12 @@ FMA_PER_EVAL = {"fwd": 9, "grad": 18}
 DESC_FMA_PER_ATOM = lambda M1, M2: 4 * M1 * M2  # noqa: E731
 
 
+# DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
+# `ncu --set full` capture of its current version (profiles/<kernel>_<workload>_<dtype>.md);
+# absent means no capture of the current kernel exists and `traffic` is reported as null.
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad"): 83890176 + 34167040}
+
+
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
     return NSM * FMA_LANES[dtype] * 2 * mhz * 1e6 / 1e12
 
@@ -252,7 +258,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall):
     achieved = flops[dom] / (mean[dom] * 1e-3) / 1e12
     path_tflops = (flops["fwd"] + flops["grad"]) / ((mean["fwd"] + mean["grad"]) * 1e-3) / 1e12
     roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
-                "frac": round(achieved / pk, 4), "traffic": None, "kernel": f"dp_tabulate_fusion_{dom}",
+                "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom)),
+                "kernel": f"dp_tabulate_fusion_{dom}",
                 "peak_basis": (f"FP{64 if args.dtype == 'f64' else 32} FMA pipe: {NSM} SMs x "
                                f"{FMA_LANES[args.dtype]} lanes/clk x 2 flop x {SM_MAX_MHZ:.0f} MHz"),
                 "fwd_grad_frac": round(path_tflops / pk, 4)}

@@ -115,7 +115,10 @@ int dp_embedding_net_nodes_f64(const double *params, const int32_t *widths, int 
  * The brackets of a, b, c are evaluated in double-double arithmetic (they
  * cancel to O(Dt^5) relative) and rounded once.
  *   y, dy, d2y  [npair][nint + 1][M1] f64 node values (device).
- *   table       [npair][nint][M1][6] (a, b, c, d, e, f), f64 or rounded to f32.
+ *   table       [npair][nint][3][M1][2], f64 or rounded to f32: per interval a
+ *               pair-planar block -- the (a, b) pairs of channels 0..M1-1, then
+ *               the (c, d) pairs, then the (e, f) pairs -- so that lanes reading
+ *               consecutive channels make fully coalesced loads.
  * Errors: DP_ERR_NULL, DP_ERR_SHAPE (npair < 1, M1 < 1), DP_ERR_TABLE_INFO,
  * DP_ERR_CUDA.
  */
@@ -133,7 +136,7 @@ int dp_table_build_f32(const double *y, const double *dy, const double *d2y, int
  * upper) uses l = floor((s - lower)/stride0), s in [upper, upper_ext) uses
  * n0 + floor((s - upper)/stride1); s < lower evaluates the first node, s >=
  * upper_ext the last node; NaN s gives NaN in that atom's T.
- *   table   [npair][nint][M1][6] (from dp_table_build_*), npair = ntypes^2
+ *   table   [npair][nint][3][M1][2] (from dp_table_build_*), npair = ntypes^2
  *   s       [nloc][nnei]      embedding input per row
  *   Rt      [nloc][nnei][4]   environment-matrix rows
  *   nvalid  [nloc][ntypes] int32, real rows per type segment; entries are

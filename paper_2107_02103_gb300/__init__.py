@@ -140,12 +140,12 @@ def dp_embedding_net_nodes(params: torch.Tensor, widths, info: dp_table_info, ou
 
 
 def dp_table_build(y, dy, d2y, info: dp_table_info, dtype=torch.float64, out=None) -> torch.Tensor:
-    """Quintic coefficient table [npair][nint][M1][6] in `dtype` from f64 node values."""
+    """Quintic coefficient table [npair][nint][3][M1][2] (pair-planar a..f) in `dtype` from f64 node values."""
     y = _dev(y, "y", torch.float64)
     npair, nn, M1 = (int(x) for x in y.shape)
     dy = _dev(dy, "dy", torch.float64, y.shape)
     d2y = _dev(d2y, "d2y", torch.float64, y.shape)
-    shape = (npair, nn - 1, M1, 6)
+    shape = (npair, nn - 1, 3, M1, 2)
     table = torch.empty(shape, dtype=dtype, device=y.device) if out is None else _dev(out, "out", dtype, shape)
     fn = getattr(_lib, f"dp_table_build_{_suffix(dtype)}")
     _check(fn(_ptr(y), _ptr(dy), _ptr(d2y), npair, M1, ctypes.byref(info), _ptr(table), _stream(y)))
@@ -170,6 +170,8 @@ def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
         nvalid = _dev(nvalid, "nvalid", torch.int32, (nloc, ntypes))
     if atype is not None:
         atype = _dev(atype, "atype", torch.int32, (nloc,))
+    if table.dim() != 5 or table.shape[-3] != 3 or table.shape[-1] != 2:
+        raise ValueError("table must be [npair][nint][3][M1][2] (from dp_table_build)")
     M1 = int(table.shape[-2])
     return dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1
 
@@ -234,6 +236,11 @@ class Model:
         if ntypes * ntypes != npair:
             raise ValueError("params must hold ntypes^2 pair rows")
         return cls(info=info, table=table, ntypes=ntypes, M1=int(widths[-1]))
+
+
+def table_rows(table: torch.Tensor) -> torch.Tensor:
+    """View a pair-planar table [npair][nint][3][M1][2] as [npair][nint][M1][6] rows (a, b, c, d, e, f)."""
+    return table.permute(0, 1, 3, 2, 4).reshape(table.shape[0], table.shape[1], table.shape[3], 6)
 
 
 EXPORTS = tuple(_SIGS)

@@ -74,6 +74,69 @@ __device__ __forceinline__ int locate(const TableGeom &g, double s, double &t, b
   return 0;
 }
 
+// The same grid and search in f32 arithmetic, for the f32 kernels: there the
+// FP64 pipe is 64x slower than the FFMA pipe, so even a per-neighbour double
+// search would cost as much as the channel work it serves.  The oracle runs
+// the search in double on the same f32 inputs; the two can differ only at a
+// node (where both intervals give the same value, the table being C2) and by
+// the f32 rounding of t (~1e-7 absolute), far inside the f32 tolerance.
+struct TableGeomF {
+  float lower, upper, upper_ext, stride0, stride1, inv0, inv1;
+  int32_t n0, n1, nint;
+};
+
+inline TableGeomF to_f32(const TableGeom &g) {
+  TableGeomF f;
+  f.lower = (float)g.lower;
+  f.upper = (float)g.upper;
+  f.upper_ext = (float)g.upper_ext;
+  f.stride0 = (float)g.stride0;
+  f.stride1 = (float)g.stride1;
+  f.inv0 = (float)g.inv0;
+  f.inv1 = (float)g.inv1;
+  f.n0 = g.n0;
+  f.n1 = g.n1;
+  f.nint = g.nint;
+  return f;
+}
+
+__device__ __forceinline__ int locate(const TableGeomF &g, float s, float &t, bool &clamped) {
+  clamped = false;
+  if (s >= g.lower) {
+    if (s < g.upper) {
+      const int l = min((int)((s - g.lower) * g.inv0), g.n0 - 1);
+      t = s - fmaf((float)l, g.stride0, g.lower);
+      return l;
+    }
+    if (s < g.upper_ext) {
+      const int k = min((int)((s - g.upper) * g.inv1), g.n1 - 1);
+      t = s - fmaf((float)k, g.stride1, g.upper);
+      return g.n0 + k;
+    }
+    clamped = true;
+    t = g.n1 > 0 ? g.stride1 : g.stride0;
+    return g.nint - 1;
+  }
+  if (s < g.lower) {
+    clamped = true;
+    t = 0.0f;
+    return 0;
+  }
+  t = s;  // NaN
+  return 0;
+}
+
+// Geometry type used by the kernels of each precision.
+template <typename real> struct GeomOf;
+template <> struct GeomOf<double> {
+  using type = TableGeom;
+  static TableGeom make(const TableGeom &g) { return g; }
+};
+template <> struct GeomOf<float> {
+  using type = TableGeomF;
+  static TableGeomF make(const TableGeom &g) { return to_f32(g); }
+};
+
 // ------------------------------------------------------- vector helpers
 template <typename real> struct Vec4;
 template <> struct Vec4<double> {
@@ -94,15 +157,19 @@ __device__ __forceinline__ Vec4<float> ld4(const float *p) {
   return {a.x, a.y, a.z, a.w};
 }
 
-// The six coefficients (a, b, c, d, e, f) of one channel of one interval.
-__device__ __forceinline__ void ld6(const double *p, double c[6]) {
-  const double2 *q = reinterpret_cast<const double2 *>(p);
-  const double2 x = __ldg(q), y = __ldg(q + 1), z = __ldg(q + 2);
+// The six coefficients (a, b, c, d, e, f) of channel m of one interval.  An
+// interval's block of 6*M1 values is stored pair-planar, [3][M1][2]: the
+// (a, b) pairs of all channels, then the (c, d) pairs, then the (e, f) pairs.
+// Lanes that read consecutive channels then read consecutive 2-vectors: each
+// of the three loads of a warp is fully coalesced (no sector fetched twice).
+__device__ __forceinline__ void ld6(const double *blk, int M1, int m, double c[6]) {
+  const double2 *q = reinterpret_cast<const double2 *>(blk) + m;
+  const double2 x = __ldg(q), y = __ldg(q + M1), z = __ldg(q + 2 * M1);
   c[0] = x.x; c[1] = x.y; c[2] = y.x; c[3] = y.y; c[4] = z.x; c[5] = z.y;
 }
-__device__ __forceinline__ void ld6(const float *p, float c[6]) {
-  const float2 *q = reinterpret_cast<const float2 *>(p);
-  const float2 x = __ldg(q), y = __ldg(q + 1), z = __ldg(q + 2);
+__device__ __forceinline__ void ld6(const float *blk, int M1, int m, float c[6]) {
+  const float2 *q = reinterpret_cast<const float2 *>(blk) + m;
+  const float2 x = __ldg(q), y = __ldg(q + M1), z = __ldg(q + 2 * M1);
   c[0] = x.x; c[1] = x.y; c[2] = y.x; c[3] = y.y; c[4] = z.x; c[5] = z.y;
 }
 

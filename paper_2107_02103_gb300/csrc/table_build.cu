@@ -152,13 +152,14 @@ __global__ void __launch_bounds__(kBuildThreads)
   const dd bc = dd_add(dd_add(dd_mul_d(h, 20.0), dd_mul_d(pc, -1.0)), dd_mul_d(qc, -1.0));
 
   const double Dt3 = Dt * Dt * Dt, Dt4 = Dt3 * Dt, Dt5 = Dt4 * Dt;
-  real *out = table + (size_t)tid * 6;
-  out[0] = (real)(dd_val(ba) / (2.0 * Dt5));
-  out[1] = (real)(dd_val(bb) / (2.0 * Dt4));
-  out[2] = (real)(dd_val(bc) / (2.0 * Dt3));
-  out[3] = (real)(0.5 * q0);
-  out[4] = (real)p0;
-  out[5] = (real)y0;
+  // pair-planar block of interval (p, l): [3][M1][2] = (a, b), (c, d), (e, f) planes
+  real *blk = table + (size_t)pl * 6 * M1 + 2 * m;
+  blk[0] = (real)(dd_val(ba) / (2.0 * Dt5));
+  blk[1] = (real)(dd_val(bb) / (2.0 * Dt4));
+  blk[2 * M1] = (real)(dd_val(bc) / (2.0 * Dt3));
+  blk[2 * M1 + 1] = (real)(0.5 * q0);
+  blk[4 * M1] = (real)p0;
+  blk[4 * M1 + 1] = (real)y0;
 }
 
 template <typename real>

@@ -8,8 +8,9 @@
 // however many lanes are active, so every FP64 instruction must have 32 busy
 // lanes.  With M1 = 32 Q + RR:
 //   * Q full rounds: all 32 lanes work on the same neighbour, lane l owning
-//     channels l, l + 32, ..., l + 32 (Q-1).  The interval's coefficient row
-//     is one contiguous 6*M1 block, so each round reads 32 x 48 B coalesced.
+//     channels l, l + 32, ..., l + 32 (Q-1).  The interval's coefficients
+//     are one contiguous 6*M1 block, pair-planar, so each round's three
+//     vector loads are fully coalesced.
 //   * one packed round for the RR remaining channels: lane l serves channel
 //     32 Q + (l mod RR) of neighbour l / RR, so PK = 32 / RR neighbours share
 //     one instruction (M1 = 100: 4 remainder channels x 8 neighbours fill all
@@ -19,9 +20,12 @@
 //     l), and are handed over through shared memory: their FP64 work costs
 //     1/32 of an instruction per neighbour.
 //   * one warp per block and per atom keeps the work units small, so the
-//     block scheduler balances the SMs to within one atom.
+//     block scheduler balances the SMs to within a few atoms.
 // The packed round's partial sums meet in a shuffle reduction over the PK
-// lanes of each remainder channel, once per atom.
+// lanes of each remainder channel, once per atom.  In f32 the coefficient
+// row of the current interval is also kept in registers across consecutive
+// neighbours that share it (sorted by distance, they often do): there the
+// L1 traffic of reloading it, not the FFMA pipe, would be the limit.
 #include <utility>
 
 #include "dp_common.cuh"
@@ -40,7 +44,7 @@ struct FwdParams {
   const int32_t *__restrict__ nvalid;
   const int32_t *__restrict__ atype;
   real *__restrict__ T;
-  TableGeom geom;
+  typename GeomOf<real>::type geom;
   int64_t nloc;
   int32_t nnei, ntypes, M1, pair_stride;  // pair_stride = nint * M1 * 6
   int32_t RR, PK;                          // remainder channels, neighbours per packed round
@@ -52,7 +56,8 @@ template <typename real>
 struct alignas(16) Stage {
   real r[32][4];    // R~ rows of the staged neighbours
   real t[32];       // local variable t
-  int32_t off[32];  // element offset of the interval's coefficient row in the centre type's tables
+  int32_t off[32];  // element offset of the interval's coefficient block in the centre type's tables
+  int32_t nvb[DP_MAX_TYPES];  // valid rows per type segment of the current atom
 };
 
 template <typename real>
@@ -65,24 +70,25 @@ __device__ __forceinline__ real horner5(const real c[6], real t) {
   return fma(g, t, c[5]);
 }
 
+// One atom: T_i into P.T (the whole warp takes part).
 template <typename real, int Q>
-__global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<real> P) {
-  __shared__ Stage<real> stage[kFwdWarps];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int64_t i = (int64_t)blockIdx.x * kFwdWarps + w;
-  if (i >= P.nloc) return;  // warp-uniform
-  Stage<real> &st = stage[w];
+__device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &st, const int lane, const int64_t i) {
+  constexpr bool kCache = sizeof(real) == 4;  // reuse coefficient registers along runs (f32 only)
 
-  // valid rows per type segment (clamped into [0, sel]) and their total
-  int nvb[DP_MAX_TYPES];
+  // valid rows per type segment (clamped into [0, sel]), kept in shared memory, and their total
+  {
+    int sl = 0;  // sel[lane] without indexing the parameter array dynamically
+#pragma unroll
+    for (int q = 0; q < DP_MAX_TYPES; ++q)
+      if (lane == q) sl = P.sel[q];
+    int x = 0;
+    if (lane < P.ntypes) x = clampi(P.nvalid ? __ldg(P.nvalid + i * P.ntypes + lane) : sl, 0, sl);
+    if (lane < DP_MAX_TYPES) st.nvb[lane] = x;
+  }
+  __syncwarp();
   int nv = 0;
 #pragma unroll
-  for (int q = 0; q < DP_MAX_TYPES; ++q) {
-    int x = 0;
-    if (q < P.ntypes) x = clampi(P.nvalid ? __ldg(P.nvalid + i * P.ntypes + q) : P.sel[q], 0, P.sel[q]);
-    nvb[q] = x;
-    nv += x;
-  }
+  for (int q = 0; q < DP_MAX_TYPES; ++q) nv += st.nvb[q];
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   const real *__restrict__ tab = P.table + (size_t)alpha * P.ntypes * P.pair_stride;
   const real *__restrict__ srow = P.s + i * P.nnei;
@@ -97,44 +103,58 @@ __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<rea
 #pragma unroll
   for (int r = 0; r < (Q > 0 ? Q : 1); ++r) acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = real(0);
   real racc0 = real(0), racc1 = real(0), racc2 = real(0), racc3 = real(0);
+  real cf[kCache && Q > 0 ? Q : 1][6];  // f32: coefficient rows of the interval in use
+  real rcf[6];
+  int cur = -1, rcur = -1;
 
   for (int base = 0; base < nv; base += 32) {
     // stage: lane l prepares valid neighbour base + l
     const int v = base + lane;
     if (v < nv) {
-      int b = 0, cum = 0, lim = nvb[0], off = 0;
+      int b = 0, cum = 0, lim = st.nvb[0], off = 0;
 #pragma unroll
       for (int q = 1; q < DP_MAX_TYPES; ++q)
         if (q < P.ntypes && v >= lim) {
           b = q;
           cum = lim;
-          lim += nvb[q];
+          lim += st.nvb[q];
           off += P.sel[q - 1];
         }
       const int row = off + (v - cum);
       const Vec4<real> rr = ld4(Rrow + (size_t)row * 4);
-      double t;
+      real t;
       bool clamped;
-      const int l = locate(P.geom, (double)__ldg(srow + row), t, clamped);
+      const int l = locate(P.geom, __ldg(srow + row), t, clamped);
       st.r[lane][0] = rr.x;
       st.r[lane][1] = rr.y;
       st.r[lane][2] = rr.z;
       st.r[lane][3] = rr.w;
-      st.t[lane] = (real)t;
+      st.t[lane] = t;
       st.off[lane] = (b * P.geom.nint + l) * P.M1 * 6;
     }
     __syncwarp();
     const int cnt = min(32, nv - base);
     if (Q > 0) {
       for (int u = 0; u < cnt; ++u) {  // uniform: every lane on neighbour u
+        const int off = st.off[u];
+        const real *__restrict__ cp = tab + off;  // the interval's coefficient block
+        if (kCache && off != cur) {  // uniform branch
+          cur = off;
+#pragma unroll
+          for (int r = 0; r < Q; ++r) ld6(cp, P.M1, r * 32 + lane, cf[r]);
+        }
         const real t = st.t[u];
         const real r0 = st.r[u][0], r1 = st.r[u][1], r2 = st.r[u][2], r3 = st.r[u][3];
-        const real *__restrict__ cp = tab + st.off[u] + lane * 6;
 #pragma unroll
         for (int r = 0; r < Q; ++r) {
-          real cf[6];
-          ld6(cp + r * 32 * 6, cf);
-          const real g = horner5(cf, t);
+          real c6[6];
+          if (kCache) {
+#pragma unroll
+            for (int e = 0; e < 6; ++e) c6[e] = cf[kCache ? r : 0][e];
+          } else {
+            ld6(cp, P.M1, r * 32 + lane, c6);
+          }
+          const real g = horner5(c6, t);
           acc[r][0] = fma(r0, g, acc[r][0]);
           acc[r][1] = fma(r1, g, acc[r][1]);
           acc[r][2] = fma(r2, g, acc[r][2]);
@@ -147,9 +167,12 @@ __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<rea
         const int u = u0 + rslot;
         if (ractive && u < cnt) {
           const real t = st.t[u];
-          real cf[6];
-          ld6(tab + st.off[u] + (Q * 32 + rch) * 6, cf);
-          const real g = horner5(cf, t);
+          const int off = st.off[u];
+          if (!kCache || off != rcur) {
+            rcur = off;
+            ld6(tab + off, P.M1, Q * 32 + rch, rcf);
+          }
+          const real g = horner5(rcf, t);
           racc0 = fma(st.r[u][0], g, racc0);
           racc1 = fma(st.r[u][1], g, racc1);
           racc2 = fma(st.r[u][2], g, racc2);
@@ -192,6 +215,14 @@ __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<rea
   }
 }
 
+template <typename real, int Q>
+__global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<real> P) {
+  __shared__ Stage<real> stage[kFwdWarps];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t i = (int64_t)blockIdx.x * kFwdWarps + w;
+  if (i < P.nloc) fwd_atom<real, Q>(P, stage[w], lane, i);  // warp-uniform
+}
+
 template <typename real>
 using FwdKernel = void (*)(const FwdParams<real>);
 
@@ -218,7 +249,7 @@ int fwd(const real *table, const dp_table_info *info, const real *s, const real 
   P.nvalid = nvalid;
   P.atype = atype;
   P.T = T;
-  P.geom = g;
+  P.geom = GeomOf<real>::make(g);
   P.nloc = nloc;
   P.nnei = nnei;
   P.ntypes = ntypes;

@@ -15,10 +15,13 @@
 // same with 10 or 32 active lanes, so the valid rows of kGradChunk
 // consecutive atoms (all type segments) are packed into one flat list and
 // only the chunk's last warp can idle, instead of every atom's last warp.
-// Each thread gathers its own interval's coefficient row, which walks
-// contiguous memory as m advances; dT_i is read through the read-only cache
+// Each thread gathers its own interval's coefficients, which walk three
+// contiguous planes as m advances; dT_i is read through the read-only cache
 // (every lane of an atom reads the same address).  Threads past the valid
 // rows zero-fill the padding rows, packed the same way.
+#include <type_traits>
+#include <utility>
+
 #include "dp_common.cuh"
 
 namespace dpc {
@@ -114,7 +117,7 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 #pragma unroll 2
     for (int m = 0; m < P.M1; ++m) {
       real cf[6];
-      ld6(cp + m * 6, cf);
+      ld6(cp, P.M1, m, cf);
       const real d0 = __ldg(dTi + m), d1 = __ldg(dTi + P.M1 + m), d2 = __ldg(dTi + 2 * P.M1 + m),
                  d3 = __ldg(dTi + 3 * P.M1 + m);
       // g and g' by Horner's rule with derivative
@@ -167,6 +170,185 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
   }
 }
 
+// ---------------------------------------------------------------- f32
+// In f32 the FFMA pipe is 64x faster than FP64 and the per-thread gather of
+// a private coefficient row (32 distinct lines per load instruction) would
+// bind long before the arithmetic.  So the f32 backward works on row groups:
+// L channel lanes per neighbour row and 32/L rows per warp instruction.  The
+// L lanes of a row read L consecutive channels of the row's interval (three
+// contiguous runs of 8*L bytes in the pair-planar block), and rows that share
+// an interval -- most neighbours next to each other in distance order -- hit
+// the same sectors.
+// Each lane keeps dT for its channels in registers; the five per-row sums
+// (ds, dR~[0..3]) meet in a log2(L)-level shuffle reduction per row, which
+// is amortised over the M1/L channel rounds of that row.
+constexpr int kGradF32Warps = 4;
+
+struct GradParamsF32 {
+  const float *__restrict__ table;
+  const float *__restrict__ s;
+  const float *__restrict__ Rt;
+  const int32_t *__restrict__ nvalid;
+  const int32_t *__restrict__ atype;
+  const float *__restrict__ dT;
+  float *__restrict__ ds;
+  float *__restrict__ dRt;
+  TableGeomF geom;
+  int64_t nloc;
+  int32_t nnei, ntypes, M1, pair_stride;
+  int32_t sel[DP_MAX_TYPES];
+  float inv_nnei;
+};
+
+template <int L, int R>
+__global__ void __launch_bounds__(kGradF32Warps * 32) grad_f32_kernel(const GradParamsF32 P) {
+  constexpr int RPW = 32 / L;                  // rows per warp instruction
+  constexpr int STEP = kGradF32Warps * RPW;    // rows per block iteration
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int grp = lane / L, q = lane % L;
+  const int64_t i = blockIdx.x;  // one atom per block
+
+  int nvb[DP_MAX_TYPES];
+  int nv = 0;
+#pragma unroll
+  for (int b = 0; b < DP_MAX_TYPES; ++b) {
+    int x = 0;
+    if (b < P.ntypes) x = clampi(P.nvalid ? __ldg(P.nvalid + i * P.ntypes + b) : P.sel[b], 0, P.sel[b]);
+    nvb[b] = x;
+    nv += x;
+  }
+  const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
+  const float *__restrict__ tab = P.table + (size_t)alpha * P.ntypes * P.pair_stride;
+
+  float dt[R][4];  // dT_i for channels q, q + L, ...
+  const float *__restrict__ dTi = P.dT + i * 4 * P.M1;
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    const int m = q + L * r;
+    const bool ok = m < P.M1;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) dt[r][k] = ok ? __ldg(dTi + k * P.M1 + m) : 0.0f;
+  }
+
+  for (int vb = w * RPW; vb < nv; vb += STEP) {  // warp-uniform
+    const int v = vb + grp;
+    const bool act = v < nv;
+    float a_ds = 0.0f, a_0 = 0.0f, a_1 = 0.0f, a_2 = 0.0f, a_3 = 0.0f;
+    int row = 0;
+    bool clamped = false;
+    if (act) {
+      int b = 0, cum = 0, lim = nvb[0], off = 0;
+#pragma unroll
+      for (int c = 1; c < DP_MAX_TYPES; ++c)
+        if (c < P.ntypes && v >= lim) {
+          b = c;
+          cum = lim;
+          lim += nvb[c];
+          off += P.sel[c - 1];
+        }
+      row = off + (v - cum);
+      const Vec4<float> rr = ld4(P.Rt + (i * P.nnei + row) * 4);
+      float t;
+      const int l = locate(P.geom, __ldg(P.s + i * P.nnei + row), t, clamped);
+      const float *__restrict__ cp = tab + (size_t)(b * P.geom.nint + l) * P.M1 * 6;
+#pragma unroll
+      for (int r = 0; r < R; ++r) {
+        if (r < R - 1 || q + L * r < P.M1) {
+          float cf[6];
+          ld6(cp, P.M1, q + r * L, cf);
+          float p = fmaf(cf[0], t, cf[1]);
+          float dp = cf[0];
+          dp = fmaf(dp, t, p);
+          p = fmaf(p, t, cf[2]);
+          dp = fmaf(dp, t, p);
+          p = fmaf(p, t, cf[3]);
+          dp = fmaf(dp, t, p);
+          p = fmaf(p, t, cf[4]);
+          dp = fmaf(dp, t, p);
+          p = fmaf(p, t, cf[5]);
+          float rm = dt[r][0] * rr.x;
+          rm = fmaf(dt[r][1], rr.y, rm);
+          rm = fmaf(dt[r][2], rr.z, rm);
+          rm = fmaf(dt[r][3], rr.w, rm);
+          a_ds = fmaf(rm, dp, a_ds);
+          a_0 = fmaf(dt[r][0], p, a_0);
+          a_1 = fmaf(dt[r][1], p, a_1);
+          a_2 = fmaf(dt[r][2], p, a_2);
+          a_3 = fmaf(dt[r][3], p, a_3);
+        }
+      }
+    }
+#pragma unroll
+    for (int sh = L / 2; sh > 0; sh >>= 1) {
+      a_ds += __shfl_xor_sync(0xffffffffu, a_ds, sh);
+      a_0 += __shfl_xor_sync(0xffffffffu, a_0, sh);
+      a_1 += __shfl_xor_sync(0xffffffffu, a_1, sh);
+      a_2 += __shfl_xor_sync(0xffffffffu, a_2, sh);
+      a_3 += __shfl_xor_sync(0xffffffffu, a_3, sh);
+    }
+    if (act && q == 0) {
+      P.ds[i * P.nnei + row] = clamped ? 0.0f : a_ds * P.inv_nnei;
+      st4(P.dRt + (i * P.nnei + row) * 4, a_0 * P.inv_nnei, a_1 * P.inv_nnei, a_2 * P.inv_nnei,
+          a_3 * P.inv_nnei);
+    }
+  }
+
+  // padding rows of this atom, packed over the segments' padded tails
+  for (int pv = threadIdx.x; pv < P.nnei - nv; pv += kGradF32Warps * 32) {
+    int cum = 0, lim = P.sel[0] - nvb[0], off = 0, nvb_b = nvb[0];
+#pragma unroll
+    for (int c = 1; c < DP_MAX_TYPES; ++c)
+      if (c < P.ntypes && pv >= lim) {
+        cum = lim;
+        lim += P.sel[c] - nvb[c];
+        off += P.sel[c - 1];
+        nvb_b = nvb[c];
+      }
+    const int row = off + nvb_b + (pv - cum);
+    P.ds[i * P.nnei + row] = 0.0f;
+    st4(P.dRt + (i * P.nnei + row) * 4, 0.0f, 0.0f, 0.0f, 0.0f);
+  }
+}
+
+using GradF32Kernel = void (*)(const GradParamsF32);
+
+template <int L, int... Rs>
+GradF32Kernel pick_grad_f32(int R, std::integer_sequence<int, Rs...>) {
+  GradF32Kernel k = nullptr;
+  ((R == Rs + 1 ? (k = &grad_f32_kernel<L, Rs + 1>, 0) : 0), ...);
+  return k;
+}
+
+int grad_f32(const float *table, const TableGeom &g, const Segments &seg, const float *s, const float *Rt,
+             const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes, int M1, const float *dT,
+             float *ds, float *dRt, void *stream) {
+  GradParamsF32 P;
+  P.table = table;
+  P.s = s;
+  P.Rt = Rt;
+  P.nvalid = nvalid;
+  P.atype = atype;
+  P.dT = dT;
+  P.ds = ds;
+  P.dRt = dRt;
+  P.geom = to_f32(g);
+  P.nloc = nloc;
+  P.nnei = nnei;
+  P.ntypes = ntypes;
+  P.M1 = M1;
+  P.pair_stride = g.nint * M1 * 6;
+  for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
+  P.inv_nnei = (float)(1.0 / (double)nnei);
+  // 8 channel lanes per row up to M1 = 128 (at most 16 rounds), 16 beyond
+  const int L = M1 <= 128 ? 8 : 16;
+  const int R = (M1 + L - 1) / L;
+  GradF32Kernel k = L == 8 ? pick_grad_f32<8>(R, std::make_integer_sequence<int, 16>{})
+                           : pick_grad_f32<16>(R, std::make_integer_sequence<int, 16>{});
+  if (!k) return set_error(DP_ERR_UNSUPPORTED, "no f32 gradient kernel for M1 = %d", M1);
+  k<<<(unsigned)nloc, kGradF32Warps * 32, 0, (cudaStream_t)stream>>>(P);
+  return launch_status("dp_tabulate_fusion_grad_f32");
+}
+
 template <typename real>
 int grad(const real *table, const dp_table_info *info, const real *s, const real *Rt, const int32_t *nvalid,
          const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, const real *dT,
@@ -179,6 +361,8 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
   if (nloc == 0) return DP_OK;
   if (!dT) return set_error(DP_ERR_NULL, "dT is NULL");
   if (nloc > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
+  if constexpr (std::is_same<real, float>::value)
+    return grad_f32(table, g, seg, s, Rt, nvalid, atype, nloc, nnei, ntypes, M1, dT, ds, dRt, stream);
   GradParams<real> P;
   P.table = table;
   P.s = s;

@@ -51,8 +51,8 @@ def test_nodes_and_table(name):
         assert rel(gy, ry) < 1e-14 and rel(gdy, rdy) < 1e-13 and rel(gd2y, rd2y) < 1e-12
         same = o.table_build(gy, gdy, gd2y, info_o)     # oracle build on the GPU's nodes
         full = o.table_build(ry, rdy, rd2y, info_o)     # oracle nodes and build
-        g64 = tab64[p].cpu().numpy()
-        g32 = tab32[p].cpu().numpy().astype(np.float64)
+        g64 = dpc.table_rows(tab64)[p].cpu().numpy()
+        g32 = dpc.table_rows(tab32)[p].cpu().numpy().astype(np.float64)
         for l in list(range(0, info_o.nint, 7)) + [info_o.n0 - 1, info_o.n0, info_o.nint - 1]:
             Dt = info_o.stride0 if l < info_o.n0 else info_o.stride1
             for t in (0.0, 0.37 * Dt, Dt):
