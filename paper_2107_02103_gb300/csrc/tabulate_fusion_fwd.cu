@@ -26,6 +26,7 @@
 // row of the current interval is also kept in registers across consecutive
 // neighbours that share it (sorted by distance, they often do): there the
 // L1 traffic of reloading it, not the FFMA pipe, would be the limit.
+#include <type_traits>
 #include <utility>
 
 #include "dp_common.cuh"
@@ -68,6 +69,50 @@ __device__ __forceinline__ real horner5(const real c[6], real t) {
   g = fma(g, t, c[3]);
   g = fma(g, t, c[4]);
   return fma(g, t, c[5]);
+}
+
+// One neighbour (interval block offset `off`, local t, R~ row r) folded into
+// the lane's Q channel rounds.  kCache: the coefficients of the interval in
+// use stay in cf across neighbours that share it (the branch is uniform).
+template <typename real, int Q, bool kCache>
+__device__ __forceinline__ void fwd_neighbour(const FwdParams<real> &P, const real *__restrict__ tab, const int lane,
+                                              const int off, const real t, const real *r,
+                                              real (&acc)[Q > 0 ? Q : 1][4], real (&cf)[kCache && Q > 0 ? Q : 1][6],
+                                              int &cur) {
+  const real r0 = r[0], r1 = r[1], r2 = r[2], r3 = r[3];
+  if (kCache) {
+    if (off != cur) {
+      cur = off;
+      using V2 = typename std::conditional<sizeof(real) == 8, double2, float2>::type;
+      const V2 *q0 = reinterpret_cast<const V2 *>(tab + off) + lane;
+      const V2 *q1 = q0 + P.M1, *q2 = q1 + P.M1;
+#pragma unroll
+      for (int k = 0; k < Q; ++k) {
+        const V2 x = __ldg(q0 + 32 * k), y = __ldg(q1 + 32 * k), z = __ldg(q2 + 32 * k);
+        cf[kCache ? k : 0][0] = x.x;
+        cf[kCache ? k : 0][1] = x.y;
+        cf[kCache ? k : 0][2] = y.x;
+        cf[kCache ? k : 0][3] = y.y;
+        cf[kCache ? k : 0][4] = z.x;
+        cf[kCache ? k : 0][5] = z.y;
+      }
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < Q; ++k) {
+    real c6[6];
+    if (kCache) {
+#pragma unroll
+      for (int e = 0; e < 6; ++e) c6[e] = cf[kCache ? k : 0][e];
+    } else {
+      ld6(tab + off, P.M1, k * 32 + lane, c6);
+    }
+    const real g = horner5(c6, t);
+    acc[k][0] = fma(r0, g, acc[k][0]);
+    acc[k][1] = fma(r1, g, acc[k][1]);
+    acc[k][2] = fma(r2, g, acc[k][2]);
+    acc[k][3] = fma(r3, g, acc[k][3]);
+  }
 }
 
 // One atom: T_i into P.T (the whole warp takes part).
@@ -135,31 +180,21 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     __syncwarp();
     const int cnt = min(32, nv - base);
     if (Q > 0) {
-      for (int u = 0; u < cnt; ++u) {  // uniform: every lane on neighbour u
-        const int off = st.off[u];
-        const real *__restrict__ cp = tab + off;  // the interval's coefficient block
-        if (kCache && off != cur) {  // uniform branch
-          cur = off;
-#pragma unroll
-          for (int r = 0; r < Q; ++r) ld6(cp, P.M1, r * 32 + lane, cf[r]);
+      if constexpr (kCache) {
+        // f32: four staged neighbours per iteration through 16-byte shared loads
+        int u = 0;
+        for (; u + 4 <= cnt; u += 4) {
+          const float4 t4 = *reinterpret_cast<const float4 *>(&st.t[u]);
+          const int4 o4 = *reinterpret_cast<const int4 *>(&st.off[u]);
+          fwd_neighbour<real, Q, true>(P, tab, lane, o4.x, t4.x, st.r[u], acc, cf, cur);
+          fwd_neighbour<real, Q, true>(P, tab, lane, o4.y, t4.y, st.r[u + 1], acc, cf, cur);
+          fwd_neighbour<real, Q, true>(P, tab, lane, o4.z, t4.z, st.r[u + 2], acc, cf, cur);
+          fwd_neighbour<real, Q, true>(P, tab, lane, o4.w, t4.w, st.r[u + 3], acc, cf, cur);
         }
-        const real t = st.t[u];
-        const real r0 = st.r[u][0], r1 = st.r[u][1], r2 = st.r[u][2], r3 = st.r[u][3];
-#pragma unroll
-        for (int r = 0; r < Q; ++r) {
-          real c6[6];
-          if (kCache) {
-#pragma unroll
-            for (int e = 0; e < 6; ++e) c6[e] = cf[kCache ? r : 0][e];
-          } else {
-            ld6(cp, P.M1, r * 32 + lane, c6);
-          }
-          const real g = horner5(c6, t);
-          acc[r][0] = fma(r0, g, acc[r][0]);
-          acc[r][1] = fma(r1, g, acc[r][1]);
-          acc[r][2] = fma(r2, g, acc[r][2]);
-          acc[r][3] = fma(r3, g, acc[r][3]);
-        }
+        for (; u < cnt; ++u) fwd_neighbour<real, Q, true>(P, tab, lane, st.off[u], st.t[u], st.r[u], acc, cf, cur);
+      } else {
+        for (int u = 0; u < cnt; ++u)  // uniform: every lane on neighbour u
+          fwd_neighbour<real, Q, false>(P, tab, lane, st.off[u], st.t[u], st.r[u], acc, cf, cur);
       }
     }
     if (P.RR > 0) {

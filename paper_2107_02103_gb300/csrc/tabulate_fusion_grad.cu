@@ -178,10 +178,13 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 // L lanes of a row read L consecutive channels of the row's interval (three
 // contiguous runs of 8*L bytes in the pair-planar block), and rows that share
 // an interval -- most neighbours next to each other in distance order -- hit
-// the same sectors.
-// Each lane keeps dT for its channels in registers; the five per-row sums
-// (ds, dR~[0..3]) meet in a log2(L)-level shuffle reduction per row, which
-// is amortised over the M1/L channel rounds of that row.
+// the same sectors.  Each warp prepares 32 rows at a time (segment lookup,
+// interval search, R~ load) spread over its lanes, and the row groups read
+// them back as shared-memory broadcasts.  dT_i sits in shared memory as
+// [M1][4] (one 16-byte load per channel round), which keeps the register
+// count low enough for the occupancy that hides the coefficient loads.  The
+// five per-row sums (ds, dR~[0..3]) meet in a log2(L)-level shuffle
+// reduction per row, amortised over the M1/L channel rounds of that row.
 constexpr int kGradF32Warps = 4;
 
 struct GradParamsF32 {
@@ -200,13 +203,24 @@ struct GradParamsF32 {
   float inv_nnei;
 };
 
+// Per-warp staging of 32 valid rows: prepared once per row, lane-distributed,
+// then read by the row groups as shared-memory broadcasts.
+struct alignas(16) RowStage {
+  float4 r[32];     // R~ rows
+  float t[32];      // local variable t
+  int32_t blk[32];  // element offset of the interval's coefficient block (centre type's tables)
+  int32_t row[32];  // row index, with bit 30 set when s was clamped (ds = 0)
+};
+
 template <int L, int R>
 __global__ void __launch_bounds__(kGradF32Warps * 32) grad_f32_kernel(const GradParamsF32 P) {
-  constexpr int RPW = 32 / L;                  // rows per warp instruction
-  constexpr int STEP = kGradF32Warps * RPW;    // rows per block iteration
+  constexpr int RPW = 32 / L;  // rows per warp instruction
+  constexpr int kClamped = 1 << 30;
+  __shared__ RowStage stage[kGradF32Warps];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int grp = lane / L, q = lane % L;
   const int64_t i = blockIdx.x;  // one atom per block
+  RowStage &st = stage[w];
 
   int nvb[DP_MAX_TYPES];
   int nv = 0;
@@ -219,24 +233,24 @@ __global__ void __launch_bounds__(kGradF32Warps * 32) grad_f32_kernel(const Grad
   }
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   const float *__restrict__ tab = P.table + (size_t)alpha * P.ntypes * P.pair_stride;
+  float *__restrict__ ds_i = P.ds + i * P.nnei;
+  float *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
 
-  float dt[R][4];  // dT_i for channels q, q + L, ...
-  const float *__restrict__ dTi = P.dT + i * 4 * P.M1;
-#pragma unroll
-  for (int r = 0; r < R; ++r) {
-    const int m = q + L * r;
-    const bool ok = m < P.M1;
-#pragma unroll
-    for (int k = 0; k < 4; ++k) dt[r][k] = ok ? __ldg(dTi + k * P.M1 + m) : 0.0f;
+  // dT_i transposed to [L*R][4] in shared memory (zero past M1): one 16-byte load per channel round
+  __shared__ float4 dts[L * R];
+  {
+    const float *__restrict__ dTi = P.dT + i * 4 * P.M1;
+    for (int m = threadIdx.x; m < L * R; m += kGradF32Warps * 32)
+      dts[m] = m < P.M1 ? make_float4(__ldg(dTi + m), __ldg(dTi + P.M1 + m), __ldg(dTi + 2 * P.M1 + m),
+                                      __ldg(dTi + 3 * P.M1 + m))
+                        : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
   }
+  __syncthreads();
 
-  for (int vb = w * RPW; vb < nv; vb += STEP) {  // warp-uniform
-    const int v = vb + grp;
-    const bool act = v < nv;
-    float a_ds = 0.0f, a_0 = 0.0f, a_1 = 0.0f, a_2 = 0.0f, a_3 = 0.0f;
-    int row = 0;
-    bool clamped = false;
-    if (act) {
+  for (int base = 32 * w; base < nv; base += 32 * kGradF32Warps) {  // warp-uniform
+    const int cnt = min(32, nv - base);
+    if (lane < cnt) {  // stage row base + lane
+      const int v = base + lane;
       int b = 0, cum = 0, lim = nvb[0], off = 0;
 #pragma unroll
       for (int c = 1; c < DP_MAX_TYPES; ++c)
@@ -246,51 +260,69 @@ __global__ void __launch_bounds__(kGradF32Warps * 32) grad_f32_kernel(const Grad
           lim += nvb[c];
           off += P.sel[c - 1];
         }
-      row = off + (v - cum);
+      const int row = off + (v - cum);
       const Vec4<float> rr = ld4(P.Rt + (i * P.nnei + row) * 4);
       float t;
+      bool clamped;
       const int l = locate(P.geom, __ldg(P.s + i * P.nnei + row), t, clamped);
-      const float *__restrict__ cp = tab + (size_t)(b * P.geom.nint + l) * P.M1 * 6;
+      st.r[lane] = make_float4(rr.x, rr.y, rr.z, rr.w);
+      st.t[lane] = t;
+      st.blk[lane] = (b * P.geom.nint + l) * P.M1 * 6;
+      st.row[lane] = row | (clamped ? kClamped : 0);
+    }
+    __syncwarp();
+    for (int u0 = 0; u0 < cnt; u0 += RPW) {  // warp-uniform
+      const int u = u0 + grp;
+      const bool act = u < cnt;
+      float a_ds = 0.0f, a_0 = 0.0f, a_1 = 0.0f, a_2 = 0.0f, a_3 = 0.0f;
+      if (act) {
+        const float4 rr = st.r[u];
+        const float t = st.t[u];
+        const float2 *q0 = reinterpret_cast<const float2 *>(tab + st.blk[u]) + q;
+        const float2 *q1 = q0 + P.M1, *q2 = q1 + P.M1;
 #pragma unroll
-      for (int r = 0; r < R; ++r) {
-        if (r < R - 1 || q + L * r < P.M1) {
-          float cf[6];
-          ld6(cp, P.M1, q + r * L, cf);
-          float p = fmaf(cf[0], t, cf[1]);
-          float dp = cf[0];
-          dp = fmaf(dp, t, p);
-          p = fmaf(p, t, cf[2]);
-          dp = fmaf(dp, t, p);
-          p = fmaf(p, t, cf[3]);
-          dp = fmaf(dp, t, p);
-          p = fmaf(p, t, cf[4]);
-          dp = fmaf(dp, t, p);
-          p = fmaf(p, t, cf[5]);
-          float rm = dt[r][0] * rr.x;
-          rm = fmaf(dt[r][1], rr.y, rm);
-          rm = fmaf(dt[r][2], rr.z, rm);
-          rm = fmaf(dt[r][3], rr.w, rm);
-          a_ds = fmaf(rm, dp, a_ds);
-          a_0 = fmaf(dt[r][0], p, a_0);
-          a_1 = fmaf(dt[r][1], p, a_1);
-          a_2 = fmaf(dt[r][2], p, a_2);
-          a_3 = fmaf(dt[r][3], p, a_3);
+        for (int r = 0; r < R; ++r) {
+          if (r < R - 1 || q + L * r < P.M1) {
+            const float2 ab = __ldg(q0 + L * r), cd = __ldg(q1 + L * r), ef = __ldg(q2 + L * r);
+            const float4 d = dts[q + L * r];
+            float p = fmaf(ab.x, t, ab.y);
+            float dp = ab.x;
+            dp = fmaf(dp, t, p);
+            p = fmaf(p, t, cd.x);
+            dp = fmaf(dp, t, p);
+            p = fmaf(p, t, cd.y);
+            dp = fmaf(dp, t, p);
+            p = fmaf(p, t, ef.x);
+            dp = fmaf(dp, t, p);
+            p = fmaf(p, t, ef.y);
+            float rm = d.x * rr.x;
+            rm = fmaf(d.y, rr.y, rm);
+            rm = fmaf(d.z, rr.z, rm);
+            rm = fmaf(d.w, rr.w, rm);
+            a_ds = fmaf(rm, dp, a_ds);
+            a_0 = fmaf(d.x, p, a_0);
+            a_1 = fmaf(d.y, p, a_1);
+            a_2 = fmaf(d.z, p, a_2);
+            a_3 = fmaf(d.w, p, a_3);
+          }
         }
       }
-    }
 #pragma unroll
-    for (int sh = L / 2; sh > 0; sh >>= 1) {
-      a_ds += __shfl_xor_sync(0xffffffffu, a_ds, sh);
-      a_0 += __shfl_xor_sync(0xffffffffu, a_0, sh);
-      a_1 += __shfl_xor_sync(0xffffffffu, a_1, sh);
-      a_2 += __shfl_xor_sync(0xffffffffu, a_2, sh);
-      a_3 += __shfl_xor_sync(0xffffffffu, a_3, sh);
+      for (int sh = L / 2; sh > 0; sh >>= 1) {
+        a_ds += __shfl_xor_sync(0xffffffffu, a_ds, sh);
+        a_0 += __shfl_xor_sync(0xffffffffu, a_0, sh);
+        a_1 += __shfl_xor_sync(0xffffffffu, a_1, sh);
+        a_2 += __shfl_xor_sync(0xffffffffu, a_2, sh);
+        a_3 += __shfl_xor_sync(0xffffffffu, a_3, sh);
+      }
+      if (act && q == 0) {
+        const int rw = st.row[u];
+        const int row = rw & (kClamped - 1);
+        ds_i[row] = (rw & kClamped) ? 0.0f : a_ds * P.inv_nnei;
+        st4(dR_i + (size_t)row * 4, a_0 * P.inv_nnei, a_1 * P.inv_nnei, a_2 * P.inv_nnei, a_3 * P.inv_nnei);
+      }
     }
-    if (act && q == 0) {
-      P.ds[i * P.nnei + row] = clamped ? 0.0f : a_ds * P.inv_nnei;
-      st4(P.dRt + (i * P.nnei + row) * 4, a_0 * P.inv_nnei, a_1 * P.inv_nnei, a_2 * P.inv_nnei,
-          a_3 * P.inv_nnei);
-    }
+    __syncwarp();
   }
 
   // padding rows of this atom, packed over the segments' padded tails
@@ -305,8 +337,8 @@ __global__ void __launch_bounds__(kGradF32Warps * 32) grad_f32_kernel(const Grad
         nvb_b = nvb[c];
       }
     const int row = off + nvb_b + (pv - cum);
-    P.ds[i * P.nnei + row] = 0.0f;
-    st4(P.dRt + (i * P.nnei + row) * 4, 0.0f, 0.0f, 0.0f, 0.0f);
+    ds_i[row] = 0.0f;
+    st4(dR_i + (size_t)row * 4, 0.0f, 0.0f, 0.0f, 0.0f);
   }
 }
 

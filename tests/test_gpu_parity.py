@@ -254,3 +254,38 @@ def test_paper_sized(name, kw, dtype, nsample):
         atoms[0], atoms[-1] = 0, w.nloc - 1
     ref = run_oracle(w, dtype, atoms=atoms)
     assert_parity(got, ref, dtype, atoms=atoms)
+
+
+@pytest.mark.parametrize("pad", [0.2, 0.3, 0.4, 0.5])
+def test_alcumg_padding_sweep(pad):
+    """The Al-Cu-Mg-like padding sweep (10-60 % empty rows), small cells, every atom."""
+    w = workload("alcumg", pad=pad, cells=(6, 6, 6))
+    assert_parity(run_product(w, torch.float64), run_oracle(w, torch.float64), torch.float64)
+
+
+@pytest.mark.parametrize("dtype", [torch.float64, torch.float32])
+def test_water_large_sampled(dtype):
+    """1,048,576 atoms in the benchmark's launch configuration; 256 sampled atoms (first and last
+    included) gathered on the device and compared with the oracle; plus the identity
+    <dR~, R~> = <dT, T> over ALL atoms, which holds at any size."""
+    dpc = lib()
+    w = workload("water_large")
+    model = product_model(w, dtype)
+    x = to_dev(w, dtype)
+    T = dpc.dp_tabulate_fusion_fwd(model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
+    D = dpc.dp_descriptor_contract(T, w.M2)
+    ds, dRt = dpc.dp_tabulate_fusion_grad(model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel,
+                                          x["dT"])
+    torch.cuda.synchronize()
+    rng = np.random.default_rng(7)
+    atoms = np.sort(rng.choice(w.nloc, 256, replace=False))
+    atoms[0], atoms[-1] = 0, w.nloc - 1
+    idx = torch.from_numpy(atoms).cuda()
+    got = {k: v.index_select(0, idx).double().cpu().numpy() for k, v in dict(T=T, D=D, ds=ds, dRt=dRt).items()}
+    ref = run_oracle(w, dtype, atoms=atoms)
+    assert_parity(got, ref, dtype)
+    lhs = float((dRt.double() * x["Rt"].double()).sum())
+    rhs = float((x["dT"].double() * T.double()).sum())
+    assert abs(lhs - rhs) <= TOL[dtype] * 10 * max(1.0, abs(rhs)), (lhs, rhs)
+    del T, D, ds, dRt, x, model
+    torch.cuda.empty_cache()
