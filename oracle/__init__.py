@@ -89,6 +89,8 @@ def load(path: str | None = None):
     lib.or_grad.restype = ctypes.c_int
     lib.or_descriptor.argtypes = [P, i64, ctypes.c_int, ctypes.c_int, P]
     lib.or_descriptor.restype = None
+    lib.or_descriptor_grad.argtypes = [P, P, i64, ctypes.c_int, ctypes.c_int, P]
+    lib.or_descriptor_grad.restype = None
     lib.or_embed_rows.argtypes = [P, ctypes.POINTER(Info), P, P, ctypes.c_int, ctypes.c_int, P, ctypes.c_int, P,
                                   i64, P, P]
     lib.or_embed_rows.restype = None
@@ -232,6 +234,15 @@ class Oracle:
         D = np.empty((n, M, M2))
         self.lib.or_descriptor(_p(T), n, M, int(M2), _p(D))
         return D
+
+    def descriptor_grad(self, T, dD):
+        T, dD = _c(T, np.float64), _c(dD, np.float64)
+        n, four, M = T.shape
+        M2 = dD.shape[-1]
+        assert dD.shape == (n, M, M2)
+        dT = np.empty_like(T)
+        self.lib.or_descriptor_grad(_p(T), _p(dD), n, M, int(M2), _p(dT))
+        return dT
 
     def embed_rows(self, table, info, s, atype, sel, atoms=None, deriv=False):
         table, s = (_c(a, np.float64) for a in (table, s))

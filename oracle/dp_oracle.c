@@ -20,7 +20,8 @@
  *     the table only for valid neighbours (Sec. II, kernel fusion and the
  *     skip of padded rows), in double;
  *   - its gradient dE/ds and dE/dR~ from an upstream dE/dT, in double;
- *   - the descriptor D_i = S_i (S_i^<)^T with S_i = T_i^T (Sec. II), in double;
+ *   - the descriptor D_i = S_i (S_i^<)^T with S_i = T_i^T (Sec. II), and its
+ *     gradient dE/dT from an upstream dE/dD, in double;
  *   - the embedding matrix G itself, through the table or straight from the
  *     net, for the explicit and uncompressed comparisons.
  *
@@ -437,6 +438,28 @@ void or_descriptor(const double *T, int64_t n, int M, int M2, double *D) {
         double v = 0.0;
         for (int k = 0; k < 4; ++k) v += Ta[k * M + m] * Ta[k * M + q];
         Da[(size_t)m * M2 + q] = v;
+      }
+  }
+}
+
+/*
+ * Gradient of the descriptor.  D[m][n] = sum_k T[k][m] T[k][n] (n < M2) is
+ * quadratic in T, so for an upstream dD = dE/dD ([n][M][M2] like D):
+ *   dE/dT[k][m] = sum_{n<M2} dD[m][n] T[k][n]  +  [m < M2] sum_{m'} dD[m'][m] T[k][m']
+ * (the first term through the S_i factor, the second through S_i^<).
+ */
+void or_descriptor_grad(const double *T, const double *dD, int64_t n, int M, int M2, double *dT) {
+  for (int64_t a = 0; a < n; ++a) {
+    const double *Ta = T + (size_t)a * 4 * M;
+    const double *Ga = dD + (size_t)a * M * M2;
+    double *dTa = dT + (size_t)a * 4 * M;
+    for (int k = 0; k < 4; ++k)
+      for (int m = 0; m < M; ++m) {
+        double v = 0.0;
+        for (int q = 0; q < M2; ++q) v += Ga[(size_t)m * M2 + q] * Ta[k * M + q];
+        if (m < M2)
+          for (int mp = 0; mp < M; ++mp) v += Ga[(size_t)mp * M2 + m] * Ta[k * M + mp];
+        dTa[k * M + m] = v;
       }
   }
 }

@@ -430,7 +430,30 @@ def pin_descriptor(o):
     assert _rel(D3, D) < 1e-13
 
 
+def pin_descriptor_grad(o):
+    """dE/dT of D = S (S^<)^T: exact central differences (D is quadratic), the Euler identity
+    <dT, T> = 2 <dD, D>, and the matrix form dS = dD S^< + [dD^T S in the first M2 rows] by matmul."""
+    rng = np.random.default_rng(21)
+    n, M, M2 = 5, 13, 4
+    T = rng.normal(size=(n, 4, M))
+    dD = rng.normal(size=(n, M, M2))
+    dT = o.descriptor_grad(T, dD)
+    L = lambda TT: float(np.sum(dD * o.descriptor(TT, M2)))  # noqa: E731
+    assert abs(float(np.sum(dT * T)) - 2.0 * L(T)) <= 1e-12 * max(1.0, abs(L(T)))
+    for (a, k, m) in ((0, 0, 0), (1, 2, 3), (2, 3, 12), (4, 1, 7), (3, 0, 4)):
+        Tp, Tm = T.copy(), T.copy()
+        Tp[a, k, m] += 0.5
+        Tm[a, k, m] -= 0.5
+        fd = (L(Tp) - L(Tm)) / 1.0
+        assert abs(dT[a, k, m] - fd) <= 1e-11 * max(1.0, abs(fd)), (a, k, m, dT[a, k, m], fd)
+    for a in range(n):
+        S = T[a].T
+        dS = dD[a] @ S[:M2]
+        dS[:M2] += dD[a].T @ S
+        assert _rel(dT[a], dS.T) < 1e-14
+
+
 ALL_PINS = [pin_net_skip_wiring, pin_net_single_neuron, pin_net_derivatives_fd, pin_table_info, pin_locate,
             pin_table_nodes, pin_table_quintic_exact, pin_table_sin_bound, pin_compressed_vs_net,
             pin_fwd_brute_force, pin_fwd_constant_G, pin_fwd_vs_explicit_G, pin_fwd_padding, pin_fwd_symmetries,
-            pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor]
+            pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor, pin_descriptor_grad]

@@ -42,6 +42,10 @@ MUTANTS = [
      "for (int j = 0; j < sel[beta]; ++j) {\n        int r = off[beta] + j;"),
     ("grad: clamp ignored", "double dg = clamped ? 0.0 : poly_dg(c, t);", "double dg = poly_dg(c, t);"),
     ("descriptor: wrong k on S^<", "v += Ta[k * M + m] * Ta[k * M + q];", "v += Ta[k * M + m] * Ta[((k + 1) % 4) * M + q];"),
+    ("descriptor grad: S^< term dropped", "if (m < M2)\n          for (int mp = 0; mp < M; ++mp)",
+     "if (m < 0)\n          for (int mp = 0; mp < M; ++mp)"),
+    ("descriptor grad: transposed dD", "v += Ga[(size_t)mp * M2 + m] * Ta[k * M + mp];",
+     "v += Ga[(size_t)m * M2 + (mp % M2)] * Ta[k * M + mp];"),
 ]
 
 
