@@ -159,6 +159,23 @@ int dp_tabulate_fusion_fwd_f32(const float *table, const dp_table_info *info, co
                                const int32_t *sel, int M1, float *T, void *stream);
 
 /*
+ * Forward and descriptor in one pass (Sec. II: T_i, then D_i = S_i (S_i^<)^T
+ * with S_i = T_i^T): the same T as dp_tabulate_fusion_fwd_* and
+ *   D[i][m][n] = sum_k T[i][k][m] * T[i][k][n],  n < M2,
+ * formed while T_i is still on chip (no second read of T).  Arguments as
+ * dp_tabulate_fusion_fwd_* plus M2 and D [nloc][M1][M2] (output).
+ * Extra errors: DP_ERR_SHAPE (M2 < 1 or M2 > M1), DP_ERR_UNSUPPORTED (M2 > 32).
+ */
+int dp_tabulate_fusion_fwd_descriptor_f64(const double *table, const dp_table_info *info, const double *s,
+                                          const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                          int nnei, int ntypes, const int32_t *sel, int M1, int M2, double *T,
+                                          double *D, void *stream);
+int dp_tabulate_fusion_fwd_descriptor_f32(const float *table, const dp_table_info *info, const float *s,
+                                          const float *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                          int nnei, int ntypes, const int32_t *sel, int M1, int M2, float *T,
+                                          float *D, void *stream);
+
+/*
  * Backward of the fused forward (Sec. II: the compressed model serves both
  * the forward and the backward propagation, which yields forces and virials).
  * Given dT = dE/dT_i:
@@ -188,6 +205,20 @@ int dp_tabulate_fusion_grad_f32(const float *table, const dp_table_info *info, c
  */
 int dp_descriptor_contract_f64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream);
 int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, float *D, void *stream);
+
+/*
+ * Backward of the descriptor (Sec. II: D_i = S_i (S_i^<)^T is quadratic in
+ * S_i = T_i^T; the backward propagation of the compressed model runs through
+ * it before reaching the tabulated embedding).  Given dD = dE/dD:
+ *   dT[i][k][m] = sum_{n<M2} dD[i][m][n] T[i][k][n] + [m < M2] sum_{m'} dD[i][m'][m] T[i][k][m']
+ *   T [nloc][4][M1], dD [nloc][M1][M2] inputs;  dT [nloc][4][M1] output, fully
+ *   overwritten (feed it to dp_tabulate_fusion_grad_*).
+ * Errors, limits and the nloc == 0 rule as dp_descriptor_contract_*.
+ */
+int dp_descriptor_contract_grad_f64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,
+                                    void *stream);
+int dp_descriptor_contract_grad_f32(const float *T, const float *dD, int64_t nloc, int M1, int M2, float *dT,
+                                    void *stream);
 
 #ifdef __cplusplus
 }

@@ -60,12 +60,18 @@ _SIGS = {
                                     _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_fwd_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
                                     _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_descriptor_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                               ctypes.c_int, ctypes.c_int, _P, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_descriptor_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                               ctypes.c_int, ctypes.c_int, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
                                      _P, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
                                      _P, _P, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_f64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_f32": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_descriptor_contract_grad_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_descriptor_contract_grad_f32": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
 }
 for _name, (_args, _res) in _SIGS.items():
     _fn = getattr(_lib, _name)
@@ -188,6 +194,22 @@ def dp_tabulate_fusion_fwd(table, info: dp_table_info, s, Rt, nvalid, atype, sel
     return T
 
 
+def dp_tabulate_fusion_fwd_descriptor(table, info: dp_table_info, s, Rt, nvalid, atype, sel, M2: int, out=None):
+    """(T [nloc][4][M1], D [nloc][M1][M2]) in one pass: T as dp_tabulate_fusion_fwd, D = S (S^<)^T."""
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
+                                                                                      sel)
+    if out is None:
+        T = torch.empty((nloc, 4, M1), dtype=dtype, device=s.device)
+        D = torch.empty((nloc, M1, int(M2)), dtype=dtype, device=s.device)
+    else:
+        T = _dev(out[0], "T", dtype, (nloc, 4, M1))
+        D = _dev(out[1], "D", dtype, (nloc, M1, int(M2)))
+    fn = getattr(_lib, f"dp_tabulate_fusion_fwd_descriptor_{_suffix(dtype)}")
+    _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
+              selc, M1, int(M2), _ptr(T), _ptr(D), _stream(s)))
+    return T, D
+
+
 def dp_tabulate_fusion_grad(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None):
     """(ds [nloc][nnei], dRt [nloc][nnei][4]) from dT = dE/dT [nloc][4][M1]."""
     dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
@@ -216,6 +238,22 @@ def dp_descriptor_contract(T, M2: int, out=None) -> torch.Tensor:
     fn = getattr(_lib, f"dp_descriptor_contract_{_suffix(T.dtype)}")
     _check(fn(_ptr(T), nloc, M1, int(M2), _ptr(D), _stream(T)))
     return D
+
+
+def dp_descriptor_contract_grad(T, dD, out=None) -> torch.Tensor:
+    """dT [nloc][4][M1] = dE/dT from dD = dE/dD [nloc][M1][M2] through D = S (S^<)^T."""
+    T = _dev(T, "T", None)
+    nloc, four, M1 = (int(x) for x in T.shape)
+    if four != 4:
+        raise ValueError("T must be [nloc][4][M1]")
+    dD = _dev(dD, "dD", T.dtype)
+    if dD.dim() != 3 or dD.shape[0] != nloc or dD.shape[1] != M1:
+        raise ValueError("dD must be [nloc][M1][M2]")
+    M2 = int(dD.shape[2])
+    dT = torch.empty_like(T) if out is None else _dev(out, "out", T.dtype, T.shape)
+    fn = getattr(_lib, f"dp_descriptor_contract_grad_{_suffix(T.dtype)}")
+    _check(fn(_ptr(T), _ptr(dD), nloc, M1, M2, _ptr(dT), _stream(T)))
+    return dT
 
 
 @dataclass

@@ -43,6 +43,73 @@ __global__ void __launch_bounds__(kDescWarps * 32)
   }
 }
 
+// Backward of the descriptor: D[m][n] = sum_k T[k][m] T[k][n] (n < M2) is
+// quadratic in T, so for dD = dE/dD
+//   dT[k][m] = sum_{n<M2} dD[m][n] T[k][n] + [m < M2] sum_{m'} dD[m'][m] T[k][m'].
+// One warp per atom.  The 4*M1 (m, k) pairs of the first term are spread
+// over the lanes (lane l: pairs l, l + 32, ...; 8 rows x 4 k per step, so the
+// dD row reads of a step are 8 rows of M2 values); the 4*M2 (k, m) pairs of
+// the second term walk the M1 rows of dD, each step reading one row.  Both
+// terms meet in shared memory and dT is written coalesced.
+template <typename real>
+__global__ void __launch_bounds__(kDescWarps * 32)
+    descriptor_grad_kernel(const real *__restrict__ T, const real *__restrict__ dD, int64_t nloc, int M1, int M2,
+                           real *__restrict__ dT) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t i = (int64_t)blockIdx.x * kDescWarps + w;
+  if (i >= nloc) return;  // warp-uniform; no block-wide barrier below
+  real *Ts = reinterpret_cast<real *>(smem_raw) + (size_t)w * 8 * M1;  // [4][M1]
+  real *Gs = Ts + 4 * M1;                                              // [4][M1] partial dT
+  const real *__restrict__ Ti = T + i * 4 * M1;
+  const real *__restrict__ Di = dD + i * (int64_t)M1 * M2;
+  for (int e = lane; e < 4 * M1; e += 32) Ts[e] = __ldg(Ti + e);
+  __syncwarp();
+  // first term, pairs p = 4 m + k
+  for (int p = lane; p < 4 * M1; p += 32) {
+    const int m = p >> 2, k = p & 3;
+    const real *__restrict__ row = Di + (size_t)m * M2;
+    const real *tk = Ts + k * M1;
+    real v = real(0);
+    for (int n = 0; n < M2; ++n) v = fma(__ldg(row + n), tk[n], v);
+    Gs[k * M1 + m] = v;
+  }
+  __syncwarp();
+  // second term, pairs p = M2 k + m (m < M2)
+  for (int p = lane; p < 4 * M2; p += 32) {
+    const int k = p / M2, m = p - k * M2;
+    const real *tk = Ts + k * M1;
+    real v = real(0);
+    for (int mp = 0; mp < M1; ++mp) v = fma(__ldg(Di + (size_t)mp * M2 + m), tk[mp], v);
+    Gs[k * M1 + m] += v;
+  }
+  __syncwarp();
+  real *__restrict__ dTi = dT + i * 4 * M1;
+  for (int e = lane; e < 4 * M1; e += 32) dTi[e] = Gs[e];
+}
+
+template <typename real>
+int descriptor_grad(const real *T, const real *dD, int64_t nloc, int M1, int M2, real *dT, void *stream) {
+  clear_error();
+  if (nloc < 0 || M1 < 1 || M2 < 1 || M2 > M1)
+    return set_error(DP_ERR_SHAPE, "need nloc >= 0 and 1 <= M2 <= M1 (nloc %lld, M1 %d, M2 %d)", (long long)nloc, M1,
+                     M2);
+  if (M1 > 4096) return set_error(DP_ERR_UNSUPPORTED, "M1 = %d > 4096", M1);
+  if (nloc == 0) return DP_OK;
+  if (!T || !dD || !dT) return set_error(DP_ERR_NULL, "T, dD or dT is NULL");
+  const int64_t blocks = (nloc + kDescWarps - 1) / kDescWarps;
+  if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
+  const size_t smem = (size_t)kDescWarps * 8 * M1 * sizeof(real);
+  if (smem > 48 * 1024) {
+    const cudaError_t e = cudaFuncSetAttribute(descriptor_grad_kernel<real>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_descriptor_contract_grad: %s", cudaGetErrorString(e));
+  }
+  descriptor_grad_kernel<real>
+      <<<(unsigned)blocks, kDescWarps * 32, smem, (cudaStream_t)stream>>>(T, dD, nloc, M1, M2, dT);
+  return launch_status("dp_descriptor_contract_grad");
+}
+
 template <typename real>
 int descriptor(const real *T, int64_t nloc, int M1, int M2, real *D, void *stream) {
   clear_error();
@@ -76,6 +143,16 @@ int dp_descriptor_contract_f64(const double *T, int64_t nloc, int M1, int M2, do
 
 int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, float *D, void *stream) {
   return dpc::descriptor<float>(T, nloc, M1, M2, D, stream);
+}
+
+int dp_descriptor_contract_grad_f64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,
+                                    void *stream) {
+  return dpc::descriptor_grad<double>(T, dD, nloc, M1, M2, dT, stream);
+}
+
+int dp_descriptor_contract_grad_f32(const float *T, const float *dD, int64_t nloc, int M1, int M2, float *dT,
+                                    void *stream) {
+  return dpc::descriptor_grad<float>(T, dD, nloc, M1, M2, dT, stream);
 }
 
 }  // extern "C"

@@ -45,10 +45,12 @@ struct FwdParams {
   const int32_t *__restrict__ nvalid;
   const int32_t *__restrict__ atype;
   real *__restrict__ T;
+  real *__restrict__ D;  // optional fused descriptor output [nloc][M1][M2] (NULL: T only)
   typename GeomOf<real>::type geom;
   int64_t nloc;
   int32_t nnei, ntypes, M1, pair_stride;  // pair_stride = nint * M1 * 6
   int32_t RR, PK;                          // remainder channels, neighbours per packed round
+  int32_t M2;                              // descriptor width when D is set (M2 <= 32)
   int32_t sel[DP_MAX_TYPES];
   real inv_nnei;
 };
@@ -71,33 +73,34 @@ __device__ __forceinline__ real horner5(const real c[6], real t) {
   return fma(g, t, c[5]);
 }
 
+// The coefficients of this lane's Q channels of the interval block at `off`.
+template <typename real, int Q>
+__device__ __forceinline__ void fwd_load_cf(const FwdParams<real> &P, const real *__restrict__ tab, const int lane,
+                                            const int off, real (&cf)[Q > 0 ? Q : 1][6]) {
+  using V2 = typename std::conditional<sizeof(real) == 8, double2, float2>::type;
+  const V2 *q0 = reinterpret_cast<const V2 *>(tab + off) + lane;
+  const V2 *q1 = q0 + P.M1, *q2 = q1 + P.M1;
+#pragma unroll
+  for (int k = 0; k < Q; ++k) {
+    const V2 x = __ldg(q0 + 32 * k), y = __ldg(q1 + 32 * k), z = __ldg(q2 + 32 * k);
+    cf[k][0] = x.x;
+    cf[k][1] = x.y;
+    cf[k][2] = y.x;
+    cf[k][3] = y.y;
+    cf[k][4] = z.x;
+    cf[k][5] = z.y;
+  }
+}
+
 // One neighbour (interval block offset `off`, local t, R~ row r) folded into
-// the lane's Q channel rounds.  kCache: the coefficients of the interval in
-// use stay in cf across neighbours that share it (the branch is uniform).
+// the lane's Q channel rounds.  kCache: cf already holds the interval's
+// coefficients; otherwise they are loaded here, round by round.
 template <typename real, int Q, bool kCache>
 __device__ __forceinline__ void fwd_neighbour(const FwdParams<real> &P, const real *__restrict__ tab, const int lane,
                                               const int off, const real t, const real *r,
                                               real (&acc)[Q > 0 ? Q : 1][4], real (&cf)[kCache && Q > 0 ? Q : 1][6],
                                               int &cur) {
   const real r0 = r[0], r1 = r[1], r2 = r[2], r3 = r[3];
-  if (kCache) {
-    if (off != cur) {
-      cur = off;
-      using V2 = typename std::conditional<sizeof(real) == 8, double2, float2>::type;
-      const V2 *q0 = reinterpret_cast<const V2 *>(tab + off) + lane;
-      const V2 *q1 = q0 + P.M1, *q2 = q1 + P.M1;
-#pragma unroll
-      for (int k = 0; k < Q; ++k) {
-        const V2 x = __ldg(q0 + 32 * k), y = __ldg(q1 + 32 * k), z = __ldg(q2 + 32 * k);
-        cf[kCache ? k : 0][0] = x.x;
-        cf[kCache ? k : 0][1] = x.y;
-        cf[kCache ? k : 0][2] = y.x;
-        cf[kCache ? k : 0][3] = y.y;
-        cf[kCache ? k : 0][4] = z.x;
-        cf[kCache ? k : 0][5] = z.y;
-      }
-    }
-  }
 #pragma unroll
   for (int k = 0; k < Q; ++k) {
     real c6[6];
@@ -115,7 +118,68 @@ __device__ __forceinline__ void fwd_neighbour(const FwdParams<real> &P, const re
   }
 }
 
-// One atom: T_i into P.T (the whole warp takes part).
+// D_i = S_i (S_i^<)^T from T_i still in registers (Sec. II, the descriptor):
+// D[m][n] = sum_k T[k][m] T[k][n], n < M2 <= 32.  T[k][n] for n < M2 is held
+// by round 0, lane n (or, when M1 < 32, by remainder lane n) and reaches the
+// other lanes by shuffles.  Main-round rows m = 32 r + lane are computed by
+// their owners; the RR remainder rows are spread as (row, n) pairs over all
+// 32 lanes so that no FMA instruction runs with a handful of lanes.
+template <typename real, int Q>
+__device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, const real (&acc)[Q > 0 ? Q : 1][4],
+                                                   real rq0, real rq1, real rq2, real rq3, const int lane,
+                                                   const int64_t i) {
+  const int M1 = P.M1, M2 = P.M2;
+  real *__restrict__ Di = P.D + i * (int64_t)M1 * M2;
+  for (int n = 0; n < M2; ++n) {  // uniform
+    real t0, t1, t2, t3;
+    if (Q > 0) {
+      t0 = __shfl_sync(0xffffffffu, acc[0][0], n);
+      t1 = __shfl_sync(0xffffffffu, acc[0][1], n);
+      t2 = __shfl_sync(0xffffffffu, acc[0][2], n);
+      t3 = __shfl_sync(0xffffffffu, acc[0][3], n);
+    } else {
+      t0 = __shfl_sync(0xffffffffu, rq0, n);
+      t1 = __shfl_sync(0xffffffffu, rq1, n);
+      t2 = __shfl_sync(0xffffffffu, rq2, n);
+      t3 = __shfl_sync(0xffffffffu, rq3, n);
+    }
+#pragma unroll
+    for (int r = 0; r < Q; ++r) {
+      real d = acc[r][0] * t0;
+      d = fma(acc[r][1], t1, d);
+      d = fma(acc[r][2], t2, d);
+      d = fma(acc[r][3], t3, d);
+      Di[(size_t)(r * 32 + lane) * M2 + n] = d;
+    }
+  }
+  const int npairs = P.RR * M2;
+  for (int p0 = 0; p0 < npairs; p0 += 32) {  // uniform
+    const int p = p0 + lane;
+    const bool ok = p < npairs;
+    const int j = ok ? p / M2 : 0, n = ok ? p - j * M2 : 0;
+    const real a0 = __shfl_sync(0xffffffffu, rq0, j), a1 = __shfl_sync(0xffffffffu, rq1, j);
+    const real a2 = __shfl_sync(0xffffffffu, rq2, j), a3 = __shfl_sync(0xffffffffu, rq3, j);
+    real b0, b1, b2, b3;
+    if (Q > 0) {
+      b0 = __shfl_sync(0xffffffffu, acc[0][0], n);
+      b1 = __shfl_sync(0xffffffffu, acc[0][1], n);
+      b2 = __shfl_sync(0xffffffffu, acc[0][2], n);
+      b3 = __shfl_sync(0xffffffffu, acc[0][3], n);
+    } else {
+      b0 = __shfl_sync(0xffffffffu, rq0, n);
+      b1 = __shfl_sync(0xffffffffu, rq1, n);
+      b2 = __shfl_sync(0xffffffffu, rq2, n);
+      b3 = __shfl_sync(0xffffffffu, rq3, n);
+    }
+    real d = a0 * b0;
+    d = fma(a1, b1, d);
+    d = fma(a2, b2, d);
+    d = fma(a3, b3, d);
+    if (ok) Di[(size_t)(Q * 32 + j) * M2 + n] = d;
+  }
+}
+
+// One atom: T_i into P.T (the whole warp takes part).// One atom: T_i into P.T (the whole warp takes part).
 template <typename real, int Q>
 __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &st, const int lane, const int64_t i) {
   constexpr bool kCache = sizeof(real) == 4;  // reuse coefficient registers along runs (f32 only)
@@ -181,17 +245,20 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     const int cnt = min(32, nv - base);
     if (Q > 0) {
       if constexpr (kCache) {
-        // f32: four staged neighbours per iteration through 16-byte shared loads
+        // f32: walk the batch run by run.  Neighbours are sorted by distance
+        // inside a type segment, so consecutive ones often share an interval:
+        // its coefficients are loaded once at the start of the run (a real
+        // branch, not loads predicated on every neighbour) and reused.
         int u = 0;
-        for (; u + 4 <= cnt; u += 4) {
-          const float4 t4 = *reinterpret_cast<const float4 *>(&st.t[u]);
-          const int4 o4 = *reinterpret_cast<const int4 *>(&st.off[u]);
-          fwd_neighbour<real, Q, true>(P, tab, lane, o4.x, t4.x, st.r[u], acc, cf, cur);
-          fwd_neighbour<real, Q, true>(P, tab, lane, o4.y, t4.y, st.r[u + 1], acc, cf, cur);
-          fwd_neighbour<real, Q, true>(P, tab, lane, o4.z, t4.z, st.r[u + 2], acc, cf, cur);
-          fwd_neighbour<real, Q, true>(P, tab, lane, o4.w, t4.w, st.r[u + 3], acc, cf, cur);
+        while (u < cnt) {  // uniform
+          const int off = st.off[u];
+          cur = off;
+          fwd_load_cf<real, Q>(P, tab, lane, off, cf);
+          do {
+            fwd_neighbour<real, Q, true>(P, tab, lane, off, st.t[u], st.r[u], acc, cf, cur);
+            ++u;
+          } while (u < cnt && st.off[u] == off);
         }
-        for (; u < cnt; ++u) fwd_neighbour<real, Q, true>(P, tab, lane, st.off[u], st.t[u], st.r[u], acc, cf, cur);
       } else {
         for (int u = 0; u < cnt; ++u)  // uniform: every lane on neighbour u
           fwd_neighbour<real, Q, false>(P, tab, lane, st.off[u], st.t[u], st.r[u], acc, cf, cur);
@@ -221,11 +288,13 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
   real *__restrict__ Ti = P.T + i * 4 * P.M1;
 #pragma unroll
   for (int r = 0; r < Q; ++r) {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) acc[r][k] *= P.inv_nnei;  // acc now holds T_i
     const int m = r * 32 + lane;
-    Ti[m] = acc[r][0] * P.inv_nnei;
-    Ti[P.M1 + m] = acc[r][1] * P.inv_nnei;
-    Ti[2 * P.M1 + m] = acc[r][2] * P.inv_nnei;
-    Ti[3 * P.M1 + m] = acc[r][3] * P.inv_nnei;
+    Ti[m] = acc[r][0];
+    Ti[P.M1 + m] = acc[r][1];
+    Ti[2 * P.M1 + m] = acc[r][2];
+    Ti[3 * P.M1 + m] = acc[r][3];
   }
   if (P.RR > 0) {
     // lanes rch, rch + RR, ..., rch + (PK-1) RR hold partial sums of channel 32 Q + rch
@@ -240,14 +309,19 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
         racc3 += x3;
       }
     }
+    racc0 *= P.inv_nnei;
+    racc1 *= P.inv_nnei;
+    racc2 *= P.inv_nnei;
+    racc3 *= P.inv_nnei;
     if (lane < P.RR) {
       const int m = Q * 32 + lane;
-      Ti[m] = racc0 * P.inv_nnei;
-      Ti[P.M1 + m] = racc1 * P.inv_nnei;
-      Ti[2 * P.M1 + m] = racc2 * P.inv_nnei;
-      Ti[3 * P.M1 + m] = racc3 * P.inv_nnei;
+      Ti[m] = racc0;
+      Ti[P.M1 + m] = racc1;
+      Ti[2 * P.M1 + m] = racc2;
+      Ti[3 * P.M1 + m] = racc3;
     }
   }
+  if (P.D) descriptor_epilogue<real, Q>(P, acc, racc0, racc1, racc2, racc3, lane, i);
 }
 
 template <typename real, int Q>
@@ -270,12 +344,18 @@ FwdKernel<real> pick_fwd(int Q, std::integer_sequence<int, Qs...>) {
 
 template <typename real>
 int fwd(const real *table, const dp_table_info *info, const real *s, const real *Rt, const int32_t *nvalid,
-        const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, real *T, void *stream) {
+        const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, real *T, void *stream,
+        int M2 = 0, real *D = nullptr, bool want_D = false) {
   clear_error();
   TableGeom g;
   Segments seg;
-  int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, T, &g, &seg);
+  int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, want_D ? (const void *)D : T, &g,
+                             &seg);
   if (rc) return rc;
+  if (want_D) {
+    if (M2 < 1 || M2 > M1) return set_error(DP_ERR_SHAPE, "need 1 <= M2 <= M1 (M1 %d, M2 %d)", M1, M2);
+    if (M2 > 32) return set_error(DP_ERR_UNSUPPORTED, "fused descriptor needs M2 <= 32 (M2 = %d)", M2);
+  }
   if (nloc == 0) return DP_OK;
   FwdParams<real> P;
   P.table = table;
@@ -284,6 +364,8 @@ int fwd(const real *table, const dp_table_info *info, const real *s, const real 
   P.nvalid = nvalid;
   P.atype = atype;
   P.T = T;
+  P.D = want_D ? D : nullptr;
+  P.M2 = want_D ? M2 : 0;
   P.geom = GeomOf<real>::make(g);
   P.nloc = nloc;
   P.nnei = nnei;
@@ -319,6 +401,20 @@ int dp_tabulate_fusion_fwd_f32(const float *table, const dp_table_info *info, co
                                const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
                                const int32_t *sel, int M1, float *T, void *stream) {
   return dpc::fwd<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream);
+}
+
+int dp_tabulate_fusion_fwd_descriptor_f64(const double *table, const dp_table_info *info, const double *s,
+                                          const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                          int nnei, int ntypes, const int32_t *sel, int M1, int M2, double *T,
+                                          double *D, void *stream) {
+  return dpc::fwd<double>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream, M2, D, true);
+}
+
+int dp_tabulate_fusion_fwd_descriptor_f32(const float *table, const dp_table_info *info, const float *s,
+                                          const float *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                          int nnei, int ntypes, const int32_t *sel, int M1, int M2, float *T,
+                                          float *D, void *stream) {
+  return dpc::fwd<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream, M2, D, true);
 }
 
 }  // extern "C"
