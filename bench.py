@@ -58,6 +58,19 @@ def rank_seed(seed: int, rank: int) -> int:
     return seed + 7919 * rank
 
 
+def rank_workload(args, rank: int, world: int, **kw):
+    """This rank's share of the work.  weak: its own seeded instance of the whole workload (per-GPU work
+    fixed as N grows).  strong: one instance, its atoms split into contiguous ranges over the ranks."""
+    import workloads as W
+    if getattr(args, "scaling", "weak") == "weak":
+        return W.make(args.workload, seed=rank_seed(args.seed, rank), **kw)
+    w = W.make(args.workload, seed=args.seed, **kw)
+    lo, hi = W.shard(w.nloc, rank, world)
+    part = {k: getattr(w, k)[lo:hi] for k in ("s", "Rt", "nvalid", "atype", "dT")}
+    w.__dict__.update(part, pos=None, box=None, name=f"{w.name}[{lo}:{hi}]")
+    return w
+
+
 def reduce_over_ranks(total_s: float, evals: float, world: int, device) -> tuple[float, float]:
     """Max of the timed seconds and sum of the work over ranks (timing only; the data path has no collective)."""
     if world == 1:
@@ -148,7 +161,7 @@ def run_native(args, rank, world, local_rank):
     kw = {}
     if args.workload == "alcumg":
         kw["pad"] = args.pad
-    w = W.make(args.workload, seed=rank_seed(args.seed, rank), **kw)
+    w = rank_workload(args, rank, world, **kw)
     info = dpc.dp_table_info_make(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
     model = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, dtype)
     sel = [int(x) for x in w.sel]
@@ -299,8 +312,10 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall):
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sum(step_ms) / len(step_ms), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": args.dtype, "data": "synthetic",
-        "config": {"workload": workload_label(w), "parallelism": f"replicas x{world} (independent seeded instances)",
+        "scaling": args.scaling, "vs_baseline": None, "dtype": args.dtype, "data": "synthetic",
+        "config": {"workload": workload_label(w),
+                   "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
+                                   else f"atoms split over {world} ranks"),
                    "step": "fwd + descriptor + grad", "l2": "flushed between steps (256 MiB write)",
                    "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4)},
         "atoms_per_s": w.nloc * world * args.steps / total_s,
@@ -413,6 +428,8 @@ def main():
     ap.add_argument("--seed", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
+    ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
+                    help="weak: one instance per rank; strong: one instance split over the ranks")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3:

@@ -73,16 +73,35 @@ __device__ __forceinline__ real horner5(const real c[6], real t) {
   return fma(g, t, c[5]);
 }
 
-// The coefficients of this lane's Q channels of the interval block at `off`.
+// One neighbour (interval block offset `off`, local t, R~ row r) folded into
+// the lane's Q channel rounds, coefficients loaded round by round (f64).
 template <typename real, int Q>
-__device__ __forceinline__ void fwd_load_cf(const FwdParams<real> &P, const real *__restrict__ tab, const int lane,
-                                            const int off, real (&cf)[Q > 0 ? Q : 1][6]) {
-  using V2 = typename std::conditional<sizeof(real) == 8, double2, float2>::type;
-  const V2 *q0 = reinterpret_cast<const V2 *>(tab + off) + lane;
-  const V2 *q1 = q0 + P.M1, *q2 = q1 + P.M1;
+__device__ __forceinline__ void fwd_neighbour(const FwdParams<real> &P, const real *__restrict__ tab, const int lane,
+                                              const int off, const real t, const real *r,
+                                              real (&acc)[Q > 0 ? Q : 1][4]) {
+  const real r0 = r[0], r1 = r[1], r2 = r[2], r3 = r[3];
 #pragma unroll
   for (int k = 0; k < Q; ++k) {
-    const V2 x = __ldg(q0 + 32 * k), y = __ldg(q1 + 32 * k), z = __ldg(q2 + 32 * k);
+    real c6[6];
+    ld6(tab + off, P.M1, k * 32 + lane, c6);
+    const real g = horner5(c6, t);
+    acc[k][0] = fma(r0, g, acc[k][0]);
+    acc[k][1] = fma(r1, g, acc[k][1]);
+    acc[k][2] = fma(r2, g, acc[k][2]);
+    acc[k][3] = fma(r3, g, acc[k][3]);
+  }
+}
+
+// f32: the coefficients of this lane's Q channels of the interval block at
+// `off`, loaded once per run of neighbours that share the interval.
+template <int Q>
+__device__ __forceinline__ void fwd_load_cf(const FwdParams<float> &P, const float *__restrict__ tab, const int lane,
+                                            const int off, float (&cf)[Q > 0 ? Q : 1][6]) {
+  const float2 *q0 = reinterpret_cast<const float2 *>(tab + off) + lane;
+  const float2 *q1 = q0 + P.M1, *q2 = q1 + P.M1;
+#pragma unroll
+  for (int k = 0; k < Q; ++k) {
+    const float2 x = __ldg(q0 + 32 * k), y = __ldg(q1 + 32 * k), z = __ldg(q2 + 32 * k);
     cf[k][0] = x.x;
     cf[k][1] = x.y;
     cf[k][2] = y.x;
@@ -92,29 +111,18 @@ __device__ __forceinline__ void fwd_load_cf(const FwdParams<real> &P, const real
   }
 }
 
-// One neighbour (interval block offset `off`, local t, R~ row r) folded into
-// the lane's Q channel rounds.  kCache: cf already holds the interval's
-// coefficients; otherwise they are loaded here, round by round.
-template <typename real, int Q, bool kCache>
-__device__ __forceinline__ void fwd_neighbour(const FwdParams<real> &P, const real *__restrict__ tab, const int lane,
-                                              const int off, const real t, const real *r,
-                                              real (&acc)[Q > 0 ? Q : 1][4], real (&cf)[kCache && Q > 0 ? Q : 1][6],
-                                              int &cur) {
-  const real r0 = r[0], r1 = r[1], r2 = r[2], r3 = r[3];
+// f32: one neighbour folded into the lane's Q channel rounds with the
+// interval's coefficients already in registers.
+template <int Q>
+__device__ __forceinline__ void fwd_neighbour_cached(const float t, const float4 r, float (&acc)[Q > 0 ? Q : 1][4],
+                                                     const float (&cf)[Q > 0 ? Q : 1][6]) {
 #pragma unroll
   for (int k = 0; k < Q; ++k) {
-    real c6[6];
-    if (kCache) {
-#pragma unroll
-      for (int e = 0; e < 6; ++e) c6[e] = cf[kCache ? k : 0][e];
-    } else {
-      ld6(tab + off, P.M1, k * 32 + lane, c6);
-    }
-    const real g = horner5(c6, t);
-    acc[k][0] = fma(r0, g, acc[k][0]);
-    acc[k][1] = fma(r1, g, acc[k][1]);
-    acc[k][2] = fma(r2, g, acc[k][2]);
-    acc[k][3] = fma(r3, g, acc[k][3]);
+    const float g = horner5(cf[k], t);
+    acc[k][0] = fmaf(r.x, g, acc[k][0]);
+    acc[k][1] = fmaf(r.y, g, acc[k][1]);
+    acc[k][2] = fmaf(r.z, g, acc[k][2]);
+    acc[k][3] = fmaf(r.w, g, acc[k][3]);
   }
 }
 
@@ -182,7 +190,7 @@ __device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, co
 // One atom: T_i into P.T (the whole warp takes part).// One atom: T_i into P.T (the whole warp takes part).
 template <typename real, int Q>
 __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &st, const int lane, const int64_t i) {
-  constexpr bool kCache = sizeof(real) == 4;  // reuse coefficient registers along runs (f32 only)
+  constexpr bool kCache = sizeof(real) == 4;  // f32: coefficients reused along runs of equal intervals
 
   // valid rows per type segment (clamped into [0, sel]), kept in shared memory, and their total
   {
@@ -212,10 +220,9 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
 #pragma unroll
   for (int r = 0; r < (Q > 0 ? Q : 1); ++r) acc[r][0] = acc[r][1] = acc[r][2] = acc[r][3] = real(0);
   real racc0 = real(0), racc1 = real(0), racc2 = real(0), racc3 = real(0);
-  real cf[kCache && Q > 0 ? Q : 1][6];  // f32: coefficient rows of the interval in use
   real rcf[6];
-  int cur = -1, rcur = -1;
-
+  int rcur = -1;
+  real cf[Q > 0 ? Q : 1][6];  // f32: coefficients of the interval in use
   for (int base = 0; base < nv; base += 32) {
     // stage: lane l prepares valid neighbour base + l
     const int v = base + lane;
@@ -252,16 +259,15 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
         int u = 0;
         while (u < cnt) {  // uniform
           const int off = st.off[u];
-          cur = off;
-          fwd_load_cf<real, Q>(P, tab, lane, off, cf);
+          fwd_load_cf<Q>(P, tab, lane, off, cf);
           do {
-            fwd_neighbour<real, Q, true>(P, tab, lane, off, st.t[u], st.r[u], acc, cf, cur);
+            fwd_neighbour_cached<Q>(st.t[u], *reinterpret_cast<const float4 *>(st.r[u]), acc, cf);
             ++u;
           } while (u < cnt && st.off[u] == off);
         }
       } else {
         for (int u = 0; u < cnt; ++u)  // uniform: every lane on neighbour u
-          fwd_neighbour<real, Q, false>(P, tab, lane, st.off[u], st.t[u], st.r[u], acc, cf, cur);
+          fwd_neighbour<real, Q>(P, tab, lane, st.off[u], st.t[u], st.r[u], acc);
       }
     }
     if (P.RR > 0) {

@@ -289,3 +289,22 @@ def test_water_large_sampled(dtype):
     assert abs(lhs - rhs) <= TOL[dtype] * 10 * max(1.0, abs(rhs)), (lhs, rhs)
     del T, D, ds, dRt, x, model
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("dtype", [torch.float64, torch.float32])
+def test_normalised_environment_matrix(dtype):
+    """The paper's normalisation of the 4-vectors (s shifted by its mean and scaled by its std, the
+    xyz columns by their joint std): s takes negative values, so the table starts below zero."""
+    base = W.water(seed=52, nmol=128, widths=(1, 8, 16, 32), M2=8)
+    off = np.concatenate([[0], np.cumsum(base.sel)])
+    valid = np.zeros(base.s.shape, bool)
+    for b in range(base.ntypes):
+        valid[:, off[b]:off[b + 1]] = np.arange(base.sel[b])[None, :] < base.nvalid[:, b:b + 1]
+    sv = base.s[valid]
+    xyz = base.Rt[..., 1:][valid]
+    norm = (float(sv.mean()), float(sv.std()), float(xyz.std()))
+    w = W.water(seed=52, nmol=128, widths=(1, 8, 16, 32), M2=8, norm=norm)
+    assert w.s_min < 0.0
+    got = run_product(w, dtype)
+    ref = run_oracle(w, dtype)
+    assert_parity(got, ref, dtype)

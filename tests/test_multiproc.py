@@ -32,7 +32,13 @@ def _worker(rank, world, port, q):
             workload, pad, seed, dtype, steps, warmup = "tiny", 0.3, 1, "f64", 2, 3
 
         ref = bench.run_reference(A, rank, world) if rank == 1 else "skipped"
-        q.put((rank, total, evals, float(w.evals), sums, ref))
+
+        class S:
+            workload, seed, scaling = "tiny", 1, "strong"
+
+        part = bench.rank_workload(S, rank, world)
+        _, strong_evals = bench.reduce_over_ranks(0.0, float(part.evals), world, torch.device("cpu"))
+        q.put((rank, total, evals, float(w.evals), sums, ref, strong_evals, part.nloc))
     finally:
         dist.destroy_process_group()
 
@@ -54,8 +60,11 @@ def test_two_ranks_gloo():
         assert p.exitcode == 0
     ev = [out[r][3] for r in range(world)]
     for r in range(world):
-        _, total, evals, _, sums, _ = out[r]
+        _, total, evals, _, sums = out[r][:5]
         assert total == 2.5  # max over ranks
         assert evals == sum(ev)  # work of all ranks
         assert sums[0] != sums[1]  # independent seeded instances
     assert out[1][5] is None  # the reference arm runs on rank 0 only
+    full = W.tiny(seed=1)
+    assert out[0][6] == out[1][6] == float(full.evals)  # strong scaling: the shards cover the instance
+    assert out[0][7] + out[1][7] == full.nloc
