@@ -176,12 +176,14 @@ def run_native(args, rank, world, local_rank):
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 256 MiB > 126 MiB L2
     stream = torch.cuda.current_stream(dev)
 
+    fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
+
     def step(ev=None, x=None, o=None):
         x = x or d
         o = o or dict(T=T, D=D, ds=ds, dRt=dRt)
         if ev:
             ev[0].record(stream)
-        dpc.dp_tabulate_fusion_fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
+        fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
         if ev:
             ev[1].record(stream)
         dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"])
@@ -316,7 +318,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall):
         "config": {"workload": workload_label(w),
                    "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
                                    else f"atoms split over {world} ranks"),
-                   "step": "fwd + descriptor + grad", "l2": "flushed between steps (256 MiB write)",
+                   "step": "fwd + descriptor + grad", "algo": args.algo,
+                   "l2": "flushed between steps (256 MiB write)",
                    "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4)},
         "atoms_per_s": w.nloc * world * args.steps / total_s,
         "roofline": roofline,
@@ -428,6 +431,8 @@ def main():
     ap.add_argument("--seed", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
+    ap.add_argument("--algo", choices=["direct", "moments"], default="direct",
+                    help="direct: per-neighbour evaluation (the paper's fused kernel); moments: interval moments")
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")
     ap.add_argument("--no-cpu-baseline", action="store_true")

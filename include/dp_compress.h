@@ -159,6 +159,24 @@ int dp_tabulate_fusion_fwd_f32(const float *table, const dp_table_info *info, co
                                const int32_t *sel, int M1, float *T, void *stream);
 
 /*
+ * The same forward by interval moments.  Neighbours are sorted by distance
+ * inside a type segment (Sec. II), so consecutive valid rows often fall in
+ * the same table interval l.  For such a run the per-neighbour sum regroups
+ * exactly as
+ *   sum_{j in run} R~_j[k] g_m(t_j) = sum_q C_{l,m,q} W[k][q],   W[k][q] = sum_{j in run} R~_j[k] t_j^q,
+ * with C_{l,m,q} the t^q coefficient: 24 FMA per channel per run instead of
+ * 9 per channel per neighbour.  Runs of 3 or more rows go this way, shorter
+ * ones neighbour by neighbour.  Same arguments, results and errors as
+ * dp_tabulate_fusion_fwd_* (equal up to rounding order).
+ */
+int dp_tabulate_fusion_fwd_moments_f64(const double *table, const dp_table_info *info, const double *s,
+                                       const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                       int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *stream);
+int dp_tabulate_fusion_fwd_moments_f32(const float *table, const dp_table_info *info, const float *s,
+                                       const float *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                       int nnei, int ntypes, const int32_t *sel, int M1, float *T, void *stream);
+
+/*
  * Forward and descriptor in one pass (Sec. II: T_i, then D_i = S_i (S_i^<)^T
  * with S_i = T_i^T): the same T as dp_tabulate_fusion_fwd_* and
  *   D[i][m][n] = sum_k T[i][k][m] * T[i][k][n],  n < M2,

@@ -60,6 +60,10 @@ _SIGS = {
                                     _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_fwd_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
                                     _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_moments_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                            ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_moments_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                            ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_fwd_descriptor_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                                ctypes.c_int, ctypes.c_int, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_fwd_descriptor_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
@@ -184,11 +188,20 @@ def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
 
 def dp_tabulate_fusion_fwd(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None) -> torch.Tensor:
     """T [nloc][4][M1] = (1/nnei) R~^T G with G from the table, valid rows only."""
+    return _fwd("dp_tabulate_fusion_fwd", table, info, s, Rt, nvalid, atype, sel, out)
+
+
+def dp_tabulate_fusion_fwd_moments(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None) -> torch.Tensor:
+    """The same T through interval moments (runs of neighbours sharing a table interval)."""
+    return _fwd("dp_tabulate_fusion_fwd_moments", table, info, s, Rt, nvalid, atype, sel, out)
+
+
+def _fwd(name, table, info, s, Rt, nvalid, atype, sel, out):
     dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
                                                                                       sel)
     shape = (nloc, 4, M1)
     T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
-    fn = getattr(_lib, f"dp_tabulate_fusion_fwd_{_suffix(dtype)}")
+    fn = getattr(_lib, f"{name}_{_suffix(dtype)}")
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(T), _stream(s)))
     return T

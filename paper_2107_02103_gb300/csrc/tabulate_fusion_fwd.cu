@@ -63,6 +63,19 @@ struct alignas(16) Stage {
   int32_t nvb[DP_MAX_TYPES];  // valid rows per type segment of the current atom
 };
 
+// Extra staging of the interval-moment variant: powers t^0..t^5 of every
+// staged neighbour and the 24 moments W[k][q] of the run being contracted.
+template <typename real>
+struct alignas(16) MomentStage {
+  real tp[32][6];
+  real w[24];
+};
+
+// Runs at least this long go through interval moments; shorter ones are
+// evaluated neighbour by neighbour (a run costs n + 24 Q FMA instructions in
+// moments against 9 Q n per neighbour).
+constexpr int kMinMomentRun = 3;
+
 template <typename real>
 __device__ __forceinline__ real horner5(const real c[6], real t) {
   // g = ((((a t + b) t + c) t + d) t + e) t + f
@@ -187,9 +200,14 @@ __device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, co
   }
 }
 
-// One atom: T_i into P.T (the whole warp takes part).// One atom: T_i into P.T (the whole warp takes part).
-template <typename real, int Q>
-__device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &st, const int lane, const int64_t i) {
+// One atom: T_i into P.T (the whole warp takes part).// One atom: T_i into P.T (the whole warp takes part).  kMoments: runs of
+// neighbours sharing an interval are contracted through their moments
+//   W[k][q] = sum_{j in run} R~_j[k] t_j^q,   T[k][m] += sum_q C_{l,m,q} W[k][q]
+// (C_{l,m,q} the t^q coefficient of channel m on interval l): the same sum as
+// the per-neighbour evaluation, associated per interval.
+template <typename real, int Q, bool kMoments>
+__device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &st, MomentStage<real> &ms,
+                                         const int lane, const int64_t i) {
   constexpr bool kCache = sizeof(real) == 4;  // f32: coefficients reused along runs of equal intervals
 
   // valid rows per type segment (clamped into [0, sel]), kept in shared memory, and their total
@@ -247,10 +265,56 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
       st.r[lane][3] = rr.w;
       st.t[lane] = t;
       st.off[lane] = (b * P.geom.nint + l) * P.M1 * 6;
+      if constexpr (kMoments) {
+        const real t2 = t * t, t3 = t2 * t;
+        ms.tp[lane][0] = real(1);
+        ms.tp[lane][1] = t;
+        ms.tp[lane][2] = t2;
+        ms.tp[lane][3] = t3;
+        ms.tp[lane][4] = t2 * t2;
+        ms.tp[lane][5] = t3 * t2;
+      }
     }
     __syncwarp();
     const int cnt = min(32, nv - base);
-    if (Q > 0) {
+    if (Q > 0 && kMoments) {
+      int u = 0;
+      while (u < cnt) {  // uniform, run by run
+        const int off = st.off[u];
+        int e = u + 1;
+        while (e < cnt && st.off[e] == off) ++e;
+        if (e - u >= kMinMomentRun) {
+          real wv = real(0);
+          if (lane < 24) {
+            const int k = lane / 6, q = lane - 6 * (lane / 6);
+            for (int j = u; j < e; ++j) wv = fma(st.r[j][k], ms.tp[j][q], wv);
+            ms.w[lane] = wv;
+          }
+          __syncwarp();
+          real W[4][6];
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+#pragma unroll
+            for (int q = 0; q < 6; ++q) W[k][q] = ms.w[6 * k + q];
+#pragma unroll
+          for (int r = 0; r < Q; ++r) {
+            real c6[6];  // (a, b, c, d, e, f) = coefficients of t^5 .. t^0
+            ld6(tab + off, P.M1, r * 32 + lane, c6);
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              real v = acc[r][k];
+#pragma unroll
+              for (int q = 0; q < 6; ++q) v = fma(c6[5 - q], W[k][q], v);
+              acc[r][k] = v;
+            }
+          }
+          __syncwarp();
+        } else {
+          for (int j = u; j < e; ++j) fwd_neighbour<real, Q>(P, tab, lane, off, st.t[j], st.r[j], acc);
+        }
+        u = e;
+      }
+    } else if (Q > 0) {
       if constexpr (kCache) {
         // f32: walk the batch run by run.  Neighbours are sorted by distance
         // inside a type segment, so consecutive ones often share an interval:
@@ -330,28 +394,29 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
   if (P.D) descriptor_epilogue<real, Q>(P, acc, racc0, racc1, racc2, racc3, lane, i);
 }
 
-template <typename real, int Q>
+template <typename real, int Q, bool kMoments>
 __global__ void __launch_bounds__(kFwdWarps * 32) fwd_kernel(const FwdParams<real> P) {
   __shared__ Stage<real> stage[kFwdWarps];
+  __shared__ MomentStage<real> mstage[kMoments ? kFwdWarps : 1];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t i = (int64_t)blockIdx.x * kFwdWarps + w;
-  if (i < P.nloc) fwd_atom<real, Q>(P, stage[w], lane, i);  // warp-uniform
+  if (i < P.nloc) fwd_atom<real, Q, kMoments>(P, stage[w], mstage[kMoments ? w : 0], lane, i);  // warp-uniform
 }
 
 template <typename real>
 using FwdKernel = void (*)(const FwdParams<real>);
 
-template <typename real, int... Qs>
+template <typename real, bool kMoments, int... Qs>
 FwdKernel<real> pick_fwd(int Q, std::integer_sequence<int, Qs...>) {
   FwdKernel<real> k = nullptr;
-  ((Q == Qs ? (k = &fwd_kernel<real, Qs>, 0) : 0), ...);
+  ((Q == Qs ? (k = &fwd_kernel<real, Qs, kMoments>, 0) : 0), ...);
   return k;
 }
 
 template <typename real>
 int fwd(const real *table, const dp_table_info *info, const real *s, const real *Rt, const int32_t *nvalid,
         const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, real *T, void *stream,
-        int M2 = 0, real *D = nullptr, bool want_D = false) {
+        int M2 = 0, real *D = nullptr, bool want_D = false, bool moments = false) {
   clear_error();
   TableGeom g;
   Segments seg;
@@ -383,7 +448,8 @@ int fwd(const real *table, const dp_table_info *info, const real *s, const real 
   P.PK = P.RR > 0 ? 32 / P.RR : 1;
   for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
   P.inv_nnei = (real)(1.0 / (double)nnei);
-  FwdKernel<real> k = pick_fwd<real>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
+  FwdKernel<real> k = moments ? pick_fwd<real, true>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{})
+                              : pick_fwd<real, false>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
   if (!k) return set_error(DP_ERR_UNSUPPORTED, "no forward kernel for M1 = %d", M1);
   const int64_t blocks = (nloc + kFwdWarps - 1) / kFwdWarps;
   if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
@@ -407,6 +473,20 @@ int dp_tabulate_fusion_fwd_f32(const float *table, const dp_table_info *info, co
                                const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
                                const int32_t *sel, int M1, float *T, void *stream) {
   return dpc::fwd<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream);
+}
+
+int dp_tabulate_fusion_fwd_moments_f64(const double *table, const dp_table_info *info, const double *s,
+                                       const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                       int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *stream) {
+  return dpc::fwd<double>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream, 0, nullptr, false,
+                          true);
+}
+
+int dp_tabulate_fusion_fwd_moments_f32(const float *table, const dp_table_info *info, const float *s,
+                                       const float *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                       int nnei, int ntypes, const int32_t *sel, int M1, float *T, void *stream) {
+  return dpc::fwd<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream, 0, nullptr, false,
+                         true);
 }
 
 int dp_tabulate_fusion_fwd_descriptor_f64(const double *table, const dp_table_info *info, const double *s,

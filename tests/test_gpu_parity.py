@@ -308,3 +308,46 @@ def test_normalised_environment_matrix(dtype):
     got = run_product(w, dtype)
     ref = run_oracle(w, dtype)
     assert_parity(got, ref, dtype)
+
+
+MOMENT_CASES = [
+    ("tiny", {}, torch.float64, None), ("tiny", {}, torch.float32, None),
+    ("water", dict(nmol=256), torch.float64, None), ("water", dict(nmol=256), torch.float32, None),
+    ("cu85", dict(cells=(6, 6, 6)), torch.float64, None), ("cu85", dict(cells=(6, 6, 6)), torch.float32, None),
+    ("alcumg", dict(pad=0.1, cells=(6, 6, 6)), torch.float64, None),
+    ("cu85", {}, torch.float64, None), ("alcumg", dict(pad=0.3), torch.float64, 384),
+]
+
+
+@pytest.mark.parametrize("name,kw,dtype,nsample", MOMENT_CASES,
+                         ids=[f"{c[0]}-{c[1]}-{str(c[2])[6:]}" for c in MOMENT_CASES])
+def test_moments_forward(name, kw, dtype, nsample):
+    """The interval-moment forward gives the oracle's T (and equals the per-neighbour forward up to rounding)."""
+    dpc = lib()
+    w = workload(name, **kw)
+    model = product_model(w, dtype)
+    x = to_dev(w, dtype)
+    T = dpc.dp_tabulate_fusion_fwd_moments(model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
+    T0 = dpc.dp_tabulate_fusion_fwd(model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
+    torch.cuda.synchronize()
+    atoms = None
+    if nsample:
+        rng = np.random.default_rng(3)
+        atoms = np.sort(rng.choice(w.nloc, nsample, replace=False))
+    ref = run_oracle(w, dtype, atoms=atoms)
+    got = T.double().cpu().numpy()
+    assert rel(got if atoms is None else got[atoms], ref["T"]) <= TOL[dtype]
+    assert rel(got, T0.double().cpu().numpy()) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("M1,widths", [(1, (1, 1)), (37, (1, 5, 37)), (64, (1, 16, 32, 64)), (200, (1, 50, 100, 200))])
+def test_moments_forward_shapes(M1, widths):
+    """Long runs (neighbours bunched in s) through every channel-round shape of the moment path."""
+    dpc = lib()
+    w = W.tiny(seed=90 + M1, nloc=11, nreal=27, sel=30, widths=widths, M2=1, rmin=2.6, rmax=3.0)
+    for dtype in (torch.float64, torch.float32):
+        model = product_model(w, dtype)
+        x = to_dev(w, dtype)
+        T = dpc.dp_tabulate_fusion_fwd_moments(model.table, model.info, x["s"], x["Rt"], x["nvalid"], None, w.sel)
+        torch.cuda.synchronize()
+        assert rel(T.double().cpu().numpy(), run_oracle(w, dtype)["T"]) <= TOL[dtype]
