@@ -177,6 +177,7 @@ def run_native(args, rank, world, local_rank):
     stream = torch.cuda.current_stream(dev)
 
     fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
+    grad = dpc.dp_tabulate_fusion_grad_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_grad
 
     def step(ev=None, x=None, o=None):
         x = x or d
@@ -189,8 +190,7 @@ def run_native(args, rank, world, local_rank):
         dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"])
         if ev:
             ev[2].record(stream)
-        dpc.dp_tabulate_fusion_grad(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, x["dT"],
-                                    out=(o["ds"], o["dRt"]))
+        grad(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, x["dT"], out=(o["ds"], o["dRt"]))
         if ev:
             ev[3].record(stream)
 

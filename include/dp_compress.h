@@ -214,6 +214,26 @@ int dp_tabulate_fusion_grad_f32(const float *table, const dp_table_info *info, c
                                 const int32_t *sel, int M1, const float *dT, float *ds, float *dRt, void *stream);
 
 /*
+ * The same backward by interval moments.  For a run of consecutive valid
+ * rows in one table interval l (rows are sorted by distance inside a type
+ * segment, Sec. II), with C_{l,m,q} the t^q coefficient of g_m on l,
+ *   H[k][q] = sum_m dT[i][k][m] C_{l,m,q}
+ * is formed once per run (24 FMA per channel), and each row follows from it:
+ *   dRt[i][row][k] = (1/nnei) sum_q t^q H[k][q]
+ *   ds[i][row]     = (1/nnei) sum_k R~[i][row][k] sum_{q>=1} q t^(q-1) H[k][q]
+ * (the channel sums of dp_tabulate_fusion_grad_* taken in the other order).
+ * Same arguments, results, limits and errors as dp_tabulate_fusion_grad_*.
+ */
+int dp_tabulate_fusion_grad_moments_f64(const double *table, const dp_table_info *info, const double *s,
+                                        const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                        int nnei, int ntypes, const int32_t *sel, int M1, const double *dT, double *ds,
+                                        double *dRt, void *stream);
+int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info *info, const float *s,
+                                        const float *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                        int nnei, int ntypes, const int32_t *sel, int M1, const float *dT, float *ds,
+                                        float *dRt, void *stream);
+
+/*
  * Descriptor (Sec. II): with S_i = T_i^T (M1 x 4) and S_i^< its first M2
  * rows, D_i = S_i (S_i^<)^T, i.e. D[i][m][n] = sum_k T[i][k][m] * T[i][k][n].
  *   T [nloc][4][M1] input,  D [nloc][M1][M2] output.

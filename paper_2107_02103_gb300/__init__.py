@@ -72,6 +72,10 @@ _SIGS = {
                                      _P, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, ctypes.c_int,
                                      _P, _P, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_moments_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                             ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_moments_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                             ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_f64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_f32": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_grad_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
@@ -225,6 +229,15 @@ def dp_tabulate_fusion_fwd_descriptor(table, info: dp_table_info, s, Rt, nvalid,
 
 def dp_tabulate_fusion_grad(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None):
     """(ds [nloc][nnei], dRt [nloc][nnei][4]) from dT = dE/dT [nloc][4][M1]."""
+    return _grad("dp_tabulate_fusion_grad", table, info, s, Rt, nvalid, atype, sel, dT, out)
+
+
+def dp_tabulate_fusion_grad_moments(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None):
+    """The same (ds, dRt) through interval moments (runs of rows sharing a table interval)."""
+    return _grad("dp_tabulate_fusion_grad_moments", table, info, s, Rt, nvalid, atype, sel, dT, out)
+
+
+def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
     dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
                                                                                       sel)
     dT = _dev(dT, "dT", dtype, (nloc, 4, M1))
@@ -234,7 +247,7 @@ def dp_tabulate_fusion_grad(table, info: dp_table_info, s, Rt, nvalid, atype, se
     else:
         ds = _dev(out[0], "ds", dtype, (nloc, nnei))
         dRt = _dev(out[1], "dRt", dtype, (nloc, nnei, 4))
-    fn = getattr(_lib, f"dp_tabulate_fusion_grad_{_suffix(dtype)}")
+    fn = getattr(_lib, f"{name}_{_suffix(dtype)}")
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(dT), _ptr(ds), _ptr(dRt), _stream(s)))
     return ds, dRt

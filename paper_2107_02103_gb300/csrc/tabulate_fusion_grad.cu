@@ -42,6 +42,7 @@ struct GradParams {
   real *__restrict__ ds;
   real *__restrict__ dRt;
   TableGeom geom;
+  typename GeomOf<real>::type lgeom;  // the same geometry in the precision of real (moment kernel)
   int64_t nloc;
   int32_t nnei, ntypes, M1, pair_stride;
   int32_t sel[DP_MAX_TYPES];
@@ -168,6 +169,208 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
     P.ds[i * P.nnei + row] = real(0);
     st4(P.dRt + (i * P.nnei + row) * 4, real(0), real(0), real(0), real(0));
   }
+}
+
+// ------------------------------------------------------- interval moments
+// The same backward regrouped per run of consecutive valid rows that share a
+// table interval l (neighbours are sorted by distance inside a segment):
+//   H[k][q] = sum_m dT[k][m] C_{l,m,q}                 (C_{l,m,q}: t^q coefficient)
+//   dE/dR~_j[k] = (1/N_c) sum_q t_j^q H[k][q]
+//   dE/ds_j     = (1/N_c) sum_k R~_j[k] sum_{q>=1} q t_j^(q-1) H[k][q]
+// One warp per atom.  For each run the lanes form H over their channels
+// (24 FMA per channel) and a reduce-scatter butterfly sums the 24 values
+// over the lanes (24 DADD); then every lane takes one row of the batch and
+// evaluates its 5 outputs from its run's H (about 50 FMA per row).  A run
+// costs ~100 warp instructions plus ~1.5 per row, against 56 per row for the
+// per-row kernel.
+constexpr int kMomentWarps = 1;
+
+template <typename real>
+struct alignas(16) MomentGradStage {
+  real r[32][4];     // R~ rows of the batch
+  real t[32];        // local variable t
+  real H[32][24];    // H of each run of the batch, [run][4*k + q... laid out k-major]
+  int32_t off[32];   // interval block offset
+  int32_t row[32];   // row index, bit 30 set when s was clamped
+  int32_t run[32];   // run index of each row of the batch
+  int32_t nvb[DP_MAX_TYPES];
+};
+
+template <typename real, int Q>
+__global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const GradParams<real> P) {
+  constexpr int kClamped = 1 << 30;
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int lane = threadIdx.x & 31;
+  const int64_t i = blockIdx.x;  // one atom per block (one warp)
+  MomentGradStage<real> &st = *reinterpret_cast<MomentGradStage<real> *>(smem_raw);
+  real *dts = reinterpret_cast<real *>(smem_raw + sizeof(MomentGradStage<real>));  // [M1][4]
+  const int M1 = P.M1, RR = M1 - 32 * Q;
+
+  {  // counts in shared memory
+    int sl = 0;
+#pragma unroll
+    for (int q = 0; q < DP_MAX_TYPES; ++q)
+      if (lane == q) sl = P.sel[q];
+    int x = 0;
+    if (lane < P.ntypes) x = clampi(P.nvalid ? __ldg(P.nvalid + i * P.ntypes + lane) : sl, 0, sl);
+    if (lane < DP_MAX_TYPES) st.nvb[lane] = x;
+  }
+  {
+    const real *__restrict__ dTi = P.dT + i * 4 * M1;
+    for (int e = lane; e < 4 * M1; e += 32) {
+      const int k = e / M1, m = e - k * M1;
+      dts[m * 4 + k] = __ldg(dTi + e);
+    }
+  }
+  __syncwarp();
+  int nv = 0;
+#pragma unroll
+  for (int q = 0; q < DP_MAX_TYPES; ++q) nv += st.nvb[q];
+  const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
+  const real *__restrict__ tab = P.table + (size_t)alpha * P.ntypes * P.pair_stride;
+  real *__restrict__ ds_i = P.ds + i * P.nnei;
+  real *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
+
+  for (int base = 0; base < nv; base += 32) {
+    const int cnt = min(32, nv - base);
+    if (lane < cnt) {  // stage row base + lane
+      const int v = base + lane;
+      int b = 0, cum = 0, lim = st.nvb[0], off = 0;
+#pragma unroll
+      for (int c = 1; c < DP_MAX_TYPES; ++c)
+        if (c < P.ntypes && v >= lim) {
+          b = c;
+          cum = lim;
+          lim += st.nvb[c];
+          off += P.sel[c - 1];
+        }
+      const int row = off + (v - cum);
+      const Vec4<real> rr = ld4(P.Rt + (i * P.nnei + row) * 4);
+      real t;
+      bool clamped;
+      const int l = locate(P.lgeom, __ldg(P.s + i * P.nnei + row), t, clamped);
+      st.r[lane][0] = rr.x;
+      st.r[lane][1] = rr.y;
+      st.r[lane][2] = rr.z;
+      st.r[lane][3] = rr.w;
+      st.t[lane] = (real)t;
+      st.off[lane] = (b * P.geom.nint + l) * M1 * 6;
+      st.row[lane] = row | (clamped ? kClamped : 0);
+    }
+    __syncwarp();
+    // runs of the batch: H of each, written to st.H[run]
+    int nrun = 0;
+    for (int u = 0; u < cnt;) {  // uniform
+      const int off = st.off[u];
+      int e = u + 1;
+      while (e < cnt && st.off[e] == off) ++e;
+      if (lane >= u && lane < e) st.run[lane] = nrun;
+      real h[24];
+#pragma unroll
+      for (int x = 0; x < 24; ++x) h[x] = real(0);
+      const real *__restrict__ blk = tab + off;
+#pragma unroll
+      for (int r = 0; r <= Q; ++r) {
+        const int m = 32 * r + lane;
+        if (r < Q || lane < RR) {  // last round: the RR remainder channels
+          real c6[6];  // (a..f): coefficients of t^5 .. t^0
+          ld6(blk, M1, m, c6);
+          const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
+#pragma unroll
+          for (int q = 0; q < 6; ++q) {
+            h[0 * 6 + q] = fma(d0, c6[5 - q], h[0 * 6 + q]);
+            h[1 * 6 + q] = fma(d1, c6[5 - q], h[1 * 6 + q]);
+            h[2 * 6 + q] = fma(d2, c6[5 - q], h[2 * 6 + q]);
+            h[3 * 6 + q] = fma(d3, c6[5 - q], h[3 * 6 + q]);
+          }
+        }
+      }
+      // reduce-scatter of the 24 sums over the 32 lanes: 24 -> 12 -> 6 -> 3 (+1 pad) -> 2 -> 1
+      {
+        const bool bA = lane & 16, bB = lane & 8, bC = lane & 4, bD = lane & 2, bE = lane & 1;
+#pragma unroll
+        for (int x = 0; x < 12; ++x) {
+          const real snd = bA ? h[x] : h[x + 12], kp = bA ? h[x + 12] : h[x];
+          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 16);
+        }
+#pragma unroll
+        for (int x = 0; x < 6; ++x) {
+          const real snd = bB ? h[x] : h[x + 6], kp = bB ? h[x + 6] : h[x];
+          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 8);
+        }
+#pragma unroll
+        for (int x = 0; x < 3; ++x) {
+          const real snd = bC ? h[x] : h[x + 3], kp = bC ? h[x + 3] : h[x];
+          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 4);
+        }
+        h[3] = real(0);
+#pragma unroll
+        for (int x = 0; x < 2; ++x) {
+          const real snd = bD ? h[x] : h[x + 2], kp = bD ? h[x + 2] : h[x];
+          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 2);
+        }
+        {
+          const real snd = bE ? h[0] : h[1], kp = bE ? h[1] : h[0];
+          h[0] = kp + __shfl_xor_sync(0xffffffffu, snd, 1);
+        }
+        const int idx = (bA ? 12 : 0) + (bB ? 6 : 0) + (bC ? 3 : 0) + (bD ? 2 : 0) + (bE ? 1 : 0);
+        if (!(bD && bE)) st.H[nrun][idx] = h[0];
+      }
+      ++nrun;
+      u = e;
+    }
+    __syncwarp();
+    if (lane < cnt) {  // row base + lane from its run's H
+      const real *Hr = st.H[st.run[lane]];
+      const real t = st.t[lane];
+      const real t2 = t * t, t3 = t2 * t, t4 = t3 * t, t5 = t4 * t;
+      const real r0 = st.r[lane][0], r1 = st.r[lane][1], r2 = st.r[lane][2], r3 = st.r[lane][3];
+      real dR[4], G[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const real *hk = Hr + 6 * k;  // H[k][q], q = 0..5
+        real v = fma(hk[5], t5, fma(hk[4], t4, fma(hk[3], t3, fma(hk[2], t2, fma(hk[1], t, hk[0])))));
+        dR[k] = v;
+        real gq = fma(real(5) * hk[5], t4, fma(real(4) * hk[4], t3, fma(real(3) * hk[3], t2, fma(real(2) * hk[2], t, hk[1]))));
+        G[k] = gq;
+      }
+      real dsv = r0 * G[0];
+      dsv = fma(r1, G[1], dsv);
+      dsv = fma(r2, G[2], dsv);
+      dsv = fma(r3, G[3], dsv);
+      const int rw = st.row[lane];
+      const int row = rw & (kClamped - 1);
+      ds_i[row] = (rw & kClamped) ? real(0) : dsv * P.inv_nnei;
+      st4(dR_i + (size_t)row * 4, dR[0] * P.inv_nnei, dR[1] * P.inv_nnei, dR[2] * P.inv_nnei, dR[3] * P.inv_nnei);
+    }
+    __syncwarp();
+  }
+
+  // padding rows, packed over the segments' padded tails
+  for (int pv = lane; pv < P.nnei - nv; pv += 32) {
+    int cum = 0, lim = P.sel[0] - st.nvb[0], off = 0, nvb_b = st.nvb[0];
+#pragma unroll
+    for (int c = 1; c < DP_MAX_TYPES; ++c)
+      if (c < P.ntypes && pv >= lim) {
+        cum = lim;
+        lim += P.sel[c] - st.nvb[c];
+        off += P.sel[c - 1];
+        nvb_b = st.nvb[c];
+      }
+    const int row = off + nvb_b + (pv - cum);
+    ds_i[row] = real(0);
+    st4(dR_i + (size_t)row * 4, real(0), real(0), real(0), real(0));
+  }
+}
+
+template <typename real>
+using GradKernel = void (*)(const GradParams<real>);
+
+template <typename real, int... Qs>
+GradKernel<real> pick_grad_moments(int Q, std::integer_sequence<int, Qs...>) {
+  GradKernel<real> k = nullptr;
+  ((Q == Qs ? (k = &grad_moments_kernel<real, Qs>, 0) : 0), ...);
+  return k;
 }
 
 // ---------------------------------------------------------------- f32
@@ -384,7 +587,7 @@ int grad_f32(const float *table, const TableGeom &g, const Segments &seg, const 
 template <typename real>
 int grad(const real *table, const dp_table_info *info, const real *s, const real *Rt, const int32_t *nvalid,
          const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, const real *dT,
-         real *ds, real *dRt, void *stream) {
+         real *ds, real *dRt, void *stream, bool moments = false) {
   clear_error();
   TableGeom g;
   Segments seg;
@@ -394,7 +597,7 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
   if (!dT) return set_error(DP_ERR_NULL, "dT is NULL");
   if (nloc > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
   if constexpr (std::is_same<real, float>::value)
-    return grad_f32(table, g, seg, s, Rt, nvalid, atype, nloc, nnei, ntypes, M1, dT, ds, dRt, stream);
+    if (!moments) return grad_f32(table, g, seg, s, Rt, nvalid, atype, nloc, nnei, ntypes, M1, dT, ds, dRt, stream);
   GradParams<real> P;
   P.table = table;
   P.s = s;
@@ -405,6 +608,7 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
   P.ds = ds;
   P.dRt = dRt;
   P.geom = g;
+  P.lgeom = GeomOf<real>::make(g);
   P.nloc = nloc;
   P.nnei = nnei;
   P.ntypes = ntypes;
@@ -412,6 +616,18 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
   P.pair_stride = g.nint * M1 * 6;
   for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
   P.inv_nnei = (real)(1.0 / (double)nnei);
+  if (moments) {
+    GradKernel<real> k =
+        pick_grad_moments<real>(M1 / 32, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
+    if (!k) return set_error(DP_ERR_UNSUPPORTED, "no moment gradient kernel for M1 = %d", M1);
+    const size_t smem = sizeof(MomentGradStage<real>) + (size_t)4 * M1 * sizeof(real);
+    if (smem > 48 * 1024) {
+      const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_tabulate_fusion_grad_moments: %s", cudaGetErrorString(e));
+    }
+    k<<<(unsigned)nloc, kMomentWarps * 32, smem, (cudaStream_t)stream>>>(P);
+    return launch_status("dp_tabulate_fusion_grad_moments");
+  }
   const int64_t ychunks = ((int64_t)kGradChunk * nnei + kGradThreads - 1) / kGradThreads;
   if (ychunks > 65535) return set_error(DP_ERR_SHAPE, "nnei = %d too large", nnei);
   const int64_t xchunks = (nloc + kGradChunk - 1) / kGradChunk;
@@ -437,6 +653,20 @@ int dp_tabulate_fusion_grad_f32(const float *table, const dp_table_info *info, c
                                 const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
                                 const int32_t *sel, int M1, const float *dT, float *ds, float *dRt, void *stream) {
   return dpc::grad<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, stream);
+}
+
+int dp_tabulate_fusion_grad_moments_f64(const double *table, const dp_table_info *info, const double *s,
+                                        const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                        int nnei, int ntypes, const int32_t *sel, int M1, const double *dT, double *ds,
+                                        double *dRt, void *stream) {
+  return dpc::grad<double>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, stream, true);
+}
+
+int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info *info, const float *s,
+                                        const float *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                        int nnei, int ntypes, const int32_t *sel, int M1, const float *dT, float *ds,
+                                        float *dRt, void *stream) {
+  return dpc::grad<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, stream, true);
 }
 
 }  // extern "C"

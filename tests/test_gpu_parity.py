@@ -351,3 +351,68 @@ def test_moments_forward_shapes(M1, widths):
         T = dpc.dp_tabulate_fusion_fwd_moments(model.table, model.info, x["s"], x["Rt"], x["nvalid"], None, w.sel)
         torch.cuda.synchronize()
         assert rel(T.double().cpu().numpy(), run_oracle(w, dtype)["T"]) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("name,kw,dtype,nsample", MOMENT_CASES,
+                         ids=[f"{c[0]}-{c[1]}-{str(c[2])[6:]}" for c in MOMENT_CASES])
+def test_moments_grad(name, kw, dtype, nsample):
+    """The interval-moment backward gives the oracle's ds and dR~, padding rows zeroed over stale outputs."""
+    dpc = lib()
+    w = workload(name, **kw)
+    model = product_model(w, dtype)
+    x = to_dev(w, dtype)
+    args = (model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel, x["dT"])
+    stale = (torch.full((w.nloc, w.nnei), 7.0, dtype=dtype, device="cuda"),
+             torch.full((w.nloc, w.nnei, 4), -3.0, dtype=dtype, device="cuda"))
+    ds, dRt = dpc.dp_tabulate_fusion_grad_moments(*args, out=stale)
+    ds0, dRt0 = dpc.dp_tabulate_fusion_grad(*args)
+    torch.cuda.synchronize()
+    atoms = None
+    if nsample:
+        rng = np.random.default_rng(4)
+        atoms = np.sort(rng.choice(w.nloc, nsample, replace=False))
+    ref = run_oracle(w, dtype, atoms=atoms)
+    got = dict(ds=ds.double().cpu().numpy(), dRt=dRt.double().cpu().numpy())
+    assert_parity(got, ref, dtype, atoms=atoms, keys=("ds", "dRt"))
+    assert rel(got["ds"], ds0.double().cpu().numpy()) <= TOL[dtype]
+    assert rel(got["dRt"], dRt0.double().cpu().numpy()) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("M1,widths", [(1, (1, 1)), (37, (1, 5, 37)), (64, (1, 16, 32, 64)), (200, (1, 50, 100, 200)),
+                                       (256, (1, 64, 128, 256))])
+def test_moments_grad_shapes(M1, widths):
+    """Long runs and every channel-round shape of the moment backward, with clamped and NaN inputs."""
+    dpc = lib()
+    w = W.tiny(seed=95 + M1, nloc=11, nreal=27, sel=30, widths=widths, M2=1, rmin=2.6, rmax=3.0)
+    s = w.s.copy()
+    s[0, 0], s[1, 2], s[2, 1] = w.s_max * 7.0, w.s_min - 1.0, np.nan  # past the coarse segment, below, NaN
+    w2 = W.Workload(**{**w.__dict__, "s": s})
+    for dtype in (torch.float64, torch.float32):
+        model = product_model(w2, dtype)
+        x = to_dev(w2, dtype)
+        ds, dRt = dpc.dp_tabulate_fusion_grad_moments(model.table, model.info, x["s"], x["Rt"], x["nvalid"], None,
+                                                      w2.sel, x["dT"])
+        torch.cuda.synchronize()
+        ref = run_oracle(w2, dtype)
+        got = dict(ds=ds.double().cpu().numpy(), dRt=dRt.double().cpu().numpy())
+        nan = np.isnan(ref["ds"])
+        assert np.array_equal(np.isnan(got["ds"]), nan)
+        got["ds"][nan] = ref["ds"][nan] = 0.0
+        nanr = np.isnan(ref["dRt"])
+        assert np.array_equal(np.isnan(got["dRt"]), nanr)
+        got["dRt"][nanr] = ref["dRt"][nanr] = 0.0
+        assert_parity(got, ref, dtype, keys=("ds", "dRt"))
+
+
+def test_moments_grad_no_valid_rows():
+    """Atoms without real neighbours: every row is padding and gets zeros over stale outputs."""
+    dpc = lib()
+    w = W.tiny(seed=7, nloc=3, nreal=5, sel=8)
+    model = product_model(w, torch.float64)
+    x = to_dev(w, torch.float64)
+    stale = (torch.ones((w.nloc, w.nnei), dtype=torch.float64, device="cuda"),
+             torch.ones((w.nloc, w.nnei, 4), dtype=torch.float64, device="cuda"))
+    ds, dRt = dpc.dp_tabulate_fusion_grad_moments(model.table, model.info, x["s"], x["Rt"],
+                                                  torch.zeros_like(x["nvalid"]), x["atype"], w.sel, x["dT"], out=stale)
+    torch.cuda.synchronize()
+    assert not ds.abs().max().item() and not dRt.abs().max().item()
