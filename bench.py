@@ -6,6 +6,9 @@ D = S S<^T (dp_descriptor_contract) and the backward from a given dE/dT
 (dp_tabulate_fusion_grad).  The table build (compression) is setup and is
 not timed.  Metric: valid neighbour x channel evaluations per second for
 fwd + grad (each valid (atom, neighbour, channel) triple counts once).
+--algo moments (default) runs the interval-moment forward and backward,
+--algo direct the per-row ones; both give the same outputs, and the
+roofline fraction is taken on the FMAs of the algorithm that ran.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload cu85] [--dtype f64]
   python bench.py --impl reference ...   # the oracle on the host cores (bounded sample)
@@ -41,6 +44,43 @@ FMA_LANES = {"f64": 2, "f32": 128}
 # algorithmic FMAs per valid neighbour x channel
 FMA_PER_EVAL = {"fwd": 9, "grad": 18}
 DESC_FMA_PER_ATOM = lambda M1, M2: 4 * M1 * M2  # noqa: E731
+
+
+# Interval-moment path: a run of L consecutive valid rows of one atom in one table
+# interval costs, in FMAs, the cheaper of its per-row form and its moment form:
+#   forward   min(9 M1 L,  24 M1 + 24 L)   (W[k][q] = sum_j R~_jk t_j^q, then T += C_l W)
+#   backward  min(18 M1 L, 24 M1 + 40 L)   (H[k][q] = sum_m dT_km C_lmq, then each row from H)
+MOMENT_FMA = {"fwd": (9, 24, 24), "grad": (18, 24, 40)}
+
+
+def interval_runs(w, info, n0: int, n1: int):
+    """Lengths of the runs of consecutive valid rows that share an atom, a type segment and a table
+    interval (the interval search of the kernels, on the host in f64)."""
+    off = np.concatenate([[0], np.cumsum(w.sel)])
+    valid = np.zeros(w.s.shape, bool)
+    seg = np.zeros(w.s.shape[1], np.int64)
+    for b in range(w.ntypes):
+        valid[:, off[b]:off[b + 1]] = np.arange(w.sel[b])[None, :] < w.nvalid[:, b:b + 1]
+        seg[off[b]:off[b + 1]] = b
+    s = w.s
+    nint = n0 + n1
+    with np.errstate(invalid="ignore"):
+        fine = np.minimum(np.floor((s - info.lower) / info.stride0), n0 - 1)
+        coarse = n0 + np.minimum(np.floor((s - info.upper) / info.stride1), n1 - 1)
+        l = np.where(s < info.lower, 0, np.where(s < info.upper, fine, np.where(s < info.upper_ext, coarse, nint - 1)))
+    key = (np.arange(w.nloc)[:, None] * w.ntypes + seg[None, :]) * nint + np.nan_to_num(l).astype(np.int64)
+    k = key[valid]  # row-major: atom, then segment, then row
+    if k.size == 0:
+        return np.zeros(0, np.int64)
+    starts = np.flatnonzero(np.concatenate([[True], k[1:] != k[:-1]]))
+    return np.diff(np.concatenate([starts, [k.size]]))
+
+
+def moment_fmas(runs, M1: int) -> dict:
+    out = {}
+    for kern, (per_row, per_run, per_row_m) in MOMENT_FMA.items():
+        out[kern] = float(np.minimum(per_row * M1 * runs, per_run * M1 + per_row_m * runs).sum())
+    return out
 
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
@@ -228,7 +268,10 @@ def run_native(args, rank, world, local_rank):
                                                 world, barrier, evals_all)
     if rank != 0:
         return None
-    return report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall)
+    fmas = None
+    if args.algo == "moments":
+        fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
+    return report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas)
 
 
 def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_all):
@@ -292,11 +335,13 @@ def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_al
             "d2h_bytes_per_step": d2h, "pipelined": "double-buffered, uploads and downloads on their own streams"}
 
 
-def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall):
+def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas=None):
     value = evals_all * args.steps / total_s
-    # ---- roofline of the dominant kernel (FMA pipe of the path's dtype)
+    # ---- roofline of the dominant kernel (FMA pipe of the path's dtype), on the FMAs of the
+    # algorithm the kernels run: per-row evaluation, or interval moments (fmas, from the run lengths)
     mean = {k: sum(v) / len(v) for k, v in k_ms.items()}
-    flops = {"fwd": 2.0 * FMA_PER_EVAL["fwd"] * w.evals, "grad": 2.0 * FMA_PER_EVAL["grad"] * w.evals,
+    fmas = fmas or {"fwd": FMA_PER_EVAL["fwd"] * w.evals, "grad": FMA_PER_EVAL["grad"] * w.evals}
+    flops = {"fwd": 2.0 * fmas["fwd"], "grad": 2.0 * fmas["grad"],
              "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
     pk = peak_tflops(args.dtype)
     kernels = {k: {"ms": round(mean[k], 4), "share": round(mean[k] / sum(mean.values()), 4),
@@ -319,6 +364,9 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall):
                    "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
                                    else f"atoms split over {world} ranks"),
                    "step": "fwd + descriptor + grad", "algo": args.algo,
+                   "fma_basis": ("interval moments: per run min(9 M1 L, 24 M1 + 24 L) fwd, "
+                                 "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
+                                 else "per row: 9 M1 fwd, 18 M1 grad"),
                    "l2": "flushed between steps (256 MiB write)",
                    "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4)},
         "atoms_per_s": w.nloc * world * args.steps / total_s,
@@ -431,7 +479,7 @@ def main():
     ap.add_argument("--seed", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
-    ap.add_argument("--algo", choices=["direct", "moments"], default="direct",
+    ap.add_argument("--algo", choices=["direct", "moments"], default="moments",
                     help="direct: per-neighbour evaluation (the paper's fused kernel); moments: interval moments")
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")

@@ -200,11 +200,13 @@ __device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, co
   }
 }
 
-// One atom: T_i into P.T (the whole warp takes part).// One atom: T_i into P.T (the whole warp takes part).  kMoments: runs of
+// One atom: T_i into P.T (the whole warp takes part).  kMoments: runs of
 // neighbours sharing an interval are contracted through their moments
 //   W[k][q] = sum_{j in run} R~_j[k] t_j^q,   T[k][m] += sum_q C_{l,m,q} W[k][q]
 // (C_{l,m,q} the t^q coefficient of channel m on interval l): the same sum as
-// the per-neighbour evaluation, associated per interval.
+// the per-neighbour evaluation, associated per interval.  A run that reaches
+// the end of a 32-row batch keeps its partial W for the next batch, so that a
+// run costs one T update however the batches cut it.
 template <typename real, int Q, bool kMoments>
 __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &st, MomentStage<real> &ms,
                                          const int lane, const int64_t i) {
@@ -241,6 +243,31 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
   real rcf[6];
   int rcur = -1;
   real cf[Q > 0 ? Q : 1][6];  // f32: coefficients of the interval in use
+  // T += C_l W for the run in interval block `off`, W[6k + q] held by lanes 0..23 (uniform call)
+  auto apply_moments = [&](int off, real wv) {
+    if (lane < 24) ms.w[lane] = wv;
+    __syncwarp();
+    real W[4][6];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+      for (int q = 0; q < 6; ++q) W[k][q] = ms.w[6 * k + q];
+#pragma unroll
+    for (int r = 0; r < (Q > 0 ? Q : 1); ++r) {
+      real c6[6];  // (a, b, c, d, e, f) = coefficients of t^5 .. t^0
+      ld6(tab + off, P.M1, r * 32 + lane, c6);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        real v = acc[r][k];
+#pragma unroll
+        for (int q = 0; q < 6; ++q) v = fma(c6[5 - q], W[k][q], v);
+        acc[r][k] = v;
+      }
+    }
+    __syncwarp();
+  };
+  int carry_off = -1;  // run left open at the end of the previous batch (uniform)
+  real wcarry = real(0);  // its partial W on lanes 0..23
   for (int base = 0; base < nv; base += 32) {
     // stage: lane l prepares valid neighbour base + l
     const int v = base + lane;
@@ -278,42 +305,35 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     __syncwarp();
     const int cnt = min(32, nv - base);
     if (Q > 0 && kMoments) {
+      if (carry_off >= 0 && st.off[0] != carry_off) {  // the open run ended with the last batch
+        apply_moments(carry_off, wcarry);
+        carry_off = -1;
+      }
+      int next_carry = -1;
       int u = 0;
       while (u < cnt) {  // uniform, run by run
         const int off = st.off[u];
         int e = u + 1;
         while (e < cnt && st.off[e] == off) ++e;
-        if (e - u >= kMinMomentRun) {
-          real wv = real(0);
+        const bool cont = u == 0 && off == carry_off;
+        if (cont || e - u >= kMinMomentRun) {
+          real wv = cont ? wcarry : real(0);
           if (lane < 24) {
             const int k = lane / 6, q = lane - 6 * (lane / 6);
             for (int j = u; j < e; ++j) wv = fma(st.r[j][k], ms.tp[j][q], wv);
-            ms.w[lane] = wv;
           }
-          __syncwarp();
-          real W[4][6];
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-#pragma unroll
-            for (int q = 0; q < 6; ++q) W[k][q] = ms.w[6 * k + q];
-#pragma unroll
-          for (int r = 0; r < Q; ++r) {
-            real c6[6];  // (a, b, c, d, e, f) = coefficients of t^5 .. t^0
-            ld6(tab + off, P.M1, r * 32 + lane, c6);
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-              real v = acc[r][k];
-#pragma unroll
-              for (int q = 0; q < 6; ++q) v = fma(c6[5 - q], W[k][q], v);
-              acc[r][k] = v;
-            }
+          if (e == cnt && base + 32 < nv) {  // may go on in the next batch: keep W open
+            wcarry = wv;
+            next_carry = off;
+          } else {
+            apply_moments(off, wv);
           }
-          __syncwarp();
         } else {
           for (int j = u; j < e; ++j) fwd_neighbour<real, Q>(P, tab, lane, off, st.t[j], st.r[j], acc);
         }
         u = e;
       }
+      carry_off = next_carry;
     } else if (Q > 0) {
       if constexpr (kCache) {
         // f32: walk the batch run by run.  Neighbours are sorted by distance

@@ -180,21 +180,66 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 // One warp per atom.  For each run the lanes form H over their channels
 // (24 FMA per channel) and a reduce-scatter butterfly sums the 24 values
 // over the lanes (24 DADD); then every lane takes one row of the batch and
-// evaluates its 5 outputs from its run's H (about 50 FMA per row).  A run
-// costs ~100 warp instructions plus ~1.5 per row, against 56 per row for the
-// per-row kernel.
+// evaluates its outputs from its run's H (about 40 FMA per row).  A run costs
+// ~(24 ceil(M1/32) + 24) warp instructions plus ~1.5 per row, against
+// 18 M1/32 per row for the per-row evaluation, so in f64 runs shorter than
+// min_grad_run rows are queued and evaluated per row instead: one row per
+// lane, all channels in turn, 32 queued rows at a time.  In f32 the per-row
+// loop is bound by its scattered coefficient loads rather than by the FMA
+// pipe, and every run goes through H.
 constexpr int kMomentWarps = 1;
+template <typename real>
+constexpr int min_grad_run() { return sizeof(real) == 8 ? 3 : 1; }
 
 template <typename real>
 struct alignas(16) MomentGradStage {
   real r[32][4];     // R~ rows of the batch
   real t[32];        // local variable t
-  real H[32][24];    // H of each run of the batch, [run][4*k + q... laid out k-major]
+  // H of each long run of the batch, H[run][6*k + q], and two slots for the
+  // last run of a batch, whose H is kept for the next batch's first rows
+  real H[32 / min_grad_run<real>() + 2][25];  // rows padded to 25: lanes reading different runs hit different banks
+  real qr[64][4];    // queue of rows of short runs: R~, t, block offset, row
+  real qt[64];
+  int32_t qoff[64];
+  int32_t qrow[64];
   int32_t off[32];   // interval block offset
   int32_t row[32];   // row index, bit 30 set when s was clamped
-  int32_t run[32];   // run index of each row of the batch
+  int32_t run[32];   // run index of each row of the batch, -1 for queued rows
   int32_t nvb[DP_MAX_TYPES];
 };
+
+// One queued row on this lane: the per-row backward over all channels.
+template <typename real>
+__device__ __forceinline__ void grad_row_direct(const real *__restrict__ blk, const real *dts, int M1, const real t,
+                                                const real r0, const real r1, const real r2, const real r3,
+                                                real &a_ds, real &a_0, real &a_1, real &a_2, real &a_3) {
+  a_ds = a_0 = a_1 = a_2 = a_3 = real(0);
+#pragma unroll 2
+  for (int m = 0; m < M1; ++m) {
+    real cf[6];
+    ld6(blk, M1, m, cf);
+    const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
+    real p = fma(cf[0], t, cf[1]);  // g and g' by Horner's rule with derivative
+    real dp = cf[0];
+    dp = fma(dp, t, p);
+    p = fma(p, t, cf[2]);
+    dp = fma(dp, t, p);
+    p = fma(p, t, cf[3]);
+    dp = fma(dp, t, p);
+    p = fma(p, t, cf[4]);
+    dp = fma(dp, t, p);
+    p = fma(p, t, cf[5]);
+    real rm = d0 * r0;
+    rm = fma(d1, r1, rm);
+    rm = fma(d2, r2, rm);
+    rm = fma(d3, r3, rm);
+    a_ds = fma(rm, dp, a_ds);
+    a_0 = fma(d0, p, a_0);
+    a_1 = fma(d1, p, a_1);
+    a_2 = fma(d2, p, a_2);
+    a_3 = fma(d3, p, a_3);
+  }
+}
 
 template <typename real, int Q>
 __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const GradParams<real> P) {
@@ -231,6 +276,94 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
   real *__restrict__ ds_i = P.ds + i * P.nnei;
   real *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
 
+  // queued rows: lane j evaluates queue entry j (when j < n)
+  auto drain = [&](int n) {
+    if (lane < n) {
+      real a_ds, a0, a1, a2, a3;
+      grad_row_direct(tab + st.qoff[lane], dts, M1, st.qt[lane], st.qr[lane][0], st.qr[lane][1], st.qr[lane][2],
+                      st.qr[lane][3], a_ds, a0, a1, a2, a3);
+      const int rw = st.qrow[lane];
+      const int row = rw & (kClamped - 1);
+      ds_i[row] = (rw & kClamped) ? real(0) : a_ds * P.inv_nnei;
+      st4(dR_i + (size_t)row * 4, a0 * P.inv_nnei, a1 * P.inv_nnei, a2 * P.inv_nnei, a3 * P.inv_nnei);
+    }
+  };
+  // H[slot] of the run in interval block `off` (uniform call; all lanes)
+  auto form_H = [&](int off, int slot) {
+    real h[24];
+#pragma unroll
+    for (int x = 0; x < 24; ++x) h[x] = real(0);
+    const real *__restrict__ blk = tab + off;
+#pragma unroll
+    for (int r = 0; r <= Q; ++r) {
+      const int m = 32 * r + lane;
+      if (r < Q || lane < RR) {  // last round: the RR remainder channels
+        real c6[6];  // (a..f): coefficients of t^5 .. t^0
+        ld6(blk, M1, m, c6);
+        const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
+#pragma unroll
+        for (int q = 0; q < 6; ++q) {
+          h[0 * 6 + q] = fma(d0, c6[5 - q], h[0 * 6 + q]);
+          h[1 * 6 + q] = fma(d1, c6[5 - q], h[1 * 6 + q]);
+          h[2 * 6 + q] = fma(d2, c6[5 - q], h[2 * 6 + q]);
+          h[3 * 6 + q] = fma(d3, c6[5 - q], h[3 * 6 + q]);
+        }
+      }
+    }
+    // reduce-scatter of the 24 sums over the 32 lanes: 24 -> 12 -> 6 -> 3 (+1 pad) -> 2 -> 1
+    const bool bA = lane & 16, bB = lane & 8, bC = lane & 4, bD = lane & 2, bE = lane & 1;
+#pragma unroll
+    for (int x = 0; x < 12; ++x) {
+      const real snd = bA ? h[x] : h[x + 12], kp = bA ? h[x + 12] : h[x];
+      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 16);
+    }
+#pragma unroll
+    for (int x = 0; x < 6; ++x) {
+      const real snd = bB ? h[x] : h[x + 6], kp = bB ? h[x + 6] : h[x];
+      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 8);
+    }
+#pragma unroll
+    for (int x = 0; x < 3; ++x) {
+      const real snd = bC ? h[x] : h[x + 3], kp = bC ? h[x + 3] : h[x];
+      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 4);
+    }
+    h[3] = real(0);
+#pragma unroll
+    for (int x = 0; x < 2; ++x) {
+      const real snd = bD ? h[x] : h[x + 2], kp = bD ? h[x + 2] : h[x];
+      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 2);
+    }
+    {
+      const real snd = bE ? h[0] : h[1], kp = bE ? h[1] : h[0];
+      h[0] = kp + __shfl_xor_sync(0xffffffffu, snd, 1);
+    }
+    const int idx = (bA ? 12 : 0) + (bB ? 6 : 0) + (bC ? 3 : 0) + (bD ? 2 : 0) + (bE ? 1 : 0);
+    if (!(bD && bE)) st.H[slot][idx] = h[0];
+  };
+  // outputs of one row (this lane) from its run's H
+  auto eval_row = [&](const real *Hr, real t, real r0, real r1, real r2, real r3, int rw) {
+    const real t2 = t * t, t3 = t2 * t, t4 = t3 * t, t5 = t4 * t;
+    real dR[4], G[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const real *hk = Hr + 6 * k;  // H[k][q], q = 0..5
+      dR[k] = fma(hk[5], t5, fma(hk[4], t4, fma(hk[3], t3, fma(hk[2], t2, fma(hk[1], t, hk[0])))));
+      G[k] = fma(real(5) * hk[5], t4,
+                 fma(real(4) * hk[4], t3, fma(real(3) * hk[3], t2, fma(real(2) * hk[2], t, hk[1]))));
+    }
+    real dsv = r0 * G[0];
+    dsv = fma(r1, G[1], dsv);
+    dsv = fma(r2, G[2], dsv);
+    dsv = fma(r3, G[3], dsv);
+    const int row = rw & (kClamped - 1);
+    ds_i[row] = (rw & kClamped) ? real(0) : dsv * P.inv_nnei;
+    st4(dR_i + (size_t)row * 4, dR[0] * P.inv_nnei, dR[1] * P.inv_nnei, dR[2] * P.inv_nnei, dR[3] * P.inv_nnei);
+  };
+  constexpr int kSlots = 32 / min_grad_run<real>();
+  int nq = 0;           // queued rows (uniform)
+  int carry_off = -1;   // interval block of the last batch's last run, if its H is kept
+  int carry_slot = kSlots;
+
   for (int base = 0; base < nv; base += 32) {
     const int cnt = min(32, nv - base);
     if (lane < cnt) {  // stage row base + lane
@@ -253,97 +386,94 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
       st.r[lane][1] = rr.y;
       st.r[lane][2] = rr.z;
       st.r[lane][3] = rr.w;
-      st.t[lane] = (real)t;
+      st.t[lane] = t;
       st.off[lane] = (b * P.geom.nint + l) * M1 * 6;
       st.row[lane] = row | (clamped ? kClamped : 0);
     }
     __syncwarp();
-    // runs of the batch: H of each, written to st.H[run]
-    int nrun = 0;
-    for (int u = 0; u < cnt;) {  // uniform
+    int nrun = 0, next_off = -1, next_slot = carry_slot;
+    for (int u = 0; u < cnt;) {  // runs of the batch (uniform control flow)
       const int off = st.off[u];
       int e = u + 1;
       while (e < cnt && st.off[e] == off) ++e;
-      if (lane >= u && lane < e) st.run[lane] = nrun;
-      real h[24];
-#pragma unroll
-      for (int x = 0; x < 24; ++x) h[x] = real(0);
-      const real *__restrict__ blk = tab + off;
-#pragma unroll
-      for (int r = 0; r <= Q; ++r) {
-        const int m = 32 * r + lane;
-        if (r < Q || lane < RR) {  // last round: the RR remainder channels
-          real c6[6];  // (a..f): coefficients of t^5 .. t^0
-          ld6(blk, M1, m, c6);
-          const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
-#pragma unroll
-          for (int q = 0; q < 6; ++q) {
-            h[0 * 6 + q] = fma(d0, c6[5 - q], h[0 * 6 + q]);
-            h[1 * 6 + q] = fma(d1, c6[5 - q], h[1 * 6 + q]);
-            h[2 * 6 + q] = fma(d2, c6[5 - q], h[2 * 6 + q]);
-            h[3 * 6 + q] = fma(d3, c6[5 - q], h[3 * 6 + q]);
-          }
+      if (u == 0 && off == carry_off) {  // the previous batch's last run goes on: its H is kept
+        if (lane < e) st.run[lane] = carry_slot;
+        if (e == cnt) next_off = off;
+      } else if (e - u < min_grad_run<real>()) {  // short run: queue its rows
+        const int j = u + lane;
+        if (j < e) {
+          st.run[j] = -1;
+          st.qr[nq + lane][0] = st.r[j][0];
+          st.qr[nq + lane][1] = st.r[j][1];
+          st.qr[nq + lane][2] = st.r[j][2];
+          st.qr[nq + lane][3] = st.r[j][3];
+          st.qt[nq + lane] = st.t[j];
+          st.qoff[nq + lane] = off;
+          st.qrow[nq + lane] = st.row[j];
         }
+        nq += e - u;
+      } else {
+        int slot = nrun;
+        if (e == cnt) {  // the batch's last run may go on in the next batch: keep its H
+          slot = next_slot = carry_slot == kSlots ? kSlots + 1 : kSlots;
+          next_off = off;
+        } else {
+          ++nrun;
+        }
+        if (lane >= u && lane < e) st.run[lane] = slot;
+        form_H(off, slot);
       }
-      // reduce-scatter of the 24 sums over the 32 lanes: 24 -> 12 -> 6 -> 3 (+1 pad) -> 2 -> 1
-      {
-        const bool bA = lane & 16, bB = lane & 8, bC = lane & 4, bD = lane & 2, bE = lane & 1;
-#pragma unroll
-        for (int x = 0; x < 12; ++x) {
-          const real snd = bA ? h[x] : h[x + 12], kp = bA ? h[x + 12] : h[x];
-          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 16);
-        }
-#pragma unroll
-        for (int x = 0; x < 6; ++x) {
-          const real snd = bB ? h[x] : h[x + 6], kp = bB ? h[x + 6] : h[x];
-          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 8);
-        }
-#pragma unroll
-        for (int x = 0; x < 3; ++x) {
-          const real snd = bC ? h[x] : h[x + 3], kp = bC ? h[x + 3] : h[x];
-          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 4);
-        }
-        h[3] = real(0);
-#pragma unroll
-        for (int x = 0; x < 2; ++x) {
-          const real snd = bD ? h[x] : h[x + 2], kp = bD ? h[x + 2] : h[x];
-          h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 2);
-        }
-        {
-          const real snd = bE ? h[0] : h[1], kp = bE ? h[1] : h[0];
-          h[0] = kp + __shfl_xor_sync(0xffffffffu, snd, 1);
-        }
-        const int idx = (bA ? 12 : 0) + (bB ? 6 : 0) + (bC ? 3 : 0) + (bD ? 2 : 0) + (bE ? 1 : 0);
-        if (!(bD && bE)) st.H[nrun][idx] = h[0];
-      }
-      ++nrun;
       u = e;
     }
+    carry_off = next_off;
+    carry_slot = next_slot;
     __syncwarp();
-    if (lane < cnt) {  // row base + lane from its run's H
-      const real *Hr = st.H[st.run[lane]];
-      const real t = st.t[lane];
-      const real t2 = t * t, t3 = t2 * t, t4 = t3 * t, t5 = t4 * t;
-      const real r0 = st.r[lane][0], r1 = st.r[lane][1], r2 = st.r[lane][2], r3 = st.r[lane][3];
-      real dR[4], G[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const real *hk = Hr + 6 * k;  // H[k][q], q = 0..5
-        real v = fma(hk[5], t5, fma(hk[4], t4, fma(hk[3], t3, fma(hk[2], t2, fma(hk[1], t, hk[0])))));
-        dR[k] = v;
-        real gq = fma(real(5) * hk[5], t4, fma(real(4) * hk[4], t3, fma(real(3) * hk[3], t2, fma(real(2) * hk[2], t, hk[1]))));
-        G[k] = gq;
+    if (lane < cnt && st.run[lane] >= 0)
+      eval_row(st.H[st.run[lane]], st.t[lane], st.r[lane][0], st.r[lane][1], st.r[lane][2], st.r[lane][3],
+               st.row[lane]);
+    if (nq >= 32) {  // a full queue: one row per lane, then keep the overflow
+      drain(32);
+      __syncwarp();
+      if (lane < nq - 32) {
+        st.qr[lane][0] = st.qr[32 + lane][0];
+        st.qr[lane][1] = st.qr[32 + lane][1];
+        st.qr[lane][2] = st.qr[32 + lane][2];
+        st.qr[lane][3] = st.qr[32 + lane][3];
+        st.qt[lane] = st.qt[32 + lane];
+        st.qoff[lane] = st.qoff[32 + lane];
+        st.qrow[lane] = st.qrow[32 + lane];
       }
-      real dsv = r0 * G[0];
-      dsv = fma(r1, G[1], dsv);
-      dsv = fma(r2, G[2], dsv);
-      dsv = fma(r3, G[3], dsv);
-      const int rw = st.row[lane];
-      const int row = rw & (kClamped - 1);
-      ds_i[row] = (rw & kClamped) ? real(0) : dsv * P.inv_nnei;
-      st4(dR_i + (size_t)row * 4, dR[0] * P.inv_nnei, dR[1] * P.inv_nnei, dR[2] * P.inv_nnei, dR[3] * P.inv_nnei);
+      nq -= 32;
     }
     __syncwarp();
+  }
+  if (nq > 0) {
+    // The rest of the queue costs 18 M1 warp FMA per row-per-lane pass however
+    // few lanes it fills, or ~24 (ceil(M1/32) + 1) per run through H: take the cheaper.
+    int nr = 1;
+    for (int u = 1; u < nq; ++u) nr += st.qoff[u] != st.qoff[u - 1];
+    if (nr * 24 * ((M1 + 31) / 32 + 1) < 18 * M1) {
+      for (int u = 0; u < nq;) {  // groups of at most kSlots runs
+        const int g0 = u;
+        int nrun = 0;
+        while (u < nq && nrun < kSlots) {
+          const int off = st.qoff[u];
+          int e = u + 1;
+          while (e < nq && st.qoff[e] == off) ++e;
+          if (lane >= u && lane < e) st.run[lane] = nrun;
+          form_H(off, nrun);
+          ++nrun;
+          u = e;
+        }
+        __syncwarp();
+        if (lane >= g0 && lane < u)
+          eval_row(st.H[st.run[lane]], st.qt[lane], st.qr[lane][0], st.qr[lane][1], st.qr[lane][2], st.qr[lane][3],
+                   st.qrow[lane]);
+        __syncwarp();
+      }
+    } else {
+      drain(nq);
+    }
   }
 
   // padding rows, packed over the segments' padded tails

@@ -1,0 +1,62 @@
+"""The bench's FMA accounting for the interval-moment path (CPU only): run lengths against a
+row-by-row walk, and the per-run cost rule on hand-made runs."""
+import math
+
+import numpy as np
+
+import bench
+import oracle
+import workloads as W
+
+
+def _walk_runs(w, info):
+    """Row by row: a new run starts at every atom, type segment or interval change."""
+    off = np.concatenate([[0], np.cumsum(w.sel)])
+    runs = []
+    for i in range(w.nloc):
+        prev, n = None, 0
+        for b in range(w.ntypes):
+            for j in range(int(w.nvalid[i, b])):
+                x = float(w.s[i, off[b] + j])
+                if x < info.lower:
+                    l = 0
+                elif x < info.upper:
+                    l = min(int(math.floor((x - info.lower) / info.stride0)), info.n0 - 1)
+                elif x < info.upper_ext:
+                    l = info.n0 + min(int(math.floor((x - info.upper) / info.stride1)), info.n1 - 1)
+                else:
+                    l = info.n0 + info.n1 - 1
+                if (b, l) == prev:
+                    n += 1
+                else:
+                    if n:
+                        runs.append(n)
+                    prev, n = (b, l), 1
+        if n:
+            runs.append(n)
+    return np.array(runs)
+
+
+def test_interval_runs_match_a_row_walk():
+    o = oracle.default()
+    for w in (W.water(seed=3, nmol=128), W.tiny(seed=4, nloc=17, nreal=29, sel=31, rmin=2.6, rmax=3.0)):
+        info = o.table_info(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+        s = w.s.copy()
+        s[0, 0], s[1, 1] = info.upper_ext + 1.0, info.lower - 1.0  # clamped rows join the end intervals
+        w = W.Workload(**{**w.__dict__, "s": s})
+        got = bench.interval_runs(w, info, info.n0, info.n1)
+        ref = _walk_runs(w, info)
+        assert np.array_equal(got, ref)
+        assert got.sum() == int(w.nvalid.sum())
+
+
+def test_moment_fmas_take_the_cheaper_form():
+    M1 = 100
+    runs = np.array([1, 2, 3, 10, 400])
+    f = bench.moment_fmas(runs, M1)
+    fwd = sum(min(9 * M1 * L, 24 * M1 + 24 * L) for L in runs)
+    grad = sum(min(18 * M1 * L, 24 * M1 + 40 * L) for L in runs)
+    assert f == {"fwd": float(fwd), "grad": float(grad)}
+    # singletons stay per row, long runs go through moments
+    assert bench.moment_fmas(np.array([1]), M1)["fwd"] == 9 * M1
+    assert bench.moment_fmas(np.array([400]), M1)["grad"] == 24 * M1 + 40 * 400
