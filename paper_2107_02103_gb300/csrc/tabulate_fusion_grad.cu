@@ -177,71 +177,239 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 //   H[k][q] = sum_m dT[k][m] C_{l,m,q}                 (C_{l,m,q}: t^q coefficient)
 //   dE/dR~_j[k] = (1/N_c) sum_q t_j^q H[k][q]
 //   dE/ds_j     = (1/N_c) sum_k R~_j[k] sum_{q>=1} q t_j^(q-1) H[k][q]
-// One warp per atom.  For each run the lanes form H over their channels
-// (24 FMA per channel) and a reduce-scatter butterfly sums the 24 values
-// over the lanes (24 DADD); then every lane takes one row of the batch and
-// evaluates its outputs from its run's H (about 40 FMA per row).  A run costs
-// ~(24 ceil(M1/32) + 24) warp instructions plus ~1.5 per row, against
-// 18 M1/32 per row for the per-row evaluation, so in f64 runs shorter than
-// min_grad_run rows are queued and evaluated per row instead: one row per
-// lane, all channels in turn, 32 queued rows at a time.  In f32 the per-row
-// loop is bound by its scattered coefficient loads rather than by the FMA
-// pipe, and every run goes through H.
+// One warp per atom.  Rows are staged 32 at a time (one per lane) into a
+// chunk of up to kChunkRows rows and cut into runs; a run that reaches the end
+// of a batch stays open for the next one.  When the chunk is full, the H of
+// its runs are formed G runs at a time: lane = (run p, channel lane c) with
+// C = 32/G channel lanes per run, each lane summing 24 products over the
+// channels c, c + C, ... and a reduce-scatter over the C lanes finishing the
+// sums.  Per run that is 24 M1/32 FMA (the sum itself) plus 24 log-steps'
+// worth of DADD shared by G runs: with G = 8 the adds cost ~2 per run instead
+// of 24 with one run across the warp.  Then every staged row (one per lane)
+// follows from its run's H by Horner's rule with derivative (~45 FMA).  The
+// H of an open run is kept for the next chunk.
+//
+// In f64 a single-row run is cheaper evaluated directly (18 M1 FMA over the
+// channels, against 24 M1 for its H): such rows are queued and evaluated
+// G = 8 rows at a time in the same lane layout, the five outputs of a row
+// finished by a reduce-scatter over its C lanes.  In f32 the per-row form is
+// bound by its scattered coefficient loads, and every run goes through H.
 constexpr int kMomentWarps = 1;
+constexpr int kChunkRows = 128;  // rows staged per chunk
 template <typename real>
-constexpr int min_grad_run() { return sizeof(real) == 8 ? 3 : 1; }
+constexpr int min_grad_run() { return sizeof(real) == 8 ? 2 : 1; }
+// H slots per chunk (plus one for an open run's H), and the most runs one batch can add
+template <typename real>
+constexpr int chunk_runs() { return sizeof(real) == 8 ? 32 : 64; }
+template <typename real>
+constexpr int batch_runs() { return 32 / min_grad_run<real>() + 1; }
 
 template <typename real>
 struct alignas(16) MomentGradStage {
-  real r[32][4];     // R~ rows of the batch
-  real t[32];        // local variable t
-  // H of each long run of the batch, H[run][6*k + q], and two slots for the
-  // last run of a batch, whose H is kept for the next batch's first rows
-  real H[32 / min_grad_run<real>() + 2][25];  // rows padded to 25: lanes reading different runs hit different banks
-  real qr[64][4];    // queue of rows of short runs: R~, t, block offset, row
-  real qt[64];
-  int32_t qoff[64];
+  real r[kChunkRows][4];  // R~ rows of the chunk
+  real t[kChunkRows];     // local variable t
+  real H[chunk_runs<real>() + 1][25];  // H[run][6*k + q]; rows padded to 25 so that lanes reading different runs hit different banks
+  int32_t qoff[64];  // queue of single-row runs: interval block offset and row (t and R~ are read again)
   int32_t qrow[64];
-  int32_t off[32];   // interval block offset
-  int32_t row[32];   // row index, bit 30 set when s was clamped
-  int32_t run[32];   // run index of each row of the batch, -1 for queued rows
+  int32_t off[kChunkRows];      // interval block offset of each staged row
+  int32_t row[kChunkRows];      // row index, bit 30 set when s was clamped
+  int32_t slot[kChunkRows];     // H slot of the row's run, -1 for queued rows
+  int32_t run_off[chunk_runs<real>() + 1];  // interval block offset of each H slot
   int32_t nvb[DP_MAX_TYPES];
 };
 
-// One queued row on this lane: the per-row backward over all channels.
-template <typename real>
-__device__ __forceinline__ void grad_row_direct(const real *__restrict__ blk, const real *dts, int M1, const real t,
-                                                const real r0, const real r1, const real r2, const real r3,
-                                                real &a_ds, real &a_0, real &a_1, real &a_2, real &a_3) {
-  a_ds = a_0 = a_1 = a_2 = a_3 = real(0);
-#pragma unroll 2
-  for (int m = 0; m < M1; ++m) {
-    real cf[6];
-    ld6(blk, M1, m, cf);
-    const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
-    real p = fma(cf[0], t, cf[1]);  // g and g' by Horner's rule with derivative
-    real dp = cf[0];
-    dp = fma(dp, t, p);
-    p = fma(p, t, cf[2]);
-    dp = fma(dp, t, p);
-    p = fma(p, t, cf[3]);
-    dp = fma(dp, t, p);
-    p = fma(p, t, cf[4]);
-    dp = fma(dp, t, p);
-    p = fma(p, t, cf[5]);
-    real rm = d0 * r0;
-    rm = fma(d1, r1, rm);
-    rm = fma(d2, r2, rm);
-    rm = fma(d3, r3, rm);
-    a_ds = fma(rm, dp, a_ds);
-    a_0 = fma(d0, p, a_0);
-    a_1 = fma(d1, p, a_1);
-    a_2 = fma(d2, p, a_2);
-    a_3 = fma(d3, p, a_3);
+__host__ __device__ constexpr int ilog2(int c) { return c > 1 ? 1 + ilog2(c / 2) : 0; }
+
+// Values a lane holds after `step` halvings of n values (an odd count is
+// padded with a zero before it is halved; a single value is not split).
+__host__ __device__ constexpr int rs_count(int n, int step) {
+  for (int k = 0; k < step; ++k)
+    if (n > 1) n = (n + 1) / 2;
+  return n;
+}
+
+// Reduce-scatter of N partial sums over groups of C lanes (C a power of two,
+// groups aligned to C): each step halves the values a lane holds and adds the
+// partner lane's other half; once a lane holds one value the remaining steps
+// add it to the partner's and the lower lane keeps it.  On return the lane
+// holds the group's totals of components base .. base + nreal - 1 in
+// h[0 .. nreal-1]; h needs room for N + 1 values (the padding zero).
+template <int n, int mask, typename real>
+__device__ __forceinline__ void rs_step(real *h, int lane, int &base, int &nreal) {
+  if constexpr (mask >= 1) {
+    const bool hi = lane & mask;
+    if constexpr (n == 1) {
+      h[0] += __shfl_xor_sync(0xffffffffu, h[0], mask);
+      if (hi) nreal = 0;
+      rs_step<1, mask / 2>(h, lane, base, nreal);
+    } else {
+      if constexpr ((n & 1) != 0) h[n] = real(0);
+      constexpr int half = (n + 1) / 2;
+#pragma unroll
+      for (int x = 0; x < half; ++x) {
+        const real snd = hi ? h[x] : h[x + half], kp = hi ? h[x + half] : h[x];
+        h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, mask);
+      }
+      if (hi) {
+        base += half;
+        nreal = max(nreal - half, 0);
+      } else {
+        nreal = min(nreal, half);
+      }
+      rs_step<half, mask / 2>(h, lane, base, nreal);
+    }
   }
 }
 
-template <typename real, int Q>
+template <int N, int C, typename real>
+__device__ __forceinline__ void reduce_scatter(real *h, int lane, int &base, int &nreal) {
+  base = 0;
+  nreal = N;
+  rs_step<N, C / 2>(h, lane, base, nreal);
+}
+
+// H of the runs in slots s0 .. s0+G-1 (those below nrun): lane = (run p, channel lane c),
+// C = 32/G channel lanes per run, each summing over the channels c, c + C, ...
+template <int G, typename real>
+__device__ __forceinline__ void form_H_group(MomentGradStage<real> &st, const real *__restrict__ tab,
+                                             const real *dts, int M1, int s0, int nrun, int lane) {
+  constexpr int C = 32 / G;
+  const int p = lane / C, c = lane - p * C;
+  const int slot = s0 + p;
+  const bool valid = slot < nrun;
+  const real *__restrict__ blk = tab + st.run_off[valid ? slot : s0];
+  real h[25];
+#pragma unroll
+  for (int x = 0; x < 24; ++x) h[x] = real(0);
+#pragma unroll 2
+  for (int m = c; m < M1; m += C) {
+    real c6[6];  // (a..f): coefficients of t^5 .. t^0
+    ld6(blk, M1, m, c6);
+    const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
+#pragma unroll
+    for (int q = 0; q < 6; ++q) {
+      h[0 * 6 + q] = fma(d0, c6[5 - q], h[0 * 6 + q]);
+      h[1 * 6 + q] = fma(d1, c6[5 - q], h[1 * 6 + q]);
+      h[2 * 6 + q] = fma(d2, c6[5 - q], h[2 * 6 + q]);
+      h[3 * 6 + q] = fma(d3, c6[5 - q], h[3 * 6 + q]);
+    }
+  }
+  int base, nreal;
+  reduce_scatter<24, C>(h, lane, base, nreal);
+  if (valid) {
+#pragma unroll
+    for (int x = 0; x < rs_count(24, ilog2(C)); ++x)
+      if (x < nreal) st.H[slot][base + x] = h[x];
+  }
+}
+
+// Per-row backward of queued rows q0 .. q0+G-1 (those below nq): lane = (row p, channel lane c),
+// each lane summing the five outputs over the channels c, c + C, ... (18 FMA per channel).
+template <int G, typename real>
+__device__ __forceinline__ void grad_rows_group(const GradParams<real> &P, const MomentGradStage<real> &st,
+                                                const real *__restrict__ tab, const real *dts, int64_t i, int q0,
+                                                int nq, int lane) {
+  constexpr int kClamped = 1 << 30;
+  constexpr int C = 32 / G;
+  const int p = lane / C, c = lane - p * C;
+  const int q = q0 + p;
+  const bool valid = q < nq;
+  const int e = valid ? q : q0;
+  const int rw = st.qrow[e];
+  const int row = rw & (kClamped - 1);
+  const Vec4<real> rr = ld4(P.Rt + (i * P.nnei + row) * 4);
+  real t;
+  bool clamped;
+  locate(P.lgeom, __ldg(P.s + i * P.nnei + row), t, clamped);
+  const real *__restrict__ blk = tab + st.qoff[e];
+  const int M1 = P.M1;
+  real a[6];  // ds, dR~[0..3], and room for the padding zero
+#pragma unroll
+  for (int x = 0; x < 5; ++x) a[x] = real(0);
+#pragma unroll 2
+  for (int m = c; m < M1; m += C) {
+    real cf[6];
+    ld6(blk, M1, m, cf);
+    const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
+    real g = fma(cf[0], t, cf[1]);  // g and g' by Horner's rule with derivative
+    real dg = cf[0];
+    dg = fma(dg, t, g);
+    g = fma(g, t, cf[2]);
+    dg = fma(dg, t, g);
+    g = fma(g, t, cf[3]);
+    dg = fma(dg, t, g);
+    g = fma(g, t, cf[4]);
+    dg = fma(dg, t, g);
+    g = fma(g, t, cf[5]);
+    real rm = d0 * rr.x;
+    rm = fma(d1, rr.y, rm);
+    rm = fma(d2, rr.z, rm);
+    rm = fma(d3, rr.w, rm);
+    a[0] = fma(rm, dg, a[0]);
+    a[1] = fma(d0, g, a[1]);
+    a[2] = fma(d1, g, a[2]);
+    a[3] = fma(d2, g, a[3]);
+    a[4] = fma(d3, g, a[4]);
+  }
+  int base, nreal;
+  reduce_scatter<5, C>(a, lane, base, nreal);
+  if (valid) {
+    real *__restrict__ ds_i = P.ds + i * P.nnei;
+    real *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
+#pragma unroll
+    for (int x = 0; x < rs_count(5, ilog2(C)); ++x)
+      if (x < nreal) {
+        const int comp = base + x;
+        if (comp == 0)
+          ds_i[row] = (rw & kClamped) ? real(0) : a[x] * P.inv_nnei;
+        else
+          dR_i[(size_t)row * 4 + comp - 1] = a[x] * P.inv_nnei;
+      }
+  }
+}
+
+// Group size for `rem` runs or rows left: G = 8 for 7 or more, then 4, 2, 1.
+__device__ __forceinline__ int h_group_size(int rem) { return rem >= 7 ? 8 : rem >= 4 ? 4 : rem >= 2 ? 2 : 1; }
+
+template <typename real>
+__device__ __forceinline__ void form_H_runs(MomentGradStage<real> &st, const real *__restrict__ tab, const real *dts,
+                                            int M1, int nrun, int lane) {
+  for (int s0 = 0; s0 < nrun;) {  // uniform
+    const int G = h_group_size(nrun - s0);
+    if (G == 8)
+      form_H_group<8>(st, tab, dts, M1, s0, nrun, lane);
+    else if (G == 4)
+      form_H_group<4>(st, tab, dts, M1, s0, nrun, lane);
+    else if (G == 2)
+      form_H_group<2>(st, tab, dts, M1, s0, nrun, lane);
+    else
+      form_H_group<1>(st, tab, dts, M1, s0, nrun, lane);
+    s0 += G;
+  }
+}
+
+// Queued rows q0 .. n-1 in groups: G = 8 while `all` is false (the rest stays queued), else down to 1.
+template <typename real>
+__device__ __forceinline__ int grad_rows_queued(const GradParams<real> &P, const MomentGradStage<real> &st,
+                                                const real *__restrict__ tab, const real *dts, int64_t i, int n,
+                                                bool all, int lane) {
+  int q0 = 0;
+  while (n - q0 >= 8 || (all && q0 < n)) {  // uniform
+    const int G = h_group_size(n - q0);
+    if (G == 8)
+      grad_rows_group<8>(P, st, tab, dts, i, q0, n, lane);
+    else if (G == 4)
+      grad_rows_group<4>(P, st, tab, dts, i, q0, n, lane);
+    else if (G == 2)
+      grad_rows_group<2>(P, st, tab, dts, i, q0, n, lane);
+    else
+      grad_rows_group<1>(P, st, tab, dts, i, q0, n, lane);
+    q0 += G;
+  }
+  return q0;
+}
+
+template <typename real>
 __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const GradParams<real> P) {
   constexpr int kClamped = 1 << 30;
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -249,7 +417,7 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
   const int64_t i = blockIdx.x;  // one atom per block (one warp)
   MomentGradStage<real> &st = *reinterpret_cast<MomentGradStage<real> *>(smem_raw);
   real *dts = reinterpret_cast<real *>(smem_raw + sizeof(MomentGradStage<real>));  // [M1][4]
-  const int M1 = P.M1, RR = M1 - 32 * Q;
+  const int M1 = P.M1;
 
   {  // counts in shared memory
     int sl = 0;
@@ -276,80 +444,24 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
   real *__restrict__ ds_i = P.ds + i * P.nnei;
   real *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
 
-  // queued rows: lane j evaluates queue entry j (when j < n)
-  auto drain = [&](int n) {
-    if (lane < n) {
-      real a_ds, a0, a1, a2, a3;
-      grad_row_direct(tab + st.qoff[lane], dts, M1, st.qt[lane], st.qr[lane][0], st.qr[lane][1], st.qr[lane][2],
-                      st.qr[lane][3], a_ds, a0, a1, a2, a3);
-      const int rw = st.qrow[lane];
-      const int row = rw & (kClamped - 1);
-      ds_i[row] = (rw & kClamped) ? real(0) : a_ds * P.inv_nnei;
-      st4(dR_i + (size_t)row * 4, a0 * P.inv_nnei, a1 * P.inv_nnei, a2 * P.inv_nnei, a3 * P.inv_nnei);
-    }
-  };
-  // H[slot] of the run in interval block `off` (uniform call; all lanes)
-  auto form_H = [&](int off, int slot) {
-    real h[24];
-#pragma unroll
-    for (int x = 0; x < 24; ++x) h[x] = real(0);
-    const real *__restrict__ blk = tab + off;
-#pragma unroll
-    for (int r = 0; r <= Q; ++r) {
-      const int m = 32 * r + lane;
-      if (r < Q || lane < RR) {  // last round: the RR remainder channels
-        real c6[6];  // (a..f): coefficients of t^5 .. t^0
-        ld6(blk, M1, m, c6);
-        const real d0 = dts[m * 4 + 0], d1 = dts[m * 4 + 1], d2 = dts[m * 4 + 2], d3 = dts[m * 4 + 3];
-#pragma unroll
-        for (int q = 0; q < 6; ++q) {
-          h[0 * 6 + q] = fma(d0, c6[5 - q], h[0 * 6 + q]);
-          h[1 * 6 + q] = fma(d1, c6[5 - q], h[1 * 6 + q]);
-          h[2 * 6 + q] = fma(d2, c6[5 - q], h[2 * 6 + q]);
-          h[3 * 6 + q] = fma(d3, c6[5 - q], h[3 * 6 + q]);
-        }
-      }
-    }
-    // reduce-scatter of the 24 sums over the 32 lanes: 24 -> 12 -> 6 -> 3 (+1 pad) -> 2 -> 1
-    const bool bA = lane & 16, bB = lane & 8, bC = lane & 4, bD = lane & 2, bE = lane & 1;
-#pragma unroll
-    for (int x = 0; x < 12; ++x) {
-      const real snd = bA ? h[x] : h[x + 12], kp = bA ? h[x + 12] : h[x];
-      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 16);
-    }
-#pragma unroll
-    for (int x = 0; x < 6; ++x) {
-      const real snd = bB ? h[x] : h[x + 6], kp = bB ? h[x + 6] : h[x];
-      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 8);
-    }
-#pragma unroll
-    for (int x = 0; x < 3; ++x) {
-      const real snd = bC ? h[x] : h[x + 3], kp = bC ? h[x + 3] : h[x];
-      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 4);
-    }
-    h[3] = real(0);
-#pragma unroll
-    for (int x = 0; x < 2; ++x) {
-      const real snd = bD ? h[x] : h[x + 2], kp = bD ? h[x + 2] : h[x];
-      h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, 2);
-    }
-    {
-      const real snd = bE ? h[0] : h[1], kp = bE ? h[1] : h[0];
-      h[0] = kp + __shfl_xor_sync(0xffffffffu, snd, 1);
-    }
-    const int idx = (bA ? 12 : 0) + (bB ? 6 : 0) + (bC ? 3 : 0) + (bD ? 2 : 0) + (bE ? 1 : 0);
-    if (!(bD && bE)) st.H[slot][idx] = h[0];
-  };
-  // outputs of one row (this lane) from its run's H
+  // outputs of one row (this lane) from its run's H, by Horner's rule with derivative
   auto eval_row = [&](const real *Hr, real t, real r0, real r1, real r2, real r3, int rw) {
-    const real t2 = t * t, t3 = t2 * t, t4 = t3 * t, t5 = t4 * t;
     real dR[4], G[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const real *hk = Hr + 6 * k;  // H[k][q], q = 0..5
-      dR[k] = fma(hk[5], t5, fma(hk[4], t4, fma(hk[3], t3, fma(hk[2], t2, fma(hk[1], t, hk[0])))));
-      G[k] = fma(real(5) * hk[5], t4,
-                 fma(real(4) * hk[4], t3, fma(real(3) * hk[3], t2, fma(real(2) * hk[2], t, hk[1]))));
+      real p = fma(hk[5], t, hk[4]);
+      real dp = hk[5];
+      dp = fma(dp, t, p);
+      p = fma(p, t, hk[3]);
+      dp = fma(dp, t, p);
+      p = fma(p, t, hk[2]);
+      dp = fma(dp, t, p);
+      p = fma(p, t, hk[1]);
+      dp = fma(dp, t, p);
+      p = fma(p, t, hk[0]);
+      dR[k] = p;
+      G[k] = dp;
     }
     real dsv = r0 * G[0];
     dsv = fma(r1, G[1], dsv);
@@ -359,14 +471,15 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     ds_i[row] = (rw & kClamped) ? real(0) : dsv * P.inv_nnei;
     st4(dR_i + (size_t)row * 4, dR[0] * P.inv_nnei, dR[1] * P.inv_nnei, dR[2] * P.inv_nnei, dR[3] * P.inv_nnei);
   };
-  constexpr int kSlots = 32 / min_grad_run<real>();
-  int nq = 0;           // queued rows (uniform)
-  int carry_off = -1;   // interval block of the last batch's last run, if its H is kept
-  int carry_slot = kSlots;
+  constexpr int kCarrySlot = chunk_runs<real>();
 
+  int nrows = 0, nrun = 0;  // staged rows and runs of the chunk (uniform)
+  int nq = 0;               // queued rows (uniform)
+  int last_off = -1, last_slot = -1;
+  bool last_open = false;   // the last run may go on in the next batch
   for (int base = 0; base < nv; base += 32) {
     const int cnt = min(32, nv - base);
-    if (lane < cnt) {  // stage row base + lane
+    if (lane < cnt) {  // stage row base + lane at chunk position nrows + lane
       const int v = base + lane;
       int b = 0, cum = 0, lim = st.nvb[0], off = 0;
 #pragma unroll
@@ -382,99 +495,77 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
       real t;
       bool clamped;
       const int l = locate(P.lgeom, __ldg(P.s + i * P.nnei + row), t, clamped);
-      st.r[lane][0] = rr.x;
-      st.r[lane][1] = rr.y;
-      st.r[lane][2] = rr.z;
-      st.r[lane][3] = rr.w;
-      st.t[lane] = t;
-      st.off[lane] = (b * P.geom.nint + l) * M1 * 6;
-      st.row[lane] = row | (clamped ? kClamped : 0);
+      const int j = nrows + lane;
+      st.r[j][0] = rr.x;
+      st.r[j][1] = rr.y;
+      st.r[j][2] = rr.z;
+      st.r[j][3] = rr.w;
+      st.t[j] = t;
+      st.off[j] = (b * P.geom.nint + l) * M1 * 6;
+      st.row[j] = row | (clamped ? kClamped : 0);
     }
     __syncwarp();
-    int nrun = 0, next_off = -1, next_slot = carry_slot;
-    for (int u = 0; u < cnt;) {  // runs of the batch (uniform control flow)
-      const int off = st.off[u];
-      int e = u + 1;
-      while (e < cnt && st.off[e] == off) ++e;
-      if (u == 0 && off == carry_off) {  // the previous batch's last run goes on: its H is kept
-        if (lane < e) st.run[lane] = carry_slot;
-        if (e == cnt) next_off = off;
-      } else if (e - u < min_grad_run<real>()) {  // short run: queue its rows
-        const int j = u + lane;
-        if (j < e) {
-          st.run[j] = -1;
-          st.qr[nq + lane][0] = st.r[j][0];
-          st.qr[nq + lane][1] = st.r[j][1];
-          st.qr[nq + lane][2] = st.r[j][2];
-          st.qr[nq + lane][3] = st.r[j][3];
-          st.qt[nq + lane] = st.t[j];
-          st.qoff[nq + lane] = off;
-          st.qrow[nq + lane] = st.row[j];
-        }
-        nq += e - u;
+    const bool more = base + cnt < nv;
+    // run starts of the batch: rows whose interval block differs from the previous row's
+    const int myoff = lane < cnt ? st.off[nrows + lane] : -1;
+    const int prevoff = __shfl_up_sync(0xffffffffu, myoff, 1);
+    unsigned starts = __ballot_sync(0xffffffffu, lane < cnt && (lane == 0 || myoff != prevoff));
+    while (starts) {  // uniform, run by run
+      const int u = __ffs(starts) - 1;
+      starts &= starts - 1;
+      const int e = starts ? __ffs(starts) - 1 : cnt;
+      const int off = __shfl_sync(0xffffffffu, myoff, u);
+      int slot;
+      if (u == 0 && last_open && off == last_off) {
+        slot = last_slot;  // the previous batch's last run goes on
+      } else if (e - u >= min_grad_run<real>() || (e == cnt && more)) {
+        slot = nrun++;
+        if (lane == 0) st.run_off[slot] = off;
       } else {
-        int slot = nrun;
-        if (e == cnt) {  // the batch's last run may go on in the next batch: keep its H
-          slot = next_slot = carry_slot == kSlots ? kSlots + 1 : kSlots;
-          next_off = off;
-        } else {
-          ++nrun;
+        slot = -1;  // a single-row run: queue it
+        if (lane == 0) {
+          st.qoff[nq] = off;
+          st.qrow[nq] = st.row[nrows + u];
         }
-        if (lane >= u && lane < e) st.run[lane] = slot;
-        form_H(off, slot);
+        ++nq;
       }
-      u = e;
+      if (lane >= u && lane < e) st.slot[nrows + lane] = slot;
+      if (e == cnt) {
+        last_off = off;
+        last_slot = slot;
+        last_open = more && slot >= 0;
+      }
     }
-    carry_off = next_off;
-    carry_slot = next_slot;
+    nrows += cnt;
     __syncwarp();
-    if (lane < cnt && st.run[lane] >= 0)
-      eval_row(st.H[st.run[lane]], st.t[lane], st.r[lane][0], st.r[lane][1], st.r[lane][2], st.r[lane][3],
-               st.row[lane]);
-    if (nq >= 32) {  // a full queue: one row per lane, then keep the overflow
-      drain(32);
+    if (nrows + 32 > kChunkRows || nrun + batch_runs<real>() > chunk_runs<real>() || !more) {  // chunk full, or the atom's last rows
+      form_H_runs(st, tab, dts, M1, nrun, lane);
       __syncwarp();
-      if (lane < nq - 32) {
-        st.qr[lane][0] = st.qr[32 + lane][0];
-        st.qr[lane][1] = st.qr[32 + lane][1];
-        st.qr[lane][2] = st.qr[32 + lane][2];
-        st.qr[lane][3] = st.qr[32 + lane][3];
-        st.qt[lane] = st.qt[32 + lane];
-        st.qoff[lane] = st.qoff[32 + lane];
-        st.qrow[lane] = st.qrow[32 + lane];
+      for (int j = lane; j < nrows; j += 32) {
+        const int sl = st.slot[j];
+        if (sl >= 0) eval_row(st.H[sl], st.t[j], st.r[j][0], st.r[j][1], st.r[j][2], st.r[j][3], st.row[j]);
       }
-      nq -= 32;
+      __syncwarp();
+      if (last_open && last_slot != kCarrySlot) {  // keep the open run's H for the next chunk
+        if (lane < 24) st.H[kCarrySlot][lane] = st.H[last_slot][lane];
+        last_slot = kCarrySlot;
+      }
+      nrows = 0;
+      nrun = 0;
+      __syncwarp();
     }
-    __syncwarp();
-  }
-  if (nq > 0) {
-    // The rest of the queue costs 18 M1 warp FMA per row-per-lane pass however
-    // few lanes it fills, or ~24 (ceil(M1/32) + 1) per run through H: take the cheaper.
-    int nr = 1;
-    for (int u = 1; u < nq; ++u) nr += st.qoff[u] != st.qoff[u - 1];
-    if (nr * 24 * ((M1 + 31) / 32 + 1) < 18 * M1) {
-      for (int u = 0; u < nq;) {  // groups of at most kSlots runs
-        const int g0 = u;
-        int nrun = 0;
-        while (u < nq && nrun < kSlots) {
-          const int off = st.qoff[u];
-          int e = u + 1;
-          while (e < nq && st.qoff[e] == off) ++e;
-          if (lane >= u && lane < e) st.run[lane] = nrun;
-          form_H(off, nrun);
-          ++nrun;
-          u = e;
-        }
-        __syncwarp();
-        if (lane >= g0 && lane < u)
-          eval_row(st.H[st.run[lane]], st.qt[lane], st.qr[lane][0], st.qr[lane][1], st.qr[lane][2], st.qr[lane][3],
-                   st.qrow[lane]);
-        __syncwarp();
+    if (nq >= 8) {  // single-row runs, 8 at a time; fewer than 8 stay queued
+      const int done = grad_rows_queued(P, st, tab, dts, i, nq, false, lane);
+      __syncwarp();
+      if (lane < nq - done) {
+        st.qoff[lane] = st.qoff[done + lane];
+        st.qrow[lane] = st.qrow[done + lane];
       }
-    } else {
-      drain(nq);
+      nq -= done;
+      __syncwarp();
     }
   }
+  grad_rows_queued(P, st, tab, dts, i, nq, true, lane);
 
   // padding rows, packed over the segments' padded tails
   for (int pv = lane; pv < P.nnei - nv; pv += 32) {
@@ -491,16 +582,6 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     ds_i[row] = real(0);
     st4(dR_i + (size_t)row * 4, real(0), real(0), real(0), real(0));
   }
-}
-
-template <typename real>
-using GradKernel = void (*)(const GradParams<real>);
-
-template <typename real, int... Qs>
-GradKernel<real> pick_grad_moments(int Q, std::integer_sequence<int, Qs...>) {
-  GradKernel<real> k = nullptr;
-  ((Q == Qs ? (k = &grad_moments_kernel<real, Qs>, 0) : 0), ...);
-  return k;
 }
 
 // ---------------------------------------------------------------- f32
@@ -747,9 +828,7 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
   for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
   P.inv_nnei = (real)(1.0 / (double)nnei);
   if (moments) {
-    GradKernel<real> k =
-        pick_grad_moments<real>(M1 / 32, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
-    if (!k) return set_error(DP_ERR_UNSUPPORTED, "no moment gradient kernel for M1 = %d", M1);
+    void (*k)(const GradParams<real>) = &grad_moments_kernel<real>;
     const size_t smem = sizeof(MomentGradStage<real>) + (size_t)4 * M1 * sizeof(real);
     if (smem > 48 * 1024) {
       const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
