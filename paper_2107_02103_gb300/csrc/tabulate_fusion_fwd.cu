@@ -64,11 +64,16 @@ struct alignas(16) Stage {
 };
 
 // Extra staging of the interval-moment variant: powers t^0..t^5 of every
-// staged neighbour and the 24 moments W[k][q] of the run being contracted.
+// staged neighbour, the 24 moments W[k][q] of the last runs contracted (kept
+// until the remainder channels of up to kPendRuns runs are done in one packed
+// round), their interval blocks, and the rows of the batch's short runs.
+constexpr int kPendRuns = 8;
 template <typename real>
 struct alignas(16) MomentStage {
   real tp[32][6];
-  real w[24];
+  real w[kPendRuns][24];
+  int32_t poff[kPendRuns];
+  int32_t srow[32];
 };
 
 // Runs at least this long go through interval moments; shorter ones are
@@ -244,14 +249,40 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
   int rcur = -1;
   real cf[Q > 0 ? Q : 1][6];  // f32: coefficients of the interval in use
   // T += C_l W for the run in interval block `off`, W[6k + q] held by lanes 0..23 (uniform call)
+  // remainder channels 32 Q + rch of the pending runs: lane (rslot, rch) takes run rslot (uniform call)
+  int npend = 0;
+  auto flush_remainder = [&]() {
+    __syncwarp();
+    if (ractive && rslot < npend) {
+      real c6[6];
+      ld6(tab + ms.poff[rslot], P.M1, Q * 32 + rch, c6);
+      const real *w = ms.w[rslot];
+      real v0 = racc0, v1 = racc1, v2 = racc2, v3 = racc3;
+#pragma unroll
+      for (int q = 0; q < 6; ++q) {
+        v0 = fma(c6[5 - q], w[q], v0);
+        v1 = fma(c6[5 - q], w[6 + q], v1);
+        v2 = fma(c6[5 - q], w[12 + q], v2);
+        v3 = fma(c6[5 - q], w[18 + q], v3);
+      }
+      racc0 = v0;
+      racc1 = v1;
+      racc2 = v2;
+      racc3 = v3;
+    }
+    __syncwarp();
+    npend = 0;
+  };
+  const int pend_cap = P.PK < kPendRuns ? P.PK : kPendRuns;
   auto apply_moments = [&](int off, real wv) {
-    if (lane < 24) ms.w[lane] = wv;
+    if (lane < 24) ms.w[npend][lane] = wv;
+    if (lane == 0) ms.poff[npend] = off;
     __syncwarp();
     real W[4][6];
 #pragma unroll
     for (int k = 0; k < 4; ++k)
 #pragma unroll
-      for (int q = 0; q < 6; ++q) W[k][q] = ms.w[6 * k + q];
+      for (int q = 0; q < 6; ++q) W[k][q] = ms.w[npend][6 * k + q];
 #pragma unroll
     for (int r = 0; r < (Q > 0 ? Q : 1); ++r) {
       real c6[6];  // (a, b, c, d, e, f) = coefficients of t^5 .. t^0
@@ -265,6 +296,7 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
       }
     }
     __syncwarp();
+    if (P.RR > 0 && ++npend == pend_cap) flush_remainder();
   };
   int carry_off = -1;  // run left open at the end of the previous batch (uniform)
   real wcarry = real(0);  // its partial W on lanes 0..23
@@ -304,17 +336,23 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     }
     __syncwarp();
     const int cnt = min(32, nv - base);
+    int nshort = cnt;  // rows whose remainder channels go through the packed per-neighbour round
     if (Q > 0 && kMoments) {
+      nshort = 0;
       if (carry_off >= 0 && st.off[0] != carry_off) {  // the open run ended with the last batch
         apply_moments(carry_off, wcarry);
         carry_off = -1;
       }
       int next_carry = -1;
-      int u = 0;
-      while (u < cnt) {  // uniform, run by run
-        const int off = st.off[u];
-        int e = u + 1;
-        while (e < cnt && st.off[e] == off) ++e;
+      // run starts of the batch: rows whose interval block differs from the previous row's
+      const int myoff = lane < cnt ? st.off[lane] : -1;
+      const int prevoff = __shfl_up_sync(0xffffffffu, myoff, 1);
+      unsigned starts = __ballot_sync(0xffffffffu, lane < cnt && (lane == 0 || myoff != prevoff));
+      while (starts) {  // uniform, run by run
+        const int u = __ffs(starts) - 1;
+        starts &= starts - 1;
+        const int e = starts ? __ffs(starts) - 1 : cnt;
+        const int off = __shfl_sync(0xffffffffu, myoff, u);
         const bool cont = u == 0 && off == carry_off;
         if (cont || e - u >= kMinMomentRun) {
           real wv = cont ? wcarry : real(0);
@@ -330,8 +368,9 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
           }
         } else {
           for (int j = u; j < e; ++j) fwd_neighbour<real, Q>(P, tab, lane, off, st.t[j], st.r[j], acc);
+          if (lane >= u && lane < e) ms.srow[nshort + lane - u] = lane;  // their remainder channels: packed round
+          nshort += e - u;
         }
-        u = e;
       }
       carry_off = next_carry;
     } else if (Q > 0) {
@@ -355,9 +394,11 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
       }
     }
     if (P.RR > 0) {
-      for (int u0 = 0; u0 < cnt; u0 += P.PK) {  // packed round: PK neighbours x RR channels
-        const int u = u0 + rslot;
-        if (ractive && u < cnt) {
+      __syncwarp();
+      for (int u0 = 0; u0 < nshort; u0 += P.PK) {  // packed round: PK neighbours x RR channels
+        const int x = u0 + rslot;
+        if (ractive && x < nshort) {
+          const int u = (Q > 0 && kMoments) ? ms.srow[x] : x;
           const real t = st.t[u];
           const int off = st.off[u];
           if (!kCache || off != rcur) {
@@ -374,6 +415,8 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     }
     __syncwarp();
   }
+
+  if (Q > 0 && kMoments && npend > 0) flush_remainder();
 
   real *__restrict__ Ti = P.T + i * 4 * P.M1;
 #pragma unroll
