@@ -84,9 +84,9 @@ def moment_fmas(runs, M1: int) -> dict:
 
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
-# `ncu --set full` capture of its current version (profiles/<kernel>_<workload>_<dtype>.md);
+# `ncu --set full` capture of its current version (profiles/<kernel>_<algo>_<workload>_<dtype>.md);
 # absent means no capture of the current kernel exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad"): 83780352 + 34432256}
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83860224 + 32249344}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
@@ -351,7 +351,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     achieved = flops[dom] / (mean[dom] * 1e-3) / 1e12
     path_tflops = (flops["fwd"] + flops["grad"]) / ((mean["fwd"] + mean["grad"]) * 1e-3) / 1e12
     roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
-                "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom)),
+                "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
                 "kernel": f"dp_tabulate_fusion_{dom}",
                 "peak_basis": (f"FP{64 if args.dtype == 'f64' else 32} FMA pipe: {NSM} SMs x "
                                f"{FMA_LANES[args.dtype]} lanes/clk x 2 flop x {SM_MAX_MHZ:.0f} MHz"),
@@ -470,7 +470,7 @@ def run_reference(args, rank, world):
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--steps", type=int, default=500)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="cu85", choices=["tiny", "cu85", "cugeo", "water", "alcumg", "water_large"])
