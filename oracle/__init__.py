@@ -94,6 +94,12 @@ def load(path: str | None = None):
     lib.or_embed_rows.argtypes = [P, ctypes.POINTER(Info), P, P, ctypes.c_int, ctypes.c_int, P, ctypes.c_int, P,
                                   i64, P, P]
     lib.or_embed_rows.restype = None
+    lib.or_switch.argtypes = [dbl, dbl, dbl, ctypes.c_int, P]
+    lib.or_switch.restype = dbl
+    lib.or_env_mat.argtypes = [i64, P, P, ctypes.c_int, dbl, dbl, ctypes.c_int, P, P, P]
+    lib.or_env_mat.restype = None
+    lib.or_force_virial.argtypes = [i64, i64, P, P, ctypes.c_int, dbl, dbl, ctypes.c_int, P, P, P, P, P]
+    lib.or_force_virial.restype = None
     if path is None:
         _lib = lib
     return lib
@@ -256,6 +262,36 @@ class Oracle:
         self.lib.or_embed_rows(_p(table), ctypes.byref(info), _p(s), _p(atype_a), nnei, sel.size, _p(sel), M, _p(at),
                                n, _p(G), _p(dG))
         return (G, dG) if deriv else G
+
+
+    def switch(self, r, rcs, rc, kind=0):
+        """(s(r), s'(r)) of the weighting function (kind 0 cosine, 1 the paper's quintic)."""
+        d = ctypes.c_double()
+        v = self.lib.or_switch(float(r), float(rcs), float(rc), int(kind), ctypes.byref(d))
+        return v, d.value
+
+    def env_mat(self, coord, nlist, rcs, rc, kind=0, norm=None):
+        """(s [nloc][nnei], R~ [nloc][nnei][4]) from coordinates [nall][3] and nlist [nloc][nnei] (-1 = padding)."""
+        coord, nlist = _c(coord, np.float64), _c(nlist, np.int32)
+        nloc, nnei = nlist.shape
+        nrm = None if norm is None else _c(np.asarray(norm, dtype=np.float64), np.float64)
+        s = np.empty((nloc, nnei))
+        Rt = np.empty((nloc, nnei, 4))
+        self.lib.or_env_mat(nloc, _p(coord), _p(nlist), nnei, float(rcs), float(rc), int(kind), _p(nrm), _p(s), _p(Rt))
+        return s, Rt
+
+    def force_virial(self, coord, nlist, rcs, rc, ds, dRt, kind=0, norm=None):
+        """(F [nall][3], W [3][3]) from dE/ds [nloc][nnei] and dE/dR~ [nloc][nnei][4]."""
+        coord, nlist = _c(coord, np.float64), _c(nlist, np.int32)
+        ds, dRt = _c(ds, np.float64), _c(dRt, np.float64)
+        nloc, nnei = nlist.shape
+        nall = coord.shape[0]
+        nrm = None if norm is None else _c(np.asarray(norm, dtype=np.float64), np.float64)
+        F = np.empty((nall, 3))
+        W = np.empty((3, 3))
+        self.lib.or_force_virial(nloc, nall, _p(coord), _p(nlist), nnei, float(rcs), float(rc), int(kind), _p(nrm),
+                                 _p(ds), _p(dRt), _p(F), _p(W))
+        return F, W
 
 
 _default = None

@@ -23,7 +23,11 @@
  *   - the descriptor D_i = S_i (S_i^<)^T with S_i = T_i^T (Sec. II), and its
  *     gradient dE/dT from an upstream dE/dD, in double;
  *   - the embedding matrix G itself, through the table or straight from the
- *     net, for the explicit and uncompressed comparisons.
+ *     net, for the explicit and uncompressed comparisons;
+ *   - the environment matrix from coordinates and a neighbour list (Sec. II,
+ *     the weighting function s(r) and the 4-vector rows with their
+ *     normalisation), and the forces and virial that follow from dE/ds and
+ *     dE/dR~ by the chain rule through those rows.
  *
  * Pins: every function here is pinned by tests that do not re-run its own
  * formula (closed forms, exactly reproduced polynomials, a sin() error
@@ -492,4 +496,128 @@ void or_embed_rows(const double *table, const or_info *in, const double *s, cons
         }
       }
   }
+}
+
+/* ------------------------------------------------- environment matrix */
+
+/*
+ * Weighting function s(r) and its derivative (Sec. II).  With
+ * u = (r - rcs)/(rc - rcs):
+ *   r < rcs:         s = 1/r
+ *   rcs <= r < rc:   s = w(u)/r
+ *   r >= rc:         s = 0
+ * kind 1 is the paper's switch w = u^3 (-6u^2 + 15u - 10) + 1; kind 0 is the
+ * cosine switch of the benchmark configurations, w = cos(pi u)/2 + 1/2.
+ */
+static void or_weight(double r, double rcs, double rc, int kind, double *sv, double *dsv) {
+  if (r < rcs) {
+    *sv = 1.0 / r;
+    *dsv = -1.0 / (r * r);
+    return;
+  }
+  if (r >= rc) {
+    *sv = 0.0;
+    *dsv = 0.0;
+    return;
+  }
+  double u = (r - rcs) / (rc - rcs);
+  double w, dw;  /* w(u) and dw/du */
+  if (kind == 1) {
+    w = u * u * u * (-6.0 * u * u + 15.0 * u - 10.0) + 1.0;
+    dw = -30.0 * u * u * (u - 1.0) * (u - 1.0);
+  } else {
+    const double pi = 3.14159265358979323846;
+    w = 0.5 * cos(pi * u) + 0.5;
+    dw = -0.5 * pi * sin(pi * u);
+  }
+  *sv = w / r;
+  *dsv = dw / ((rc - rcs) * r) - w / (r * r);
+}
+
+double or_switch(double r, double rcs, double rc, int kind, double *ds_dr) {
+  double sv, dsv;
+  or_weight(r, rcs, rc, kind, &sv, &dsv);
+  if (ds_dr) *ds_dr = dsv;
+  return sv;
+}
+
+/*
+ * Rows of the environment matrix (Sec. II).  For atom i < nloc and row q of
+ * nlist (index j into coord, -1 on padding rows): d = r_j - r_i, r = |d|,
+ *   R~ = ( (s(r) - mean)/std,  s(r) d_x / r / std_all,  s(r) d_y / r / std_all,  s(r) d_z / r / std_all )
+ * with norm = {mean, std, std_all} (NULL: {0, 1, 1}); the embedding input
+ * s of the row is its first entry.  Padding rows are zero.
+ */
+void or_env_mat(int64_t nloc, const double *coord, const int32_t *nlist, int nnei, double rcs, double rc, int kind,
+                const double *norm, double *s, double *Rt) {
+  const double mean = norm ? norm[0] : 0.0, sd = norm ? norm[1] : 1.0, sa = norm ? norm[2] : 1.0;
+  for (int64_t i = 0; i < nloc; ++i)
+    for (int q = 0; q < nnei; ++q) {
+      const int64_t row = i * nnei + q;
+      const int32_t j = nlist[row];
+      if (j < 0) {
+        s[row] = 0.0;
+        for (int k = 0; k < 4; ++k) Rt[4 * row + k] = 0.0;
+        continue;
+      }
+      double d[3], r2 = 0.0;
+      for (int a = 0; a < 3; ++a) {
+        d[a] = coord[3 * (int64_t)j + a] - coord[3 * i + a];
+        r2 += d[a] * d[a];
+      }
+      const double r = sqrt(r2);
+      const double sv = or_switch(r, rcs, rc, kind, NULL);
+      const double sh = (sv - mean) / sd;
+      s[row] = sh;
+      Rt[4 * row + 0] = sh;
+      for (int a = 0; a < 3; ++a) Rt[4 * row + 1 + a] = sv * d[a] / r / sa;
+    }
+}
+
+/*
+ * Forces and virial from the gradients of the rows (the derivatives of E_i
+ * with respect to atom i and its neighbours, Sec. II).  For a valid row
+ * (i, j) with d = r_j - r_i, the energy depends on d through s (the
+ * embedding input) and R~; with ds = dE/ds and dR = dE/dR~ of the row,
+ *   dE/dd_b = (ds + dR_0) s'(r) d_b / (r std)
+ *           + sum_a dR_{1+a} / std_all * ( s'(r) d_a d_b / r^2 + s(r) (delta_ab / r - d_a d_b / r^3) ).
+ * Then F_i += dE/dd, F_j -= dE/dd (F = -dE/dr; d = r_j - r_i), and the
+ * virial W_ab = - sum over rows of d_a dE/dd_b.  F has nall rows (every
+ * index nlist can hold); both outputs are overwritten.
+ */
+void or_force_virial(int64_t nloc, int64_t nall, const double *coord, const int32_t *nlist, int nnei, double rcs,
+                     double rc, int kind, const double *norm, const double *ds, const double *dRt, double *F,
+                     double *W) {
+  const double sd = norm ? norm[1] : 1.0, sa = norm ? norm[2] : 1.0;
+  for (int64_t a = 0; a < 3 * nall; ++a) F[a] = 0.0;
+  for (int a = 0; a < 9; ++a) W[a] = 0.0;
+  for (int64_t i = 0; i < nloc; ++i)
+    for (int q = 0; q < nnei; ++q) {
+      const int64_t row = i * nnei + q;
+      const int32_t j = nlist[row];
+      if (j < 0) continue;
+      double d[3], r2 = 0.0;
+      for (int a = 0; a < 3; ++a) {
+        d[a] = coord[3 * (int64_t)j + a] - coord[3 * i + a];
+        r2 += d[a] * d[a];
+      }
+      const double r = sqrt(r2);
+      double sv, dsv;
+      or_weight(r, rcs, rc, kind, &sv, &dsv);
+      double g[3];
+      for (int b = 0; b < 3; ++b) {
+        double v = (ds[row] + dRt[4 * row + 0]) * dsv * d[b] / (r * sd);
+        for (int a = 0; a < 3; ++a) {
+          const double dab = (a == b) ? 1.0 : 0.0;
+          v += dRt[4 * row + 1 + a] / sa * (dsv * d[a] * d[b] / r2 + sv * (dab / r - d[a] * d[b] / (r2 * r)));
+        }
+        g[b] = v;
+      }
+      for (int b = 0; b < 3; ++b) {
+        F[3 * i + b] += g[b];
+        F[3 * (int64_t)j + b] -= g[b];
+      }
+      for (int a = 0; a < 3; ++a)
+        for (int b = 0; b < 3; ++b) W[3 * a + b] -= d[a] * g[b];
+    }
 }

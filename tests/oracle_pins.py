@@ -453,7 +453,146 @@ def pin_descriptor_grad(o):
         assert _rel(dT[a], dS.T) < 1e-14
 
 
+# ------------------------------------------------- environment matrix, forces
+
+def pin_switch(o):
+    """s(r) at hand-computable points, s'(r) against central differences, and smoothness at rcs and rc.
+
+    u = 1/2 gives w = 1/2 for both switches; u = 1/4 gives 0.896484375 (quintic, exact in binary)
+    and (1 + cos(pi/4))/2 (cosine, library cos).  Both switches and their first derivatives are
+    continuous at r = rcs and r = rc (the paper's stated purpose of the switch)."""
+    rcs, rc = 2.0, 6.0
+    for kind in (0, 1):
+        v, d = o.switch(1.5, rcs, rc, kind)
+        assert abs(v - 1.0 / 1.5) < 1e-15 and abs(d + 1.0 / 2.25) < 1e-15
+        v, _ = o.switch(4.0, rcs, rc, kind)  # u = 1/2
+        assert abs(v - 0.5 / 4.0) < 1e-15, (kind, v)
+        assert o.switch(6.0, rcs, rc, kind) == (0.0, 0.0) and o.switch(7.0, rcs, rc, kind)[0] == 0.0
+        for r in (2.3, 3.1, 4.7, 5.9):
+            h = 1e-6
+            fd = (o.switch(r + h, rcs, rc, kind)[0] - o.switch(r - h, rcs, rc, kind)[0]) / (2 * h)
+            assert abs(fd - o.switch(r, rcs, rc, kind)[1]) < 1e-8, (kind, r)
+        for r0 in (rcs, rc):  # value and slope continuous
+            e = 1e-9
+            lo, hi = o.switch(r0 - e, rcs, rc, kind), o.switch(r0 + e, rcs, rc, kind)
+            assert abs(lo[0] - hi[0]) < 1e-8 and abs(lo[1] - hi[1]) < 1e-6, (kind, r0, lo, hi)
+    assert abs(o.switch(3.0, rcs, rc, 1)[0] - 0.896484375 / 3.0) < 1e-15
+    assert abs(o.switch(3.0, rcs, rc, 0)[0] - (0.5 + 0.5 * math.cos(math.pi / 4)) / 3.0) < 1e-15
+
+
+def pin_env_mat_hand(o):
+    """One neighbour at d = (1, 2, 2), r = 3, inside rcs: R~ = (1/3, 1/9, 2/9, 2/9); with the paper's
+    normalisation (mean 0.1, std 2, std_all 3) every entry maps as stated; padding rows are zero."""
+    coord = np.array([[0.5, -1.0, 2.0], [1.5, 1.0, 4.0], [9.0, 9.0, 9.0]])
+    nlist = np.array([[1, -1, -1], [0, 2, -1]], dtype=np.int32)
+    s, Rt = o.env_mat(coord, nlist, 4.0, 20.0)
+    assert _rel(Rt[0, 0], [1 / 3, 1 / 9, 2 / 9, 2 / 9]) < 1e-15 and s[0, 0] == Rt[0, 0, 0]
+    assert not Rt[0, 1:].any() and not s[0, 1:].any() and not Rt[1, 2].any()
+    assert _rel(Rt[1, 0], [1 / 3, -1 / 9, -2 / 9, -2 / 9]) < 1e-15  # the reverse pair
+    s2, Rt2 = o.env_mat(coord, nlist, 4.0, 20.0, norm=(0.1, 2.0, 3.0))
+    assert _rel(Rt2[0, 0], [(1 / 3 - 0.1) / 2, 1 / 27, 2 / 27, 2 / 27]) < 1e-15 and s2[0, 0] == Rt2[0, 0, 0]
+
+
+def pin_env_mat_matches_generator(o):
+    """Rows from coordinates + neighbour list (periodic images as extra coordinates) equal the rows the
+    workload generator builds on its own (minimum image, its own series cos) — two independent codes."""
+    for w in (W.cu(seed=11, cells=(6, 6, 6), sel=256, fill=0.8, widths=(1, 4)),
+              W.water(seed=12, nmol=160, widths=(1, 4), norm=(0.05, 0.1, 0.2))):
+        coord, nlist, _ = W.ghost_system(w)
+        e = w.env
+        s, Rt = o.env_mat(coord, nlist, e["rcs"], e["rc"], e["kind"], e["norm"])
+        assert _rel(s, w.s) < 1e-12 and _rel(Rt, w.Rt) < 1e-12, (w.name, _rel(s, w.s), _rel(Rt, w.Rt))
+
+
+def _cluster(seed, n=36, L=7.0, rc=4.0, types=2, sel=(20, 30)):
+    """Non-periodic random cluster with a brute-force neighbour list (type, then distance)."""
+    x = W.uniform(seed, (n, 3), 0.0, L)
+    t = (np.arange(n) % types).astype(np.int32)
+    off = np.concatenate([[0], np.cumsum(sel)])
+    nlist = -np.ones((n, int(off[-1])), dtype=np.int32)
+    nvalid = np.zeros((n, types), dtype=np.int32)
+    for i in range(n):
+        d = np.linalg.norm(x - x[i], axis=1)
+        for b in range(types):
+            js = [j for j in np.argsort(d, kind="stable") if j != i and t[j] == b and d[j] < rc][:sel[b]]
+            nlist[i, off[b]:off[b] + len(js)] = js
+            nvalid[i, b] = len(js)
+    return x, t, nlist, nvalid, np.array(sel, dtype=np.int32)
+
+
+def _chain_energy(o, x, t, nlist, nvalid, sel, env, params, widths, info, tabs, dD, M2):
+    s, Rt = o.env_mat(x, nlist, env[0], env[1], env[2], env[3])
+    T = o.fwd(tabs, info, s, Rt, nvalid, t, sel)
+    return float(np.sum(dD * o.descriptor(T, M2))), s, Rt, T
+
+
+def _chain_forces(o, x, t, nlist, nvalid, sel, env, tabs, info, dD, M2):
+    E, s, Rt, T = _chain_energy(o, x, t, nlist, nvalid, sel, env, None, None, info, tabs, dD, M2)
+    dT = o.descriptor_grad(T, dD)
+    ds, dRt = o.grad(tabs, info, s, Rt, nvalid, t, sel, dT)
+    F, Wv = o.force_virial(x, nlist, env[0], env[1], ds, dRt, env[2], env[3])
+    return E, F, Wv
+
+
+def _cluster_model(o, seed, kind, norm):
+    x, t, nlist, nvalid, sel = _cluster(seed)
+    env = (1.5, 4.0, kind, norm)
+    s, _ = o.env_mat(x, nlist, *env[:2], kind, norm)
+    widths = [1, 4, 8]
+    params = W.net_params(seed + 1, widths, 4)
+    valid = nlist >= 0
+    info = o.table_info(float(s[valid].min()) - 0.05, float(s[valid].max()) + 0.05)
+    tabs = o.tables(params, widths, info)
+    dD = W.normal(seed + 2, (x.shape[0], 8, 3))
+    return x, t, nlist, nvalid, sel, env, tabs, info, dD
+
+
+def pin_force_fd(o):
+    """Forces of E = sum_i <dD_i, D_i> (coordinates -> rows -> table -> T -> D) against central
+    differences of E in every coordinate of four atoms, both switches, with and without normalisation."""
+    for seed, kind, norm in ((21, 0, None), (22, 1, (0.2, 0.3, 0.25))):
+        x, t, nlist, nvalid, sel, env, tabs, info, dD = _cluster_model(o, seed, kind, norm)
+        E, F, _ = _chain_forces(o, x, t, nlist, nvalid, sel, env, tabs, info, dD, 3)
+        h = 1e-5
+        for a in (0, 7, 18, 35):
+            for b in range(3):
+                xp, xm = x.copy(), x.copy()
+                xp[a, b] += h
+                xm[a, b] -= h
+                Ep = _chain_energy(o, xp, t, nlist, nvalid, sel, env, None, None, info, tabs, dD, 3)[0]
+                Em = _chain_energy(o, xm, t, nlist, nvalid, sel, env, None, None, info, tabs, dD, 3)[0]
+                fd = -(Ep - Em) / (2 * h)
+                assert abs(fd - F[a, b]) <= 1e-6 * max(1.0, np.abs(F).max()), (seed, a, b, fd, F[a, b])
+
+
+def pin_force_invariants(o):
+    """Translation invariance (sum of forces 0), the virial as sum_a r_a (x) F_a for a cluster, and
+    rotation covariance (E unchanged, F rotated, W -> R W R^T) — Sec. II's symmetries."""
+    x, t, nlist, nvalid, sel, env, tabs, info, dD = _cluster_model(o, 31, 0, None)
+    E, F, Wv = _chain_forces(o, x, t, nlist, nvalid, sel, env, tabs, info, dD, 3)
+    scale = np.abs(F).max()
+    assert np.abs(F.sum(axis=0)).max() < 1e-12 * scale * x.shape[0]
+    assert _rel(Wv, np.einsum("ia,ib->ab", x, F)) < 1e-12
+    c, sn = math.cos(0.7), math.sin(0.7)
+    Rz = np.array([[c, -sn, 0], [sn, c, 0], [0, 0, 1.0]])
+    c2, s2 = math.cos(-1.1), math.sin(-1.1)
+    Rx = np.array([[1.0, 0, 0], [0, c2, -s2], [0, s2, c2]])
+    R = Rz @ Rx
+    E2, F2, W2 = _chain_forces(o, x @ R.T, t, nlist, nvalid, sel, env, tabs, info, dD, 3)
+    assert abs(E2 - E) <= 1e-12 * max(1.0, abs(E))
+    assert _rel(F2, F @ R.T) < 1e-11 and _rel(W2, R @ Wv @ R.T) < 1e-11
+    # an energy that is not rotation invariant, E = sum_i <dT_i, T_i> with dT fixed, has a
+    # non-symmetric virial; it is still sum_a r_a (x) F_a
+    s, Rt = o.env_mat(x, nlist, env[0], env[1], env[2], env[3])
+    dT = W.normal(33, (x.shape[0], 4, 8))
+    ds, dRt = o.grad(tabs, info, s, Rt, nvalid, t, sel, dT)
+    F3, W3 = o.force_virial(x, nlist, env[0], env[1], ds, dRt, env[2], env[3])
+    ref = np.einsum("ia,ib->ab", x, F3)
+    assert _rel(W3, ref) < 1e-12 and _rel(ref, ref.T) > 1e-3
+
+
 ALL_PINS = [pin_net_skip_wiring, pin_net_single_neuron, pin_net_derivatives_fd, pin_table_info, pin_locate,
             pin_table_nodes, pin_table_quintic_exact, pin_table_sin_bound, pin_compressed_vs_net,
             pin_fwd_brute_force, pin_fwd_constant_G, pin_fwd_vs_explicit_G, pin_fwd_padding, pin_fwd_symmetries,
-            pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor, pin_descriptor_grad]
+            pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor, pin_descriptor_grad,
+            pin_switch, pin_env_mat_hand, pin_env_mat_matches_generator, pin_force_fd, pin_force_invariants]

@@ -46,6 +46,18 @@ MUTANTS = [
      "if (m < 0)\n          for (int mp = 0; mp < M; ++mp)"),
     ("descriptor grad: transposed dD", "v += Ga[(size_t)mp * M2 + m] * Ta[k * M + mp];",
      "v += Ga[(size_t)m * M2 + (mp % M2)] * Ta[k * M + mp];"),
+    ("switch: sign of dw/du", "dw = -30.0 * u * u * (u - 1.0) * (u - 1.0);", "dw = 30.0 * u * u * (u - 1.0) * (u - 1.0);"),
+    ("switch: s' without -w/r^2", "*dsv = dw / ((rc - rcs) * r) - w / (r * r);", "*dsv = dw / ((rc - rcs) * r);"),
+    ("switch: cosine of u, not pi u", "w = 0.5 * cos(pi * u) + 0.5;", "w = 0.5 * cos(u) + 0.5;"),
+    ("env mat: xyz not divided by r", "Rt[4 * row + 1 + a] = sv * d[a] / r / sa;", "Rt[4 * row + 1 + a] = sv * d[a] / sa;"),
+    ("env mat: xyz scaled by std of s", "Rt[4 * row + 1 + a] = sv * d[a] / r / sa;",
+     "Rt[4 * row + 1 + a] = sv * d[a] / r / sd;"),
+    ("force: s column gradient dropped from the first R~ entry",
+     "double v = (ds[row] + dRt[4 * row + 0]) * dsv * d[b] / (r * sd);", "double v = ds[row] * dsv * d[b] / (r * sd);"),
+    ("force: reaction on j with the wrong sign", "F[3 * (int64_t)j + b] -= g[b];", "F[3 * (int64_t)j + b] += g[b];"),
+    ("force: delta term of d(d/r) dropped", "sv * (dab / r - d[a] * d[b] / (r2 * r))", "sv * (0.0 / r - d[a] * d[b] / (r2 * r))"),
+    ("virial: sign", "W[3 * a + b] -= d[a] * g[b];", "W[3 * a + b] += d[a] * g[b];"),
+    ("virial: transposed", "W[3 * a + b] -= d[a] * g[b];", "W[3 * a + b] -= d[b] * g[a];"),
 ]
 
 

@@ -68,7 +68,7 @@ def _get_lib():
         lib.wl_species.restype = None
         lib.wl_water.argtypes = [u64, i32, i32, dbl, dbl, dbl, dbl, P, P]
         lib.wl_water.restype = i64
-        lib.wl_envmat.argtypes = [i64, P, P, P, i32, P, dbl, dbl, i32, P, P, P, P, P, P, i32]
+        lib.wl_envmat.argtypes = [i64, P, P, P, i32, P, dbl, dbl, i32, P, P, P, P, P, P, i32, P, P]
         lib.wl_envmat.restype = i32
         _lib = lib
     return _lib
@@ -163,6 +163,7 @@ class Workload:
     stats: dict = field(default_factory=dict)
     pos: np.ndarray | None = None
     box: np.ndarray | None = None
+    env: dict | None = None  # rcs, rc, switch kind, normalisation, nlist [nloc][nnei], image shift [nloc][nnei][3]
 
     @property
     def nloc(self) -> int:
@@ -214,6 +215,8 @@ def _envmat(pos, types, box, ntypes, sel, rcs, rc, kind=0, norm=None, nthreads=0
     nvalid = np.empty((natoms, ntypes), dtype=np.int32)
     stats = np.zeros(4, dtype=np.int64)
     srange = np.zeros(2, dtype=np.float64)
+    nlist = np.empty((natoms, nnei), dtype=np.int32)
+    shift = np.empty((natoms, nnei, 3), dtype=np.int8)
     box = np.ascontiguousarray(box, dtype=np.float64)
     normp = None
     if norm is not None:
@@ -221,12 +224,14 @@ def _envmat(pos, types, box, ntypes, sel, rcs, rc, kind=0, norm=None, nthreads=0
         normp = _ptr(norm_a)
     rc_ = lib.wl_envmat(natoms, _ptr(np.ascontiguousarray(pos)), _ptr(np.ascontiguousarray(types, dtype=np.int32)),
                         _ptr(box), ntypes, _ptr(sel), rcs, rc, kind, normp, _ptr(s), _ptr(Rt), _ptr(nvalid),
-                        _ptr(stats), _ptr(srange), nthreads)
+                        _ptr(stats), _ptr(srange), nthreads, _ptr(nlist), _ptr(shift))
     if rc_ != 0:
         raise RuntimeError(f"wl_envmat failed ({rc_})")
     st = {"real_neighbours_total": int(stats[0]), "rows_dropped_by_sel": int(stats[1]),
           "max_real_neighbours": int(stats[2]), "rows_kept": int(stats[3])}
-    return s, Rt, nvalid, st, float(srange[0]), float(srange[1])
+    env = {"rcs": float(rcs), "rc": float(rc), "kind": int(kind),
+           "norm": None if norm is None else tuple(float(x) for x in norm), "nlist": nlist, "shift": shift}
+    return s, Rt, nvalid, st, float(srange[0]), float(srange[1]), env
 
 
 def tiny(seed: int = 1, nloc: int = 64, nreal: int = 24, sel: int = 32, widths=(1, 8, 16, 32), M2: int = 4,
@@ -269,13 +274,13 @@ def cu(seed: int = 2, fill: float | None = 0.85, a: float | None = None, cells=(
     lib.wl_fcc(_sub_seed(seed, 1), nx, ny, nz, a, jitter, _ptr(pos), _ptr(box))
     types = np.zeros(nat, dtype=np.int32)
     sela = np.array([sel], dtype=np.int32)
-    s, Rt, nvalid, st, smin, smax = _envmat(pos, types, box, 1, sela, rcs, rc)
+    s, Rt, nvalid, st, smin, smax, env = _envmat(pos, types, box, 1, sela, rcs, rc)
     widths = list(widths)
     st.update({"lattice_constant": round(a, 6), "rcs": rcs, "rc": rc, "box": [float(x) for x in box]})
     return Workload(name=name or ("cu85" if fill else "cu"), seed=seed, ntypes=1, sel=sela,
                     widths=widths, M2=M2, s=s, Rt=Rt, nvalid=nvalid, atype=types,
                     params=net_params(_sub_seed(seed, 2), widths, 1), dT=_dT(seed, nat, widths[-1]),
-                    s_min=smin, s_max=smax, stats=st, pos=pos, box=box)
+                    s_min=smin, s_max=smax, stats=st, pos=pos, box=box, env=env)
 
 
 def water(seed: int = 3, nmol: int = 4096, extra_o: int = 0, density: float = 0.0334, sel=(46, 92),
@@ -292,13 +297,13 @@ def water(seed: int = 3, nmol: int = 4096, extra_o: int = 0, density: float = 0.
         raise RuntimeError(f"wl_water failed ({att})")
     box = np.array([L, L, L], dtype=np.float64)
     sela = np.array(sel, dtype=np.int32)
-    s, Rt, nvalid, st, smin, smax = _envmat(pos, types, box, 2, sela, rcs, rc, norm=norm)
+    s, Rt, nvalid, st, smin, smax, env = _envmat(pos, types, box, 2, sela, rcs, rc, norm=norm)
     widths = list(widths)
     st.update({"box": L, "rcs": rcs, "rc": rc, "placement_attempts": int(att), "molecules": nmol,
                "extra_O": extra_o})
     return Workload(name=name, seed=seed, ntypes=2, sel=sela, widths=widths, M2=M2, s=s, Rt=Rt, nvalid=nvalid,
                     atype=types, params=net_params(_sub_seed(seed, 2), widths, 4), dT=_dT(seed, nat, widths[-1]),
-                    s_min=smin, s_max=smax, stats=st, pos=pos, box=box)
+                    s_min=smin, s_max=smax, stats=st, pos=pos, box=box, env=env)
 
 
 def alcumg(seed: int = 4, pad: float | None = 0.3, cells=(16, 16, 32), sel=(400, 60, 40),
@@ -324,7 +329,7 @@ def alcumg(seed: int = 4, pad: float | None = 0.3, cells=(16, 16, 32), sel=(400,
     order = np.argsort(types, kind="stable")
     pos = np.ascontiguousarray(pos[order])
     types = np.ascontiguousarray(types[order])
-    s, Rt, nvalid, st, smin, smax = _envmat(pos, types, box, 3, sela, rcs, rc)
+    s, Rt, nvalid, st, smin, smax, env = _envmat(pos, types, box, 3, sela, rcs, rc)
     widths = list(widths)
     achieved_pad = 1.0 - float(nvalid.astype(np.int64).sum()) / float(nat * nnei)
     st.update({"lattice_constant": round(a, 6), "pad_target": pad, "pad_achieved": round(achieved_pad, 4),
@@ -332,7 +337,7 @@ def alcumg(seed: int = 4, pad: float | None = 0.3, cells=(16, 16, 32), sel=(400,
     return Workload(name=name or (f"alcumg_pad{int(round(pad * 100))}" if pad is not None else "alcumg_a405"),
                     seed=seed, ntypes=3, sel=sela, widths=widths, M2=M2, s=s, Rt=Rt, nvalid=nvalid, atype=types,
                     params=net_params(_sub_seed(seed, 2), widths, 9), dT=_dT(seed, nat, widths[-1]),
-                    s_min=smin, s_max=smax, stats=st, pos=pos, box=box)
+                    s_min=smin, s_max=smax, stats=st, pos=pos, box=box, env=env)
 
 
 def water_large(seed: int = 5, nmol: int = 349525, extra_o: int = 1, **kw) -> Workload:
@@ -362,3 +367,28 @@ def shard(nloc: int, rank: int, world: int) -> tuple[int, int]:
     base, rem = divmod(nloc, world)
     lo = rank * base + min(rank, rem)
     return lo, lo + base + (1 if rank < rem else 0)
+
+
+def ghost_system(w: Workload):
+    """Coordinates with periodic images as extra atoms, for inputs given as positions and a neighbour list.
+
+    Returns (coord [nall][3] f64, nlist [nloc][nnei] int32 indexing coord, -1 on padding rows,
+    owner [nall] int32: the local atom each coordinate is a copy of).  Neighbour rows whose image
+    shift is zero point at the local atom itself; every other (atom, shift) pair becomes one
+    image, placed at r_j + shift * box.
+    """
+    if w.env is None or w.pos is None:
+        raise ValueError(f"workload {w.name} has no positions and neighbour list")
+    nl, sh = w.env["nlist"], w.env["shift"].astype(np.int64)
+    nloc = w.nloc
+    code = (sh[..., 0] + 1) * 9 + (sh[..., 1] + 1) * 3 + (sh[..., 2] + 1)  # 13 = no shift
+    need = (nl >= 0) & (code != 13)
+    key = nl.astype(np.int64) * 27 + code
+    uniq, inv = np.unique(key[need], return_inverse=True)
+    j_img, c_img = uniq // 27, uniq % 27
+    shv = np.stack([c_img // 9 - 1, (c_img // 3) % 3 - 1, c_img % 3 - 1], axis=1).astype(np.float64)
+    coord = np.concatenate([w.pos, w.pos[j_img] + shv * w.box[None, :]], axis=0)
+    nlist = nl.copy()
+    nlist[need] = (nloc + inv).astype(np.int32)
+    owner = np.concatenate([np.arange(nloc), j_img]).astype(np.int32)
+    return np.ascontiguousarray(coord), np.ascontiguousarray(nlist), owner

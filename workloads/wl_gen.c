@@ -365,6 +365,7 @@ int64_t wl_water(uint64_t seed, int nmol, int extra_o, double L, double r_oo_min
 typedef struct {
   double r, d[3];
   int32_t j, t;
+  int8_t sh[3];
 } cand_t;
 
 static int cand_cmp(const void *pa, const void *pb) {
@@ -387,10 +388,13 @@ static int cand_cmp(const void *pa, const void *pb) {
  * stats (int64[4]): total real neighbours before the cap, rows dropped by
  * the cap, maximum per-atom real count, rows kept.
  * srange (double[2]): min and max of s over kept rows.
+ * nlist (int32 [natoms][nnei], optional): the neighbour index of each row,
+ * -1 on padding rows; shift (int8 [natoms][nnei][3], optional): the periodic
+ * image of that neighbour, r_j + shift * box being the position the row uses.
  */
 int wl_envmat(int64_t natoms, const double *pos, const int32_t *types, const double box[3], int ntypes,
               const int32_t *sel, double rcs, double rc, int kind, const double *norm, double *s, double *Rt,
-              int32_t *nvalid, int64_t *stats, double *srange, int nthreads) {
+              int32_t *nvalid, int64_t *stats, double *srange, int nthreads, int32_t *nlist, int8_t *shift) {
   if (ntypes < 1 || ntypes > 64) return -1;
   for (int d = 0; d < 3; ++d)
     if (box[d] < 2.0 * rc) return -4; /* minimum image needs L >= 2 rc */
@@ -476,14 +480,20 @@ int wl_envmat(int64_t natoms, const double *pos, const int32_t *types, const dou
             for (int32_t j = head[cj]; j >= 0; j = next[j]) {
               if (j == i) continue;
               double dv[3], r2 = 0.0;
+              int8_t sh[3];
               for (int d = 0; d < 3; ++d) {
                 double dd = pos[3 * j + d] - pos[3 * i + d];
-                dd -= box[d] * nearbyint(dd / box[d]);
+                const double k = nearbyint(dd / box[d]);
+                dd -= box[d] * k;
+                sh[d] = (int8_t)(-k);
                 dv[d] = dd;
                 r2 += dd * dd;
               }
               if (r2 >= rc * rc) continue;
               cand_t cd;
+              cd.sh[0] = sh[0];
+              cd.sh[1] = sh[1];
+              cd.sh[2] = sh[2];
               cd.r = sqrt(r2);
               cd.d[0] = dv[0];
               cd.d[1] = dv[1];
@@ -519,6 +529,12 @@ int wl_envmat(int64_t natoms, const double *pos, const int32_t *types, const dou
           Rt[4 * row + 1] = sx;
           Rt[4 * row + 2] = sy;
           Rt[4 * row + 3] = sz;
+          if (nlist) nlist[row] = cand[k].j;
+          if (shift) {
+            shift[3 * row + 0] = cand[k].sh[0];
+            shift[3 * row + 1] = cand[k].sh[1];
+            shift[3 * row + 2] = cand[k].sh[2];
+          }
           if (sh < smin) smin = sh;
           if (sh > smax) smax = sh;
           ++kept;
@@ -527,6 +543,8 @@ int wl_envmat(int64_t natoms, const double *pos, const int32_t *types, const dou
           int64_t row = i * nnei + off[t] + q;
           s[row] = 0.0;
           Rt[4 * row + 0] = Rt[4 * row + 1] = Rt[4 * row + 2] = Rt[4 * row + 3] = 0.0;
+          if (nlist) nlist[row] = -1;
+          if (shift) shift[3 * row + 0] = shift[3 * row + 1] = shift[3 * row + 2] = 0;
         }
         nvalid[i * ntypes + t] = kept;
         tot_kept += kept;
