@@ -258,6 +258,67 @@ int dp_descriptor_contract_grad_f64(const double *T, const double *dD, int64_t n
 int dp_descriptor_contract_grad_f32(const float *T, const float *dD, int64_t nloc, int M1, int M2, float *dT,
                                     void *stream);
 
+/* ------------------------------------------------------------------------
+ * Environment matrix front end and force / virial back end (Sec. II: the
+ * weighting function s(r), the 4-vector rows and their normalisation; the
+ * forces and virials follow from the derivatives of E with respect to atom i
+ * and its neighbours).
+ *
+ * Coordinates: coord [nall][3], every position a neighbour list can point
+ * at (local atoms first, nloc of them, then periodic images or ghost atoms,
+ * as a domain decomposition provides them).  Neighbour list: nlist
+ * [nloc][nnei] int32, row q of atom i holds the index j into coord of the
+ * neighbour (the formatted list of Sec. II: per type segment the neighbours
+ * sorted by distance, then -1 on every padding row).  d = coord[j] - coord[i].
+ */
+typedef struct dp_env_info {
+  double rcs, rc;        /* smooth cutoff and cutoff, 0 < rcs < rc                     */
+  int32_t kind;          /* 1: the paper's switch u^3(-6u^2+15u-10)+1; 0: cos(pi u)/2+1/2 */
+  double mean, std;      /* normalisation of s: (s - mean) / std, std > 0 (0 and 1 = none) */
+  double std_all;        /* normalisation of the xyz entries, > 0 (1 = none)           */
+} dp_env_info;
+
+/*
+ * Rows of the environment matrix (Sec. II), u = (r - rcs)/(rc - rcs):
+ *   s(r) = 1/r (r < rcs),  w(u)/r (rcs <= r < rc),  0 (r >= rc)
+ *   R~ = ( (s(r) - mean)/std,  s(r) d_x/(r std_all),  s(r) d_y/(r std_all),  s(r) d_z/(r std_all) )
+ * and s (the embedding input) = R~[0].  Rows with j < 0 are zero.
+ *   coord [nall][3], nlist [nloc][nnei] inputs; env (host);
+ *   s [nloc][nnei], Rt [nloc][nnei][4], nvalid [nloc][ntypes] int32 outputs
+ *   (nvalid[i][b] = number of rows of segment b with j >= 0; with a formatted
+ *   list these are the segment's first rows, as the fusion kernels expect).
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (nloc < 0, nnei < 1, sum(sel) != nnei),
+ * DP_ERR_UNSUPPORTED (ntypes > DP_MAX_TYPES), DP_ERR_TABLE_INFO (env not as
+ * stated), DP_ERR_CUDA.  nloc == 0 returns DP_OK without reading any pointer.
+ * Indices j must lie in [0, nall); they are not checked on the device.
+ */
+int dp_env_mat_f64(const double *coord, const int32_t *nlist, int64_t nloc, int nnei, int ntypes,
+                   const int32_t *sel, const dp_env_info *env, double *s, double *Rt, int32_t *nvalid,
+                   void *stream);
+int dp_env_mat_f32(const float *coord, const int32_t *nlist, int64_t nloc, int nnei, int ntypes, const int32_t *sel,
+                   const dp_env_info *env, float *s, float *Rt, int32_t *nvalid, void *stream);
+
+/*
+ * Forces and virial from ds = dE/ds [nloc][nnei] and dRt = dE/dR~
+ * [nloc][nnei][4] (the outputs of dp_tabulate_fusion_grad_*), by the chain
+ * rule through the rows above.  For a row (i, j) the gradient with respect to
+ * d is
+ *   g = (ds + dRt_0) s'(r)/(r std) d  +  (s'(r)/r^2 - s(r)/r^3) (dRt_xyz . d)/std_all d  +  s(r)/(r std_all) dRt_xyz
+ * and F[i] += g, F[j] -= g (F = -dE/dr), virial[a][b] -= d_a g_b, summed
+ * over all rows with j >= 0.
+ *   F [nall][3] and virial [3][3] outputs, fully overwritten (forces on
+ *   images / ghosts land on their own rows: fold them onto their owners as
+ *   the domain decomposition requires).  Summation order is not fixed
+ *   (atomic adds), so results agree with any serial order up to rounding.
+ * Errors as dp_env_mat_* (nall < nloc is DP_ERR_SHAPE).
+ */
+int dp_force_virial_f64(const double *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,
+                        const dp_env_info *env, const double *ds, const double *dRt, double *F, double *virial,
+                        void *stream);
+int dp_force_virial_f32(const float *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,
+                        const dp_env_info *env, const float *ds, const float *dRt, float *F, float *virial,
+                        void *stream);
+
 #ifdef __cplusplus
 }
 #endif

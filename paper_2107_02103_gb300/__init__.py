@@ -40,6 +40,22 @@ class dp_table_info(ctypes.Structure):
                 f"stride0={self.stride0!r}, stride1={self.stride1!r})")
 
 
+class dp_env_info(ctypes.Structure):
+    """Environment-matrix parameters (mirror of the C struct): cutoffs, switch kind, normalisation."""
+    _fields_ = [("rcs", ctypes.c_double), ("rc", ctypes.c_double), ("kind", ctypes.c_int32),
+                ("mean", ctypes.c_double), ("std", ctypes.c_double), ("std_all", ctypes.c_double)]
+
+    def __repr__(self):
+        return (f"dp_env_info(rcs={self.rcs!r}, rc={self.rc!r}, kind={self.kind!r}, mean={self.mean!r}, "
+                f"std={self.std!r}, std_all={self.std_all!r})")
+
+
+def env_info(rcs: float, rc: float, kind: int = 0, norm=None) -> dp_env_info:
+    """dp_env_info from cutoffs, switch kind (0 cosine, 1 the paper's quintic) and norm = (mean, std, std_all)."""
+    mean, std, std_all = (0.0, 1.0, 1.0) if norm is None else (float(x) for x in norm)
+    return dp_env_info(float(rcs), float(rc), int(kind), mean, std, std_all)
+
+
 class DPError(RuntimeError):
     def __init__(self, code: int, msg: str):
         super().__init__(f"[{code}] {msg}")
@@ -49,6 +65,7 @@ class DPError(RuntimeError):
 _P = ctypes.c_void_p
 _I32, _I64, _D = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
 _INFO = ctypes.POINTER(dp_table_info)
+_ENV = ctypes.POINTER(dp_env_info)
 _SIGS = {
     "dp_last_error": ([], ctypes.c_char_p),
     "dp_table_info_make": ([_D, _D, _D, _D, _D, _INFO], ctypes.c_int),
@@ -76,6 +93,10 @@ _SIGS = {
                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_moments_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
+    "dp_env_mat_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
+    "dp_env_mat_f32": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
+    "dp_force_virial_f64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_force_virial_f32": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_f64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_f32": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_grad_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
@@ -251,6 +272,54 @@ def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(dT), _ptr(ds), _ptr(dRt), _stream(s)))
     return ds, dRt
+
+
+def dp_env_mat(coord, nlist, sel, env: dp_env_info, out=None):
+    """(s [nloc][nnei], Rt [nloc][nnei][4], nvalid [nloc][ntypes] int32) from coord [nall][3] and nlist [nloc][nnei]."""
+    coord = _dev(coord, "coord", None)
+    dtype = coord.dtype
+    if coord.dim() != 2 or coord.shape[1] != 3:
+        raise ValueError("coord must be [nall][3]")
+    nlist = _dev(nlist, "nlist", torch.int32)
+    nloc, nnei = (int(x) for x in nlist.shape)
+    selc, ntypes, nsum = _sel_arr(sel)
+    if nsum != nnei:
+        raise ValueError(f"sum(sel) = {nsum} != nnei = {nnei}")
+    if out is None:
+        s = torch.empty((nloc, nnei), dtype=dtype, device=coord.device)
+        Rt = torch.empty((nloc, nnei, 4), dtype=dtype, device=coord.device)
+        nvalid = torch.empty((nloc, ntypes), dtype=torch.int32, device=coord.device)
+    else:
+        s = _dev(out[0], "s", dtype, (nloc, nnei))
+        Rt = _dev(out[1], "Rt", dtype, (nloc, nnei, 4))
+        nvalid = _dev(out[2], "nvalid", torch.int32, (nloc, ntypes))
+    fn = getattr(_lib, f"dp_env_mat_{_suffix(dtype)}")
+    _check(fn(_ptr(coord), _ptr(nlist), nloc, nnei, ntypes, selc, ctypes.byref(env), _ptr(s), _ptr(Rt), _ptr(nvalid),
+              _stream(coord)))
+    return s, Rt, nvalid
+
+
+def dp_force_virial(coord, nlist, env: dp_env_info, ds, dRt, out=None):
+    """(F [nall][3], virial [3][3]) from dE/ds [nloc][nnei] and dE/dRt [nloc][nnei][4]."""
+    coord = _dev(coord, "coord", None)
+    dtype = coord.dtype
+    if coord.dim() != 2 or coord.shape[1] != 3:
+        raise ValueError("coord must be [nall][3]")
+    nall = int(coord.shape[0])
+    nlist = _dev(nlist, "nlist", torch.int32)
+    nloc, nnei = (int(x) for x in nlist.shape)
+    ds = _dev(ds, "ds", dtype, (nloc, nnei))
+    dRt = _dev(dRt, "dRt", dtype, (nloc, nnei, 4))
+    if out is None:
+        F = torch.empty((nall, 3), dtype=dtype, device=coord.device)
+        W = torch.empty((3, 3), dtype=dtype, device=coord.device)
+    else:
+        F = _dev(out[0], "F", dtype, (nall, 3))
+        W = _dev(out[1], "virial", dtype, (3, 3))
+    fn = getattr(_lib, f"dp_force_virial_{_suffix(dtype)}")
+    _check(fn(_ptr(coord), _ptr(nlist), nloc, nall, nnei, ctypes.byref(env), _ptr(ds), _ptr(dRt), _ptr(F), _ptr(W),
+              _stream(coord)))
+    return F, W
 
 
 def dp_descriptor_contract(T, M2: int, out=None) -> torch.Tensor:

@@ -109,6 +109,23 @@ def test_validation_codes_without_gpu(dpc):
     assert lib.dp_embedding_net_nodes_f64(fake, w, 2, 1, ctypes.byref(info), fake, fake, fake,
                                           None) == dpc.DP_ERR_UNSUPPORTED
     assert dpc.dp_last_error() != ""
+    env = dpc.env_info(0.5, 6.0)
+    assert lib.dp_env_mat_f64(fake, fake, -1, 7, 2, sel, ctypes.byref(env), fake, fake, fake, None) == dpc.DP_ERR_SHAPE
+    assert lib.dp_env_mat_f64(fake, fake, 5, 8, 2, sel, ctypes.byref(env), fake, fake, fake, None) == dpc.DP_ERR_SHAPE
+    assert lib.dp_env_mat_f32(fake, fake, 5, 7, 2, sel, None, fake, fake, fake, None) == dpc.DP_ERR_NULL
+    for bad in (dpc.env_info(6.0, 0.5), dpc.env_info(0.0, 6.0), dpc.env_info(0.5, 6.0, kind=2),
+                dpc.env_info(0.5, 6.0, norm=(0.0, 0.0, 1.0)), dpc.env_info(0.5, 6.0, norm=(0.0, 1.0, -1.0))):
+        assert lib.dp_env_mat_f64(fake, fake, 5, 7, 2, sel, ctypes.byref(bad), fake, fake, fake,
+                                  None) == dpc.DP_ERR_TABLE_INFO
+    assert lib.dp_env_mat_f64(None, None, 0, 7, 2, sel, ctypes.byref(env), None, None, None, None) == dpc.DP_OK
+    assert lib.dp_env_mat_f64(None, fake, 5, 7, 2, sel, ctypes.byref(env), fake, fake, fake, None) == dpc.DP_ERR_NULL
+    fv = lib.dp_force_virial_f64
+    assert fv(fake, fake, 5, 4, 7, ctypes.byref(env), fake, fake, fake, fake, None) == dpc.DP_ERR_SHAPE  # nall < nloc
+    assert fv(fake, fake, 5, 9, 0, ctypes.byref(env), fake, fake, fake, fake, None) == dpc.DP_ERR_SHAPE
+    assert fv(fake, fake, 5, 9, 7, ctypes.byref(env), fake, fake, fake, None, None) == dpc.DP_ERR_NULL
+    assert fv(fake, None, 5, 9, 7, ctypes.byref(env), fake, fake, fake, fake, None) == dpc.DP_ERR_NULL
+    bad = dpc.env_info(0.5, 6.0, kind=3)
+    assert fv(fake, fake, 5, 9, 7, ctypes.byref(bad), fake, fake, fake, fake, None) == dpc.DP_ERR_TABLE_INFO
 
 
 def test_binding_rejects_cpu_tensors(dpc):
