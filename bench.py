@@ -44,6 +44,18 @@ FMA_LANES = {"f64": 2, "f32": 128}
 # algorithmic FMAs per valid neighbour x channel
 FMA_PER_EVAL = {"fwd": 9, "grad": 18}
 DESC_FMA_PER_ATOM = lambda M1, M2: 4 * M1 * M2  # noqa: E731
+# backward of D: dT[k][m] = sum_n dD[m][n] T[k][n] + [m < M2] sum_m' dD[m'][m] T[k][m']
+DESC_GRAD_FMA_PER_ATOM = lambda M1, M2: 8 * M1 * M2  # noqa: E731
+
+
+def chain_bytes(w, esize: int, nall: int) -> dict:
+    """Algorithmic DRAM bytes of the chain's front and back end (the unique data each one must move):
+    env_mat reads the neighbour list and the coordinates once and writes s, R~ (every row) and the counts;
+    force_virial reads the neighbour list, the coordinates, ds and dR~ once and writes forces and virial."""
+    rows = w.nloc * w.nnei
+    coord = 3 * esize * nall
+    return {"env_mat": rows * (4 + 5 * esize) + coord + 4 * w.nloc * w.ntypes,
+            "force_virial": rows * (4 + 5 * esize) + 2 * coord + 9 * esize}
 
 
 # Interval-moment path: a run of L consecutive valid rows of one atom in one table
@@ -86,7 +98,7 @@ def moment_fmas(runs, M1: int) -> dict:
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
 # `ncu --set full` capture of its current version (profiles/<kernel>_<algo>_<workload>_<dtype>.md);
 # absent means no capture of the current kernel exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83860224 + 32249344}
+PROFILED_DRAM_BYTES = {}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
@@ -188,11 +200,76 @@ class ClockSampler:
 
 
 # --------------------------------------------------------------- native arm
+def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
+    """Host inputs, resident device inputs and outputs, the kernel names and one step of the path.
+
+    Default step: fwd -> descriptor -> grad, from resident s, R~, nvalid, atype and a given dE/dT.
+    --chain: the whole descriptor chain from coordinates to forces, env_mat -> fwd -> descriptor ->
+    descriptor_grad (a given dE/dD) -> grad -> force_virial, from resident coordinates (periodic images
+    as extra rows), the neighbour list, atype and dE/dD."""
+    import torch
+
+    import workloads as W
+    fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
+    grad = dpc.dp_tabulate_fusion_grad_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_grad
+    T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
+    D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
+    ds = torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev)
+    dRt = torch.empty((w.nloc, w.nnei, 4), dtype=dtype, device=dev)
+    if not args.chain:
+        host = {"s": np.ascontiguousarray(w.s.astype(npdt)), "Rt": np.ascontiguousarray(w.Rt.astype(npdt)),
+                "nvalid": w.nvalid, "atype": w.atype, "dT": np.ascontiguousarray(w.dT.astype(npdt))}
+        d = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
+        outs = dict(T=T, D=D, ds=ds, dRt=dRt)
+        names = ["fwd", "descriptor", "grad"]
+
+        def step(rec, x, o):
+            rec(0)
+            fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
+            rec(1)
+            dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"])
+            rec(2)
+            grad(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, x["dT"], out=(o["ds"], o["dRt"]))
+            rec(3)
+        return host, d, outs, names, step
+
+    coord, nlist, _ = W.ghost_system(w)
+    nv = w.env["norm"]
+    env = dpc.env_info(w.env["rcs"], w.env["rc"], w.env["kind"], nv)
+    dD = W.normal(W._sub_seed(w.seed, 404), (w.nloc, w.M1, w.M2))
+    host = {"coord": np.ascontiguousarray(coord.astype(npdt)), "nlist": nlist, "atype": w.atype,
+            "dD": np.ascontiguousarray(dD.astype(npdt))}
+    d = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
+    work = dict(s=torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev),
+                Rt=torch.empty((w.nloc, w.nnei, 4), dtype=dtype, device=dev),
+                nvalid=torch.empty((w.nloc, w.ntypes), dtype=torch.int32, device=dev),
+                dT=torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev), T=T, ds=ds, dRt=dRt)
+    outs = dict(D=D, F=torch.empty((coord.shape[0], 3), dtype=dtype, device=dev),
+                virial=torch.empty((3, 3), dtype=dtype, device=dev))
+    names = ["env_mat", "fwd", "descriptor", "descriptor_grad", "grad", "force_virial"]
+
+    def step(rec, x, o):
+        rec(0)
+        dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]))
+        rec(1)
+        fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
+        rec(2)
+        dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"])
+        rec(3)
+        dpc.dp_descriptor_contract_grad(work["T"], x["dD"], out=work["dT"])
+        rec(4)
+        grad(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, work["dT"],
+             out=(work["ds"], work["dRt"]))
+        rec(5)
+        dpc.dp_force_virial(x["coord"], x["nlist"], env, work["ds"], work["dRt"], out=(o["F"], o["virial"]))
+        rec(6)
+    return host, d, outs, names, step
+
+
 def run_native(args, rank, world, local_rank):
     import torch
 
     import paper_2107_02103_gb300 as dpc
-    import workloads as W
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
@@ -202,47 +279,28 @@ def run_native(args, rank, world, local_rank):
     if args.workload == "alcumg":
         kw["pad"] = args.pad
     w = rank_workload(args, rank, world, **kw)
+    if args.chain and w.env is None:
+        raise SystemExit(f"--chain needs positions and a neighbour list; workload {w.name} has none")
     info = dpc.dp_table_info_make(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
     model = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, dtype)
     sel = [int(x) for x in w.sel]
-
-    host = {"s": np.ascontiguousarray(w.s.astype(npdt)), "Rt": np.ascontiguousarray(w.Rt.astype(npdt)),
-            "nvalid": w.nvalid, "atype": w.atype, "dT": np.ascontiguousarray(w.dT.astype(npdt))}
-    d = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
-    T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
-    D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
-    ds = torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev)
-    dRt = torch.empty((w.nloc, w.nnei, 4), dtype=dtype, device=dev)
+    host, d, outs, names, step = build_step(args, w, dpc, model, info, sel, dtype, npdt, dev)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 256 MiB > 126 MiB L2
     stream = torch.cuda.current_stream(dev)
+    nk = len(names)
 
-    fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
-    grad = dpc.dp_tabulate_fusion_grad_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_grad
-
-    def step(ev=None, x=None, o=None):
-        x = x or d
-        o = o or dict(T=T, D=D, ds=ds, dRt=dRt)
-        if ev:
-            ev[0].record(stream)
-        fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
-        if ev:
-            ev[1].record(stream)
-        dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"])
-        if ev:
-            ev[2].record(stream)
-        grad(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, x["dT"], out=(o["ds"], o["dRt"]))
-        if ev:
-            ev[3].record(stream)
+    def run_step(ev=None, x=None, o=None):
+        step((lambda k: ev[k].record(stream)) if ev else (lambda k: None), x or d, o or outs)
 
     for _ in range(args.warmup):
-        step()
+        run_step()
     torch.cuda.synchronize(dev)
 
     def barrier():
         if world > 1:
             torch.distributed.barrier()
 
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
     vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
     clocks = ClockSampler(vis[local_rank] if local_rank < len(vis) else str(local_rank))
     barrier()
@@ -252,31 +310,32 @@ def run_native(args, rank, world, local_rank):
     t_wall0 = time.perf_counter()
     for k in range(args.steps):
         flush.zero_()  # evict the previous step's data from L2 (outside the timed events)
-        step(evs[k])
+        run_step(evs[k])
     torch.cuda.synchronize(dev)
     t_wall = time.perf_counter() - t_wall0
     barrier()
     clk = clocks.stop() if rank == 0 else None
 
-    step_ms = [e[0].elapsed_time(e[3]) for e in evs]
-    k_ms = {"fwd": [e[0].elapsed_time(e[1]) for e in evs], "descriptor": [e[1].elapsed_time(e[2]) for e in evs],
-            "grad": [e[2].elapsed_time(e[3]) for e in evs]}
+    step_ms = [e[0].elapsed_time(e[nk]) for e in evs]
+    k_ms = {n: [e[j].elapsed_time(e[j + 1]) for e in evs] for j, n in enumerate(names)}
     total_s, evals_all = reduce_over_ranks(sum(step_ms) / 1e3, float(w.evals), world, dev)
 
     # ---- end to end through the public API: pinned host inputs -> device -> path -> host results
-    e2e = None if args.no_e2e else measure_e2e(args, host, d, dict(T=T, D=D, ds=ds, dRt=dRt), step, stream, dev,
-                                                world, barrier, evals_all)
+    e2e = None if args.no_e2e else measure_e2e(args, host, d, outs, run_step, stream, dev, world, barrier,
+                                                evals_all)
     if rank != 0:
         return None
     fmas = None
     if args.algo == "moments":
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
-    return report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas)
+    nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
+    return report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall)
 
 
 def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_all):
     """The metric end to end through the public API with host buffers: every step uploads its inputs
-    (s, R~, nvalid, atype, dT) from pinned host memory and downloads its results (T, D, ds, dR~).  Steps
+    (s, R~, nvalid, atype, dT; with --chain coordinates, neighbour list, atype, dE/dD) from pinned host
+    memory and downloads its results (T, D, ds, dR~; with --chain D, forces and virial).  Steps
     are pipelined the way a streaming caller would run them: double-buffered device inputs and outputs,
     the upload of step k+1 and the download of step k-1 on their own streams while step k computes."""
     import torch
@@ -335,18 +394,26 @@ def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_al
             "d2h_bytes_per_step": d2h, "pipelined": "double-buffered, uploads and downloads on their own streams"}
 
 
-def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas=None):
+def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas=None, nall=0):
     value = evals_all * args.steps / total_s
     # ---- roofline of the dominant kernel (FMA pipe of the path's dtype), on the FMAs of the
     # algorithm the kernels run: per-row evaluation, or interval moments (fmas, from the run lengths)
     mean = {k: sum(v) / len(v) for k, v in k_ms.items()}
     fmas = fmas or {"fwd": FMA_PER_EVAL["fwd"] * w.evals, "grad": FMA_PER_EVAL["grad"] * w.evals}
     flops = {"fwd": 2.0 * fmas["fwd"], "grad": 2.0 * fmas["grad"],
-             "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
+             "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc,
+             "descriptor_grad": 2.0 * DESC_GRAD_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
+    nbytes = chain_bytes(w, 8 if args.dtype == "f64" else 4, nall) if args.chain else {}
     pk = peak_tflops(args.dtype)
-    kernels = {k: {"ms": round(mean[k], 4), "share": round(mean[k] / sum(mean.values()), 4),
-                   "tflops": round(flops[k] / (mean[k] * 1e-3) / 1e12, 4),
-                   "frac": round(flops[k] / (mean[k] * 1e-3) / 1e12 / pk, 4)} for k in mean}
+    kernels = {}
+    for k in mean:
+        e = {"ms": round(mean[k], 4), "share": round(mean[k] / sum(mean.values()), 4)}
+        if k in flops:
+            e["tflops"] = round(flops[k] / (mean[k] * 1e-3) / 1e12, 4)
+            e["frac"] = round(flops[k] / (mean[k] * 1e-3) / 1e12 / pk, 4)
+        if k in nbytes:
+            e["gbs"] = round(nbytes[k] / (mean[k] * 1e-3) / 1e9, 1)
+        kernels[k] = e
     dom = max(mean, key=mean.get)
     achieved = flops[dom] / (mean[dom] * 1e-3) / 1e12
     path_tflops = (flops["fwd"] + flops["grad"]) / ((mean["fwd"] + mean["grad"]) * 1e-3) / 1e12
@@ -363,7 +430,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         "config": {"workload": workload_label(w),
                    "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
                                    else f"atoms split over {world} ranks"),
-                   "step": "fwd + descriptor + grad", "algo": args.algo,
+                   "step": ("env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain
+                            else "fwd + descriptor + grad"), "algo": args.algo,
                    "fma_basis": ("interval moments: per run min(9 M1 L, 24 M1 + 24 L) fwd, "
                                  "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
                                  else "per row: 9 M1 fwd, 18 M1 grad"),
@@ -373,7 +441,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         "roofline": roofline,
         "kernels": kernels,
         "e2e": e2e,
-        "gpu_launches": 3 * args.steps * world,
+        "gpu_launches": len(k_ms) * args.steps * world,
         "clocks": clk,
         "wall_s_timed_region": round(t_wall, 4),
     }
@@ -497,6 +565,8 @@ def main():
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--chain", action="store_true",
+                    help="time the whole chain from coordinates to forces (env_mat ... force_virial)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -305,6 +305,7 @@ __device__ __forceinline__ void form_H_group(MomentGradStage<real> &st, const re
 
 // Per-row backward of queued rows q0 .. q0+G-1 (those below nq): lane = (row p, channel lane c),
 // each lane summing the five outputs over the channels c, c + C, ... (18 FMA per channel).
+// dts holds dT_i / N_c, so the sums are the outputs.
 template <int G, typename real>
 __device__ __forceinline__ void grad_rows_group(const GradParams<real> &P, const MomentGradStage<real> &st,
                                                 const real *__restrict__ tab, const real *dts, int64_t i, int q0,
@@ -361,9 +362,9 @@ __device__ __forceinline__ void grad_rows_group(const GradParams<real> &P, const
       if (x < nreal) {
         const int comp = base + x;
         if (comp == 0)
-          ds_i[row] = (rw & kClamped) ? real(0) : a[x] * P.inv_nnei;
+          ds_i[row] = (rw & kClamped) ? real(0) : a[x];
         else
-          dR_i[(size_t)row * 4 + comp - 1] = a[x] * P.inv_nnei;
+          dR_i[(size_t)row * 4 + comp - 1] = a[x];
       }
   }
 }
@@ -428,11 +429,11 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     if (lane < P.ntypes) x = clampi(P.nvalid ? __ldg(P.nvalid + i * P.ntypes + lane) : sl, 0, sl);
     if (lane < DP_MAX_TYPES) st.nvb[lane] = x;
   }
-  {
+  {  // dT_i / N_c, transposed: the 1/N_c of every output is folded in here, once per atom
     const real *__restrict__ dTi = P.dT + i * 4 * M1;
     for (int e = lane; e < 4 * M1; e += 32) {
       const int k = e / M1, m = e - k * M1;
-      dts[m * 4 + k] = __ldg(dTi + e);
+      dts[m * 4 + k] = __ldg(dTi + e) * P.inv_nnei;
     }
   }
   __syncwarp();
@@ -468,8 +469,8 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     dsv = fma(r2, G[2], dsv);
     dsv = fma(r3, G[3], dsv);
     const int row = rw & (kClamped - 1);
-    ds_i[row] = (rw & kClamped) ? real(0) : dsv * P.inv_nnei;
-    st4(dR_i + (size_t)row * 4, dR[0] * P.inv_nnei, dR[1] * P.inv_nnei, dR[2] * P.inv_nnei, dR[3] * P.inv_nnei);
+    ds_i[row] = (rw & kClamped) ? real(0) : dsv;
+    st4(dR_i + (size_t)row * 4, dR[0], dR[1], dR[2], dR[3]);
   };
   constexpr int kCarrySlot = chunk_runs<real>();
 
