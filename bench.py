@@ -41,6 +41,9 @@ SM_MAX_MHZ = 2070.0
 # FP64 / FP32 FMA lanes per SM per clock: GB300 is specified at 1.25 TFLOP/s FP64
 # (2 lanes/clk/SM at 2.07 GHz over 152 SMs) and 128 FP32 lanes/clk/SM.
 FMA_LANES = {"f64": 2, "f32": 128}
+# df64 (double-float) arithmetic runs on the FP32 pipe; one df64 FMA is 12 FP32 instructions
+# (FMUL, 3 FFMA for the exact product and the cross terms, 8 FADD for the exact sum and the lows).
+DF64_OPS_PER_FMA = 12
 # algorithmic FMAs per valid neighbour x channel
 FMA_PER_EVAL = {"fwd": 9, "grad": 18}
 DESC_FMA_PER_ATOM = lambda M1, M2: 4 * M1 * M2  # noqa: E731
@@ -102,7 +105,18 @@ PROFILED_DRAM_BYTES = {}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
+    """FMA-pipe peak in TFLOP/s (an FMA = 2 flop); for df64 the FP32 pipe's rate of df64 FMAs."""
+    if dtype == "df64":
+        return NSM * FMA_LANES["f32"] * 2 * mhz * 1e6 / 1e12 / DF64_OPS_PER_FMA
     return NSM * FMA_LANES[dtype] * 2 * mhz * 1e6 / 1e12
+
+
+def peak_basis(dtype: str) -> str:
+    if dtype == "df64":
+        return (f"FP32 pipe: {NSM} SMs x {FMA_LANES['f32']} lanes/clk x {SM_MAX_MHZ:.0f} MHz / "
+                f"{DF64_OPS_PER_FMA} FP32 instructions per df64 FMA, x 2 flop")
+    return (f"FP{64 if dtype == 'f64' else 32} FMA pipe: {NSM} SMs x {FMA_LANES[dtype]} lanes/clk x 2 flop x "
+            f"{SM_MAX_MHZ:.0f} MHz")
 
 
 def rank_seed(seed: int, rank: int) -> int:
@@ -212,6 +226,7 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     import workloads as W
     fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
     grad = dpc.dp_tabulate_fusion_grad_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_grad
+    arith = dpc.DF64 if args.dtype == "df64" else None  # the table picks the fusion kernels' arithmetic
     T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
     D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
     ds = torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev)
@@ -227,7 +242,7 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
             rec(0)
             fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
             rec(1)
-            dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"])
+            dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"], arith=arith)
             rec(2)
             grad(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, x["dT"], out=(o["ds"], o["dRt"]))
             rec(3)
@@ -254,9 +269,9 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
         rec(1)
         fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
         rec(2)
-        dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"])
+        dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"], arith=arith)
         rec(3)
-        dpc.dp_descriptor_contract_grad(work["T"], x["dD"], out=work["dT"])
+        dpc.dp_descriptor_contract_grad(work["T"], x["dD"], out=work["dT"], arith=arith)
         rec(4)
         grad(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, work["dT"],
              out=(work["ds"], work["dRt"]))
@@ -273,8 +288,8 @@ def run_native(args, rank, world, local_rank):
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
-    dtype = torch.float64 if args.dtype == "f64" else torch.float32
-    npdt = np.float64 if args.dtype == "f64" else np.float32
+    dtype = torch.float32 if args.dtype == "f32" else torch.float64
+    npdt = np.float32 if args.dtype == "f32" else np.float64
     kw = {}
     if args.workload == "alcumg":
         kw["pad"] = args.pad
@@ -282,7 +297,8 @@ def run_native(args, rank, world, local_rank):
     if args.chain and w.env is None:
         raise SystemExit(f"--chain needs positions and a neighbour list; workload {w.name} has none")
     info = dpc.dp_table_info_make(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
-    model = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, dtype)
+    model = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info,
+                               dpc.DF64 if args.dtype == "df64" else dtype)
     sel = [int(x) for x in w.sel]
     host, d, outs, names, step = build_step(args, w, dpc, model, info, sel, dtype, npdt, dev)
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)  # 256 MiB > 126 MiB L2
@@ -403,7 +419,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     flops = {"fwd": 2.0 * fmas["fwd"], "grad": 2.0 * fmas["grad"],
              "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc,
              "descriptor_grad": 2.0 * DESC_GRAD_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
-    nbytes = chain_bytes(w, 8 if args.dtype == "f64" else 4, nall) if args.chain else {}
+    nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
     pk = peak_tflops(args.dtype)
     kernels = {}
     for k in mean:
@@ -420,8 +436,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
                 "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
                 "kernel": f"dp_tabulate_fusion_{dom}",
-                "peak_basis": (f"FP{64 if args.dtype == 'f64' else 32} FMA pipe: {NSM} SMs x "
-                               f"{FMA_LANES[args.dtype]} lanes/clk x 2 flop x {SM_MAX_MHZ:.0f} MHz"),
+                "peak_basis": peak_basis(args.dtype),
                 "fwd_grad_frac": round(path_tflops / pk, 4)}
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -556,7 +571,8 @@ def main():
     ap.add_argument("--impl", choices=["native", "reference"], default="native")
     ap.add_argument("--workload", default="cu85", choices=["tiny", "cu85", "cugeo", "water", "alcumg", "water_large"])
     ap.add_argument("--pad", type=float, default=0.3, help="alcumg padding fraction")
-    ap.add_argument("--dtype", choices=["f64", "f32"], default="f64")
+    ap.add_argument("--dtype", choices=["f64", "f32", "df64"], default="f64",
+                    help="df64: f64 arrays, double-float arithmetic on the FP32 pipes (moment path)")
     ap.add_argument("--seed", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
@@ -570,6 +586,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.dtype == "df64" and args.algo != "moments":
+        ap.error("--dtype df64 runs the moment path only")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

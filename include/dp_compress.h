@@ -238,8 +238,9 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  * rows, D_i = S_i (S_i^<)^T, i.e. D[i][m][n] = sum_k T[i][k][m] * T[i][k][n].
  *   T [nloc][4][M1] input,  D [nloc][M1][M2] output.
  * Errors: DP_ERR_NULL, DP_ERR_SHAPE (nloc < 0, M1 < 1, M2 < 1, M2 > M1),
- * DP_ERR_UNSUPPORTED (M1 > 4096), DP_ERR_CUDA.  nloc == 0 returns DP_OK
- * without reading T or D.
+ * DP_ERR_UNSUPPORTED (M1 > 4096, or T_i of four atoms not fitting in 227 KB
+ * of shared memory: M1 > 1816 in f64, 3632 in f32), DP_ERR_CUDA.  nloc == 0
+ * returns DP_OK without reading T or D.
  */
 int dp_descriptor_contract_f64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream);
 int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, float *D, void *stream);
@@ -251,12 +252,50 @@ int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, flo
  *   dT[i][k][m] = sum_{n<M2} dD[i][m][n] T[i][k][n] + [m < M2] sum_{m'} dD[i][m'][m] T[i][k][m']
  *   T [nloc][4][M1], dD [nloc][M1][M2] inputs;  dT [nloc][4][M1] output, fully
  *   overwritten (feed it to dp_tabulate_fusion_grad_*).
- * Errors, limits and the nloc == 0 rule as dp_descriptor_contract_*.
+ * Errors, limits and the nloc == 0 rule as dp_descriptor_contract_*; the
+ * backward stages T_i and dT_i (M1 > 908 in f64, 1816 in f32 is
+ * DP_ERR_UNSUPPORTED).
  */
 int dp_descriptor_contract_grad_f64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,
                                     void *stream);
 int dp_descriptor_contract_grad_f32(const float *T, const float *dD, int64_t nloc, int M1, int M2, float *dT,
                                     void *stream);
+
+/* ------------------------------------------------------------------------
+ * df64 variant: double inputs and outputs, double-float arithmetic.
+ *
+ * The same operations as the *_f64 calls above (Sec. II; same arguments,
+ * layouts, limits, errors and nloc == 0 rule), computed in double-float
+ * ("df64") arithmetic: every intermediate is the unevaluated sum of two
+ * floats (48 significant bits), multiplied and accumulated through
+ * error-free transformations on the FP32 pipes, which on GB300 retire 64
+ * times the FP64 pipe's lanes per clock.  s, R~, dE/dT, dE/dD, T, D, ds and
+ * dR~ are double arrays as in the *_f64 calls; results agree with them to a
+ * few 1e-13 (max-norm relative on the paper's shapes; the rounding of df64
+ * is 2^-48 per operation against 2^-53 in double).  Values must lie within
+ * float's exponent range: magnitudes below ~1e-38 (relative parts below
+ * ~1e-38 / 2^-24) flush towards zero, above ~3e38 overflow.
+ *
+ * dp_descriptor_contract_grad_df64 also stages dD_i: it needs
+ * M1 (8 + M2) <= 7264 (DP_ERR_UNSUPPORTED beyond).
+ *
+ * The table is built for this arithmetic: [npair][nint][3][M1][4] float,
+ * per interval the (a.hi, a.lo, b.hi, b.lo) vectors of all channels, then
+ * (c, d), then (e, f) -- each coefficient of dp_table_build_f64 split into a
+ * float and the float rounding of its remainder.
+ * ---------------------------------------------------------------------- */
+int dp_table_build_df64(const double *y, const double *dy, const double *d2y, int npair, int M1,
+                        const dp_table_info *info, float *table, void *stream);
+int dp_tabulate_fusion_fwd_moments_df64(const float *table, const dp_table_info *info, const double *s,
+                                        const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                        int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *stream);
+int dp_tabulate_fusion_grad_moments_df64(const float *table, const dp_table_info *info, const double *s,
+                                         const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                         int nnei, int ntypes, const int32_t *sel, int M1, const double *dT,
+                                         double *ds, double *dRt, void *stream);
+int dp_descriptor_contract_df64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream);
+int dp_descriptor_contract_grad_df64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,
+                                     void *stream);
 
 /* ------------------------------------------------------------------------
  * Environment matrix front end and force / virial back end (Sec. II: the

@@ -101,6 +101,13 @@ _SIGS = {
     "dp_descriptor_contract_f32": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_grad_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_grad_f32": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_table_build_df64": ([_P, _P, _P, ctypes.c_int, ctypes.c_int, _INFO, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_moments_df64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                             ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_moments_df64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
+    "dp_descriptor_contract_df64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_descriptor_contract_grad_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
 }
 for _name, (_args, _res) in _SIGS.items():
     _fn = getattr(_lib, _name)
@@ -137,12 +144,23 @@ def _dev(t: torch.Tensor, name: str, dtype=None, shape=None):
     return t
 
 
+# Arithmetic "df64": double arrays, double-float arithmetic; its table is float [npair][nint][3][M1][4].
+DF64 = "df64"
+
+
 def _suffix(dtype) -> str:
     if dtype == torch.float64:
         return "f64"
     if dtype == torch.float32:
         return "f32"
+    if dtype == DF64:
+        return "df64"
     raise TypeError(f"unsupported dtype {dtype}")
+
+
+def is_df64_table(table: torch.Tensor) -> bool:
+    """A table from dp_table_build(..., dtype="df64"): float, (hi, lo) pairs in a last dimension of 4."""
+    return table.dtype == torch.float32 and table.dim() == 5 and table.shape[-1] == 4
 
 
 def dp_table_info_make(s_min: float, s_max: float, stride0: float = 0.01, stride1: float = 0.1,
@@ -175,13 +193,15 @@ def dp_embedding_net_nodes(params: torch.Tensor, widths, info: dp_table_info, ou
 
 
 def dp_table_build(y, dy, d2y, info: dp_table_info, dtype=torch.float64, out=None) -> torch.Tensor:
-    """Quintic coefficient table [npair][nint][3][M1][2] (pair-planar a..f) in `dtype` from f64 node values."""
+    """Quintic coefficient table [npair][nint][3][M1][2] (pair-planar a..f) in `dtype` from f64 node values;
+    dtype="df64": float [npair][nint][3][M1][4], each coefficient as a (hi, lo) float pair."""
     y = _dev(y, "y", torch.float64)
     npair, nn, M1 = (int(x) for x in y.shape)
     dy = _dev(dy, "dy", torch.float64, y.shape)
     d2y = _dev(d2y, "d2y", torch.float64, y.shape)
-    shape = (npair, nn - 1, 3, M1, 2)
-    table = torch.empty(shape, dtype=dtype, device=y.device) if out is None else _dev(out, "out", dtype, shape)
+    shape = (npair, nn - 1, 3, M1, 4 if dtype == DF64 else 2)
+    tdt = torch.float32 if dtype == DF64 else dtype
+    table = torch.empty(shape, dtype=tdt, device=y.device) if out is None else _dev(out, "out", tdt, shape)
     fn = getattr(_lib, f"dp_table_build_{_suffix(dtype)}")
     _check(fn(_ptr(y), _ptr(dy), _ptr(d2y), npair, M1, ctypes.byref(info), _ptr(table), _stream(y)))
     return table
@@ -193,8 +213,9 @@ def _sel_arr(sel):
 
 
 def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
-    dtype = table.dtype
-    table = _dev(table, "table", dtype)
+    df = isinstance(table, torch.Tensor) and is_df64_table(table)
+    table = _dev(table, "table", None)
+    dtype = torch.float64 if df else table.dtype
     s = _dev(s, "s", dtype)
     nloc, nnei = (int(x) for x in s.shape)
     Rt = _dev(Rt, "Rt", dtype, (nloc, nnei, 4))
@@ -205,10 +226,10 @@ def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
         nvalid = _dev(nvalid, "nvalid", torch.int32, (nloc, ntypes))
     if atype is not None:
         atype = _dev(atype, "atype", torch.int32, (nloc,))
-    if table.dim() != 5 or table.shape[-3] != 3 or table.shape[-1] != 2:
-        raise ValueError("table must be [npair][nint][3][M1][2] (from dp_table_build)")
+    if table.dim() != 5 or table.shape[-3] != 3 or table.shape[-1] != (4 if df else 2):
+        raise ValueError("table must be [npair][nint][3][M1][2] (or [..][4] for df64) from dp_table_build")
     M1 = int(table.shape[-2])
-    return dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1
+    return dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, (DF64 if df else dtype)
 
 
 def dp_tabulate_fusion_fwd(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None) -> torch.Tensor:
@@ -221,12 +242,21 @@ def dp_tabulate_fusion_fwd_moments(table, info: dp_table_info, s, Rt, nvalid, at
     return _fwd("dp_tabulate_fusion_fwd_moments", table, info, s, Rt, nvalid, atype, sel, out)
 
 
+def dp_tabulate_fusion_fwd_moments_df64(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None):
+    """T of dp_tabulate_fusion_fwd_moments in df64 arithmetic: f64 s, Rt and T, a df64 table."""
+    if not is_df64_table(table):
+        raise TypeError("table must come from dp_table_build(..., dtype='df64')")
+    return _fwd("dp_tabulate_fusion_fwd_moments", table, info, s, Rt, nvalid, atype, sel, out)
+
+
 def _fwd(name, table, info, s, Rt, nvalid, atype, sel, out):
-    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
-                                                                                      sel)
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, arith = _fusion_inputs(table, s, Rt, nvalid,
+                                                                                             atype, sel)
+    if arith == DF64 and not name.endswith("_moments"):
+        raise TypeError(f"{name} has no df64 form; use the _moments call")
     shape = (nloc, 4, M1)
     T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
-    fn = getattr(_lib, f"{name}_{_suffix(dtype)}")
+    fn = getattr(_lib, f"{name}_{_suffix(arith)}")
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(T), _stream(s)))
     return T
@@ -234,8 +264,10 @@ def _fwd(name, table, info, s, Rt, nvalid, atype, sel, out):
 
 def dp_tabulate_fusion_fwd_descriptor(table, info: dp_table_info, s, Rt, nvalid, atype, sel, M2: int, out=None):
     """(T [nloc][4][M1], D [nloc][M1][M2]) in one pass: T as dp_tabulate_fusion_fwd, D = S (S^<)^T."""
-    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
-                                                                                      sel)
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, arith = _fusion_inputs(table, s, Rt, nvalid,
+                                                                                             atype, sel)
+    if arith == DF64:
+        raise TypeError("dp_tabulate_fusion_fwd_descriptor has no df64 form")
     if out is None:
         T = torch.empty((nloc, 4, M1), dtype=dtype, device=s.device)
         D = torch.empty((nloc, M1, int(M2)), dtype=dtype, device=s.device)
@@ -258,9 +290,18 @@ def dp_tabulate_fusion_grad_moments(table, info: dp_table_info, s, Rt, nvalid, a
     return _grad("dp_tabulate_fusion_grad_moments", table, info, s, Rt, nvalid, atype, sel, dT, out)
 
 
+def dp_tabulate_fusion_grad_moments_df64(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None):
+    """(ds, dRt) of dp_tabulate_fusion_grad_moments in df64 arithmetic: f64 arrays, a df64 table."""
+    if not is_df64_table(table):
+        raise TypeError("table must come from dp_table_build(..., dtype='df64')")
+    return _grad("dp_tabulate_fusion_grad_moments", table, info, s, Rt, nvalid, atype, sel, dT, out)
+
+
 def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
-    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1 = _fusion_inputs(table, s, Rt, nvalid, atype,
-                                                                                      sel)
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, arith = _fusion_inputs(table, s, Rt, nvalid,
+                                                                                             atype, sel)
+    if arith == DF64 and not name.endswith("_moments"):
+        raise TypeError(f"{name} has no df64 form; use the _moments call")
     dT = _dev(dT, "dT", dtype, (nloc, 4, M1))
     if out is None:
         ds = torch.empty((nloc, nnei), dtype=dtype, device=s.device)
@@ -268,7 +309,7 @@ def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
     else:
         ds = _dev(out[0], "ds", dtype, (nloc, nnei))
         dRt = _dev(out[1], "dRt", dtype, (nloc, nnei, 4))
-    fn = getattr(_lib, f"{name}_{_suffix(dtype)}")
+    fn = getattr(_lib, f"{name}_{_suffix(arith)}")
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(dT), _ptr(ds), _ptr(dRt), _stream(s)))
     return ds, dRt
@@ -322,21 +363,23 @@ def dp_force_virial(coord, nlist, env: dp_env_info, ds, dRt, out=None):
     return F, W
 
 
-def dp_descriptor_contract(T, M2: int, out=None) -> torch.Tensor:
-    """D [nloc][M1][M2] = S (S^<)^T with S = T^T."""
+def dp_descriptor_contract(T, M2: int, out=None, arith=None) -> torch.Tensor:
+    """D [nloc][M1][M2] = S (S^<)^T with S = T^T (arith="df64": f64 arrays, df64 arithmetic)."""
     T = _dev(T, "T", None)
     nloc, four, M1 = (int(x) for x in T.shape)
     if four != 4:
         raise ValueError("T must be [nloc][4][M1]")
     shape = (nloc, M1, int(M2))
     D = torch.empty(shape, dtype=T.dtype, device=T.device) if out is None else _dev(out, "out", T.dtype, shape)
-    fn = getattr(_lib, f"dp_descriptor_contract_{_suffix(T.dtype)}")
+    if arith == DF64 and T.dtype != torch.float64:
+        raise TypeError("df64 descriptor takes f64 arrays")
+    fn = getattr(_lib, f"dp_descriptor_contract_{_suffix(arith or T.dtype)}")
     _check(fn(_ptr(T), nloc, M1, int(M2), _ptr(D), _stream(T)))
     return D
 
 
-def dp_descriptor_contract_grad(T, dD, out=None) -> torch.Tensor:
-    """dT [nloc][4][M1] = dE/dT from dD = dE/dD [nloc][M1][M2] through D = S (S^<)^T."""
+def dp_descriptor_contract_grad(T, dD, out=None, arith=None) -> torch.Tensor:
+    """dT [nloc][4][M1] = dE/dT from dD = dE/dD [nloc][M1][M2] through D = S (S^<)^T (arith as above)."""
     T = _dev(T, "T", None)
     nloc, four, M1 = (int(x) for x in T.shape)
     if four != 4:
@@ -346,9 +389,26 @@ def dp_descriptor_contract_grad(T, dD, out=None) -> torch.Tensor:
         raise ValueError("dD must be [nloc][M1][M2]")
     M2 = int(dD.shape[2])
     dT = torch.empty_like(T) if out is None else _dev(out, "out", T.dtype, T.shape)
-    fn = getattr(_lib, f"dp_descriptor_contract_grad_{_suffix(T.dtype)}")
+    if arith == DF64 and T.dtype != torch.float64:
+        raise TypeError("df64 descriptor backward takes f64 arrays")
+    fn = getattr(_lib, f"dp_descriptor_contract_grad_{_suffix(arith or T.dtype)}")
     _check(fn(_ptr(T), _ptr(dD), nloc, M1, M2, _ptr(dT), _stream(T)))
     return dT
+
+
+def dp_descriptor_contract_df64(T, M2: int, out=None) -> torch.Tensor:
+    """dp_descriptor_contract in df64 arithmetic (f64 T and D)."""
+    return dp_descriptor_contract(T, M2, out, arith=DF64)
+
+
+def dp_descriptor_contract_grad_df64(T, dD, out=None) -> torch.Tensor:
+    """dp_descriptor_contract_grad in df64 arithmetic (f64 T, dD and dT)."""
+    return dp_descriptor_contract_grad(T, dD, out, arith=DF64)
+
+
+def dp_table_build_df64(y, dy, d2y, info: dp_table_info, out=None) -> torch.Tensor:
+    """dp_table_build(..., dtype="df64")."""
+    return dp_table_build(y, dy, d2y, info, DF64, out)
 
 
 @dataclass

@@ -5,6 +5,7 @@
 // output tile is contiguous, so lane l computes elements l, l + 32, ... of it
 // in storage order: every FP64 instruction has 32 busy lanes (M1*M2 is a
 // multiple of 32 for the paper's shapes) and every store is coalesced.
+// Both kernels also run in df64 arithmetic on double arrays (io_t).
 #include "dp_common.cuh"
 
 namespace dpc {
@@ -15,16 +16,16 @@ constexpr int kDescWarps = 4;
 
 template <typename real>
 __global__ void __launch_bounds__(kDescWarps * 32)
-    descriptor_kernel(const real *__restrict__ T, int64_t nloc, int M1, int M2, real *__restrict__ D) {
+    descriptor_kernel(const io_t<real> *__restrict__ T, int64_t nloc, int M1, int M2, io_t<real> *__restrict__ D) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t i = (int64_t)blockIdx.x * kDescWarps + w;
   if (i >= nloc) return;  // warp-uniform; no block-wide barrier below
   real *Ts = reinterpret_cast<real *>(smem_raw) + (size_t)w * 4 * M1;
-  const real *__restrict__ Ti = T + i * 4 * M1;
-  for (int e = lane; e < 4 * M1; e += 32) Ts[e] = __ldg(Ti + e);
+  const io_t<real> *__restrict__ Ti = T + i * 4 * M1;
+  for (int e = lane; e < 4 * M1; e += 32) Ts[e] = from_io<real>(__ldg(Ti + e));
   __syncwarp();
-  real *__restrict__ Di = D + i * (int64_t)M1 * M2;
+  io_t<real> *__restrict__ Di = D + i * (int64_t)M1 * M2;
   const int total = M1 * M2;
   int m = lane / M2, n = lane - m * M2;
   const int dm = 32 / M2, dn = 32 - dm * M2;  // advance of (m, n) per 32 elements
@@ -33,7 +34,7 @@ __global__ void __launch_bounds__(kDescWarps * 32)
     v = fma(Ts[M1 + m], Ts[M1 + n], v);
     v = fma(Ts[2 * M1 + m], Ts[2 * M1 + n], v);
     v = fma(Ts[3 * M1 + m], Ts[3 * M1 + n], v);
-    Di[e] = v;
+    Di[e] = to_io(v);
     m += dm;
     n += dn;
     if (n >= M2) {
@@ -41,6 +42,13 @@ __global__ void __launch_bounds__(kDescWarps * 32)
       ++m;
     }
   }
+}
+
+// Shared memory per warp of the descriptor backward, in elements: T_i and the partial dT_i
+// ([4][M1] each), and in df64 also dD_i ([M1][M2]).
+template <typename real>
+__host__ __device__ constexpr size_t desc_grad_smem_per_warp(int M1, int M2) {
+  return (size_t)8 * M1 + (is_df64<real> ? (size_t)M1 * M2 : 0);
 }
 
 // Backward of the descriptor: D[m][n] = sum_k T[k][m] T[k][n] (n < M2) is
@@ -53,25 +61,34 @@ __global__ void __launch_bounds__(kDescWarps * 32)
 // terms meet in shared memory and dT is written coalesced.
 template <typename real>
 __global__ void __launch_bounds__(kDescWarps * 32)
-    descriptor_grad_kernel(const real *__restrict__ T, const real *__restrict__ dD, int64_t nloc, int M1, int M2,
-                           real *__restrict__ dT) {
+    descriptor_grad_kernel(const io_t<real> *__restrict__ T, const io_t<real> *__restrict__ dD, int64_t nloc, int M1,
+                           int M2, io_t<real> *__restrict__ dT) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t i = (int64_t)blockIdx.x * kDescWarps + w;
   if (i >= nloc) return;  // warp-uniform; no block-wide barrier below
-  real *Ts = reinterpret_cast<real *>(smem_raw) + (size_t)w * 8 * M1;  // [4][M1]
-  real *Gs = Ts + 4 * M1;                                              // [4][M1] partial dT
-  const real *__restrict__ Ti = T + i * 4 * M1;
-  const real *__restrict__ Di = dD + i * (int64_t)M1 * M2;
-  for (int e = lane; e < 4 * M1; e += 32) Ts[e] = __ldg(Ti + e);
+  real *Ts = reinterpret_cast<real *>(smem_raw) + (size_t)w * desc_grad_smem_per_warp<real>(M1, M2);  // [4][M1]
+  real *Gs = Ts + 4 * M1;                                                                              // [4][M1]
+  const io_t<real> *__restrict__ Ti = T + i * 4 * M1;
+  const io_t<real> *__restrict__ Di = dD + i * (int64_t)M1 * M2;
+  for (int e = lane; e < 4 * M1; e += 32) Ts[e] = from_io<real>(__ldg(Ti + e));
+  // df64: dD_i converted once into shared memory ([M1][M2] after Gs); every element is read 8 times
+  const real *Ds = Gs + 4 * M1;
+  if constexpr (is_df64<real>) {
+    real *Dw = Gs + 4 * M1;
+    for (int e = lane; e < M1 * M2; e += 32) Dw[e] = from_io<real>(__ldg(Di + e));
+  }
   __syncwarp();
+  auto dd = [&](int e) -> real {
+    if constexpr (is_df64<real>) return Ds[e];
+    else return __ldg(Di + e);
+  };
   // first term, pairs p = 4 m + k
   for (int p = lane; p < 4 * M1; p += 32) {
     const int m = p >> 2, k = p & 3;
-    const real *__restrict__ row = Di + (size_t)m * M2;
     const real *tk = Ts + k * M1;
     real v = real(0);
-    for (int n = 0; n < M2; ++n) v = fma(__ldg(row + n), tk[n], v);
+    for (int n = 0; n < M2; ++n) v = fma(dd(m * M2 + n), tk[n], v);
     Gs[k * M1 + m] = v;
   }
   __syncwarp();
@@ -80,16 +97,17 @@ __global__ void __launch_bounds__(kDescWarps * 32)
     const int k = p / M2, m = p - k * M2;
     const real *tk = Ts + k * M1;
     real v = real(0);
-    for (int mp = 0; mp < M1; ++mp) v = fma(__ldg(Di + (size_t)mp * M2 + m), tk[mp], v);
+    for (int mp = 0; mp < M1; ++mp) v = fma(dd(mp * M2 + m), tk[mp], v);
     Gs[k * M1 + m] += v;
   }
   __syncwarp();
-  real *__restrict__ dTi = dT + i * 4 * M1;
-  for (int e = lane; e < 4 * M1; e += 32) dTi[e] = Gs[e];
+  io_t<real> *__restrict__ dTi = dT + i * 4 * M1;
+  for (int e = lane; e < 4 * M1; e += 32) dTi[e] = to_io(Gs[e]);
 }
 
 template <typename real>
-int descriptor_grad(const real *T, const real *dD, int64_t nloc, int M1, int M2, real *dT, void *stream) {
+int descriptor_grad(const io_t<real> *T, const io_t<real> *dD, int64_t nloc, int M1, int M2, io_t<real> *dT,
+                    void *stream) {
   clear_error();
   if (nloc < 0 || M1 < 1 || M2 < 1 || M2 > M1)
     return set_error(DP_ERR_SHAPE, "need nloc >= 0 and 1 <= M2 <= M1 (nloc %lld, M1 %d, M2 %d)", (long long)nloc, M1,
@@ -99,7 +117,8 @@ int descriptor_grad(const real *T, const real *dD, int64_t nloc, int M1, int M2,
   if (!T || !dD || !dT) return set_error(DP_ERR_NULL, "T, dD or dT is NULL");
   const int64_t blocks = (nloc + kDescWarps - 1) / kDescWarps;
   if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
-  const size_t smem = (size_t)kDescWarps * 8 * M1 * sizeof(real);
+  const size_t smem = (size_t)kDescWarps * desc_grad_smem_per_warp<real>(M1, M2) * sizeof(real);
+  if (smem > 227 * 1024) return set_error(DP_ERR_UNSUPPORTED, "M1 = %d, M2 = %d need too much shared memory", M1, M2);
   if (smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(descriptor_grad_kernel<real>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -111,7 +130,7 @@ int descriptor_grad(const real *T, const real *dD, int64_t nloc, int M1, int M2,
 }
 
 template <typename real>
-int descriptor(const real *T, int64_t nloc, int M1, int M2, real *D, void *stream) {
+int descriptor(const io_t<real> *T, int64_t nloc, int M1, int M2, io_t<real> *D, void *stream) {
   clear_error();
   if (nloc < 0 || M1 < 1 || M2 < 1 || M2 > M1)
     return set_error(DP_ERR_SHAPE, "need nloc >= 0 and 1 <= M2 <= M1 (nloc %lld, M1 %d, M2 %d)", (long long)nloc, M1,
@@ -122,6 +141,7 @@ int descriptor(const real *T, int64_t nloc, int M1, int M2, real *D, void *strea
   const int64_t blocks = (nloc + kDescWarps - 1) / kDescWarps;
   if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
   const size_t smem = (size_t)kDescWarps * 4 * M1 * sizeof(real);
+  if (smem > 227 * 1024) return set_error(DP_ERR_UNSUPPORTED, "M1 = %d needs too much shared memory", M1);
   if (smem > 48 * 1024) {
     const cudaError_t e = cudaFuncSetAttribute(descriptor_kernel<real>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                (int)smem);
@@ -143,6 +163,15 @@ int dp_descriptor_contract_f64(const double *T, int64_t nloc, int M1, int M2, do
 
 int dp_descriptor_contract_f32(const float *T, int64_t nloc, int M1, int M2, float *D, void *stream) {
   return dpc::descriptor<float>(T, nloc, M1, M2, D, stream);
+}
+
+int dp_descriptor_contract_df64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream) {
+  return dpc::descriptor<dpc::df64>(T, nloc, M1, M2, D, stream);
+}
+
+int dp_descriptor_contract_grad_df64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,
+                                     void *stream) {
+  return dpc::descriptor_grad<dpc::df64>(T, dD, nloc, M1, M2, dT, stream);
 }
 
 int dp_descriptor_contract_grad_f64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,

@@ -8,8 +8,11 @@
 #include <cstdint>
 
 #include "dp_compress.h"
+#include "dp_df64.cuh"
 
 namespace dpc {
+
+using dfl::df64;
 
 // ---------------------------------------------------------------- errors
 int set_error(int code, const char *fmt, ...);  // stores the message, returns code
@@ -126,7 +129,16 @@ __device__ __forceinline__ int locate(const TableGeomF &g, float s, float &t, bo
   return 0;
 }
 
-// Geometry type used by the kernels of each precision.
+// df64 kernels search in double (one search per neighbour row, off the FP32
+// pipes that carry their arithmetic) and split t into a df64.
+__device__ __forceinline__ int locate(const TableGeom &g, double s, df64 &t, bool &clamped) {
+  double td;
+  const int l = locate(g, s, td, clamped);
+  t = dfl::split(td);
+  return l;
+}
+
+// Geometry type used by the kernels of each arithmetic.
 template <typename real> struct GeomOf;
 template <> struct GeomOf<double> {
   using type = TableGeom;
@@ -136,6 +148,55 @@ template <> struct GeomOf<float> {
   using type = TableGeomF;
   static TableGeomF make(const TableGeom &g) { return to_f32(g); }
 };
+template <> struct GeomOf<df64> {
+  using type = TableGeom;
+  static TableGeom make(const TableGeom &g) { return g; }
+};
+
+// Element type of the arrays a kernel of arithmetic `real` reads and writes
+// (s, R~, dE/dT, T, ds, dR~): the arithmetic type itself, except df64
+// kernels, which take and return double.  Tables are stored in the
+// arithmetic type (a df64 table holds (hi, lo) float pairs).
+template <typename real> constexpr bool is_df64 = false;
+template <> constexpr bool is_df64<df64> = true;
+
+template <typename real> struct IoOf { using type = real; };
+template <> struct IoOf<df64> { using type = double; };
+template <typename real>
+using io_t = typename IoOf<real>::type;
+
+__device__ __forceinline__ double to_io(const double x) { return x; }
+__device__ __forceinline__ float to_io(const float x) { return x; }
+__device__ __forceinline__ double to_io(const df64 x) { return dfl::join(x); }
+
+template <typename real>
+__device__ __forceinline__ real from_io(const io_t<real> x) { return x; }
+template <>
+__device__ __forceinline__ df64 from_io<df64>(const double x) { return dfl::split(x); }
+
+// A double in the arithmetic type, on the device (table coefficients).
+template <typename real>
+__device__ __forceinline__ real dcvt(const double x) { return (real)x; }
+template <>
+__device__ __forceinline__ df64 dcvt<df64>(const double x) { return dfl::from_double(x); }
+
+// A host-side double in the arithmetic type (kernel parameters).
+template <typename real>
+inline real host_cvt(const double x) { return (real)x; }
+template <>
+inline df64 host_cvt<df64>(const double x) { return dfl::from_double(x); }
+
+// Warp shuffles of one value of any arithmetic type (a df64 moves as two floats).
+__device__ __forceinline__ double shfl(const double v, const int src) { return __shfl_sync(0xffffffffu, v, src); }
+__device__ __forceinline__ float shfl(const float v, const int src) { return __shfl_sync(0xffffffffu, v, src); }
+__device__ __forceinline__ df64 shfl(const df64 v, const int src) {
+  return df64(__shfl_sync(0xffffffffu, v.hi, src), __shfl_sync(0xffffffffu, v.lo, src));
+}
+__device__ __forceinline__ double shfl_xor(const double v, const int m) { return __shfl_xor_sync(0xffffffffu, v, m); }
+__device__ __forceinline__ float shfl_xor(const float v, const int m) { return __shfl_xor_sync(0xffffffffu, v, m); }
+__device__ __forceinline__ df64 shfl_xor(const df64 v, const int m) {
+  return df64(__shfl_xor_sync(0xffffffffu, v.hi, m), __shfl_xor_sync(0xffffffffu, v.lo, m));
+}
 
 // ------------------------------------------------------- vector helpers
 template <typename real> struct Vec4;
@@ -144,6 +205,9 @@ template <> struct Vec4<double> {
 };
 template <> struct Vec4<float> {
   float x, y, z, w;
+};
+template <> struct Vec4<df64> {
+  df64 x, y, z, w;
 };
 
 // Four consecutive values (an environment-matrix row, a dT column).
@@ -155,6 +219,14 @@ __device__ __forceinline__ Vec4<double> ld4(const double *p) {
 __device__ __forceinline__ Vec4<float> ld4(const float *p) {
   const float4 a = __ldg(reinterpret_cast<const float4 *>(p));
   return {a.x, a.y, a.z, a.w};
+}
+// Four consecutive I/O values in the arithmetic type `real`.
+template <typename real>
+__device__ __forceinline__ Vec4<real> ld4r(const io_t<real> *p) { return ld4(p); }
+template <>
+__device__ __forceinline__ Vec4<df64> ld4r<df64>(const double *p) {
+  const Vec4<double> v = ld4(p);
+  return {dfl::split(v.x), dfl::split(v.y), dfl::split(v.z), dfl::split(v.w)};
 }
 
 // The six coefficients (a, b, c, d, e, f) of channel m of one interval.  An
@@ -173,12 +245,23 @@ __device__ __forceinline__ void ld6(const float *blk, int M1, int m, float c[6])
   c[0] = x.x; c[1] = x.y; c[2] = y.x; c[3] = y.y; c[4] = z.x; c[5] = z.y;
 }
 
+// df64 table: the (a, b) pair of a channel is one 16-byte (a.hi, a.lo, b.hi, b.lo) vector.
+__device__ __forceinline__ void ld6(const df64 *blk, int M1, int m, df64 c[6]) {
+  const float4 *q = reinterpret_cast<const float4 *>(blk) + m;
+  const float4 x = __ldg(q), y = __ldg(q + M1), z = __ldg(q + 2 * M1);
+  c[0] = df64(x.x, x.y); c[1] = df64(x.z, x.w); c[2] = df64(y.x, y.y);
+  c[3] = df64(y.z, y.w); c[4] = df64(z.x, z.y); c[5] = df64(z.z, z.w);
+}
+
 __device__ __forceinline__ void st4(double *p, double a, double b, double c, double d) {
   reinterpret_cast<double2 *>(p)[0] = make_double2(a, b);
   reinterpret_cast<double2 *>(p)[1] = make_double2(c, d);
 }
 __device__ __forceinline__ void st4(float *p, float a, float b, float c, float d) {
   *reinterpret_cast<float4 *>(p) = make_float4(a, b, c, d);
+}
+__device__ __forceinline__ void st4(double *p, df64 a, df64 b, df64 c, df64 d) {
+  st4(p, to_io(a), to_io(b), to_io(c), to_io(d));
 }
 
 __device__ __forceinline__ int clampi(int x, int lo, int hi) { return min(max(x, lo), hi); }

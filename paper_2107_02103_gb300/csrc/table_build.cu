@@ -154,12 +154,12 @@ __global__ void __launch_bounds__(kBuildThreads)
   const double Dt3 = Dt * Dt * Dt, Dt4 = Dt3 * Dt, Dt5 = Dt4 * Dt;
   // pair-planar block of interval (p, l): [3][M1][2] = (a, b), (c, d), (e, f) planes
   real *blk = table + (size_t)pl * 6 * M1 + 2 * m;
-  blk[0] = (real)(dd_val(ba) / (2.0 * Dt5));
-  blk[1] = (real)(dd_val(bb) / (2.0 * Dt4));
-  blk[2 * M1] = (real)(dd_val(bc) / (2.0 * Dt3));
-  blk[2 * M1 + 1] = (real)(0.5 * q0);
-  blk[4 * M1] = (real)p0;
-  blk[4 * M1 + 1] = (real)y0;
+  blk[0] = dcvt<real>(dd_val(ba) / (2.0 * Dt5));
+  blk[1] = dcvt<real>(dd_val(bb) / (2.0 * Dt4));
+  blk[2 * M1] = dcvt<real>(dd_val(bc) / (2.0 * Dt3));
+  blk[2 * M1 + 1] = dcvt<real>(0.5 * q0);
+  blk[4 * M1] = dcvt<real>(p0);
+  blk[4 * M1 + 1] = dcvt<real>(y0);
 }
 
 template <typename real>
@@ -228,6 +228,11 @@ int dp_table_build_f64(const double *y, const double *dy, const double *d2y, int
 int dp_table_build_f32(const double *y, const double *dy, const double *d2y, int npair, int M1,
                        const dp_table_info *info, float *table, void *stream) {
   return dpc::table_build<float>(y, dy, d2y, npair, M1, info, table, stream);
+}
+
+int dp_table_build_df64(const double *y, const double *dy, const double *d2y, int npair, int M1,
+                        const dp_table_info *info, float *table, void *stream) {
+  return dpc::table_build<dpc::df64>(y, dy, d2y, npair, M1, info, reinterpret_cast<dpc::df64 *>(table), stream);
 }
 
 }  // extern "C"

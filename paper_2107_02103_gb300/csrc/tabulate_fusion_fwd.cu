@@ -21,6 +21,9 @@
 //     1/32 of an instruction per neighbour.
 //   * one warp per block and per atom keeps the work units small, so the
 //     block scheduler balances the SMs to within a few atoms.
+// The same kernels run in df64 (double-float) arithmetic on the FP32 pipes
+// for double inputs and outputs: the templates are written against the
+// arithmetic type `real` and read / write arrays of io_t<real>.
 // The packed round's partial sums meet in a shuffle reduction over the PK
 // lanes of each remainder channel, once per atom.  In f32 the coefficient
 // row of the current interval is also kept in registers across consecutive
@@ -40,12 +43,12 @@ constexpr int kFwdWarps = 1;
 template <typename real>
 struct FwdParams {
   const real *__restrict__ table;
-  const real *__restrict__ s;
-  const real *__restrict__ Rt;
+  const io_t<real> *__restrict__ s;
+  const io_t<real> *__restrict__ Rt;
   const int32_t *__restrict__ nvalid;
   const int32_t *__restrict__ atype;
-  real *__restrict__ T;
-  real *__restrict__ D;  // optional fused descriptor output [nloc][M1][M2] (NULL: T only)
+  io_t<real> *__restrict__ T;
+  io_t<real> *__restrict__ D;  // optional fused descriptor output [nloc][M1][M2] (NULL: T only)
   typename GeomOf<real>::type geom;
   int64_t nloc;
   int32_t nnei, ntypes, M1, pair_stride;  // pair_stride = nint * M1 * 6
@@ -155,19 +158,19 @@ __device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, co
                                                    real rq0, real rq1, real rq2, real rq3, const int lane,
                                                    const int64_t i) {
   const int M1 = P.M1, M2 = P.M2;
-  real *__restrict__ Di = P.D + i * (int64_t)M1 * M2;
+  io_t<real> *__restrict__ Di = P.D + i * (int64_t)M1 * M2;
   for (int n = 0; n < M2; ++n) {  // uniform
     real t0, t1, t2, t3;
     if (Q > 0) {
-      t0 = __shfl_sync(0xffffffffu, acc[0][0], n);
-      t1 = __shfl_sync(0xffffffffu, acc[0][1], n);
-      t2 = __shfl_sync(0xffffffffu, acc[0][2], n);
-      t3 = __shfl_sync(0xffffffffu, acc[0][3], n);
+      t0 = shfl(acc[0][0], n);
+      t1 = shfl(acc[0][1], n);
+      t2 = shfl(acc[0][2], n);
+      t3 = shfl(acc[0][3], n);
     } else {
-      t0 = __shfl_sync(0xffffffffu, rq0, n);
-      t1 = __shfl_sync(0xffffffffu, rq1, n);
-      t2 = __shfl_sync(0xffffffffu, rq2, n);
-      t3 = __shfl_sync(0xffffffffu, rq3, n);
+      t0 = shfl(rq0, n);
+      t1 = shfl(rq1, n);
+      t2 = shfl(rq2, n);
+      t3 = shfl(rq3, n);
     }
 #pragma unroll
     for (int r = 0; r < Q; ++r) {
@@ -175,7 +178,7 @@ __device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, co
       d = fma(acc[r][1], t1, d);
       d = fma(acc[r][2], t2, d);
       d = fma(acc[r][3], t3, d);
-      Di[(size_t)(r * 32 + lane) * M2 + n] = d;
+      Di[(size_t)(r * 32 + lane) * M2 + n] = to_io(d);
     }
   }
   const int npairs = P.RR * M2;
@@ -183,25 +186,25 @@ __device__ __forceinline__ void descriptor_epilogue(const FwdParams<real> &P, co
     const int p = p0 + lane;
     const bool ok = p < npairs;
     const int j = ok ? p / M2 : 0, n = ok ? p - j * M2 : 0;
-    const real a0 = __shfl_sync(0xffffffffu, rq0, j), a1 = __shfl_sync(0xffffffffu, rq1, j);
-    const real a2 = __shfl_sync(0xffffffffu, rq2, j), a3 = __shfl_sync(0xffffffffu, rq3, j);
+    const real a0 = shfl(rq0, j), a1 = shfl(rq1, j);
+    const real a2 = shfl(rq2, j), a3 = shfl(rq3, j);
     real b0, b1, b2, b3;
     if (Q > 0) {
-      b0 = __shfl_sync(0xffffffffu, acc[0][0], n);
-      b1 = __shfl_sync(0xffffffffu, acc[0][1], n);
-      b2 = __shfl_sync(0xffffffffu, acc[0][2], n);
-      b3 = __shfl_sync(0xffffffffu, acc[0][3], n);
+      b0 = shfl(acc[0][0], n);
+      b1 = shfl(acc[0][1], n);
+      b2 = shfl(acc[0][2], n);
+      b3 = shfl(acc[0][3], n);
     } else {
-      b0 = __shfl_sync(0xffffffffu, rq0, n);
-      b1 = __shfl_sync(0xffffffffu, rq1, n);
-      b2 = __shfl_sync(0xffffffffu, rq2, n);
-      b3 = __shfl_sync(0xffffffffu, rq3, n);
+      b0 = shfl(rq0, n);
+      b1 = shfl(rq1, n);
+      b2 = shfl(rq2, n);
+      b3 = shfl(rq3, n);
     }
     real d = a0 * b0;
     d = fma(a1, b1, d);
     d = fma(a2, b2, d);
     d = fma(a3, b3, d);
-    if (ok) Di[(size_t)(Q * 32 + j) * M2 + n] = d;
+    if (ok) Di[(size_t)(Q * 32 + j) * M2 + n] = to_io(d);
   }
 }
 
@@ -233,8 +236,8 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
   for (int q = 0; q < DP_MAX_TYPES; ++q) nv += st.nvb[q];
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   const real *__restrict__ tab = P.table + (size_t)alpha * P.ntypes * P.pair_stride;
-  const real *__restrict__ srow = P.s + i * P.nnei;
-  const real *__restrict__ Rrow = P.Rt + i * P.nnei * 4;
+  const io_t<real> *__restrict__ srow = P.s + i * P.nnei;
+  const io_t<real> *__restrict__ Rrow = P.Rt + i * P.nnei * 4;
 
   // packed-round role of this lane: neighbour slot and remainder channel
   const int rslot = P.RR > 0 ? lane / P.RR : 0;
@@ -314,7 +317,7 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
           off += P.sel[q - 1];
         }
       const int row = off + (v - cum);
-      const Vec4<real> rr = ld4(Rrow + (size_t)row * 4);
+      const Vec4<real> rr = ld4r<real>(Rrow + (size_t)row * 4);
       real t;
       bool clamped;
       const int l = locate(P.geom, __ldg(srow + row), t, clamped);
@@ -339,8 +342,13 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     int nshort = cnt;  // rows whose remainder channels go through the packed per-neighbour round
     if (Q > 0 && kMoments) {
       nshort = 0;
+      // W of a contracted run waiting for its T update (uniform): first the run left open by the
+      // last batch if this batch does not continue it, then each contracted run of this batch.
+      // The update has this one call site, so its (large) code is inlined once.
+      int apply_off = -1;
+      real apply_w = wcarry;
       if (carry_off >= 0 && st.off[0] != carry_off) {  // the open run ended with the last batch
-        apply_moments(carry_off, wcarry);
+        apply_off = carry_off;
         carry_off = -1;
       }
       int next_carry = -1;
@@ -348,7 +356,12 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
       const int myoff = lane < cnt ? st.off[lane] : -1;
       const int prevoff = __shfl_up_sync(0xffffffffu, myoff, 1);
       unsigned starts = __ballot_sync(0xffffffffu, lane < cnt && (lane == 0 || myoff != prevoff));
-      while (starts) {  // uniform, run by run
+      while (starts || apply_off >= 0) {  // uniform, run by run
+        if (apply_off >= 0) {
+          apply_moments(apply_off, apply_w);
+          apply_off = -1;
+          continue;
+        }
         const int u = __ffs(starts) - 1;
         starts &= starts - 1;
         const int e = starts ? __ffs(starts) - 1 : cnt;
@@ -364,7 +377,8 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
             wcarry = wv;
             next_carry = off;
           } else {
-            apply_moments(off, wv);
+            apply_off = off;
+            apply_w = wv;
           }
         } else {
           for (int j = u; j < e; ++j) fwd_neighbour<real, Q>(P, tab, lane, off, st.t[j], st.r[j], acc);
@@ -418,23 +432,23 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
 
   if (Q > 0 && kMoments && npend > 0) flush_remainder();
 
-  real *__restrict__ Ti = P.T + i * 4 * P.M1;
+  io_t<real> *__restrict__ Ti = P.T + i * 4 * P.M1;
 #pragma unroll
   for (int r = 0; r < Q; ++r) {
 #pragma unroll
     for (int k = 0; k < 4; ++k) acc[r][k] *= P.inv_nnei;  // acc now holds T_i
     const int m = r * 32 + lane;
-    Ti[m] = acc[r][0];
-    Ti[P.M1 + m] = acc[r][1];
-    Ti[2 * P.M1 + m] = acc[r][2];
-    Ti[3 * P.M1 + m] = acc[r][3];
+    Ti[m] = to_io(acc[r][0]);
+    Ti[P.M1 + m] = to_io(acc[r][1]);
+    Ti[2 * P.M1 + m] = to_io(acc[r][2]);
+    Ti[3 * P.M1 + m] = to_io(acc[r][3]);
   }
   if (P.RR > 0) {
     // lanes rch, rch + RR, ..., rch + (PK-1) RR hold partial sums of channel 32 Q + rch
     for (int k = 1; k < P.PK; ++k) {
       const int src = lane + k * P.RR;
-      const real x0 = __shfl_sync(0xffffffffu, racc0, src & 31), x1 = __shfl_sync(0xffffffffu, racc1, src & 31);
-      const real x2 = __shfl_sync(0xffffffffu, racc2, src & 31), x3 = __shfl_sync(0xffffffffu, racc3, src & 31);
+      const real x0 = shfl(racc0, src & 31), x1 = shfl(racc1, src & 31);
+      const real x2 = shfl(racc2, src & 31), x3 = shfl(racc3, src & 31);
       if (lane < P.RR) {
         racc0 += x0;
         racc1 += x1;
@@ -448,10 +462,10 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
     racc3 *= P.inv_nnei;
     if (lane < P.RR) {
       const int m = Q * 32 + lane;
-      Ti[m] = racc0;
-      Ti[P.M1 + m] = racc1;
-      Ti[2 * P.M1 + m] = racc2;
-      Ti[3 * P.M1 + m] = racc3;
+      Ti[m] = to_io(racc0);
+      Ti[P.M1 + m] = to_io(racc1);
+      Ti[2 * P.M1 + m] = to_io(racc2);
+      Ti[3 * P.M1 + m] = to_io(racc3);
     }
   }
   if (P.D) descriptor_epilogue<real, Q>(P, acc, racc0, racc1, racc2, racc3, lane, i);
@@ -477,9 +491,10 @@ FwdKernel<real> pick_fwd(int Q, std::integer_sequence<int, Qs...>) {
 }
 
 template <typename real>
-int fwd(const real *table, const dp_table_info *info, const real *s, const real *Rt, const int32_t *nvalid,
-        const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, real *T, void *stream,
-        int M2 = 0, real *D = nullptr, bool want_D = false, bool moments = false) {
+int fwd(const real *table, const dp_table_info *info, const io_t<real> *s, const io_t<real> *Rt,
+        const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1,
+        io_t<real> *T, void *stream, int M2 = 0, io_t<real> *D = nullptr, bool want_D = false,
+        bool moments = false) {
   clear_error();
   TableGeom g;
   Segments seg;
@@ -510,9 +525,12 @@ int fwd(const real *table, const dp_table_info *info, const real *s, const real 
   P.RR = M1 - 32 * Q;
   P.PK = P.RR > 0 ? 32 / P.RR : 1;
   for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
-  P.inv_nnei = (real)(1.0 / (double)nnei);
-  FwdKernel<real> k = moments ? pick_fwd<real, true>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{})
-                              : pick_fwd<real, false>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
+  P.inv_nnei = host_cvt<real>(1.0 / (double)nnei);
+  FwdKernel<real> k = nullptr;
+  if (moments)
+    k = pick_fwd<real, true>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
+  else if constexpr (!std::is_same<real, df64>::value)  // df64 runs the moment form only
+    k = pick_fwd<real, false>(Q, std::make_integer_sequence<int, DP_MAX_M1 / 32 + 1>{});
   if (!k) return set_error(DP_ERR_UNSUPPORTED, "no forward kernel for M1 = %d", M1);
   const int64_t blocks = (nloc + kFwdWarps - 1) / kFwdWarps;
   if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
@@ -550,6 +568,13 @@ int dp_tabulate_fusion_fwd_moments_f32(const float *table, const dp_table_info *
                                        int nnei, int ntypes, const int32_t *sel, int M1, float *T, void *stream) {
   return dpc::fwd<float>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, stream, 0, nullptr, false,
                          true);
+}
+
+int dp_tabulate_fusion_fwd_moments_df64(const float *table, const dp_table_info *info, const double *s,
+                                        const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                        int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *stream) {
+  return dpc::fwd<dpc::df64>(reinterpret_cast<const dpc::df64 *>(table), info, s, Rt, nvalid, atype, nloc, nnei,
+                             ntypes, sel, M1, T, stream, 0, nullptr, false, true);
 }
 
 int dp_tabulate_fusion_fwd_descriptor_f64(const double *table, const dp_table_info *info, const double *s,

@@ -34,13 +34,13 @@ constexpr int kGradChunk = 16;  // atoms whose valid rows are packed together
 template <typename real>
 struct GradParams {
   const real *__restrict__ table;
-  const real *__restrict__ s;
-  const real *__restrict__ Rt;
+  const io_t<real> *__restrict__ s;
+  const io_t<real> *__restrict__ Rt;
   const int32_t *__restrict__ nvalid;
   const int32_t *__restrict__ atype;
-  const real *__restrict__ dT;
-  real *__restrict__ ds;
-  real *__restrict__ dRt;
+  const io_t<real> *__restrict__ dT;
+  io_t<real> *__restrict__ ds;
+  io_t<real> *__restrict__ dRt;
   TableGeom geom;
   typename GeomOf<real>::type lgeom;  // the same geometry in the precision of real (moment kernel)
   int64_t nloc;
@@ -239,7 +239,7 @@ __device__ __forceinline__ void rs_step(real *h, int lane, int &base, int &nreal
   if constexpr (mask >= 1) {
     const bool hi = lane & mask;
     if constexpr (n == 1) {
-      h[0] += __shfl_xor_sync(0xffffffffu, h[0], mask);
+      h[0] += shfl_xor(h[0], mask);
       if (hi) nreal = 0;
       rs_step<1, mask / 2>(h, lane, base, nreal);
     } else {
@@ -248,7 +248,7 @@ __device__ __forceinline__ void rs_step(real *h, int lane, int &base, int &nreal
 #pragma unroll
       for (int x = 0; x < half; ++x) {
         const real snd = hi ? h[x] : h[x + half], kp = hi ? h[x + half] : h[x];
-        h[x] = kp + __shfl_xor_sync(0xffffffffu, snd, mask);
+        h[x] = kp + shfl_xor(snd, mask);
       }
       if (hi) {
         base += half;
@@ -268,6 +268,12 @@ __device__ __forceinline__ void reduce_scatter(real *h, int lane, int &base, int
   rs_step<N, C / 2>(h, lane, base, nreal);
 }
 
+// Channel loops are unrolled twice in f64 and f32.  In df64 every FMA is
+// twelve instructions: the loop bodies are large already, and a kernel that
+// no longer fits the instruction cache stalls on instruction fetch.
+template <typename real>
+constexpr int kUnrollM = is_df64<real> ? 1 : 2;
+
 // H of the runs in slots s0 .. s0+G-1 (those below nrun): lane = (run p, channel lane c),
 // C = 32/G channel lanes per run, each summing over the channels c, c + C, ...
 template <int G, typename real>
@@ -281,7 +287,7 @@ __device__ __forceinline__ void form_H_group(MomentGradStage<real> &st, const re
   real h[25];
 #pragma unroll
   for (int x = 0; x < 24; ++x) h[x] = real(0);
-#pragma unroll 2
+#pragma unroll kUnrollM<real>
   for (int m = c; m < M1; m += C) {
     real c6[6];  // (a..f): coefficients of t^5 .. t^0
     ld6(blk, M1, m, c6);
@@ -318,7 +324,7 @@ __device__ __forceinline__ void grad_rows_group(const GradParams<real> &P, const
   const int e = valid ? q : q0;
   const int rw = st.qrow[e];
   const int row = rw & (kClamped - 1);
-  const Vec4<real> rr = ld4(P.Rt + (i * P.nnei + row) * 4);
+  const Vec4<real> rr = ld4r<real>(P.Rt + (i * P.nnei + row) * 4);
   real t;
   bool clamped;
   locate(P.lgeom, __ldg(P.s + i * P.nnei + row), t, clamped);
@@ -327,7 +333,7 @@ __device__ __forceinline__ void grad_rows_group(const GradParams<real> &P, const
   real a[6];  // ds, dR~[0..3], and room for the padding zero
 #pragma unroll
   for (int x = 0; x < 5; ++x) a[x] = real(0);
-#pragma unroll 2
+#pragma unroll kUnrollM<real>
   for (int m = c; m < M1; m += C) {
     real cf[6];
     ld6(blk, M1, m, cf);
@@ -355,28 +361,41 @@ __device__ __forceinline__ void grad_rows_group(const GradParams<real> &P, const
   int base, nreal;
   reduce_scatter<5, C>(a, lane, base, nreal);
   if (valid) {
-    real *__restrict__ ds_i = P.ds + i * P.nnei;
-    real *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
+    io_t<real> *__restrict__ ds_i = P.ds + i * P.nnei;
+    io_t<real> *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
 #pragma unroll
     for (int x = 0; x < rs_count(5, ilog2(C)); ++x)
       if (x < nreal) {
         const int comp = base + x;
         if (comp == 0)
-          ds_i[row] = (rw & kClamped) ? real(0) : a[x];
+          ds_i[row] = (rw & kClamped) ? io_t<real>(0) : to_io(a[x]);
         else
-          dR_i[(size_t)row * 4 + comp - 1] = a[x];
+          dR_i[(size_t)row * 4 + comp - 1] = to_io(a[x]);
       }
   }
 }
 
-// Group size for `rem` runs or rows left: G = 8 for 7 or more, then 4, 2, 1.
-__device__ __forceinline__ int h_group_size(int rem) { return rem >= 7 ? 8 : rem >= 4 ? 4 : rem >= 2 ? 2 : 1; }
+// Group size for `rem` runs or rows left: G = 8 for 7 or more, then 4, 2, 1.  df64 keeps two
+// of the four shapes (8 for 5 or more, else 1): each shape is another copy of a large loop.
+template <typename real>
+__device__ __forceinline__ int h_group_size(int rem) {
+  if constexpr (is_df64<real>) return rem >= 5 ? 8 : 1;
+  return rem >= 7 ? 8 : rem >= 4 ? 4 : rem >= 2 ? 2 : 1;
+}
 
 template <typename real>
 __device__ __forceinline__ void form_H_runs(MomentGradStage<real> &st, const real *__restrict__ tab, const real *dts,
                                             int M1, int nrun, int lane) {
   for (int s0 = 0; s0 < nrun;) {  // uniform
-    const int G = h_group_size(nrun - s0);
+    const int G = h_group_size<real>(nrun - s0);
+    if constexpr (is_df64<real>) {
+      if (G == 8)
+        form_H_group<8>(st, tab, dts, M1, s0, nrun, lane);
+      else
+        form_H_group<1>(st, tab, dts, M1, s0, nrun, lane);
+      s0 += G;
+      continue;
+    }
     if (G == 8)
       form_H_group<8>(st, tab, dts, M1, s0, nrun, lane);
     else if (G == 4)
@@ -396,7 +415,15 @@ __device__ __forceinline__ int grad_rows_queued(const GradParams<real> &P, const
                                                 bool all, int lane) {
   int q0 = 0;
   while (n - q0 >= 8 || (all && q0 < n)) {  // uniform
-    const int G = h_group_size(n - q0);
+    const int G = h_group_size<real>(n - q0);
+    if constexpr (is_df64<real>) {
+      if (G == 8)
+        grad_rows_group<8>(P, st, tab, dts, i, q0, n, lane);
+      else
+        grad_rows_group<1>(P, st, tab, dts, i, q0, n, lane);
+      q0 += G;
+      continue;
+    }
     if (G == 8)
       grad_rows_group<8>(P, st, tab, dts, i, q0, n, lane);
     else if (G == 4)
@@ -430,10 +457,10 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     if (lane < DP_MAX_TYPES) st.nvb[lane] = x;
   }
   {  // dT_i / N_c, transposed: the 1/N_c of every output is folded in here, once per atom
-    const real *__restrict__ dTi = P.dT + i * 4 * M1;
+    const io_t<real> *__restrict__ dTi = P.dT + i * 4 * M1;
     for (int e = lane; e < 4 * M1; e += 32) {
       const int k = e / M1, m = e - k * M1;
-      dts[m * 4 + k] = __ldg(dTi + e) * P.inv_nnei;
+      dts[m * 4 + k] = from_io<real>(__ldg(dTi + e)) * P.inv_nnei;
     }
   }
   __syncwarp();
@@ -442,8 +469,8 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
   for (int q = 0; q < DP_MAX_TYPES; ++q) nv += st.nvb[q];
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   const real *__restrict__ tab = P.table + (size_t)alpha * P.ntypes * P.pair_stride;
-  real *__restrict__ ds_i = P.ds + i * P.nnei;
-  real *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
+  io_t<real> *__restrict__ ds_i = P.ds + i * P.nnei;
+  io_t<real> *__restrict__ dR_i = P.dRt + i * P.nnei * 4;
 
   // outputs of one row (this lane) from its run's H, by Horner's rule with derivative
   auto eval_row = [&](const real *Hr, real t, real r0, real r1, real r2, real r3, int rw) {
@@ -469,7 +496,7 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     dsv = fma(r2, G[2], dsv);
     dsv = fma(r3, G[3], dsv);
     const int row = rw & (kClamped - 1);
-    ds_i[row] = (rw & kClamped) ? real(0) : dsv;
+    ds_i[row] = (rw & kClamped) ? io_t<real>(0) : to_io(dsv);
     st4(dR_i + (size_t)row * 4, dR[0], dR[1], dR[2], dR[3]);
   };
   constexpr int kCarrySlot = chunk_runs<real>();
@@ -492,7 +519,7 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
           off += P.sel[c - 1];
         }
       const int row = off + (v - cum);
-      const Vec4<real> rr = ld4(P.Rt + (i * P.nnei + row) * 4);
+      const Vec4<real> rr = ld4r<real>(P.Rt + (i * P.nnei + row) * 4);
       real t;
       bool clamped;
       const int l = locate(P.lgeom, __ldg(P.s + i * P.nnei + row), t, clamped);
@@ -580,8 +607,8 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
         nvb_b = st.nvb[c];
       }
     const int row = off + nvb_b + (pv - cum);
-    ds_i[row] = real(0);
-    st4(dR_i + (size_t)row * 4, real(0), real(0), real(0), real(0));
+    ds_i[row] = io_t<real>(0);
+    st4(dR_i + (size_t)row * 4, io_t<real>(0), io_t<real>(0), io_t<real>(0), io_t<real>(0));
   }
 }
 
@@ -797,9 +824,9 @@ int grad_f32(const float *table, const TableGeom &g, const Segments &seg, const 
 }
 
 template <typename real>
-int grad(const real *table, const dp_table_info *info, const real *s, const real *Rt, const int32_t *nvalid,
-         const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, const real *dT,
-         real *ds, real *dRt, void *stream, bool moments = false) {
+int grad(const real *table, const dp_table_info *info, const io_t<real> *s, const io_t<real> *Rt,
+         const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1,
+         const io_t<real> *dT, io_t<real> *ds, io_t<real> *dRt, void *stream, bool moments = false) {
   clear_error();
   TableGeom g;
   Segments seg;
@@ -827,7 +854,7 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
   P.M1 = M1;
   P.pair_stride = g.nint * M1 * 6;
   for (int b = 0; b < DP_MAX_TYPES; ++b) P.sel[b] = seg.sel[b];
-  P.inv_nnei = (real)(1.0 / (double)nnei);
+  P.inv_nnei = host_cvt<real>(1.0 / (double)nnei);
   if (moments) {
     void (*k)(const GradParams<real>) = &grad_moments_kernel<real>;
     const size_t smem = sizeof(MomentGradStage<real>) + (size_t)4 * M1 * sizeof(real);
@@ -838,12 +865,16 @@ int grad(const real *table, const dp_table_info *info, const real *s, const real
     k<<<(unsigned)nloc, kMomentWarps * 32, smem, (cudaStream_t)stream>>>(P);
     return launch_status("dp_tabulate_fusion_grad_moments");
   }
+  if constexpr (std::is_same<real, df64>::value) {
+    return set_error(DP_ERR_UNSUPPORTED, "df64 runs the moment form only");
+  } else {
   const int64_t ychunks = ((int64_t)kGradChunk * nnei + kGradThreads - 1) / kGradThreads;
   if (ychunks > 65535) return set_error(DP_ERR_SHAPE, "nnei = %d too large", nnei);
   const int64_t xchunks = (nloc + kGradChunk - 1) / kGradChunk;
   dim3 grid((unsigned)xchunks, (unsigned)ychunks);
   grad_kernel<real><<<grid, kGradThreads, 0, (cudaStream_t)stream>>>(P);
   return launch_status("dp_tabulate_fusion_grad");
+  }
 }
 
 }  // namespace
@@ -870,6 +901,14 @@ int dp_tabulate_fusion_grad_moments_f64(const double *table, const dp_table_info
                                         int nnei, int ntypes, const int32_t *sel, int M1, const double *dT, double *ds,
                                         double *dRt, void *stream) {
   return dpc::grad<double>(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, stream, true);
+}
+
+int dp_tabulate_fusion_grad_moments_df64(const float *table, const dp_table_info *info, const double *s,
+                                         const double *Rt, const int32_t *nvalid, const int32_t *atype, int64_t nloc,
+                                         int nnei, int ntypes, const int32_t *sel, int M1, const double *dT,
+                                         double *ds, double *dRt, void *stream) {
+  return dpc::grad<dpc::df64>(reinterpret_cast<const dpc::df64 *>(table), info, s, Rt, nvalid, atype, nloc, nnei,
+                              ntypes, sel, M1, dT, ds, dRt, stream, true);
 }
 
 int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info *info, const float *s,
