@@ -51,6 +51,17 @@ DESC_FMA_PER_ATOM = lambda M1, M2: 4 * M1 * M2  # noqa: E731
 DESC_GRAD_FMA_PER_ATOM = lambda M1, M2: 8 * M1 * M2  # noqa: E731
 
 
+def footprint(w, esize: int, hbm_bytes: float = 280e9) -> dict:
+    """Device memory of one fwd + descriptor + grad pass per atom (the memory side of Sec. III's
+    comparison): s, R~, T, dE/dT, D, ds, dR~ and the two int32 count / type arrays.  An uncompressed
+    model also materialises the embedding matrix G and keeps every embedding-net layer's output per
+    neighbour row for its backward: sum(widths[1:]) values per row.  Atoms per GPU = hbm_bytes / that."""
+    ours = esize * (5 * w.nnei + 8 * w.M1 + w.M1 * w.M2 + 5 * w.nnei) + 4 * (w.ntypes + 1)
+    net = esize * w.nnei * sum(int(x) for x in w.widths[1:])
+    return {"bytes_per_atom": ours, "uncompressed_extra_bytes_per_atom": net,
+            "atoms_per_280GB": int(hbm_bytes // ours), "atoms_per_280GB_uncompressed": int(hbm_bytes // (ours + net))}
+
+
 def chain_bytes(w, esize: int, nall: int) -> dict:
     """Algorithmic DRAM bytes of the chain's front and back end (the unique data each one must move):
     env_mat reads the neighbour list and the coordinates once and writes s, R~ (every row) and the counts;
@@ -451,7 +462,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                                  "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
                                  else "per row: 9 M1 fwd, 18 M1 grad"),
                    "l2": "flushed between steps (256 MiB write)",
-                   "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4)},
+                   "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4),
+                   "footprint": footprint(w, 4 if args.dtype == "f32" else 8)},
         "atoms_per_s": w.nloc * world * args.steps / total_s,
         "roofline": roofline,
         "kernels": kernels,

@@ -73,33 +73,46 @@ __host__ __device__ __forceinline__ df64 from_double(const double x) {
 __host__ __device__ __forceinline__ double to_double(const df64 a) { return (double)a.hi + (double)a.lo; }
 
 // The same two conversions for the kernels, by integer operations on the bit
-// patterns instead of FP64 conversion instructions: those run on the FP64
-// pipe, where four of them per value would cost more than the df64
-// arithmetic they feed.
+// patterns only.  Conversion instructions between float and double execute on
+// GB300's FP64 pipe (64 cycles per warp instruction on a sub-partition), and
+// a rare-case fallback to them is if-converted by the compiler into every
+// call; so the special cases are integer selects as well.
 //
-// split: hi = x with its significand cut to 24 bits (a normal float), lo =
-// the remaining 29 bits cut to 24, |x - hi - lo| < 2^-47 |x|.  Values outside
-// [2^-79, 2^128) in magnitude (zero, tiny, huge, inf, NaN) take from_double.
+// split: hi = x with its significand cut to 24 bits, lo = the remaining 29
+// bits cut to 24: |x - hi - lo| < 2^-47 |x| for 2^-79 <= |x| < 2^128.  Below
+// that lo is 0 (|x| < 2^-79: 24 bits kept) and below 2^-126 hi is 0 too; at
+// or above 2^128 hi is +-inf, and NaN stays NaN.
 __device__ __forceinline__ df64 split(const double x) {
   const unsigned hw = (unsigned)__double2hiint(x), lw = (unsigned)__double2loint(x);
   const unsigned e = (hw >> 20) & 0x7ffu;  // biased double exponent
-  if (e - 944u > 206u) return from_double(x);
   const unsigned sign = hw & 0x80000000u;
-  const float hi = __uint_as_float(sign | ((e - 896u) << 23) | ((hw & 0xfffffu) << 3) | (lw >> 29));
-  // bits 28..5 of the low word (an integer below 2^24, exact as a float), scaled by their weight
-  const float r = __uint2float_rn((lw & 0x1fffffffu) >> 5);
-  const float scale = __uint_as_float((e - 943u) << 23);  // 2^(e - 1075 + 5), a normal float for e >= 944
+  const unsigned m23 = ((hw & 0xfffffu) << 3) | (lw >> 29);
+  unsigned hb = sign | ((e - 896u) << 23) | m23;              // normal float range: 897 <= e <= 1150
+  hb = e < 897u ? sign : hb;                                   // tiny: signed zero
+  const unsigned nan = (e == 0x7ffu && ((hw & 0xfffffu) | lw)) ? 0x400000u : 0u;
+  hb = e > 1150u ? (sign | 0x7f800000u | nan) : hb;            // huge, inf, NaN
+  // bits 28..5 of the low word: an integer below 2^24, made exact as a float from two 12-bit halves
+  // (2^23 + h - 2^23 is exact for h < 2^23), then scaled by its weight
+  const unsigned r24 = (lw & 0x1fffffffu) >> 5;
+  const float ra = __fsub_rn(__uint_as_float(0x4b000000u | (r24 >> 12)), 8388608.0f);
+  const float rb = __fsub_rn(__uint_as_float(0x4b000000u | (r24 & 0xfffu)), 8388608.0f);
+  const float r = __fmaf_rn(ra, 4096.0f, rb);
+  const float scale = __uint_as_float(e - 943u < 207u ? (e - 943u) << 23 : 0u);  // 2^(e-1070); 0 outside
   const float lo = __uint_as_float(__float_as_uint(__fmul_rn(r, scale)) ^ sign);
-  return df64(hi, lo);
+  return df64(__uint_as_float(hb), lo);
 }
 
-// A normal float widened to double by moving its fields (exact); zero,
-// subnormal, inf and NaN take the conversion instruction.
+// A float widened to double by moving its fields (exact for normal floats);
+// zero and subnormals give a signed zero, inf and NaN keep their kind.
 __device__ __forceinline__ double widen(const float f) {
   const unsigned b = __float_as_uint(f);
-  const unsigned e = (b >> 23) & 0xffu;
-  if (e - 1u > 253u) return (double)f;
-  return __hiloint2double((int)((b & 0x80000000u) | ((e + 896u) << 20) | ((b & 0x7fffffu) >> 3)), (int)(b << 29));
+  const unsigned e = (b >> 23) & 0xffu, m = b & 0x7fffffu;
+  const unsigned sign = b & 0x80000000u;
+  unsigned hw = sign | ((e + 896u) << 20) | (m >> 3), lw = m << 29;
+  hw = e == 0xffu ? (sign | 0x7ff00000u | (m >> 3) | (m ? 0x80000u : 0u)) : hw;
+  hw = e == 0u ? sign : hw;
+  lw = e == 0u ? 0u : lw;
+  return __hiloint2double((int)hw, (int)lw);
 }
 
 // hi + lo in double: one FP64 add.

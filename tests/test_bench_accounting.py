@@ -60,3 +60,13 @@ def test_moment_fmas_take_the_cheaper_form():
     # singletons stay per row, long runs go through moments
     assert bench.moment_fmas(np.array([1]), M1)["fwd"] == 9 * M1
     assert bench.moment_fmas(np.array([400]), M1)["grad"] == 24 * M1 + 40 * 400
+
+
+def test_footprint_counts_every_array():
+    """Bytes per atom of the pass: s and R~ in, ds and dR~ out (5 values per row each way), T and dT
+    (4 M1 each), D (M1 M2), two int32 arrays; the uncompressed model adds every layer output per row."""
+    w = W.tiny()
+    f = bench.footprint(w, 8)
+    assert f["bytes_per_atom"] == 8 * (10 * 32 + 8 * 32 + 32 * 4) + 4 * 2
+    assert f["uncompressed_extra_bytes_per_atom"] == 8 * 32 * (8 + 16 + 32)
+    assert f["atoms_per_280GB"] > f["atoms_per_280GB_uncompressed"] > 0
