@@ -277,7 +277,7 @@ int dp_descriptor_contract_grad_f32(const float *T, const float *dD, int64_t nlo
  * ~1e-38 / 2^-24) flush towards zero, above ~3e38 overflow.
  *
  * dp_descriptor_contract_grad_df64 also stages dD_i: it needs
- * M1 (8 + M2) <= 7264 (DP_ERR_UNSUPPORTED beyond).
+ * M1 (9 + M2) <= 7264 (DP_ERR_UNSUPPORTED beyond).
  *
  * The table is built for this arithmetic: [npair][nint][3][M1][4] float,
  * per interval the (a.hi, a.lo, b.hi, b.lo) vectors of all channels, then

@@ -6,6 +6,8 @@
 // in storage order: every FP64 instruction has 32 busy lanes (M1*M2 is a
 // multiple of 32 for the paper's shapes) and every store is coalesced.
 // Both kernels also run in df64 arithmetic on double arrays (io_t).
+#include <type_traits>
+
 #include "dp_common.cuh"
 
 namespace dpc {
@@ -44,11 +46,19 @@ __global__ void __launch_bounds__(kDescWarps * 32)
   }
 }
 
+// dD_i is staged in shared memory (read once, coalesced, converted once) in df64, where each
+// element, read eight times, would otherwise cost eight conversions.  In f64 and f32 the
+// second read of each element hits L1; staging there made the f32 kernel load-bound (both
+// operands of every FMA from shared memory: 0.100 -> 0.146 ms on the water-like input).
+template <typename real>
+constexpr bool kStageDD = is_df64<real>;
+
 // Shared memory per warp of the descriptor backward, in elements: T_i and the partial dT_i
-// ([4][M1] each), and in df64 also dD_i ([M1][M2]).
+// ([4][M1] each), and dD_i ([M1][M2 + 1], rows padded so that the eight rows one
+// instruction reads fall in different banks) where it is staged.
 template <typename real>
 __host__ __device__ constexpr size_t desc_grad_smem_per_warp(int M1, int M2) {
-  return (size_t)8 * M1 + (is_df64<real> ? (size_t)M1 * M2 : 0);
+  return (size_t)8 * M1 + (kStageDD<real> ? (size_t)M1 * (M2 + 1) : 0);
 }
 
 // Backward of the descriptor: D[m][n] = sum_k T[k][m] T[k][n] (n < M2) is
@@ -72,23 +82,26 @@ __global__ void __launch_bounds__(kDescWarps * 32)
   const io_t<real> *__restrict__ Ti = T + i * 4 * M1;
   const io_t<real> *__restrict__ Di = dD + i * (int64_t)M1 * M2;
   for (int e = lane; e < 4 * M1; e += 32) Ts[e] = from_io<real>(__ldg(Ti + e));
-  // df64: dD_i converted once into shared memory ([M1][M2] after Gs); every element is read 8 times
+  // dD_i into shared memory ([M1][M2] after Gs) where staged; every element is read 8 times
   const real *Ds = Gs + 4 * M1;
-  if constexpr (is_df64<real>) {
+  if constexpr (kStageDD<real>) {
     real *Dw = Gs + 4 * M1;
-    for (int e = lane; e < M1 * M2; e += 32) Dw[e] = from_io<real>(__ldg(Di + e));
+    for (int e = lane; e < M1 * M2; e += 32) {
+      const int r = e / M2;
+      Dw[e + r] = from_io<real>(__ldg(Di + e));
+    }
   }
   __syncwarp();
-  auto dd = [&](int e) -> real {
-    if constexpr (is_df64<real>) return Ds[e];
-    else return __ldg(Di + e);
+  auto dd = [&](int m, int n) -> real {  // dD_i[m][n]
+    if constexpr (kStageDD<real>) return Ds[m * (M2 + 1) + n];
+    else return __ldg(Di + (size_t)m * M2 + n);
   };
   // first term, pairs p = 4 m + k
   for (int p = lane; p < 4 * M1; p += 32) {
     const int m = p >> 2, k = p & 3;
     const real *tk = Ts + k * M1;
     real v = real(0);
-    for (int n = 0; n < M2; ++n) v = fma(dd(m * M2 + n), tk[n], v);
+    for (int n = 0; n < M2; ++n) v = fma(dd(m, n), tk[n], v);
     Gs[k * M1 + m] = v;
   }
   __syncwarp();
@@ -97,7 +110,7 @@ __global__ void __launch_bounds__(kDescWarps * 32)
     const int k = p / M2, m = p - k * M2;
     const real *tk = Ts + k * M1;
     real v = real(0);
-    for (int mp = 0; mp < M1; ++mp) v = fma(dd(mp * M2 + m), tk[mp], v);
+    for (int mp = 0; mp < M1; ++mp) v = fma(dd(mp, m), tk[mp], v);
     Gs[k * M1 + m] += v;
   }
   __syncwarp();
