@@ -356,7 +356,55 @@ def run_native(args, rank, world, local_rank):
     if args.algo == "moments":
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
     nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
-    return report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall)
+    out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall)
+    if world == 1 and not args.no_variants and not args.chain and args.dtype == "f64" and args.algo == "moments":
+        out["variants"] = measure_variants(args, w, dpc, info, sel, d, outs, flush, stream, dev, fmas)
+    return out
+
+
+def measure_variants(args, w, dpc, info, sel, d, ref_outs, flush, stream, dev, fmas):
+    """The same step by the other f64-accurate kernels, on the same resident inputs, timed the same way
+    (L2 flushed between steps, CUDA events per kernel): the per-row kernels (the paper's per-neighbour
+    evaluation) and the df64 moment kernels (double arrays, double-float arithmetic on the FP32 pipes),
+    with the max-norm relative difference of each output from the default path's."""
+    import torch
+    model_df = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, dpc.DF64)
+    model_64 = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, torch.float64)
+    nsteps = max(3, min(args.steps, 100))
+    res = {}
+    for name, model, fwd, grad, arith in (
+            ("f64_per_row", model_64, dpc.dp_tabulate_fusion_fwd, dpc.dp_tabulate_fusion_grad, None),
+            ("df64_moments", model_df, dpc.dp_tabulate_fusion_fwd_moments, dpc.dp_tabulate_fusion_grad_moments,
+             dpc.DF64)):
+        o = {k: torch.empty_like(v) for k, v in ref_outs.items()}
+
+        def step(rec):
+            rec(0)
+            fwd(model.table, info, d["s"], d["Rt"], d["nvalid"], d["atype"], sel, out=o["T"])
+            rec(1)
+            dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"], arith=arith)
+            rec(2)
+            grad(model.table, info, d["s"], d["Rt"], d["nvalid"], d["atype"], sel, d["dT"], out=(o["ds"], o["dRt"]))
+            rec(3)
+        for _ in range(args.warmup):
+            step(lambda k: None)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(nsteps)]
+        torch.cuda.synchronize(dev)
+        for k in range(nsteps):
+            flush.zero_()
+            step(lambda j, k=k: evs[k][j].record(stream))
+        torch.cuda.synchronize(dev)
+        ms = {n: sum(e[j].elapsed_time(e[j + 1]) for e in evs) / nsteps for j, n in enumerate(("fwd", "descriptor", "grad"))}
+        tot = sum(ms.values())
+        pk = peak_tflops("df64" if arith else "f64")
+        fm = fmas if arith else {"fwd": FMA_PER_EVAL["fwd"] * w.evals, "grad": FMA_PER_EVAL["grad"] * w.evals}
+        diff = {k: float(((o[k] - ref_outs[k]).abs().max() / ref_outs[k].abs().max()).item()) for k in ref_outs}
+        res[name] = {"value": w.evals / (tot * 1e-3), "unit": UNIT, "ms_per_step": round(tot, 4), "steps": nsteps,
+                     "dtype": "df64" if arith else "f64",
+                     "kernels": {k: {"ms": round(v, 4)} for k, v in ms.items()},
+                     "frac": {k: round(2.0 * fm[k] / (ms[k] * 1e-3) / 1e12 / pk, 4) for k in ("fwd", "grad")},
+                     "peak_tflops": round(pk, 4), "max_rel_diff_vs_default": diff}
+    return res
 
 
 def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_all):
@@ -593,6 +641,8 @@ def main():
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip the per-row and df64 timings added to the default f64 line")
     ap.add_argument("--chain", action="store_true",
                     help="time the whole chain from coordinates to forces (env_mat ... force_virial)")
     args = ap.parse_args()

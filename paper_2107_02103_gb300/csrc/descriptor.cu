@@ -6,8 +6,6 @@
 // in storage order: every FP64 instruction has 32 busy lanes (M1*M2 is a
 // multiple of 32 for the paper's shapes) and every store is coalesced.
 // Both kernels also run in df64 arithmetic on double arrays (io_t).
-#include <type_traits>
-
 #include "dp_common.cuh"
 
 namespace dpc {
