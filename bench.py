@@ -276,7 +276,7 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
 
     def step(rec, x, o):
         rec(0)
-        dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]))
+        dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]), arith=arith)
         rec(1)
         fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
         rec(2)
@@ -287,7 +287,8 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
         grad(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, work["dT"],
              out=(work["ds"], work["dRt"]))
         rec(5)
-        dpc.dp_force_virial(x["coord"], x["nlist"], env, work["ds"], work["dRt"], out=(o["F"], o["virial"]))
+        dpc.dp_force_virial(x["coord"], x["nlist"], env, work["ds"], work["dRt"], out=(o["F"], o["virial"]),
+                            arith=arith)
         rec(6)
     return host, d, outs, names, step
 

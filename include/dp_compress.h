@@ -284,6 +284,7 @@ int dp_descriptor_contract_grad_f32(const float *T, const float *dD, int64_t nlo
  * (c, d), then (e, f) -- each coefficient of dp_table_build_f64 split into a
  * float and the float rounding of its remainder.
  * ---------------------------------------------------------------------- */
+struct dp_env_info;
 int dp_table_build_df64(const double *y, const double *dy, const double *d2y, int npair, int M1,
                         const dp_table_info *info, float *table, void *stream);
 int dp_tabulate_fusion_fwd_moments_df64(const float *table, const dp_table_info *info, const double *s,
@@ -296,6 +297,15 @@ int dp_tabulate_fusion_grad_moments_df64(const float *table, const dp_table_info
 int dp_descriptor_contract_df64(const double *T, int64_t nloc, int M1, int M2, double *D, void *stream);
 int dp_descriptor_contract_grad_df64(const double *T, const double *dD, int64_t nloc, int M1, int M2, double *dT,
                                      void *stream);
+/* dp_env_mat_f64 and dp_force_virial_f64 (declared below) in df64: the square root by Karp and
+   Markstein's method, the reciprocal by a Newton-Raphson step, sin and cos of pi u by Taylor
+   series on a reduced argument, each to about 2^-46 relative. */
+int dp_env_mat_df64(const double *coord, const int32_t *nlist, int64_t nloc, int nnei, int ntypes,
+                    const int32_t *sel, const struct dp_env_info *env, double *s, double *Rt, int32_t *nvalid,
+                    void *stream);
+int dp_force_virial_df64(const double *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,
+                         const struct dp_env_info *env, const double *ds, const double *dRt, double *F,
+                         double *virial, void *stream);
 
 /* ------------------------------------------------------------------------
  * Environment matrix front end and force / virial back end (Sec. II: the

@@ -108,6 +108,8 @@ _SIGS = {
                                               ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_df64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_grad_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_env_mat_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
+    "dp_force_virial_df64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
 }
 for _name, (_args, _res) in _SIGS.items():
     _fn = getattr(_lib, _name)
@@ -315,9 +317,12 @@ def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
     return ds, dRt
 
 
-def dp_env_mat(coord, nlist, sel, env: dp_env_info, out=None):
-    """(s [nloc][nnei], Rt [nloc][nnei][4], nvalid [nloc][ntypes] int32) from coord [nall][3] and nlist [nloc][nnei]."""
+def dp_env_mat(coord, nlist, sel, env: dp_env_info, out=None, arith=None):
+    """(s [nloc][nnei], Rt [nloc][nnei][4], nvalid [nloc][ntypes] int32) from coord [nall][3] and nlist [nloc][nnei]
+    (arith="df64": f64 arrays, df64 arithmetic)."""
     coord = _dev(coord, "coord", None)
+    if arith == DF64 and coord.dtype != torch.float64:
+        raise TypeError("df64 takes f64 arrays")
     dtype = coord.dtype
     if coord.dim() != 2 or coord.shape[1] != 3:
         raise ValueError("coord must be [nall][3]")
@@ -334,15 +339,17 @@ def dp_env_mat(coord, nlist, sel, env: dp_env_info, out=None):
         s = _dev(out[0], "s", dtype, (nloc, nnei))
         Rt = _dev(out[1], "Rt", dtype, (nloc, nnei, 4))
         nvalid = _dev(out[2], "nvalid", torch.int32, (nloc, ntypes))
-    fn = getattr(_lib, f"dp_env_mat_{_suffix(dtype)}")
+    fn = getattr(_lib, f"dp_env_mat_{_suffix(arith or dtype)}")
     _check(fn(_ptr(coord), _ptr(nlist), nloc, nnei, ntypes, selc, ctypes.byref(env), _ptr(s), _ptr(Rt), _ptr(nvalid),
               _stream(coord)))
     return s, Rt, nvalid
 
 
-def dp_force_virial(coord, nlist, env: dp_env_info, ds, dRt, out=None):
-    """(F [nall][3], virial [3][3]) from dE/ds [nloc][nnei] and dE/dRt [nloc][nnei][4]."""
+def dp_force_virial(coord, nlist, env: dp_env_info, ds, dRt, out=None, arith=None):
+    """(F [nall][3], virial [3][3]) from dE/ds [nloc][nnei] and dE/dRt [nloc][nnei][4] (arith as dp_env_mat)."""
     coord = _dev(coord, "coord", None)
+    if arith == DF64 and coord.dtype != torch.float64:
+        raise TypeError("df64 takes f64 arrays")
     dtype = coord.dtype
     if coord.dim() != 2 or coord.shape[1] != 3:
         raise ValueError("coord must be [nall][3]")
@@ -357,7 +364,7 @@ def dp_force_virial(coord, nlist, env: dp_env_info, ds, dRt, out=None):
     else:
         F = _dev(out[0], "F", dtype, (nall, 3))
         W = _dev(out[1], "virial", dtype, (3, 3))
-    fn = getattr(_lib, f"dp_force_virial_{_suffix(dtype)}")
+    fn = getattr(_lib, f"dp_force_virial_{_suffix(arith or dtype)}")
     _check(fn(_ptr(coord), _ptr(nlist), nloc, nall, nnei, ctypes.byref(env), _ptr(ds), _ptr(dRt), _ptr(F), _ptr(W),
               _stream(coord)))
     return F, W
@@ -404,6 +411,16 @@ def dp_descriptor_contract_df64(T, M2: int, out=None) -> torch.Tensor:
 def dp_descriptor_contract_grad_df64(T, dD, out=None) -> torch.Tensor:
     """dp_descriptor_contract_grad in df64 arithmetic (f64 T, dD and dT)."""
     return dp_descriptor_contract_grad(T, dD, out, arith=DF64)
+
+
+def dp_env_mat_df64(coord, nlist, sel, env: dp_env_info, out=None):
+    """dp_env_mat in df64 arithmetic (f64 arrays)."""
+    return dp_env_mat(coord, nlist, sel, env, out, arith=DF64)
+
+
+def dp_force_virial_df64(coord, nlist, env: dp_env_info, ds, dRt, out=None):
+    """dp_force_virial in df64 arithmetic (f64 arrays)."""
+    return dp_force_virial(coord, nlist, env, ds, dRt, out, arith=DF64)
 
 
 def dp_table_build_df64(y, dy, d2y, info: dp_table_info, out=None) -> torch.Tensor:

@@ -118,5 +118,82 @@ __device__ __forceinline__ double widen(const float f) {
 // hi + lo in double: one FP64 add.
 __device__ __forceinline__ double join(const df64 a) { return __dadd_rn(widen(a.hi), widen(a.lo)); }
 
+// ---------------------------------------------------------------- functions
+// (s, e) with s + e == a + b exactly, for |a| >= |b| (or a == 0): Dekker's fast two-sum.
+__device__ __forceinline__ df64 fast_two_sum(const float a, const float b) {
+  const float s = __fadd_rn(a, b);
+  return df64(s, __fsub_rn(b, __fsub_rn(s, a)));
+}
+
+__device__ __forceinline__ df64 operator-(const df64 a) { return df64(-a.hi, -a.lo); }
+__device__ __forceinline__ bool operator<(const df64 a, const df64 b) {
+  return a.hi < b.hi || (a.hi == b.hi && a.lo < b.lo);
+}
+__device__ __forceinline__ df64 operator-(const df64 a, const df64 b) { return a + (-b); }
+
+// The float nearest a df64 (up to one rounding).  Results are left unnormalised, and after
+// a cancellation the whole value can sit in lo (hi == 0), so a float stand-in is hi + lo.
+__device__ __forceinline__ float approx(const df64 a) { return __fadd_rn(a.hi, a.lo); }
+
+// 1 / a: the float reciprocal q0 refined by one Newton-Raphson step whose residual
+// e = 1 - a q0 is formed in df64 (q = q0 + q0 e); relative error about 2^-46.
+__device__ __forceinline__ df64 rcp(const df64 a) {
+  const float q0 = __frcp_rn(approx(a));
+  const df64 e = fma(-a, df64(q0), df64(1.0f));
+  return fast_two_sum(q0, __fmul_rn(q0, approx(e)));
+}
+
+// sqrt(a) for a > 0, after Karp and Markstein: y = a x with x the float 1/sqrt(a), corrected
+// by (x / 2)(a - y^2) with the residual formed in df64; relative error about 2^-46.
+__device__ __forceinline__ df64 sqrt(const df64 a) {
+  const float ah = approx(a);
+  const float x = __frsqrt_rn(ah);
+  const float y = __fmul_rn(ah, x);
+  const df64 r = fma(df64(-y), df64(y), a);
+  return fast_two_sum(y, __fmul_rn(__fmul_rn(0.5f, x), approx(r)));
+}
+
+// sin(pi u) and cos(pi u) for u in [0, 1] (the cosine switch): with x = u - 1/2,
+// sin(pi u) = cos(pi x) and cos(pi u) = -sin(pi x); for |x| > 1/4 the pair comes from
+// x' = 1/2 - |x| instead (sin(pi x) = sign(x) cos(pi x'), cos(pi x) = sin(pi x')).  On
+// |z| = |pi x| <= pi/4 the Taylor series of sin to z^17 and of cos to z^18 leave terms below
+// 2^-52 relative; they are summed by Horner's rule in w = z^2.  The coefficients are
+// (-1)^k / (2k+1)! and (-1)^k / (2k)!, and pi, each as the float nearest to it plus the float
+// nearest to the rest.
+__device__ __forceinline__ void sincospi(const df64 u, df64 *sn, df64 *cs) {
+  const df64 x = u + df64(-0.5f);
+  const float xa = approx(x);
+  const bool flip = fabsf(xa) > 0.25f;
+  const bool neg = xa < 0.0f;
+  const df64 ax = neg ? -x : x;
+  const df64 xr = flip ? df64(0.5f) - ax : ax;  // in [0, 1/4]
+  const df64 z = xr * df64(3.1415927e+00f, -8.742278e-08f);
+  const df64 w = z * z;
+  df64 s = df64(2.8114574e-15f, -1.0462085e-22f);
+  s = fma(s, w, df64(-7.6471636e-13f, -1.22007105e-20f));
+  s = fma(s, w, df64(1.6059044e-10f, -5.3525265e-18f));
+  s = fma(s, w, df64(-2.5052108e-08f, -4.417623e-16f));
+  s = fma(s, w, df64(2.7557319e-06f, 3.7935712e-14f));
+  s = fma(s, w, df64(-1.984127e-04f, 2.7255969e-12f));
+  s = fma(s, w, df64(8.333334e-03f, -4.346172e-10f));
+  s = fma(s, w, df64(-1.6666667e-01f, 4.967054e-09f));
+  s = fma(s * w, z, z);  // sin(z)
+  df64 c = df64(-1.5619207e-16f, -1.5404471e-24f);
+  c = fma(c, w, df64(4.7794773e-14f, 7.625444e-22f));
+  c = fma(c, w, df64(-1.1470745e-11f, -2.3722077e-19f));
+  c = fma(c, w, df64(2.0876756e-09f, 1.1082839e-16f));
+  c = fma(c, w, df64(-2.755732e-07f, 7.575112e-15f));
+  c = fma(c, w, df64(2.4801588e-05f, -3.406996e-13f));
+  c = fma(c, w, df64(-1.3888889e-03f, 3.3631094e-11f));
+  c = fma(c, w, df64(4.1666668e-02f, -1.2417635e-09f));
+  c = fma(c, w, df64(-0.5f));
+  c = fma(c, w, df64(1.0f));  // cos(z)
+  // sin(pi x) and cos(pi x) for the signed x
+  df64 sx = flip ? c : s, cx = flip ? s : c;
+  sx = neg ? -sx : sx;
+  *sn = cx;   // sin(pi u) = cos(pi x)
+  *cs = -sx;  // cos(pi u) = -sin(pi x)
+}
+
 }  // namespace dfl
 }  // namespace dpc

@@ -8,7 +8,9 @@
 // coalesced, the neighbour coordinates are gathered (they stay in L2).  The
 // arithmetic per row is a square root, a reciprocal, the switch (a sine and
 // cosine for the cosine switch) and a few dozen FMA; both kernels are FP64
-// bound in f64, like the fusion kernels around them.
+// bound in f64, like the fusion kernels around them.  The df64 instances
+// (double arrays, double-float arithmetic) take the square root, the
+// reciprocal and sin/cos(pi u) from dp_df64.cuh.
 #include <cuda_runtime.h>
 
 #include "dp_common.cuh"
@@ -20,21 +22,32 @@ constexpr int kEnvWarps = 4;  // atoms per block
 
 template <typename real>
 struct EnvParams {
-  const real *__restrict__ coord;
+  const io_t<real> *__restrict__ coord;
   const int32_t *__restrict__ nlist;
-  real *__restrict__ s;
-  real *__restrict__ Rt;
+  io_t<real> *__restrict__ s;
+  io_t<real> *__restrict__ Rt;
   int32_t *__restrict__ nvalid;
-  const real *__restrict__ ds;
-  const real *__restrict__ dRt;
-  real *__restrict__ F;
-  real *__restrict__ virial;
+  const io_t<real> *__restrict__ ds;
+  const io_t<real> *__restrict__ dRt;
+  io_t<real> *__restrict__ F;
+  io_t<real> *__restrict__ virial;
   int64_t nloc;
   int32_t nnei, ntypes;
   int32_t sel[DP_MAX_TYPES];
   real rcs, rc, inv_width, mean, inv_std, inv_std_all;
   int32_t kind;
 };
+
+__device__ __forceinline__ double recip(const double x) { return 1.0 / x; }
+__device__ __forceinline__ float recip(const float x) { return 1.0f / x; }
+__device__ __forceinline__ df64 recip(const df64 x) { return dfl::rcp(x); }
+__device__ __forceinline__ void sin_cos_pi(const double u, double *s, double *c) { sincospi(u, s, c); }
+__device__ __forceinline__ void sin_cos_pi(const float u, float *s, float *c) { sincospif(u, s, c); }
+__device__ __forceinline__ void sin_cos_pi(const df64 u, df64 *s, df64 *c) { dfl::sincospi(u, s, c); }
+template <typename real>
+__device__ __forceinline__ real half_pi() { return real(1.57079632679489661923); }
+template <>
+__device__ __forceinline__ df64 half_pi<df64>() { return df64(1.5707964e+00f, -4.371139e-08f); }
 
 // s(r) and ds/dr of the weighting function (Sec. II).  u = (r - rcs)/(rc - rcs);
 // kind 1: w = u^3 (-6u^2 + 15u - 10) + 1 (the paper's switch), w' = -30 u^2 (u - 1)^2;
@@ -53,12 +66,9 @@ __device__ __forceinline__ void weight(const EnvParams<real> &P, real r, real in
       dw = real(-30) * u2 * um * um;
     } else {
       real sn, cs;
-      if constexpr (sizeof(real) == 8)
-        sincospi(u, &sn, &cs);
-      else
-        sincospif(u, &sn, &cs);
+      sin_cos_pi(u, &sn, &cs);
       w = fma(real(0.5), cs, real(0.5));
-      dw = real(-0.5) * real(3.14159265358979323846) * sn;
+      dw = -(half_pi<real>() * sn);
     }
     sv = w * inv_r;
     dsv = (dw * P.inv_width - w * inv_r) * inv_r;
@@ -86,7 +96,9 @@ __global__ void __launch_bounds__(kEnvWarps * 32) env_mat_kernel(const EnvParams
   const int lane = threadIdx.x & 31;
   const int64_t i = (int64_t)blockIdx.x * kEnvWarps + (threadIdx.x >> 5);
   if (i >= P.nloc) return;  // warp-uniform
-  const real xi = P.coord[3 * i], yi = P.coord[3 * i + 1], zi = P.coord[3 * i + 2];
+  // d = r_j - r_i is formed in the arrays' own precision before it enters the arithmetic type:
+  // in df64 that keeps its relative accuracy independent of how far the atoms sit from the origin
+  const io_t<real> xi = P.coord[3 * i], yi = P.coord[3 * i + 1], zi = P.coord[3 * i + 2];
   int count = 0;  // lane b < ntypes: rows of segment b with a neighbour
   for (int q0 = 0; q0 < P.nnei; q0 += 32) {
     const int q = q0 + lane;
@@ -95,11 +107,12 @@ __global__ void __launch_bounds__(kEnvWarps * 32) env_mat_kernel(const EnvParams
     if (q < P.nnei) {
       real sh = real(0), rx = real(0), ry = real(0), rz = real(0);
       if (j >= 0) {
-        const real dx = P.coord[3 * (int64_t)j] - xi, dy = P.coord[3 * (int64_t)j + 1] - yi,
-                   dz = P.coord[3 * (int64_t)j + 2] - zi;
+        const real dx = from_io<real>(P.coord[3 * (int64_t)j] - xi),
+                   dy = from_io<real>(P.coord[3 * (int64_t)j + 1] - yi),
+                   dz = from_io<real>(P.coord[3 * (int64_t)j + 2] - zi);
         const real r2 = fma(dx, dx, fma(dy, dy, dz * dz));
         const real r = sqrt(r2);
-        const real inv_r = real(1) / r;
+        const real inv_r = recip(r);
         real sv, dsv;
         weight(P, r, inv_r, sv, dsv);
         const real a = sv * inv_r * P.inv_std_all;
@@ -108,7 +121,7 @@ __global__ void __launch_bounds__(kEnvWarps * 32) env_mat_kernel(const EnvParams
         ry = a * dy;
         rz = a * dz;
       }
-      P.s[row] = sh;
+      P.s[row] = to_io(sh);
       st4(P.Rt + row * 4, sh, rx, ry, rz);
     }
     const int b = q < P.nnei ? segment_of(P, q) : 0;
@@ -125,7 +138,7 @@ __global__ void __launch_bounds__(kEnvWarps * 32) env_mat_kernel(const EnvParams
 template <typename real>
 __device__ __forceinline__ real warp_sum(real v) {
 #pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  for (int o = 16; o > 0; o >>= 1) v += shfl_xor(v, o);
   return v;
 }
 
@@ -134,7 +147,7 @@ __global__ void __launch_bounds__(kEnvWarps * 32) force_virial_kernel(const EnvP
   const int lane = threadIdx.x & 31;
   const int64_t i = (int64_t)blockIdx.x * kEnvWarps + (threadIdx.x >> 5);
   if (i >= P.nloc) return;  // warp-uniform
-  const real xi = P.coord[3 * i], yi = P.coord[3 * i + 1], zi = P.coord[3 * i + 2];
+  const io_t<real> xi = P.coord[3 * i], yi = P.coord[3 * i + 1], zi = P.coord[3 * i + 2];
   real f0 = real(0), f1 = real(0), f2 = real(0);  // force on atom i from this lane's rows
   real w[9];
 #pragma unroll
@@ -144,15 +157,15 @@ __global__ void __launch_bounds__(kEnvWarps * 32) force_virial_kernel(const EnvP
     const int64_t row = i * P.nnei + q;
     const int j = q < P.nnei ? __ldg(P.nlist + row) : -1;
     if (j >= 0) {
-      const real d[3] = {P.coord[3 * (int64_t)j] - xi, P.coord[3 * (int64_t)j + 1] - yi,
-                         P.coord[3 * (int64_t)j + 2] - zi};
+      const real d[3] = {from_io<real>(P.coord[3 * (int64_t)j] - xi), from_io<real>(P.coord[3 * (int64_t)j + 1] - yi),
+                         from_io<real>(P.coord[3 * (int64_t)j + 2] - zi)};
       const real r2 = fma(d[0], d[0], fma(d[1], d[1], d[2] * d[2]));
       const real r = sqrt(r2);
-      const real inv_r = real(1) / r;
+      const real inv_r = recip(r);
       real sv, dsv;
       weight(P, r, inv_r, sv, dsv);
-      const Vec4<real> gR = ld4(P.dRt + row * 4);
-      const real g0 = __ldg(P.ds + row) + gR.x;  // the s column feeds both the table input and R~[0]
+      const Vec4<real> gR = ld4r<real>(P.dRt + row * 4);
+      const real g0 = from_io<real>(__ldg(P.ds + row)) + gR.x;  // the s column feeds both the table input and R~[0]
       const real p = fma(gR.y, d[0], fma(gR.z, d[1], gR.w * d[2]));
       // g = (g0 s'/(r std) + (s'/r^2 - s/r^3) p / std_all) d + s/(r std_all) dR~_xyz
       const real cd = fma(g0 * dsv, inv_r * P.inv_std, (dsv - sv * inv_r) * inv_r * inv_r * p * P.inv_std_all);
@@ -161,9 +174,9 @@ __global__ void __launch_bounds__(kEnvWarps * 32) force_virial_kernel(const EnvP
       f0 += g[0];
       f1 += g[1];
       f2 += g[2];
-      atomicAdd(P.F + 3 * (int64_t)j, -g[0]);
-      atomicAdd(P.F + 3 * (int64_t)j + 1, -g[1]);
-      atomicAdd(P.F + 3 * (int64_t)j + 2, -g[2]);
+      atomicAdd(P.F + 3 * (int64_t)j, to_io(-g[0]));
+      atomicAdd(P.F + 3 * (int64_t)j + 1, to_io(-g[1]));
+      atomicAdd(P.F + 3 * (int64_t)j + 2, to_io(-g[2]));
 #pragma unroll
       for (int a = 0; a < 3; ++a)
 #pragma unroll
@@ -176,16 +189,16 @@ __global__ void __launch_bounds__(kEnvWarps * 32) force_virial_kernel(const EnvP
 #pragma unroll
   for (int x = 0; x < 9; ++x) w[x] = warp_sum(w[x]);
   if (lane == 0) {
-    atomicAdd(P.F + 3 * i, f0);
-    atomicAdd(P.F + 3 * i + 1, f1);
-    atomicAdd(P.F + 3 * i + 2, f2);
+    atomicAdd(P.F + 3 * i, to_io(f0));
+    atomicAdd(P.F + 3 * i + 1, to_io(f1));
+    atomicAdd(P.F + 3 * i + 2, to_io(f2));
   }
   if (lane < 9) {
     real v = w[0];
 #pragma unroll
     for (int x = 1; x < 9; ++x)
       if (lane == x) v = w[x];
-    atomicAdd(P.virial + lane, v);
+    atomicAdd(P.virial + lane, to_io(v));
   }
 }
 
@@ -202,18 +215,18 @@ int check_env(const dp_env_info *env) {
 
 template <typename real>
 void fill_env(EnvParams<real> &P, const dp_env_info *env) {
-  P.rcs = (real)env->rcs;
-  P.rc = (real)env->rc;
-  P.inv_width = (real)(1.0 / (env->rc - env->rcs));
-  P.mean = (real)env->mean;
-  P.inv_std = (real)(1.0 / env->std);
-  P.inv_std_all = (real)(1.0 / env->std_all);
+  P.rcs = host_cvt<real>(env->rcs);
+  P.rc = host_cvt<real>(env->rc);
+  P.inv_width = host_cvt<real>(1.0 / (env->rc - env->rcs));
+  P.mean = host_cvt<real>(env->mean);
+  P.inv_std = host_cvt<real>(1.0 / env->std);
+  P.inv_std_all = host_cvt<real>(1.0 / env->std_all);
   P.kind = env->kind;
 }
 
 template <typename real>
-int env_mat(const real *coord, const int32_t *nlist, int64_t nloc, int nnei, int ntypes, const int32_t *sel,
-            const dp_env_info *env, real *s, real *Rt, int32_t *nvalid, void *stream) {
+int env_mat(const io_t<real> *coord, const int32_t *nlist, int64_t nloc, int nnei, int ntypes, const int32_t *sel,
+            const dp_env_info *env, io_t<real> *s, io_t<real> *Rt, int32_t *nvalid, void *stream) {
   clear_error();
   if (nloc < 0) return set_error(DP_ERR_SHAPE, "nloc = %lld < 0", (long long)nloc);
   Segments seg;
@@ -240,8 +253,9 @@ int env_mat(const real *coord, const int32_t *nlist, int64_t nloc, int nnei, int
 }
 
 template <typename real>
-int force_virial(const real *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,
-                 const dp_env_info *env, const real *ds, const real *dRt, real *F, real *virial, void *stream) {
+int force_virial(const io_t<real> *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,
+                 const dp_env_info *env, const io_t<real> *ds, const io_t<real> *dRt, io_t<real> *F,
+                 io_t<real> *virial, void *stream) {
   clear_error();
   if (nloc < 0) return set_error(DP_ERR_SHAPE, "nloc = %lld < 0", (long long)nloc);
   if (nall < nloc) return set_error(DP_ERR_SHAPE, "nall = %lld < nloc = %lld", (long long)nall, (long long)nloc);
@@ -252,8 +266,9 @@ int force_virial(const real *coord, const int32_t *nlist, int64_t nloc, int64_t 
   if (nloc > 0 && (!coord || !nlist || !ds || !dRt)) return set_error(DP_ERR_NULL, "dp_force_virial: NULL input");
   const int64_t blocks = (nloc + kEnvWarps - 1) / kEnvWarps;
   if (blocks > 2147483647LL) return set_error(DP_ERR_SHAPE, "nloc too large");
-  cudaError_t e = cudaMemsetAsync(virial, 0, 9 * sizeof(real), (cudaStream_t)stream);
-  if (e == cudaSuccess && nall > 0) e = cudaMemsetAsync(F, 0, (size_t)nall * 3 * sizeof(real), (cudaStream_t)stream);
+  cudaError_t e = cudaMemsetAsync(virial, 0, 9 * sizeof(io_t<real>), (cudaStream_t)stream);
+  if (e == cudaSuccess && nall > 0)
+    e = cudaMemsetAsync(F, 0, (size_t)nall * 3 * sizeof(io_t<real>), (cudaStream_t)stream);
   if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_force_virial: %s", cudaGetErrorString(e));
   if (nloc == 0) return DP_OK;
   EnvParams<real> P{};
@@ -290,6 +305,18 @@ int dp_force_virial_f64(const double *coord, const int32_t *nlist, int64_t nloc,
                         const dp_env_info *env, const double *ds, const double *dRt, double *F, double *virial,
                         void *stream) {
   return dpc::force_virial<double>(coord, nlist, nloc, nall, nnei, env, ds, dRt, F, virial, stream);
+}
+
+int dp_env_mat_df64(const double *coord, const int32_t *nlist, int64_t nloc, int nnei, int ntypes,
+                    const int32_t *sel, const dp_env_info *env, double *s, double *Rt, int32_t *nvalid,
+                    void *stream) {
+  return dpc::env_mat<dpc::df64>(coord, nlist, nloc, nnei, ntypes, sel, env, s, Rt, nvalid, stream);
+}
+
+int dp_force_virial_df64(const double *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,
+                         const dp_env_info *env, const double *ds, const double *dRt, double *F, double *virial,
+                         void *stream) {
+  return dpc::force_virial<dpc::df64>(coord, nlist, nloc, nall, nnei, env, ds, dRt, F, virial, stream);
 }
 
 int dp_force_virial_f32(const float *coord, const int32_t *nlist, int64_t nloc, int64_t nall, int nnei,

@@ -458,7 +458,8 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
   }
   {  // dT_i / N_c, transposed: the 1/N_c of every output is folded in here, once per atom
     const io_t<real> *__restrict__ dTi = P.dT + i * 4 * M1;
-    for (int e = lane; e < 4 * M1; e += 32) {
+#pragma unroll 4
+    for (int e = lane; e < 4 * M1; e += 32) {  // unrolled: several loads in flight per lane
       const int k = e / M1, m = e - k * M1;
       dts[m * 4 + k] = from_io<real>(__ldg(dTi + e)) * P.inv_nnei;
     }

@@ -155,3 +155,79 @@ def test_df64_water_large_sampled():
     got = run_df64(w)
     ref = run_oracle(w, F64, atoms=atoms)
     assert_parity(got, ref, F64, atoms=atoms)
+
+
+# ------------------------------------------------------------- front and back end in df64
+from test_gpu_env_force import SYSTEMS, _system  # noqa: E402
+
+
+@pytest.mark.parametrize("name,kw,kind,norm", SYSTEMS, ids=[f"{s[0]}-k{s[2]}-n{s[3] is not None}" for s in SYSTEMS])
+def test_df64_env_mat_and_forces(name, kw, kind, norm):
+    """s, R~, counts, forces and virial in df64 against the oracle (both switches, normalised or not)."""
+    dpc = lib()
+    w, coord, nlist, _, env = _system(name, kw, kind, norm)
+    cg, ng = torch.from_numpy(coord).cuda(), torch.from_numpy(nlist).cuda()
+    ei = dpc.env_info(*env)
+    s, Rt, nvalid = dpc.dp_env_mat_df64(cg, ng, w.sel, ei)
+    ds = W.normal(7, nlist.shape)
+    dRt = W.normal(8, nlist.shape + (4,))
+    stale = (torch.full((coord.shape[0], 3), 5.0, dtype=F64, device="cuda"),
+             torch.full((3, 3), 5.0, dtype=F64, device="cuda"))
+    F, Wv = dpc.dp_force_virial_df64(cg, ng, ei, torch.from_numpy(ds).cuda(), torch.from_numpy(dRt).cuda(), out=stale)
+    torch.cuda.synchronize()
+    o = oracle.default()
+    so, Rto = o.env_mat(coord, nlist, *env)
+    Fo, Wo = o.force_virial(coord, nlist, env[0], env[1], ds, dRt, env[2], env[3])
+    assert np.array_equal(nvalid.cpu().numpy(), w.nvalid)
+    errs = {k: rel(g, r) for k, g, r in (("s", s.cpu().numpy(), so), ("Rt", Rt.cpu().numpy(), Rto),
+                                          ("F", F.cpu().numpy(), Fo), ("virial", Wv.cpu().numpy(), Wo))}
+    print(f"df64 env/force {name} kind={kind} norm={norm is not None}: {errs}")
+    assert all(e <= TOL[F64] for e in errs.values()), errs
+    assert not s.cpu().numpy()[nlist < 0].any()
+
+
+def test_df64_forces_through_the_whole_chain():
+    """coordinates -> rows -> T -> D -> dE/dT -> dE/ds, dE/dR~ -> forces, virial, every kernel in df64,
+    against the oracle's chain; the folded forces of the periodic system sum to zero."""
+    dpc = lib()
+    w, coord, nlist, owner, env = _system("water", dict(seed=45, nmol=256), 1, None)
+    model = df64_model(w)
+    cg, ng, at = torch.from_numpy(coord).cuda(), torch.from_numpy(nlist).cuda(), torch.from_numpy(w.atype).cuda()
+    ei = dpc.env_info(*env)
+    dD = W.normal(46, (w.nloc, w.M1, w.M2))
+    s, Rt, nvalid = dpc.dp_env_mat_df64(cg, ng, w.sel, ei)
+    T = dpc.dp_tabulate_fusion_fwd_moments_df64(model.table, model.info, s, Rt, nvalid, at, w.sel)
+    dT = dpc.dp_descriptor_contract_grad_df64(T, torch.from_numpy(dD).cuda())
+    ds, dRt = dpc.dp_tabulate_fusion_grad_moments_df64(model.table, model.info, s, Rt, nvalid, at, w.sel, dT)
+    F, Wv = dpc.dp_force_virial_df64(cg, ng, ei, ds, dRt)
+    torch.cuda.synchronize()
+    o = oracle.default()
+    info, tabs = oracle_tables(w, F64)
+    so, Rto = o.env_mat(coord, nlist, *env)
+    To = o.fwd(tabs, info, so, Rto, w.nvalid, w.atype, w.sel)
+    dso, dRo = o.grad(tabs, info, so, Rto, w.nvalid, w.atype, w.sel, o.descriptor_grad(To, dD))
+    Fo, Wo = o.force_virial(coord, nlist, env[0], env[1], dso, dRo, env[2], env[3])
+    assert rel(F.cpu().numpy(), Fo) <= TOL[F64] and rel(Wv.cpu().numpy(), Wo) <= TOL[F64]
+    folded = np.zeros((w.nloc, 3))
+    np.add.at(folded, owner, F.cpu().numpy())
+    assert np.abs(folded.sum(axis=0)).max() <= 1e-9 * np.abs(folded).max()
+
+
+def test_df64_env_edges():
+    """A neighbour exactly at rc gives s = 0 and no force; u = 1/2 gives w = 1/2 exactly; padding rows."""
+    dpc = lib()
+    for kind in (0, 1):
+        ei = dpc.env_info(1.0, 3.0, kind=kind)
+        coord = torch.tensor([[0.0, 0.0, 0.0], [3.0, 0.0, 0.0], [3.0, 2.0, 0.0]], dtype=F64, device="cuda")
+        nl = torch.tensor([[-1, -1, -1, -1], [0, 2, -1, -1]], dtype=torch.int32, device="cuda")
+        s, Rt, nv = dpc.dp_env_mat_df64(coord, nl, [4], ei)
+        torch.cuda.synchronize()
+        assert nv.cpu().tolist() == [[0], [2]]
+        assert not s[0].abs().max().item() and s[1, 0].item() == 0.0
+        assert abs(s[1, 1].item() - 0.25) <= 1e-15
+        F, Wv = dpc.dp_force_virial_df64(coord, nl, ei, torch.ones((2, 4), dtype=F64, device="cuda"),
+                                         torch.ones((2, 4, 4), dtype=F64, device="cuda"))
+        torch.cuda.synchronize()
+        Fo, Wo = oracle.default().force_virial(coord.cpu().numpy(), nl.cpu().numpy(), 1.0, 3.0, np.ones((2, 4)),
+                                               np.ones((2, 4, 4)), kind)
+        assert rel(F.cpu().numpy(), Fo) <= TOL[F64] and rel(Wv.cpu().numpy(), Wo) <= TOL[F64]
