@@ -196,11 +196,19 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 // bound by its scattered coefficient loads, and every run goes through H.
 constexpr int kMomentWarps = 1;
 constexpr int kChunkRows = 128;  // rows staged per chunk
+// df64: every run goes through H, and a row's four k components are evaluated in a loop.  Each
+// df64 FMA is twelve instructions; the per-row path for single-row runs and the unrolled row
+// evaluation made the kernel too large for the instruction cache (ncu: 2.0 cycles per issued
+// instruction stalled on instruction fetch).  Without them the cu85 backward went from 0.533 to
+// 0.459 ms and the water one from 1.018 to 0.758 ms, although single rows now cost 24 M1 + 40
+// FMA instead of 18 M1.
+constexpr int kDf64MinGradRun = 1;     // shortest run that goes through H in df64
+constexpr bool kDf64RolledEval = true;  // evaluate a row's k components in a loop in df64
 template <typename real>
-constexpr int min_grad_run() { return sizeof(real) == 8 ? 2 : 1; }
+constexpr int min_grad_run() { return is_df64<real> ? kDf64MinGradRun : sizeof(real) == 8 ? 2 : 1; }
 // H slots per chunk (plus one for an open run's H), and the most runs one batch can add
 template <typename real>
-constexpr int chunk_runs() { return sizeof(real) == 8 ? 32 : 64; }
+constexpr int chunk_runs() { return min_grad_run<real>() == 2 ? 32 : 64; }
 template <typename real>
 constexpr int batch_runs() { return 32 / min_grad_run<real>() + 1; }
 
@@ -475,30 +483,52 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
 
   // outputs of one row (this lane) from its run's H, by Horner's rule with derivative
   auto eval_row = [&](const real *Hr, real t, real r0, real r1, real r2, real r3, int rw) {
-    real dR[4], G[4];
-#pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const real *hk = Hr + 6 * k;  // H[k][q], q = 0..5
-      real p = fma(hk[5], t, hk[4]);
-      real dp = hk[5];
-      dp = fma(dp, t, p);
-      p = fma(p, t, hk[3]);
-      dp = fma(dp, t, p);
-      p = fma(p, t, hk[2]);
-      dp = fma(dp, t, p);
-      p = fma(p, t, hk[1]);
-      dp = fma(dp, t, p);
-      p = fma(p, t, hk[0]);
-      dR[k] = p;
-      G[k] = dp;
-    }
-    real dsv = r0 * G[0];
-    dsv = fma(r1, G[1], dsv);
-    dsv = fma(r2, G[2], dsv);
-    dsv = fma(r3, G[3], dsv);
     const int row = rw & (kClamped - 1);
+    real dsv = real(0);
+    if constexpr (is_df64<real> && kDf64RolledEval) {
+      // one k component per iteration: a quarter of the code, each output stored as it is done
+#pragma unroll 1
+      for (int k = 0; k < 4; ++k) {
+        const real *hk = Hr + 6 * k;
+        real p = fma(hk[5], t, hk[4]);
+        real dp = hk[5];
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[3]);
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[2]);
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[1]);
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[0]);
+        const real rk = k == 0 ? r0 : k == 1 ? r1 : k == 2 ? r2 : r3;
+        dsv = fma(rk, dp, dsv);
+        dR_i[(size_t)row * 4 + k] = to_io(p);
+      }
+    } else {
+      real dR[4], G[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const real *hk = Hr + 6 * k;  // H[k][q], q = 0..5
+        real p = fma(hk[5], t, hk[4]);
+        real dp = hk[5];
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[3]);
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[2]);
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[1]);
+        dp = fma(dp, t, p);
+        p = fma(p, t, hk[0]);
+        dR[k] = p;
+        G[k] = dp;
+      }
+      dsv = r0 * G[0];
+      dsv = fma(r1, G[1], dsv);
+      dsv = fma(r2, G[2], dsv);
+      dsv = fma(r3, G[3], dsv);
+      st4(dR_i + (size_t)row * 4, dR[0], dR[1], dR[2], dR[3]);
+    }
     ds_i[row] = (rw & kClamped) ? io_t<real>(0) : to_io(dsv);
-    st4(dR_i + (size_t)row * 4, dR[0], dR[1], dR[2], dR[3]);
   };
   constexpr int kCarrySlot = chunk_runs<real>();
 
@@ -583,7 +613,7 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
       nrun = 0;
       __syncwarp();
     }
-    if (nq >= 8) {  // single-row runs, 8 at a time; fewer than 8 stay queued
+    if (min_grad_run<real>() > 1 && nq >= 8) {  // single-row runs, 8 at a time; fewer than 8 stay queued
       const int done = grad_rows_queued(P, st, tab, dts, i, nq, false, lane);
       __syncwarp();
       if (lane < nq - done) {
@@ -594,7 +624,7 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
       __syncwarp();
     }
   }
-  grad_rows_queued(P, st, tab, dts, i, nq, true, lane);
+  if constexpr (min_grad_run<real>() > 1) grad_rows_queued(P, st, tab, dts, i, nq, true, lane);
 
   // padding rows, packed over the segments' padded tails
   for (int pv = lane; pv < P.nnei - nv; pv += 32) {
