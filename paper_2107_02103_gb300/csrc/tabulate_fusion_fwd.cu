@@ -473,7 +473,8 @@ __device__ __forceinline__ void fwd_atom(const FwdParams<real> &P, Stage<real> &
       Ti[3 * P.M1 + m] = to_io(racc3);
     }
   }
-  if (P.D) descriptor_epilogue<real, Q>(P, acc, racc0, racc1, racc2, racc3, lane, i);
+  if constexpr (!kMoments)  // the fused descriptor is offered with the per-row forward only
+    if (P.D) descriptor_epilogue<real, Q>(P, acc, racc0, racc1, racc2, racc3, lane, i);
 }
 
 template <typename real, int Q, bool kMoments>
