@@ -112,7 +112,7 @@ def moment_fmas(runs, M1: int) -> dict:
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
 # `ncu --set full` capture of its current version (profiles/<kernel>_<algo>_<workload>_<dtype>.md);
 # absent means no capture of the current kernel exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83842304 + 32110592}
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
