@@ -91,6 +91,8 @@ def load(path: str | None = None):
     lib.or_descriptor.restype = None
     lib.or_descriptor_grad.argtypes = [P, P, i64, ctypes.c_int, ctypes.c_int, P]
     lib.or_descriptor_grad.restype = None
+    lib.or_fitting.argtypes = [P, i64, P, ctypes.c_int, P, P, i64, P, P, P, ctypes.c_int]
+    lib.or_fitting.restype = ctypes.c_int
     lib.or_embed_rows.argtypes = [P, ctypes.POINTER(Info), P, P, ctypes.c_int, ctypes.c_int, P, ctypes.c_int, P,
                                   i64, P, P]
     lib.or_embed_rows.restype = None
@@ -249,6 +251,22 @@ class Oracle:
         dT = np.empty_like(T)
         self.lib.or_descriptor_grad(_p(T), _p(dD), n, M, int(M2), _p(dT))
         return dT
+
+    def fitting(self, params, widths, D, atype=None, g=None, grad=True, nthreads=0):
+        """Atomic energies E [n] of the fitting net and, with grad, dE_i/dD_i [n][widths[0]] (scaled by g)."""
+        params = _c(np.atleast_2d(params), np.float64)
+        w = _c(widths, np.int32)
+        D = _c(D.reshape(D.shape[0], -1), np.float64)
+        n = D.shape[0]
+        assert D.shape[1] == w[0]
+        at = None if atype is None else _c(atype, np.int32)
+        gg = None if g is None else _c(g, np.float64)
+        E = np.empty(n)
+        dD = np.empty((n, int(w[0]))) if grad else None
+        if self.lib.or_fitting(_p(params), params.shape[1], _p(w), len(w) - 1, _p(D), _p(at), n, _p(gg), _p(E),
+                               _p(dD), nthreads):
+            raise ValueError("or_fitting failed")
+        return (E, dD) if grad else E
 
     def embed_rows(self, table, info, s, atype, sel, atoms=None, deriv=False):
         table, s = (_c(a, np.float64) for a in (table, s))

@@ -621,3 +621,100 @@ void or_force_virial(int64_t nloc, int64_t nall, const double *coord, const int3
         for (int b = 0; b < 3; ++b) W[3 * a + b] -= d[a] * g[b];
     }
 }
+
+/* ----------------------------------------------------------- fitting net */
+
+/*
+ * Fitting net (Sec. II: the descriptor D_i is passed to a fully connected
+ * network that outputs the atomic energy E_i; the total energy is
+ * E = sum_i E_i).  For centre type t the net has nlayer layers with widths
+ * widths[0..nlayer], widths[0] = the length of D_i, widths[nlayer] = 1:
+ *   hidden layer l (l < nlayer - 1):  v_l = tanh(v_{l-1} W_l + b_l) (+ v_{l-1} when the widths agree)
+ *   output layer:                     E_i = v_{nlayer-1} W_nlayer + b_nlayer
+ * params [ntypes][P], layer by layer W_l [a][b] row-major then b_l [b].
+ * E [n]; when dD is not NULL also dE_i/dD_i [n][widths[0]] by the chain rule
+ * backwards through the layers (d tanh(z)/dz = 1 - tanh(z)^2), scaled by
+ * g[i] (NULL: 1).  Returns -1 for a width above OR_FITW or bad sizes.
+ */
+#define OR_FITW 4096
+int or_fitting(const double *params, int64_t P, const int32_t *widths, int nlayer, const double *D,
+               const int32_t *atype, int64_t n, const double *g, double *E, double *dD, int nthreads) {
+  if (nlayer < 1 || widths[nlayer] != 1) return -1;
+  int hid = 0;  // sum of the hidden widths
+  for (int l = 0; l <= nlayer; ++l)
+    if (widths[l] < 1 || widths[l] > OR_FITW) return -1;
+  for (int l = 1; l < nlayer; ++l) hid += widths[l];
+  int err = 0;
+#ifdef _OPENMP
+  if (nthreads <= 0) nthreads = omp_get_max_threads();
+#pragma omp parallel for num_threads(nthreads) schedule(dynamic, 4) reduction(| : err)
+#endif
+  for (int64_t i = 0; i < n; ++i) {
+    double *act = malloc(sizeof(double) * (size_t)(hid + widths[0]));  // the layer outputs v_0 .. v_{nlayer-1}
+    double *tn = malloc(sizeof(double) * (size_t)(hid > 0 ? hid : 1));  // tanh of every hidden layer
+    double *gv = malloc(sizeof(double) * (size_t)OR_FITW * 2);
+    if (!act || !tn || !gv) {
+      err |= 1;
+      free(act);
+      free(tn);
+      free(gv);
+      continue;
+    }
+    const double *pp = params + (size_t)(atype ? atype[i] : 0) * P;
+    for (int k = 0; k < widths[0]; ++k) act[k] = D[(size_t)i * widths[0] + k];
+    // forward
+    const double *p = pp;
+    int off_in = 0, off_out = widths[0], off_t = 0;
+    for (int l = 1; l < nlayer; ++l) {
+      const int a = widths[l - 1], b = widths[l];
+      const double *W = p, *bias = p + (size_t)a * b;
+      p += (size_t)a * b + b;
+      for (int o = 0; o < b; ++o) {
+        double z = bias[o];
+        for (int k = 0; k < a; ++k) z += act[off_in + k] * W[(size_t)k * b + o];
+        const double t = tanh(z);
+        tn[off_t + o] = t;
+        act[off_out + o] = t + (b == a ? act[off_in + o] : 0.0);
+      }
+      off_in = off_out;
+      off_out += b;
+      off_t += b;
+    }
+    const int a = widths[nlayer - 1];
+    const double *Wo = p, *bo = p + a;
+    double e = bo[0];
+    for (int k = 0; k < a; ++k) e += act[off_in + k] * Wo[k];
+    E[i] = e;
+    if (dD) {
+      // backward: gv holds dE_i/dv_l for the current layer
+      const double gi = g ? g[i] : 1.0;
+      double *cur = gv, *nxt = gv + OR_FITW;
+      for (int k = 0; k < a; ++k) cur[k] = gi * Wo[k];
+      // walk the hidden layers from the last to the first; their parameters precede Wo
+      const double *pl = Wo;
+      int toff = off_t;
+      for (int l = nlayer - 1; l >= 1; --l) {
+        const int ai = widths[l - 1], bo_ = widths[l];
+        pl -= (size_t)ai * bo_ + bo_;
+        const double *W = pl;
+        toff -= bo_;
+        for (int k = 0; k < ai; ++k) nxt[k] = 0.0;
+        for (int o = 0; o < bo_; ++o) {
+          const double t = tn[toff + o];
+          const double gz = cur[o] * (1.0 - t * t);
+          for (int k = 0; k < ai; ++k) nxt[k] += gz * W[(size_t)k * bo_ + o];
+        }
+        if (bo_ == ai)
+          for (int k = 0; k < ai; ++k) nxt[k] += cur[k];
+        double *s = cur;
+        cur = nxt;
+        nxt = s;
+      }
+      for (int k = 0; k < widths[0]; ++k) dD[(size_t)i * widths[0] + k] = cur[k];
+    }
+    free(act);
+    free(tn);
+    free(gv);
+  }
+  return err ? -1 : 0;
+}

@@ -591,8 +591,67 @@ def pin_force_invariants(o):
     assert _rel(W3, ref) < 1e-12 and _rel(ref, ref.T) > 1e-3
 
 
+# ------------------------------------------------------------------ fitting net
+
+def pin_fitting_hand(o):
+    """Nets small enough to evaluate by hand with math.tanh: widths (2, 1, 1) is
+    E = w_o tanh(D W_1 + b_1) + b_o and dE/dD_k = w_o (1 - tanh^2) W_1[k]; widths (3, 2, 2, 1) with
+    W_2 = 0 shows the skip of the equal-width layer: v_2 = tanh(b_2) + v_1."""
+    W1, b1, wo, bo = np.array([0.3, -0.7]), 0.2, 1.5, -0.4
+    params = np.concatenate([W1, [b1], [wo], [bo]])
+    D = np.array([[0.9, 0.25], [-1.2, 0.4]])
+    E, dD = o.fitting(params, [2, 1, 1], D)
+    for i in range(2):
+        z = D[i] @ W1 + b1
+        assert abs(E[i] - (wo * math.tanh(z) + bo)) < 1e-15
+        assert _rel(dD[i], wo * (1 - math.tanh(z) ** 2) * W1) < 1e-15
+    Wa = np.array([[0.1, -0.2], [0.3, 0.05], [-0.6, 0.4]])
+    ba, bb, wout, bout = np.array([0.5, -0.1]), np.array([0.7, 0.2]), np.array([2.0, -1.0]), 0.3
+    params = np.concatenate([Wa.ravel(), ba, np.zeros(4), bb, wout, [bout]])
+    D = np.array([[1.0, -2.0, 0.5]])
+    E = o.fitting(params, [3, 2, 2, 1], D, grad=False)
+    v1 = np.tanh(D[0] @ Wa + ba)
+    v2 = np.tanh(bb) + v1
+    assert abs(E[0] - (v2 @ wout + bout)) < 1e-15
+
+
+def pin_fitting_fd(o):
+    """dE_i/dD_i against central differences of E_i (a 40-wide input, three 24-wide hidden layers
+    with skips, two centre types), and linearity of the gradient in the upstream weights g."""
+    widths = [40, 24, 24, 24, 1]
+    params = W.net_params(61, widths, 2)
+    D = W.normal(62, (5, 40))
+    at = np.array([0, 1, 1, 0, 1], dtype=np.int32)
+    E, dD = o.fitting(params, widths, D, at)
+    h = 1e-6
+    for i in (0, 2, 4):
+        for k in (0, 7, 39):
+            Dp, Dm = D.copy(), D.copy()
+            Dp[i, k] += h
+            Dm[i, k] -= h
+            fd = (o.fitting(params, widths, Dp, at, grad=False)[i] - o.fitting(params, widths, Dm, at, grad=False)[i]) / (2 * h)
+            assert abs(fd - dD[i, k]) <= 1e-8 * max(1.0, np.abs(dD).max()), (i, k, fd, dD[i, k])
+    g = np.array([0.5, -2.0, 1.0, 3.0, 0.0])
+    _, dDg = o.fitting(params, widths, D, at, g=g)
+    assert _rel(dDg, g[:, None] * dD) < 1e-15
+
+
+def pin_fitting_types(o):
+    """Each atom uses its own centre type's parameters: a two-type batch equals two one-type batches."""
+    widths = [10, 6, 6, 1]
+    params = W.net_params(63, widths, 2)
+    D = W.normal(64, (6, 10))
+    at = np.array([1, 0, 1, 1, 0, 0], dtype=np.int32)
+    E, dD = o.fitting(params, widths, D, at)
+    for t in (0, 1):
+        sel = at == t
+        Et, dDt = o.fitting(params[t], widths, D[sel])
+        assert _rel(E[sel], Et) < 1e-15 and _rel(dD[sel], dDt) < 1e-15
+
+
 ALL_PINS = [pin_net_skip_wiring, pin_net_single_neuron, pin_net_derivatives_fd, pin_table_info, pin_locate,
             pin_table_nodes, pin_table_quintic_exact, pin_table_sin_bound, pin_compressed_vs_net,
             pin_fwd_brute_force, pin_fwd_constant_G, pin_fwd_vs_explicit_G, pin_fwd_padding, pin_fwd_symmetries,
             pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor, pin_descriptor_grad,
-            pin_switch, pin_env_mat_hand, pin_env_mat_matches_generator, pin_force_fd, pin_force_invariants]
+            pin_switch, pin_env_mat_hand, pin_env_mat_matches_generator, pin_force_fd, pin_force_invariants,
+            pin_fitting_hand, pin_fitting_fd, pin_fitting_types]

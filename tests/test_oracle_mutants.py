@@ -58,6 +58,12 @@ MUTANTS = [
     ("force: delta term of d(d/r) dropped", "sv * (dab / r - d[a] * d[b] / (r2 * r))", "sv * (0.0 / r - d[a] * d[b] / (r2 * r))"),
     ("virial: sign", "W[3 * a + b] -= d[a] * g[b];", "W[3 * a + b] += d[a] * g[b];"),
     ("virial: transposed", "W[3 * a + b] -= d[a] * g[b];", "W[3 * a + b] -= d[b] * g[a];"),
+    ("fitting: skip missing", "act[off_out + o] = t + (b == a ? act[off_in + o] : 0.0);", "act[off_out + o] = t;"),
+    ("fitting: backward skip missing", "for (int k = 0; k < ai; ++k) nxt[k] += cur[k];", "for (int k = 0; k < ai; ++k) nxt[k] += 0.0;"),
+    ("fitting: tanh' with the wrong sign", "const double gz = cur[o] * (1.0 - t * t);", "const double gz = cur[o] * (1.0 + t * t);"),
+    ("fitting: transposed weights", "for (int k = 0; k < a; ++k) z += act[off_in + k] * W[(size_t)k * b + o];",
+     "for (int k = 0; k < a; ++k) z += act[off_in + k] * W[(size_t)o * a + k];"),
+    ("fitting: centre type ignored", "const double *pp = params + (size_t)(atype ? atype[i] : 0) * P;", "const double *pp = params;"),
 ]
 
 
