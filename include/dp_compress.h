@@ -368,6 +368,58 @@ int dp_force_virial_f32(const float *coord, const int32_t *nlist, int64_t nloc, 
                         const dp_env_info *env, const float *ds, const float *dRt, float *F, float *virial,
                         void *stream);
 
+/* ------------------------------------------------------------------------
+ * Fitting net (Sec. II: the descriptor D_i is passed to a fully connected
+ * network that outputs the atomic energy E_i; the total energy is
+ * E = sum_i E_i).  Each centre type t has its own net of nlayer layers with
+ * widths widths[0..nlayer] (host), widths[0] = the length of D_i (M1 * M2),
+ * widths[nlayer] = 1:
+ *   v_0 = D_i
+ *   v_l = tanh(v_{l-1} W_l + b_l) (+ v_{l-1} when widths[l] == widths[l-1]),  0 < l < nlayer
+ *   E_i = v_{nlayer-1} W_nlayer + b_nlayer
+ *   params      [ntypes][P]: per type, layer by layer, W_l [widths[l-1]][widths[l]]
+ *               row-major then b_l [widths[l]]; P = sum_l (widths[l-1] + 1) widths[l].
+ *   type_start  [ntypes + 1] HOST int64: the atoms of centre type t are rows
+ *               type_start[t] .. type_start[t+1] - 1 (atoms sorted by centre
+ *               type, as in every workload here); type_start[0] = 0 and
+ *               nloc = type_start[ntypes].
+ *   D    [nloc][widths[0]] input (the descriptor, flattened)
+ *   E    [nloc] output
+ *   act  [nloc][H] output, H = the sum of the hidden widths: tanh(v_{l-1} W_l + b_l)
+ *        of every hidden layer, in layer order -- what the backward needs.
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (widths[nlayer] != 1, type_start not
+ * increasing or not starting at 0, more than 4,194,240 atoms of one type),
+ * DP_ERR_UNSUPPORTED (nlayer or ntypes above DP_MAX_LAYERS / DP_MAX_TYPES),
+ * DP_ERR_CUDA.  nloc == 0 reads no device pointer.
+ */
+int dp_fitting_fwd_f64(const double *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
+                       const double *D, double *E, double *act, void *stream);
+int dp_fitting_fwd_f32(const float *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
+                       const float *D, float *E, float *act, void *stream);
+
+/*
+ * Backward of the fitting net: dD[i] = g_i dE_i/dD_i, the chain rule through
+ * the layers in reverse (d tanh(z)/dz = 1 - tanh(z)^2; an identity skip
+ * passes dE/dv_l on to v_{l-1}).
+ *   act   [nloc][H] from dp_fitting_fwd_* on the same D
+ *   g     [nloc] upstream dE/dE_i, or NULL for all ones (E = sum_i E_i)
+ *   dD    [nloc][widths[0]] output (feed it to dp_descriptor_contract_grad_*)
+ *   work  [2][nloc][max hidden width] scratch, caller-owned, overwritten
+ *         (NULL allowed when the net has a single hidden layer).
+ * Errors as dp_fitting_fwd_*; a net without hidden layers is DP_ERR_UNSUPPORTED.
+ */
+int dp_fitting_grad_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                        const int64_t *type_start, const double *act, const double *g, double *dD, double *work,
+                        void *stream);
+int dp_fitting_grad_f32(const float *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
+                        const float *act, const float *g, float *dD, float *work, void *stream);
+/* The same in df64 arithmetic (double arrays; tanh itself in double). */
+int dp_fitting_fwd_df64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                        const int64_t *type_start, const double *D, double *E, double *act, void *stream);
+int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                         const int64_t *type_start, const double *act, const double *g, double *dD, double *work,
+                         void *stream);
+
 #ifdef __cplusplus
 }
 #endif

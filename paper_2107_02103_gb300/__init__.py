@@ -108,6 +108,12 @@ _SIGS = {
                                               ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_df64": ([_P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
     "dp_descriptor_contract_grad_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _P], ctypes.c_int),
+    "dp_fitting_fwd_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_fwd_f32": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_fwd_df64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_grad_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_grad_f32": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_grad_df64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_env_mat_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_df64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
 }
@@ -426,6 +432,58 @@ def dp_force_virial_df64(coord, nlist, env: dp_env_info, ds, dRt, out=None):
 def dp_table_build_df64(y, dy, d2y, info: dp_table_info, out=None) -> torch.Tensor:
     """dp_table_build(..., dtype="df64")."""
     return dp_table_build(y, dy, d2y, info, DF64, out)
+
+
+def _fit_shape(params, widths, type_start):
+    widths = [int(x) for x in widths]
+    ts = [int(x) for x in type_start]
+    ntypes = len(ts) - 1
+    P = sum((widths[l - 1] + 1) * widths[l] for l in range(1, len(widths)))
+    if params.dim() != 2 or params.shape[0] != ntypes or params.shape[1] != P:
+        raise ValueError(f"params must be [ntypes={ntypes}][{P}]")
+    H = sum(widths[1:-1])
+    return ((ctypes.c_int32 * len(widths))(*widths), len(widths) - 1, ntypes, (ctypes.c_int64 * len(ts))(*ts), ts[-1],
+            widths, H)
+
+
+def dp_fitting_fwd(params, widths, type_start, D, out=None, arith=None):
+    """(E [nloc], act [nloc][H]) of the fitting net; D [nloc][widths[0]] (a [nloc][M1][M2] descriptor is
+    flattened), atoms sorted by centre type with type_start [ntypes+1] (host); arith="df64" as elsewhere."""
+    params = _dev(params, "params", None)
+    dtype = params.dtype
+    w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
+    D = _dev(D, "D", dtype)
+    if D.shape[0] != nloc or D.numel() != nloc * widths[0]:
+        raise ValueError(f"D must hold [{nloc}][{widths[0]}]")
+    if out is None:
+        E = torch.empty((nloc,), dtype=dtype, device=params.device)
+        act = torch.empty((nloc, max(H, 1)), dtype=dtype, device=params.device)
+    else:
+        E = _dev(out[0], "E", dtype, (nloc,))
+        act = _dev(out[1], "act", dtype, (nloc, max(H, 1)))
+    fn = getattr(_lib, f"dp_fitting_fwd_{_suffix(arith or dtype)}")
+    _check(fn(_ptr(params), w, nlayer, ntypes, ts, _ptr(D), _ptr(E), _ptr(act), _stream(params)))
+    return E, act
+
+
+def dp_fitting_grad(params, widths, type_start, act, g=None, out=None, work=None, arith=None):
+    """dD [nloc][widths[0]] = g_i dE_i/dD_i from the forward's act; g [nloc] or None (all ones)."""
+    params = _dev(params, "params", None)
+    dtype = params.dtype
+    w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
+    act = _dev(act, "act", dtype, (nloc, max(H, 1)))
+    if g is not None:
+        g = _dev(g, "g", dtype, (nloc,))
+    dD = torch.empty((nloc, widths[0]), dtype=dtype, device=params.device) if out is None else \
+        _dev(out, "out", dtype, (nloc, widths[0]))
+    maxh = max(widths[1:-1]) if len(widths) > 2 else 1
+    if work is None:
+        work = torch.empty((2, nloc, maxh), dtype=dtype, device=params.device)
+    else:
+        work = _dev(work, "work", dtype, (2, nloc, maxh))
+    fn = getattr(_lib, f"dp_fitting_grad_{_suffix(arith or dtype)}")
+    _check(fn(_ptr(params), w, nlayer, ntypes, ts, _ptr(act), _ptr(g), _ptr(dD), _ptr(work), _stream(params)))
+    return dD
 
 
 @dataclass

@@ -132,6 +132,13 @@ def net_params(seed: int, widths, npair: int) -> np.ndarray:
     return out
 
 
+def fitting_net(seed: int, in_width: int, hidden=(240, 240, 240), ntypes: int = 1):
+    """Random fitting-net parameters, one row per centre type: widths (in_width, *hidden, 1), the
+    layout of net_params (W ~ N(0, 1/fan_in), b ~ N(0, 1)).  The paper's nets are (240, 240, 240)."""
+    widths = [int(in_width), *[int(h) for h in hidden], 1]
+    return widths, net_params(_sub_seed(seed, 505), widths, ntypes)
+
+
 @dataclass
 class Workload:
     """One synthetic batch of the tabulate-fusion path, host arrays.
