@@ -62,6 +62,27 @@ def footprint(w, esize: int, hbm_bytes: float = 280e9) -> dict:
             "atoms_per_280GB": int(hbm_bytes // ours), "atoms_per_280GB_uncompressed": int(hbm_bytes // (ours + net))}
 
 
+# the C entry point behind each timed kernel
+KERNEL_API = {"fwd": "dp_tabulate_fusion_fwd", "grad": "dp_tabulate_fusion_grad", "descriptor": "dp_descriptor_contract",
+              "descriptor_grad": "dp_descriptor_contract_grad", "fitting_fwd": "dp_fitting_fwd",
+              "fitting_grad": "dp_fitting_grad", "env_mat": "dp_env_mat", "force_virial": "dp_force_virial"}
+
+
+def fitting_model(w):
+    """The fitting net of the --fitting chain: the paper's (240, 240, 240) hidden layers per centre type
+    on the flattened descriptor, random-init (seeded) weights."""
+    import workloads as W
+    return W.fitting_net(W._sub_seed(w.seed, 606), w.M1 * w.M2, (240, 240, 240), w.ntypes)
+
+
+def fitting_fmas(w, widths) -> dict:
+    """FMAs per step of the fitting net: every layer's w_{l-1} w_l per atom forward, the hidden layers'
+    again backward (the output layer's backward is a scaling of its weights)."""
+    f = sum(widths[l - 1] * widths[l] for l in range(1, len(widths)))
+    b = sum(widths[l - 1] * widths[l] for l in range(1, len(widths) - 1))
+    return {"fitting_fwd": f * w.nloc, "fitting_grad": b * w.nloc}
+
+
 def chain_bytes(w, esize: int, nall: int) -> dict:
     """Algorithmic DRAM bytes of the chain's front and back end (the unique data each one must move):
     env_mat reads the neighbour list and the coordinates once and writes s, R~ (every row) and the counts;
@@ -262,9 +283,14 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     coord, nlist, _ = W.ghost_system(w)
     nv = w.env["norm"]
     env = dpc.env_info(w.env["rcs"], w.env["rc"], w.env["kind"], nv)
-    dD = W.normal(W._sub_seed(w.seed, 404), (w.nloc, w.M1, w.M2))
-    host = {"coord": np.ascontiguousarray(coord.astype(npdt)), "nlist": nlist, "atype": w.atype,
-            "dD": np.ascontiguousarray(dD.astype(npdt))}
+    host = {"coord": np.ascontiguousarray(coord.astype(npdt)), "nlist": nlist, "atype": w.atype}
+    if args.fitting:  # the energy of the whole model: dE/dD comes from the fitting net
+        fwidths, fparams = fitting_model(w)
+        fpar = torch.from_numpy(np.ascontiguousarray(fparams.astype(npdt))).to(dev)  # parameters stay resident
+        ts = [0] + [int(x) for x in np.cumsum(w.ncentre())]
+    else:
+        dD = W.normal(W._sub_seed(w.seed, 404), (w.nloc, w.M1, w.M2))
+        host["dD"] = np.ascontiguousarray(dD.astype(npdt))
     d = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
     work = dict(s=torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev),
                 Rt=torch.empty((w.nloc, w.nnei, 4), dtype=dtype, device=dev),
@@ -273,23 +299,41 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     outs = dict(D=D, F=torch.empty((coord.shape[0], 3), dtype=dtype, device=dev),
                 virial=torch.empty((3, 3), dtype=dtype, device=dev))
     names = ["env_mat", "fwd", "descriptor", "descriptor_grad", "grad", "force_virial"]
+    if args.fitting:
+        H = sum(fwidths[1:-1])
+        outs["E"] = torch.empty((w.nloc,), dtype=dtype, device=dev)
+        work["act"] = torch.empty((w.nloc, H), dtype=dtype, device=dev)
+        work["dD"] = torch.empty((w.nloc, w.M1 * w.M2), dtype=dtype, device=dev)
+        work["fit_scratch"] = torch.empty((2, w.nloc, max(fwidths[1:-1])), dtype=dtype, device=dev)
+        names = ["env_mat", "fwd", "descriptor", "fitting_fwd", "fitting_grad", "descriptor_grad", "grad",
+                 "force_virial"]
 
     def step(rec, x, o):
-        rec(0)
+        k = 0
+        rec(k)
         dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]), arith=arith)
-        rec(1)
+        rec(k := k + 1)
         fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
-        rec(2)
+        rec(k := k + 1)
         dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"], arith=arith)
-        rec(3)
-        dpc.dp_descriptor_contract_grad(work["T"], x["dD"], out=work["dT"], arith=arith)
-        rec(4)
+        rec(k := k + 1)
+        if args.fitting:
+            dpc.dp_fitting_fwd(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), arith=arith)
+            rec(k := k + 1)
+            dpc.dp_fitting_grad(fpar, fwidths, ts, work["act"], out=work["dD"], work=work["fit_scratch"],
+                                arith=arith)
+            rec(k := k + 1)
+            dD_in = work["dD"].view(w.nloc, w.M1, w.M2)
+        else:
+            dD_in = x["dD"]
+        dpc.dp_descriptor_contract_grad(work["T"], dD_in, out=work["dT"], arith=arith)
+        rec(k := k + 1)
         grad(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, work["dT"],
              out=(work["ds"], work["dRt"]))
-        rec(5)
+        rec(k := k + 1)
         dpc.dp_force_virial(x["coord"], x["nlist"], env, work["ds"], work["dRt"], out=(o["F"], o["virial"]),
                             arith=arith)
-        rec(6)
+        rec(k := k + 1)
     return host, d, outs, names, step
 
 
@@ -410,8 +454,9 @@ def measure_variants(args, w, dpc, info, sel, d, ref_outs, flush, stream, dev, f
 
 def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_all):
     """The metric end to end through the public API with host buffers: every step uploads its inputs
-    (s, R~, nvalid, atype, dT; with --chain coordinates, neighbour list, atype, dE/dD) from pinned host
-    memory and downloads its results (T, D, ds, dR~; with --chain D, forces and virial).  Steps
+    (s, R~, nvalid, atype, dT; with --chain coordinates, neighbour list, atype and dE/dD or, with
+    --fitting, nothing more) from pinned host memory and downloads its results (T, D, ds, dR~; with
+    --chain D, forces and virial, and with --fitting the atomic energies).  Steps
     are pipelined the way a streaming caller would run them: double-buffered device inputs and outputs,
     the upload of step k+1 and the download of step k-1 on their own streams while step k computes."""
     import torch
@@ -479,6 +524,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     flops = {"fwd": 2.0 * fmas["fwd"], "grad": 2.0 * fmas["grad"],
              "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc,
              "descriptor_grad": 2.0 * DESC_GRAD_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
+    if getattr(args, "fitting", False):
+        flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w)[0]).items()})
     nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
     pk = peak_tflops(args.dtype)
     kernels = {}
@@ -495,7 +542,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     path_tflops = (flops["fwd"] + flops["grad"]) / ((mean["fwd"] + mean["grad"]) * 1e-3) / 1e12
     roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
                 "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
-                "kernel": f"dp_tabulate_fusion_{dom}",
+                "kernel": KERNEL_API[dom],
                 "peak_basis": peak_basis(args.dtype),
                 "fwd_grad_frac": round(path_tflops / pk, 4)}
     out = {
@@ -505,7 +552,9 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         "config": {"workload": workload_label(w),
                    "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
                                    else f"atoms split over {world} ranks"),
-                   "step": ("env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain
+                   "step": (("env_mat + fwd + descriptor + fitting_fwd + fitting_grad + descriptor_grad + grad + "
+                             "force_virial (energy and forces of the whole model)") if args.fitting else
+                            "env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain
                             else "fwd + descriptor + grad"), "algo": args.algo,
                    "fma_basis": ("interval moments: per run min(9 M1 L, 24 M1 + 24 L) fwd, "
                                  "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
@@ -646,11 +695,15 @@ def main():
                     help="skip the per-row and df64 timings added to the default f64 line")
     ap.add_argument("--chain", action="store_true",
                     help="time the whole chain from coordinates to forces (env_mat ... force_virial)")
+    ap.add_argument("--fitting", action="store_true",
+                    help="with --chain: add the fitting net, so the step yields the model's energy and forces")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     if args.dtype == "df64" and args.algo != "moments":
         ap.error("--dtype df64 runs the moment path only")
+    if args.fitting and not args.chain:
+        ap.error("--fitting extends the --chain step")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
