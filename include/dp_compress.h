@@ -413,6 +413,28 @@ int dp_fitting_grad_f64(const double *params, const int32_t *widths, int nlayer,
                         void *stream);
 int dp_fitting_grad_f32(const float *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
                         const float *act, const float *g, float *dD, float *work, void *stream);
+/*
+ * dp_fitting_grad_f64 without a work argument, for callers that cannot
+ * allocate device memory or hand the library a scratch buffer -- an MD
+ * engine that sizes all device memory at start-up and passes a plugin only
+ * its inputs and outputs, where an allocation would synchronise the device
+ * mid-step.  (The paper has no counterpart; this is an interface for such
+ * callers.)  The scratch, 2 x nloc x (widest hidden layer) doubles, lives in
+ * a fixed 8 MiB array inside the library (1,048,576 doubles: 2,184 atoms at
+ * width 240), which every GPU that loads the library keeps until the process
+ * exits; larger problems return DP_ERR_UNSUPPORTED -- use the call with a
+ * work buffer.  Nothing is allocated: no cudaMalloc, no cudaFree, no
+ * allocating library routine.  The first call on a device looks the array's
+ * address up (cudaGetSymbolAddress) and keeps it; make that first call
+ * before any stream capture.  Every call on a device uses the same array and
+ * it keeps the last call's contents; the kernels overwrite every element they
+ * read, so nothing needs clearing, but calls that overlap on the GPU (on
+ * different streams, or from different threads) race on it.  Results are
+ * those of dp_fitting_grad_f64.  Arguments and errors as dp_fitting_grad_f64.
+ */
+int dp_fitting_grad_noalloc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                                const int64_t *type_start, const double *act, const double *g, double *dD,
+                                void *stream);
 /* The same in df64 arithmetic (double arrays; tanh itself in double). */
 int dp_fitting_fwd_df64(const double *params, const int32_t *widths, int nlayer, int ntypes,
                         const int64_t *type_start, const double *D, double *E, double *act, void *stream);

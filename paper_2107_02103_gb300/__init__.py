@@ -114,6 +114,7 @@ _SIGS = {
     "dp_fitting_grad_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_fitting_grad_f32": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_fitting_grad_df64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_grad_noalloc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_env_mat_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_df64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
 }
@@ -483,6 +484,21 @@ def dp_fitting_grad(params, widths, type_start, act, g=None, out=None, work=None
         work = _dev(work, "work", dtype, (2, nloc, maxh))
     fn = getattr(_lib, f"dp_fitting_grad_{_suffix(arith or dtype)}")
     _check(fn(_ptr(params), w, nlayer, ntypes, ts, _ptr(act), _ptr(g), _ptr(dD), _ptr(work), _stream(params)))
+    return dD
+
+
+def dp_fitting_grad_noalloc_f64(params, widths, type_start, act, g=None, out=None):
+    """dp_fitting_grad in f64 with the library's fixed scratch array: no work buffer and no device
+    allocation by the library (for callers that cannot allocate; see include/dp_compress.h)."""
+    params = _dev(params, "params", torch.float64)
+    w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
+    act = _dev(act, "act", torch.float64, (nloc, max(H, 1)))
+    if g is not None:
+        g = _dev(g, "g", torch.float64, (nloc,))
+    dD = torch.empty((nloc, widths[0]), dtype=torch.float64, device=params.device) if out is None else \
+        _dev(out, "out", torch.float64, (nloc, widths[0]))
+    _check(_lib.dp_fitting_grad_noalloc_f64(_ptr(params), w, nlayer, ntypes, ts, _ptr(act), _ptr(g), _ptr(dD),
+                                            _stream(params)))
     return dD
 
 

@@ -19,6 +19,8 @@
 // (f64) or the FP32 pipe (f32, df64).
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "dp_common.cuh"
 
 namespace dpc {
@@ -318,10 +320,74 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
   return DP_OK;
 }
 
+// ------------------------------------------------- backward without allocation
+// Some callers cannot hand this library a scratch buffer: an MD engine's force
+// loop that owns all device memory, sized once at start-up, and gives a plugin
+// only its input and output arrays -- allocating there would synchronise the
+// device in the middle of a time step and fragment the engine's pool.  For
+// them dp_fitting_grad_noalloc_f64 takes its scratch (the two buffers the
+// backward passes between layers) from this fixed array, which every GPU that
+// loads the library keeps until the process exits.
+constexpr size_t kStaticScratchDoubles = (size_t)1 << 20;  // 8 MiB
+static __device__ __align__(256) double g_fit_scratch[kStaticScratchDoubles];
+
+constexpr int kMaxScratchDevices = 64;
+std::atomic<double *> g_fit_scratch_addr[kMaxScratchDevices];  // per device, filled on its first call
+
+// Device address of the array on the current device.  In host code the array's
+// name only stands in for it; the address comes from the runtime, looked up on
+// the first call on each device and kept.
+int static_scratch(double **out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_fitting_grad_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
+  if (dev < 0 || dev >= kMaxScratchDevices)
+    return set_error(DP_ERR_UNSUPPORTED, "dp_fitting_grad_noalloc: device %d beyond the %d it tracks", dev,
+                     kMaxScratchDevices);
+  double *p = g_fit_scratch_addr[dev].load(std::memory_order_acquire);
+  if (!p) {
+    void *q = nullptr;
+    e = cudaGetSymbolAddress(&q, g_fit_scratch);
+    if (e != cudaSuccess)
+      return set_error(DP_ERR_CUDA, "dp_fitting_grad_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+    p = static_cast<double *>(q);
+    g_fit_scratch_addr[dev].store(p, std::memory_order_release);
+  }
+  *out = p;
+  return DP_OK;
+}
+
+int fitting_grad_noalloc(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                         const int64_t *type_start, const double *act, const double *g, double *dD, void *stream) {
+  clear_error();
+  FitShape s;
+  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
+  if (rc) return rc;
+  const int64_t nloc = s.start[ntypes];
+  const size_t need = nlayer > 2 ? (size_t)2 * (size_t)nloc * (size_t)s.maxh : 0;
+  if (need > kStaticScratchDoubles)
+    return set_error(DP_ERR_UNSUPPORTED,
+                     "dp_fitting_grad_noalloc: needs 2 x %lld atoms x %d = %zu doubles of scratch, the static array "
+                     "holds %zu; use dp_fitting_grad_f64 with a work buffer",
+                     (long long)nloc, s.maxh, need, kStaticScratchDoubles);
+  double *work = nullptr;
+  if (need > 0 && nloc > 0) {
+    rc = static_scratch(&work);
+    if (rc) return rc;
+  }
+  return fitting_grad<double>(params, widths, nlayer, ntypes, type_start, act, g, dD, work, stream);
+}
+
 }  // namespace
 }  // namespace dpc
 
 extern "C" {
+
+int dp_fitting_grad_noalloc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                                const int64_t *type_start, const double *act, const double *g, double *dD,
+                                void *stream) {
+  return dpc::fitting_grad_noalloc(params, widths, nlayer, ntypes, type_start, act, g, dD, stream);
+}
 
 int dp_fitting_fwd_f64(const double *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
                        const double *D, double *E, double *act, void *stream) {
