@@ -13,8 +13,8 @@
 // equal-width layers (the skips telescope: v_l = t_l + v_{l-1}), formed as
 // the operand is loaded.
 //
-// GEMM tiling: 64 x 64 output tiles, 256 threads with 4 x 4 outputs each,
-// 16-deep slices of both operands staged in shared memory.  Every FMA
+// GEMM tiling: small output tiles (FitTile below), 256 threads, 16-deep
+// slices of both operands staged in shared memory.  Every FMA
 // instruction has its 32 lanes busy; the kernels are bound by the FP64 pipe
 // (f64) or the FP32 pipe (f32, df64).
 #include <cuda_runtime.h>
@@ -26,7 +26,40 @@
 namespace dpc {
 namespace {
 
-constexpr int kBM = 64, kBN = 64, kBK = 16, kFitThreads = 256;
+// Output tile kBM x kBN per block, kTM x kTN per thread, 256 threads.
+template <int BM, int BN, int TM, int TN>
+struct Tile {
+  static constexpr int kBM = BM, kBN = BN, kTM = TM, kTN = TN, kTX = BN / TN;  // kTX: threads across columns
+  static_assert((BM / TM) * (BN / TN) == 256, "tile shape");
+};
+// By arithmetic and direction, measured on GB300 with the 240-wide nets of cu85 and water.  f64 is
+// bound by the FP64 pipe alone, so its tiles are small: a type's few thousand atoms must still make
+// many blocks per SM, or the SMs that get one block more than the others set the time (64 x 64
+// tiles give 256 blocks for 4096 atoms on 152 SMs, 84 % at best; 16 x 16 tiles 3840, 97 %).  The
+// backward's loader spends FP64 work on every element of A it stages (the factor 1 - t^2), once per
+// column tile, so there wider tiles (16 x 48) pay for themselves.  df64 and f32 feed the FP32 pipes,
+// where the shared-memory operand loads per product start to count: larger tiles.
+template <typename real, bool kFwd>
+struct FitTile {
+  using T = Tile<16, 48, 1, 3>;
+};
+template <>
+struct FitTile<double, true> {
+  using T = Tile<16, 16, 1, 1>;
+};
+template <bool kFwd>
+struct FitTile<float, kFwd> {
+  using T = Tile<64, 64, 4, 4>;
+};
+template <>
+struct FitTile<df64, true> {
+  using T = Tile<32, 48, 2, 3>;
+};
+template <>
+struct FitTile<df64, false> {
+  using T = Tile<64, 64, 4, 4>;
+};
+constexpr int kBK = 16, kFitThreads = 256;
 constexpr int kMaxChain = DP_MAX_LAYERS + 1;
 
 __device__ __forceinline__ double tanh_r(const double z) { return tanh(z); }
@@ -84,25 +117,27 @@ __device__ __forceinline__ real load_b(const FitGemm<real> &P, int k, int nn) {
 
 template <typename real, bool kFwd>
 __global__ void __launch_bounds__(kFitThreads) fit_gemm_kernel(const FitGemm<real> P) {
+  using TL = typename FitTile<real, kFwd>::T;
+  constexpr int kBM = TL::kBM, kBN = TL::kBN, kTM = TL::kTM, kTN = TL::kTN, kTX = TL::kTX;
   __shared__ real As[kBK][kBM + 1];
   __shared__ real Bs[kBK][kBN];
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  const int tx = threadIdx.x % kTX, ty = threadIdx.x / kTX;
   const int64_t m0 = (int64_t)blockIdx.y * kBM;
   const int n0 = blockIdx.x * kBN;
-  real acc[4][4];
+  real acc[kTM][kTN];
 #pragma unroll
-  for (int a = 0; a < 4; ++a)
+  for (int a = 0; a < kTM; ++a)
 #pragma unroll
-    for (int b = 0; b < 4; ++b) acc[a][b] = real(0);
+    for (int b = 0; b < kTN; ++b) acc[a][b] = real(0);
   for (int k0 = 0; k0 < P.K; k0 += kBK) {
-    // A slice [kBM][kBK] and B slice [kBK][kBN]: 1024 elements each, 4 per thread
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int e = threadIdx.x + q * kFitThreads;
+    // A slice [kBM][kBK] and B slice [kBK][kBN], spread over the threads
+    for (int e = threadIdx.x; e < kBM * kBK; e += kFitThreads) {
       const int am = e / kBK, ak = e - am * kBK;  // consecutive threads: consecutive k of one row
       const int64_t row = m0 + am;
       const int k = k0 + ak;
       As[ak][am] = (row < P.n && k < P.K) ? load_a<real, kFwd>(P, P.r0 + row, k) : real(0);
+    }
+    for (int e = threadIdx.x; e < kBK * kBN; e += kFitThreads) {
       const int bk = e / kBN, bn = e - bk * kBN;
       const int kb = k0 + bk, nb = n0 + bn;
       Bs[bk][bn] = (kb < P.K && nb < P.N) ? load_b<real, kFwd>(P, kb, nb) : real(0);
@@ -110,27 +145,26 @@ __global__ void __launch_bounds__(kFitThreads) fit_gemm_kernel(const FitGemm<rea
     __syncthreads();
 #pragma unroll
     for (int kk = 0; kk < kBK; ++kk) {
-      real a[4], b[4];
+      real a[kTM], b[kTN];
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        a[q] = As[kk][ty + 16 * q];
-        b[q] = Bs[kk][tx + 16 * q];
-      }
+      for (int q = 0; q < kTM; ++q) a[q] = As[kk][ty + (kBM / kTM) * q];
 #pragma unroll
-      for (int p = 0; p < 4; ++p)
+      for (int q = 0; q < kTN; ++q) b[q] = Bs[kk][tx + kTX * q];
 #pragma unroll
-        for (int q = 0; q < 4; ++q) acc[p][q] = fma(a[p], b[q], acc[p][q]);
+      for (int p = 0; p < kTM; ++p)
+#pragma unroll
+        for (int q = 0; q < kTN; ++q) acc[p][q] = fma(a[p], b[q], acc[p][q]);
     }
     __syncthreads();
   }
-  // epilogue: rows ty + 16 p, columns tx + 16 q (consecutive threads write consecutive columns)
+  // epilogue: rows ty + (kBM / kTM) p, columns tx + kTX q (consecutive threads write consecutive columns)
 #pragma unroll
-  for (int p = 0; p < 4; ++p) {
-    const int64_t row = m0 + ty + 16 * p;
+  for (int p = 0; p < kTM; ++p) {
+    const int64_t row = m0 + ty + (kBM / kTM) * p;
     if (row >= P.n) continue;
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int nn = n0 + tx + 16 * q;
+    for (int q = 0; q < kTN; ++q) {
+      const int nn = n0 + tx + kTX * q;
       if (nn >= P.N) continue;
       real v = acc[p][q];
       if constexpr (kFwd) {
@@ -222,11 +256,20 @@ void chain_sources(const FitShape &s, int l, const io_t<real> *D, const io_t<rea
   }
 }
 
+template <typename real, bool kFwd>
+int launch_gemm(const FitGemm<real> &G, cudaStream_t st, const char *who) {
+  using TL = typename FitTile<real, kFwd>::T;
+  const dim3 grid((unsigned)((G.N + TL::kBN - 1) / TL::kBN), (unsigned)((G.n + TL::kBM - 1) / TL::kBM));
+  if (grid.y > 65535u) return set_error(DP_ERR_SHAPE, "%s: too many atoms of one type (%lld)", who, (long long)G.n);
+  fit_gemm_kernel<real, kFwd><<<grid, kFitThreads, 0, st>>>(G);
+  return launch_status(who);
+}
+
 template <typename real>
 int fitting_fwd(const io_t<real> *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
                 const io_t<real> *D, io_t<real> *E, io_t<real> *act, void *stream) {
   clear_error();
-  FitShape s;
+  FitShape s{};
   int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
@@ -248,10 +291,7 @@ int fitting_fwd(const io_t<real> *params, const int32_t *widths, int nlayer, int
       G.bias = G.W + (size_t)G.K * G.N;
       G.out = act + s.aoff[l];
       G.ldo = s.H;
-      dim3 grid((unsigned)((G.N + kBN - 1) / kBN), (unsigned)((n + kBM - 1) / kBM));
-      if (grid.y > 65535u) return set_error(DP_ERR_SHAPE, "too many atoms of one type (%lld)", (long long)n);
-      fit_gemm_kernel<real, true><<<grid, kFitThreads, 0, st>>>(G);
-      rc = launch_status("dp_fitting_fwd");
+      rc = launch_gemm<real, true>(G, st, "dp_fitting_fwd");
       if (rc) return rc;
     }
     G.K = s.w[nlayer - 1];
@@ -269,7 +309,7 @@ template <typename real>
 int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start,
                  const io_t<real> *act, const io_t<real> *g, io_t<real> *dD, io_t<real> *work, void *stream) {
   clear_error();
-  FitShape s;
+  FitShape s{};
   int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
@@ -307,10 +347,7 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
         G.out = buf[cur];
         G.ldo = s.maxh;
       }
-      dim3 grid((unsigned)((G.N + kBN - 1) / kBN), (unsigned)((n + kBM - 1) / kBM));
-      if (grid.y > 65535u) return set_error(DP_ERR_SHAPE, "too many atoms of one type (%lld)", (long long)n);
-      fit_gemm_kernel<real, false><<<grid, kFitThreads, 0, st>>>(G);
-      rc = launch_status("dp_fitting_grad");
+      rc = launch_gemm<real, false>(G, st, "dp_fitting_grad");
       if (rc) return rc;
       S = G.out;
       ldS = G.ldo;
@@ -360,7 +397,7 @@ int static_scratch(double **out) {
 int fitting_grad_noalloc(const double *params, const int32_t *widths, int nlayer, int ntypes,
                          const int64_t *type_start, const double *act, const double *g, double *dD, void *stream) {
   clear_error();
-  FitShape s;
+  FitShape s{};
   int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
