@@ -62,6 +62,22 @@ def footprint(w, esize: int, hbm_bytes: float = 280e9) -> dict:
             "atoms_per_280GB": int(hbm_bytes // ours), "atoms_per_280GB_uncompressed": int(hbm_bytes // (ours + net))}
 
 
+# f64 fitting GEMMs on the tensor cores: every operand element is split into 11 digits and the 66 digit
+# products with s + t <= 12 run as fp16 MMAs, so a GEMM of 2 n K N FP64 flop issues 66 times as many
+# fp16 MMA flop; their roofline is the dense 16-bit tensor rate (fp16 and bf16 run at the same rate).
+TC_DIGIT_PRODUCTS = 66
+
+
+def tensor_peak() -> tuple:
+    """(TFLOP/s, basis): the measured dense bf16 GEMM burst rate, else the stated fallback."""
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured dense bf16 GEMM burst (MEASURED_PEAKS.json)"
+    except (OSError, KeyError, ValueError):
+        return 1900.0, "fallback 1.9 PFLOP/s dense bf16"
+
+
 # the C entry point behind each timed kernel
 KERNEL_API = {"fwd": "dp_tabulate_fusion_fwd", "grad": "dp_tabulate_fusion_grad", "descriptor": "dp_descriptor_contract",
               "descriptor_grad": "dp_descriptor_contract_grad", "fitting_fwd": "dp_fitting_fwd",
@@ -305,6 +321,9 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
         work["act"] = torch.empty((w.nloc, H), dtype=dtype, device=dev)
         work["dD"] = torch.empty((w.nloc, w.M1 * w.M2), dtype=dtype, device=dev)
         work["fit_scratch"] = torch.empty((2, w.nloc, max(fwidths[1:-1])), dtype=dtype, device=dev)
+        if args.fitting_tc:
+            work["fit_tc"] = torch.empty((dpc.dp_fitting_tc_work_bytes(fwidths, w.nloc),), dtype=torch.uint8,
+                                         device=dev)
         names = ["env_mat", "fwd", "descriptor", "fitting_fwd", "fitting_grad", "descriptor_grad", "grad",
                  "force_virial"]
 
@@ -317,7 +336,13 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
         rec(k := k + 1)
         dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"], arith=arith)
         rec(k := k + 1)
-        if args.fitting:
+        if args.fitting and args.fitting_tc:
+            dpc.dp_fitting_fwd_tc_f64(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), work=work["fit_tc"])
+            rec(k := k + 1)
+            dpc.dp_fitting_grad_tc_f64(fpar, fwidths, ts, work["act"], out=work["dD"], work=work["fit_tc"])
+            rec(k := k + 1)
+            dD_in = work["dD"].view(w.nloc, w.M1, w.M2)
+        elif args.fitting:
             dpc.dp_fitting_fwd(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), arith=arith)
             rec(k := k + 1)
             dpc.dp_fitting_grad(fpar, fwidths, ts, work["act"], out=work["dD"], work=work["fit_scratch"],
@@ -528,6 +553,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w)[0]).items()})
     nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
     pk = peak_tflops(args.dtype)
+    tc = bool(getattr(args, "fitting_tc", False))
+    tpk, tbasis = tensor_peak()
     kernels = {}
     for k in mean:
         e = {"ms": round(mean[k], 4), "share": round(mean[k] / sum(mean.values()), 4)}
@@ -536,15 +563,23 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
             e["frac"] = round(flops[k] / (mean[k] * 1e-3) / 1e12 / pk, 4)
         if k in nbytes:
             e["gbs"] = round(nbytes[k] / (mean[k] * 1e-3) / 1e9, 1)
+        if tc and k in ("fitting_fwd", "fitting_grad"):  # FP64-equivalent above; the MMAs it takes here
+            e["tensor_tflops"] = round(TC_DIGIT_PRODUCTS * flops[k] / (mean[k] * 1e-3) / 1e12, 2)
+            e["tensor_frac"] = round(e["tensor_tflops"] / tpk, 4)
         kernels[k] = e
     dom = max((k for k in mean if k in flops), key=mean.get)  # the roofline covers the FMA-counted kernels
     achieved = flops[dom] / (mean[dom] * 1e-3) / 1e12
     path_tflops = (flops["fwd"] + flops["grad"]) / ((mean["fwd"] + mean["grad"]) * 1e-3) / 1e12
+    api = KERNEL_API[dom] + ("_tc_f64" if tc and dom.startswith("fitting") else "")
     roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
                 "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
-                "kernel": KERNEL_API[dom],
+                "kernel": api,
                 "peak_basis": peak_basis(args.dtype),
                 "fwd_grad_frac": round(path_tflops / pk, 4)}
+    if tc and dom.startswith("fitting"):
+        roofline.update({"bound": "tensor", "achieved": kernels[dom]["tensor_tflops"], "peak": round(tpk, 1),
+                         "frac": kernels[dom]["tensor_frac"], "traffic": None,
+                         "peak_basis": f"{tbasis}; achieved counts all {TC_DIGIT_PRODUCTS} fp16 digit products"})
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sum(step_ms) / len(step_ms), "higher_is_better": True,
@@ -560,6 +595,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                                  "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
                                  else "per row: 9 M1 fwd, 18 M1 grad"),
                    "l2": "flushed between steps (256 MiB write)",
+                   **({"fitting_gemm": ("tensor cores: f64 by exact 11-digit splitting, fp16 MMAs"
+                                        if tc else "FP64 pipe")} if getattr(args, "fitting", False) else {}),
                    "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4),
                    "footprint": footprint(w, 4 if args.dtype == "f32" else 8)},
         "atoms_per_s": w.nloc * world * args.steps / total_s,
@@ -697,6 +734,8 @@ def main():
                     help="time the whole chain from coordinates to forces (env_mat ... force_virial)")
     ap.add_argument("--fitting", action="store_true",
                     help="with --chain: add the fitting net, so the step yields the model's energy and forces")
+    ap.add_argument("--fitting-tc", action="store_true",
+                    help="with --fitting --dtype f64: the fitting net's GEMMs on the tensor cores (exact splitting)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -704,6 +743,8 @@ def main():
         ap.error("--dtype df64 runs the moment path only")
     if args.fitting and not args.chain:
         ap.error("--fitting extends the --chain step")
+    if args.fitting_tc and (not args.fitting or args.dtype != "f64"):
+        ap.error("--fitting-tc needs --fitting and --dtype f64")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -36,6 +36,7 @@
 #ifndef DP_COMPRESS_H
 #define DP_COMPRESS_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -441,6 +442,35 @@ int dp_fitting_fwd_df64(const double *params, const int32_t *widths, int nlayer,
 int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer, int ntypes,
                          const int64_t *type_start, const double *act, const double *g, double *dD, double *work,
                          void *stream);
+
+/*
+ * The f64 fitting net with its hidden-layer GEMMs on the tensor cores.  Same
+ * inputs, outputs and results as dp_fitting_fwd_f64 / dp_fitting_grad_f64
+ * (Sec. II: E_i from D_i, and dE_i/dD_i), to f64 accuracy: every GEMM operand
+ * element is split exactly into eleven 5-bit digits scaled by its row's (A)
+ * or column's (B) power of two, the digit products run as fp16 MMAs whose
+ * fp32 sums are exact integers (at most 1024 of K per partial sum), and those
+ * partial sums are combined in f64.  Per output the error is below about
+ * K 2^-51 max_k |a_ik| max_k |b_kj| (an f64 dot product: K 2^-53 sum_k
+ * |a_ik b_kj|).  A row or column holding inf or NaN gives NaN outputs.  The
+ * paper computes the net in double; this is that computation on hardware
+ * whose FP64 rate is ~480 times below its fp16 tensor rate.
+ *   work, work_bytes  device scratch, caller-owned, 256-byte aligned, at least
+ *                     dp_fitting_tc_work_bytes(widths, nlayer, nloc) bytes:
+ *                     the weights' digit planes (rebuilt on every call) and,
+ *                     for the backward, the two [nloc][max hidden width]
+ *                     buffers between layers.  Calls sharing a work buffer
+ *                     must not overlap on the GPU.
+ * Errors as the f64 calls, plus DP_ERR_NULL / DP_ERR_SHAPE for a missing,
+ * short or misaligned work buffer.
+ */
+size_t dp_fitting_tc_work_bytes(const int32_t *widths, int nlayer, int64_t nloc); /* 0 on bad widths */
+int dp_fitting_fwd_tc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                          const int64_t *type_start, const double *D, double *E, double *act, void *work,
+                          size_t work_bytes, void *stream);
+int dp_fitting_grad_tc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
+                           const int64_t *type_start, const double *act, const double *g, double *dD, void *work,
+                           size_t work_bytes, void *stream);
 
 #ifdef __cplusplus
 }

@@ -115,6 +115,11 @@ _SIGS = {
     "dp_fitting_grad_f32": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_fitting_grad_df64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_fitting_grad_noalloc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P], ctypes.c_int),
+    "dp_fitting_tc_work_bytes": ([_P, ctypes.c_int, _I64], ctypes.c_size_t),
+    "dp_fitting_fwd_tc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P],
+                              ctypes.c_int),
+    "dp_fitting_grad_tc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P],
+                               ctypes.c_int),
     "dp_env_mat_df64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_df64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
 }
@@ -499,6 +504,60 @@ def dp_fitting_grad_noalloc_f64(params, widths, type_start, act, g=None, out=Non
         _dev(out, "out", torch.float64, (nloc, widths[0]))
     _check(_lib.dp_fitting_grad_noalloc_f64(_ptr(params), w, nlayer, ntypes, ts, _ptr(act), _ptr(g), _ptr(dD),
                                             _stream(params)))
+    return dD
+
+
+def dp_fitting_tc_work_bytes(widths, nloc) -> int:
+    """Bytes of device scratch dp_fitting_fwd_tc_f64 / dp_fitting_grad_tc_f64 need for nloc atoms."""
+    widths = [int(x) for x in widths]
+    w = (ctypes.c_int32 * len(widths))(*widths)
+    n = int(_lib.dp_fitting_tc_work_bytes(w, len(widths) - 1, int(nloc)))
+    if n == 0 and len(widths) > 2:
+        raise ValueError(f"bad fitting-net widths {widths}")
+    return n
+
+
+def _tc_work(work, widths, nloc, device):
+    need = dp_fitting_tc_work_bytes(widths, nloc)
+    if work is None:
+        return torch.empty((max(need, 1),), dtype=torch.uint8, device=device)
+    if not work.is_cuda or work.dtype != torch.uint8 or not work.is_contiguous() or work.numel() < need:
+        raise ValueError(f"work must be a contiguous CUDA uint8 tensor of at least {need} bytes")
+    return work
+
+
+def dp_fitting_fwd_tc_f64(params, widths, type_start, D, out=None, work=None):
+    """dp_fitting_fwd in f64 with the hidden-layer GEMMs on the tensor cores (exact digit splitting);
+    work: a uint8 CUDA tensor of dp_fitting_tc_work_bytes(widths, nloc) bytes, or None to allocate one."""
+    params = _dev(params, "params", torch.float64)
+    w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
+    D = _dev(D, "D", torch.float64)
+    if D.shape[0] != nloc or D.numel() != nloc * widths[0]:
+        raise ValueError(f"D must hold [{nloc}][{widths[0]}]")
+    if out is None:
+        E = torch.empty((nloc,), dtype=torch.float64, device=params.device)
+        act = torch.empty((nloc, max(H, 1)), dtype=torch.float64, device=params.device)
+    else:
+        E = _dev(out[0], "E", torch.float64, (nloc,))
+        act = _dev(out[1], "act", torch.float64, (nloc, max(H, 1)))
+    work = _tc_work(work, widths, nloc, params.device)
+    _check(_lib.dp_fitting_fwd_tc_f64(_ptr(params), w, nlayer, ntypes, ts, _ptr(D), _ptr(E), _ptr(act), _ptr(work),
+                                      work.numel(), _stream(params)))
+    return E, act
+
+
+def dp_fitting_grad_tc_f64(params, widths, type_start, act, g=None, out=None, work=None):
+    """dp_fitting_grad in f64 with the GEMMs on the tensor cores; work as dp_fitting_fwd_tc_f64."""
+    params = _dev(params, "params", torch.float64)
+    w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
+    act = _dev(act, "act", torch.float64, (nloc, max(H, 1)))
+    if g is not None:
+        g = _dev(g, "g", torch.float64, (nloc,))
+    dD = torch.empty((nloc, widths[0]), dtype=torch.float64, device=params.device) if out is None else \
+        _dev(out, "out", torch.float64, (nloc, widths[0]))
+    work = _tc_work(work, widths, nloc, params.device)
+    _check(_lib.dp_fitting_grad_tc_f64(_ptr(params), w, nlayer, ntypes, ts, _ptr(act), _ptr(g), _ptr(dD),
+                                       _ptr(work), work.numel(), _stream(params)))
     return dD
 
 

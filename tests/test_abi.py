@@ -20,7 +20,7 @@ def dpc():
 
 def declared():
     src = open(HEADER).read()
-    return sorted(set(re.findall(r"^\s*(?:int|const char \*)\s*(dp_\w+)\s*\(", src, flags=re.M)))
+    return sorted(set(re.findall(r"^\s*(?:int|size_t|const char \*)\s*(dp_\w+)\s*\(", src, flags=re.M)))
 
 
 def test_header_declares_the_boundary():
