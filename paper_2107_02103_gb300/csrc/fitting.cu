@@ -376,22 +376,29 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
 // against K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column
 // with an inf or NaN gives NaN outputs.
 //
-// Block tile 32 x 80 (ten warps of 16 x 16), 32-deep K slices: per slice the
-// block's A rows are split into 11 fp16 digit planes in shared memory (their
-// exponents found by a pass over the rows first), the pre-split B planes are
-// copied in, and each warp runs the 66 digit products of its tile as
-// m16n8k16 MMAs with fp32 accumulators, one per diagonal.
+// Block tile 64 x 48 (eight warps of 16 x 24: two per SM sub-partition, so
+// that each sub-partition's tensor unit gets the same work), 32-deep K slices,
+// two slices in shared memory: while the warps multiply one slice, the next
+// slice's digit planes arrive by cp.async.  The planes are made by a separate
+// pass, once per element: B's when the call starts, A's per chunk of rows
+// before each GEMM (with each row's exponent).  Each warp runs the 66 digit
+// products of its tile as m16n8k16 MMAs with fp32 accumulators, one per
+// diagonal and 8-column tile.  A is always a plain matrix: the forward keeps
+// each layer's input v_l (its tanh outputs plus the skip) in a work buffer,
+// and the backward's epilogue writes dE/dv (for the next skip) and
+// dE/dv (1 - t^2) (the next A).
 namespace tc {
 constexpr int kS = 11;  // digits per operand element
-constexpr int kBM = 32, kBN = 80, kBK = 32;
+constexpr int kBM = 64, kBN = 48, kBK = 32;
 constexpr int kLd = kBK + 8;  // shared row stride in halves (80 B): the 8 rows an ldmatrix reads hit 8 distinct bank groups
-constexpr int kWarpsN = kBN / 16, kWarps = (kBM / 16) * kWarpsN, kThreads = 32 * kWarps;
+constexpr int kNT = 3;  // 8-column MMA tiles per warp: warp tile 16 x 24
+constexpr int kWarpsN = kBN / (8 * kNT), kWarps = (kBM / 16) * kWarpsN, kThreads = 32 * kWarps;  // 4 x 2 warps
+static_assert(kWarps == 8, "two warps per SM sub-partition: more than 8 leave some with a third warp");
 constexpr int kFlushK = 1024;
 constexpr int kNonFinite = 1 << 20;  // exponent of a row or column holding inf or NaN
 constexpr size_t kSmemA = (size_t)kS * kBM * kLd * 2, kSmemB = (size_t)kS * kBN * kLd * 2;
-constexpr size_t kSmem = kSmemA + kSmemB + (size_t)(kBM + kBN) * sizeof(int);
+constexpr size_t kSmemE = (size_t)(kBM + kBN) * sizeof(int);  // row and column exponents
 static_assert((size_t)kS * kFlushK * 961 < (1u << 24), "fp32 diagonal sums must stay exact");
-static_assert((kS * kBN * (kBK / 8)) % kThreads == 0, "B copy: whole rounds");
 
 __host__ __device__ constexpr int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
@@ -435,6 +442,10 @@ __device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
                : "r"(addr));
 }
 
+__device__ __forceinline__ void ldmatrix_x2(uint32_t (&r)[2], uint32_t addr) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+}
+
 __device__ __forceinline__ void mma_f16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
   asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
                : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
@@ -445,99 +456,129 @@ __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src));
 }
 
-// B of one layer as digit planes [kS][Np][Kp] (fp16, column n's K values contiguous) and the column
-// exponents F [Np]; columns >= N and rows >= K are zero.  Forward: B[k][n] = W[k][n] (W is [K][N]);
-// backward: B[k][n] = W[n][k].  One warp per column.
-__global__ void __launch_bounds__(128) split_b_kernel(const double *__restrict__ W, int K, int N, bool fwd, int Np,
-                                                      int Kp, uint32_t *__restrict__ planes, int *__restrict__ Fexp) {
+// Rows of a matrix as digit planes [kS][rows_p][Kp] (fp16, a row's K values contiguous) with the
+// rows' exponents [rows_p]: element (r, k) of the source is X[r ld_r + k ld_k]; rows >= nrows and
+// columns >= K are zero.  One warp per row.  Used for the A operand (rows of the layer input) and
+// for B (forward: the columns of W, ld_r = 1, ld_k = N; backward: the rows of W).
+__global__ void __launch_bounds__(128) split_rows_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
+                                                         int64_t nrows, int K, int64_t rows_p, int Kp,
+                                                         uint32_t *__restrict__ planes, int *__restrict__ exps) {
   const int lane = threadIdx.x & 31;
-  const int n = blockIdx.x * 4 + (threadIdx.x >> 5);
-  if (n >= Np) return;  // warp-uniform
-  auto w = [&](int k) {
-    return (n < N && k < K) ? (fwd ? W[(size_t)k * N + n] : W[(size_t)n * K + k]) : 0.0;
-  };
+  const int64_t r = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (r >= rows_p) return;  // warp-uniform
+  const double *__restrict__ xr = X + (r < nrows ? r : 0) * ld_r;
+  auto x = [&](int k) { return (r < nrows && k < K) ? __ldg(xr + k * ld_k) : 0.0; };
   int eb = 0;
-  for (int k = lane; k < K; k += 32) eb = max(eb, exp_bits(w(k)));
-  const int F = exp_of_max(__reduce_max_sync(0xffffffffu, eb));
-  if (lane == 0) Fexp[n] = F;
+  for (int k = lane; k < K; k += 32) eb = max(eb, exp_bits(x(k)));
+  const int E = exp_of_max(__reduce_max_sync(0xffffffffu, eb));
+  if (lane == 0) exps[r] = E;
   for (int c2 = lane; c2 < Kp / 2; c2 += 32) {
-    const double x0 = w(2 * c2), x1 = w(2 * c2 + 1);
+    const double x0 = x(2 * c2), x1 = x(2 * c2 + 1);
     uint32_t h[kS];
-    digit_pairs(fixed55(x0, F), fixed55(x1, F), sign_pair(x0, x1), h);
+    digit_pairs(fixed55(x0, E), fixed55(x1, E), sign_pair(x0, x1), h);
 #pragma unroll
-    for (int s = 0; s < kS; ++s) planes[((size_t)s * Np + n) * (Kp / 2) + c2] = h[s];
+    for (int s = 0; s < kS; ++s) planes[((size_t)s * rows_p + r) * (Kp / 2) + c2] = h[s];
   }
 }
 
+// One hidden-layer GEMM of a chunk of one type's atoms: rows r0 .. r0 + n - 1 of the plain
+// row-major A [*][K] (as digit planes) times B (digit planes), K cut into ksplit shares (grid z) so
+// that even a few thousand atoms give enough blocks for every SM; the shares' f64 results go to
+// `part`, and epilogue_kernel sums them and applies the layer's epilogue.
+struct TcGemm {
+  int64_t r0, n;  // output rows r0 .. r0 + n - 1; A's planes hold rows 0 .. n - 1 of this chunk
+  int K, N;
+  const double *A;  // the layer input itself (forward: its skip term)
+  int64_t lda;
+  const uint16_t *aplanes;  // [kS][Mp][Kp]
+  const int *Eexp;          // [Mp]
+  int64_t Mp;
+  const uint16_t *planes;   // B: [kS][Np][Kp]
+  const int *Fexp;
+  int Np, Kp;
+  double *part;             // [ksplit][Mp][Np]: the f64 result of each share of K (grid z)
+  int slices_per_split;
+  bool skip;
+  // forward
+  const double *bias;
+  double *act;
+  int64_t ldact;
+  double *V;
+  int64_t ldv;
+  // backward
+  const double *S;  // NULL: S(row, col) = g_row wo_col
+  int64_t ldS;
+  const double *g, *wo;
+  const double *T;  // tanh outputs of the layer below (NULL: the last GEMM)
+  int64_t ldT;
+  double *Snext, *Z;
+  int64_t ldz;
+  double *out;
+  int64_t ldo;
+};
+
+constexpr size_t kStage = kSmemA + kSmemB;
+
 template <bool kFwd>
-__global__ void __launch_bounds__(kThreads) gemm_kernel(const FitGemm<double> P, const uint16_t *__restrict__ planes,
-                                                        const int *__restrict__ Fexp, int Np, int Kp) {
+__global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   extern __shared__ __align__(16) unsigned char smem[];
-  uint16_t *As = reinterpret_cast<uint16_t *>(smem);           // [kS][kBM][kLd]
-  uint16_t *Bs = reinterpret_cast<uint16_t *>(smem + kSmemA);  // [kS][kBN][kLd]
-  int *sE = reinterpret_cast<int *>(smem + kSmemA + kSmemB);   // row exponents [kBM]
-  int *sF = sE + kBM;                                          // column exponents [kBN]
+  int *sE = reinterpret_cast<int *>(smem + 2 * kStage);  // row exponents [kBM]
+  int *sF = sE + kBM;                                    // column exponents [kBN]
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int wm = warp / kWarpsN, wn = warp - wm * kWarpsN;
   const int64_t m0 = (int64_t)blockIdx.y * kBM;
   const int n0 = blockIdx.x * kBN;
-
-  // row exponents of the block's rows over the whole of K, and the columns' exponents
-  for (int r = warp; r < kBM; r += kWarps) {
-    const int64_t row = m0 + r;
-    int eb = 0;
-    if (row < P.n)
-      for (int k = lane; k < P.K; k += 32) eb = max(eb, exp_bits(load_a<double, kFwd>(P, P.r0 + row, k)));
-    eb = __reduce_max_sync(0xffffffffu, eb);
-    if (lane == 0) sE[r] = exp_of_max(eb);
+  for (int c = threadIdx.x; c < kBM + kBN; c += kThreads) {
+    if (c < kBM)
+      sE[c] = P.Eexp[m0 + c];
+    else
+      sF[c - kBM] = P.Fexp[n0 + c - kBM];
   }
-  for (int c = threadIdx.x; c < kBN; c += kThreads) sF[c] = Fexp[n0 + c];
-  __syncthreads();
 
-  float acc[kS][2][4];
+  // the digit planes of slice k0, A then B: kS x (kBM + kBN) rows of kBK halves, 16 B a copy
+  auto copy_slice = [&](int k0, int buf) {
+    uint16_t *As = reinterpret_cast<uint16_t *>(smem + buf * kStage);
+    uint16_t *Bs = reinterpret_cast<uint16_t *>(smem + buf * kStage + kSmemA);
+#pragma unroll 1
+    for (int e = threadIdx.x; e < kS * (kBM + kBN) * (kBK / 8); e += kThreads) {
+      const int s = e / ((kBM + kBN) * (kBK / 8)), rem = e - s * (kBM + kBN) * (kBK / 8);
+      const int rr = rem / (kBK / 8), kc = rem - rr * (kBK / 8);
+      if (rr < kBM)
+        cp_async16(smem_u32(As + (s * kBM + rr) * kLd + kc * 8),
+                   P.aplanes + ((size_t)s * P.Mp + m0 + rr) * P.Kp + k0 + kc * 8);
+      else
+        cp_async16(smem_u32(Bs + (s * kBN + rr - kBM) * kLd + kc * 8),
+                   P.planes + ((size_t)s * P.Np + n0 + rr - kBM) * P.Kp + k0 + kc * 8);
+    }
+    asm volatile("cp.async.commit_group;");
+  };
+
+  float acc[kS][kNT][4];
 #pragma unroll
   for (int d = 0; d < kS; ++d)
 #pragma unroll
-    for (int j = 0; j < 2; ++j)
+    for (int j = 0; j < kNT; ++j)
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[d][j][c] = 0.f;
-  double acc64[2][4];
+  double acc64[kNT][4];
 #pragma unroll
-  for (int j = 0; j < 2; ++j)
+  for (int j = 0; j < kNT; ++j)
 #pragma unroll
     for (int c = 0; c < 4; ++c) acc64[j][c] = 0.0;
 
+  copy_slice(blockIdx.z * P.slices_per_split * kBK, 0);
+  asm volatile("cp.async.wait_all;" ::: "memory");
+  __syncthreads();
+  // this block's share of K: slices i0 .. i1 - 1
+  const int i0 = blockIdx.z * P.slices_per_split;
+  const int i1 = min((P.K + kBK - 1) / kBK, i0 + P.slices_per_split);
   int since_flush = 0;
-  for (int k0 = 0; k0 < P.K; k0 += kBK) {  // uniform
-    // B planes: kS x kBN rows of kBK halves, 16 B per copy
-#pragma unroll 1
-    for (int e = threadIdx.x; e < kS * kBN * (kBK / 8); e += kThreads) {
-      const int s = e / (kBN * (kBK / 8)), rem = e - s * kBN * (kBK / 8);
-      const int nn = rem / (kBK / 8), kc = rem - nn * (kBK / 8);
-      cp_async16(smem_u32(Bs + (s * kBN + nn) * kLd + kc * 8),
-                 planes + ((size_t)s * Np + n0 + nn) * Kp + k0 + kc * 8);
-    }
-    asm volatile("cp.async.commit_group;");
-    // A: the block's rows split into digit planes, two adjacent columns per thread
-    uint32_t *As32 = reinterpret_cast<uint32_t *>(As);
-#pragma unroll 1
-    for (int e = threadIdx.x; e < kBM * kBK / 2; e += kThreads) {
-      const int r = e / (kBK / 2), c2 = e - r * (kBK / 2);
-      const int64_t row = m0 + r;
-      const int k = k0 + 2 * c2;
-      double x0 = 0.0, x1 = 0.0;
-      if (row < P.n) {
-        if (k < P.K) x0 = load_a<double, kFwd>(P, P.r0 + row, k);
-        if (k + 1 < P.K) x1 = load_a<double, kFwd>(P, P.r0 + row, k + 1);
-      }
-      const int E = sE[r];
-      uint32_t h[kS];
-      digit_pairs(fixed55(x0, E), fixed55(x1, E), sign_pair(x0, x1), h);
-#pragma unroll
-      for (int s = 0; s < kS; ++s) As32[(s * kBM + r) * (kLd / 2) + c2] = h[s];
-    }
-    asm volatile("cp.async.wait_all;" ::: "memory");
-    __syncthreads();
+  for (int i = i0; i < i1; ++i) {  // uniform
+    const int cur = (i - i0) & 1;
+    const bool more = i + 1 < i1;
+    if (more) copy_slice((i + 1) * kBK, cur ^ 1);  // the next slice's copies fly while this one multiplies
+    const uint16_t *As = reinterpret_cast<const uint16_t *>(smem + cur * kStage);
+    const uint16_t *Bs = reinterpret_cast<const uint16_t *>(smem + cur * kStage + kSmemA);
 #pragma unroll
     for (int ks = 0; ks < kBK / 16; ++ks) {
       uint32_t a[kS][4];
@@ -546,25 +587,27 @@ __global__ void __launch_bounds__(kThreads) gemm_kernel(const FitGemm<double> P,
         ldmatrix_x4(a[s], smem_u32(As + (s * kBM + wm * 16 + (lane & 15)) * kLd + ks * 16 + (lane >> 4) * 8));
 #pragma unroll
       for (int t = 0; t < kS; ++t) {
-        uint32_t b[4];
-        ldmatrix_x4(b, smem_u32(Bs + (t * kBN + wn * 16 + (lane & 7) + ((lane >> 4) << 3)) * kLd + ks * 16 +
-                                ((lane >> 3) & 1) * 8));
+        // B fragments of the warp's three 8-column tiles: an x4 load for the first two, an x2 for the third
+        const uint16_t *bt = Bs + (t * kBN + wn * 8 * kNT) * kLd + ks * 16 + ((lane >> 3) & 1) * 8;
+        uint32_t b[4], b2[2];
+        ldmatrix_x4(b, smem_u32(bt + ((lane & 7) + ((lane >> 4) << 3)) * kLd));
+        ldmatrix_x2(b2, smem_u32(bt + (16 + (lane & 7)) * kLd));
 #pragma unroll
         for (int s = 0; s + t < kS; ++s) {  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
           mma_f16(acc[s + t][0], a[s], b[0], b[1]);
           mma_f16(acc[s + t][1], a[s], b[2], b[3]);
+          mma_f16(acc[s + t][2], a[s], b2[0], b2[1]);
         }
       }
     }
-    __syncthreads();
     since_flush += kBK;
-    if (since_flush == kFlushK || k0 + kBK >= P.K) {  // uniform: the diagonals into f64, smallest first
+    if (since_flush == kFlushK || !more) {  // uniform: the diagonals into f64, smallest first
       since_flush = 0;
 #pragma unroll
       for (int d = kS - 1; d >= 0; --d) {
         const double scale = __hiloint2double((1023 - 5 * (d + 2)) << 20, 0);  // 32^-(d + 2)
 #pragma unroll
-        for (int j = 0; j < 2; ++j)
+        for (int j = 0; j < kNT; ++j)
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
             acc64[j][c] = fma(dfl::widen(acc[d][j][c]), scale, acc64[j][c]);
@@ -572,33 +615,80 @@ __global__ void __launch_bounds__(kThreads) gemm_kernel(const FitGemm<double> P,
           }
       }
     }
+    asm volatile("cp.async.wait_all;" ::: "memory");  // buffer cur ^ 1 was last read before the previous barrier
+    __syncthreads();
   }
 
-  // epilogue: lane (gid, tig) holds rows gid and gid + 8, columns 2 tig and 2 tig + 1 of each 8-wide tile
+  // the share's f64 result, scaled by the row and column powers of two: lane (gid, tig) holds rows
+  // gid and gid + 8, columns 2 tig and 2 tig + 1 of each 8-wide tile (planes are padded: no bounds)
   const int gid = lane >> 2, tig = lane & 3;
+  double *part = P.part + (size_t)blockIdx.z * P.Mp * P.Np;
 #pragma unroll
-  for (int j = 0; j < 2; ++j)
+  for (int j = 0; j < kNT; ++j)
 #pragma unroll
-    for (int c = 0; c < 4; ++c) {
-      const int rl = wm * 16 + gid + (c >= 2 ? 8 : 0), cl = wn * 16 + j * 8 + 2 * tig + (c & 1);
-      const int64_t row = m0 + rl;
-      const int nn = n0 + cl;
-      if (row >= P.n || nn >= P.N) continue;
-      const int E = sE[rl], F = sF[cl];
-      double v = (E >= kNonFinite || F >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
-                                                     : scalbn(acc64[j][c], E + F);
-      if constexpr (kFwd) {
-        v = tanh(v + P.bias[nn]);
-      } else if (P.skip) {
-        const int64_t r = P.r0 + row;
-        v += P.S ? P.S[r * P.ldS + nn] : (P.g ? P.g[r] : 1.0) * P.wo[nn];
-      }
-      P.out[(P.r0 + row) * P.ldo + nn] = v;
+    for (int h = 0; h < 2; ++h) {
+      const int rl = wm * 16 + gid + 8 * h, cl = wn * 8 * kNT + j * 8 + 2 * tig;
+      const int E = sE[rl];
+      double2 v;
+      v.x = (E >= kNonFinite || sF[cl] >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
+                                                     : scalbn(acc64[j][2 * h], E + sF[cl]);
+      v.y = (E >= kNonFinite || sF[cl + 1] >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
+                                                         : scalbn(acc64[j][2 * h + 1], E + sF[cl + 1]);
+      *reinterpret_cast<double2 *>(part + (size_t)(m0 + rl) * P.Np + n0 + cl) = v;
     }
 }
 
+// The layer's epilogue over the chunk's n x N outputs, from the shares' partial results summed in
+// a fixed order (so a call's results do not depend on timing):
+//   forward:  t = tanh(acc + bias); act[row][col] = t; V[row][col] = t (+ A[row][col] when the layer
+//             keeps its width: the identity skip, v_l = t_l + v_{l-1})
+//   backward: s = acc (+ S[row][col] or g_row wo_col when the layer kept its width); then either
+//             out[row][col] = s (dE/dD, the last GEMM) or S_next[row][col] = s and
+//             Z[row][col] = s (1 - t_prev^2) with t_prev = T[row][col] (the next GEMM's A)
+template <bool kFwd>
+__global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int ksplit) {
+  const int64_t total = P.n * P.N;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t rc = e / P.N;
+    const int nn = (int)(e - rc * P.N);
+    const int64_t row = P.r0 + rc;
+    double v = P.part[rc * P.Np + nn];
+    for (int z = 1; z < ksplit; ++z) v += P.part[((size_t)z * P.Mp + rc) * P.Np + nn];
+    if constexpr (kFwd) {
+      const double t = tanh(v + P.bias[nn]);
+      P.act[row * P.ldact + nn] = t;
+      P.V[row * P.ldv + nn] = P.skip ? t + P.A[row * P.lda + nn] : t;
+    } else {
+      if (P.skip) v += P.S ? P.S[row * P.ldS + nn] : (P.g ? P.g[row] : 1.0) * P.wo[nn];
+      if (P.T) {
+        const double t = P.T[row * P.ldT + nn];
+        P.Snext[row * P.ldz + nn] = v;
+        P.Z[row * P.ldz + nn] = v * fma(-t, t, 1.0);
+      } else {
+        P.out[row * P.ldo + nn] = v;
+      }
+    }
+  }
+}
+
+// dz of the last hidden layer: Z[row][k] = g_row wo_k (1 - t_k^2), t its tanh outputs
+__global__ void __launch_bounds__(256) last_dz_kernel(int64_t r0, int64_t n, int K, const double *__restrict__ g,
+                                                      const double *__restrict__ wo, const double *__restrict__ T,
+                                                      int64_t ldT, double *__restrict__ Z, int64_t ldz) {
+  const int64_t total = n * K;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t row = r0 + e / K;
+    const int k = (int)(e - (e / K) * K);
+    const double t = T[row * ldT + k];
+    Z[row * ldz + k] = (g ? g[row] : 1.0) * wo[k] * fma(-t, t, 1.0);
+  }
+}
+
 // Where the B planes and column exponents of each hidden-layer GEMM of one type sit in the work
-// buffer (forward: layers 1 .. L-1; backward: L-1 .. 1), and the bytes they take.
+// buffer (forward: layers 1 .. L-1; backward: L-1 .. 1).  After them come the A planes and row
+// exponents of one chunk of at most kChunkRows atoms, and the [nloc][max hidden width] buffers
+// between layers (forward: 2, backward: 4).
+constexpr int64_t kChunkRows = 16384;
 struct Layer {
   int K, N, Np, Kp;
   size_t planes, fexp;  // byte offsets
@@ -620,38 +710,105 @@ size_t layout(const FitShape &s, bool fwd, Layer *out) {
   return off;
 }
 
-size_t work_bytes(const FitShape &s, int64_t nloc) {
+struct WorkMap {
+  size_t bplanes;          // bytes of the B planes (the larger of the two directions)
+  size_t aplanes, aexp;    // byte offsets of the A planes and row exponents of one chunk
+  int64_t Mp;              // rows of A planes per chunk
+  int Kpmax;
+  size_t part;             // byte offset of the shares' partial results
+  size_t buffers;          // byte offset of the buffers between layers
+};
+
+// K shares of one GEMM: enough that tiles x shares reaches kTargetBlocks (~6.7 waves of one block
+// per SM on 152 SMs), but at least kMinShareSlices slices per share (a block's first slice arrives
+// before any MMA can start; shorter shares spend their time waiting for it).  Shares x tiles x
+// tile stays below kTargetBlocks x tile + Mp x Np, which bounds the partial-result buffer.
+constexpr int64_t kTargetBlocks = 1024;
+constexpr int kMinShareSlices = 8;
+int ksplit_for(int64_t Mp, int Np, int Kp) {
+  const int64_t tiles = (Mp / kBM) * (Np / kBN);
+  const int slices = Kp / kBK;
+  const int64_t want = std::min<int64_t>((kTargetBlocks + tiles - 1) / tiles, std::max(1, slices / kMinShareSlices));
+  const int per = (int)((slices + want - 1) / want);
+  return (slices + per - 1) / per;  // no empty share
+}
+WorkMap work_map(const FitShape &s, int64_t nloc) {
   Layer L[DP_MAX_LAYERS];
-  size_t b = std::max(layout(s, true, L), layout(s, false, L));
-  if (s.nlayer > 2) b += (size_t)2 * (size_t)nloc * (size_t)s.maxh * sizeof(double);
-  return b;
+  WorkMap m{};
+  m.bplanes = std::max(layout(s, true, L), layout(s, false, L));
+  int kmax = 1;
+  for (int l = 0; l < s.nlayer; ++l) kmax = std::max(kmax, s.w[l]);  // every GEMM's K is a layer width
+  m.Kpmax = (int)round_up(kmax, kBK);
+  int64_t maxn = 0;  // rows of the largest type
+  for (int t = 0; t < s.ntypes; ++t) maxn = std::max<int64_t>(maxn, s.start[t + 1] - s.start[t]);
+  m.Mp = round_up(std::min<int64_t>(std::max<int64_t>(maxn, 1), kChunkRows), kBM);
+  m.aplanes = m.bplanes;
+  m.aexp = m.aplanes + (size_t)round_up((int64_t)kS * m.Mp * m.Kpmax * 2, 256);
+  m.part = m.aexp + (size_t)round_up(m.Mp * 4, 256);
+  int Npmax = kBN;
+  for (int l = 0; l < s.nlayer; ++l) Npmax = std::max(Npmax, (int)round_up(s.w[l], kBN));
+  m.buffers = m.part + (size_t)round_up((kTargetBlocks * kBM * kBN + m.Mp * Npmax) * 8, 256);
+  return m;
+}
+
+size_t work_bytes(const FitShape &s, int64_t nloc) {
+  const WorkMap m = work_map(s, nloc);
+  return m.buffers + (s.nlayer > 1 ? (size_t)4 * (size_t)nloc * (size_t)s.maxh * sizeof(double) : 0);
 }
 
 int set_smem() {
   static std::atomic<bool> done{false};
   if (done.load(std::memory_order_acquire)) return DP_OK;
   for (auto k : {&gemm_kernel<true>, &gemm_kernel<false>}) {
-    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem);
+    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(2 * kStage + kSmemE));
     if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_fitting_*_tc_f64: %s", cudaGetErrorString(e));
   }
   done.store(true, std::memory_order_release);
   return DP_OK;
 }
 
-int split(const double *W, const Layer &L, bool fwd, unsigned char *work, cudaStream_t st, const char *who) {
-  split_b_kernel<<<(unsigned)((L.Np + 3) / 4), 128, 0, st>>>(W, L.K, L.N, fwd, L.Np, L.Kp,
-                                                            reinterpret_cast<uint32_t *>(work + L.planes),
-                                                            reinterpret_cast<int *>(work + L.fexp));
+int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp,
+               unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
+  split_rows_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp,
+                                                                   reinterpret_cast<uint32_t *>(planes),
+                                                                   reinterpret_cast<int *>(exps));
   return launch_status(who);
 }
 
+// The weights of one layer as B planes: forward B[k][n] = W[k][n] (W is [K][N]), backward B[k][n] = W[n][k]
+int split_b(const double *W, const Layer &L, bool fwd, unsigned char *work, cudaStream_t st, const char *who) {
+  return fwd ? split_rows(W, 1, L.N, L.N, L.K, L.Np, L.Kp, work + L.planes, work + L.fexp, st, who)
+             : split_rows(W, L.K, 1, L.N, L.K, L.Np, L.Kp, work + L.planes, work + L.fexp, st, who);
+}
+
+// G over its rows in chunks of at most kChunkRows: each chunk's A rows split into planes, then the GEMM
 template <bool kFwd>
-int gemm(const FitGemm<double> &G, const Layer &L, const unsigned char *work, cudaStream_t st, const char *who) {
-  const dim3 grid((unsigned)(L.Np / kBN), (unsigned)((G.n + kBM - 1) / kBM));
-  if (grid.y > 65535u) return set_error(DP_ERR_SHAPE, "%s: too many atoms of one type (%lld)", who, (long long)G.n);
-  gemm_kernel<kFwd><<<grid, kThreads, kSmem, st>>>(G, reinterpret_cast<const uint16_t *>(work + L.planes),
-                                                   reinterpret_cast<const int *>(work + L.fexp), L.Np, L.Kp);
-  return launch_status(who);
+int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaStream_t st, const char *who) {
+  G.planes = reinterpret_cast<const uint16_t *>(work + L.planes);
+  G.Fexp = reinterpret_cast<const int *>(work + L.fexp);
+  G.Np = L.Np;
+  G.Kp = L.Kp;
+  G.aplanes = reinterpret_cast<const uint16_t *>(work + m.aplanes);
+  G.Eexp = reinterpret_cast<const int *>(work + m.aexp);
+  G.part = reinterpret_cast<double *>(work + m.part);
+  const int64_t r_end = G.r0 + G.n;
+  for (int64_t r0 = G.r0; r0 < r_end; r0 += kChunkRows) {
+    TcGemm C = G;
+    C.r0 = r0;
+    C.n = std::min<int64_t>(kChunkRows, r_end - r0);
+    C.Mp = round_up(C.n, kBM);
+    int rc = split_rows(G.A + r0 * G.lda, G.lda, 1, C.n, G.K, C.Mp, L.Kp, work + m.aplanes, work + m.aexp, st, who);
+    if (rc) return rc;
+    const int ksplit = ksplit_for(C.Mp, L.Np, L.Kp);
+    C.slices_per_split = (L.Kp / kBK + ksplit - 1) / ksplit;
+    const dim3 grid((unsigned)(L.Np / kBN), (unsigned)(C.Mp / kBM), (unsigned)ksplit);
+    gemm_kernel<kFwd><<<grid, kThreads, 2 * kStage + kSmemE, st>>>(C);
+    if ((rc = launch_status(who))) return rc;
+    const int64_t total = C.n * C.N;
+    epilogue_kernel<kFwd><<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(C, ksplit);
+    if ((rc = launch_status(who))) return rc;
+  }
+  return DP_OK;
 }
 
 int check_work(const FitShape &s, int64_t nloc, const void *work, size_t nbytes, const char *who) {
@@ -677,30 +834,45 @@ int fwd(const double *params, const int32_t *widths, int nlayer, int ntypes, con
   unsigned char *wk = static_cast<unsigned char *>(work);
   Layer L[DP_MAX_LAYERS];
   layout(s, true, L);
+  const WorkMap m = work_map(s, nloc);
+  double *V[2] = {reinterpret_cast<double *>(wk + m.buffers), nullptr};
+  V[1] = V[0] + (size_t)nloc * s.maxh;
   for (int t = 0; t < ntypes; ++t) {
     const int64_t n = s.start[t + 1] - s.start[t];
     if (n == 0) continue;
     const double *pt = params + (size_t)t * s.P;
     for (int l = 1; l < nlayer; ++l)  // this type's weights as digit planes (the previous type's are done with)
-      if ((rc = split(pt + s.woff[l], L[l - 1], true, wk, st, who))) return rc;
-    FitGemm<double> G{};
-    G.r0 = s.start[t];
-    G.n = n;
+      if ((rc = split_b(pt + s.woff[l], L[l - 1], true, wk, st, who))) return rc;
+    const double *in = D;  // v_{l-1}: D, then the layer outputs with their skips
+    int64_t ldin = s.w[0];
     for (int l = 1; l < nlayer; ++l) {
+      TcGemm G{};
+      G.r0 = s.start[t];
+      G.n = n;
       G.K = s.w[l - 1];
       G.N = s.w[l];
-      chain_sources<double>(s, l, D, act, G);
-      G.W = pt + s.woff[l];
-      G.bias = G.W + (size_t)G.K * G.N;
-      G.out = act + s.aoff[l];
-      G.ldo = s.H;
-      if ((rc = gemm<true>(G, L[l - 1], wk, st, who))) return rc;
+      G.A = in;
+      G.lda = ldin;
+      G.skip = s.w[l] == s.w[l - 1];
+      G.bias = pt + s.woff[l] + (size_t)G.K * G.N;
+      G.act = act + s.aoff[l];
+      G.ldact = s.H;
+      G.V = V[(l - 1) & 1];
+      G.ldv = s.maxh;
+      if ((rc = gemm<true>(G, L[l - 1], wk, m, st, who))) return rc;
+      in = G.V;
+      ldin = G.ldv;
     }
-    G.K = s.w[nlayer - 1];
-    G.N = 1;
-    chain_sources<double>(s, nlayer, D, act, G);
-    G.wo = pt + s.woff[nlayer];
-    fit_out_kernel<double><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(G, G.wo + G.K, E);
+    FitGemm<double> O{};  // output layer: E_i = v_{L-1} . wo + bo
+    O.r0 = s.start[t];
+    O.n = n;
+    O.K = s.w[nlayer - 1];
+    O.N = 1;
+    O.src[0] = in;
+    O.lds[0] = ldin;
+    O.nsrc = 1;
+    O.wo = pt + s.woff[nlayer];
+    fit_out_kernel<double><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(O, O.wo + O.K, E);
     if ((rc = launch_status(who))) return rc;
   }
   return DP_OK;
@@ -721,43 +893,52 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
   Layer L[DP_MAX_LAYERS];
-  Layer Lf[DP_MAX_LAYERS];
-  const size_t planes = std::max(layout(s, true, Lf), layout(s, false, L));
-  double *buf[2] = {reinterpret_cast<double *>(wk + planes),
-                    reinterpret_cast<double *>(wk + planes) + (size_t)nloc * s.maxh};
+  layout(s, false, L);
+  const WorkMap m = work_map(s, nloc);
+  double *buf = reinterpret_cast<double *>(wk + m.buffers);
+  const size_t bs = (size_t)nloc * s.maxh;
+  double *Z[2] = {buf, buf + bs}, *Sb[2] = {buf + 2 * bs, buf + 3 * bs};
   for (int t = 0; t < ntypes; ++t) {
     const int64_t n = s.start[t + 1] - s.start[t];
     if (n == 0) continue;
     const double *pt = params + (size_t)t * s.P;
     for (int q = 0; q + 1 < nlayer; ++q)
-      if ((rc = split(pt + s.woff[nlayer - 1 - q], L[q], false, wk, st, who))) return rc;
-    FitGemm<double> G{};
-    G.r0 = s.start[t];
-    G.n = n;
-    G.g = g;
-    G.wo = pt + s.woff[nlayer];
-    const double *S = nullptr;
-    int64_t ldS = 0;
+      if ((rc = split_b(pt + s.woff[nlayer - 1 - q], L[q], false, wk, st, who))) return rc;
+    const double *wo = pt + s.woff[nlayer];
+    {  // dz of the last hidden layer
+      const int K = s.w[nlayer - 1];
+      const int64_t total = n * K;
+      const unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 8);
+      last_dz_kernel<<<blocks, 256, 0, st>>>(s.start[t], n, K, g, wo, act + s.aoff[nlayer - 1], s.H, Z[0], s.maxh);
+      if ((rc = launch_status(who))) return rc;
+    }
+    const double *S = nullptr;  // dE/dv of the layer being walked; NULL: g wo (the last hidden layer)
     int cur = 0;
     for (int l = nlayer - 1; l >= 1; --l) {
+      TcGemm G{};
+      G.r0 = s.start[t];
+      G.n = n;
       G.K = s.w[l];
       G.N = s.w[l - 1];
-      G.S = S;
-      G.ldS = ldS;
-      G.T = act + s.aoff[l];
-      G.ldT = s.H;
-      G.W = pt + s.woff[l];
+      G.A = Z[cur];
+      G.lda = s.maxh;
       G.skip = s.w[l] == s.w[l - 1];
-      if (l == 1) {
+      G.S = S;
+      G.ldS = s.maxh;
+      G.g = g;
+      G.wo = wo;
+      if (l > 1) {
+        G.T = act + s.aoff[l - 1];
+        G.ldT = s.H;
+        G.Snext = Sb[cur];
+        G.Z = Z[cur ^ 1];
+        G.ldz = s.maxh;
+      } else {
         G.out = dD;
         G.ldo = s.w[0];
-      } else {
-        G.out = buf[cur];
-        G.ldo = s.maxh;
       }
-      if ((rc = gemm<false>(G, L[nlayer - 1 - l], wk, st, who))) return rc;
-      S = G.out;
-      ldS = G.ldo;
+      if ((rc = gemm<false>(G, L[nlayer - 1 - l], wk, m, st, who))) return rc;
+      S = G.Snext;
       cur ^= 1;
     }
   }
