@@ -195,5 +195,44 @@ __device__ __forceinline__ void sincospi(const df64 u, df64 *sn, df64 *cs) {
   *cs = -sx;  // cos(pi u) = -sin(pi x)
 }
 
+// tanh(x) for a double x, computed in df64 on the FP32 pipes and rounded to double once (relative
+// error a few 1e-15; the FP64 pipe runs a handful of instructions per call instead of a whole tanh).
+// |x| >= 19.1 gives +-1, what tanh rounds to in double there, |x| < 1e-20 gives x; NaN stays NaN.
+// Otherwise, with u = expm1(-2|x|) in (-1, 0], tanh(|x|) = -u / (2 + u): no cancellation for small
+// |x|.  expm1(y) for y = -2|x| in (-38.2, 0]: Cody and Waite's reduction y = k ln2 + r with
+// k = rint(y / ln2), |r| <~ ln2 / 2, ln2 in three parts whose first two carry 16 significant bits
+// (so k times them is exact in float for |k| < 256); expm1(r) = r (1 + r (1/2! + r (1/3! + ...)))
+// by its Taylor series to r^13 (the next term is below 2^-50 of the sum); then
+// expm1(y) = 2^k expm1(r) + (2^k - 1).  The coefficients 1/n! are each the float nearest to them
+// plus the float nearest to the rest.
+__device__ __forceinline__ double tanh_d(const double x) {
+  const double ax = fabs(x);
+  if (!(ax < 19.1)) return x != x ? x : copysign(1.0, x);
+  if (ax < 1e-20) return x;  // tanh(x) = x (1 - x^2 / 3 ...); and split keeps all 48 bits only above 2^-79
+  const df64 y = split(-2.0 * ax);
+  const float kf = rintf(y.hi * 1.44269504f);  // |k| <= 28
+  df64 r = y + df64(-kf * 0.69314575f);        // k c1, k c2 exact
+  r = r + df64(-kf * 1.4285906e-06f);
+  r = r + df64(-kf) * df64(1.619851e-11f);
+  df64 q = df64(1.6059044e-10f, -5.3525265e-18f);  // 1/13!
+  q = fma(q, r, df64(2.0876756e-09f, 1.1082839e-16f));
+  q = fma(q, r, df64(2.5052108e-08f, 4.417623e-16f));
+  q = fma(q, r, df64(2.755732e-07f, -7.575112e-15f));
+  q = fma(q, r, df64(2.7557319e-06f, 3.7935712e-14f));
+  q = fma(q, r, df64(2.4801588e-05f, -3.406996e-13f));
+  q = fma(q, r, df64(1.984127e-04f, -2.7255969e-12f));
+  q = fma(q, r, df64(1.3888889e-03f, -3.3631094e-11f));
+  q = fma(q, r, df64(8.333334e-03f, -4.346172e-10f));
+  q = fma(q, r, df64(4.1666668e-02f, -1.2417635e-09f));
+  q = fma(q, r, df64(1.6666667e-01f, -4.967054e-09f));
+  q = fma(q, r, df64(0.5f));
+  q = fma(q, r, df64(1.0f));
+  const df64 em = q * r;                                            // expm1(r)
+  const float p2 = __uint_as_float((unsigned)(127 + (int)kf) << 23);  // 2^k, k >= -28
+  const df64 u = fma(em, df64(p2), df64(p2) + df64(-1.0f));        // expm1(y)
+  const df64 t = (-u) * rcp(u + df64(2.0f));
+  return copysign(join(t), x);
+}
+
 }  // namespace dfl
 }  // namespace dpc

@@ -446,8 +446,9 @@ __device__ __forceinline__ void ldmatrix_x2(uint32_t (&r)[2], uint32_t addr) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
 }
 
+// (not volatile: a pure function of its registers, so the compiler may interleave it with the loads)
 __device__ __forceinline__ void mma_f16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
                : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
                : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
@@ -535,20 +536,37 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
       sF[c - kBM] = P.Fexp[n0 + c - kBM];
   }
 
-  // the digit planes of slice k0, A then B: kS x (kBM + kBN) rows of kBK halves, 16 B a copy
+  // the digit planes of slice k0, A then B: kS x (kBM + kBN) rows of kBK halves, 16 B a copy.  A
+  // thread keeps the same (row, 16-byte column) pairs for every slice and plane; its addresses step
+  // by one plane's stride from plane to plane.
+  constexpr int kPairs = (kBM + kBN) * (kBK / 8);             // (row, column) pairs per plane
+  constexpr int kPairsPer = (kPairs + kThreads - 1) / kThreads;
+  const uint16_t *src[kPairsPer];
+  uint32_t dst[kPairsPer];
+  size_t sstride[kPairsPer];
+#pragma unroll
+  for (int q = 0; q < kPairsPer; ++q) {
+    const int e = min(threadIdx.x + q * kThreads, kPairs - 1);  // spare threads repeat the last copy
+    const int rr = e / (kBK / 8), kc = e - rr * (kBK / 8);
+    if (rr < kBM) {
+      src[q] = P.aplanes + (size_t)(m0 + rr) * P.Kp + kc * 8;
+      sstride[q] = (size_t)P.Mp * P.Kp;
+      dst[q] = smem_u32(smem) + 2u * (uint32_t)(rr * kLd + kc * 8);
+    } else {
+      src[q] = P.planes + (size_t)(n0 + rr - kBM) * P.Kp + kc * 8;
+      sstride[q] = (size_t)P.Np * P.Kp;
+      dst[q] = smem_u32(smem + kSmemA) + 2u * (uint32_t)((rr - kBM) * kLd + kc * 8);
+    }
+  }
   auto copy_slice = [&](int k0, int buf) {
-    uint16_t *As = reinterpret_cast<uint16_t *>(smem + buf * kStage);
-    uint16_t *Bs = reinterpret_cast<uint16_t *>(smem + buf * kStage + kSmemA);
-#pragma unroll 1
-    for (int e = threadIdx.x; e < kS * (kBM + kBN) * (kBK / 8); e += kThreads) {
-      const int s = e / ((kBM + kBN) * (kBK / 8)), rem = e - s * (kBM + kBN) * (kBK / 8);
-      const int rr = rem / (kBK / 8), kc = rem - rr * (kBK / 8);
-      if (rr < kBM)
-        cp_async16(smem_u32(As + (s * kBM + rr) * kLd + kc * 8),
-                   P.aplanes + ((size_t)s * P.Mp + m0 + rr) * P.Kp + k0 + kc * 8);
-      else
-        cp_async16(smem_u32(Bs + (s * kBN + rr - kBM) * kLd + kc * 8),
-                   P.planes + ((size_t)s * P.Np + n0 + rr - kBM) * P.Kp + k0 + kc * 8);
+#pragma unroll
+    for (int q = 0; q < kPairsPer; ++q) {
+      const bool a_side = dst[q] < smem_u32(smem) + kSmemA;
+      const uint32_t dplane = 2u * (a_side ? kBM : kBN) * kLd;  // bytes between planes in shared memory
+      const uint16_t *sp = src[q] + k0;
+      uint32_t dp = dst[q] + buf * (uint32_t)kStage;
+#pragma unroll
+      for (int s = 0; s < kS; ++s, sp += sstride[q], dp += dplane) cp_async16(dp, sp);
     }
     asm volatile("cp.async.commit_group;");
   };
@@ -587,17 +605,23 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
         ldmatrix_x4(a[s], smem_u32(As + (s * kBM + wm * 16 + (lane & 15)) * kLd + ks * 16 + (lane >> 4) * 8));
 #pragma unroll
       for (int t = 0; t < kS; ++t) {
-        // B fragments of the warp's three 8-column tiles: an x4 load for the first two, an x2 for the third
+        // B fragments of the warp's 8-column tiles: x4 loads for pairs of tiles, an x2 for an odd last one
         const uint16_t *bt = Bs + (t * kBN + wn * 8 * kNT) * kLd + ks * 16 + ((lane >> 3) & 1) * 8;
-        uint32_t b[4], b2[2];
-        ldmatrix_x4(b, smem_u32(bt + ((lane & 7) + ((lane >> 4) << 3)) * kLd));
-        ldmatrix_x2(b2, smem_u32(bt + (16 + (lane & 7)) * kLd));
+        uint32_t b[kNT][2];
 #pragma unroll
-        for (int s = 0; s + t < kS; ++s) {  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
-          mma_f16(acc[s + t][0], a[s], b[0], b[1]);
-          mma_f16(acc[s + t][1], a[s], b[2], b[3]);
-          mma_f16(acc[s + t][2], a[s], b2[0], b2[1]);
+        for (int j = 0; j + 1 < kNT; j += 2) {
+          uint32_t r[4];
+          ldmatrix_x4(r, smem_u32(bt + (8 * j + (lane & 7) + ((lane >> 4) << 3)) * kLd));
+          b[j][0] = r[0];
+          b[j][1] = r[1];
+          b[j + 1][0] = r[2];
+          b[j + 1][1] = r[3];
         }
+        if constexpr (kNT % 2) ldmatrix_x2(b[kNT - 1], smem_u32(bt + (8 * (kNT - 1) + (lane & 7)) * kLd));
+#pragma unroll
+        for (int s = 0; s + t < kS; ++s)  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
+#pragma unroll
+          for (int j = 0; j < kNT; ++j) mma_f16(acc[s + t][j], a[s], b[j][0], b[j][1]);
       }
     }
     since_flush += kBK;
@@ -655,7 +679,7 @@ __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int kspli
     double v = P.part[rc * P.Np + nn];
     for (int z = 1; z < ksplit; ++z) v += P.part[((size_t)z * P.Mp + rc) * P.Np + nn];
     if constexpr (kFwd) {
-      const double t = tanh(v + P.bias[nn]);
+      const double t = dfl::tanh_d(v + P.bias[nn]);
       P.act[row * P.ldact + nn] = t;
       P.V[row * P.ldv + nn] = P.skip ? t + P.A[row * P.lda + nn] : t;
     } else {

@@ -122,3 +122,26 @@ def test_tc_work_buffer_rules_and_reuse():
     E0, act0 = dpc.dp_fitting_fwd_tc_f64(p, widths, [0, 0, 0], torch.empty((0, 70), dtype=torch.float64,
                                                                             device="cuda"))
     assert E0.numel() == 0
+
+
+def test_tc_forward_tanh_against_numpy():
+    """The forward's tanh (evaluated in double-float on the FP32 pipes, rounded to double once) read
+    through a 1 -> 1 -> 1 net with W = 1, b = 0, so that act = tanh(D): within 3e-14 relative of
+    numpy's tanh from 1e-300 to 19, exactly +-1 beyond 19.1, x itself below 1e-20, NaN kept."""
+    dpc = lib()
+    widths = [1, 1, 1]
+    params = np.array([[1.0, 0.0, 1.0, 0.0]])
+    z = np.concatenate([np.linspace(-25.0, 25.0, 4001), 10.0 ** np.linspace(-300, 1.28, 2000),
+                        -(10.0 ** np.linspace(-300, 1.28, 2000)), [0.0, -0.0, 19.1, -19.1, 19.0999, np.nan]])
+    ts = np.array([0, z.size], dtype=np.int64)
+    E, act = dpc.dp_fitting_fwd_tc_f64(_cuda(params), widths, ts, _cuda(z[:, None]))
+    t = act.cpu().numpy()[:, 0]
+    ref = np.tanh(z)
+    ok = ~np.isnan(z)
+    relerr = np.abs(t[ok] - ref[ok]) / np.maximum(np.abs(ref[ok]), 1e-300)
+    assert relerr.max() <= 3e-14, (relerr.max(), z[ok][np.argmax(relerr)])
+    big = np.abs(z) >= 19.1
+    assert np.array_equal(t[big], np.sign(z[big]))
+    assert np.isnan(t[~ok]).all()
+    tiny = np.abs(z) < 1e-20
+    assert np.array_equal(t[tiny], z[tiny])
