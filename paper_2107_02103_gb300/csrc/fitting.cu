@@ -64,11 +64,11 @@ struct FitTile<df64, false> {
 constexpr int kBK = 16, kFitThreads = 256;
 constexpr int kMaxChain = DP_MAX_LAYERS + 1;
 
-__device__ __forceinline__ double tanh_r(const double z) { return tanh(z); }
+// f64 and df64: tanh evaluated in double-float on the FP32 pipes (dfl::tanh_d), not on the FP64
+// pipe, where a double tanh costs about a tenth of a 240-deep layer's products
+__device__ __forceinline__ double tanh_r(const double z) { return dfl::tanh_d(z); }
 __device__ __forceinline__ float tanh_r(const float z) { return tanhf(z); }
-// df64: tanh in double on the FP64 pipe (one per output element, against a
-// K-long df64 dot product per element on the FP32 pipes)
-__device__ __forceinline__ df64 tanh_r(const df64 z) { return dfl::split(tanh(dfl::join(z))); }
+__device__ __forceinline__ df64 tanh_r(const df64 z) { return dfl::split(dfl::tanh_d(dfl::join(z))); }
 
 template <typename real>
 struct FitGemm {
