@@ -74,10 +74,11 @@ def test_fitting_skip_on_the_input_layer_and_errors():
         dpc.dp_fitting_fwd(p, widths, [0, 70, 71], torch.from_numpy(D).cuda())
 
 
-@pytest.mark.parametrize("arith", ["f64", "df64"])
+@pytest.mark.parametrize("arith", ["f64", "df64", "f64-tc"])
 def test_energy_and_forces_of_the_whole_model(arith):
     """Coordinates -> s, R~ -> T -> D -> E_i (fitting net) and back: dE/dD -> dE/dT -> dE/ds, dE/dR~ ->
-    forces and virial, every step on the GPU, against the oracle's chain; the folded forces sum to zero."""
+    forces and virial, every step on the GPU, against the oracle's chain; the folded forces sum to zero.
+    f64-tc: the fitting net's GEMMs on the tensor cores (dp_fitting_*_tc_f64)."""
     dpc = lib()
     from test_gpu_env_force import _system
     w, coord, nlist, owner, env = _system("water", dict(seed=47, nmol=128), 0, None)
@@ -95,8 +96,12 @@ def test_energy_and_forces_of_the_whole_model(arith):
     T = fwd(model.table, model.info, s, Rt, nvalid, at, w.sel)
     D = dpc.dp_descriptor_contract(T, w.M2, arith=a)
     fp = torch.from_numpy(fparams).cuda()
-    E, act = dpc.dp_fitting_fwd(fp, widths, ts, D, arith=a)
-    dD = dpc.dp_fitting_grad(fp, widths, ts, act, arith=a)
+    if arith == "f64-tc":
+        E, act = dpc.dp_fitting_fwd_tc_f64(fp, widths, ts, D)
+        dD = dpc.dp_fitting_grad_tc_f64(fp, widths, ts, act)
+    else:
+        E, act = dpc.dp_fitting_fwd(fp, widths, ts, D, arith=a)
+        dD = dpc.dp_fitting_grad(fp, widths, ts, act, arith=a)
     dT = dpc.dp_descriptor_contract_grad(T, dD.reshape(D.shape), arith=a)
     ds, dRt = grad(model.table, model.info, s, Rt, nvalid, at, w.sel, dT)
     F, Wv = dpc.dp_force_virial(cg, ng, ei, ds, dRt, arith=a)
