@@ -398,6 +398,9 @@ constexpr int kFlushK = 1024;
 constexpr int kNonFinite = 1 << 20;  // exponent of a row or column holding inf or NaN
 constexpr size_t kSmemA = (size_t)kS * kBM * kLd * 2, kSmemB = (size_t)kS * kBN * kLd * 2;
 constexpr size_t kSmemE = (size_t)(kBM + kBN) * sizeof(int);  // row and column exponents
+// f64 accumulators of every thread's 4 kNT outputs, [output][thread]: touched only at the flushes,
+// so kept in shared memory rather than in registers (the MMA loop needs those for its fragments)
+constexpr size_t kSmemAcc = (size_t)4 * 3 * 256 * sizeof(double);
 static_assert((size_t)kS * kFlushK * 961 < (1u << 24), "fp32 diagonal sums must stay exact");
 
 __host__ __device__ constexpr int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
@@ -519,6 +522,9 @@ struct TcGemm {
 };
 
 constexpr size_t kStage = kSmemA + kSmemB;
+constexpr size_t kSmemTotal = 2 * kStage + kSmemE + kSmemAcc;
+static_assert(kSmemAcc == (size_t)4 * kNT * kThreads * sizeof(double), "accumulator area");
+static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
 
 template <bool kFwd>
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
@@ -578,11 +584,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
     for (int j = 0; j < kNT; ++j)
 #pragma unroll
       for (int c = 0; c < 4; ++c) acc[d][j][c] = 0.f;
-  double acc64[kNT][4];
+  double *acc64 = reinterpret_cast<double *>(smem + 2 * kStage + kSmemE) + threadIdx.x;  // [4 kNT][kThreads]
 #pragma unroll
-  for (int j = 0; j < kNT; ++j)
-#pragma unroll
-    for (int c = 0; c < 4; ++c) acc64[j][c] = 0.0;
+  for (int x = 0; x < 4 * kNT; ++x) acc64[x * kThreads] = 0.0;
 
   copy_slice(blockIdx.z * P.slices_per_split * kBK, 0);
   asm volatile("cp.async.wait_all;" ::: "memory");
@@ -603,11 +607,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
 #pragma unroll
       for (int s = 0; s < kS; ++s)
         ldmatrix_x4(a[s], smem_u32(As + (s * kBM + wm * 16 + (lane & 15)) * kLd + ks * 16 + (lane >> 4) * 8));
-#pragma unroll
-      for (int t = 0; t < kS; ++t) {
-        // B fragments of the warp's 8-column tiles: x4 loads for pairs of tiles, an x2 for an odd last one
+      // B fragments of digit plane t for the warp's 8-column tiles: x4 loads for pairs of tiles, an x2
+      // for an odd last one; plane t + 1's are loaded while plane t's MMAs issue
+      auto load_b = [&](int t, uint32_t (&b)[kNT][2]) {
         const uint16_t *bt = Bs + (t * kBN + wn * 8 * kNT) * kLd + ks * 16 + ((lane >> 3) & 1) * 8;
-        uint32_t b[kNT][2];
 #pragma unroll
         for (int j = 0; j + 1 < kNT; j += 2) {
           uint32_t r[4];
@@ -618,26 +621,33 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
           b[j + 1][1] = r[3];
         }
         if constexpr (kNT % 2) ldmatrix_x2(b[kNT - 1], smem_u32(bt + (8 * (kNT - 1) + (lane & 7)) * kLd));
+      };
+      uint32_t b[2][kNT][2];
+      load_b(0, b[0]);
+#pragma unroll
+      for (int t = 0; t < kS; ++t) {
+        if (t + 1 < kS) load_b(t + 1, b[(t + 1) & 1]);
 #pragma unroll
         for (int s = 0; s + t < kS; ++s)  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
 #pragma unroll
-          for (int j = 0; j < kNT; ++j) mma_f16(acc[s + t][j], a[s], b[j][0], b[j][1]);
+          for (int j = 0; j < kNT; ++j) mma_f16(acc[s + t][j], a[s], b[t & 1][j][0], b[t & 1][j][1]);
       }
     }
     since_flush += kBK;
     if (since_flush == kFlushK || !more) {  // uniform: the diagonals into f64, smallest first
       since_flush = 0;
 #pragma unroll
-      for (int d = kS - 1; d >= 0; --d) {
-        const double scale = __hiloint2double((1023 - 5 * (d + 2)) << 20, 0);  // 32^-(d + 2)
+      for (int j = 0; j < kNT; ++j)
 #pragma unroll
-        for (int j = 0; j < kNT; ++j)
+        for (int c = 0; c < 4; ++c) {
+          double v = acc64[(4 * j + c) * kThreads];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            acc64[j][c] = fma(dfl::widen(acc[d][j][c]), scale, acc64[j][c]);
+          for (int d = kS - 1; d >= 0; --d) {
+            v = fma(dfl::widen(acc[d][j][c]), __hiloint2double((1023 - 5 * (d + 2)) << 20, 0), v);  // 32^-(d+2)
             acc[d][j][c] = 0.f;
           }
-      }
+          acc64[(4 * j + c) * kThreads] = v;
+        }
     }
     asm volatile("cp.async.wait_all;" ::: "memory");  // buffer cur ^ 1 was last read before the previous barrier
     __syncthreads();
@@ -655,9 +665,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
       const int E = sE[rl];
       double2 v;
       v.x = (E >= kNonFinite || sF[cl] >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
-                                                     : scalbn(acc64[j][2 * h], E + sF[cl]);
+                                                     : scalbn(acc64[(4 * j + 2 * h) * kThreads], E + sF[cl]);
       v.y = (E >= kNonFinite || sF[cl + 1] >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
-                                                         : scalbn(acc64[j][2 * h + 1], E + sF[cl + 1]);
+                                                         : scalbn(acc64[(4 * j + 2 * h + 1) * kThreads], E + sF[cl + 1]);
       *reinterpret_cast<double2 *>(part + (size_t)(m0 + rl) * P.Np + n0 + cl) = v;
     }
 }
@@ -784,7 +794,7 @@ int set_smem() {
   static std::atomic<bool> done{false};
   if (done.load(std::memory_order_acquire)) return DP_OK;
   for (auto k : {&gemm_kernel<true>, &gemm_kernel<false>}) {
-    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)(2 * kStage + kSmemE));
+    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemTotal);
     if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_fitting_*_tc_f64: %s", cudaGetErrorString(e));
   }
   done.store(true, std::memory_order_release);
@@ -826,7 +836,7 @@ int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaSt
     const int ksplit = ksplit_for(C.Mp, L.Np, L.Kp);
     C.slices_per_split = (L.Kp / kBK + ksplit - 1) / ksplit;
     const dim3 grid((unsigned)(L.Np / kBN), (unsigned)(C.Mp / kBM), (unsigned)ksplit);
-    gemm_kernel<kFwd><<<grid, kThreads, 2 * kStage + kSmemE, st>>>(C);
+    gemm_kernel<kFwd><<<grid, kThreads, kSmemTotal, st>>>(C);
     if ((rc = launch_status(who))) return rc;
     const int64_t total = C.n * C.N;
     epilogue_kernel<kFwd><<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(C, ksplit);
