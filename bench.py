@@ -62,10 +62,10 @@ def footprint(w, esize: int, hbm_bytes: float = 280e9) -> dict:
             "atoms_per_280GB": int(hbm_bytes // ours), "atoms_per_280GB_uncompressed": int(hbm_bytes // (ours + net))}
 
 
-# f64 fitting GEMMs on the tensor cores: every operand element is split into 11 digits and the 66 digit
-# products with s + t <= 12 run as fp16 MMAs, so a GEMM of 2 n K N FP64 flop issues 66 times as many
+# f64 fitting GEMMs on the tensor cores: every operand element is split into 9 digits and the 45 digit
+# products with s + t <= 10 run as fp16 MMAs, so a GEMM of 2 n K N FP64 flop issues 45 times as many
 # fp16 MMA flop; their roofline is the dense 16-bit tensor rate (fp16 and bf16 run at the same rate).
-TC_DIGIT_PRODUCTS = 66
+TC_DIGIT_PRODUCTS = 45
 
 
 def tensor_peak() -> tuple:
@@ -595,7 +595,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                                  "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
                                  else "per row: 9 M1 fwd, 18 M1 grad"),
                    "l2": "flushed between steps (256 MiB write)",
-                   **({"fitting_gemm": ("tensor cores: f64 by exact 11-digit splitting, fp16 MMAs"
+                   **({"fitting_gemm": ("tensor cores (tcgen05): f64 by exact 9-digit splitting, fp16 MMAs"
                                         if tc else "FP64 pipe")} if getattr(args, "fitting", False) else {}),
                    "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4),
                    "footprint": footprint(w, 4 if args.dtype == "f32" else 8)},

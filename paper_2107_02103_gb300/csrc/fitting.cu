@@ -360,48 +360,57 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
 }
 
 // ------------------------------------------------- f64 GEMMs on the tensor cores
-// GB300 retires FP64 at 2 lanes per clock per SM, fp16 products on the tensor
-// cores (mma.sync, measured) at about 480 times that rate.  An f64 GEMM
-// C = A B is recovered from fp16 products by splitting every operand element
-// into base-32 digits (the error-free splitting of Ozaki et al.):
-//   a_ik = 2^E_i sum_{s=1..11} A_s[i][k] 32^-s + r_ik,  A_s integers in [-31, 31],  |r_ik| < 2^(E_i - 55),
+// GB300 retires FP64 at 2 lanes per clock per SM but fp16 products on its
+// tcgen05 tensor cores at ~1000 times that rate.  An f64 GEMM C = A B is
+// recovered from fp16 products by splitting every operand element into base-64
+// digits (the error-free splitting of Ozaki et al.):
+//   a_ik = 2^E_i sum_{s=1..9} A_s[i][k] 64^-s + r_ik,  A_s integers in [-63, 63],  |r_ik| < 2^(E_i - 54),
 // with max_k |a_ik| < 2^E_i, and likewise b_kj with a column exponent F_j, so that
-//   C_ij = 2^(E_i + F_j) sum_{d=2..12} 32^-d sum_{s+t=d} (A_s B_t)_ij + (terms with s + t > 12 and the r).
-// Every (A_s B_t)_ij is a sum of integer products |A_s B_t| <= 961, so its fp32
-// sum on the tensor cores is exact while it stays below 2^24: the 11 diagonals
-// d are summed in fp32 over at most kFlushK = 1024 of K at a time (11 pairs x
-// 1024 x 961 < 2^24) and then added into an f64 accumulator.  What rounds is
-// that f64 accumulation (11 adds per 1024 of K), the 55-bit truncation of the
-// operands and the dropped terms: |error| <~ K 2^-51 max_k|a_ik| max_k|b_kj|,
-// against K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column
-// with an inf or NaN gives NaN outputs.
+//   C_ij = 2^(E_i + F_j) sum_{d=2..10} 64^-d sum_{s+t=d} (A_s B_t)_ij + (terms with s + t > 10 and the r).
+// Every (A_s B_t)_ij is a sum of integer products |A_s B_t| <= 3969; a diagonal
+// d has at most 9 of them, so its fp32 sum on the tensor cores is exact while
+// a block's share of K is at most kMaxShareK = 448 (9 x 448 x 3969 < 2^24).
+// The 9 diagonal sums of an output are then combined with one rounding: the
+// two largest exactly in f64, the rest in float-float (its rounding lies some
+// 2^-60 below the result), one f64 add for the two.  What rounds is that add,
+// the adds of the shares' f64 results (epilogue_kernel), the 54-bit truncation
+// of the operands and the dropped terms: |error| <~ K 2^-50 max_k|a_ik|
+// max_k|b_kj|, against K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row
+// or column with an inf or NaN gives NaN outputs.
 //
-// Block tile 64 x 48 (eight warps of 16 x 24: two per SM sub-partition, so
-// that each sub-partition's tensor unit gets the same work), 32-deep K slices,
-// two slices in shared memory: while the warps multiply one slice, the next
-// slice's digit planes arrive by cp.async.  The planes are made by a separate
-// pass, once per element: B's when the call starts, A's per chunk of rows
-// before each GEMM (with each row's exponent).  Each warp runs the 66 digit
-// products of its tile as m16n8k16 MMAs with fp32 accumulators, one per
-// diagonal and 8-column tile.  A is always a plain matrix: the forward keeps
-// each layer's input v_l (its tanh outputs plus the skip) in a work buffer,
-// and the backward's epilogue writes dE/dv (for the next skip) and
-// dE/dv (1 - t^2) (the next A).
+// gemm_kernel: one CTA of 128 threads per 128 x 48 output tile and share of K,
+// one CTA per SM (its 9 diagonal accumulators take 432 of the SM's 512 TMEM
+// columns).  The digit planes of A (per chunk of rows, with the row exponents)
+// and B (per call) are made by split_rows_kernel, once per element.  K slices
+// of 16 pass through four shared-memory stages in the tcgen05 K-major layout
+// without swizzle (8-row x 16-byte core matrices), filled by cp.async; one
+// thread issues the 45 digit-product MMAs (M = 128, N = 48, K = 16, fp16 in,
+// fp32 accumulators in TMEM, one per diagonal) of a stage and commits them to
+// the stage's mbarrier, which frees the stage for the slice four ahead.  At
+// the end each warp reads its 32 TMEM lanes (rows), combines the diagonals and
+// writes the share's f64 result; epilogue_kernel sums the shares in a fixed
+// order and applies the layer's epilogue.  A is always a plain matrix: the
+// forward keeps each layer's input v_l (tanh outputs plus the skip) in a work
+// buffer, the backward writes dE/dv (for the next skip) and dE/dv (1 - t^2)
+// (the next A).  Every wait on an mbarrier is bounded; a wait that gives up
+// makes the tile's outputs NaN.
 namespace tc {
-constexpr int kS = 11;  // digits per operand element
-constexpr int kBM = 64, kBN = 48, kBK = 32;
-constexpr int kLd = kBK + 8;  // shared row stride in halves (80 B): the 8 rows an ldmatrix reads hit 8 distinct bank groups
-constexpr int kNT = 3;  // 8-column MMA tiles per warp: warp tile 16 x 24
-constexpr int kWarpsN = kBN / (8 * kNT), kWarps = (kBM / 16) * kWarpsN, kThreads = 32 * kWarps;  // 4 x 2 warps
-static_assert(kWarps == 8, "two warps per SM sub-partition: more than 8 leave some with a third warp");
-constexpr int kFlushK = 1024;
+constexpr int kS = 9;      // digits per operand element
+constexpr int kBits = 6;   // bits per digit
+constexpr int kFrac = kS * kBits;  // 54 fractional bits
+constexpr int kTM = 128, kTN = 48, kTK = 16;  // CTA tile; K per stage (one MMA)
+constexpr int kStages = 4;
+constexpr int kThreads = 384;  // 12 warps: every thread copies one 16-byte slot of every plane; three warps per TMEM lane quadrant
+constexpr int kMaxShareK = 448;
 constexpr int kNonFinite = 1 << 20;  // exponent of a row or column holding inf or NaN
-constexpr size_t kSmemA = (size_t)kS * kBM * kLd * 2, kSmemB = (size_t)kS * kBN * kLd * 2;
-constexpr size_t kSmemE = (size_t)(kBM + kBN) * sizeof(int);  // row and column exponents
-// f64 accumulators of every thread's 4 kNT outputs, [output][thread]: touched only at the flushes,
-// so kept in shared memory rather than in registers (the MMA loop needs those for its fragments)
-constexpr size_t kSmemAcc = (size_t)4 * 3 * 256 * sizeof(double);
-static_assert((size_t)kS * kFlushK * 961 < (1u << 24), "fp32 diagonal sums must stay exact");
+constexpr uint32_t kLBO = 128, kSBO = 256;  // core matrices: next along K at +128 B, next 8 rows at +256 B
+constexpr int kPlaneA = kTM * kTK * 2, kPlaneB = kTN * kTK * 2;  // bytes of one digit plane in a stage
+constexpr int kStageBytes = kS * (kPlaneA + kPlaneB);
+constexpr uint32_t kTmemCols = 512;  // allocation (a power of two); kS * kTN = 432 used
+constexpr size_t kSmemTotal = (size_t)kStages * kStageBytes + 64;
+static_assert((size_t)kS * kMaxShareK * 63 * 63 < (1u << 24), "fp32 diagonal sums must stay exact");
+static_assert(kMaxShareK % kTK == 0 && kS * kTN <= (int)kTmemCols, "shares and TMEM");
+static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
 
 __host__ __device__ constexpr int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
@@ -409,13 +418,13 @@ __device__ __forceinline__ int exp_bits(double x) { return (int)(((uint64_t)__do
 // E with max |x| < 2^E from the largest biased exponent (normal x: |x| < 2^(eb - 1022))
 __device__ __forceinline__ int exp_of_max(int ebmax) { return ebmax == 0x7ff ? kNonFinite : max(ebmax, 1) - 1022; }
 
-// |x| 2^-E as an integer with 55 fractional bits, truncated; below 2^55 since |x| < 2^E
-__device__ __forceinline__ uint64_t fixed55(double x, int E) {
+// |x| 2^-E as an integer with kFrac fractional bits, truncated; below 2^kFrac since |x| < 2^E
+__device__ __forceinline__ uint64_t fixed_point(double x, int E) {
   const uint64_t b = (uint64_t)__double_as_longlong(x);
   const int eb = (int)((b >> 52) & 0x7ff);
   const uint64_t mant = b & 0xfffffffffffffull;
   const uint64_t m = eb ? (mant | (1ull << 52)) : mant;
-  const int sh = (eb ? eb - 1075 : -1074) - E + 55;  // |x| 2^(55 - E) = m 2^sh, sh <= 2 for finite x
+  const int sh = (eb ? eb - 1075 : -1074) - E + kFrac;  // |x| 2^(kFrac - E) = m 2^sh, sh <= 1 for finite x
   if (sh >= 0) return m << min(sh, 10);
   return sh > -64 ? m >> -sh : 0ull;
 }
@@ -423,9 +432,11 @@ __device__ __forceinline__ uint64_t fixed55(double x, int E) {
 // The kS digits of two fixed-point values, digit s of both packed as an fp16 pair (element 0 in the
 // low half), each with its element's sign: 0x6400 | d is the fp16 1024 + d, and 1024 comes off exactly.
 __device__ __forceinline__ void digit_pairs(uint64_t f0, uint64_t f1, uint32_t sign2, uint32_t (&h)[kS]) {
+  constexpr uint32_t kMask = (1u << kBits) - 1;
 #pragma unroll
   for (int s = 1; s <= kS; ++s) {
-    const uint32_t d0 = (uint32_t)(f0 >> (55 - 5 * s)) & 31u, d1 = (uint32_t)(f1 >> (55 - 5 * s)) & 31u;
+    const uint32_t d0 = (uint32_t)(f0 >> (kFrac - kBits * s)) & kMask;
+    const uint32_t d1 = (uint32_t)(f1 >> (kFrac - kBits * s)) & kMask;
     uint32_t v;
     asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(v) : "r"(0x64006400u | d0 | (d1 << 16)), "r"(0x64006400u));
     h[s - 1] = v ^ sign2;
@@ -438,23 +449,6 @@ __device__ __forceinline__ uint32_t sign_pair(double x0, double x1) {
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void ldmatrix_x2(uint32_t (&r)[2], uint32_t addr) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
-}
-
-// (not volatile: a pure function of its registers, so the compiler may interleave it with the loads)
-__device__ __forceinline__ void mma_f16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
-               : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-               : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
 
 __device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src));
@@ -479,16 +473,16 @@ __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restric
   for (int c2 = lane; c2 < Kp / 2; c2 += 32) {
     const double x0 = x(2 * c2), x1 = x(2 * c2 + 1);
     uint32_t h[kS];
-    digit_pairs(fixed55(x0, E), fixed55(x1, E), sign_pair(x0, x1), h);
+    digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
 #pragma unroll
     for (int s = 0; s < kS; ++s) planes[((size_t)s * rows_p + r) * (Kp / 2) + c2] = h[s];
   }
 }
 
 // One hidden-layer GEMM of a chunk of one type's atoms: rows r0 .. r0 + n - 1 of the plain
-// row-major A [*][K] (as digit planes) times B (digit planes), K cut into ksplit shares (grid z) so
-// that even a few thousand atoms give enough blocks for every SM; the shares' f64 results go to
-// `part`, and epilogue_kernel sums them and applies the layer's epilogue.
+// row-major A [*][K] (as digit planes) times B (digit planes), K cut into shares of at most
+// kMaxShareK (grid z); the shares' f64 results go to `part`, and epilogue_kernel sums them and
+// applies the layer's epilogue.
 struct TcGemm {
   int64_t r0, n;  // output rows r0 .. r0 + n - 1; A's planes hold rows 0 .. n - 1 of this chunk
   int K, N;
@@ -521,155 +515,161 @@ struct TcGemm {
   int64_t ldo;
 };
 
-constexpr size_t kStage = kSmemA + kSmemB;
-constexpr size_t kSmemTotal = 2 * kStage + kSmemE + kSmemAcc;
-static_assert(kSmemAcc == (size_t)4 * kNT * kThreads * sizeof(double), "accumulator area");
-static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
+// shared-memory descriptor of a K-major operand without swizzle (tcgen05): start address, the byte
+// offsets of the next core matrix along K (leading) and along the rows (stride), version 1
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFF) >> 4) | ((uint64_t)(kLBO >> 4) << 16) | ((uint64_t)(kSBO >> 4) << 32) |
+         (1ull << 46);
+}
+// instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A and B f16 (0), both K-major, N >> 3 at
+// bit 17, M >> 4 at bit 24
+constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(kTN >> 3) << 17) | ((uint32_t)(kTM >> 4) << 24);
 
-template <bool kFwd>
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  uint32_t done = 0;
+  for (int it = 0; it < (1 << 24) && !done; ++it)
+    asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+                 : "=r"(done)
+                 : "r"(bar), "r"(parity)
+                 : "memory");
+  return done != 0;
+}
+
+__device__ __forceinline__ void cp_async_wait_pending(int n) {  // at most n of this thread's copy groups pending
+  if (n >= 2)
+    asm volatile("cp.async.wait_group 2;" ::: "memory");
+  else if (n == 1)
+    asm volatile("cp.async.wait_group 1;" ::: "memory");
+  else
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
-  extern __shared__ __align__(16) unsigned char smem[];
-  int *sE = reinterpret_cast<int *>(smem + 2 * kStage);  // row exponents [kBM]
-  int *sF = sE + kBM;                                    // column exponents [kBN]
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int wm = warp / kWarpsN, wn = warp - wm * kWarpsN;
-  const int64_t m0 = (int64_t)blockIdx.y * kBM;
-  const int n0 = blockIdx.x * kBN;
-  for (int c = threadIdx.x; c < kBM + kBN; c += kThreads) {
-    if (c < kBM)
-      sE[c] = P.Eexp[m0 + c];
-    else
-      sF[c - kBM] = P.Fexp[n0 + c - kBM];
+  extern __shared__ __align__(1024) unsigned char smem[];
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);  // one per stage
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + kStages);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t m0 = (int64_t)blockIdx.y * kTM;
+  const int n0 = blockIdx.x * kTN;
+  const int slices_total = P.Kp / kTK;
+  const int i0 = blockIdx.z * P.slices_per_split;
+  const int nsl = min(slices_total - i0, P.slices_per_split);  // > 0: no empty share
+
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s)
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bars + s)));
+    asm volatile("fence.mbarrier_init.release.cluster;");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                 "r"(kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
 
-  // the digit planes of slice k0, A then B: kS x (kBM + kBN) rows of kBK halves, 16 B a copy.  A
-  // thread keeps the same (row, 16-byte column) pairs for every slice and plane; its addresses step
-  // by one plane's stride from plane to plane.
-  constexpr int kPairs = (kBM + kBN) * (kBK / 8);             // (row, column) pairs per plane
-  constexpr int kPairsPer = (kPairs + kThreads - 1) / kThreads;
-  const uint16_t *src[kPairsPer];
-  uint32_t dst[kPairsPer];
-  size_t sstride[kPairsPer];
+  // copies of slice j into stage st: thread tid < 2 (kTM + kTN) owns one 16-byte slot (a row and
+  // one of its two 8-k chunks) of A (first 2 kTM threads) or B, and copies it for every plane, from
+  // the plane's row in global memory to its place in the core-matrix layout
+  const uint32_t sbase = smem_u32(smem);
+  const bool loader = tid < 2 * (kTM + kTN);
+  const bool a_side = tid < 2 * kTM;
+  const int lr = (a_side ? tid : tid - 2 * kTM) >> 1, lc = tid & 1;
+  const uint16_t *lsrc = !loader ? P.planes
+                         : a_side ? P.aplanes + (size_t)(m0 + lr) * P.Kp + 8 * lc
+                                  : P.planes + (size_t)(n0 + lr) * P.Kp + 8 * lc;
+  const size_t lsstride = a_side ? (size_t)P.Mp * P.Kp : (size_t)P.Np * P.Kp;  // halves between planes
+  const uint32_t ldst = (a_side ? 0u : (uint32_t)(kS * kPlaneA)) + (lr >> 3) * kSBO + lc * kLBO + (lr & 7) * 16;
+  const uint32_t ldstride = a_side ? kPlaneA : kPlaneB;
+  auto load_slice = [&](int j, int st) {
+    if (loader) {
+      const uint16_t *src = lsrc + (i0 + j) * kTK;
+      uint32_t dst = sbase + st * kStageBytes + ldst;
 #pragma unroll
-  for (int q = 0; q < kPairsPer; ++q) {
-    const int e = min(threadIdx.x + q * kThreads, kPairs - 1);  // spare threads repeat the last copy
-    const int rr = e / (kBK / 8), kc = e - rr * (kBK / 8);
-    if (rr < kBM) {
-      src[q] = P.aplanes + (size_t)(m0 + rr) * P.Kp + kc * 8;
-      sstride[q] = (size_t)P.Mp * P.Kp;
-      dst[q] = smem_u32(smem) + 2u * (uint32_t)(rr * kLd + kc * 8);
-    } else {
-      src[q] = P.planes + (size_t)(n0 + rr - kBM) * P.Kp + kc * 8;
-      sstride[q] = (size_t)P.Np * P.Kp;
-      dst[q] = smem_u32(smem + kSmemA) + 2u * (uint32_t)((rr - kBM) * kLd + kc * 8);
-    }
-  }
-  auto copy_slice = [&](int k0, int buf) {
-#pragma unroll
-    for (int q = 0; q < kPairsPer; ++q) {
-      const bool a_side = dst[q] < smem_u32(smem) + kSmemA;
-      const uint32_t dplane = 2u * (a_side ? kBM : kBN) * kLd;  // bytes between planes in shared memory
-      const uint16_t *sp = src[q] + k0;
-      uint32_t dp = dst[q] + buf * (uint32_t)kStage;
-#pragma unroll
-      for (int s = 0; s < kS; ++s, sp += sstride[q], dp += dplane) cp_async16(dp, sp);
+      for (int s = 0; s < kS; ++s, src += lsstride, dst += ldstride) cp_async16(dst, src);
     }
     asm volatile("cp.async.commit_group;");
   };
 
-  float acc[kS][kNT][4];
-#pragma unroll
-  for (int d = 0; d < kS; ++d)
-#pragma unroll
-    for (int j = 0; j < kNT; ++j)
-#pragma unroll
-      for (int c = 0; c < 4; ++c) acc[d][j][c] = 0.f;
-  double *acc64 = reinterpret_cast<double *>(smem + 2 * kStage + kSmemE) + threadIdx.x;  // [4 kNT][kThreads]
-#pragma unroll
-  for (int x = 0; x < 4 * kNT; ++x) acc64[x * kThreads] = 0.0;
-
-  copy_slice(blockIdx.z * P.slices_per_split * kBK, 0);
-  asm volatile("cp.async.wait_all;" ::: "memory");
+  const int pre = min(kStages - 1, nsl);
+  for (int j = 0; j < pre; ++j) load_slice(j, j);
+  asm volatile("tcgen05.fence::before_thread_sync;");
   __syncthreads();
-  // this block's share of K: slices i0 .. i1 - 1
-  const int i0 = blockIdx.z * P.slices_per_split;
-  const int i1 = min((P.K + kBK - 1) / kBK, i0 + P.slices_per_split);
-  int since_flush = 0;
-  for (int i = i0; i < i1; ++i) {  // uniform
-    const int cur = (i - i0) & 1;
-    const bool more = i + 1 < i1;
-    if (more) copy_slice((i + 1) * kBK, cur ^ 1);  // the next slice's copies fly while this one multiplies
-    const uint16_t *As = reinterpret_cast<const uint16_t *>(smem + cur * kStage);
-    const uint16_t *Bs = reinterpret_cast<const uint16_t *>(smem + cur * kStage + kSmemA);
-#pragma unroll
-    for (int ks = 0; ks < kBK / 16; ++ks) {
-      uint32_t a[kS][4];
-#pragma unroll
-      for (int s = 0; s < kS; ++s)
-        ldmatrix_x4(a[s], smem_u32(As + (s * kBM + wm * 16 + (lane & 15)) * kLd + ks * 16 + (lane >> 4) * 8));
-      // B fragments of digit plane t for the warp's 8-column tiles: x4 loads for pairs of tiles, an x2
-      // for an odd last one; plane t + 1's are loaded while plane t's MMAs issue
-      auto load_b = [&](int t, uint32_t (&b)[kNT][2]) {
-        const uint16_t *bt = Bs + (t * kBN + wn * 8 * kNT) * kLd + ks * 16 + ((lane >> 3) & 1) * 8;
-#pragma unroll
-        for (int j = 0; j + 1 < kNT; j += 2) {
-          uint32_t r[4];
-          ldmatrix_x4(r, smem_u32(bt + (8 * j + (lane & 7) + ((lane >> 4) << 3)) * kLd));
-          b[j][0] = r[0];
-          b[j][1] = r[1];
-          b[j + 1][0] = r[2];
-          b[j + 1][1] = r[3];
-        }
-        if constexpr (kNT % 2) ldmatrix_x2(b[kNT - 1], smem_u32(bt + (8 * (kNT - 1) + (lane & 7)) * kLd));
-      };
-      uint32_t b[2][kNT][2];
-      load_b(0, b[0]);
+  asm volatile("tcgen05.fence::after_thread_sync;");
+  const uint32_t tmem = *tmem_holder;
+
+  bool ok = true;
+  for (int i = 0; i < nsl; ++i) {  // uniform
+    cp_async_wait_pending(min(kStages - 2, nsl - 1 - i));  // slice i's copies (this thread's) have landed
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the copies, visible to the tensor core
+    __syncthreads();
+    if (tid == 0 && ok) {
+      asm volatile("tcgen05.fence::after_thread_sync;");
+      const uint32_t stage = sbase + (i % kStages) * kStageBytes;
 #pragma unroll
       for (int t = 0; t < kS; ++t) {
-        if (t + 1 < kS) load_b(t + 1, b[(t + 1) & 1]);
+        const uint64_t bd = smem_desc(stage + kS * kPlaneA + t * kPlaneB);
 #pragma unroll
-        for (int s = 0; s + t < kS; ++s)  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
-#pragma unroll
-          for (int j = 0; j < kNT; ++j) mma_f16(acc[s + t][j], a[s], b[t & 1][j][0], b[t & 1][j][1]);
-      }
-    }
-    since_flush += kBK;
-    if (since_flush == kFlushK || !more) {  // uniform: the diagonals into f64, smallest first
-      since_flush = 0;
-#pragma unroll
-      for (int j = 0; j < kNT; ++j)
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          double v = acc64[(4 * j + c) * kThreads];
-#pragma unroll
-          for (int d = kS - 1; d >= 0; --d) {
-            v = fma(dfl::widen(acc[d][j][c]), __hiloint2double((1023 - 5 * (d + 2)) << 20, 0), v);  // 32^-(d+2)
-            acc[d][j][c] = 0.f;
-          }
-          acc64[(4 * j + c) * kThreads] = v;
+        for (int s = 0; s + t < kS; ++s) {  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
+          const uint64_t ad = smem_desc(stage + s * kPlaneA);
+          const uint32_t acc = (i > 0 || t > 0) ? 1u : 0u;  // a diagonal's first product overwrites
+          asm volatile(
+              "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+              " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem + (uint32_t)((s + t) * kTN)),
+              "l"(ad), "l"(bd), "r"(kIdesc), "r"(acc));
         }
+      }
+      asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(bars + i % kStages)));
     }
-    asm volatile("cp.async.wait_all;" ::: "memory");  // buffer cur ^ 1 was last read before the previous barrier
-    __syncthreads();
+    // refill the stage of slice i - 1 with slice i + kStages - 1 once slice i - 1's MMAs are done
+    const int j = i + kStages - 1;
+    if (j < nsl) {
+      if (i >= 1) ok = ok && mbar_wait(smem_u32(bars + (i - 1) % kStages), (uint32_t)(((i - 1) / kStages) & 1));
+      load_slice(j, j % kStages);
+    }
+  }
+  // all MMAs of the share done: the last slice's commit tracks every earlier one
+  ok = ok && mbar_wait(smem_u32(bars + (nsl - 1) % kStages), (uint32_t)(((nsl - 1) / kStages) & 1));
+  asm volatile("tcgen05.fence::after_thread_sync;");
+
+  // combine the diagonals of row 32 (warp % 4) + lane (the warp's TMEM lane quadrant), the warp's
+  // third of the columns, 8 at a time
+  const int rl = 32 * (warp & 3) + lane;
+  const int E = P.Eexp[m0 + rl];
+  double *outp = P.part + ((size_t)blockIdx.z * P.Mp + m0 + rl) * P.Np + n0;
+  const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
+  constexpr int kColsPerWarp = kTN / (kThreads / 128);
+  static_assert(kColsPerWarp % 8 == 0, "column share");
+#pragma unroll 1
+  for (int c0 = (warp >> 2) * kColsPerWarp; c0 < (warp >> 2) * kColsPerWarp + kColsPerWarp; c0 += 8) {
+    float v[kS][8];
+#pragma unroll
+    for (int d = 0; d < kS; ++d)
+      asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                   : "=f"(v[d][0]), "=f"(v[d][1]), "=f"(v[d][2]), "=f"(v[d][3]), "=f"(v[d][4]), "=f"(v[d][5]),
+                     "=f"(v[d][6]), "=f"(v[d][7])
+                   : "r"(trow + (uint32_t)(d * kTN + c0)));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      // diagonals 2 and 3 (d = 0, 1) exactly in f64; 4 .. 10 in float-float, smallest first
+      dfl::df64 lo(0.0f);
+#pragma unroll
+      for (int d = kS - 1; d >= 2; --d) {
+        const float x = v[d][c] * __uint_as_float((uint32_t)(127 - kBits * (d + 2)) << 23);  // exact: 64^-(d+2)
+        lo = lo + dfl::df64(x);
+      }
+      double r = fma(dfl::widen(v[0][c]), 0x1p-12, dfl::widen(v[1][c]) * 0x1p-18);  // exact
+      r += dfl::join(lo);
+      const int F = P.Fexp[n0 + c0 + c];
+      r = (!ok || E >= kNonFinite || F >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll) : scalbn(r, E + F);
+      outp[c0 + c] = r;
+    }
   }
 
-  // the share's f64 result, scaled by the row and column powers of two: lane (gid, tig) holds rows
-  // gid and gid + 8, columns 2 tig and 2 tig + 1 of each 8-wide tile (planes are padded: no bounds)
-  const int gid = lane >> 2, tig = lane & 3;
-  double *part = P.part + (size_t)blockIdx.z * P.Mp * P.Np;
-#pragma unroll
-  for (int j = 0; j < kNT; ++j)
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int rl = wm * 16 + gid + 8 * h, cl = wn * 8 * kNT + j * 8 + 2 * tig;
-      const int E = sE[rl];
-      double2 v;
-      v.x = (E >= kNonFinite || sF[cl] >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
-                                                     : scalbn(acc64[(4 * j + 2 * h) * kThreads], E + sF[cl]);
-      v.y = (E >= kNonFinite || sF[cl + 1] >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll)
-                                                         : scalbn(acc64[(4 * j + 2 * h + 1) * kThreads], E + sF[cl + 1]);
-      *reinterpret_cast<double2 *>(part + (size_t)(m0 + rl) * P.Np + n0 + cl) = v;
-    }
+  asm volatile("tcgen05.fence::before_thread_sync;");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;");
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
 }
 
 // The layer's epilogue over the chunk's n x N outputs, from the shares' partial results summed in
@@ -734,8 +734,8 @@ size_t layout(const FitShape &s, bool fwd, Layer *out) {
     Layer &L = out[q];
     L.K = fwd ? s.w[l - 1] : s.w[l];
     L.N = fwd ? s.w[l] : s.w[l - 1];
-    L.Np = (int)round_up(L.N, kBN);
-    L.Kp = (int)round_up(L.K, kBK);
+    L.Np = (int)round_up(L.N, kTN);
+    L.Kp = (int)round_up(L.K, kTK);
     L.planes = off;
     off += (size_t)round_up((int64_t)kS * L.Np * L.Kp * 2, 256);
     L.fexp = off;
@@ -753,35 +753,45 @@ struct WorkMap {
   size_t buffers;          // byte offset of the buffers between layers
 };
 
-// K shares of one GEMM: enough that tiles x shares reaches kTargetBlocks (~6.7 waves of one block
-// per SM on 152 SMs), but at least kMinShareSlices slices per share (a block's first slice arrives
-// before any MMA can start; shorter shares spend their time waiting for it).  Shares x tiles x
-// tile stays below kTargetBlocks x tile + Mp x Np, which bounds the partial-result buffer.
-constexpr int64_t kTargetBlocks = 1024;
-constexpr int kMinShareSlices = 8;
+// K shares of one GEMM: at most kMaxShareK each (the exactness bound), and more when the tiles
+// alone would not give every SM a few CTAs (one CTA per SM), but at least kMinShareSlices slices
+// each (a CTA's pipeline fill and combine are paid once per share).
+constexpr int kMaxShareSlices = kMaxShareK / kTK;
+constexpr int64_t kTargetCtas = 4 * 152;
+constexpr int kMinShareSlices = 6;
 int ksplit_for(int64_t Mp, int Np, int Kp) {
-  const int64_t tiles = (Mp / kBM) * (Np / kBN);
-  const int slices = Kp / kBK;
-  const int64_t want = std::min<int64_t>((kTargetBlocks + tiles - 1) / tiles, std::max(1, slices / kMinShareSlices));
-  const int per = (int)((slices + want - 1) / want);
-  return (slices + per - 1) / per;  // no empty share
+  const int64_t tiles = (Mp / kTM) * (Np / kTN);
+  const int slices = Kp / kTK;
+  int want = (int)std::min<int64_t>((kTargetCtas + tiles - 1) / tiles, std::max(1, slices / kMinShareSlices));
+  want = std::max(want, (slices + kMaxShareSlices - 1) / kMaxShareSlices);
+  const int per = (slices + want - 1) / want;
+  return (slices + per - 1) / per;  // no empty share; per <= kMaxShareSlices
 }
+
 WorkMap work_map(const FitShape &s, int64_t nloc) {
   Layer L[DP_MAX_LAYERS];
   WorkMap m{};
   m.bplanes = std::max(layout(s, true, L), layout(s, false, L));
   int kmax = 1;
   for (int l = 0; l < s.nlayer; ++l) kmax = std::max(kmax, s.w[l]);  // every GEMM's K is a layer width
-  m.Kpmax = (int)round_up(kmax, kBK);
+  m.Kpmax = (int)round_up(kmax, kTK);
   int64_t maxn = 0;  // rows of the largest type
   for (int t = 0; t < s.ntypes; ++t) maxn = std::max<int64_t>(maxn, s.start[t + 1] - s.start[t]);
-  m.Mp = round_up(std::min<int64_t>(std::max<int64_t>(maxn, 1), kChunkRows), kBM);
+  m.Mp = round_up(std::min<int64_t>(std::max<int64_t>(maxn, 1), kChunkRows), kTM);
   m.aplanes = m.bplanes;
   m.aexp = m.aplanes + (size_t)round_up((int64_t)kS * m.Mp * m.Kpmax * 2, 256);
   m.part = m.aexp + (size_t)round_up(m.Mp * 4, 256);
-  int Npmax = kBN;
-  for (int l = 0; l < s.nlayer; ++l) Npmax = std::max(Npmax, (int)round_up(s.w[l], kBN));
-  m.buffers = m.part + (size_t)round_up((kTargetBlocks * kBM * kBN + m.Mp * Npmax) * 8, 256);
+  // shares x Mp x Np over the GEMMs: below kTargetCtas tiles plus the largest chunk's Mp x Np, or
+  // the exactness bound's shares at the largest chunk (a smaller chunk stays under both)
+  int Npmax = kTN;
+  for (int l = 0; l < s.nlayer; ++l) Npmax = std::max(Npmax, (int)round_up(s.w[l], kTN));
+  int64_t part = kTargetCtas * kTM * kTN + m.Mp * Npmax;
+  for (int q = 0; q + 1 < s.nlayer; ++q)
+    for (int dir = 0; dir < 2; ++dir) {
+      layout(s, dir == 0, L);
+      part = std::max<int64_t>(part, (int64_t)ksplit_for(m.Mp, L[q].Np, L[q].Kp) * m.Mp * L[q].Np);
+    }
+  m.buffers = m.part + (size_t)round_up(part * 8, 256);
   return m;
 }
 
@@ -793,10 +803,8 @@ size_t work_bytes(const FitShape &s, int64_t nloc) {
 int set_smem() {
   static std::atomic<bool> done{false};
   if (done.load(std::memory_order_acquire)) return DP_OK;
-  for (auto k : {&gemm_kernel<true>, &gemm_kernel<false>}) {
-    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemTotal);
-    if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_fitting_*_tc_f64: %s", cudaGetErrorString(e));
-  }
+  const cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemTotal);
+  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_fitting_*_tc_f64: %s", cudaGetErrorString(e));
   done.store(true, std::memory_order_release);
   return DP_OK;
 }
@@ -830,13 +838,13 @@ int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaSt
     TcGemm C = G;
     C.r0 = r0;
     C.n = std::min<int64_t>(kChunkRows, r_end - r0);
-    C.Mp = round_up(C.n, kBM);
+    C.Mp = round_up(C.n, kTM);
     int rc = split_rows(G.A + r0 * G.lda, G.lda, 1, C.n, G.K, C.Mp, L.Kp, work + m.aplanes, work + m.aexp, st, who);
     if (rc) return rc;
     const int ksplit = ksplit_for(C.Mp, L.Np, L.Kp);
-    C.slices_per_split = (L.Kp / kBK + ksplit - 1) / ksplit;
-    const dim3 grid((unsigned)(L.Np / kBN), (unsigned)(C.Mp / kBM), (unsigned)ksplit);
-    gemm_kernel<kFwd><<<grid, kThreads, kSmemTotal, st>>>(C);
+    C.slices_per_split = (L.Kp / kTK + ksplit - 1) / ksplit;
+    const dim3 grid((unsigned)(L.Np / kTN), (unsigned)(C.Mp / kTM), (unsigned)ksplit);
+    gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(C);
     if ((rc = launch_status(who))) return rc;
     const int64_t total = C.n * C.N;
     epilogue_kernel<kFwd><<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(C, ksplit);
@@ -988,6 +996,7 @@ size_t work_bytes_api(const int32_t *widths, int nlayer, int64_t nloc) {
   return work_bytes(s, nloc);
 }
 }  // namespace tc
+
 
 // ------------------------------------------------- backward without allocation
 // Some callers cannot hand this library a scratch buffer: an MD engine's force
