@@ -370,13 +370,14 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
 // Every (A_s B_t)_ij is a sum of integer products |A_s B_t| <= 3969; a diagonal
 // d has at most 9 of them, so its fp32 sum on the tensor cores is exact while
 // a block's share of K is at most kMaxShareK = 448 (9 x 448 x 3969 < 2^24).
-// The 9 diagonal sums of an output are then combined with one rounding: the
-// two largest exactly in f64, the rest in float-float (its rounding lies some
-// 2^-60 below the result), one f64 add for the two.  What rounds is that add,
-// the adds of the shares' f64 results (epilogue_kernel), the 54-bit truncation
-// of the operands and the dropped terms: |error| <~ K 2^-50 max_k|a_ik|
-// max_k|b_kj|, against K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row
-// or column with an inf or NaN gives NaN outputs.
+// The 9 diagonal sums of an output are combined on the FP32 pipe into four
+// floats (the two largest by an exact two-sum, the rest in float-float, whose
+// rounding lies ~2^-60 below the result); epilogue_kernel adds the shares'
+// floats into a three-float sum by exact two-sums and converts it to f64 once.
+// What rounds is that conversion, the 54-bit truncation of the operands and
+// the dropped terms: |error| <~ K 2^-50 max_k|a_ik| max_k|b_kj|, against
+// K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column with an
+// inf or NaN gives NaN outputs.
 //
 // gemm_kernel: one CTA of 128 threads per 128 x 48 output tile and share of K,
 // one CTA per SM (its 9 diagonal accumulators take 432 of the SM's 512 TMEM
@@ -388,8 +389,8 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
 // fp32 accumulators in TMEM, one per diagonal) of a stage and commits them to
 // the stage's mbarrier, which frees the stage for the slice four ahead.  At
 // the end each warp reads its 32 TMEM lanes (rows), combines the diagonals and
-// writes the share's f64 result; epilogue_kernel sums the shares in a fixed
-// order and applies the layer's epilogue.  A is always a plain matrix: the
+// writes the share's result as four floats; epilogue_kernel sums the shares in
+// a fixed order, scales by 2^(E+F) and applies the layer's epilogue.  A is always a plain matrix: the
 // forward keeps each layer's input v_l (tanh outputs plus the skip) in a work
 // buffer, the backward writes dE/dv (for the next skip) and dE/dv (1 - t^2)
 // (the next A).  Every wait on an mbarrier is bounded; a wait that gives up
@@ -494,7 +495,7 @@ struct TcGemm {
   const uint16_t *planes;   // B: [kS][Np][Kp]
   const int *Fexp;
   int Np, Kp;
-  double *part;             // [ksplit][Mp][Np]: the f64 result of each share of K (grid z)
+  float4 *part;             // [ksplit][Mp][Np]: each share's result (grid z) as four floats, see gemm_kernel
   int slices_per_split;
   bool skip;
   // forward
@@ -634,8 +635,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   // combine the diagonals of row 32 (warp % 4) + lane (the warp's TMEM lane quadrant), the warp's
   // third of the columns, 8 at a time
   const int rl = 32 * (warp & 3) + lane;
-  const int E = P.Eexp[m0 + rl];
-  double *outp = P.part + ((size_t)blockIdx.z * P.Mp + m0 + rl) * P.Np + n0;
+  float4 *outp = P.part + ((size_t)blockIdx.z * P.Mp + m0 + rl) * P.Np + n0;
   const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
   constexpr int kColsPerWarp = kTN / (kThreads / 128);
   static_assert(kColsPerWarp % 8 == 0, "column share");
@@ -651,18 +651,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
-      // diagonals 2 and 3 (d = 0, 1) exactly in f64; 4 .. 10 in float-float, smallest first
+      // sum_d v_d 64^-(d+2) as four floats on the FP32 pipe: diagonals 2 and 3 (d = 0, 1) as an exact
+      // two-sum, 4 .. 10 in float-float, smallest first (its rounding lies ~2^-60 below the sum).
+      // The scaling by 2^(E+F), and all f64 arithmetic, is left to epilogue_kernel.
       dfl::df64 lo(0.0f);
 #pragma unroll
       for (int d = kS - 1; d >= 2; --d) {
         const float x = v[d][c] * __uint_as_float((uint32_t)(127 - kBits * (d + 2)) << 23);  // exact: 64^-(d+2)
         lo = lo + dfl::df64(x);
       }
-      double r = fma(dfl::widen(v[0][c]), 0x1p-12, dfl::widen(v[1][c]) * 0x1p-18);  // exact
-      r += dfl::join(lo);
-      const int F = P.Fexp[n0 + c0 + c];
-      r = (!ok || E >= kNonFinite || F >= kNonFinite) ? __longlong_as_double(0x7ff8000000000000ll) : scalbn(r, E + F);
-      outp[c0 + c] = r;
+      const float a = v[0][c] * 0x1p-12f, b = v[1][c] * 0x1p-18f;  // exact
+      const float s = __fadd_rn(a, b), bb = __fsub_rn(s, a);
+      const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+      outp[c0 + c] = ok ? make_float4(s, e, lo.hi, lo.lo) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
     }
   }
 
@@ -686,8 +687,31 @@ __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int kspli
     const int64_t rc = e / P.N;
     const int nn = (int)(e - rc * P.N);
     const int64_t row = P.r0 + rc;
-    double v = P.part[rc * P.Np + nn];
-    for (int z = 1; z < ksplit; ++z) v += P.part[((size_t)z * P.Mp + rc) * P.Np + nn];
+    // the shares' four floats each, added into a three-float sum by exact two-sums on the FP32 pipe
+    // (only the last component rounds, ~2^-72 below the sum), then one conversion to f64 and the
+    // scaling by the row and column powers of two
+    float s0 = 0.f, s1 = 0.f, s2 = 0.f;
+    auto add = [&](float x) {
+      float t = __fadd_rn(s0, x), z = __fsub_rn(t, s0);
+      const float e0 = __fadd_rn(__fsub_rn(s0, __fsub_rn(t, z)), __fsub_rn(x, z));
+      s0 = t;
+      t = __fadd_rn(s1, e0);
+      z = __fsub_rn(t, s1);
+      const float e1 = __fadd_rn(__fsub_rn(s1, __fsub_rn(t, z)), __fsub_rn(e0, z));
+      s1 = t;
+      s2 = __fadd_rn(s2, e1);
+    };
+    for (int z = 0; z < ksplit; ++z) {
+      const float4 q = P.part[((size_t)z * P.Mp + rc) * P.Np + nn];
+      add(q.x);
+      add(q.y);
+      add(q.z);
+      add(q.w);
+    }
+    const int E = P.Eexp[rc], F = P.Fexp[nn];
+    double v = __dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2));
+    v = (E >= kNonFinite || F >= kNonFinite || s0 != s0) ? __longlong_as_double(0x7ff8000000000000ll)
+                                                          : scalbn(v, E + F);
     if constexpr (kFwd) {
       const double t = dfl::tanh_d(v + P.bias[nn]);
       P.act[row * P.ldact + nn] = t;
@@ -791,7 +815,7 @@ WorkMap work_map(const FitShape &s, int64_t nloc) {
       layout(s, dir == 0, L);
       part = std::max<int64_t>(part, (int64_t)ksplit_for(m.Mp, L[q].Np, L[q].Kp) * m.Mp * L[q].Np);
     }
-  m.buffers = m.part + (size_t)round_up(part * 8, 256);
+  m.buffers = m.part + (size_t)round_up(part * 16, 256);
   return m;
 }
 
@@ -832,7 +856,7 @@ int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaSt
   G.Kp = L.Kp;
   G.aplanes = reinterpret_cast<const uint16_t *>(work + m.aplanes);
   G.Eexp = reinterpret_cast<const int *>(work + m.aexp);
-  G.part = reinterpret_cast<double *>(work + m.part);
+  G.part = reinterpret_cast<float4 *>(work + m.part);
   const int64_t r_end = G.r0 + G.n;
   for (int64_t r0 = G.r0; r0 < r_end; r0 += kChunkRows) {
     TcGemm C = G;
