@@ -401,14 +401,14 @@ constexpr int kBits = 6;   // bits per digit
 constexpr int kFrac = kS * kBits;  // 54 fractional bits
 constexpr int kTM = 128, kTN = 48, kTK = 16;  // CTA tile; K per stage (one MMA)
 constexpr int kStages = 4;
-constexpr int kThreads = 384;  // 12 warps: every thread copies one 16-byte slot of every plane; three warps per TMEM lane quadrant
+constexpr int kThreads = 128;  // one warp per TMEM lane quadrant; lane 0 of warps 0 and 1: producer and MMA issuer
 constexpr int kMaxShareK = 448;
 constexpr int kNonFinite = 1 << 20;  // exponent of a row or column holding inf or NaN
 constexpr uint32_t kLBO = 128, kSBO = 256;  // core matrices: next along K at +128 B, next 8 rows at +256 B
 constexpr int kPlaneA = kTM * kTK * 2, kPlaneB = kTN * kTK * 2;  // bytes of one digit plane in a stage
 constexpr int kStageBytes = kS * (kPlaneA + kPlaneB);
 constexpr uint32_t kTmemCols = 512;  // allocation (a power of two); kS * kTN = 432 used
-constexpr size_t kSmemTotal = (size_t)kStages * kStageBytes + 64;
+constexpr size_t kSmemTotal = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16;
 static_assert((size_t)kS * kMaxShareK * 63 * 63 < (1u << 24), "fp32 diagonal sums must stay exact");
 static_assert(kMaxShareK % kTK == 0 && kS * kTN <= (int)kTmemCols, "shares and TMEM");
 static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
@@ -451,17 +451,17 @@ __device__ __forceinline__ uint32_t sign_pair(double x0, double x1) {
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src));
-}
-
-// Rows of a matrix as digit planes [kS][rows_p][Kp] (fp16, a row's K values contiguous) with the
-// rows' exponents [rows_p]: element (r, k) of the source is X[r ld_r + k ld_k]; rows >= nrows and
-// columns >= K are zero.  One warp per row.  Used for the A operand (rows of the layer input) and
-// for B (forward: the columns of W, ld_r = 1, ld_k = N; backward: the rows of W).
+// Rows of a matrix as digit planes, laid out as the shared-memory image of each (tile of RT rows,
+// 16-deep K slice) block that gemm_kernel copies in one piece: block (r / RT, k / 16) holds the kS
+// planes of those rows and columns, plane s at s RT 32 bytes, and in a plane the tcgen05 K-major
+// core matrices (8 rows x 8 k = 128 bytes; the second 8 k of the slice at +128 B, the next 8 rows
+// at +256 B).  Also the rows' exponents [rows_p].  Element (r, k) of the source is X[r ld_r + k ld_k];
+// rows >= nrows and columns >= K are zero.  One warp per row.  Used for the A operand (rows of the
+// layer input, RT = kTM) and for B (RT = kTN; forward: the columns of W, ld_r = 1, ld_k = N;
+// backward: the rows of W).
 __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
-                                                         int64_t nrows, int K, int64_t rows_p, int Kp,
-                                                         uint32_t *__restrict__ planes, int *__restrict__ exps) {
+                                                         int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
+                                                         unsigned char *__restrict__ planes, int *__restrict__ exps) {
   const int lane = threadIdx.x & 31;
   const int64_t r = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
   if (r >= rows_p) return;  // warp-uniform
@@ -471,12 +471,17 @@ __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restric
   for (int k = lane; k < K; k += 32) eb = max(eb, exp_bits(x(k)));
   const int E = exp_of_max(__reduce_max_sync(0xffffffffu, eb));
   if (lane == 0) exps[r] = E;
+  const size_t plane = (size_t)RT * kTK * 2, block = kS * plane;
+  const int ri = (int)(r % RT);
+  unsigned char *rowbase = planes + (size_t)(r / RT) * (Kp / kTK) * block + (ri >> 3) * kSBO + (ri & 7) * 16;
   for (int c2 = lane; c2 < Kp / 2; c2 += 32) {
-    const double x0 = x(2 * c2), x1 = x(2 * c2 + 1);
+    const int k = 2 * c2;
+    const double x0 = x(k), x1 = x(k + 1);
     uint32_t h[kS];
     digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
+    unsigned char *dst = rowbase + (size_t)(k / kTK) * block + ((k % kTK) >> 3) * kLBO + (k & 7) * 2;
 #pragma unroll
-    for (int s = 0; s < kS; ++s) planes[((size_t)s * rows_p + r) * (Kp / 2) + c2] = h[s];
+    for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
   }
 }
 
@@ -489,10 +494,10 @@ struct TcGemm {
   int K, N;
   const double *A;  // the layer input itself (forward: its skip term)
   int64_t lda;
-  const uint16_t *aplanes;  // [kS][Mp][Kp]
+  const unsigned char *aplanes;  // A's blocks [Mp / kTM][Kp / kTK] of kS x kPlaneA bytes
   const int *Eexp;          // [Mp]
   int64_t Mp;
-  const uint16_t *planes;   // B: [kS][Np][Kp]
+  const unsigned char *planes;   // B's blocks [Np / kTN][Kp / kTK] of kS x kPlaneB bytes
   const int *Fexp;
   int Np, Kp;
   float4 *part;             // [ksplit][Mp][Np]: each share's result (grid z) as four floats, see gemm_kernel
@@ -536,29 +541,26 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   return done != 0;
 }
 
-__device__ __forceinline__ void cp_async_wait_pending(int n) {  // at most n of this thread's copy groups pending
-  if (n >= 2)
-    asm volatile("cp.async.wait_group 2;" ::: "memory");
-  else if (n == 1)
-    asm volatile("cp.async.wait_group 1;" ::: "memory");
-  else
-    asm volatile("cp.async.wait_group 0;" ::: "memory");
-}
-
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   extern __shared__ __align__(1024) unsigned char smem[];
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);  // one per stage
-  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bars + kStages);
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);  // stage loaded
+  uint64_t *empty = full + kStages;                                               // stage's MMAs done
+  uint64_t *done = empty + kStages;                                               // every MMA done (one use)
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(done + 1);
+  int *flags = reinterpret_cast<int *>(tmem_holder + 1);                          // producer / issuer ok
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t m0 = (int64_t)blockIdx.y * kTM;
   const int n0 = blockIdx.x * kTN;
-  const int slices_total = P.Kp / kTK;
+  const int nslices = P.Kp / kTK;
   const int i0 = blockIdx.z * P.slices_per_split;
-  const int nsl = min(slices_total - i0, P.slices_per_split);  // > 0: no empty share
+  const int nsl = min(nslices - i0, P.slices_per_split);  // > 0: no empty share
 
   if (tid == 0) {
-    for (int s = 0; s < kStages; ++s)
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bars + s)));
+    for (int s = 0; s < kStages; ++s) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(full + s)));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(empty + s)));
+    }
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(done)));
     asm volatile("fence.mbarrier_init.release.cluster;");
   }
   if (warp == 0) {
@@ -566,51 +568,47 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
                  "r"(kTmemCols));
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
   }
-
-  // copies of slice j into stage st: thread tid < 2 (kTM + kTN) owns one 16-byte slot (a row and
-  // one of its two 8-k chunks) of A (first 2 kTM threads) or B, and copies it for every plane, from
-  // the plane's row in global memory to its place in the core-matrix layout
-  const uint32_t sbase = smem_u32(smem);
-  const bool loader = tid < 2 * (kTM + kTN);
-  const bool a_side = tid < 2 * kTM;
-  const int lr = (a_side ? tid : tid - 2 * kTM) >> 1, lc = tid & 1;
-  const uint16_t *lsrc = !loader ? P.planes
-                         : a_side ? P.aplanes + (size_t)(m0 + lr) * P.Kp + 8 * lc
-                                  : P.planes + (size_t)(n0 + lr) * P.Kp + 8 * lc;
-  const size_t lsstride = a_side ? (size_t)P.Mp * P.Kp : (size_t)P.Np * P.Kp;  // halves between planes
-  const uint32_t ldst = (a_side ? 0u : (uint32_t)(kS * kPlaneA)) + (lr >> 3) * kSBO + lc * kLBO + (lr & 7) * 16;
-  const uint32_t ldstride = a_side ? kPlaneA : kPlaneB;
-  auto load_slice = [&](int j, int st) {
-    if (loader) {
-      const uint16_t *src = lsrc + (i0 + j) * kTK;
-      uint32_t dst = sbase + st * kStageBytes + ldst;
-#pragma unroll
-      for (int s = 0; s < kS; ++s, src += lsstride, dst += ldstride) cp_async16(dst, src);
-    }
-    asm volatile("cp.async.commit_group;");
-  };
-
-  const int pre = min(kStages - 1, nsl);
-  for (int j = 0; j < pre; ++j) load_slice(j, j);
   asm volatile("tcgen05.fence::before_thread_sync;");
   __syncthreads();
   asm volatile("tcgen05.fence::after_thread_sync;");
   const uint32_t tmem = *tmem_holder;
-
+  const uint32_t sbase = smem_u32(smem);
   bool ok = true;
-  for (int i = 0; i < nsl; ++i) {  // uniform
-    cp_async_wait_pending(min(kStages - 2, nsl - 1 - i));  // slice i's copies (this thread's) have landed
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // the copies, visible to the tensor core
-    __syncthreads();
-    if (tid == 0 && ok) {
+
+  if (warp == 0 && lane == 0) {
+    // producer: each slice's A and B blocks, one bulk copy each, counted in bytes on the stage's
+    // "full" barrier; a stage is reused once the MMAs that read it have completed ("empty")
+    const unsigned char *asrc = P.aplanes + ((size_t)blockIdx.y * nslices + i0) * (kS * kPlaneA);
+    const unsigned char *bsrc = P.planes + ((size_t)blockIdx.x * nslices + i0) * (kS * kPlaneB);
+    for (int j = 0; j < nsl && ok; ++j) {
+      const int st = j % kStages;
+      if (j >= kStages) ok = mbar_wait(smem_u32(empty + st), (uint32_t)((j / kStages - 1) & 1));
+      if (!ok) break;
+      const uint32_t bar = smem_u32(full + st), dst = sbase + st * kStageBytes;
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"((uint32_t)kStageBytes)
+                   : "memory");
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                   "l"(asrc + (size_t)j * (kS * kPlaneA)), "r"((uint32_t)(kS * kPlaneA)), "r"(bar)
+                   : "memory");
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       dst + kS * kPlaneA),
+                   "l"(bsrc + (size_t)j * (kS * kPlaneB)), "r"((uint32_t)(kS * kPlaneB)), "r"(bar)
+                   : "memory");
+    }
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer: the 45 digit products of each slice once it has landed, then a commit that frees the stage
+    for (int i = 0; i < nsl && ok; ++i) {
+      const int st = i % kStages;
+      ok = mbar_wait(smem_u32(full + st), (uint32_t)((i / kStages) & 1));
+      if (!ok) break;
       asm volatile("tcgen05.fence::after_thread_sync;");
-      const uint32_t stage = sbase + (i % kStages) * kStageBytes;
+      const uint64_t a0 = smem_desc(sbase + st * kStageBytes), b0 = smem_desc(sbase + st * kStageBytes + kS * kPlaneA);
 #pragma unroll
       for (int t = 0; t < kS; ++t) {
-        const uint64_t bd = smem_desc(stage + kS * kPlaneA + t * kPlaneB);
+        const uint64_t bd = b0 + (uint64_t)((t * kPlaneB) >> 4);  // start-address field, in 16-byte units
 #pragma unroll
         for (int s = 0; s + t < kS; ++s) {  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
-          const uint64_t ad = smem_desc(stage + s * kPlaneA);
+          const uint64_t ad = a0 + (uint64_t)((s * kPlaneA) >> 4);
           const uint32_t acc = (i > 0 || t > 0) ? 1u : 0u;  // a diagonal's first product overwrites
           asm volatile(
               "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
@@ -619,17 +617,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
         }
       }
       asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bars + i % kStages)));
+          smem_u32(empty + st)));
     }
-    // refill the stage of slice i - 1 with slice i + kStages - 1 once slice i - 1's MMAs are done
-    const int j = i + kStages - 1;
-    if (j < nsl) {
-      if (i >= 1) ok = ok && mbar_wait(smem_u32(bars + (i - 1) % kStages), (uint32_t)(((i - 1) / kStages) & 1));
-      load_slice(j, j % kStages);
-    }
+    // one more commit, on a barrier used once: it completes when every MMA issued above has (also
+    // after a wait that gave up, so that nobody waits on it in vain)
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(done)));
   }
-  // all MMAs of the share done: the last slice's commit tracks every earlier one
-  ok = ok && mbar_wait(smem_u32(bars + (nsl - 1) % kStages), (uint32_t)(((nsl - 1) / kStages) & 1));
+  if (lane == 0 && warp < 2) flags[warp] = ok;
+  __syncwarp();
+  // The other warps wait here rather than on a stage barrier: a parity wait can only tell apart the
+  // current phase and the one before, and they would start it phases ahead of the MMAs.
+  __syncthreads();
+  ok = flags[0] && flags[1];
+  ok = mbar_wait(smem_u32(done), 0) && ok;
   asm volatile("tcgen05.fence::after_thread_sync;");
 
   // combine the diagonals of row 32 (warp % 4) + lane (the warp's TMEM lane quadrant), the warp's
@@ -833,28 +833,27 @@ int set_smem() {
   return DP_OK;
 }
 
-int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp,
+int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
                unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
-  split_rows_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp,
-                                                                   reinterpret_cast<uint32_t *>(planes),
+  split_rows_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT, planes,
                                                                    reinterpret_cast<int *>(exps));
   return launch_status(who);
 }
 
 // The weights of one layer as B planes: forward B[k][n] = W[k][n] (W is [K][N]), backward B[k][n] = W[n][k]
 int split_b(const double *W, const Layer &L, bool fwd, unsigned char *work, cudaStream_t st, const char *who) {
-  return fwd ? split_rows(W, 1, L.N, L.N, L.K, L.Np, L.Kp, work + L.planes, work + L.fexp, st, who)
-             : split_rows(W, L.K, 1, L.N, L.K, L.Np, L.Kp, work + L.planes, work + L.fexp, st, who);
+  return fwd ? split_rows(W, 1, L.N, L.N, L.K, L.Np, L.Kp, kTN, work + L.planes, work + L.fexp, st, who)
+             : split_rows(W, L.K, 1, L.N, L.K, L.Np, L.Kp, kTN, work + L.planes, work + L.fexp, st, who);
 }
 
 // G over its rows in chunks of at most kChunkRows: each chunk's A rows split into planes, then the GEMM
 template <bool kFwd>
 int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaStream_t st, const char *who) {
-  G.planes = reinterpret_cast<const uint16_t *>(work + L.planes);
+  G.planes = work + L.planes;
   G.Fexp = reinterpret_cast<const int *>(work + L.fexp);
   G.Np = L.Np;
   G.Kp = L.Kp;
-  G.aplanes = reinterpret_cast<const uint16_t *>(work + m.aplanes);
+  G.aplanes = work + m.aplanes;
   G.Eexp = reinterpret_cast<const int *>(work + m.aexp);
   G.part = reinterpret_cast<float4 *>(work + m.part);
   const int64_t r_end = G.r0 + G.n;
@@ -863,7 +862,7 @@ int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaSt
     C.r0 = r0;
     C.n = std::min<int64_t>(kChunkRows, r_end - r0);
     C.Mp = round_up(C.n, kTM);
-    int rc = split_rows(G.A + r0 * G.lda, G.lda, 1, C.n, G.K, C.Mp, L.Kp, work + m.aplanes, work + m.aexp, st, who);
+    int rc = split_rows(G.A + r0 * G.lda, G.lda, 1, C.n, G.K, C.Mp, L.Kp, kTM, work + m.aplanes, work + m.aexp, st, who);
     if (rc) return rc;
     const int ksplit = ksplit_for(C.Mp, L.Np, L.Kp);
     C.slices_per_split = (L.Kp / kTK + ksplit - 1) / ksplit;
