@@ -456,30 +456,48 @@ __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)_
 // planes of those rows and columns, plane s at s RT 32 bytes, and in a plane the tcgen05 K-major
 // core matrices (8 rows x 8 k = 128 bytes; the second 8 k of the slice at +128 B, the next 8 rows
 // at +256 B).  Also the rows' exponents [rows_p].  Element (r, k) of the source is X[r ld_r + k ld_k];
-// rows >= nrows and columns >= K are zero.  One warp per row.  Used for the A operand (rows of the
+// rows >= nrows and columns >= K are zero (row_exps_kernel first finds the exponents).  Used for the A operand (rows of the
 // layer input, RT = kTM) and for B (RT = kTN; forward: the columns of W, ld_r = 1, ld_k = N;
 // backward: the rows of W).
-__global__ void __launch_bounds__(128) split_rows_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
-                                                         int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
-                                                         unsigned char *__restrict__ planes, int *__restrict__ exps) {
+__global__ void __launch_bounds__(128) row_exps_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
+                                                       int64_t nrows, int K, int64_t rows_p, int *__restrict__ exps) {
+  // one warp per row: E with max_k |x_rk| < 2^E
   const int lane = threadIdx.x & 31;
   const int64_t r = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
   if (r >= rows_p) return;  // warp-uniform
+  int eb = 0;
+  if (r < nrows)
+    for (int k = lane; k < K; k += 32) eb = max(eb, exp_bits(__ldg(X + r * ld_r + k * ld_k)));
+  eb = __reduce_max_sync(0xffffffffu, eb);
+  if (lane == 0) exps[r] = exp_of_max(eb);
+}
+
+constexpr int kSplitK = 64;  // K per warp of split_rows_kernel
+__global__ void __launch_bounds__(128) split_rows_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
+                                                         int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
+                                                         unsigned char *__restrict__ planes,
+                                                         const int *__restrict__ exps) {
+  // one warp per (group of 8 rows, kSplitK of K): lane = (row ri8 = lane / 4, pair of k kp = lane % 4),
+  // so that per plane and 8 k the warp writes one whole 128-byte core matrix
+  const int lane = threadIdx.x & 31, ri8 = lane >> 2, kp = lane & 3;
+  const int kchunks = (Kp + kSplitK - 1) / kSplitK;
+  const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int64_t g = w / kchunks;  // 8-row group
+  if (g * 8 >= rows_p) return;    // warp-uniform
+  const int kc = (int)(w - g * kchunks);
+  const int64_t r = g * 8 + ri8;
   const double *__restrict__ xr = X + (r < nrows ? r : 0) * ld_r;
   auto x = [&](int k) { return (r < nrows && k < K) ? __ldg(xr + k * ld_k) : 0.0; };
-  int eb = 0;
-  for (int k = lane; k < K; k += 32) eb = max(eb, exp_bits(x(k)));
-  const int E = exp_of_max(__reduce_max_sync(0xffffffffu, eb));
-  if (lane == 0) exps[r] = E;
+  const int E = exps[r];
   const size_t plane = (size_t)RT * kTK * 2, block = kS * plane;
   const int ri = (int)(r % RT);
-  unsigned char *rowbase = planes + (size_t)(r / RT) * (Kp / kTK) * block + (ri >> 3) * kSBO + (ri & 7) * 16;
-  for (int c2 = lane; c2 < Kp / 2; c2 += 32) {
-    const int k = 2 * c2;
+  unsigned char *rowbase = planes + (size_t)(r / RT) * (Kp / kTK) * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
+  for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
+    const int k = k0 + 2 * kp;
     const double x0 = x(k), x1 = x(k + 1);
     uint32_t h[kS];
     digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
-    unsigned char *dst = rowbase + (size_t)(k / kTK) * block + ((k % kTK) >> 3) * kLBO + (k & 7) * 2;
+    unsigned char *dst = rowbase + (size_t)(k0 / kTK) * block + ((k0 % kTK) >> 3) * kLBO;
 #pragma unroll
     for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
   }
@@ -680,6 +698,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
 //   backward: s = acc (+ S[row][col] or g_row wo_col when the layer kept its width); then either
 //             out[row][col] = s (dE/dD, the last GEMM) or S_next[row][col] = s and
 //             Z[row][col] = s (1 - t_prev^2) with t_prev = T[row][col] (the next GEMM's A)
+// f 2^e as a double, exactly, by moving fields (f finite; |e| < 900, so a normal result stays normal
+// and a float that is zero stays zero; float subnormals, which the sums do not produce, widen to 0)
+__device__ __forceinline__ double widen_pow2(float f, int e) {
+  const double d = dfl::widen(f);
+  const long long b = __double_as_longlong(d);
+  return (b & 0x7fffffffffffffffll) ? __longlong_as_double(b + ((long long)e << 52)) : d;
+}
+
 template <bool kFwd>
 __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int ksplit) {
   const int64_t total = P.n * P.N;
@@ -709,9 +735,13 @@ __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int kspli
       add(q.w);
     }
     const int E = P.Eexp[rc], F = P.Fexp[nn];
-    double v = __dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2));
-    v = (E >= kNonFinite || F >= kNonFinite || s0 != s0) ? __longlong_as_double(0x7ff8000000000000ll)
-                                                          : scalbn(v, E + F);
+    double v;
+    if (E >= kNonFinite || F >= kNonFinite || s0 != s0)
+      v = __longlong_as_double(0x7ff8000000000000ll);
+    else if (E + F > -900 && E + F < 900)  // the scaling moves exponent fields only (sums stay normal)
+      v = __dadd_rn(__dadd_rn(widen_pow2(s0, E + F), widen_pow2(s1, E + F)), widen_pow2(s2, E + F));
+    else
+      v = scalbn(__dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2)), E + F);
     if constexpr (kFwd) {
       const double t = dfl::tanh_d(v + P.bias[nn]);
       P.act[row * P.ldact + nn] = t;
@@ -835,8 +865,13 @@ int set_smem() {
 
 int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
                unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
-  split_rows_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT, planes,
-                                                                   reinterpret_cast<int *>(exps));
+  row_exps_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p,
+                                                                 reinterpret_cast<int *>(exps));
+  int rc = launch_status(who);
+  if (rc) return rc;
+  const int64_t warps = rows_p / 8 * ((Kp + kSplitK - 1) / kSplitK);
+  split_rows_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT, planes,
+                                                                 reinterpret_cast<const int *>(exps));
   return launch_status(who);
 }
 
