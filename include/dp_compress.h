@@ -444,23 +444,24 @@ int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer
                          void *stream);
 
 /*
- * The f64 fitting net with its hidden-layer GEMMs on the tensor cores.  Same
- * inputs, outputs and results as dp_fitting_fwd_f64 / dp_fitting_grad_f64
- * (Sec. II: E_i from D_i, and dE_i/dD_i), to f64 accuracy: every GEMM operand
- * element is split exactly into eleven 5-bit digits scaled by its row's (A)
- * or column's (B) power of two, the digit products run as fp16 MMAs whose
- * fp32 sums are exact integers (at most 1024 of K per partial sum), and those
- * partial sums are combined in f64.  Per output the error is below about
- * K 2^-51 max_k |a_ik| max_k |b_kj| (an f64 dot product: K 2^-53 sum_k
+ * The f64 fitting net with its hidden-layer GEMMs on the tensor cores
+ * (tcgen05).  Same inputs, outputs and results as dp_fitting_fwd_f64 /
+ * dp_fitting_grad_f64 (Sec. II: E_i from D_i, and dE_i/dD_i), to f64
+ * accuracy: every GEMM operand element is split exactly into nine 6-bit
+ * digits scaled by its row's (A) or column's (B) power of two, the 45 digit
+ * products that matter run as fp16 MMAs whose fp32 sums are exact integers
+ * (at most 448 of K per partial sum), and those sums are recombined exactly
+ * before one rounding to f64.  Per output the error is below about
+ * K 2^-50 max_k |a_ik| max_k |b_kj| (an f64 dot product: K 2^-53 sum_k
  * |a_ik b_kj|).  A row or column holding inf or NaN gives NaN outputs.  The
  * paper computes the net in double; this is that computation on hardware
- * whose FP64 rate is ~480 times below its fp16 tensor rate.
+ * whose FP64 rate is ~1000 times below its fp16 tensor rate.
  *   work, work_bytes  device scratch, caller-owned, 256-byte aligned, at least
  *                     dp_fitting_tc_work_bytes(widths, nlayer, nloc) bytes:
- *                     the weights' digit planes (rebuilt on every call) and,
- *                     for the backward, the two [nloc][max hidden width]
- *                     buffers between layers.  Calls sharing a work buffer
- *                     must not overlap on the GPU.
+ *                     the operands' digit planes (the weights' rebuilt on
+ *                     every call), partial results, and the [nloc][max hidden
+ *                     width] buffers between layers.  Calls sharing a work
+ *                     buffer must not overlap on the GPU.
  * Errors as the f64 calls, plus DP_ERR_NULL / DP_ERR_SHAPE for a missing,
  * short or misaligned work buffer.
  */
