@@ -735,7 +735,8 @@ def main():
     ap.add_argument("--fitting", action="store_true",
                     help="with --chain: add the fitting net, so the step yields the model's energy and forces")
     ap.add_argument("--fitting-tc", action="store_true",
-                    help="with --fitting --dtype f64: the fitting net's GEMMs on the tensor cores (exact splitting)")
+                    help="with --fitting and double arrays (f64, df64): the fitting net's f64 GEMMs on the tensor "
+                         "cores (exact splitting)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -743,8 +744,8 @@ def main():
         ap.error("--dtype df64 runs the moment path only")
     if args.fitting and not args.chain:
         ap.error("--fitting extends the --chain step")
-    if args.fitting_tc and (not args.fitting or args.dtype != "f64"):
-        ap.error("--fitting-tc needs --fitting and --dtype f64")
+    if args.fitting_tc and (not args.fitting or args.dtype not in ("f64", "df64")):
+        ap.error("--fitting-tc needs --fitting and double arrays (--dtype f64 or df64)")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
