@@ -381,20 +381,23 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
 //
 // gemm_kernel: one CTA of 128 threads per 128 x 48 output tile and share of K,
 // one CTA per SM (its 9 diagonal accumulators take 432 of the SM's 512 TMEM
-// columns).  The digit planes of A (per chunk of rows, with the row exponents)
-// and B (per call) are made by split_rows_kernel, once per element.  K slices
-// of 16 pass through four shared-memory stages in the tcgen05 K-major layout
-// without swizzle (8-row x 16-byte core matrices), filled by cp.async; one
-// thread issues the 45 digit-product MMAs (M = 128, N = 48, K = 16, fp16 in,
-// fp32 accumulators in TMEM, one per diagonal) of a stage and commits them to
-// the stage's mbarrier, which frees the stage for the slice four ahead.  At
-// the end each warp reads its 32 TMEM lanes (rows), combines the diagonals and
-// writes the share's result as four floats; epilogue_kernel sums the shares in
-// a fixed order, scales by 2^(E+F) and applies the layer's epilogue.  A is always a plain matrix: the
-// forward keeps each layer's input v_l (tanh outputs plus the skip) in a work
-// buffer, the backward writes dE/dv (for the next skip) and dE/dv (1 - t^2)
-// (the next A).  Every wait on an mbarrier is bounded; a wait that gives up
-// makes the tile's outputs NaN.
+// columns).  The digit planes of A (per chunk of rows) and B (per call) are
+// made by split_rows_kernel, once per element, as the shared-memory image of
+// each (tile, 16-deep K slice) block: the tcgen05 K-major layout without
+// swizzle (8-row x 16-byte core matrices).  Lane 0 of warp 0 moves a slice's
+// A and B blocks into one of four stages with two bulk async copies counted in
+// bytes on the stage's "full" mbarrier; lane 0 of warp 1 issues the slice's 45
+// digit-product MMAs (M 128, N 48, K 16, fp16 in, fp32 accumulators in TMEM,
+// one per diagonal) and commits them to the stage's "empty" mbarrier, which
+// the producer waits on before refilling the stage.  A last commit on a
+// barrier used once releases the four warps, which read their TMEM lane
+// quadrant (rows), combine the diagonals and write the share's result as four
+// floats; epilogue_kernel sums the shares in a fixed order, scales by 2^(E+F)
+// and applies the layer's epilogue.  A is always a plain matrix: the forward
+// keeps each layer's input v_l (tanh outputs plus the skip) in a work buffer,
+// the backward writes dE/dv (for the next skip) and dE/dv (1 - t^2) (the next
+// A).  Every wait on an mbarrier is bounded; a wait that gives up makes the
+// tile's outputs NaN.
 namespace tc {
 constexpr int kS = 9;      // digits per operand element
 constexpr int kBits = 6;   // bits per digit
