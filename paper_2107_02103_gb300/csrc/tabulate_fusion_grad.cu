@@ -178,7 +178,7 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 //   dE/dR~_j[k] = (1/N_c) sum_q t_j^q H[k][q]
 //   dE/ds_j     = (1/N_c) sum_k R~_j[k] sum_{q>=1} q t_j^(q-1) H[k][q]
 // One warp per atom.  Rows are staged 32 at a time (one per lane) into a
-// chunk of up to kChunkRows rows and cut into runs; a run that reaches the end
+// chunk of up to chunk_rows() rows and cut into runs; a run that reaches the end
 // of a batch stays open for the next one.  When the chunk is full, the H of
 // its runs are formed G runs at a time: lane = (run p, channel lane c) with
 // C = 32/G channel lanes per run, each lane summing 24 products over the
@@ -195,7 +195,13 @@ __global__ void __launch_bounds__(kGradThreads) grad_kernel(const GradParams<rea
 // finished by a reduce-scatter over its C lanes.  In f32 the per-row form is
 // bound by its scattered coefficient loads, and every run goes through H.
 constexpr int kMomentWarps = 1;
-constexpr int kChunkRows = 128;  // rows staged per chunk
+// Rows staged per chunk and H slots per chunk.  df64 uses smaller chunks: its staging takes twice
+// the bytes of f32's, and a one-warp block with 24 KB of shared memory left ~8 warps per SM, too few
+// to hide the latencies of its long FP32 sequences (measured: 96 rows and 32 runs took the cu85
+// backward from 0.459 to 0.427 ms and the water one from 0.757 to 0.688 ms; f64 keeps 128 rows).
+constexpr int kDf64ChunkRows = 96;  // 64 measured the same to within 2 %
+template <typename real>
+constexpr int chunk_rows() { return is_df64<real> ? kDf64ChunkRows : 128; }
 // df64: every run goes through H, and a row's four k components are evaluated in a loop.  Each
 // df64 FMA is twelve instructions; the per-row path for single-row runs and the unrolled row
 // evaluation made the kernel too large for the instruction cache (ncu: 2.0 cycles per issued
@@ -208,20 +214,20 @@ template <typename real>
 constexpr int min_grad_run() { return is_df64<real> ? kDf64MinGradRun : sizeof(real) == 8 ? 2 : 1; }
 // H slots per chunk (plus one for an open run's H), and the most runs one batch can add
 template <typename real>
-constexpr int chunk_runs() { return min_grad_run<real>() == 2 ? 32 : 64; }
+constexpr int chunk_runs() { return min_grad_run<real>() == 2 || is_df64<real> ? 32 : 64; }
 template <typename real>
 constexpr int batch_runs() { return 32 / min_grad_run<real>() + 1; }
 
 template <typename real>
 struct alignas(16) MomentGradStage {
-  real r[kChunkRows][4];  // R~ rows of the chunk
-  real t[kChunkRows];     // local variable t
+  real r[chunk_rows<real>()][4];  // R~ rows of the chunk
+  real t[chunk_rows<real>()];     // local variable t
   real H[chunk_runs<real>() + 1][25];  // H[run][6*k + q]; rows padded to 25 so that lanes reading different runs hit different banks
   int32_t qoff[64];  // queue of single-row runs: interval block offset and row (t and R~ are read again)
   int32_t qrow[64];
-  int32_t off[kChunkRows];      // interval block offset of each staged row
-  int32_t row[kChunkRows];      // row index, bit 30 set when s was clamped
-  int32_t slot[kChunkRows];     // H slot of the row's run, -1 for queued rows
+  int32_t off[chunk_rows<real>()];   // interval block offset of each staged row
+  int32_t row[chunk_rows<real>()];   // row index, bit 30 set when s was clamped
+  int32_t slot[chunk_rows<real>()];  // H slot of the row's run, -1 for queued rows
   int32_t run_off[chunk_runs<real>() + 1];  // interval block offset of each H slot
   int32_t nvb[DP_MAX_TYPES];
 };
@@ -597,7 +603,7 @@ __global__ void __launch_bounds__(kMomentWarps * 32) grad_moments_kernel(const G
     }
     nrows += cnt;
     __syncwarp();
-    if (nrows + 32 > kChunkRows || nrun + batch_runs<real>() > chunk_runs<real>() || !more) {  // chunk full, or the atom's last rows
+    if (nrows + 32 > chunk_rows<real>() || nrun + batch_runs<real>() > chunk_runs<real>() || !more) {  // chunk full, or the atom's last rows
       form_H_runs(st, tab, dts, M1, nrun, lane);
       __syncwarp();
       for (int j = lane; j < nrows; j += 32) {
