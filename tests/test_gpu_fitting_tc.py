@@ -145,3 +145,24 @@ def test_tc_forward_tanh_against_numpy():
     assert np.isnan(t[~ok]).all()
     tiny = np.abs(z) < 1e-20
     assert np.array_equal(t[tiny], z[tiny])
+
+
+def test_tc_many_atoms_in_row_chunks():
+    """More atoms of one type than one chunk of digit planes holds (16,384), a second type after
+    them, a width that is no multiple of 48: against the FP64-pipe path (1e-13) and the oracle on a
+    sample of atoms."""
+    dpc = lib()
+    widths, params = W.fitting_net(51, 40, (56, 56), 2)
+    ts = np.array([0, 20000, 20300], dtype=np.int64)
+    D = W.normal(52, (20300, 40), 0.0, 0.3)
+    E, act, dD = _tc(dpc, params, widths, ts, D)
+    p = _cuda(params)
+    E2, act2 = dpc.dp_fitting_fwd(p, widths, ts, _cuda(D))
+    dD2 = dpc.dp_fitting_grad(p, widths, ts, act2)
+    torch.cuda.synchronize()
+    assert rel(E, E2.cpu().numpy()) <= 1e-13
+    assert rel(dD, dD2.cpu().numpy()) <= 1e-13
+    pick = np.r_[0:5, 16380:16390, 19995:20005, 20295:20300]
+    at = np.repeat(np.arange(2), [20000, 300]).astype(np.int32)
+    Eo, dDo = oracle.default().fitting(params, widths, D[pick], at[pick])
+    assert rel(E[pick], Eo) <= F64 and rel(dD[pick], dDo) <= F64
