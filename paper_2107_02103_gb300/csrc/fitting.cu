@@ -549,8 +549,10 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
          (1ull << 46);
 }
 // instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A and B f16 (0), both K-major, N >> 3 at
-// bit 17, M >> 4 at bit 24
-constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(kTN >> 3) << 17) | ((uint32_t)(kTM >> 4) << 24);
+// bit 17 (set per MMA), M >> 4 at bit 24
+constexpr uint32_t kIdescNoN = (1u << 4) | ((uint32_t)(kTM >> 4) << 24);  // N >> 3 goes in at bit 17
+constexpr int kMaxPlanesPerMma = 256 / kTN;  // N <= 256 for M = 128
+static_assert(kTN % 16 == 0 && kMaxPlanesPerMma >= 1, "MMA N: multiples of 16 up to 256");
 
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   uint32_t done = 0;
@@ -624,17 +626,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
       if (!ok) break;
       asm volatile("tcgen05.fence::after_thread_sync;");
       const uint64_t a0 = smem_desc(sbase + st * kStageBytes), b0 = smem_desc(sbase + st * kStageBytes + kS * kPlaneA);
+      // Digit s of A against digits t = 0 .. kS-1-s of B in one MMA: B's planes lie back to back in
+      // the stage (48 rows each, one row stride), so together they are one operand of 48 (kS - s)
+      // rows, and with the accumulator address moved by s diagonals the block of plane t lands on
+      // diagonal s + t.  N is at most 256, so up to 5 planes (240 columns) per MMA: 13 MMAs per
+      // slice instead of 45, each reading its A tile once for up to 240 columns.
 #pragma unroll
-      for (int t = 0; t < kS; ++t) {
-        const uint64_t bd = b0 + (uint64_t)((t * kPlaneB) >> 4);  // start-address field, in 16-byte units
+      for (int s = 0; s < kS; ++s) {
+        const uint64_t ad = a0 + (uint64_t)((s * kPlaneA) >> 4);  // start-address field, in 16-byte units
 #pragma unroll
-        for (int s = 0; s + t < kS; ++s) {  // digits s + 1 and t + 1: diagonal s + t + 2 <= kS + 1
-          const uint64_t ad = a0 + (uint64_t)((s * kPlaneA) >> 4);
-          const uint32_t acc = (i > 0 || t > 0) ? 1u : 0u;  // a diagonal's first product overwrites
+        for (int t0 = 0; t0 < kS - s; t0 += kMaxPlanesPerMma) {
+          const int np = min(kMaxPlanesPerMma, kS - s - t0);
+          const uint64_t bd = b0 + (uint64_t)((t0 * kPlaneB) >> 4);
+          const uint32_t idesc = kIdescNoN | ((uint32_t)((np * kTN) >> 3) << 17);
+          const uint32_t acc = (i > 0 || s > 0) ? 1u : 0u;  // digit 1 of A writes every diagonal first
           asm volatile(
               "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-              " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem + (uint32_t)((s + t) * kTN)),
-              "l"(ad), "l"(bd), "r"(kIdesc), "r"(acc));
+              " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem + (uint32_t)((s + t0) * kTN)),
+              "l"(ad), "l"(bd), "r"(idesc), "r"(acc));
         }
       }
       asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
