@@ -720,10 +720,9 @@ __device__ __forceinline__ double widen_pow2(float f, int e) {
 
 template <bool kFwd>
 __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int ksplit) {
-  const int64_t total = P.n * P.N;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t rc = e / P.N;
-    const int nn = (int)(e - rc * P.N);
+  // rows over the grid, columns over the block (no 64-bit division per element)
+  for (int64_t rc = blockIdx.x; rc < P.n; rc += gridDim.x)
+  for (int nn = threadIdx.x; nn < P.N; nn += blockDim.x) {
     const int64_t row = P.r0 + rc;
     // the shares' four floats each, added into a three-float sum by exact two-sums on the FP32 pipe
     // (only the last component rounds, ~2^-72 below the sum), then one conversion to f64 and the
@@ -775,10 +774,9 @@ __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int kspli
 __global__ void __launch_bounds__(256) last_dz_kernel(int64_t r0, int64_t n, int K, const double *__restrict__ g,
                                                       const double *__restrict__ wo, const double *__restrict__ T,
                                                       int64_t ldT, double *__restrict__ Z, int64_t ldz) {
-  const int64_t total = n * K;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t row = r0 + e / K;
-    const int k = (int)(e - (e / K) * K);
+  for (int64_t rr = blockIdx.x; rr < n; rr += gridDim.x)
+  for (int k = threadIdx.x; k < K; k += blockDim.x) {
+    const int64_t row = r0 + rr;
     const double t = T[row * ldT + k];
     Z[row * ldz + k] = (g ? g[row] : 1.0) * wo[k] * fma(-t, t, 1.0);
   }
@@ -916,8 +914,7 @@ int gemm(TcGemm G, const Layer &L, unsigned char *work, const WorkMap &m, cudaSt
     const dim3 grid((unsigned)(L.Np / kTN), (unsigned)(C.Mp / kTM), (unsigned)ksplit);
     gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(C);
     if ((rc = launch_status(who))) return rc;
-    const int64_t total = C.n * C.N;
-    epilogue_kernel<kFwd><<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(C, ksplit);
+    epilogue_kernel<kFwd><<<(unsigned)std::min<int64_t>(C.n, 152 * 32), 256, 0, st>>>(C, ksplit);
     if ((rc = launch_status(who))) return rc;
   }
   return DP_OK;
@@ -1019,9 +1016,9 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
     const double *wo = pt + s.woff[nlayer];
     {  // dz of the last hidden layer
       const int K = s.w[nlayer - 1];
-      const int64_t total = n * K;
-      const unsigned blocks = (unsigned)std::min<int64_t>((total + 255) / 256, 152 * 8);
-      last_dz_kernel<<<blocks, 256, 0, st>>>(s.start[t], n, K, g, wo, act + s.aoff[nlayer - 1], s.H, Z[0], s.maxh);
+      last_dz_kernel<<<(unsigned)std::min<int64_t>(n, 152 * 32), 256, 0, st>>>(s.start[t], n, K, g, wo,
+                                                                             act + s.aoff[nlayer - 1], s.H, Z[0],
+                                                                             s.maxh);
       if ((rc = launch_status(who))) return rc;
     }
     const double *S = nullptr;  // dE/dv of the layer being walked; NULL: g wo (the last hidden layer)
