@@ -417,6 +417,9 @@ def run_native(args, rank, world, local_rank):
     k_ms = {n: [e[j].elapsed_time(e[j + 1]) for e in evs] for j, n in enumerate(names)}
     total_s, evals_all = reduce_over_ranks(sum(step_ms) / 1e3, float(w.evals), world, dev)
 
+    # ---- the same step captured once as a CUDA graph (the chain's many launches in one)
+    graph = measure_graph(run_step, flush, dev, args.steps) if (args.chain and not args.no_graph) else None
+
     # ---- end to end through the public API: pinned host inputs -> device -> path -> host results
     e2e = None if args.no_e2e else measure_e2e(args, host, d, outs, run_step, stream, dev, world, barrier,
                                                 evals_all)
@@ -427,9 +430,42 @@ def run_native(args, rank, world, local_rank):
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
     nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
     out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall)
+    if graph is not None:
+        graph["evals_per_s"] = w.evals / (graph["ms_per_step"] * 1e-3)
+        out["graph"] = graph
     if world == 1 and not args.no_variants and not args.chain and args.dtype == "f64" and args.algo == "moments":
         out["variants"] = measure_variants(args, w, dpc, info, sel, d, outs, flush, stream, dev, fmas)
     return out
+
+
+def measure_graph(run_step, flush, dev, nsteps):
+    """The step captured once as a CUDA graph and replayed: its launches (a few dozen in the chain with
+    the fitting net) leave the host as one.  The library's calls allocate nothing and never wait, so
+    they capture as they are; one eager step on the capture stream first does their one-time setup.
+    Inputs resident, L2 flushed between replays (outside the events), CUDA events around each replay."""
+    import torch
+    side = torch.cuda.Stream(device=dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    with torch.cuda.stream(side):
+        run_step()
+    torch.cuda.current_stream(dev).wait_stream(side)
+    torch.cuda.synchronize(dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        run_step()
+    g.replay()
+    torch.cuda.synchronize(dev)
+    st = torch.cuda.current_stream(dev)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(nsteps)]
+    for e0, e1 in evs:
+        flush.zero_()
+        e0.record(st)
+        g.replay()
+        e1.record(st)
+    torch.cuda.synchronize(dev)
+    ms = sum(a.elapsed_time(b) for a, b in evs) / nsteps
+    return {"ms_per_step": round(ms, 4), "replays": nsteps,
+            "note": "the same step captured once as a CUDA graph and replayed (per-kernel times above: eager)"}
 
 
 def measure_variants(args, w, dpc, info, sel, d, ref_outs, flush, stream, dev, fmas):
@@ -728,6 +764,7 @@ def main():
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true", help="with --chain: skip the CUDA-graph replay timing")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the per-row and df64 timings added to the default f64 line")
     ap.add_argument("--chain", action="store_true",
