@@ -274,6 +274,15 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     import workloads as W
     fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
     grad = dpc.dp_tabulate_fusion_grad_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_grad
+    if args.algo == "tc":  # the per-interval contraction on the tensor cores; its scratch stays resident
+        tcw = torch.empty((dpc.dp_tabulate_tc_work_bytes(info, w.nloc, w.nnei, w.ntypes, w.M1),), dtype=torch.uint8,
+                          device=dev)
+
+        def fwd(*a, out=None):
+            return dpc.dp_tabulate_fusion_fwd_tc_f64(*a, out=out, work=tcw)
+
+        def grad(*a, out=None):
+            return dpc.dp_tabulate_fusion_grad_tc_f64(*a, out=out, work=tcw)
     arith = dpc.DF64 if args.dtype == "df64" else None  # the table picks the fusion kernels' arithmetic
     T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
     D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
@@ -426,7 +435,7 @@ def run_native(args, rank, world, local_rank):
     if rank != 0:
         return None
     fmas = None
-    if args.algo == "moments":
+    if args.algo in ("moments", "tc"):
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
     nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
     out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall)
@@ -759,7 +768,7 @@ def main():
     ap.add_argument("--seed", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
-    ap.add_argument("--algo", choices=["direct", "moments"], default="moments",
+    ap.add_argument("--algo", choices=["direct", "moments", "tc"], default="moments",
                     help="direct: per-neighbour evaluation (the paper's fused kernel); moments: interval moments")
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")
@@ -779,6 +788,8 @@ def main():
         ap.error("--warmup must be >= 3")
     if args.dtype == "df64" and args.algo != "moments":
         ap.error("--dtype df64 runs the moment path only")
+    if args.algo == "tc" and args.dtype != "f64":
+        ap.error("--algo tc is the f64 path (exact digit splitting on the tensor cores)")
     if args.fitting and not args.chain:
         ap.error("--fitting extends the --chain step")
     if args.fitting_tc and (not args.fitting or args.dtype not in ("f64", "df64")):

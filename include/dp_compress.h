@@ -235,6 +235,50 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
                                         float *dRt, void *stream);
 
 /*
+ * The f64 forward and backward with the per-interval contraction on the
+ * tensor cores (tcgen05).  Same arguments, results, limits and errors as
+ * dp_tabulate_fusion_fwd_f64 / dp_tabulate_fusion_grad_f64, plus a work
+ * buffer.  With u = t / Delta_l in [0, 1] (Delta_l = stride0 on the fine
+ * grid, stride1 on the coarse one) and c'_q = c_q Delta_l^q, the interval
+ * moments of the rows of atom i,
+ *   W[k][(b, l, q)] = sum_{valid rows j of segment b in interval l} R~[i][j][k] u_j^q,
+ * turn the forward into a GEMM over K = (neighbour type b, interval l, q):
+ *   T[i][k][m] = (1/nnei) sum_{(b, l, q)} W[k][(b, l, q)] c'_q(pair (atype[i], b), l, m),
+ * and the backward into the transposed one, dW[k][(b, l, q)] =
+ * (1/nnei) sum_m dT[i][k][m] c'_q(..., l, m), from which every valid row
+ * takes dRt[i][j][k] = sum_q dW[k][(b, l, q)] u_j^q and ds[i][j] =
+ * sum_k R~[i][j][k] sum_{q>=1} q dW[k][(b, l, q)] u_j^(q-1) / Delta_l (0
+ * where s was clamped).  Both GEMMs run exactly as in dp_fitting_*_tc_f64:
+ * nine 6-bit digits per element, scaled by the row's or column's power of
+ * two, fp16 MMAs with exact fp32 sums (at most 448 of K per partial sum),
+ * one rounding to f64; per output the error is below about
+ * K 2^-50 max|row| max|column| (K: the used intervals x 8, or M1).  Only
+ * the intervals some atom of a 12-atom tile uses enter its GEMM.  Rows need
+ * not be sorted, though sorted rows (one run per interval) do the least
+ * FP64 work.  NaN s gives NaN in that atom's T (forward) and in that row's
+ * ds and dRt (backward); inf or NaN in dT gives NaN in the atom's rows.
+ *   work, work_bytes  device scratch, caller-owned, 256-byte aligned, at
+ *                     least dp_tabulate_tc_work_bytes(info, nloc, nnei,
+ *                     ntypes, M1) bytes (one size for both directions): the
+ *                     scaled coefficients and their digit planes (rebuilt
+ *                     on every call), the moments or their gradients per
+ *                     (atom, interval), flags of the used intervals, and
+ *                     partial results, for chunks of at most 4104 atoms.
+ *                     Calls sharing a work buffer must not overlap on the GPU.
+ * Extra errors: DP_ERR_NULL / DP_ERR_SHAPE for a missing, short or
+ * misaligned work buffer.
+ */
+size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nnei, int ntypes,
+                                 int M1); /* 0 on bad sizes or table info */
+int dp_tabulate_fusion_fwd_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+                                  const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                  const int32_t *sel, int M1, double *T, void *work, size_t work_bytes, void *stream);
+int dp_tabulate_fusion_grad_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                   const int32_t *sel, int M1, const double *dT, double *ds, double *dRt, void *work,
+                                   size_t work_bytes, void *stream);
+
+/*
  * Descriptor (Sec. II): with S_i = T_i^T (M1 x 4) and S_i^< its first M2
  * rows, D_i = S_i (S_i^<)^T, i.e. D[i][m][n] = sum_k T[i][k][m] * T[i][k][n].
  *   T [nloc][4][M1] input,  D [nloc][M1][M2] output.

@@ -93,6 +93,11 @@ _SIGS = {
                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_moments_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
+    "dp_tabulate_tc_work_bytes": ([_INFO, _I64, ctypes.c_int, ctypes.c_int, ctypes.c_int], ctypes.c_size_t),
+    "dp_tabulate_fusion_fwd_tc_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                       ctypes.c_int, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_tc_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                        ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
     "dp_env_mat_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_env_mat_f32": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_f64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
@@ -326,6 +331,66 @@ def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
     fn = getattr(_lib, f"{name}_{_suffix(arith)}")
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(dT), _ptr(ds), _ptr(dRt), _stream(s)))
+    return ds, dRt
+
+
+def dp_tabulate_tc_work_bytes(info: dp_table_info, nloc, nnei, ntypes, M1) -> int:
+    """Bytes of device scratch dp_tabulate_fusion_{fwd,grad}_tc_f64 need (one size for both)."""
+    n = int(_lib.dp_tabulate_tc_work_bytes(ctypes.byref(info), int(nloc), int(nnei), int(ntypes), int(M1)))
+    if n == 0:
+        raise ValueError(_lib.dp_last_error().decode())
+    return n
+
+
+def _tab_tc_work(work, info, nloc, nnei, ntypes, M1, device):
+    need = dp_tabulate_tc_work_bytes(info, nloc, nnei, ntypes, M1)
+    if work is None:
+        return torch.empty((need,), dtype=torch.uint8, device=device)
+    if not work.is_cuda or work.dtype != torch.uint8 or not work.is_contiguous() or work.numel() < need:
+        raise ValueError(f"work must be a contiguous CUDA uint8 tensor of at least {need} bytes")
+    return work
+
+
+def _tc_inputs(table, s, Rt, nvalid, atype, sel):
+    r = _fusion_inputs(table, s, Rt, nvalid, atype, sel)
+    if r[-1] != torch.float64:
+        raise TypeError("the tensor-core calls take an f64 table and f64 arrays")
+    return r
+
+
+def dp_tabulate_fusion_fwd_tc_f64(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None, work=None):
+    """T of dp_tabulate_fusion_fwd in f64 with the per-interval contraction on the tensor cores (interval
+    moments times the scaled table, an exact digit-split GEMM); work: a uint8 CUDA tensor of
+    dp_tabulate_tc_work_bytes(...) bytes, or None to allocate one."""
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, _ = _tc_inputs(table, s, Rt, nvalid, atype, sel)
+    shape = (nloc, 4, M1)
+    T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
+    if nloc == 0:
+        return T
+    work = _tab_tc_work(work, info, nloc, nnei, ntypes, M1, s.device)
+    _check(_lib.dp_tabulate_fusion_fwd_tc_f64(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid),
+                                              _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(T), _ptr(work),
+                                              work.numel(), _stream(s)))
+    return T
+
+
+def dp_tabulate_fusion_grad_tc_f64(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None, work=None):
+    """(ds, dRt) of dp_tabulate_fusion_grad in f64 with the per-interval contraction on the tensor cores;
+    work as dp_tabulate_fusion_fwd_tc_f64."""
+    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, _ = _tc_inputs(table, s, Rt, nvalid, atype, sel)
+    dT = _dev(dT, "dT", dtype, (nloc, 4, M1))
+    if out is None:
+        ds = torch.empty((nloc, nnei), dtype=dtype, device=s.device)
+        dRt = torch.empty((nloc, nnei, 4), dtype=dtype, device=s.device)
+    else:
+        ds = _dev(out[0], "ds", dtype, (nloc, nnei))
+        dRt = _dev(out[1], "dRt", dtype, (nloc, nnei, 4))
+    if nloc == 0:
+        return ds, dRt
+    work = _tab_tc_work(work, info, nloc, nnei, ntypes, M1, s.device)
+    _check(_lib.dp_tabulate_fusion_grad_tc_f64(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid),
+                                               _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(dT), _ptr(ds),
+                                               _ptr(dRt), _ptr(work), work.numel(), _stream(s)))
     return ds, dRt
 
 

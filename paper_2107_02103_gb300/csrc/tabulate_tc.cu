@@ -1,0 +1,724 @@
+// Tabulated embedding + contraction (Sec. II, kernel fusion) in f64 with the
+// per-interval contraction on the tcgen05 tensor cores.
+//
+// The fused forward is a sum over the valid neighbour rows j of atom i,
+//   T_i[k][m] = (1/N_c) sum_j R~_j[k] g_m^l(t_j),  g_m^l(t) = sum_q c_q^{l,m} t^q (q = 0..5),
+// l the row's interval and t its offset from the interval's left node.  With
+// u = t / Delta_l (Delta_l the interval's step, so 0 <= u <= 1) and the scaled
+// coefficients c'_q^{l,m} = c_q^{l,m} Delta_l^q, it regroups per interval into
+// moments of the rows that fall in it,
+//   W_i[k][(l, q)] = sum_{j in l} R~_j[k] u_j^q,     T_i[k][m] = (1/N_c) sum_{(l, q)} W_i[k][(l, q)] c'_q^{l,m},
+// a GEMM whose K index is (neighbour type, interval, power): the same sum as
+// the per-row evaluation, associated per interval.  The backward is the
+// transposed GEMM,
+//   dW_i[k][(l, q)] = (1/N_c) sum_m dT_i[k][m] c'_q^{l,m},
+//   dE/dR~_j[k] = sum_q dW_i[k][(l, q)] u_j^q,
+//   dE/ds_j     = sum_k R~_j[k] sum_{q >= 1} q dW_i[k][(l, q)] u_j^(q-1) / Delta_l   (0 where s_j was clamped).
+// The FP64 pipe keeps the per-row work (24 FMAs per row for W, 40 for the
+// derivatives); the per-interval work (24 M1 FMAs per interval and atom in
+// each direction), which is most of it, runs as exact digit-split GEMMs on
+// the tensor cores (tc_gemm.cuh), at f64 accuracy.
+//
+// K layout, per centre type: key = beta nint + l (neighbour type beta, interval
+// l), and column 8 key + q of the GEMM holds power q (q = 6, 7 are zero), so a
+// 16-deep K slice is two intervals.  An atom touches only the intervals its
+// rows fall in: the W values are stored per run of rows (one slot per
+// interval an atom uses, found through a per-atom map), and the GEMMs skip the
+// slices (forward) or output tiles (backward) that no atom of a tile uses.
+//
+// Per chunk of at most kChunkAtoms atoms and per centre type alpha:
+//   forward:  runs_kernel<true> (map, W, column exponents, slice flags),
+//             split_mom_kernel (W -> B digit planes, used slices only),
+//             gemm_kernel (A = C'_alpha^T: channels x K, B = W^T: K x (atom, k)),
+//             fwd_epilogue_kernel (shares -> T for the atoms of type alpha);
+//   backward: runs_kernel<false> (map, tile flags), split of dT (B), gemm_kernel
+//             (A = C'_alpha: K x channels, B = dT^T) scattering each used
+//             (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
+// C'_alpha and its digit planes are made per call from the table.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "dp_common.cuh"
+#include "tc_gemm.cuh"
+
+namespace dpc {
+namespace {
+namespace tt {
+using namespace tc;
+
+constexpr int kQ = 8;                 // K entries per interval: u^0 .. u^5 and two zeros
+constexpr int kCols = 4;              // GEMM columns per atom: k = 0 .. 3
+constexpr int kTileAtoms = kTN / kCols;  // 12 atoms per 48-column tile
+constexpr int64_t kChunkAtoms = 4104;    // a multiple of 12 (16,416 columns)
+constexpr int kShareSlices = 14;         // used K slices per forward share
+constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' results per chunk
+static_assert(kShareSlices <= kMaxShareSlices, "share within the exactness bound");
+static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
+
+// Sizes shared by the kernels and the work-buffer layout.
+struct Shape {
+  int ntypes, nint, nkeys, M1, cap;
+  int Kp;    // round_up(8 nkeys, 16): K of the forward GEMM, rows of the backward A
+  int nsl;   // Kp / 16
+  int Mpf;   // round_up(M1, 128): rows of the forward A
+  int Kpm;   // round_up(M1, 16): K of the backward GEMM
+  int Mpb;   // round_up(Kp, 128): rows of the backward A
+  int64_t chunk, Np, ntiles;  // atoms per chunk, its columns round_up(4 chunk, 48), Np / 48
+  int zmax;                   // forward shares per tile at most
+};
+
+struct Layout {
+  size_t cp, afwd, efwd, abwd, ebwd, map, occ, fexp, bplanes, w, part, total;
+};
+
+Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1) {
+  Shape s{};
+  s.ntypes = ntypes;
+  s.nint = g.nint;
+  s.nkeys = ntypes * g.nint;
+  s.M1 = M1;
+  s.cap = std::min(nnei, s.nkeys);
+  s.Kp = (int)round_up((int64_t)s.nkeys * kQ, kTK);
+  s.nsl = s.Kp / kTK;
+  s.Mpf = (int)round_up(M1, kTM);
+  s.Kpm = (int)round_up(M1, kTK);
+  s.Mpb = (int)round_up(s.Kp, kTM);
+  s.zmax = (s.nsl + kShareSlices - 1) / kShareSlices;
+  int64_t chunk = std::min<int64_t>(round_up(std::max<int64_t>(nloc, 1), kTileAtoms), kChunkAtoms);
+  while (chunk > kTileAtoms &&
+         (size_t)s.zmax * s.Mpf * round_up(kCols * chunk, kTN) * sizeof(float4) > kPartBudget)
+    chunk = round_up(chunk / 2, kTileAtoms);
+  s.chunk = chunk;
+  s.Np = round_up(kCols * chunk, kTN);
+  s.ntiles = s.Np / kTN;
+  return s;
+}
+
+Layout make_layout(const Shape &s) {
+  Layout L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off += (size_t)round_up((int64_t)bytes, 256);
+    return at;
+  };
+  const size_t nt = (size_t)s.ntypes;
+  L.cp = take(nt * s.Kp * s.M1 * sizeof(double));
+  L.afwd = take(nt * kS * (size_t)s.Mpf * s.Kp * 2);
+  L.efwd = take(nt * s.Mpf * sizeof(int));
+  L.abwd = take(nt * kS * (size_t)s.Mpb * s.Kpm * 2);
+  L.ebwd = take(nt * s.Mpb * sizeof(int));
+  L.map = take((size_t)s.chunk * s.nkeys * sizeof(int));
+  L.occ = take(nt * s.ntiles * std::max(s.nsl, s.Mpb / kTM));
+  L.fexp = take((size_t)s.Np * sizeof(int));
+  L.bplanes = take((size_t)s.ntiles * std::max(s.nsl, s.Kpm / kTK) * kS * kPlaneB);
+  L.w = take((size_t)s.chunk * s.cap * 24 * sizeof(float4));  // backward float4 slots; forward doubles fit
+  L.part = take((size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
+  L.total = off;
+  return L;
+}
+
+// C'[alpha][8 key + q][m] = c_q Delta_l^q (key = beta nint + l; q >= 6 and rows past the keys: 0).
+// The interval's block of the table is pair-planar [3][M1][2] holding (a, b, c, d, e, f), the
+// coefficients of t^5 .. t^0.
+__global__ void __launch_bounds__(256) coef_kernel(const double *__restrict__ table, TableGeom g, int ntypes, int M1,
+                                                   int Kp, double *__restrict__ Cp) {
+  const int64_t total = (int64_t)ntypes * Kp * M1;
+  for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total; x += (int64_t)gridDim.x * blockDim.x) {
+    const int m = (int)(x % M1);
+    const int64_t rest = x / M1;
+    const int r = (int)(rest % Kp), alpha = (int)(rest / Kp);
+    const int key = r >> 3, q = r & 7;
+    double v = 0.0;
+    if (q < 6 && key < ntypes * g.nint) {
+      const int beta = key / g.nint, l = key - beta * g.nint;
+      const double *blk = table + ((size_t)(alpha * ntypes + beta) * g.nint + l) * M1 * 6;
+      const int j = 5 - q;  // position of t^q's coefficient in (a .. f)
+      const double c = blk[(size_t)(j >> 1) * 2 * M1 + 2 * m + (j & 1)];
+      const double delta = l < g.n0 ? g.stride0 : g.stride1;
+      double p = 1.0;
+      for (int e = 0; e < q; ++e) p *= delta;
+      v = c * p;
+    }
+    Cp[x] = v;
+  }
+}
+
+struct RunsParams {
+  const double *s, *Rt;
+  const int32_t *nvalid, *atype;
+  TableGeom g;
+  int64_t atom0, natoms, ntiles;
+  int nnei, ntypes, nkeys, cap;
+  int sel[DP_MAX_TYPES];
+  int *map;            // [natoms][nkeys]: run slot of the key, or -1
+  double *W;           // forward: [natoms][cap][24] moments W[k][q] at 6 k + q
+  int *fexp;           // forward: [Np] exponents of the columns 4 a + k
+  unsigned char *occ;  // [ntypes][ntiles][occ_cols]
+  int occ_cols;        // forward: K slices; backward: 128-row tiles of the backward A
+  int keys_per_unit;   // keys per flag: 2 (a 16-deep slice) or 16 (128 rows of 8 per key)
+};
+
+struct alignas(16) RunsStage {
+  double r[32][4];
+  double tp[32][6];
+  int key[32];
+  int nvb[DP_MAX_TYPES];
+};
+
+// Valid rows per type segment of atom i (clamped into [0, sel]) into nvb; returns their total.
+__device__ __forceinline__ int valid_rows(const int32_t *nvalid, const int *sel, int ntypes, int64_t i, int lane,
+                                          int *nvb) {
+  int sl = 0;
+#pragma unroll
+  for (int q = 0; q < DP_MAX_TYPES; ++q)
+    if (lane == q) sl = sel[q];
+  int x = 0;
+  if (lane < ntypes) x = clampi(nvalid ? __ldg(nvalid + i * ntypes + lane) : sl, 0, sl);
+  if (lane < DP_MAX_TYPES) nvb[lane] = x;
+  __syncwarp();
+  int nv = 0;
+#pragma unroll
+  for (int q = 0; q < DP_MAX_TYPES; ++q) nv += nvb[q];
+  return nv;
+}
+
+// Row index of valid row v (type segments in order, the valid rows of each first) and its segment.
+__device__ __forceinline__ int valid_row(int v, const int *nvb, const int *sel, int ntypes, int &b) {
+  int cum = 0, lim = nvb[0], off = 0;
+  b = 0;
+#pragma unroll
+  for (int q = 1; q < DP_MAX_TYPES; ++q)
+    if (q < ntypes && v >= lim) {
+      b = q;
+      cum = lim;
+      lim += nvb[q];
+      off += sel[q - 1];
+    }
+  return off + (v - cum);
+}
+
+// One warp per atom: the runs of rows sharing an interval (consecutive rows with one key; rows
+// sorted by distance give one run per interval, and a key met again adds to its slot), each
+// interval's slot in the map and its flag for the atom's tile; forward also its moments W and
+// the atom's four column exponents.
+template <bool kMom>
+__global__ void __launch_bounds__(32) runs_kernel(const RunsParams P) {
+  __shared__ RunsStage st;
+  const int lane = threadIdx.x;
+  const int64_t a = blockIdx.x;
+  const int64_t i = P.atom0 + a;
+  int *map = P.map + a * P.nkeys;
+  for (int k = lane; k < P.nkeys; k += 32) map[k] = -1;
+  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the map reset)
+  const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
+  unsigned char *occ = P.occ + ((size_t)alpha * P.ntiles + (size_t)(a / kTileAtoms)) * P.occ_cols;
+  double *Wa = kMom ? P.W + (size_t)a * P.cap * 24 : nullptr;
+  int nslot = 0;
+  int cur = -1;       // key of the open run (uniform)
+  double wv = 0.0;    // its moment W[k][q] on lane 6 k + q < 24
+  auto flush = [&]() {  // uniform
+    int slot = lane == 0 ? map[cur] : 0;
+    slot = __shfl_sync(0xffffffffu, slot, 0);
+    const bool fresh = slot < 0;
+    if (fresh) {
+      slot = nslot++;
+      if (lane == 0) {
+        map[cur] = slot;
+        occ[cur / P.keys_per_unit] = 1;
+      }
+    }
+    if (kMom && lane < 24) {
+      double *w = Wa + (size_t)slot * 24 + lane;
+      *w = fresh ? wv : *w + wv;
+    }
+    __syncwarp();
+  };
+  const double *srow = P.s + i * P.nnei;
+  const double *Rrow = P.Rt + i * P.nnei * 4;
+  for (int base = 0; base < nv; base += 32) {
+    const int v = base + lane;
+    if (v < nv) {
+      int b;
+      const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
+      double t;
+      bool clamped;
+      const int l = locate(P.g, __ldg(srow + row), t, clamped);
+      st.key[lane] = b * P.g.nint + l;
+      if constexpr (kMom) {
+        const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
+        st.r[lane][0] = rr.x;
+        st.r[lane][1] = rr.y;
+        st.r[lane][2] = rr.z;
+        st.r[lane][3] = rr.w;
+        const double u = t * (l < P.g.n0 ? P.g.inv0 : P.g.inv1);
+        const double u2 = u * u, u3 = u2 * u;
+        st.tp[lane][0] = 1.0;
+        st.tp[lane][1] = u;
+        st.tp[lane][2] = u2;
+        st.tp[lane][3] = u3;
+        st.tp[lane][4] = u2 * u2;
+        st.tp[lane][5] = u3 * u2;
+      }
+    }
+    __syncwarp();
+    const int cnt = min(32, nv - base);
+    const int mykey = lane < cnt ? st.key[lane] : -1;
+    const int prev = __shfl_up_sync(0xffffffffu, mykey, 1);
+    unsigned starts = __ballot_sync(0xffffffffu, lane < cnt && (lane == 0 || mykey != prev));
+    while (starts) {  // uniform, run by run
+      const int u0 = __ffs(starts) - 1;
+      starts &= starts - 1;
+      const int e = starts ? __ffs(starts) - 1 : cnt;
+      const int key = __shfl_sync(0xffffffffu, mykey, u0);
+      if (key != cur) {
+        if (cur >= 0) flush();
+        cur = key;
+        wv = 0.0;
+      }
+      if (kMom && lane < 24) {
+        const int k = lane / 6, q = lane - 6 * (lane / 6);
+        for (int j = u0; j < e; ++j) wv = fma(st.r[j][k], st.tp[j][q], wv);
+      }
+    }
+    __syncwarp();
+  }
+  if (cur >= 0) flush();
+  if constexpr (kMom) {
+    // column exponents: max over the atom's slots of |W[k][q]|, per k
+    int eb = 0;
+    if (lane < 24)
+      for (int sl = 0; sl < nslot; ++sl) eb = max(eb, exp_bits(Wa[(size_t)sl * 24 + lane]));
+    int m = eb;
+#pragma unroll
+    for (int q = 1; q < 6; ++q) m = max(m, __shfl_sync(0xffffffffu, eb, min(lane + q, 31)));
+    if (lane < 24 && lane % 6 == 0) P.fexp[kCols * a + lane / 6] = exp_of_max(m);
+  }
+}
+
+// The forward's B operand: B[8 key + q][4 a + k] = W_a[k][(key, q)] as digit planes with the column
+// exponents, in split_rows_kernel's block layout (RT = 48), for the slices some atom of the tile
+// uses (any centre type); the other blocks are never read.  One warp per (8 columns, 64 of K).
+__global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict__ W, const int *__restrict__ map,
+                                                        const int *__restrict__ fexp,
+                                                        const unsigned char *__restrict__ occ, int ntypes,
+                                                        int64_t ntiles, int64_t natoms, int nkeys, int cap,
+                                                        int64_t rows_p, int Kp, unsigned char *__restrict__ planes) {
+  const int lane = threadIdx.x & 31, ri8 = lane >> 2, kp = lane & 3;
+  const int kchunks = (Kp + kSplitK - 1) / kSplitK;
+  const int nsl = Kp / kTK;
+  const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int64_t g8 = w / kchunks;
+  if (g8 * 8 >= rows_p) return;  // warp-uniform
+  const int kc = (int)(w - g8 * kchunks);
+  const int64_t r = g8 * 8 + ri8;  // column 4 a + k of the GEMM
+  const int64_t a = r >> 2;
+  const int k = (int)(r & 3);
+  const int64_t tile = r / kTN;   // the same for the warp's 8 columns
+  const int E = fexp[r];
+  constexpr size_t plane = (size_t)kTN * kTK * 2, block = kS * plane;
+  const int ri = (int)(r % kTN);
+  unsigned char *rowbase = planes + (size_t)tile * nsl * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
+  const int q0 = 2 * kp;  // this lane's two powers
+  for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
+    const int sl = k0 / kTK;
+    bool used = false;
+    for (int t = 0; t < ntypes; ++t) used |= occ[((size_t)t * ntiles + tile) * nsl + sl] != 0;
+    if (!used) continue;  // uniform
+    const int key = k0 >> 3;
+    const int slot = (a < natoms && key < nkeys) ? map[a * nkeys + key] : -1;
+    const double *wp = W + ((size_t)a * cap + (slot >= 0 ? slot : 0)) * 24 + 6 * k;
+    const double x0 = (slot >= 0 && q0 < 6) ? wp[q0] : 0.0;
+    const double x1 = (slot >= 0 && q0 + 1 < 6) ? wp[q0 + 1] : 0.0;
+    uint32_t h[kS];
+    digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
+    unsigned char *dst = rowbase + (size_t)sl * block + ((k0 % kTK) >> 3) * kLBO;
+#pragma unroll
+    for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
+  }
+}
+
+// T for the atoms of type alpha of one 12-atom tile (one block): the tile's shares (one per
+// kShareSlices used slices) summed, scaled by 2^(E_m + F_(a,k)) and by 1/N_c.
+__global__ void __launch_bounds__(256) fwd_epilogue_kernel(const float4 *__restrict__ part, int Mp, int64_t Np,
+                                                           const int *__restrict__ eexp,
+                                                           const int *__restrict__ fexp,
+                                                           const unsigned char *__restrict__ occ, int nsl,
+                                                           int64_t natoms, int64_t atom0,
+                                                           const int32_t *__restrict__ atype, int ntypes, int alpha,
+                                                           int M1, double inv_nnei, double *__restrict__ T) {
+  __shared__ int nused;
+  const int64_t tile = blockIdx.x;
+  if (threadIdx.x == 0) nused = 0;
+  __syncthreads();
+  int c = 0;
+  for (int x = threadIdx.x; x < nsl; x += blockDim.x) c += occ[tile * nsl + x] != 0;
+  if (c) atomicAdd(&nused, c);
+  __syncthreads();
+  const int nz = (nused + kShareSlices - 1) / kShareSlices;
+  for (int e = threadIdx.x; e < kTN * M1; e += blockDim.x) {
+    const int col = e % kTN, m = e / kTN;  // columns fastest: the shares' reads coalesce
+    const int64_t n = tile * kTN + col, a = n >> 2;
+    const int k = (int)(n & 3);
+    if (a >= natoms) continue;
+    if (atype && clampi(atype[atom0 + a], 0, ntypes - 1) != alpha) continue;
+    double v = 0.0;  // an atom of a tile without used slices has no valid rows
+    if (nz > 0) {
+      Sum3 acc;
+      for (int z = 0; z < nz; ++z) acc.add(part[((size_t)z * Mp + m) * Np + n]);
+      v = acc.value(eexp[m], fexp[n]) * inv_nnei;
+    }
+    T[((atom0 + a) * kCols + k) * M1 + m] = v;
+  }
+}
+
+struct RowsParams {
+  const double *s, *Rt;
+  const int32_t *nvalid, *atype;
+  TableGeom g;
+  int64_t atom0;
+  int nnei, ntypes, nkeys, cap;
+  int sel[DP_MAX_TYPES];
+  const int *map;
+  const float4 *dW;    // [natoms][cap][24]: the backward GEMM's result per run slot (four floats)
+  const int *eexp;     // [ntypes][Mpb]: exponents of the backward A's rows 8 key + q
+  int Mpb;
+  const int *fexp;     // [Np]: exponents of dT's rows 4 a + k
+  double inv_nnei;
+  double *ds, *dRt;
+};
+
+struct alignas(16) RowsStage {
+  double r[32][4];
+  double u[32];
+  double dw[32][24];   // per run of the batch: dW[k][q] at 6 k + q
+  double dwq[32][24];  // q dW[k][q] / Delta_l
+  int key[32], run[32], clamped[32], row[32];
+  int nvb[DP_MAX_TYPES];
+};
+
+// One warp per atom: each run's dW finished from the GEMM's four floats (lanes 6 k + q), then
+// each valid row's dE/dR~ and dE/ds by Horner's rule in u (a lane per row); padded rows get zeros.
+__global__ void __launch_bounds__(32) rows_kernel(const RowsParams P) {
+  __shared__ RowsStage st;
+  const int lane = threadIdx.x;
+  const int64_t a = blockIdx.x;
+  const int64_t i = P.atom0 + a;
+  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);
+  const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
+  const int *map = P.map + a * P.nkeys;
+  const int *eexp = P.eexp + (size_t)alpha * P.Mpb;
+  const double *srow = P.s + i * P.nnei;
+  const double *Rrow = P.Rt + i * P.nnei * 4;
+  double *dsrow = P.ds + i * P.nnei;
+  double *drow = P.dRt + i * P.nnei * 4;
+  for (int base = 0; base < nv; base += 32) {
+    const int v = base + lane;
+    if (v < nv) {
+      int b;
+      const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
+      double t;
+      bool clamped;
+      const int l = locate(P.g, __ldg(srow + row), t, clamped);
+      const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
+      st.r[lane][0] = rr.x;
+      st.r[lane][1] = rr.y;
+      st.r[lane][2] = rr.z;
+      st.r[lane][3] = rr.w;
+      st.u[lane] = t * (l < P.g.n0 ? P.g.inv0 : P.g.inv1);
+      st.key[lane] = b * P.g.nint + l;
+      st.clamped[lane] = clamped;
+      st.row[lane] = row;
+    }
+    __syncwarp();
+    const int cnt = min(32, nv - base);
+    const int mykey = lane < cnt ? st.key[lane] : -1;
+    const int prev = __shfl_up_sync(0xffffffffu, mykey, 1);
+    unsigned starts = __ballot_sync(0xffffffffu, lane < cnt && (lane == 0 || mykey != prev));
+    int nrun = 0;
+    while (starts) {  // uniform, run by run
+      const int u0 = __ffs(starts) - 1;
+      starts &= starts - 1;
+      const int e = starts ? __ffs(starts) - 1 : cnt;
+      const int key = __shfl_sync(0xffffffffu, mykey, u0);
+      if (lane < 24) {
+        const int k = lane / 6, q = lane - 6 * (lane / 6);
+        const int slot = map[key];
+        Sum3 acc;
+        acc.add(P.dW[((size_t)a * P.cap + slot) * 24 + lane]);
+        const double d = acc.value(eexp[key * kQ + q], P.fexp[kCols * a + k]) * P.inv_nnei;
+        const int l = key % P.g.nint;
+        st.dw[nrun][lane] = d;
+        st.dwq[nrun][lane] = (double)q * d * (l < P.g.n0 ? P.g.inv0 : P.g.inv1);
+      }
+      if (lane >= u0 && lane < e) st.run[lane] = nrun;
+      ++nrun;
+    }
+    __syncwarp();
+    if (lane < cnt) {
+      const double *dw = st.dw[st.run[lane]], *dq = st.dwq[st.run[lane]];
+      const double u = st.u[lane];
+      double d4[4], ds = 0.0;
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const double *c = dw + 6 * k, *cq = dq + 6 * k;
+        double h = fma(c[5], u, c[4]);
+        h = fma(h, u, c[3]);
+        h = fma(h, u, c[2]);
+        h = fma(h, u, c[1]);
+        d4[k] = fma(h, u, c[0]);
+        double gq = fma(cq[5], u, cq[4]);
+        gq = fma(gq, u, cq[3]);
+        gq = fma(gq, u, cq[2]);
+        gq = fma(gq, u, cq[1]);
+        ds = fma(st.r[lane][k], gq, ds);
+      }
+      const int row = st.row[lane];
+      dsrow[row] = st.clamped[lane] ? 0.0 : ds;
+      st4(drow + (size_t)row * 4, d4[0], d4[1], d4[2], d4[3]);
+    }
+    __syncwarp();
+  }
+  // padded rows of each segment
+  int off = 0;
+  for (int b = 0; b < P.ntypes; ++b) {  // uniform
+    for (int j = st.nvb[b] + lane; j < P.sel[b]; j += 32) {
+      dsrow[off + j] = 0.0;
+      st4(drow + (size_t)(off + j) * 4, 0.0, 0.0, 0.0, 0.0);
+    }
+    off += P.sel[b];
+  }
+}
+
+int check_work(const Layout &L, const void *work, size_t nbytes, const char *who) {
+  if (!work) return set_error(DP_ERR_NULL, "%s: work is NULL", who);
+  if (nbytes < L.total) return set_error(DP_ERR_SHAPE, "%s: work holds %zu bytes, needs %zu", who, nbytes, L.total);
+  if (reinterpret_cast<uintptr_t>(work) % 256) return set_error(DP_ERR_SHAPE, "%s: work is not 256-byte aligned", who);
+  return DP_OK;
+}
+
+// C' of every centre type from the table, then its digit planes: forward A = C'^T (rows: the
+// channels, K: 8 key + q), backward A = C' (rows: 8 key + q, K: the channels).
+int prep(const double *table, const TableGeom &g, const Shape &s, const Layout &L, unsigned char *wk, bool fwd,
+         cudaStream_t st, const char *who) {
+  double *Cp = reinterpret_cast<double *>(wk + L.cp);
+  const int64_t total = (int64_t)s.ntypes * s.Kp * s.M1;
+  coef_kernel<<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(table, g, s.ntypes, s.M1,
+                                                                                          s.Kp, Cp);
+  int rc = launch_status(who);
+  for (int t = 0; t < s.ntypes && !rc; ++t) {
+    const double *Ct = Cp + (size_t)t * s.Kp * s.M1;
+    rc = fwd ? split_rows(Ct, 1, s.M1, s.M1, s.Kp, s.Mpf, s.Kp, kTM, wk + L.afwd + (size_t)t * kS * s.Mpf * s.Kp * 2,
+                          wk + L.efwd + (size_t)t * s.Mpf * sizeof(int), st, who)
+             : split_rows(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM, wk + L.abwd + (size_t)t * kS * s.Mpb * s.Kpm * 2,
+                          wk + L.ebwd + (size_t)t * s.Mpb * sizeof(int), st, who);
+  }
+  return rc;
+}
+
+RunsParams runs_params(const double *s, const double *Rt, const int32_t *nvalid, const int32_t *atype,
+                       const TableGeom &g, const Segments &seg, const Shape &S, const Layout &L, unsigned char *wk,
+                       int nnei) {
+  RunsParams R{};
+  R.s = s;
+  R.Rt = Rt;
+  R.nvalid = nvalid;
+  R.atype = atype;
+  R.g = g;
+  R.nnei = nnei;
+  R.ntypes = S.ntypes;
+  R.nkeys = S.nkeys;
+  R.cap = S.cap;
+  for (int b = 0; b < DP_MAX_TYPES; ++b) R.sel[b] = seg.sel[b];
+  R.map = reinterpret_cast<int *>(wk + L.map);
+  R.occ = wk + L.occ;
+  R.fexp = reinterpret_cast<int *>(wk + L.fexp);
+  return R;
+}
+
+int fwd(const double *table, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
+        const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *work,
+        size_t work_bytes, void *stream) {
+  clear_error();
+  static const char *who = "dp_tabulate_fusion_fwd_tc_f64";
+  TableGeom g;
+  Segments seg;
+  int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, T, &g, &seg);
+  if (rc) return rc;
+  if (nloc == 0) return DP_OK;
+  const Shape S = make_shape(g, nloc, nnei, ntypes, M1);
+  const Layout L = make_layout(S);
+  if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
+  const cudaStream_t st = (cudaStream_t)stream;
+  unsigned char *wk = static_cast<unsigned char *>(work);
+  if ((rc = prep(table, g, S, L, wk, true, st, who))) return rc;
+  RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
+  R.W = reinterpret_cast<double *>(wk + L.w);
+  R.occ_cols = S.nsl;
+  R.keys_per_unit = kTK / kQ;
+  float4 *part = reinterpret_cast<float4 *>(wk + L.part);
+  for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
+    const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
+    const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN;
+    const size_t occ_per_type = (size_t)ntiles * S.nsl;
+    if (cudaMemsetAsync(wk + L.occ, 0, (size_t)ntypes * occ_per_type, st) != cudaSuccess)
+      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+    R.atom0 = c0;
+    R.natoms = n;
+    R.ntiles = ntiles;
+    runs_kernel<true><<<(unsigned)n, 32, 0, st>>>(R);
+    if ((rc = launch_status(who))) return rc;
+    const int64_t warps = Np / 8 * ((S.Kp + kSplitK - 1) / kSplitK);
+    split_mom_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(R.W, R.map, R.fexp, wk + L.occ, ntypes, ntiles, n,
+                                                                   S.nkeys, S.cap, Np, S.Kp, wk + L.bplanes);
+    if ((rc = launch_status(who))) return rc;
+    for (int t = 0; t < ntypes; ++t) {
+      TcGemm G{};
+      G.aplanes = wk + L.afwd + (size_t)t * kS * S.Mpf * S.Kp * 2;
+      G.Eexp = reinterpret_cast<const int *>(wk + L.efwd) + (size_t)t * S.Mpf;
+      G.Mp = S.Mpf;
+      G.planes = wk + L.bplanes;
+      G.Fexp = R.fexp;
+      G.Np = (int)Np;
+      G.Kp = S.Kp;
+      G.part = part;
+      G.slices_per_split = kShareSlices;
+      G.kocc = wk + L.occ + (size_t)t * occ_per_type;
+      const dim3 grid((unsigned)ntiles, (unsigned)(S.Mpf / kTM), (unsigned)S.zmax);
+      gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
+      if ((rc = launch_status(who))) return rc;
+      fwd_epilogue_kernel<<<(unsigned)ntiles, 256, 0, st>>>(part, S.Mpf, Np, G.Eexp, R.fexp, G.kocc, S.nsl, n, c0,
+                                                            atype, ntypes, t, M1, 1.0 / (double)nnei, T);
+      if ((rc = launch_status(who))) return rc;
+    }
+  }
+  return DP_OK;
+}
+
+int grad(const double *table, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
+         const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, const double *dT,
+         double *ds, double *dRt, void *work, size_t work_bytes, void *stream) {
+  clear_error();
+  static const char *who = "dp_tabulate_fusion_grad_tc_f64";
+  TableGeom g;
+  Segments seg;
+  int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, ds, dRt, &g, &seg);
+  if (rc) return rc;
+  if (nloc > 0 && !dT) return set_error(DP_ERR_NULL, "%s: dT is NULL", who);
+  if (nloc == 0) return DP_OK;
+  const Shape S = make_shape(g, nloc, nnei, ntypes, M1);
+  const Layout L = make_layout(S);
+  if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
+  const cudaStream_t st = (cudaStream_t)stream;
+  unsigned char *wk = static_cast<unsigned char *>(work);
+  if ((rc = prep(table, g, S, L, wk, false, st, who))) return rc;
+  RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
+  const int mtiles = S.Mpb / kTM;
+  R.occ_cols = mtiles;
+  R.keys_per_unit = kTM / kQ;
+  float4 *dW = reinterpret_cast<float4 *>(wk + L.w);
+  RowsParams Q{};
+  Q.s = s;
+  Q.Rt = Rt;
+  Q.nvalid = nvalid;
+  Q.atype = atype;
+  Q.g = g;
+  Q.nnei = nnei;
+  Q.ntypes = ntypes;
+  Q.nkeys = S.nkeys;
+  Q.cap = S.cap;
+  for (int b = 0; b < DP_MAX_TYPES; ++b) Q.sel[b] = seg.sel[b];
+  Q.map = R.map;
+  Q.dW = dW;
+  Q.eexp = reinterpret_cast<const int *>(wk + L.ebwd);
+  Q.Mpb = S.Mpb;
+  Q.fexp = R.fexp;
+  Q.inv_nnei = 1.0 / (double)nnei;
+  Q.ds = ds;
+  Q.dRt = dRt;
+  for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
+    const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
+    const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN;
+    const size_t occ_per_type = (size_t)ntiles * mtiles;
+    if (cudaMemsetAsync(wk + L.occ, 0, (size_t)ntypes * occ_per_type, st) != cudaSuccess)
+      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+    R.atom0 = c0;
+    R.natoms = n;
+    R.ntiles = ntiles;
+    runs_kernel<false><<<(unsigned)n, 32, 0, st>>>(R);
+    if ((rc = launch_status(who))) return rc;
+    // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
+    if ((rc = split_rows(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, Np, S.Kpm, kTN, wk + L.bplanes, wk + L.fexp, st,
+                         who)))
+      return rc;
+    for (int t = 0; t < ntypes; ++t) {
+      TcGemm G{};
+      G.aplanes = wk + L.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
+      G.Eexp = Q.eexp + (size_t)t * S.Mpb;
+      G.Mp = S.Mpb;
+      G.planes = wk + L.bplanes;
+      G.Fexp = R.fexp;
+      G.Np = (int)Np;
+      G.Kp = S.Kpm;
+      G.slices_per_split = S.Kpm / kTK;
+      G.tocc = wk + L.occ + (size_t)t * occ_per_type;
+      G.scat = dW;
+      G.map = R.map;
+      G.atype = atype;
+      G.natoms = n;
+      G.atom0 = c0;
+      G.nkeys = S.nkeys;
+      G.cap = S.cap;
+      G.alpha = t;
+      G.ntypes = ntypes;
+      const dim3 grid((unsigned)ntiles, (unsigned)mtiles, 1);
+      gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
+      if ((rc = launch_status(who))) return rc;
+    }
+    Q.atom0 = c0;
+    rows_kernel<<<(unsigned)n, 32, 0, st>>>(Q);
+    if ((rc = launch_status(who))) return rc;
+  }
+  return DP_OK;
+}
+
+size_t work_bytes_api(const dp_table_info *info, int64_t nloc, int nnei, int ntypes, int M1) {
+  clear_error();
+  TableGeom g;
+  if (make_geom(info, &g)) return 0;
+  if (nloc < 0 || nnei < 1 || ntypes < 1 || ntypes > DP_MAX_TYPES || M1 < 1 || M1 > DP_MAX_M1) {
+    set_error(DP_ERR_SHAPE, "dp_tabulate_tc_work_bytes: nloc %lld, nnei %d, ntypes %d, M1 %d out of range",
+              (long long)nloc, nnei, ntypes, M1);
+    return 0;
+  }
+  return make_layout(make_shape(g, nloc, nnei, ntypes, M1)).total;
+}
+
+}  // namespace tt
+}  // namespace
+}  // namespace dpc
+
+extern "C" {
+
+size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nnei, int ntypes, int M1) {
+  return dpc::tt::work_bytes_api(info, nloc, nnei, ntypes, M1);
+}
+
+int dp_tabulate_fusion_fwd_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+                                  const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                  const int32_t *sel, int M1, double *T, void *work, size_t work_bytes,
+                                  void *stream) {
+  return dpc::tt::fwd(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, work, work_bytes, stream);
+}
+
+int dp_tabulate_fusion_grad_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                   const int32_t *sel, int M1, const double *dT, double *ds, double *dRt, void *work,
+                                   size_t work_bytes, void *stream) {
+  return dpc::tt::grad(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, work, work_bytes,
+                       stream);
+}
+
+}  // extern "C"

@@ -1,0 +1,472 @@
+// Exact f64 GEMMs on the tcgen05 tensor cores, shared by the fitting net and the
+// tensor-core form of the tabulated embedding.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cstdint>
+
+#include "dp_common.cuh"
+
+namespace dpc {
+namespace {
+
+
+// ------------------------------------------------- f64 GEMMs on the tensor cores
+// GB300 retires FP64 at 2 lanes per clock per SM but fp16 products on its
+// tcgen05 tensor cores at ~1000 times that rate.  An f64 GEMM C = A B is
+// recovered from fp16 products by splitting every operand element into base-64
+// digits (the error-free splitting of Ozaki et al.):
+//   a_ik = 2^E_i sum_{s=1..9} A_s[i][k] 64^-s + r_ik,  A_s integers in [-63, 63],  |r_ik| < 2^(E_i - 54),
+// with max_k |a_ik| < 2^E_i, and likewise b_kj with a column exponent F_j, so that
+//   C_ij = 2^(E_i + F_j) sum_{d=2..10} 64^-d sum_{s+t=d} (A_s B_t)_ij + (terms with s + t > 10 and the r).
+// Every (A_s B_t)_ij is a sum of integer products |A_s B_t| <= 3969; a diagonal
+// d has at most 9 of them, so its fp32 sum on the tensor cores is exact while
+// a block's share of K is at most kMaxShareK = 448 (9 x 448 x 3969 < 2^24).
+// The 9 diagonal sums of an output are combined on the FP32 pipe into four
+// floats (the two largest by an exact two-sum, the rest in float-float, whose
+// rounding lies ~2^-60 below the result); epilogue_kernel adds the shares'
+// floats into a three-float sum by exact two-sums and converts it to f64 once.
+// What rounds is that conversion, the 54-bit truncation of the operands and
+// the dropped terms: |error| <~ K 2^-50 max_k|a_ik| max_k|b_kj|, against
+// K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column with an
+// inf or NaN gives NaN outputs.
+//
+// gemm_kernel: one CTA of 128 threads per 128 x 48 output tile and share of K,
+// one CTA per SM (its 9 diagonal accumulators take 432 of the SM's 512 TMEM
+// columns).  The digit planes of A (per chunk of rows) and B (per call) are
+// made by split_rows_kernel, once per element, as the shared-memory image of
+// each (tile, 16-deep K slice) block: the tcgen05 K-major layout without
+// swizzle (8-row x 16-byte core matrices).  Lane 0 of warp 0 moves a slice's
+// A and B blocks into one of four stages with two bulk async copies counted in
+// bytes on the stage's "full" mbarrier; lane 0 of warp 1 issues the slice's 45
+// digit-product MMAs (M 128, N 48, K 16, fp16 in, fp32 accumulators in TMEM,
+// one per diagonal) and commits them to the stage's "empty" mbarrier, which
+// the producer waits on before refilling the stage.  A last commit on a
+// barrier used once releases the four warps, which read their TMEM lane
+// quadrant (rows), combine the diagonals and write the share's result as four
+// floats; the caller's epilogue kernel sums the shares in a fixed order,
+// scales by 2^(E+F) and finishes the outputs.  Two optional modes serve sparse
+// operands (the tabulated embedding's interval moments): a per-tile list of the
+// K slices in use (the others are zero and are skipped; the shares then cut the
+// used slices), and a per-tile flag that skips unwanted output tiles, whose
+// wanted outputs are scattered to per-run slots instead of a dense array.
+// Every wait on an mbarrier is bounded; a wait that gives up makes the tile's
+// outputs NaN.
+namespace tc {
+constexpr int kS = 9;      // digits per operand element
+constexpr int kBits = 6;   // bits per digit
+constexpr int kFrac = kS * kBits;  // 54 fractional bits
+constexpr int kTM = 128, kTN = 48, kTK = 16;  // CTA tile; K per stage (one MMA)
+constexpr int kStages = 4;
+constexpr int kThreads = 128;  // one warp per TMEM lane quadrant; lane 0 of warps 0 and 1: producer and MMA issuer
+constexpr int kMaxShareK = 448;
+constexpr int kNonFinite = 1 << 20;  // exponent of a row or column holding inf or NaN
+constexpr uint32_t kLBO = 128, kSBO = 256;  // core matrices: next along K at +128 B, next 8 rows at +256 B
+constexpr int kPlaneA = kTM * kTK * 2, kPlaneB = kTN * kTK * 2;  // bytes of one digit plane in a stage
+constexpr int kStageBytes = kS * (kPlaneA + kPlaneB);
+constexpr uint32_t kTmemCols = 512;  // allocation (a power of two); kS * kTN = 432 used
+constexpr int kMaxShareSlices = kMaxShareK / kTK;
+constexpr size_t kSmemTail = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16;  // used-slice list
+constexpr size_t kSmemTotal = kSmemTail + (kMaxShareSlices + 1) * 4;
+static_assert((size_t)kS * kMaxShareK * 63 * 63 < (1u << 24), "fp32 diagonal sums must stay exact");
+static_assert(kMaxShareK % kTK == 0 && kS * kTN <= (int)kTmemCols, "shares and TMEM");
+static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
+
+__host__ __device__ constexpr int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+__device__ __forceinline__ int exp_bits(double x) { return (int)(((uint64_t)__double_as_longlong(x) >> 52) & 0x7ff); }
+// E with max |x| < 2^E from the largest biased exponent (normal x: |x| < 2^(eb - 1022))
+__device__ __forceinline__ int exp_of_max(int ebmax) { return ebmax == 0x7ff ? kNonFinite : max(ebmax, 1) - 1022; }
+
+// |x| 2^-E as an integer with kFrac fractional bits, truncated; below 2^kFrac since |x| < 2^E
+__device__ __forceinline__ uint64_t fixed_point(double x, int E) {
+  const uint64_t b = (uint64_t)__double_as_longlong(x);
+  const int eb = (int)((b >> 52) & 0x7ff);
+  const uint64_t mant = b & 0xfffffffffffffull;
+  const uint64_t m = eb ? (mant | (1ull << 52)) : mant;
+  const int sh = (eb ? eb - 1075 : -1074) - E + kFrac;  // |x| 2^(kFrac - E) = m 2^sh, sh <= 1 for finite x
+  if (sh >= 0) return m << min(sh, 10);
+  return sh > -64 ? m >> -sh : 0ull;
+}
+
+// The kS digits of two fixed-point values, digit s of both packed as an fp16 pair (element 0 in the
+// low half), each with its element's sign: 0x6400 | d is the fp16 1024 + d, and 1024 comes off exactly.
+__device__ __forceinline__ void digit_pairs(uint64_t f0, uint64_t f1, uint32_t sign2, uint32_t (&h)[kS]) {
+  constexpr uint32_t kMask = (1u << kBits) - 1;
+#pragma unroll
+  for (int s = 1; s <= kS; ++s) {
+    const uint32_t d0 = (uint32_t)(f0 >> (kFrac - kBits * s)) & kMask;
+    const uint32_t d1 = (uint32_t)(f1 >> (kFrac - kBits * s)) & kMask;
+    uint32_t v;
+    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(v) : "r"(0x64006400u | d0 | (d1 << 16)), "r"(0x64006400u));
+    h[s - 1] = v ^ sign2;
+  }
+}
+
+__device__ __forceinline__ uint32_t sign_pair(double x0, double x1) {
+  return (uint32_t)((uint64_t)__double_as_longlong(x0) >> 63) << 15 | (uint32_t)((uint64_t)__double_as_longlong(x1) >> 63)
+                                                                          << 31;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+// Rows of a matrix as digit planes, laid out as the shared-memory image of each (tile of RT rows,
+// 16-deep K slice) block that gemm_kernel copies in one piece: block (r / RT, k / 16) holds the kS
+// planes of those rows and columns, plane s at s RT 32 bytes, and in a plane the tcgen05 K-major
+// core matrices (8 rows x 8 k = 128 bytes; the second 8 k of the slice at +128 B, the next 8 rows
+// at +256 B).  Also the rows' exponents [rows_p].  Element (r, k) of the source is X[r ld_r + k ld_k];
+// rows >= nrows and columns >= K are zero (row_exps_kernel first finds the exponents).  Used for the A operand (rows of the
+// layer input, RT = kTM) and for B (RT = kTN; forward: the columns of W, ld_r = 1, ld_k = N;
+// backward: the rows of W).
+__global__ void __launch_bounds__(128) row_exps_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
+                                                       int64_t nrows, int K, int64_t rows_p, int *__restrict__ exps) {
+  // one warp per row: E with max_k |x_rk| < 2^E
+  const int lane = threadIdx.x & 31;
+  const int64_t r = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (r >= rows_p) return;  // warp-uniform
+  int eb = 0;
+  if (r < nrows)
+    for (int k = lane; k < K; k += 32) eb = max(eb, exp_bits(__ldg(X + r * ld_r + k * ld_k)));
+  eb = __reduce_max_sync(0xffffffffu, eb);
+  if (lane == 0) exps[r] = exp_of_max(eb);
+}
+
+constexpr int kSplitK = 64;  // K per warp of split_rows_kernel
+__global__ void __launch_bounds__(128) split_rows_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
+                                                         int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
+                                                         unsigned char *__restrict__ planes,
+                                                         const int *__restrict__ exps) {
+  // one warp per (group of 8 rows, kSplitK of K): lane = (row ri8 = lane / 4, pair of k kp = lane % 4),
+  // so that per plane and 8 k the warp writes one whole 128-byte core matrix
+  const int lane = threadIdx.x & 31, ri8 = lane >> 2, kp = lane & 3;
+  const int kchunks = (Kp + kSplitK - 1) / kSplitK;
+  const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  const int64_t g = w / kchunks;  // 8-row group
+  if (g * 8 >= rows_p) return;    // warp-uniform
+  const int kc = (int)(w - g * kchunks);
+  const int64_t r = g * 8 + ri8;
+  const double *__restrict__ xr = X + (r < nrows ? r : 0) * ld_r;
+  auto x = [&](int k) { return (r < nrows && k < K) ? __ldg(xr + k * ld_k) : 0.0; };
+  const int E = exps[r];
+  const size_t plane = (size_t)RT * kTK * 2, block = kS * plane;
+  const int ri = (int)(r % RT);
+  unsigned char *rowbase = planes + (size_t)(r / RT) * (Kp / kTK) * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
+  for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
+    const int k = k0 + 2 * kp;
+    const double x0 = x(k), x1 = x(k + 1);
+    uint32_t h[kS];
+    digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
+    unsigned char *dst = rowbase + (size_t)(k0 / kTK) * block + ((k0 % kTK) >> 3) * kLBO;
+#pragma unroll
+    for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
+  }
+}
+
+// One hidden-layer GEMM of a chunk of one type's atoms: rows r0 .. r0 + n - 1 of the plain
+// row-major A [*][K] (as digit planes) times B (digit planes), K cut into shares of at most
+// kMaxShareK (grid z); the shares' f64 results go to `part`, and epilogue_kernel sums them and
+// applies the layer's epilogue.
+struct TcGemm {
+  int64_t r0, n;  // output rows r0 .. r0 + n - 1; A's planes hold rows 0 .. n - 1 of this chunk
+  int K, N;
+  const double *A;  // the layer input itself (forward: its skip term)
+  int64_t lda;
+  const unsigned char *aplanes;  // A's blocks [Mp / kTM][Kp / kTK] of kS x kPlaneA bytes
+  const int *Eexp;          // [Mp]
+  int64_t Mp;
+  const unsigned char *planes;   // B's blocks [Np / kTN][Kp / kTK] of kS x kPlaneB bytes
+  const int *Fexp;
+  int Np, Kp;
+  float4 *part;             // [ksplit][Mp][Np]: each share's result (grid z) as four floats, see gemm_kernel
+  int slices_per_split;
+  // sparse operands (NULL for dense ones)
+  const unsigned char *kocc;  // [Np / kTN][Kp / kTK]: nonzero where the B tile has a nonzero entry in the
+                              // slice; share z of a tile then takes its used slices z S .. z S + S - 1
+                              // (S = slices_per_split), and a share past its last used slice writes nothing
+  const unsigned char *tocc;  // [Np / kTN][Mp / kTM]: nonzero where the output tile is wanted
+  // scatter (with tocc): output (row 8 key + q, column 4 a + k), q < 6, key < nkeys, a < natoms, goes to
+  // scat[(a cap + slot) 24 + 6 k + q] when slot = map[a nkeys + key] >= 0 and atom atom0 + a has type
+  // alpha (atype clamped into [0, ntypes)); nothing is written to part
+  float4 *scat;
+  const int *map;
+  const int32_t *atype;
+  int64_t natoms, atom0;
+  int nkeys, cap, alpha, ntypes;
+  bool skip;
+  // forward
+  const double *bias;
+  double *act;
+  int64_t ldact;
+  double *V;
+  int64_t ldv;
+  // backward
+  const double *S;  // NULL: S(row, col) = g_row wo_col
+  int64_t ldS;
+  const double *g, *wo;
+  const double *T;  // tanh outputs of the layer below (NULL: the last GEMM)
+  int64_t ldT;
+  double *Snext, *Z;
+  int64_t ldz;
+  double *out;
+  int64_t ldo;
+};
+
+// shared-memory descriptor of a K-major operand without swizzle (tcgen05): start address, the byte
+// offsets of the next core matrix along K (leading) and along the rows (stride), version 1
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+  return (uint64_t)((saddr & 0x3FFFF) >> 4) | ((uint64_t)(kLBO >> 4) << 16) | ((uint64_t)(kSBO >> 4) << 32) |
+         (1ull << 46);
+}
+// instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A and B f16 (0), both K-major, N >> 3 at
+// bit 17 (set per MMA), M >> 4 at bit 24
+constexpr uint32_t kIdescNoN = (1u << 4) | ((uint32_t)(kTM >> 4) << 24);  // N >> 3 goes in at bit 17
+constexpr int kMaxPlanesPerMma = 256 / kTN;  // N <= 256 for M = 128
+static_assert(kTN % 16 == 0 && kMaxPlanesPerMma >= 1, "MMA N: multiples of 16 up to 256");
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  uint32_t done = 0;
+  for (int it = 0; it < (1 << 24) && !done; ++it)
+    asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+                 : "=r"(done)
+                 : "r"(bar), "r"(parity)
+                 : "memory");
+  return done != 0;
+}
+
+__global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);  // stage loaded
+  uint64_t *empty = full + kStages;                                               // stage's MMAs done
+  uint64_t *done = empty + kStages;                                               // every MMA done (one use)
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(done + 1);
+  int *flags = reinterpret_cast<int *>(tmem_holder + 1);                          // producer / issuer ok
+  int *slist = reinterpret_cast<int *>(smem + kSmemTail);                         // used slices, then their count
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int64_t m0 = (int64_t)blockIdx.y * kTM;
+  const int n0 = blockIdx.x * kTN;
+  const int nslices = P.Kp / kTK;
+  const int i0 = blockIdx.z * P.slices_per_split;
+  if (P.tocc && !P.tocc[(size_t)blockIdx.x * gridDim.y + blockIdx.y]) return;  // unwanted tile (uniform)
+  int nsl = min(nslices - i0, P.slices_per_split);  // dense: > 0, no empty share
+  if (P.kocc) {
+    // this share's used slices, in order, by a ballot over the tile's flags
+    if (warp == 0) {
+      const unsigned char *occ = P.kocc + (size_t)blockIdx.x * nslices;
+      const int last = i0 + P.slices_per_split;
+      int rank = 0;
+      for (int b = 0; b < nslices && rank < last; b += 32) {  // uniform
+        const int i = b + lane;
+        const bool used = i < nslices && occ[i] != 0;
+        const unsigned m = __ballot_sync(0xffffffffu, used);
+        const int r = rank + __popc(m & ((1u << lane) - 1u));
+        if (used && r >= i0 && r < last) slist[r - i0] = i;
+        rank += __popc(m);
+      }
+      if (lane == 0) slist[kMaxShareSlices] = min(max(rank - i0, 0), P.slices_per_split);
+    }
+    __syncthreads();
+    nsl = slist[kMaxShareSlices];
+    if (nsl == 0) return;  // uniform: no slice left for this share
+  }
+
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(full + s)));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(empty + s)));
+    }
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(done)));
+    asm volatile("fence.mbarrier_init.release.cluster;");
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                 "r"(kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;");
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t sbase = smem_u32(smem);
+  bool ok = true;
+
+  if (warp == 0 && lane == 0) {
+    // producer: each slice's A and B blocks, one bulk copy each, counted in bytes on the stage's
+    // "full" barrier; a stage is reused once the MMAs that read it have completed ("empty")
+    for (int j = 0; j < nsl && ok; ++j) {
+      const int sl = P.kocc ? slist[j] : i0 + j;
+      const unsigned char *asrc = P.aplanes + ((size_t)blockIdx.y * nslices + sl) * (kS * kPlaneA);
+      const unsigned char *bsrc = P.planes + ((size_t)blockIdx.x * nslices + sl) * (kS * kPlaneB);
+      const int st = j % kStages;
+      if (j >= kStages) ok = mbar_wait(smem_u32(empty + st), (uint32_t)((j / kStages - 1) & 1));
+      if (!ok) break;
+      const uint32_t bar = smem_u32(full + st), dst = sbase + st * kStageBytes;
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"((uint32_t)kStageBytes)
+                   : "memory");
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                   "l"(asrc), "r"((uint32_t)(kS * kPlaneA)), "r"(bar)
+                   : "memory");
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       dst + kS * kPlaneA),
+                   "l"(bsrc), "r"((uint32_t)(kS * kPlaneB)), "r"(bar)
+                   : "memory");
+    }
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer: the 45 digit products of each slice once it has landed, then a commit that frees the stage
+    for (int i = 0; i < nsl && ok; ++i) {
+      const int st = i % kStages;
+      ok = mbar_wait(smem_u32(full + st), (uint32_t)((i / kStages) & 1));
+      if (!ok) break;
+      asm volatile("tcgen05.fence::after_thread_sync;");
+      const uint64_t a0 = smem_desc(sbase + st * kStageBytes), b0 = smem_desc(sbase + st * kStageBytes + kS * kPlaneA);
+      // Digit s of A against digits t = 0 .. kS-1-s of B in one MMA: B's planes lie back to back in
+      // the stage (48 rows each, one row stride), so together they are one operand of 48 (kS - s)
+      // rows, and with the accumulator address moved by s diagonals the block of plane t lands on
+      // diagonal s + t.  N is at most 256, so up to 5 planes (240 columns) per MMA: 13 MMAs per
+      // slice instead of 45, each reading its A tile once for up to 240 columns.
+#pragma unroll
+      for (int s = 0; s < kS; ++s) {
+        const uint64_t ad = a0 + (uint64_t)((s * kPlaneA) >> 4);  // start-address field, in 16-byte units
+#pragma unroll
+        for (int t0 = 0; t0 < kS - s; t0 += kMaxPlanesPerMma) {
+          const int np = min(kMaxPlanesPerMma, kS - s - t0);
+          const uint64_t bd = b0 + (uint64_t)((t0 * kPlaneB) >> 4);
+          const uint32_t idesc = kIdescNoN | ((uint32_t)((np * kTN) >> 3) << 17);
+          const uint32_t acc = (i > 0 || s > 0) ? 1u : 0u;  // digit 1 of A writes every diagonal first
+          asm volatile(
+              "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+              " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem + (uint32_t)((s + t0) * kTN)),
+              "l"(ad), "l"(bd), "r"(idesc), "r"(acc));
+        }
+      }
+      asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+          smem_u32(empty + st)));
+    }
+    // one more commit, on a barrier used once: it completes when every MMA issued above has (also
+    // after a wait that gave up, so that nobody waits on it in vain)
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(done)));
+  }
+  if (lane == 0 && warp < 2) flags[warp] = ok;
+  __syncwarp();
+  // The other warps wait here rather than on a stage barrier: a parity wait can only tell apart the
+  // current phase and the one before, and they would start it phases ahead of the MMAs.
+  __syncthreads();
+  ok = flags[0] && flags[1];
+  ok = mbar_wait(smem_u32(done), 0) && ok;
+  asm volatile("tcgen05.fence::after_thread_sync;");
+
+  // combine the diagonals of row 32 (warp % 4) + lane (the warp's TMEM lane quadrant), the warp's
+  // third of the columns, 8 at a time
+  const int rl = 32 * (warp & 3) + lane;
+  float4 *outp = P.scat ? nullptr : P.part + ((size_t)blockIdx.z * P.Mp + m0 + rl) * P.Np + n0;
+  const int key = (int)((m0 + rl) >> 3), q = (int)((m0 + rl) & 7);  // scatter: this thread's row
+  const bool row_wanted = P.scat && q < 6 && key < P.nkeys;
+  const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
+  constexpr int kColsPerWarp = kTN / (kThreads / 128);
+  static_assert(kColsPerWarp % 8 == 0, "column share");
+#pragma unroll 1
+  for (int c0 = (warp >> 2) * kColsPerWarp; c0 < (warp >> 2) * kColsPerWarp + kColsPerWarp; c0 += 8) {
+    float v[kS][8];
+#pragma unroll
+    for (int d = 0; d < kS; ++d)
+      asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                   : "=f"(v[d][0]), "=f"(v[d][1]), "=f"(v[d][2]), "=f"(v[d][3]), "=f"(v[d][4]), "=f"(v[d][5]),
+                     "=f"(v[d][6]), "=f"(v[d][7])
+                   : "r"(trow + (uint32_t)(d * kTN + c0)));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      // sum_d v_d 64^-(d+2) as four floats on the FP32 pipe: diagonals 2 and 3 (d = 0, 1) as an exact
+      // two-sum, 4 .. 10 in float-float, smallest first (its rounding lies ~2^-60 below the sum).
+      // The scaling by 2^(E+F), and all f64 arithmetic, is left to epilogue_kernel.
+      dfl::df64 lo(0.0f);
+#pragma unroll
+      for (int d = kS - 1; d >= 2; --d) {
+        const float x = v[d][c] * __uint_as_float((uint32_t)(127 - kBits * (d + 2)) << 23);  // exact: 64^-(d+2)
+        lo = lo + dfl::df64(x);
+      }
+      const float a = v[0][c] * 0x1p-12f, b = v[1][c] * 0x1p-18f;  // exact
+      const float s = __fadd_rn(a, b), bb = __fsub_rn(s, a);
+      const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+      const float4 val = ok ? make_float4(s, e, lo.hi, lo.lo) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
+      if (outp) {
+        outp[c0 + c] = val;
+      } else if (row_wanted) {
+        const int64_t a = (int64_t)(n0 + c0 + c) >> 2;
+        const int k = (n0 + c0 + c) & 3;
+        if (a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha)) {
+          const int slot = P.map[a * P.nkeys + key];
+          if (slot >= 0) P.scat[((size_t)a * P.cap + slot) * 24 + 6 * k + q] = val;
+        }
+      }
+    }
+  }
+
+  asm volatile("tcgen05.fence::before_thread_sync;");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;");
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+}
+
+// f 2^e as a double, exactly, by moving fields (f finite; |e| < 900, so a normal result stays normal
+// and a float that is zero stays zero; float subnormals, which the sums do not produce, widen to 0)
+__device__ __forceinline__ double widen_pow2(float f, int e) {
+  const double d = dfl::widen(f);
+  const long long b = __double_as_longlong(d);
+  return (b & 0x7fffffffffffffffll) ? __longlong_as_double(b + ((long long)e << 52)) : d;
+}
+
+// The shares' results of one output summed in a fixed order: each share's four floats are added
+// into a three-float sum by exact two-sums on the FP32 pipe (only the last component rounds, ~2^-72
+// below the sum), which is converted to f64 once and scaled by the row and column powers of two.
+struct Sum3 {
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    float t = __fadd_rn(s0, x), z = __fsub_rn(t, s0);
+    const float e0 = __fadd_rn(__fsub_rn(s0, __fsub_rn(t, z)), __fsub_rn(x, z));
+    s0 = t;
+    t = __fadd_rn(s1, e0);
+    z = __fsub_rn(t, s1);
+    const float e1 = __fadd_rn(__fsub_rn(s1, __fsub_rn(t, z)), __fsub_rn(e0, z));
+    s1 = t;
+    s2 = __fadd_rn(s2, e1);
+  }
+  __device__ __forceinline__ void add(const float4 q) {
+    add(q.x);
+    add(q.y);
+    add(q.z);
+    add(q.w);
+  }
+  // the sum times 2^(E + F); NaN for a row or column with an inf or NaN, or a NaN share
+  __device__ __forceinline__ double value(int E, int F) const {
+    if (E >= kNonFinite || F >= kNonFinite || s0 != s0) return __longlong_as_double(0x7ff8000000000000ll);
+    if (E + F > -900 && E + F < 900)  // the scaling moves exponent fields only (sums stay normal)
+      return __dadd_rn(__dadd_rn(widen_pow2(s0, E + F), widen_pow2(s1, E + F)), widen_pow2(s2, E + F));
+    return scalbn(__dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2)), E + F);
+  }
+};
+
+int set_smem(const char *who) {
+  static std::atomic<bool> done{false};
+  if (done.load(std::memory_order_acquire)) return DP_OK;
+  const cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemTotal);
+  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+  done.store(true, std::memory_order_release);
+  return DP_OK;
+}
+
+int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
+               unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
+  row_exps_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p,
+                                                                 reinterpret_cast<int *>(exps));
+  int rc = launch_status(who);
+  if (rc) return rc;
+  const int64_t warps = rows_p / 8 * ((Kp + kSplitK - 1) / kSplitK);
+  split_rows_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT, planes,
+                                                                 reinterpret_cast<const int *>(exps));
+  return launch_status(who);
+}
+}  // namespace tc
+}  // namespace
+}  // namespace dpc
