@@ -20,8 +20,8 @@
 // the tensor cores (tc_gemm.cuh), at f64 accuracy.
 //
 // K layout, per centre type: key = beta nint + l (neighbour type beta, interval
-// l), and column 8 key + q of the GEMM holds power q (q = 6, 7 are zero), so a
-// 16-deep K slice is two intervals.  An atom touches only the intervals its
+// l), and column 6 key + q of the GEMM holds power q, so an interval lies in
+// one or two 16-deep K slices.  An atom touches only the intervals its
 // rows fall in: the W values are stored per run of rows (one slot per
 // interval an atom uses, found through a per-atom map), and the GEMMs skip the
 // slices (forward) or output tiles (backward) that no atom of a tile uses.
@@ -48,19 +48,20 @@ namespace {
 namespace tt {
 using namespace tc;
 
-constexpr int kQ = 8;                 // K entries per interval: u^0 .. u^5 and two zeros
+constexpr int kQ = 6;                 // K entries per interval: u^0 .. u^5
 constexpr int kCols = 4;              // GEMM columns per atom: k = 0 .. 3
 constexpr int kTileAtoms = kTN / kCols;  // 12 atoms per 48-column tile
 constexpr int64_t kChunkAtoms = 4104;    // a multiple of 12 (16,416 columns)
 constexpr int kShareSlices = 14;         // used K slices per forward share
 constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' results per chunk
+constexpr int kMaxKeys = 16384;  // ntypes x nint: an atom's key map (int16) lives in shared memory
 static_assert(kShareSlices <= kMaxShareSlices, "share within the exactness bound");
 static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
 
 // Sizes shared by the kernels and the work-buffer layout.
 struct Shape {
   int ntypes, nint, nkeys, M1, cap;
-  int Kp;    // round_up(8 nkeys, 16): K of the forward GEMM, rows of the backward A
+  int Kp;    // round_up(6 nkeys, 16): K of the forward GEMM, rows of the backward A
   int nsl;   // Kp / 16
   int Mpf;   // round_up(M1, 128): rows of the forward A
   int Kpm;   // round_up(M1, 16): K of the backward GEMM
@@ -70,7 +71,7 @@ struct Shape {
 };
 
 struct Layout {
-  size_t cp, afwd, efwd, abwd, ebwd, map, occ, fexp, bplanes, w, part, total;
+  size_t cp, afwd, efwd, abwd, ebwd, map, keys, nslots, occ, fexp, bplanes, w, part, total;
 };
 
 Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1) {
@@ -111,6 +112,8 @@ Layout make_layout(const Shape &s) {
   L.abwd = take(nt * kS * (size_t)s.Mpb * s.Kpm * 2);
   L.ebwd = take(nt * s.Mpb * sizeof(int));
   L.map = take((size_t)s.chunk * s.nkeys * sizeof(int));
+  L.keys = take((size_t)s.chunk * s.cap * sizeof(int));
+  L.nslots = take((size_t)s.chunk * sizeof(int));
   L.occ = take(nt * s.ntiles * std::max(s.nsl, s.Mpb / kTM));
   L.fexp = take((size_t)s.Np * sizeof(int));
   L.bplanes = take((size_t)s.ntiles * std::max(s.nsl, s.Kpm / kTK) * kS * kPlaneB);
@@ -120,19 +123,19 @@ Layout make_layout(const Shape &s) {
   return L;
 }
 
-// C'[alpha][8 key + q][m] = c_q Delta_l^q (key = beta nint + l; q >= 6 and rows past the keys: 0).
+// C'[alpha][6 key + q][m] = c_q Delta_l^q / N_c (key = beta nint + l; rows past the keys: 0).
 // The interval's block of the table is pair-planar [3][M1][2] holding (a, b, c, d, e, f), the
 // coefficients of t^5 .. t^0.
 __global__ void __launch_bounds__(256) coef_kernel(const double *__restrict__ table, TableGeom g, int ntypes, int M1,
-                                                   int Kp, double *__restrict__ Cp) {
+                                                   int Kp, double scale, double *__restrict__ Cp) {
   const int64_t total = (int64_t)ntypes * Kp * M1;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total; x += (int64_t)gridDim.x * blockDim.x) {
     const int m = (int)(x % M1);
     const int64_t rest = x / M1;
     const int r = (int)(rest % Kp), alpha = (int)(rest / Kp);
-    const int key = r >> 3, q = r & 7;
+    const int key = r / kQ, q = r - kQ * key;
     double v = 0.0;
-    if (q < 6 && key < ntypes * g.nint) {
+    if (key < ntypes * g.nint) {
       const int beta = key / g.nint, l = key - beta * g.nint;
       const double *blk = table + ((size_t)(alpha * ntypes + beta) * g.nint + l) * M1 * 6;
       const int j = 5 - q;  // position of t^q's coefficient in (a .. f)
@@ -140,7 +143,7 @@ __global__ void __launch_bounds__(256) coef_kernel(const double *__restrict__ ta
       const double delta = l < g.n0 ? g.stride0 : g.stride1;
       double p = 1.0;
       for (int e = 0; e < q; ++e) p *= delta;
-      v = c * p;
+      v = c * p * scale;
     }
     Cp[x] = v;
   }
@@ -154,11 +157,13 @@ struct RunsParams {
   int nnei, ntypes, nkeys, cap;
   int sel[DP_MAX_TYPES];
   int *map;            // [natoms][nkeys]: run slot of the key, or -1
+  int *keys;           // [natoms][cap]: key of each slot
+  int *nslots;         // [natoms]: slots in use
   double *W;           // forward: [natoms][cap][24] moments W[k][q] at 6 k + q
   int *fexp;           // forward: [Np] exponents of the columns 4 a + k
   unsigned char *occ;  // [ntypes][ntiles][occ_cols]
   int occ_cols;        // forward: K slices; backward: 128-row tiles of the backward A
-  int keys_per_unit;   // keys per flag: 2 (a 16-deep slice) or 16 (128 rows of 8 per key)
+  int unit;            // K entries (rows) per flag: 16 (a slice) or 128 (a tile)
 };
 
 struct alignas(16) RunsStage {
@@ -202,37 +207,44 @@ __device__ __forceinline__ int valid_row(int v, const int *nvb, const int *sel, 
 
 // One warp per atom: the runs of rows sharing an interval (consecutive rows with one key; rows
 // sorted by distance give one run per interval, and a key met again adds to its slot), each
-// interval's slot in the map and its flag for the atom's tile; forward also its moments W and
-// the atom's four column exponents.
+// interval's slot (a shared-memory map of the keys, copied out at the end with each slot's key and
+// the slot count) and its flag for the atom's tile; forward also its moments W and the atom's four
+// column exponents (over every value written, which bounds the final ones).
 template <bool kMom>
 __global__ void __launch_bounds__(32) runs_kernel(const RunsParams P) {
   __shared__ RunsStage st;
+  extern __shared__ short smap[];  // [nkeys]
   const int lane = threadIdx.x;
   const int64_t a = blockIdx.x;
   const int64_t i = P.atom0 + a;
-  int *map = P.map + a * P.nkeys;
-  for (int k = lane; k < P.nkeys; k += 32) map[k] = -1;
-  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the map reset)
+  for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
+  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the reset)
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   unsigned char *occ = P.occ + ((size_t)alpha * P.ntiles + (size_t)(a / kTileAtoms)) * P.occ_cols;
+  int *keys = P.keys + a * P.cap;
   double *Wa = kMom ? P.W + (size_t)a * P.cap * 24 : nullptr;
   int nslot = 0;
   int cur = -1;       // key of the open run (uniform)
   double wv = 0.0;    // its moment W[k][q] on lane 6 k + q < 24
+  int eb = 0;         // largest exponent field written by this lane
   auto flush = [&]() {  // uniform
-    int slot = lane == 0 ? map[cur] : 0;
-    slot = __shfl_sync(0xffffffffu, slot, 0);
+    int slot = smap[cur];
     const bool fresh = slot < 0;
+    __syncwarp();
     if (fresh) {
       slot = nslot++;
       if (lane == 0) {
-        map[cur] = slot;
-        occ[cur / P.keys_per_unit] = 1;
+        smap[cur] = (short)slot;
+        keys[slot] = cur;
+        occ[kQ * cur / P.unit] = 1;  // the key's entries 6 key .. 6 key + 5, in one or two units
+        occ[(kQ * cur + kQ - 1) / P.unit] = 1;
       }
     }
     if (kMom && lane < 24) {
       double *w = Wa + (size_t)slot * 24 + lane;
-      *w = fresh ? wv : *w + wv;
+      const double x = fresh ? wv : *w + wv;
+      *w = x;
+      eb = max(eb, exp_bits(x));
     }
     __syncwarp();
   };
@@ -286,19 +298,18 @@ __global__ void __launch_bounds__(32) runs_kernel(const RunsParams P) {
     __syncwarp();
   }
   if (cur >= 0) flush();
+  int *map = P.map + a * P.nkeys;
+  for (int k = lane; k < P.nkeys; k += 32) map[k] = smap[k];
+  if (lane == 0) P.nslots[a] = nslot;
   if constexpr (kMom) {
-    // column exponents: max over the atom's slots of |W[k][q]|, per k
-    int eb = 0;
-    if (lane < 24)
-      for (int sl = 0; sl < nslot; ++sl) eb = max(eb, exp_bits(Wa[(size_t)sl * 24 + lane]));
-    int m = eb;
+    int m = eb;  // per k: the largest over its six lanes
 #pragma unroll
     for (int q = 1; q < 6; ++q) m = max(m, __shfl_sync(0xffffffffu, eb, min(lane + q, 31)));
     if (lane < 24 && lane % 6 == 0) P.fexp[kCols * a + lane / 6] = exp_of_max(m);
   }
 }
 
-// The forward's B operand: B[8 key + q][4 a + k] = W_a[k][(key, q)] as digit planes with the column
+// The forward's B operand: B[6 key + q][4 a + k] = W_a[k][(key, q)] as digit planes with the column
 // exponents, in split_rows_kernel's block layout (RT = 48), for the slices some atom of the tile
 // uses (any centre type); the other blocks are never read.  One warp per (8 columns, 64 of K).
 __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict__ W, const int *__restrict__ map,
@@ -321,17 +332,17 @@ __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict
   constexpr size_t plane = (size_t)kTN * kTK * 2, block = kS * plane;
   const int ri = (int)(r % kTN);
   unsigned char *rowbase = planes + (size_t)tile * nsl * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
-  const int q0 = 2 * kp;  // this lane's two powers
   for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
     const int sl = k0 / kTK;
     bool used = false;
     for (int t = 0; t < ntypes; ++t) used |= occ[((size_t)t * ntiles + tile) * nsl + sl] != 0;
     if (!used) continue;  // uniform
-    const int key = k0 >> 3;
+    const int kk = k0 + 2 * kp;  // this lane's two entries, of one key (6 is even)
+    const int key = kk / kQ, q0 = kk - kQ * key;
     const int slot = (a < natoms && key < nkeys) ? map[a * nkeys + key] : -1;
     const double *wp = W + ((size_t)a * cap + (slot >= 0 ? slot : 0)) * 24 + 6 * k;
-    const double x0 = (slot >= 0 && q0 < 6) ? wp[q0] : 0.0;
-    const double x1 = (slot >= 0 && q0 + 1 < 6) ? wp[q0 + 1] : 0.0;
+    const double x0 = slot >= 0 ? wp[q0] : 0.0;
+    const double x1 = slot >= 0 ? wp[q0 + 1] : 0.0;
     uint32_t h[kS];
     digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
     unsigned char *dst = rowbase + (size_t)sl * block + ((k0 % kTK) >> 3) * kLBO;
@@ -341,36 +352,49 @@ __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict
 }
 
 // T for the atoms of type alpha of one 12-atom tile (one block): the tile's shares (one per
-// kShareSlices used slices) summed, scaled by 2^(E_m + F_(a,k)) and by 1/N_c.
+// kShareSlices used slices) summed and scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at
+// a time: read with the columns fastest (the shares' rows), written with the channels fastest (T's).
 __global__ void __launch_bounds__(256) fwd_epilogue_kernel(const float4 *__restrict__ part, int Mp, int64_t Np,
                                                            const int *__restrict__ eexp,
                                                            const int *__restrict__ fexp,
                                                            const unsigned char *__restrict__ occ, int nsl,
                                                            int64_t natoms, int64_t atom0,
                                                            const int32_t *__restrict__ atype, int ntypes, int alpha,
-                                                           int M1, double inv_nnei, double *__restrict__ T) {
+                                                           int M1, double *__restrict__ T) {
   __shared__ int nused;
+  __shared__ double tile_out[kTN][33];
+  __shared__ bool wanted[kTileAtoms];
   const int64_t tile = blockIdx.x;
   if (threadIdx.x == 0) nused = 0;
+  if (threadIdx.x < kTileAtoms) {
+    const int64_t a = tile * kTileAtoms + threadIdx.x;
+    wanted[threadIdx.x] = a < natoms && (!atype || clampi(atype[atom0 + a], 0, ntypes - 1) == alpha);
+  }
   __syncthreads();
   int c = 0;
   for (int x = threadIdx.x; x < nsl; x += blockDim.x) c += occ[tile * nsl + x] != 0;
   if (c) atomicAdd(&nused, c);
   __syncthreads();
   const int nz = (nused + kShareSlices - 1) / kShareSlices;
-  for (int e = threadIdx.x; e < kTN * M1; e += blockDim.x) {
-    const int col = e % kTN, m = e / kTN;  // columns fastest: the shares' reads coalesce
-    const int64_t n = tile * kTN + col, a = n >> 2;
-    const int k = (int)(n & 3);
-    if (a >= natoms) continue;
-    if (atype && clampi(atype[atom0 + a], 0, ntypes - 1) != alpha) continue;
-    double v = 0.0;  // an atom of a tile without used slices has no valid rows
-    if (nz > 0) {
-      Sum3 acc;
-      for (int z = 0; z < nz; ++z) acc.add(part[((size_t)z * Mp + m) * Np + n]);
-      v = acc.value(eexp[m], fexp[n]) * inv_nnei;
+  for (int m0 = 0; m0 < M1; m0 += 32) {
+    for (int e = threadIdx.x; e < kTN * 32; e += blockDim.x) {
+      const int col = e % kTN, m = m0 + e / kTN;
+      const int64_t n = tile * kTN + col;
+      double v = 0.0;  // an atom of a tile without used slices has no valid rows
+      if (m < M1 && wanted[col >> 2] && nz > 0) {
+        Sum3 acc;
+        for (int z = 0; z < nz; ++z) acc.add(part[((size_t)z * Mp + m) * Np + n]);
+        v = acc.value(eexp[m], fexp[n]);
+      }
+      tile_out[col][e / kTN] = v;
     }
-    T[((atom0 + a) * kCols + k) * M1 + m] = v;
+    __syncthreads();
+    for (int e = threadIdx.x; e < kTN * 32; e += blockDim.x) {
+      const int col = e >> 5, m = m0 + (e & 31);
+      const int64_t a = tile * kTileAtoms + (col >> 2);
+      if (m < M1 && wanted[col >> 2]) T[((atom0 + a) * kCols + (col & 3)) * M1 + m] = tile_out[col][e & 31];
+    }
+    __syncthreads();
   }
 }
 
@@ -381,12 +405,12 @@ struct RowsParams {
   int64_t atom0;
   int nnei, ntypes, nkeys, cap;
   int sel[DP_MAX_TYPES];
-  const int *map;
-  const float4 *dW;    // [natoms][cap][24]: the backward GEMM's result per run slot (four floats)
+  const int *map, *keys, *nslots;
+  float4 *dW;          // [natoms][cap][24]: the backward GEMM's result per slot (four floats), then in place
+                       // (dW, q dW / Delta) as two doubles
   const int *eexp;     // [ntypes][Mpb]: exponents of the backward A's rows 8 key + q
   int Mpb;
   const int *fexp;     // [Np]: exponents of dT's rows 4 a + k
-  double inv_nnei;
   double *ds, *dRt;
 };
 
@@ -395,27 +419,45 @@ struct alignas(16) RowsStage {
   double u[32];
   double dw[32][24];   // per run of the batch: dW[k][q] at 6 k + q
   double dwq[32][24];  // q dW[k][q] / Delta_l
-  int key[32], run[32], clamped[32], row[32];
+  int slot[32], run[32], clamped[32], row[32], rslot[32];
   int nvb[DP_MAX_TYPES];
 };
 
-// One warp per atom: each run's dW finished from the GEMM's four floats (lanes 6 k + q), then
-// each valid row's dE/dR~ and dE/ds by Horner's rule in u (a lane per row); padded rows get zeros.
+// One warp per atom: every slot's dW finished from the GEMM's four floats (all lanes, in place),
+// then per 32-row batch the batch's runs copied to shared memory and each valid row's dE/dR~ and
+// dE/ds by Horner's rule in u (a lane per row); padded rows get zeros.
 __global__ void __launch_bounds__(32) rows_kernel(const RowsParams P) {
   __shared__ RowsStage st;
+  extern __shared__ short smap[];  // [nkeys]
   const int lane = threadIdx.x;
   const int64_t a = blockIdx.x;
   const int64_t i = P.atom0 + a;
+  const int *gmap = P.map + a * P.nkeys;
+  for (int k = lane; k < P.nkeys; k += 32) smap[k] = (short)gmap[k];
   const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
-  const int *map = P.map + a * P.nkeys;
   const int *eexp = P.eexp + (size_t)alpha * P.Mpb;
+  const int *keys = P.keys + a * P.cap;
+  float4 *dWa = P.dW + (size_t)a * P.cap * 24;
+  double2 *dWd = reinterpret_cast<double2 *>(dWa);
+  const int nslot = P.nslots[a];
+  for (int x = lane; x < nslot * 24; x += 32) {
+    const int sl = x / 24, j = x - 24 * sl, k = j / 6, q = j - 6 * k;
+    const int key = keys[sl];
+    const int l = key % P.g.nint;
+    Sum3 acc;
+    acc.add(dWa[x]);
+    const double d = acc.value(eexp[key * kQ + q], P.fexp[kCols * a + k]);
+    dWd[x] = make_double2(d, d * ((double)q * (l < P.g.n0 ? P.g.inv0 : P.g.inv1)));
+  }
+  __syncwarp();
   const double *srow = P.s + i * P.nnei;
   const double *Rrow = P.Rt + i * P.nnei * 4;
   double *dsrow = P.ds + i * P.nnei;
   double *drow = P.dRt + i * P.nnei * 4;
   for (int base = 0; base < nv; base += 32) {
     const int v = base + lane;
+    int mykey = -1;
     if (v < nv) {
       int b;
       const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
@@ -428,33 +470,24 @@ __global__ void __launch_bounds__(32) rows_kernel(const RowsParams P) {
       st.r[lane][2] = rr.z;
       st.r[lane][3] = rr.w;
       st.u[lane] = t * (l < P.g.n0 ? P.g.inv0 : P.g.inv1);
-      st.key[lane] = b * P.g.nint + l;
+      mykey = b * P.g.nint + l;
       st.clamped[lane] = clamped;
       st.row[lane] = row;
     }
-    __syncwarp();
     const int cnt = min(32, nv - base);
-    const int mykey = lane < cnt ? st.key[lane] : -1;
     const int prev = __shfl_up_sync(0xffffffffu, mykey, 1);
-    unsigned starts = __ballot_sync(0xffffffffu, lane < cnt && (lane == 0 || mykey != prev));
-    int nrun = 0;
-    while (starts) {  // uniform, run by run
-      const int u0 = __ffs(starts) - 1;
-      starts &= starts - 1;
-      const int e = starts ? __ffs(starts) - 1 : cnt;
-      const int key = __shfl_sync(0xffffffffu, mykey, u0);
-      if (lane < 24) {
-        const int k = lane / 6, q = lane - 6 * (lane / 6);
-        const int slot = map[key];
-        Sum3 acc;
-        acc.add(P.dW[((size_t)a * P.cap + slot) * 24 + lane]);
-        const double d = acc.value(eexp[key * kQ + q], P.fexp[kCols * a + k]) * P.inv_nnei;
-        const int l = key % P.g.nint;
-        st.dw[nrun][lane] = d;
-        st.dwq[nrun][lane] = (double)q * d * (l < P.g.n0 ? P.g.inv0 : P.g.inv1);
-      }
-      if (lane >= u0 && lane < e) st.run[lane] = nrun;
-      ++nrun;
+    const bool start = lane < cnt && (lane == 0 || mykey != prev);
+    const unsigned starts = __ballot_sync(0xffffffffu, start);
+    const int nrun = __popc(starts);
+    const int myrun = __popc(starts & (0xffffffffu >> (31 - lane))) - 1;  // runs starting at lanes <= this one
+    if (lane < cnt) st.run[lane] = myrun;
+    if (start) st.rslot[myrun] = smap[mykey];
+    __syncwarp();
+    for (int x = lane; x < nrun * 24; x += 32) {
+      const int r = x / 24, j = x - 24 * r;
+      const double2 w = dWd[(size_t)st.rslot[r] * 24 + j];
+      st.dw[r][j] = w.x;
+      st.dwq[r][j] = w.y;
     }
     __syncwarp();
     if (lane < cnt) {
@@ -502,11 +535,11 @@ int check_work(const Layout &L, const void *work, size_t nbytes, const char *who
 // C' of every centre type from the table, then its digit planes: forward A = C'^T (rows: the
 // channels, K: 8 key + q), backward A = C' (rows: 8 key + q, K: the channels).
 int prep(const double *table, const TableGeom &g, const Shape &s, const Layout &L, unsigned char *wk, bool fwd,
-         cudaStream_t st, const char *who) {
+         int nnei, cudaStream_t st, const char *who) {
   double *Cp = reinterpret_cast<double *>(wk + L.cp);
   const int64_t total = (int64_t)s.ntypes * s.Kp * s.M1;
   coef_kernel<<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(table, g, s.ntypes, s.M1,
-                                                                                          s.Kp, Cp);
+                                                                                          s.Kp, 1.0 / (double)nnei, Cp);
   int rc = launch_status(who);
   for (int t = 0; t < s.ntypes && !rc; ++t) {
     const double *Ct = Cp + (size_t)t * s.Kp * s.M1;
@@ -533,6 +566,8 @@ RunsParams runs_params(const double *s, const double *Rt, const int32_t *nvalid,
   R.cap = S.cap;
   for (int b = 0; b < DP_MAX_TYPES; ++b) R.sel[b] = seg.sel[b];
   R.map = reinterpret_cast<int *>(wk + L.map);
+  R.keys = reinterpret_cast<int *>(wk + L.keys);
+  R.nslots = reinterpret_cast<int *>(wk + L.nslots);
   R.occ = wk + L.occ;
   R.fexp = reinterpret_cast<int *>(wk + L.fexp);
   return R;
@@ -548,16 +583,19 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
   int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, T, &g, &seg);
   if (rc) return rc;
   if (nloc == 0) return DP_OK;
+  if ((int64_t)ntypes * g.nint > kMaxKeys)
+    return set_error(DP_ERR_UNSUPPORTED, "%s: ntypes x nint = %lld intervals per centre type, at most %d", who,
+                     (long long)ntypes * g.nint, kMaxKeys);
   const Shape S = make_shape(g, nloc, nnei, ntypes, M1);
   const Layout L = make_layout(S);
   if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
-  if ((rc = prep(table, g, S, L, wk, true, st, who))) return rc;
+  if ((rc = prep(table, g, S, L, wk, true, nnei, st, who))) return rc;
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
   R.W = reinterpret_cast<double *>(wk + L.w);
   R.occ_cols = S.nsl;
-  R.keys_per_unit = kTK / kQ;
+  R.unit = kTK;
   float4 *part = reinterpret_cast<float4 *>(wk + L.part);
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
     const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
@@ -568,7 +606,7 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
     R.atom0 = c0;
     R.natoms = n;
     R.ntiles = ntiles;
-    runs_kernel<true><<<(unsigned)n, 32, 0, st>>>(R);
+    runs_kernel<true><<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     const int64_t warps = Np / 8 * ((S.Kp + kSplitK - 1) / kSplitK);
     split_mom_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(R.W, R.map, R.fexp, wk + L.occ, ntypes, ntiles, n,
@@ -590,7 +628,7 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
       gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
       if ((rc = launch_status(who))) return rc;
       fwd_epilogue_kernel<<<(unsigned)ntiles, 256, 0, st>>>(part, S.Mpf, Np, G.Eexp, R.fexp, G.kocc, S.nsl, n, c0,
-                                                            atype, ntypes, t, M1, 1.0 / (double)nnei, T);
+                                                            atype, ntypes, t, M1, T);
       if ((rc = launch_status(who))) return rc;
     }
   }
@@ -608,16 +646,19 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
   if (rc) return rc;
   if (nloc > 0 && !dT) return set_error(DP_ERR_NULL, "%s: dT is NULL", who);
   if (nloc == 0) return DP_OK;
+  if ((int64_t)ntypes * g.nint > kMaxKeys)
+    return set_error(DP_ERR_UNSUPPORTED, "%s: ntypes x nint = %lld intervals per centre type, at most %d", who,
+                     (long long)ntypes * g.nint, kMaxKeys);
   const Shape S = make_shape(g, nloc, nnei, ntypes, M1);
   const Layout L = make_layout(S);
   if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
-  if ((rc = prep(table, g, S, L, wk, false, st, who))) return rc;
+  if ((rc = prep(table, g, S, L, wk, false, nnei, st, who))) return rc;
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
   const int mtiles = S.Mpb / kTM;
   R.occ_cols = mtiles;
-  R.keys_per_unit = kTM / kQ;
+  R.unit = kTM;
   float4 *dW = reinterpret_cast<float4 *>(wk + L.w);
   RowsParams Q{};
   Q.s = s;
@@ -631,11 +672,12 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
   Q.cap = S.cap;
   for (int b = 0; b < DP_MAX_TYPES; ++b) Q.sel[b] = seg.sel[b];
   Q.map = R.map;
+  Q.keys = R.keys;
+  Q.nslots = R.nslots;
   Q.dW = dW;
   Q.eexp = reinterpret_cast<const int *>(wk + L.ebwd);
   Q.Mpb = S.Mpb;
   Q.fexp = R.fexp;
-  Q.inv_nnei = 1.0 / (double)nnei;
   Q.ds = ds;
   Q.dRt = dRt;
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
@@ -647,7 +689,7 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
     R.atom0 = c0;
     R.natoms = n;
     R.ntiles = ntiles;
-    runs_kernel<false><<<(unsigned)n, 32, 0, st>>>(R);
+    runs_kernel<false><<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
     if ((rc = split_rows(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, Np, S.Kpm, kTN, wk + L.bplanes, wk + L.fexp, st,
@@ -673,12 +715,13 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
       G.cap = S.cap;
       G.alpha = t;
       G.ntypes = ntypes;
+      G.kq = kQ;
       const dim3 grid((unsigned)ntiles, (unsigned)mtiles, 1);
       gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
       if ((rc = launch_status(who))) return rc;
     }
     Q.atom0 = c0;
-    rows_kernel<<<(unsigned)n, 32, 0, st>>>(Q);
+    rows_kernel<<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(Q);
     if ((rc = launch_status(who))) return rc;
   }
   return DP_OK;
@@ -688,9 +731,10 @@ size_t work_bytes_api(const dp_table_info *info, int64_t nloc, int nnei, int nty
   clear_error();
   TableGeom g;
   if (make_geom(info, &g)) return 0;
-  if (nloc < 0 || nnei < 1 || ntypes < 1 || ntypes > DP_MAX_TYPES || M1 < 1 || M1 > DP_MAX_M1) {
-    set_error(DP_ERR_SHAPE, "dp_tabulate_tc_work_bytes: nloc %lld, nnei %d, ntypes %d, M1 %d out of range",
-              (long long)nloc, nnei, ntypes, M1);
+  if (nloc < 0 || nnei < 1 || ntypes < 1 || ntypes > DP_MAX_TYPES || M1 < 1 || M1 > DP_MAX_M1 ||
+      (int64_t)ntypes * g.nint > kMaxKeys) {
+    set_error(DP_ERR_SHAPE, "dp_tabulate_tc_work_bytes: nloc %lld, nnei %d, ntypes %d, M1 %d (%d intervals) out of range",
+              (long long)nloc, nnei, ntypes, M1, g.nint);
     return 0;
   }
   return make_layout(make_shape(g, nloc, nnei, ntypes, M1)).total;

@@ -69,7 +69,8 @@ constexpr int kStageBytes = kS * (kPlaneA + kPlaneB);
 constexpr uint32_t kTmemCols = 512;  // allocation (a power of two); kS * kTN = 432 used
 constexpr int kMaxShareSlices = kMaxShareK / kTK;
 constexpr size_t kSmemTail = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16;  // used-slice list
-constexpr size_t kSmemTotal = kSmemTail + (kMaxShareSlices + 1) * 4;
+constexpr int kScatKeys = kTM / 4 + 1, kScatAtoms = kTN / 4;  // scatter: keys (kq >= 4) and atoms of a tile
+constexpr size_t kSmemTotal = kSmemTail + (kMaxShareSlices + 1) * 4 + kScatKeys * kScatAtoms * 4;
 static_assert((size_t)kS * kMaxShareK * 63 * 63 < (1u << 24), "fp32 diagonal sums must stay exact");
 static_assert(kMaxShareK % kTK == 0 && kS * kTN <= (int)kTmemCols, "shares and TMEM");
 static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
@@ -186,14 +187,14 @@ struct TcGemm {
                               // slice; share z of a tile then takes its used slices z S .. z S + S - 1
                               // (S = slices_per_split), and a share past its last used slice writes nothing
   const unsigned char *tocc;  // [Np / kTN][Mp / kTM]: nonzero where the output tile is wanted
-  // scatter (with tocc): output (row 8 key + q, column 4 a + k), q < 6, key < nkeys, a < natoms, goes to
-  // scat[(a cap + slot) 24 + 6 k + q] when slot = map[a nkeys + key] >= 0 and atom atom0 + a has type
-  // alpha (atype clamped into [0, ntypes)); nothing is written to part
+  // scatter (with tocc): output (row kq key + q, column 4 a + k), q < 6 <= kq, key < nkeys, a < natoms,
+  // goes to scat[(a cap + slot) 24 + 6 k + q] when slot = map[a nkeys + key] >= 0 and atom atom0 + a
+  // has type alpha (atype clamped into [0, ntypes)); nothing is written to part
   float4 *scat;
   const int *map;
   const int32_t *atype;
   int64_t natoms, atom0;
-  int nkeys, cap, alpha, ntypes;
+  int nkeys, cap, alpha, ntypes, kq;
   bool skip;
   // forward
   const double *bias;
@@ -243,12 +244,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(done + 1);
   int *flags = reinterpret_cast<int *>(tmem_holder + 1);                          // producer / issuer ok
   int *slist = reinterpret_cast<int *>(smem + kSmemTail);                         // used slices, then their count
+  int *stab = slist + kMaxShareSlices + 1;  // scatter: slot of (key, atom) of the tile, or -1
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t m0 = (int64_t)blockIdx.y * kTM;
   const int n0 = blockIdx.x * kTN;
   const int nslices = P.Kp / kTK;
   const int i0 = blockIdx.z * P.slices_per_split;
   if (P.tocc && !P.tocc[(size_t)blockIdx.x * gridDim.y + blockIdx.y]) return;  // unwanted tile (uniform)
+  if (P.scat)  // the tile's slots, loaded once and in parallel
+    for (int x = tid; x < kScatKeys * kScatAtoms; x += kThreads) {
+      const int key = (int)(m0 / P.kq) + x / kScatAtoms;
+      const int64_t a = (int64_t)(n0 / 4) + x % kScatAtoms;
+      int slot = -1;
+      if (key < P.nkeys && a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha))
+        slot = P.map[a * P.nkeys + key];
+      stab[x] = slot;
+    }
   int nsl = min(nslices - i0, P.slices_per_split);  // dense: > 0, no empty share
   if (P.kocc) {
     // this share's used slices, in order, by a ballot over the tile's flags
@@ -360,7 +371,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   // third of the columns, 8 at a time
   const int rl = 32 * (warp & 3) + lane;
   float4 *outp = P.scat ? nullptr : P.part + ((size_t)blockIdx.z * P.Mp + m0 + rl) * P.Np + n0;
-  const int key = (int)((m0 + rl) >> 3), q = (int)((m0 + rl) & 7);  // scatter: this thread's row
+  const int key = P.scat ? (int)((m0 + rl) / P.kq) : 0, q = P.scat ? (int)(m0 + rl - (int64_t)key * P.kq) : 0;
+  const int key_l = P.scat ? key - (int)(m0 / P.kq) : 0;  // this thread's row's key, in the tile
   const bool row_wanted = P.scat && q < 6 && key < P.nkeys;
   const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
   constexpr int kColsPerWarp = kTN / (kThreads / 128);
@@ -393,12 +405,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
       if (outp) {
         outp[c0 + c] = val;
       } else if (row_wanted) {
-        const int64_t a = (int64_t)(n0 + c0 + c) >> 2;
-        const int k = (n0 + c0 + c) & 3;
-        if (a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha)) {
-          const int slot = P.map[a * P.nkeys + key];
-          if (slot >= 0) P.scat[((size_t)a * P.cap + slot) * 24 + 6 * k + q] = val;
-        }
+        const int al = (c0 + c) >> 2, k = (c0 + c) & 3;  // the tile's atom, its column k
+        const int slot = stab[key_l * kScatAtoms + al];
+        if (slot >= 0) P.scat[((size_t)((n0 >> 2) + al) * P.cap + slot) * 24 + 6 * k + q] = val;
       }
     }
   }
