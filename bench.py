@@ -6,9 +6,12 @@ D = S S<^T (dp_descriptor_contract) and the backward from a given dE/dT
 (dp_tabulate_fusion_grad).  The table build (compression) is setup and is
 not timed.  Metric: valid neighbour x channel evaluations per second for
 fwd + grad (each valid (atom, neighbour, channel) triple counts once).
---algo moments (default) runs the interval-moment forward and backward,
---algo direct the per-row ones; both give the same outputs, and the
-roofline fraction is taken on the FMAs of the algorithm that ran.
+--algo tc (the default in f64) runs the interval moments with their
+per-interval contraction on the tensor cores (f64 by exact digit
+splitting), --algo moments (the default in f32 and df64) the interval
+moments on the FMA pipes, --algo direct the per-row kernels; all give the
+same outputs, and the roofline fraction is taken on the dominant kernel
+of the path that ran (inside the tc calls: the events they record).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload cu85] [--dtype f64]
   python bench.py --impl reference ...   # the oracle on the host cores (bounded sample)
@@ -139,6 +142,26 @@ def interval_runs(w, info, n0: int, n1: int):
     return np.diff(np.concatenate([starts, [k.size]]))
 
 
+# --algo tc: algorithmic FMAs of its kernels, per valid row (FP64 pipe) or per run x M1 (the
+# per-interval contraction on the tensor cores, each FMA as 45 fp16 digit products):
+#   tc_runs_moments  W[k][q] += R~_k u^q                 24 per row
+#   tc_rows          dE/dR~ and dE/ds by Horner in u     40 per row (20 + 16 + 4)
+#   tc_gemm_fwd      T += W C' per run                    24 M1 per run
+#   tc_gemm_grad     dW = dT C'^T per run                 24 M1 per run
+TC_FMA = {"tc_runs_moments": ("row", 24), "tc_rows": ("row", 40), "tc_gemm_fwd": ("run", 24),
+          "tc_gemm_grad": ("run", 24)}
+TC_KERNEL = {"tc_runs_moments": "runs_kernel<moments> (dp_tabulate_fusion_fwd_tc_f64)",
+             "tc_rows": "rows_kernel (dp_tabulate_fusion_grad_tc_f64)",
+             "tc_gemm_fwd": "gemm_kernel (dp_tabulate_fusion_fwd_tc_f64)",
+             "tc_gemm_grad": "gemm_kernel (dp_tabulate_fusion_grad_tc_f64)"}
+TC_PROFILE_EVENTS = 64  # per step: the tc calls record one after each of their kernels
+
+
+def tc_fmas(w, runs) -> dict:
+    rows = float(w.evals) / w.M1
+    return {k: (n * rows if per == "row" else n * w.M1 * float(len(runs))) for k, (per, n) in TC_FMA.items()}
+
+
 def moment_fmas(runs, M1: int) -> dict:
     out = {}
     for kern, (per_row, per_run, per_row_m) in MOMENT_FMA.items():
@@ -149,7 +172,8 @@ def moment_fmas(runs, M1: int) -> dict:
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
 # `ncu --set full` capture of its current version (profiles/<kernel>_<algo>_<workload>_<dtype>.md);
 # absent means no capture of the current kernel exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640}
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,
+                       ("cu85", "f64", "tc_rows", "tc"): 140421632 + 95273984}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
@@ -407,6 +431,11 @@ def run_native(args, rank, world, local_rank):
             torch.distributed.barrier()
 
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
+    pev, pnames = None, []
+    if args.algo == "tc":  # per-kernel times inside the tc calls, from events they record themselves
+        pev = [[torch.cuda.Event(enable_timing=True) for _ in range(TC_PROFILE_EVENTS)] for _ in range(args.steps)]
+        for e in (e for row in pev for e in row):
+            e.record(stream)  # creates the CUDA events before the timed region
     vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
     clocks = ClockSampler(vis[local_rank] if local_rank < len(vis) else str(local_rank))
     barrier()
@@ -416,7 +445,11 @@ def run_native(args, rank, world, local_rank):
     t_wall0 = time.perf_counter()
     for k in range(args.steps):
         flush.zero_()  # evict the previous step's data from L2 (outside the timed events)
+        if pev:
+            dpc.dp_profile_begin(pev[k])
         run_step(evs[k])
+        if pev:
+            pnames.append(dpc.dp_profile_end())
     torch.cuda.synchronize(dev)
     t_wall = time.perf_counter() - t_wall0
     barrier()
@@ -424,6 +457,13 @@ def run_native(args, rank, world, local_rank):
 
     step_ms = [e[0].elapsed_time(e[nk]) for e in evs]
     k_ms = {n: [e[j].elapsed_time(e[j + 1]) for e in evs] for j, n in enumerate(names)}
+    tc_ms = None
+    if pev:
+        tc_ms = {}
+        for k, nm in enumerate(pnames):
+            for i in range(1, len(nm)):
+                if nm[i] not in ("tc_fwd", "tc_grad"):  # a call's start closes nothing
+                    tc_ms.setdefault(nm[i], [0.0] * args.steps)[k] += pev[k][i - 1].elapsed_time(pev[k][i])
     total_s, evals_all = reduce_over_ranks(sum(step_ms) / 1e3, float(w.evals), world, dev)
 
     # ---- the same step captured once as a CUDA graph (the chain's many launches in one)
@@ -438,11 +478,15 @@ def run_native(args, rank, world, local_rank):
     if args.algo in ("moments", "tc"):
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
     nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
-    out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall)
+    tcf = tc_fmas(w, interval_runs(w, info, *dpc.dp_table_info_sizes(info))) if tc_ms else None
+    per_mark = {"tc_coef_split": 1 + 2 * w.ntypes, "tc_split_dT": 2, "tc_fwd": 0, "tc_grad": 0}  # kernels per mark
+    out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall, tc_ms, tcf,
+                 [sum(per_mark.get(x, 1) for x in nm) for nm in pnames])
     if graph is not None:
         graph["evals_per_s"] = w.evals / (graph["ms_per_step"] * 1e-3)
         out["graph"] = graph
-    if world == 1 and not args.no_variants and not args.chain and args.dtype == "f64" and args.algo == "moments":
+    if world == 1 and not args.no_variants and not args.chain and args.dtype == "f64" and args.algo in ("moments",
+                                                                                                         "tc"):
         out["variants"] = measure_variants(args, w, dpc, info, sel, d, outs, flush, stream, dev, fmas)
     return out
 
@@ -487,10 +531,13 @@ def measure_variants(args, w, dpc, info, sel, d, ref_outs, flush, stream, dev, f
     model_64 = dpc.Model.compress(torch.from_numpy(w.params).to(dev), w.widths, info, torch.float64)
     nsteps = max(3, min(args.steps, 100))
     res = {}
-    for name, model, fwd, grad, arith in (
-            ("f64_per_row", model_64, dpc.dp_tabulate_fusion_fwd, dpc.dp_tabulate_fusion_grad, None),
+    todo = [("f64_per_row", model_64, dpc.dp_tabulate_fusion_fwd, dpc.dp_tabulate_fusion_grad, None),
             ("df64_moments", model_df, dpc.dp_tabulate_fusion_fwd_moments, dpc.dp_tabulate_fusion_grad_moments,
-             dpc.DF64)):
+             dpc.DF64)]
+    if args.algo == "tc":
+        todo.insert(0, ("f64_moments", model_64, dpc.dp_tabulate_fusion_fwd_moments,
+                        dpc.dp_tabulate_fusion_grad_moments, None))
+    for name, model, fwd, grad, arith in todo:
         o = {k: torch.empty_like(v) for k, v in ref_outs.items()}
 
         def step(rec):
@@ -512,7 +559,8 @@ def measure_variants(args, w, dpc, info, sel, d, ref_outs, flush, stream, dev, f
         ms = {n: sum(e[j].elapsed_time(e[j + 1]) for e in evs) / nsteps for j, n in enumerate(("fwd", "descriptor", "grad"))}
         tot = sum(ms.values())
         pk = peak_tflops("df64" if arith else "f64")
-        fm = fmas if arith else {"fwd": FMA_PER_EVAL["fwd"] * w.evals, "grad": FMA_PER_EVAL["grad"] * w.evals}
+        fm = fmas if name.endswith("moments") else {"fwd": FMA_PER_EVAL["fwd"] * w.evals,
+                                                     "grad": FMA_PER_EVAL["grad"] * w.evals}
         diff = {k: float(((o[k] - ref_outs[k]).abs().max() / ref_outs[k].abs().max()).item()) for k in ref_outs}
         res[name] = {"value": w.evals / (tot * 1e-3), "unit": UNIT, "ms_per_step": round(tot, 4), "steps": nsteps,
                      "dtype": "df64" if arith else "f64",
@@ -585,7 +633,8 @@ def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_al
             "d2h_bytes_per_step": d2h, "pipelined": "double-buffered, uploads and downloads on their own streams"}
 
 
-def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas=None, nall=0):
+def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas=None, nall=0, tc_ms=None,
+           tcf=None, tc_launches=None):
     value = evals_all * args.steps / total_s
     # ---- roofline of the dominant kernel (FMA pipe of the path's dtype), on the FMAs of the
     # algorithm the kernels run: per-row evaluation, or interval moments (fmas, from the run lengths)
@@ -625,6 +674,32 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         roofline.update({"bound": "tensor", "achieved": kernels[dom]["tensor_tflops"], "peak": round(tpk, 1),
                          "frac": kernels[dom]["tensor_frac"], "traffic": None,
                          "peak_basis": f"{tbasis}; achieved counts all {TC_DIGIT_PRODUCTS} fp16 digit products"})
+    if tc_ms:  # the tensor-core tabulation: its own kernels, timed by the events its calls record
+        step_mean = sum(step_ms) / len(step_ms)
+        tmean = {k: sum(v) / len(v) for k, v in tc_ms.items()}
+        for k, ms in tmean.items():
+            e = {"ms": round(ms, 4), "share": round(ms / step_mean, 4)}
+            if k in tcf:
+                e["tflops"] = round(2.0 * tcf[k] / (ms * 1e-3) / 1e12, 4)  # FP64 (equivalent) flop
+                if k.startswith("tc_gemm"):
+                    e["tensor_tflops"] = round(TC_DIGIT_PRODUCTS * e["tflops"], 2)
+                    e["tensor_frac"] = round(e["tensor_tflops"] / tpk, 4)
+                else:
+                    e["frac"] = round(e["tflops"] / pk, 4)
+            kernels[k] = e
+        dom = max(tmean, key=tmean.get)
+        if dom in tcf:
+            e = kernels[dom]
+            gemm = dom.startswith("tc_gemm")
+            roofline = {"bound": "tensor" if gemm else "alu",
+                        "achieved": e["tensor_tflops"] if gemm else e["tflops"],
+                        "peak": round(tpk, 1) if gemm else round(pk, 4), "unit": "TFLOP/s",
+                        "frac": e["tensor_frac"] if gemm else e["frac"],
+                        "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
+                        "kernel": TC_KERNEL[dom],
+                        "peak_basis": (f"{tbasis}; achieved counts all {TC_DIGIT_PRODUCTS} fp16 digit products"
+                                       if gemm else peak_basis(args.dtype)),
+                        "fwd_grad_frac_fp64_equivalent": round(path_tflops / pk, 4)}
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sum(step_ms) / len(step_ms), "higher_is_better": True,
@@ -637,8 +712,11 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                             "env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain
                             else "fwd + descriptor + grad"), "algo": args.algo,
                    "fma_basis": ("interval moments: per run min(9 M1 L, 24 M1 + 24 L) fwd, "
-                                 "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo == "moments"
+                                 "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo in ("moments", "tc")
                                  else "per row: 9 M1 fwd, 18 M1 grad"),
+                   **({"tc": ("per-interval contraction on the tensor cores (f64 by exact 9-digit splitting, "
+                              "fp16 MMAs); per-row work on the FP64 pipe: moments 24 FMA, derivatives 40 FMA "
+                              "per valid row")} if args.algo == "tc" else {}),
                    "l2": "flushed between steps (256 MiB write)",
                    **({"fitting_gemm": ("tensor cores (tcgen05): f64 by exact 9-digit splitting, fp16 MMAs"
                                         if tc else "FP64 pipe")} if getattr(args, "fitting", False) else {}),
@@ -648,7 +726,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         "roofline": roofline,
         "kernels": kernels,
         "e2e": e2e,
-        "gpu_launches": len(k_ms) * args.steps * world,
+        # the tc fwd and grad calls count as the kernels they launched (their recorded marks)
+        "gpu_launches": (len(k_ms) * args.steps + (sum(tc_launches) - 2 * args.steps if tc_launches else 0)) * world,
         "clocks": clk,
         "wall_s_timed_region": round(t_wall, 4),
     }
@@ -768,8 +847,10 @@ def main():
     ap.add_argument("--seed", type=int, default=2)
     ap.add_argument("--cpu-seconds", type=float, default=10.0, help="oracle CPU-baseline sample length")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) measurement")
-    ap.add_argument("--algo", choices=["direct", "moments", "tc"], default="moments",
-                    help="direct: per-neighbour evaluation (the paper's fused kernel); moments: interval moments")
+    ap.add_argument("--algo", choices=["direct", "moments", "tc"], default=None,
+                    help="direct: per-neighbour evaluation (the paper's fused kernel); moments: interval moments; "
+                         "tc: interval moments with the per-interval contraction on the tensor cores (f64; the "
+                         "default for f64)")
     ap.add_argument("--scaling", choices=["weak", "strong"], default="weak",
                     help="weak: one instance per rank; strong: one instance split over the ranks")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -786,6 +867,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.algo is None:  # f64: the tensor-core path; f32 and df64: the interval moments
+        args.algo = "tc" if args.dtype == "f64" else "moments"
     if args.dtype == "df64" and args.algo != "moments":
         ap.error("--dtype df64 runs the moment path only")
     if args.algo == "tc" and args.dtype != "f64":

@@ -268,6 +268,23 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  * Extra errors: DP_ERR_NULL / DP_ERR_SHAPE for a missing, short or
  * misaligned work buffer.
  */
+/*
+ * Kernel timing hook, for profiling (off by default; not thread-safe: one
+ * profiling session per process).  dp_profile_begin hands the library n
+ * caller-created cudaEvent_t handles (as void*, created with timing enabled,
+ * owned by the caller); until dp_profile_end, the calls that launch several
+ * kernels (dp_tabulate_fusion_*_tc_f64) record the next event on their
+ * stream when they start and after each of their kernels, so that the time
+ * between consecutive events of one call is one kernel's.  dp_profile_name(i)
+ * names what event i follows ("tc_fwd" / "tc_grad" for a call's start);
+ * recording stops when the n events are used.  dp_profile_end turns the hook
+ * off and returns how many events were recorded.  Errors: DP_ERR_SHAPE (n < 0
+ * or n > 4096), DP_ERR_NULL.
+ */
+int dp_profile_begin(void *const *events, int n);
+int dp_profile_end(void);
+const char *dp_profile_name(int i);
+
 size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nnei, int ntypes,
                                  int M1); /* 0 on bad sizes or table info */
 int dp_tabulate_fusion_fwd_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,

@@ -93,6 +93,9 @@ _SIGS = {
                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_moments_f32": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                              ctypes.c_int, _P, _P, _P, _P], ctypes.c_int),
+    "dp_profile_begin": ([_P, ctypes.c_int], ctypes.c_int),
+    "dp_profile_end": ([], ctypes.c_int),
+    "dp_profile_name": ([ctypes.c_int], ctypes.c_char_p),
     "dp_tabulate_tc_work_bytes": ([_INFO, _I64, ctypes.c_int, ctypes.c_int, ctypes.c_int], ctypes.c_size_t),
     "dp_tabulate_fusion_fwd_tc_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                        ctypes.c_int, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
@@ -332,6 +335,24 @@ def _grad(name, table, info, s, Rt, nvalid, atype, sel, dT, out):
     _check(fn(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes,
               selc, M1, _ptr(dT), _ptr(ds), _ptr(dRt), _stream(s)))
     return ds, dRt
+
+
+def dp_profile_begin(events):
+    """Kernel timing hook: the multi-kernel calls record these torch.cuda.Event objects (timing enabled)
+    after each of their kernels until dp_profile_end(); returns nothing."""
+    handles = []
+    for ev in events:
+        if ev.cuda_event == 0:  # torch creates the CUDA event on its first record
+            ev.record()
+        handles.append(ev.cuda_event)
+    arr = (ctypes.c_void_p * max(len(handles), 1))(*handles)
+    _check(_lib.dp_profile_begin(arr, len(handles)))
+
+
+def dp_profile_end():
+    """Names of what each recorded event follows, in recording order; turns the hook off."""
+    n = int(_lib.dp_profile_end())
+    return [_lib.dp_profile_name(i).decode() for i in range(n)]
 
 
 def dp_tabulate_tc_work_bytes(info: dp_table_info, nloc, nnei, ntypes, M1) -> int:

@@ -18,6 +18,7 @@ using dfl::df64;
 int set_error(int code, const char *fmt, ...);  // stores the message, returns code
 void clear_error();
 int launch_status(const char *what);  // DP_ERR_CUDA if the last launch failed
+void prof_mark(const char *name, cudaStream_t st);  // kernel timing hook (dp_profile_begin)
 
 // --------------------------------------------------------- table geometry
 // dp_table_info with its derived sizes and reciprocal steps.

@@ -28,6 +28,24 @@ int launch_status(const char *what) {
   return DP_OK;
 }
 
+// Kernel timing hook (off unless dp_profile_begin was called): calls that launch several kernels
+// record the caller's events on their stream, one after each kernel, in order, with the kernel's name.
+namespace {
+constexpr int kMaxProfileEvents = 4096;
+struct Profile {
+  cudaEvent_t ev[kMaxProfileEvents];
+  const char *name[kMaxProfileEvents];
+  int n = 0, cap = 0;
+  bool on = false;
+};
+Profile g_prof;
+}  // namespace
+
+void prof_mark(const char *name, cudaStream_t st) {
+  if (!g_prof.on || g_prof.n >= g_prof.cap) return;
+  if (cudaEventRecord(g_prof.ev[g_prof.n], st) == cudaSuccess) g_prof.name[g_prof.n++] = name;
+}
+
 static bool finite(double x) { return std::isfinite(x); }
 
 int make_geom(const dp_table_info *info, TableGeom *g) {
@@ -102,6 +120,28 @@ int check_fusion_args(const void *table, const dp_table_info *info, const void *
 extern "C" {
 
 const char *dp_last_error(void) { return dpc::g_error.c_str(); }
+
+int dp_profile_begin(void *const *events, int n) {
+  dpc::clear_error();
+  if (n < 0 || n > dpc::kMaxProfileEvents)
+    return dpc::set_error(DP_ERR_SHAPE, "dp_profile_begin: n = %d outside [0, %d]", n, dpc::kMaxProfileEvents);
+  if (n > 0 && !events) return dpc::set_error(DP_ERR_NULL, "dp_profile_begin: events is NULL");
+  for (int i = 0; i < n; ++i) {
+    if (!events[i]) return dpc::set_error(DP_ERR_NULL, "dp_profile_begin: events[%d] is NULL", i);
+    dpc::g_prof.ev[i] = static_cast<cudaEvent_t>(events[i]);
+  }
+  dpc::g_prof.n = 0;
+  dpc::g_prof.cap = n;
+  dpc::g_prof.on = n > 0;
+  return DP_OK;
+}
+
+int dp_profile_end(void) {
+  dpc::g_prof.on = false;
+  return dpc::g_prof.n;
+}
+
+const char *dp_profile_name(int i) { return i >= 0 && i < dpc::g_prof.n ? dpc::g_prof.name[i] : ""; }
 
 int dp_table_info_make(double s_min, double s_max, double stride0, double stride1, double ext, dp_table_info *out) {
   dpc::clear_error();

@@ -421,6 +421,7 @@ struct alignas(16) RowsStage {
   double dwq[32][24];  // q dW[k][q] / Delta_l
   int slot[32], run[32], clamped[32], row[32], rslot[32];
   int nvb[DP_MAX_TYPES];
+  double qinv[2][kQ];  // q / Delta on the fine and the coarse grid
 };
 
 // One warp per atom: every slot's dW finished from the GEMM's four floats (all lanes, in place),
@@ -441,6 +442,8 @@ __global__ void __launch_bounds__(32) rows_kernel(const RowsParams P) {
   float4 *dWa = P.dW + (size_t)a * P.cap * 24;
   double2 *dWd = reinterpret_cast<double2 *>(dWa);
   const int nslot = P.nslots[a];
+  if (lane < 2 * kQ) st.qinv[lane / kQ][lane % kQ] = (double)(lane % kQ) * (lane < kQ ? P.g.inv0 : P.g.inv1);
+  __syncwarp();
   for (int x = lane; x < nslot * 24; x += 32) {
     const int sl = x / 24, j = x - 24 * sl, k = j / 6, q = j - 6 * k;
     const int key = keys[sl];
@@ -448,7 +451,7 @@ __global__ void __launch_bounds__(32) rows_kernel(const RowsParams P) {
     Sum3 acc;
     acc.add(dWa[x]);
     const double d = acc.value(eexp[key * kQ + q], P.fexp[kCols * a + k]);
-    dWd[x] = make_double2(d, d * ((double)q * (l < P.g.n0 ? P.g.inv0 : P.g.inv1)));
+    dWd[x] = make_double2(d, d * st.qinv[l < P.g.n0 ? 0 : 1][q]);
   }
   __syncwarp();
   const double *srow = P.s + i * P.nnei;
@@ -591,7 +594,9 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
   if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
+  prof_mark("tc_fwd", st);
   if ((rc = prep(table, g, S, L, wk, true, nnei, st, who))) return rc;
+  prof_mark("tc_coef_split", st);
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
   R.W = reinterpret_cast<double *>(wk + L.w);
   R.occ_cols = S.nsl;
@@ -608,10 +613,12 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
     R.ntiles = ntiles;
     runs_kernel<true><<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_runs_moments", st);
     const int64_t warps = Np / 8 * ((S.Kp + kSplitK - 1) / kSplitK);
     split_mom_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(R.W, R.map, R.fexp, wk + L.occ, ntypes, ntiles, n,
                                                                    S.nkeys, S.cap, Np, S.Kp, wk + L.bplanes);
     if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_split_moments", st);
     for (int t = 0; t < ntypes; ++t) {
       TcGemm G{};
       G.aplanes = wk + L.afwd + (size_t)t * kS * S.Mpf * S.Kp * 2;
@@ -627,9 +634,11 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
       const dim3 grid((unsigned)ntiles, (unsigned)(S.Mpf / kTM), (unsigned)S.zmax);
       gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
       if ((rc = launch_status(who))) return rc;
+      prof_mark("tc_gemm_fwd", st);
       fwd_epilogue_kernel<<<(unsigned)ntiles, 256, 0, st>>>(part, S.Mpf, Np, G.Eexp, R.fexp, G.kocc, S.nsl, n, c0,
                                                             atype, ntypes, t, M1, T);
       if ((rc = launch_status(who))) return rc;
+      prof_mark("tc_epilogue_fwd", st);
     }
   }
   return DP_OK;
@@ -654,7 +663,9 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
   if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
+  prof_mark("tc_grad", st);
   if ((rc = prep(table, g, S, L, wk, false, nnei, st, who))) return rc;
+  prof_mark("tc_coef_split", st);
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
   const int mtiles = S.Mpb / kTM;
   R.occ_cols = mtiles;
@@ -691,10 +702,12 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
     R.ntiles = ntiles;
     runs_kernel<false><<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_runs", st);
     // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
     if ((rc = split_rows(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, Np, S.Kpm, kTN, wk + L.bplanes, wk + L.fexp, st,
                          who)))
       return rc;
+    prof_mark("tc_split_dT", st);
     for (int t = 0; t < ntypes; ++t) {
       TcGemm G{};
       G.aplanes = wk + L.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
@@ -719,10 +732,12 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
       const dim3 grid((unsigned)ntiles, (unsigned)mtiles, 1);
       gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
       if ((rc = launch_status(who))) return rc;
+      prof_mark("tc_gemm_grad", st);
     }
     Q.atom0 = c0;
     rows_kernel<<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(Q);
     if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_rows", st);
   }
   return DP_OK;
 }
