@@ -266,7 +266,9 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  *                     partial results, for chunks of at most 4104 atoms.
  *                     Calls sharing a work buffer must not overlap on the GPU.
  * Extra errors: DP_ERR_NULL / DP_ERR_SHAPE for a missing, short or
- * misaligned work buffer.
+ * misaligned work buffer; DP_ERR_UNSUPPORTED for more than 4096 intervals
+ * per centre type (ntypes x nint), whose per-atom key map would not fit in
+ * shared memory.
  */
 /*
  * Kernel timing hook, for profiling (off by default; not thread-safe: one

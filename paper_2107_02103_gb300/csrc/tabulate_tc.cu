@@ -54,7 +54,7 @@ constexpr int kTileAtoms = kTN / kCols;  // 12 atoms per 48-column tile
 constexpr int64_t kChunkAtoms = 4104;    // a multiple of 12 (16,416 columns)
 constexpr int kShareSlices = 14;         // used K slices per forward share
 constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' results per chunk
-constexpr int kMaxKeys = 16384;  // ntypes x nint: an atom's key map (int16) lives in shared memory
+constexpr int kMaxKeys = 4096;  // ntypes x nint: each warp's key map (int16) lives in shared memory
 static_assert(kShareSlices <= kMaxShareSlices, "share within the exactness bound");
 static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
 
@@ -210,12 +210,19 @@ __device__ __forceinline__ int valid_row(int v, const int *nvb, const int *sel, 
 // interval's slot (a shared-memory map of the keys, copied out at the end with each slot's key and
 // the slot count) and its flag for the atom's tile; forward also its moments W and the atom's four
 // column exponents (over every value written, which bounds the final ones).
+// Warps (one atom each) per block of the runs and rows kernels: a few per block, so that launching
+// thousands of tiny blocks does not set the pace of a short kernel.
+constexpr int kRunsWarps = 4, kRowsWarps = 2;
+
 template <bool kMom>
-__global__ void __launch_bounds__(32) runs_kernel(const RunsParams P) {
-  __shared__ RunsStage st;
-  extern __shared__ short smap[];  // [nkeys]
-  const int lane = threadIdx.x;
-  const int64_t a = blockIdx.x;
+__global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams P) {
+  __shared__ RunsStage stw[kRunsWarps];
+  extern __shared__ short smapw[];  // [kRunsWarps][nkeys]
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t a = (int64_t)blockIdx.x * kRunsWarps + warp;
+  if (a >= P.natoms) return;  // warp-uniform
+  RunsStage &st = stw[warp];
+  short *smap = smapw + (size_t)warp * P.nkeys;
   const int64_t i = P.atom0 + a;
   for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
   const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the reset)
@@ -412,6 +419,7 @@ struct RowsParams {
   int Mpb;
   const int *fexp;     // [Np]: exponents of dT's rows 4 a + k
   double *ds, *dRt;
+  int64_t natoms;
 };
 
 struct alignas(16) RowsStage {
@@ -427,11 +435,14 @@ struct alignas(16) RowsStage {
 // One warp per atom: every slot's dW finished from the GEMM's four floats (all lanes, in place),
 // then per 32-row batch the batch's runs copied to shared memory and each valid row's dE/dR~ and
 // dE/ds by Horner's rule in u (a lane per row); padded rows get zeros.
-__global__ void __launch_bounds__(32) rows_kernel(const RowsParams P) {
-  __shared__ RowsStage st;
-  extern __shared__ short smap[];  // [nkeys]
-  const int lane = threadIdx.x;
-  const int64_t a = blockIdx.x;
+__global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams P) {
+  __shared__ RowsStage stw[kRowsWarps];
+  extern __shared__ short smapw[];  // [kRowsWarps][nkeys]
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t a = (int64_t)blockIdx.x * kRowsWarps + warp;
+  if (a >= P.natoms) return;  // warp-uniform
+  RowsStage &st = stw[warp];
+  short *smap = smapw + (size_t)warp * P.nkeys;
   const int64_t i = P.atom0 + a;
   const int *gmap = P.map + a * P.nkeys;
   for (int k = lane; k < P.nkeys; k += 32) smap[k] = (short)gmap[k];
@@ -611,7 +622,8 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
     R.atom0 = c0;
     R.natoms = n;
     R.ntiles = ntiles;
-    runs_kernel<true><<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(R);
+    runs_kernel<true><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
+                        kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_runs_moments", st);
     const int64_t warps = Np / 8 * ((S.Kp + kSplitK - 1) / kSplitK);
@@ -700,7 +712,8 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
     R.atom0 = c0;
     R.natoms = n;
     R.ntiles = ntiles;
-    runs_kernel<false><<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(R);
+    runs_kernel<false><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
+                         kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_runs", st);
     // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
@@ -735,7 +748,9 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
       prof_mark("tc_gemm_grad", st);
     }
     Q.atom0 = c0;
-    rows_kernel<<<(unsigned)n, 32, S.nkeys * sizeof(short), st>>>(Q);
+    Q.natoms = n;
+    rows_kernel<<<(unsigned)((n + kRowsWarps - 1) / kRowsWarps), 32 * kRowsWarps, kRowsWarps * S.nkeys * sizeof(short),
+                  st>>>(Q);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_rows", st);
   }
