@@ -154,7 +154,15 @@ TC_KERNEL = {"tc_runs_moments": "runs_kernel<moments> (dp_tabulate_fusion_fwd_tc
              "tc_rows": "rows_kernel (dp_tabulate_fusion_grad_tc_f64)",
              "tc_gemm_fwd": "gemm_kernel (dp_tabulate_fusion_fwd_tc_f64)",
              "tc_gemm_grad": "gemm_kernel (dp_tabulate_fusion_grad_tc_f64)"}
-TC_PROFILE_EVENTS = 64  # per step: the tc calls record one after each of their kernels
+TC_CHUNK_ATOMS = 4104  # atoms per chunk of the tc calls
+
+
+def tc_profile_events(w) -> int:
+    """Events one step of the tc calls records: a start and a mark after the coefficients per call,
+    then per chunk forward runs, split, and per centre type GEMM and epilogue; backward runs, dT split,
+    per type GEMM, rows."""
+    chunks = -(-w.nloc // TC_CHUNK_ATOMS)
+    return min(4096, 4 + chunks * (2 + 2 * w.ntypes + 3 + w.ntypes) + 8)
 
 
 def tc_fmas(w, runs) -> dict:
@@ -433,7 +441,7 @@ def run_native(args, rank, world, local_rank):
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
     pev, pnames = None, []
     if args.algo == "tc":  # per-kernel times inside the tc calls, from events they record themselves
-        pev = [[torch.cuda.Event(enable_timing=True) for _ in range(TC_PROFILE_EVENTS)] for _ in range(args.steps)]
+        pev = [[torch.cuda.Event(enable_timing=True) for _ in range(tc_profile_events(w))] for _ in range(args.steps)]
         for e in (e for row in pev for e in row):
             e.record(stream)  # creates the CUDA events before the timed region
     vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x.strip()]
