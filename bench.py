@@ -181,7 +181,7 @@ def moment_fmas(runs, M1: int) -> dict:
 # `ncu --set full` capture of its current version (profiles/<kernel>_<algo>_<workload>_<dtype>.md);
 # absent means no capture of the current kernel exists and `traffic` is reported as null.
 PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,
-                       ("cu85", "f64", "tc_rows", "tc"): 140421632 + 95273984}
+                       ("cu85", "f64", "tc_rows", "tc"): 140379392 + 95468544}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
