@@ -1,0 +1,99 @@
+"""The arithmetic of the tensor-core tabulation, restated in numpy on the CPU and held against the
+oracle (Sec. II: T_i = R~_i^T G_i / N_c and its backward): per interval l of an atom's rows, the
+moments W[k][q] = sum_j R~_jk u_j^q with u = t / Delta_l, the scaled coefficients
+c'_q = c_q Delta_l^q, T[k][m] = (1/N_c) sum_(l,q) W[k][q] c'_q[m]; backward
+dW[k][q] = (1/N_c) sum_m dT[k][m] c'_q[m], dE/dR~_jk = sum_q dW[k][q] u_j^q and
+dE/ds_j = sum_k R~_jk sum_q q dW[k][q] u_j^(q-1) / Delta_l (0 for clamped s).  These are the sums
+the GPU GEMMs compute (in exact digit-split form); a dropped power of Delta, a wrong factor q or a
+missing clamp fails here, before any GPU run.  CPU only."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads as W
+
+TOL = 1e-12
+
+
+def regrouped(o, tabs, info, w, dT, scale_delta=True, q_factor=True):
+    """T, ds, dR~ by interval moments and scaled coefficients (rows need not be sorted); the two
+    switches plant a slip (coefficients left unscaled, the derivative without its factor q)."""
+    nloc, nnei = w.s.shape
+    M1 = tabs.shape[-2]
+    off = np.concatenate([[0], np.cumsum(w.sel)])
+    T = np.zeros((nloc, 4, M1))
+    ds = np.zeros((nloc, nnei))
+    dR = np.zeros((nloc, nnei, 4))
+    for i in range(nloc):
+        alpha = int(w.atype[i]) if w.atype is not None else 0
+        rows = {}  # key (b, l) -> [(row, u, clamped)]
+        for b in range(w.ntypes):
+            for j in range(off[b], off[b] + int(w.nvalid[i, b])):
+                l, t, clamped = o.locate(info, w.s[i, j])
+                delta = info.stride0 if l < info.n0 else info.stride1
+                rows.setdefault((b, l), []).append((j, t / delta, clamped))
+        for (b, l), rr in rows.items():
+            delta = info.stride0 if l < info.n0 else info.stride1
+            c = tabs[alpha * w.ntypes + b, l]                          # [M1][6]: t^5 .. t^0
+            cp = np.stack([c[:, 5 - q] * (delta ** q if scale_delta else 1.0) for q in range(6)])  # c'_q
+            Wm = np.zeros((4, 6))
+            for j, u, _ in rr:
+                Wm += np.outer(w.Rt[i, j], u ** np.arange(6))
+            T[i] += Wm @ cp / nnei
+            dW = dT[i] @ cp.T / nnei                                   # [4][6]
+            for j, u, clamped in rr:
+                dR[i, j] = dW @ (u ** np.arange(6))
+                dq = dW[:, 1:] @ ((np.arange(1, 6) if q_factor else 1.0) * u ** np.arange(5)) / delta
+                ds[i, j] = 0.0 if clamped else float(w.Rt[i, j] @ dq)
+    return T, ds, dR
+
+
+def _check(w):
+    o = oracle.default()
+    info = o.table_info(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    tabs = o.tables(w.params, w.widths, info)
+    T, ds, dR = regrouped(o, tabs, info, w, w.dT)
+    To = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    dso, dRo = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, w.dT)
+    for got, ref in ((T, To), (ds, dso), (dR, dRo)):
+        err = np.max(np.abs(got - ref)) / np.max(np.abs(ref))
+        assert err <= TOL, err
+
+
+def test_regrouping_matches_oracle_sorted_rows():
+    _check(W.tiny(seed=3, nloc=12, nreal=20, sel=24, widths=(1, 4, 8, 16), M2=4))
+
+
+def test_regrouping_matches_oracle_two_types_unsorted_clamped():
+    """Two neighbour types and two centre types, rows shuffled inside their segments (an interval's
+    rows in several runs), and rows past the coarse segment and below the table (clamped)."""
+    w = W.water(seed=17, nmol=48, widths=(1, 4, 8), M2=4, sel=(24, 48), rc=5.0)
+    rng = np.random.default_rng(5)
+    s, Rt = w.s.copy(), w.Rt.copy()
+    off = np.concatenate([[0], np.cumsum(w.sel)])
+    for i in range(w.nloc):
+        for b in range(w.ntypes):
+            nv = int(w.nvalid[i, b])
+            p = off[b] + rng.permutation(nv)
+            s[i, off[b]:off[b] + nv], Rt[i, off[b]:off[b] + nv] = s[i, p], Rt[i, p]
+    o = oracle.default()
+    info = o.table_info(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    s[0, 0] = info.upper_ext + 1.0
+    s[1, 1] = info.lower - 0.5
+    w2 = W.Workload(**{**w.__dict__, "s": s, "Rt": Rt})
+    _check(w2)
+
+
+@pytest.mark.parametrize("mistake", ["unscaled_coefficients", "no_q_factor"])
+def test_regrouping_slips_are_caught(mistake):
+    """The comparison above notices a plausible slip in the regrouping itself."""
+    w = W.tiny(seed=4, nloc=6, nreal=16, sel=16, widths=(1, 4, 8), M2=4)
+    o = oracle.default()
+    info = o.table_info(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    tabs = o.tables(w.params, w.widths, info)
+    To = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
+    dso, _ = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, w.dT)
+    kw = {"scale_delta": False} if mistake == "unscaled_coefficients" else {"q_factor": False}
+    T, ds, _ = regrouped(o, tabs, info, w, w.dT, **kw)
+    rel = lambda a, b: np.max(np.abs(a - b)) / np.max(np.abs(b))  # noqa: E731
+    assert max(rel(T, To), rel(ds, dso)) > 1e-3
