@@ -52,10 +52,9 @@ constexpr int kQ = 6;                 // K entries per interval: u^0 .. u^5
 constexpr int kCols = 4;              // GEMM columns per atom: k = 0 .. 3
 constexpr int kTileAtoms = kTN / kCols;  // 12 atoms per 48-column tile
 constexpr int64_t kChunkAtoms = 4104;    // a multiple of 12 (16,416 columns)
-constexpr int kShareSlices = 14;         // used K slices per forward share
+constexpr int kShareSlices = kMaxShareSlices;  // used K slices per forward share (28, the exactness bound)
 constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' results per chunk
 constexpr int kMaxKeys = 4096;  // ntypes x nint: each warp's key map (int16) lives in shared memory
-static_assert(kShareSlices <= kMaxShareSlices, "share within the exactness bound");
 static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
 
 // Sizes shared by the kernels and the work-buffer layout.
@@ -358,9 +357,10 @@ __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict
   }
 }
 
-// T for the atoms of type alpha of one 12-atom tile (one block): the tile's shares (one per
-// kShareSlices used slices) summed and scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at
-// a time: read with the columns fastest (the shares' rows), written with the channels fastest (T's).
+// T for the atoms of type alpha of one 12-atom tile (one block) whose used slices take several shares
+// (one per kShareSlices; a single share's GEMM writes T itself) or none (T = 0): the shares summed and
+// scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at a time: read with the columns fastest
+// (the shares' rows), written with the channels fastest (T's).
 __global__ void __launch_bounds__(256) fwd_epilogue_kernel(const float4 *__restrict__ part, int Mp, int64_t Np,
                                                            const int *__restrict__ eexp,
                                                            const int *__restrict__ fexp,
@@ -383,6 +383,7 @@ __global__ void __launch_bounds__(256) fwd_epilogue_kernel(const float4 *__restr
   if (c) atomicAdd(&nused, c);
   __syncthreads();
   const int nz = (nused + kShareSlices - 1) / kShareSlices;
+  if (nz == 1) return;  // uniform: the GEMM wrote this tile's T itself
   for (int m0 = 0; m0 < M1; m0 += 32) {
     for (int e = threadIdx.x; e < kTN * 32; e += blockDim.x) {
       const int col = e % kTN, m = m0 + e / kTN;
@@ -643,6 +644,13 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
       G.part = part;
       G.slices_per_split = kShareSlices;
       G.kocc = wk + L.occ + (size_t)t * occ_per_type;
+      G.tout = T;  // tiles with one share write T themselves
+      G.ldt = M1;
+      G.natoms = n;
+      G.atom0 = c0;
+      G.atype = atype;
+      G.alpha = t;
+      G.ntypes = ntypes;
       const dim3 grid((unsigned)ntiles, (unsigned)(S.Mpf / kTM), (unsigned)S.zmax);
       gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
       if ((rc = launch_status(who))) return rc;

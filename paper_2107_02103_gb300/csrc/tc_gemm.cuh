@@ -70,7 +70,7 @@ constexpr uint32_t kTmemCols = 512;  // allocation (a power of two); kS * kTN = 
 constexpr int kMaxShareSlices = kMaxShareK / kTK;
 constexpr size_t kSmemTail = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16;  // used-slice list
 constexpr int kScatKeys = kTM / 4 + 1, kScatAtoms = kTN / 4;  // scatter: keys (kq >= 4) and atoms of a tile
-constexpr size_t kSmemTotal = kSmemTail + (kMaxShareSlices + 1) * 4 + kScatKeys * kScatAtoms * 4;
+constexpr size_t kSmemTotal = kSmemTail + (kMaxShareSlices + 2) * 4 + kScatKeys * kScatAtoms * 4;
 static_assert((size_t)kS * kMaxShareK * 63 * 63 < (1u << 24), "fp32 diagonal sums must stay exact");
 static_assert(kMaxShareK % kTK == 0 && kS * kTN <= (int)kTmemCols, "shares and TMEM");
 static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
@@ -165,6 +165,44 @@ __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restric
   }
 }
 
+// f 2^e as a double, exactly, by moving fields (f finite; |e| < 900, so a normal result stays normal
+// and a float that is zero stays zero; float subnormals, which the sums do not produce, widen to 0)
+__device__ __forceinline__ double widen_pow2(float f, int e) {
+  const double d = dfl::widen(f);
+  const long long b = __double_as_longlong(d);
+  return (b & 0x7fffffffffffffffll) ? __longlong_as_double(b + ((long long)e << 52)) : d;
+}
+
+// The shares' results of one output summed in a fixed order: each share's four floats are added
+// into a three-float sum by exact two-sums on the FP32 pipe (only the last component rounds, ~2^-72
+// below the sum), which is converted to f64 once and scaled by the row and column powers of two.
+struct Sum3 {
+  float s0 = 0.f, s1 = 0.f, s2 = 0.f;
+  __device__ __forceinline__ void add(float x) {
+    float t = __fadd_rn(s0, x), z = __fsub_rn(t, s0);
+    const float e0 = __fadd_rn(__fsub_rn(s0, __fsub_rn(t, z)), __fsub_rn(x, z));
+    s0 = t;
+    t = __fadd_rn(s1, e0);
+    z = __fsub_rn(t, s1);
+    const float e1 = __fadd_rn(__fsub_rn(s1, __fsub_rn(t, z)), __fsub_rn(e0, z));
+    s1 = t;
+    s2 = __fadd_rn(s2, e1);
+  }
+  __device__ __forceinline__ void add(const float4 q) {
+    add(q.x);
+    add(q.y);
+    add(q.z);
+    add(q.w);
+  }
+  // the sum times 2^(E + F); NaN for a row or column with an inf or NaN, or a NaN share
+  __device__ __forceinline__ double value(int E, int F) const {
+    if (E >= kNonFinite || F >= kNonFinite || s0 != s0) return __longlong_as_double(0x7ff8000000000000ll);
+    if (E + F > -900 && E + F < 900)  // the scaling moves exponent fields only (sums stay normal)
+      return __dadd_rn(__dadd_rn(widen_pow2(s0, E + F), widen_pow2(s1, E + F)), widen_pow2(s2, E + F));
+    return scalbn(__dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2)), E + F);
+  }
+};
+
 // One hidden-layer GEMM of a chunk of one type's atoms: rows r0 .. r0 + n - 1 of the plain
 // row-major A [*][K] (as digit planes) times B (digit planes), K cut into shares of at most
 // kMaxShareK (grid z); the shares' f64 results go to `part`, and epilogue_kernel sums them and
@@ -195,6 +233,11 @@ struct TcGemm {
   const int32_t *atype;
   int64_t natoms, atom0;
   int nkeys, cap, alpha, ntypes, kq;
+  // direct output (with kocc): a tile whose used slices fit one share writes its outputs as f64,
+  // scaled by 2^(E_row + F_col), to tout[((atom0 + a) 4 + k) ldt + row] for row < ldt and the atoms
+  // a < natoms of type alpha, and nothing to part (the forward tabulation's T)
+  double *tout;
+  int ldt;
   bool skip;
   // forward
   const double *bias;
@@ -243,8 +286,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   uint64_t *done = empty + kStages;                                               // every MMA done (one use)
   uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(done + 1);
   int *flags = reinterpret_cast<int *>(tmem_holder + 1);                          // producer / issuer ok
-  int *slist = reinterpret_cast<int *>(smem + kSmemTail);                         // used slices, then their count
-  int *stab = slist + kMaxShareSlices + 1;  // scatter: slot of (key, atom) of the tile, or -1
+  int *slist = reinterpret_cast<int *>(smem + kSmemTail);  // used slices, their count, the tile's total
+  int *stab = slist + kMaxShareSlices + 2;  // scatter: slot of (key, atom) of the tile, or -1; direct: atom wanted
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int64_t m0 = (int64_t)blockIdx.y * kTM;
   const int n0 = blockIdx.x * kTN;
@@ -260,6 +303,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
         slot = P.map[a * P.nkeys + key];
       stab[x] = slot;
     }
+  if (P.tout)
+    for (int x = tid; x < kScatAtoms; x += kThreads) {
+      const int64_t a = (int64_t)(n0 / 4) + x;
+      stab[x] = a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha);
+    }
   int nsl = min(nslices - i0, P.slices_per_split);  // dense: > 0, no empty share
   if (P.kocc) {
     // this share's used slices, in order, by a ballot over the tile's flags
@@ -267,7 +315,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
       const unsigned char *occ = P.kocc + (size_t)blockIdx.x * nslices;
       const int last = i0 + P.slices_per_split;
       int rank = 0;
-      for (int b = 0; b < nslices && rank < last; b += 32) {  // uniform
+      for (int b = 0; b < nslices && (rank < last || P.tout); b += 32) {  // uniform; direct output counts all
         const int i = b + lane;
         const bool used = i < nslices && occ[i] != 0;
         const unsigned m = __ballot_sync(0xffffffffu, used);
@@ -275,12 +323,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
         if (used && r >= i0 && r < last) slist[r - i0] = i;
         rank += __popc(m);
       }
-      if (lane == 0) slist[kMaxShareSlices] = min(max(rank - i0, 0), P.slices_per_split);
+      if (lane == 0) {
+        slist[kMaxShareSlices] = min(max(rank - i0, 0), P.slices_per_split);
+        slist[kMaxShareSlices + 1] = rank;
+      }
     }
     __syncthreads();
     nsl = slist[kMaxShareSlices];
     if (nsl == 0) return;  // uniform: no slice left for this share
   }
+  const bool direct = P.tout && P.kocc && slist[kMaxShareSlices + 1] <= P.slices_per_split;
 
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -374,6 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   const int key = P.scat ? (int)((m0 + rl) / P.kq) : 0, q = P.scat ? (int)(m0 + rl - (int64_t)key * P.kq) : 0;
   const int key_l = P.scat ? key - (int)(m0 / P.kq) : 0;  // this thread's row's key, in the tile
   const bool row_wanted = P.scat && q < 6 && key < P.nkeys;
+  const int Erow = direct && m0 + rl < P.ldt ? P.Eexp[m0 + rl] : 0;
   const uint32_t trow = tmem + ((uint32_t)(32 * (warp & 3)) << 16);
   constexpr int kColsPerWarp = kTN / (kThreads / 128);
   static_assert(kColsPerWarp % 8 == 0, "column share");
@@ -391,7 +444,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
     for (int c = 0; c < 8; ++c) {
       // sum_d v_d 64^-(d+2) as four floats on the FP32 pipe: diagonals 2 and 3 (d = 0, 1) as an exact
       // two-sum, 4 .. 10 in float-float, smallest first (its rounding lies ~2^-60 below the sum).
-      // The scaling by 2^(E+F), and all f64 arithmetic, is left to epilogue_kernel.
+      // The scaling by 2^(E+F), and all f64 arithmetic, is left to the epilogue (or, for a direct
+      // output, to the two f64 adds below).
       dfl::df64 lo(0.0f);
 #pragma unroll
       for (int d = kS - 1; d >= 2; --d) {
@@ -402,7 +456,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
       const float s = __fadd_rn(a, b), bb = __fsub_rn(s, a);
       const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
       const float4 val = ok ? make_float4(s, e, lo.hi, lo.lo) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
-      if (outp) {
+      if (direct) {
+        if (m0 + rl < P.ldt && stab[(c0 + c) >> 2]) {
+          Sum3 acc;
+          acc.add(val);
+          const int64_t a = (int64_t)(n0 >> 2) + ((c0 + c) >> 2);
+          P.tout[((P.atom0 + a) * 4 + ((c0 + c) & 3)) * P.ldt + m0 + rl] = acc.value(Erow, P.Fexp[n0 + c0 + c]);
+        }
+      } else if (outp) {
         outp[c0 + c] = val;
       } else if (row_wanted) {
         const int al = (c0 + c) >> 2, k = (c0 + c) & 3;  // the tile's atom, its column k
@@ -417,44 +478,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   asm volatile("tcgen05.fence::after_thread_sync;");
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
 }
-
-// f 2^e as a double, exactly, by moving fields (f finite; |e| < 900, so a normal result stays normal
-// and a float that is zero stays zero; float subnormals, which the sums do not produce, widen to 0)
-__device__ __forceinline__ double widen_pow2(float f, int e) {
-  const double d = dfl::widen(f);
-  const long long b = __double_as_longlong(d);
-  return (b & 0x7fffffffffffffffll) ? __longlong_as_double(b + ((long long)e << 52)) : d;
-}
-
-// The shares' results of one output summed in a fixed order: each share's four floats are added
-// into a three-float sum by exact two-sums on the FP32 pipe (only the last component rounds, ~2^-72
-// below the sum), which is converted to f64 once and scaled by the row and column powers of two.
-struct Sum3 {
-  float s0 = 0.f, s1 = 0.f, s2 = 0.f;
-  __device__ __forceinline__ void add(float x) {
-    float t = __fadd_rn(s0, x), z = __fsub_rn(t, s0);
-    const float e0 = __fadd_rn(__fsub_rn(s0, __fsub_rn(t, z)), __fsub_rn(x, z));
-    s0 = t;
-    t = __fadd_rn(s1, e0);
-    z = __fsub_rn(t, s1);
-    const float e1 = __fadd_rn(__fsub_rn(s1, __fsub_rn(t, z)), __fsub_rn(e0, z));
-    s1 = t;
-    s2 = __fadd_rn(s2, e1);
-  }
-  __device__ __forceinline__ void add(const float4 q) {
-    add(q.x);
-    add(q.y);
-    add(q.z);
-    add(q.w);
-  }
-  // the sum times 2^(E + F); NaN for a row or column with an inf or NaN, or a NaN share
-  __device__ __forceinline__ double value(int E, int F) const {
-    if (E >= kNonFinite || F >= kNonFinite || s0 != s0) return __longlong_as_double(0x7ff8000000000000ll);
-    if (E + F > -900 && E + F < 900)  // the scaling moves exponent fields only (sums stay normal)
-      return __dadd_rn(__dadd_rn(widen_pow2(s0, E + F), widen_pow2(s1, E + F)), widen_pow2(s2, E + F));
-    return scalbn(__dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2)), E + F);
-  }
-};
 
 int set_smem(const char *who) {
   static std::atomic<bool> done{false};
