@@ -97,3 +97,23 @@ def test_regrouping_slips_are_caught(mistake):
     T, ds, _ = regrouped(o, tabs, info, w, w.dT, **kw)
     rel = lambda a, b: np.max(np.abs(a - b)) / np.max(np.abs(b))  # noqa: E731
     assert max(rel(T, To), rel(ds, dso)) > 1e-3
+
+
+def test_tc_work_size_query():
+    """dp_tabulate_tc_work_bytes on the host: one size for both directions, 256-byte multiples,
+    growing with the atoms until the chunk size caps it, refusals for bad sizes and for more
+    intervals per centre type than the shared-memory key map holds."""
+    import __graft_entry__
+    __graft_entry__._load_builder().build()
+    import paper_2107_02103_gb300 as dpc
+    info = dpc.dp_table_info_make(0.0, 0.5, 0.01, 0.1, 5.0)   # 50 fine + 20 coarse intervals
+    sizes = [dpc.dp_tabulate_tc_work_bytes(info, n, 512, 1, 100) for n in (1, 100, 4104, 20000)]
+    assert all(b > 0 and b % 256 == 0 for b in sizes)
+    assert sizes[0] <= sizes[1] <= sizes[2] == sizes[3]       # chunks of at most 4104 atoms
+    assert dpc.dp_tabulate_tc_work_bytes(info, 100, 512, 3, 100) > sizes[1]   # K grows with the types
+    for bad in ((info, -1, 512, 1, 100), (info, 10, 0, 1, 100), (info, 10, 512, 9, 100), (info, 10, 512, 1, 0)):
+        with pytest.raises(ValueError):
+            dpc.dp_tabulate_tc_work_bytes(*bad)
+    wide = dpc.dp_table_info_make(0.0, 0.5, 0.0001, 0.1, 5.0)   # 5000 fine intervals
+    with pytest.raises(ValueError):
+        dpc.dp_tabulate_tc_work_bytes(wide, 10, 512, 1, 100)
