@@ -29,8 +29,9 @@
 // Per chunk of at most kChunkAtoms atoms and per centre type alpha:
 //   forward:  runs_kernel<true> (map, W, column exponents, slice flags),
 //             split_mom_kernel (W -> B digit planes, used slices only),
-//             gemm_kernel (A = C'_alpha^T: channels x K, B = W^T: K x (atom, k)),
-//             fwd_epilogue_kernel (shares -> T for the atoms of type alpha);
+//             gemm_kernel (A = C'_alpha^T: channels x K, B = W^T: K x (atom, k); a tile whose
+//             used slices fit one share writes its atoms' T directly),
+//             fwd_epilogue_kernel (T of the tiles with several shares, or none);
 //   backward: runs_kernel<false> (map, tile flags), split of dT (B), gemm_kernel
 //             (A = C'_alpha: K x channels, B = dT^T) scattering each used
 //             (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
