@@ -70,3 +70,20 @@ def test_footprint_counts_every_array():
     assert f["bytes_per_atom"] == 8 * (10 * 32 + 8 * 32 + 32 * 4) + 4 * 2
     assert f["uncompressed_extra_bytes_per_atom"] == 8 * 32 * (8 + 16 + 32)
     assert f["atoms_per_280GB"] > f["atoms_per_280GB_uncompressed"] > 0
+
+
+def test_tensor_core_path_accounting():
+    """--algo tc: the FP64 kernels' FMAs per valid row (moments 24, rows 40), the GEMMs' 24 M1 per
+    run, and enough timing events per step for every kernel mark of every chunk and centre type."""
+    w = W.tiny(seed=5, nloc=9, nreal=13, sel=16, widths=(1, 4, 8), M2=4)
+    rows = int(w.nvalid.sum())
+    runs = np.array([3, 5, 5])
+    f = bench.tc_fmas(w, runs)
+    assert f["tc_runs_moments"] == 24 * rows and f["tc_rows"] == 40 * rows
+    assert f["tc_gemm_fwd"] == f["tc_gemm_grad"] == 24 * w.M1 * len(runs)
+    assert w.evals == rows * w.M1
+    for nloc, ntypes in ((100, 1), (4104, 1), (4105, 2), (12288, 2), (32768, 3), (1048576, 2)):
+        chunks = -(-nloc // bench.TC_CHUNK_ATOMS)
+        marks = 2 + 2 + chunks * ((2 + 2 * ntypes) + (2 + ntypes + 1))  # starts, coefficients, per chunk
+        ww = W.Workload(**{**w.__dict__, "s": np.zeros((nloc, 1)), "ntypes": ntypes})
+        assert bench.tc_profile_events(ww) >= min(marks, 4096)
