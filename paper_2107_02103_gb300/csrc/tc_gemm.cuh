@@ -12,7 +12,6 @@
 namespace dpc {
 namespace {
 
-
 // ------------------------------------------------- f64 GEMMs on the tensor cores
 // GB300 retires FP64 at 2 lanes per clock per SM but fp16 products on its
 // tcgen05 tensor cores at ~1000 times that rate.  An f64 GEMM C = A B is
@@ -26,8 +25,9 @@ namespace {
 // a block's share of K is at most kMaxShareK = 448 (9 x 448 x 3969 < 2^24).
 // The 9 diagonal sums of an output are combined on the FP32 pipe into four
 // floats (the two largest by an exact two-sum, the rest in float-float, whose
-// rounding lies ~2^-60 below the result); epilogue_kernel adds the shares'
-// floats into a three-float sum by exact two-sums and converts it to f64 once.
+// rounding lies ~2^-60 below the result); the caller's epilogue (Sum3 below)
+// adds the shares' floats into a three-float sum by exact two-sums and
+// converts it to f64 once.
 // What rounds is that conversion, the 54-bit truncation of the operands and
 // the dropped terms: |error| <~ K 2^-50 max_k|a_ik| max_k|b_kj|, against
 // K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column with an
@@ -41,8 +41,9 @@ namespace {
 // swizzle (8-row x 16-byte core matrices).  Lane 0 of warp 0 moves a slice's
 // A and B blocks into one of four stages with two bulk async copies counted in
 // bytes on the stage's "full" mbarrier; lane 0 of warp 1 issues the slice's 45
-// digit-product MMAs (M 128, N 48, K 16, fp16 in, fp32 accumulators in TMEM,
-// one per diagonal) and commits them to the stage's "empty" mbarrier, which
+// digit products as 13 MMAs (M 128, K 16, fp16 in, fp32 accumulators in TMEM,
+// one 48-column block per diagonal; digit s of A against all of B's digits
+// t <= 8 - s at once, N up to 240) and commits them to the stage's "empty" mbarrier, which
 // the producer waits on before refilling the stage.  A last commit on a
 // barrier used once releases the four warps, which read their TMEM lane
 // quadrant (rows), combine the diagonals and write the share's result as four
@@ -50,7 +51,8 @@ namespace {
 // scales by 2^(E+F) and finishes the outputs.  Two optional modes serve sparse
 // operands (the tabulated embedding's interval moments): a per-tile list of the
 // K slices in use (the others are zero and are skipped; the shares then cut the
-// used slices), and a per-tile flag that skips unwanted output tiles, whose
+// used slices, and a tile whose used slices fit one share can write its f64
+// outputs itself), and a per-tile flag that skips unwanted output tiles, whose
 // wanted outputs are scattered to per-run slots instead of a dense array.
 // Every wait on an mbarrier is bounded; a wait that gives up makes the tile's
 // outputs NaN.
