@@ -87,3 +87,35 @@ def test_tensor_core_path_accounting():
         marks = 2 + 2 + chunks * ((2 + 2 * ntypes) + (2 + ntypes + 1))  # starts, coefficients, per chunk
         ww = W.Workload(**{**w.__dict__, "s": np.zeros((nloc, 1)), "ntypes": ntypes})
         assert bench.tc_profile_events(ww) >= min(marks, 4096)
+
+
+def test_report_takes_the_roofline_on_the_dominant_tc_kernel():
+    """report() with per-kernel times from the tc calls: the roofline names the dominant kernel with
+    its own algorithmic FLOPs and peak (FP64 for the rows and moments kernels, the tensor peak and 45
+    digit products for a GEMM), and the launch count includes the kernels inside the calls."""
+    import argparse
+    w = W.tiny(seed=5, nloc=9, nreal=13, sel=16, widths=(1, 4, 8), M2=4)
+    args = argparse.Namespace(dtype="f64", algo="tc", steps=2, warmup=3, scaling="weak", chain=False,
+                              fitting=False, fitting_tc=False, no_cpu_baseline=True)
+    runs = np.array([3, 5, 5])
+    tcf = bench.tc_fmas(w, runs)
+    step_ms = [1.0, 1.0]
+    k_ms = {"fwd": [0.4, 0.4], "descriptor": [0.1, 0.1], "grad": [0.5, 0.5]}
+    for dom, ms in (("tc_rows", 0.3), ("tc_gemm_grad", 0.45)):
+        tc_ms = {"tc_runs_moments": [0.2, 0.2], "tc_gemm_fwd": [0.1, 0.1], "tc_rows": [0.3, 0.3],
+                 "tc_gemm_grad": [0.05, 0.05]}
+        tc_ms[dom] = [ms, ms]
+        out = bench.report(args, w, 1, step_ms, k_ms, 2e-3, float(w.evals), None, None, 0.01,
+                           bench.moment_fmas(runs, w.M1), 0, tc_ms, tcf, [16, 16])
+        r = out["roofline"]
+        assert r["kernel"] == bench.TC_KERNEL[dom]
+        if dom == "tc_rows":
+            assert r["bound"] == "alu"
+            assert abs(r["achieved"] - 2 * 40 * w.evals / w.M1 / (ms * 1e-3) / 1e12) < 1e-3
+            assert r["peak"] == round(bench.peak_tflops("f64"), 4)
+        else:
+            assert r["bound"] == "tensor"
+            assert abs(r["achieved"] - 45 * 2 * 24 * w.M1 * len(runs) / (ms * 1e-3) / 1e12) < 0.02
+            assert r["peak"] == round(bench.tensor_peak()[0], 1)
+        assert "tensor_frac" in out["kernels"]["tc_gemm_fwd"] and "frac" in out["kernels"]["tc_rows"]
+        assert out["gpu_launches"] == 3 * 2 + 16 * 2 - 2 * 2
