@@ -488,11 +488,13 @@ int dp_fitting_grad_f32(const float *params, const int32_t *widths, int nlayer, 
  * width 240), which every GPU that loads the library keeps until the process
  * exits; larger problems return DP_ERR_UNSUPPORTED -- use the call with a
  * work buffer.  Nothing is allocated: no cudaMalloc, no cudaFree, no
- * allocating library routine.  The first call on a device looks the array's
- * address up (cudaGetSymbolAddress) and keeps it; make that first call
- * before any stream capture.  Every call on a device uses the same array and
- * it keeps the last call's contents; the kernels overwrite every element they
- * read, so nothing needs clearing, but calls that overlap on the GPU (on
+ * allocating library routine.  Every call looks the array's address up in
+ * the current context (cudaGetSymbolAddress, which allocates nothing; the
+ * first lookup on a device may load the library's kernels there, so make
+ * the first call before any stream capture).  Every call on a device uses
+ * the same array and it keeps the last call's contents; the kernels
+ * overwrite every element they read, so nothing needs clearing, but calls
+ * that overlap on the GPU (on
  * different streams, or from different threads) race on it.  Results are
  * those of dp_fitting_grad_f64.  Arguments and errors as dp_fitting_grad_f64.
  */

@@ -683,29 +683,16 @@ size_t work_bytes_api(const int32_t *widths, int nlayer, int64_t nloc) {
 constexpr size_t kStaticScratchDoubles = (size_t)1 << 20;  // 8 MiB
 static __device__ __align__(256) double g_fit_scratch[kStaticScratchDoubles];
 
-constexpr int kMaxScratchDevices = 64;
-std::atomic<double *> g_fit_scratch_addr[kMaxScratchDevices];  // per device, filled on its first call
-
-// Device address of the array on the current device.  In host code the array's
-// name only stands in for it; the address comes from the runtime, looked up on
-// the first call on each device and kept.
+// Device address of the array in the current context.  In host code the array's
+// name only stands in for it; the runtime gives the address.  It is looked up
+// on every call (the lookup allocates nothing), so that a context made anew --
+// after cudaDeviceReset, or on another device -- is served at its own address.
 int static_scratch(double **out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_fitting_grad_noalloc: cudaGetDevice: %s", cudaGetErrorString(e));
-  if (dev < 0 || dev >= kMaxScratchDevices)
-    return set_error(DP_ERR_UNSUPPORTED, "dp_fitting_grad_noalloc: device %d beyond the %d it tracks", dev,
-                     kMaxScratchDevices);
-  double *p = g_fit_scratch_addr[dev].load(std::memory_order_acquire);
-  if (!p) {
-    void *q = nullptr;
-    e = cudaGetSymbolAddress(&q, g_fit_scratch);
-    if (e != cudaSuccess)
-      return set_error(DP_ERR_CUDA, "dp_fitting_grad_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
-    p = static_cast<double *>(q);
-    g_fit_scratch_addr[dev].store(p, std::memory_order_release);
-  }
-  *out = p;
+  void *q = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&q, g_fit_scratch);
+  if (e != cudaSuccess)
+    return set_error(DP_ERR_CUDA, "dp_fitting_grad_noalloc: cudaGetSymbolAddress: %s", cudaGetErrorString(e));
+  *out = static_cast<double *>(q);
   return DP_OK;
 }
 

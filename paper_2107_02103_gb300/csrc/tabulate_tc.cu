@@ -417,7 +417,7 @@ struct RowsParams {
   const int *map, *keys, *nslots;
   float4 *dW;          // [natoms][cap][24]: the backward GEMM's result per slot (four floats), then in place
                        // (dW, q dW / Delta) as two doubles
-  const int *eexp;     // [ntypes][Mpb]: exponents of the backward A's rows 8 key + q
+  const int *eexp;     // [ntypes][Mpb]: exponents of the backward A's rows 6 key + q
   int Mpb;
   const int *fexp;     // [Np]: exponents of dT's rows 4 a + k
   double *ds, *dRt;
@@ -549,7 +549,7 @@ int check_work(const Layout &L, const void *work, size_t nbytes, const char *who
 }
 
 // C' of every centre type from the table, then its digit planes: forward A = C'^T (rows: the
-// channels, K: 8 key + q), backward A = C' (rows: 8 key + q, K: the channels).
+// channels, K: 6 key + q), backward A = C' (rows: 6 key + q, K: the channels).
 int prep(const double *table, const TableGeom &g, const Shape &s, const Layout &L, unsigned char *wk, bool fwd,
          int nnei, cudaStream_t st, const char *who) {
   double *Cp = reinterpret_cast<double *>(wk + L.cp);

@@ -49,8 +49,10 @@ CASES = [
     ("tiny", {}, None), ("water", dict(nmol=256), None), ("cu85", dict(cells=(6, 6, 6)), None),
     ("cugeo", dict(cells=(6, 6, 6)), None), ("alcumg", dict(pad=0.1, cells=(6, 6, 6)), None),
     ("alcumg", dict(pad=0.6, cells=(6, 6, 6)), None), ("cu85", {}, None), ("water", {}, 512),
-    ("alcumg", dict(pad=0.3), 384),
+    ("cugeo", {}, 512), ("alcumg", dict(pad=0.1), 384), ("alcumg", dict(pad=0.3), 384),
+    ("alcumg", dict(pad=0.6), 384),
 ]
+CHUNK = 4104  # atoms per chunk of the tensor-core calls (their work buffer holds one chunk)
 
 
 @pytest.mark.parametrize("name,kw,nsample", CASES, ids=[f"{c[0]}-{c[1]}" for c in CASES])
@@ -64,6 +66,7 @@ def test_tc_against_oracle_and_fp64_path(name, kw, nsample):
     atoms = None
     if nsample:
         atoms = np.sort(np.random.default_rng(5).choice(w.nloc, nsample, replace=False))
+        atoms[0], atoms[-1] = 0, w.nloc - 1
     ref = run_oracle(w, F64, atoms=atoms)
     assert_parity(got, ref, F64, atoms=atoms, keys=("T", "ds", "dRt"))
     pipe = _pipe(w, model, x)
@@ -160,7 +163,7 @@ def test_tc_chunks_of_atoms():
     pipe = _pipe(w, model, x)
     for k in ("T", "ds", "dRt"):
         assert rel(got[k], pipe[k]) <= CLOSE, k
-    atoms = np.r_[0:4, 4100:4108, w.nloc - 4:w.nloc]
+    atoms = np.r_[0:4, CHUNK - 4:CHUNK + 4, w.nloc - 4:w.nloc]
     assert_parity(got, run_oracle(w, F64, atoms=atoms), F64, atoms=atoms, keys=("T", "ds", "dRt"))
 
 
@@ -186,3 +189,42 @@ def test_tc_work_buffer_rules_and_reuse():
         dpc.dp_tabulate_fusion_fwd_tc_f64(*args, work=work[16:need + 16])
     with pytest.raises(ValueError):
         dpc.dp_tabulate_tc_work_bytes(model.info, w.nloc, 0, w.ntypes, w.M1)
+
+
+def test_tc_water_large_chunk_edges():
+    """The default f64 path at its largest size: 1,048,576 atoms in 256 chunks, in the benchmark's launch
+    configuration.  The oracle on 256 atoms gathered on the device: the first and last atom of 24
+    chunks spread over the run (edges from the 1st chunk to the 256th, byte offsets into R~ and dR~ past
+    2^32) and random atoms; the FP64-pipe moment path on every atom, compared on the device; and
+    the identity <dR~, R~> = <dT, T> over every atom, which holds at any size."""
+    dpc = lib()
+    w = workload("water_large")
+    nchunks = -(-w.nloc // CHUNK)
+    assert nchunks >= 64
+    model = product_model(w, F64)
+    x = to_dev(w, F64)
+    args = (model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
+    T = dpc.dp_tabulate_fusion_fwd_tc_f64(*args)
+    ds, dRt = dpc.dp_tabulate_fusion_grad_tc_f64(*args, x["dT"])
+    torch.cuda.synchronize()
+    edges = []
+    for c in np.unique(np.r_[1, 2, 3, np.linspace(4, nchunks - 1, 21).astype(int)]):
+        edges += [c * CHUNK - 1, min(c * CHUNK, w.nloc - 1)]
+    rest = np.random.default_rng(17).choice(w.nloc, 256 - len(edges) - 2, replace=False)
+    atoms = np.unique(np.r_[0, w.nloc - 1, edges, rest])
+    idx = torch.from_numpy(atoms).cuda()
+    got = {k: v.index_select(0, idx).cpu().numpy() for k, v in dict(T=T, ds=ds, dRt=dRt).items()}
+    assert_parity(got, run_oracle(w, F64, atoms=atoms), F64, keys=("T", "ds", "dRt"))
+    lhs = float((dRt * x["Rt"]).sum())
+    rhs = float((x["dT"] * T).sum())
+    assert abs(lhs - rhs) <= TOL[F64] * 10 * max(1.0, abs(rhs)), (lhs, rhs)
+    Tp = dpc.dp_tabulate_fusion_fwd_moments(*args)
+    d = float((Tp - T).abs().max() / Tp.abs().max())
+    assert d <= CLOSE, ("T", d)
+    del Tp
+    dsp, dRtp = dpc.dp_tabulate_fusion_grad_moments(*args, x["dT"])
+    for k, a, b in (("ds", ds, dsp), ("dRt", dRt, dRtp)):
+        d = float((a - b).abs().max() / b.abs().max())
+        assert d <= CLOSE, (k, d)
+    del T, ds, dRt, dsp, dRtp, x, model
+    torch.cuda.empty_cache()
