@@ -39,7 +39,7 @@ import numpy as np  # noqa: E402
 
 METRIC = "tabulate-fusion fwd+grad neighbour·channel evals/s (fp64) and % of roofline"
 UNIT = "evals/s"
-NSM = 152
+NSM = 152  # GB300; run_native reads the device's own count and passes it on
 SM_MAX_MHZ = 2070.0
 # FP64 / FP32 FMA lanes per SM per clock: GB300 is specified at 1.25 TFLOP/s FP64
 # (2 lanes/clk/SM at 2.07 GHz over 152 SMs) and 128 FP32 lanes/clk/SM.
@@ -158,9 +158,9 @@ TC_CHUNK_ATOMS = 4104  # atoms per chunk of the tc calls
 
 
 def tc_profile_events(w) -> int:
-    """Events one step of the tc calls records: a start and a mark after the coefficients per call,
-    then per chunk forward runs, split, and per centre type GEMM and epilogue; backward runs, dT split,
-    per type GEMM, rows."""
+    """Events one step of the tc calls records (an upper bound): a start per call, then per chunk forward
+    runs, split, and per centre type GEMM and epilogue; backward runs (unless the forward's are reused),
+    dT split, per type GEMM, rows."""
     chunks = -(-w.nloc // TC_CHUNK_ATOMS)
     return min(4096, 4 + chunks * (2 + 2 * w.ntypes + 3 + w.ntypes) + 8)
 
@@ -178,25 +178,66 @@ def moment_fmas(runs, M1: int) -> dict:
 
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
-# `ncu --set full` capture of its current version (profiles/<kernel>_<algo>_<workload>_<dtype>.md);
-# absent means no capture of the current kernel exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,
-                       ("cu85", "f64", "tc_rows", "tc"): 140379392 + 95468544}
+# `ncu --set full` capture of its current version; absent means no capture of the current kernel
+# exists and `traffic` is reported as null.
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640}
 
 
-def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ) -> float:
+def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ, nsm: int = NSM) -> float:
     """FMA-pipe peak in TFLOP/s (an FMA = 2 flop); for df64 the FP32 pipe's rate of df64 FMAs."""
     if dtype == "df64":
-        return NSM * FMA_LANES["f32"] * 2 * mhz * 1e6 / 1e12 / DF64_OPS_PER_FMA
-    return NSM * FMA_LANES[dtype] * 2 * mhz * 1e6 / 1e12
+        return nsm * FMA_LANES["f32"] * 2 * mhz * 1e6 / 1e12 / DF64_OPS_PER_FMA
+    return nsm * FMA_LANES[dtype] * 2 * mhz * 1e6 / 1e12
 
 
-def peak_basis(dtype: str) -> str:
+def peak_basis(dtype: str, nsm: int = NSM) -> str:
     if dtype == "df64":
-        return (f"FP32 pipe: {NSM} SMs x {FMA_LANES['f32']} lanes/clk x {SM_MAX_MHZ:.0f} MHz / "
+        return (f"FP32 pipe: {nsm} SMs x {FMA_LANES['f32']} lanes/clk x {SM_MAX_MHZ:.0f} MHz / "
                 f"{DF64_OPS_PER_FMA} FP32 instructions per df64 FMA, x 2 flop")
-    return (f"FP{64 if dtype == 'f64' else 32} FMA pipe: {NSM} SMs x {FMA_LANES[dtype]} lanes/clk x 2 flop x "
-            f"{SM_MAX_MHZ:.0f} MHz")
+    return (f"FP{64 if dtype == 'f64' else 32} FMA pipe: {nsm} SMs (the device's count) x {FMA_LANES[dtype]} "
+            f"lanes/clk x 2 flop x {SM_MAX_MHZ:.0f} MHz")
+
+
+def hbm_peak() -> tuple:
+    """(GB/s, basis): the measured copy bandwidth, else the stated fallback."""
+    path = os.path.join(os.path.dirname(os.path.abspath(__file__)), "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured copy bandwidth (MEASURED_PEAKS.json)"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback 6.8 TB/s"
+
+
+def step_bytes(w, esize: int) -> dict:
+    """Algorithmic DRAM bytes of one fwd + descriptor + grad step: the forward reads s and R~ of the valid
+    rows and writes T; the descriptor reads T and writes D; the backward reads s and R~ of the valid rows
+    and dE/dT and writes ds and dR~ of every row (padding included); tables are L2-resident."""
+    rows = float(w.evals) / w.M1
+    t = 4 * w.M1 * esize * w.nloc
+    return {"fwd": 5 * esize * rows + t, "descriptor": t + w.M1 * w.M2 * esize * w.nloc,
+            "grad": 5 * esize * rows + t + 5 * esize * w.nloc * w.nnei}
+
+
+def tc_step_bound(w, nruns: float, nsm: int, ms_step: float) -> dict:
+    """The roofline of the step the tensor-core path runs: the slowest of its FP64-pipe work (the per-row
+    moments, 24 FMA, and derivatives, 40 FMA, per valid row, and the descriptor's 4 M1 M2 per atom) at the
+    FP64 peak, its digit-product MMAs (24 M1 FMA per run and direction, 45 fp16 products each) at the
+    measured dense 16-bit tensor peak, and its algorithmic bytes at the measured HBM bandwidth."""
+    rows = float(w.evals) / w.M1
+    fp64_fma = (24 + 40) * rows + DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc
+    tensor_flop = 2.0 * TC_DIGIT_PRODUCTS * 2 * 24 * w.M1 * float(nruns)
+    hbm, hbasis = hbm_peak()
+    tpk, tbasis = tensor_peak()
+    t = {"fp64": 2.0 * fp64_fma / (peak_tflops("f64", nsm=nsm) * 1e12) * 1e3,
+         "tensor": tensor_flop / (tpk * 1e12) * 1e3,
+         "hbm": sum(step_bytes(w, 8).values()) / (hbm * 1e9) * 1e3}
+    bound = max(t, key=t.get)
+    return {"t_roof_ms": round(t[bound], 4), "bound": bound, "fp64_ms": round(t["fp64"], 4),
+            "tensor_ms": round(t["tensor"], 4), "hbm_ms": round(t["hbm"], 4), "ms_per_step": round(ms_step, 4),
+            "frac": round(t[bound] / ms_step, 4),
+            "basis": (f"fwd + descriptor + grad as the tc path computes them: FP64 {fp64_fma:.4g} FMA "
+                      f"({peak_basis('f64', nsm)}); tensor {tensor_flop:.4g} flop ({tbasis}); "
+                      f"{sum(step_bytes(w, 8).values()):.4g} B ({hbasis})")}
 
 
 def rank_seed(seed: int, rank: int) -> int:
@@ -306,15 +347,16 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     import workloads as W
     fwd = dpc.dp_tabulate_fusion_fwd_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_fwd
     grad = dpc.dp_tabulate_fusion_grad_moments if args.algo == "moments" else dpc.dp_tabulate_fusion_grad
-    if args.algo == "tc":  # the per-interval contraction on the tensor cores; its scratch stays resident
+    if args.algo == "tc":  # the per-interval contraction on the tensor cores; plan and scratch stay resident
         tcw = torch.empty((dpc.dp_tabulate_tc_work_bytes(info, w.nloc, w.nnei, w.ntypes, w.M1),), dtype=torch.uint8,
                           device=dev)
+        plan = dpc.dp_tabulate_tc_plan_f64(model.table, info, w.nnei)  # setup, once per table (like the build)
 
-        def fwd(*a, out=None):
-            return dpc.dp_tabulate_fusion_fwd_tc_f64(*a, out=out, work=tcw)
+        def fwd(table, *a, out=None):
+            return dpc.dp_tabulate_fusion_fwd_tc_f64(plan, *a, out=out, work=tcw)
 
-        def grad(*a, out=None):
-            return dpc.dp_tabulate_fusion_grad_tc_f64(*a, out=out, work=tcw)
+        def grad(table, *a, out=None):  # on the forward's inputs: it takes the forward's interval runs
+            return dpc.dp_tabulate_fusion_grad_tc_f64(plan, *a, out=out, work=tcw, flags=dpc.DP_TC_REUSE_RUNS)
     arith = dpc.DF64 if args.dtype == "df64" else None  # the table picks the fusion kernels' arithmetic
     T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
     D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
@@ -410,6 +452,7 @@ def run_native(args, rank, world, local_rank):
 
     dev = torch.device("cuda", local_rank)
     torch.cuda.set_device(dev)
+    args.nsm = int(torch.cuda.get_device_properties(dev).multi_processor_count)  # the peaks use the device's count
     dtype = torch.float32 if args.dtype == "f32" else torch.float64
     npdt = np.float32 if args.dtype == "f32" else np.float64
     kw = {}
@@ -487,7 +530,7 @@ def run_native(args, rank, world, local_rank):
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
     nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
     tcf = tc_fmas(w, interval_runs(w, info, *dpc.dp_table_info_sizes(info))) if tc_ms else None
-    per_mark = {"tc_coef_split": 1 + 2 * w.ntypes, "tc_split_dT": 2, "tc_fwd": 0, "tc_grad": 0}  # kernels per mark
+    per_mark = {"tc_split_dT": 2, "tc_fwd": 0, "tc_grad": 0}  # kernels per mark
     out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall, tc_ms, tcf,
                  [sum(per_mark.get(x, 1) for x in nm) for nm in pnames])
     if graph is not None:
@@ -566,7 +609,7 @@ def measure_variants(args, w, dpc, info, sel, d, ref_outs, flush, stream, dev, f
         torch.cuda.synchronize(dev)
         ms = {n: sum(e[j].elapsed_time(e[j + 1]) for e in evs) / nsteps for j, n in enumerate(("fwd", "descriptor", "grad"))}
         tot = sum(ms.values())
-        pk = peak_tflops("df64" if arith else "f64")
+        pk = peak_tflops("df64" if arith else "f64", nsm=getattr(args, "nsm", NSM))
         fm = fmas if name.endswith("moments") else {"fwd": FMA_PER_EVAL["fwd"] * w.evals,
                                                      "grad": FMA_PER_EVAL["grad"] * w.evals}
         diff = {k: float(((o[k] - ref_outs[k]).abs().max() / ref_outs[k].abs().max()).item()) for k in ref_outs}
@@ -654,7 +697,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     if getattr(args, "fitting", False):
         flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w)[0]).items()})
     nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
-    pk = peak_tflops(args.dtype)
+    nsm = getattr(args, "nsm", NSM)
+    pk = peak_tflops(args.dtype, nsm=nsm)
     tc = bool(getattr(args, "fitting_tc", False))
     tpk, tbasis = tensor_peak()
     kernels = {}
@@ -676,7 +720,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     roofline = {"bound": "alu", "achieved": round(achieved, 4), "peak": round(pk, 4), "unit": "TFLOP/s",
                 "frac": round(achieved / pk, 4), "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
                 "kernel": api,
-                "peak_basis": peak_basis(args.dtype),
+                "peak_basis": peak_basis(args.dtype, nsm),
                 "fwd_grad_frac": round(path_tflops / pk, 4)}
     if tc and dom.startswith("fitting"):
         roofline.update({"bound": "tensor", "achieved": kernels[dom]["tensor_tflops"], "peak": round(tpk, 1),
@@ -706,8 +750,10 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                         "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
                         "kernel": TC_KERNEL[dom],
                         "peak_basis": (f"{tbasis}; achieved counts all {TC_DIGIT_PRODUCTS} fp16 digit products"
-                                       if gemm else peak_basis(args.dtype)),
+                                       if gemm else peak_basis(args.dtype, nsm)),
                         "fwd_grad_frac_fp64_equivalent": round(path_tflops / pk, 4)}
+        if not args.chain:  # the whole step against the bound of the algorithm it runs
+            roofline["step"] = tc_step_bound(w, tcf["tc_gemm_fwd"] / (24.0 * w.M1), nsm, step_mean)
     out = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": sum(step_ms) / len(step_ms), "higher_is_better": True,
@@ -729,6 +775,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                    **({"fitting_gemm": ("tensor cores (tcgen05): f64 by exact 9-digit splitting, fp16 MMAs"
                                         if tc else "FP64 pipe")} if getattr(args, "fitting", False) else {}),
                    "evals_per_step_per_gpu": w.evals, "atoms_per_step_per_gpu": w.nloc, "fill": round(w.fill, 4),
+                   "device_sms": nsm,
                    "footprint": footprint(w, 4 if args.dtype == "f32" else 8)},
         "atoms_per_s": w.nloc * world * args.steps / total_s,
         "roofline": roofline,

@@ -236,8 +236,9 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
 
 /*
  * The f64 forward and backward with the per-interval contraction on the
- * tensor cores (tcgen05).  Same arguments, results, limits and errors as
- * dp_tabulate_fusion_fwd_f64 / dp_tabulate_fusion_grad_f64, plus a work
+ * tensor cores (tcgen05).  Same inputs, results, limits and errors as
+ * dp_tabulate_fusion_fwd_f64 / dp_tabulate_fusion_grad_f64, with the table
+ * replaced by a plan made from it once (dp_tabulate_tc_plan_f64) and a work
  * buffer.  With u = t / Delta_l in [0, 1] (Delta_l = stride0 on the fine
  * grid, stride1 on the coarse one) and c'_q = c_q Delta_l^q, the interval
  * moments of the rows of atom i,
@@ -252,24 +253,69 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  * nine 6-bit digits per element, scaled by the row's or column's power of
  * two, fp16 MMAs with exact fp32 sums (at most 448 of K per partial sum),
  * one rounding to f64; per output the error is below about
- * K 2^-50 max|row| max|column| (K: the used intervals x 8, or M1).  Only
+ * K 2^-50 max|row| max|column| (K: the used intervals x 6, or M1).  Only
  * the intervals some atom of a 12-atom tile uses enter its GEMM.  Rows need
  * not be sorted, though sorted rows (one run per interval) do the least
  * FP64 work.  NaN s gives NaN in that atom's T (forward) and in that row's
  * ds and dRt (backward); inf or NaN in dT gives NaN in the atom's rows.
+ *
+ * The plan holds the scaled coefficients c'_q / nnei of every centre type
+ * and their digit planes for both GEMMs; it depends only on the table, its
+ * info, nnei, ntypes and M1, so a caller makes it once per table (it is
+ * setup, like the table build) and passes it to every call.
+ *   dp_tabulate_tc_plan_bytes  the size of its device buffer (0 on bad sizes).
+ *   dp_tabulate_tc_plan_f64    fills `buf` (device, caller-owned, 256-byte
+ *                              aligned, at least that many bytes) from the
+ *                              table [ntypes*ntypes][nint][M1][6] (as
+ *                              dp_table_build_f64 writes it), asynchronously
+ *                              on `stream`, and the host record *plan (the
+ *                              buffer, its size and the geometry it was made
+ *                              for, which every call checks against its own
+ *                              arguments: DP_ERR_SHAPE if they differ).  The
+ *                              buffer must not change while calls use it.
  *   work, work_bytes  device scratch, caller-owned, 256-byte aligned, at
  *                     least dp_tabulate_tc_work_bytes(info, nloc, nnei,
  *                     ntypes, M1) bytes (one size for both directions): the
- *                     scaled coefficients and their digit planes (rebuilt
- *                     on every call), the moments or their gradients per
- *                     (atom, interval), flags of the used intervals, and
- *                     partial results, for chunks of at most 4104 atoms.
- *                     Calls sharing a work buffer must not overlap on the GPU.
+ *                     slot keys (int16, one per interval an atom uses), their
+ *                     counts and the used-slice flags of every atom (kept
+ *                     from the forward for the backward), and for one chunk
+ *                     of at most 4104 atoms the moments or their gradients
+ *                     per (atom, interval), the B digit planes and partial
+ *                     results.  Calls sharing a work buffer must not overlap
+ *                     on the GPU.
+ *   flags (backward)  0, or DP_TC_REUSE_RUNS: the forward call on the same
+ *                     plan, s, nvalid, atype, nloc and work buffer ran before
+ *                     this call on the stream, and nothing has written the
+ *                     work buffer or those inputs since; the backward then
+ *                     takes the forward's slot keys and slice flags instead
+ *                     of finding them again.  The library cannot check this
+ *                     contract; broken, the results are wrong.
  * Extra errors: DP_ERR_NULL / DP_ERR_SHAPE for a missing, short or
- * misaligned work buffer; DP_ERR_UNSUPPORTED for more than 4096 intervals
- * per centre type (ntypes x nint), whose per-atom key map would not fit in
- * shared memory.
+ * misaligned work or plan buffer, or a plan made for another geometry;
+ * DP_ERR_SHAPE for unknown flags; DP_ERR_UNSUPPORTED for more than 4096
+ * intervals per centre type (ntypes x nint), whose per-atom key map would
+ * not fit in shared memory.
  */
+typedef struct dp_tc_plan {
+  const void *data;   /* the plan's device buffer */
+  size_t bytes;       /* its size */
+  dp_table_info info; /* the geometry it was made for */
+  int32_t nnei, ntypes, M1;
+} dp_tc_plan;
+#define DP_TC_REUSE_RUNS 1
+size_t dp_tabulate_tc_plan_bytes(const dp_table_info *info, int nnei, int ntypes, int M1);
+int dp_tabulate_tc_plan_f64(const double *table, const dp_table_info *info, int nnei, int ntypes, int M1, void *buf,
+                            size_t bytes, dp_tc_plan *plan, void *stream);
+size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nnei, int ntypes,
+                                 int M1); /* 0 on bad sizes or table info */
+int dp_tabulate_fusion_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
+                                  const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                  const int32_t *sel, int M1, double *T, void *work, size_t work_bytes, void *stream);
+int dp_tabulate_fusion_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
+                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
+                                   const int32_t *sel, int M1, const double *dT, double *ds, double *dRt, void *work,
+                                   size_t work_bytes, int flags, void *stream);
+
 /*
  * Kernel timing hook, for profiling (off by default; not thread-safe: one
  * profiling session per process).  dp_profile_begin hands the library n
@@ -287,15 +333,17 @@ int dp_profile_begin(void *const *events, int n);
 int dp_profile_end(void);
 const char *dp_profile_name(int i);
 
-size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nnei, int ntypes,
-                                 int M1); /* 0 on bad sizes or table info */
-int dp_tabulate_fusion_fwd_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
-                                  const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
-                                  const int32_t *sel, int M1, double *T, void *work, size_t work_bytes, void *stream);
-int dp_tabulate_fusion_grad_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
-                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
-                                   const int32_t *sel, int M1, const double *dT, double *ds, double *dRt, void *work,
-                                   size_t work_bytes, void *stream);
+/*
+ * Diagnostic (not part of the paper's method): every wait of the tensor-core
+ * GEMM kernels (dp_tabulate_fusion_*_tc_f64, dp_fitting_*_tc_f64) on an
+ * mbarrier is bounded; a CTA whose wait gives up writes NaN outputs, reads
+ * no accumulator and counts one timeout on the device.  This call waits for
+ * the device to finish (cudaDeviceSynchronize), writes the count since the
+ * last call to *count (host) and clears it.  0 in normal operation.
+ * Errors: DP_ERR_NULL, DP_ERR_CUDA.
+ */
+int dp_tc_wait_timeouts(unsigned int *count);
+
 
 /*
  * Descriptor (Sec. II): with S_i = T_i^T (M1 x 4) and S_i^< its first M2

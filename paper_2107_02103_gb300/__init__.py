@@ -40,6 +40,16 @@ class dp_table_info(ctypes.Structure):
                 f"stride0={self.stride0!r}, stride1={self.stride1!r})")
 
 
+class dp_tc_plan(ctypes.Structure):
+    """Host record of a tensor-core tabulation plan (mirror of the C struct): its device buffer and the
+    geometry it was made for."""
+    _fields_ = [("data", ctypes.c_void_p), ("bytes", ctypes.c_size_t), ("info", dp_table_info),
+                ("nnei", ctypes.c_int32), ("ntypes", ctypes.c_int32), ("M1", ctypes.c_int32)]
+
+
+DP_TC_REUSE_RUNS = 1
+
+
 class dp_env_info(ctypes.Structure):
     """Environment-matrix parameters (mirror of the C struct): cutoffs, switch kind, normalisation."""
     _fields_ = [("rcs", ctypes.c_double), ("rc", ctypes.c_double), ("kind", ctypes.c_int32),
@@ -66,6 +76,7 @@ _P = ctypes.c_void_p
 _I32, _I64, _D = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
 _INFO = ctypes.POINTER(dp_table_info)
 _ENV = ctypes.POINTER(dp_env_info)
+_PLAN = ctypes.POINTER(dp_tc_plan)
 _SIGS = {
     "dp_last_error": ([], ctypes.c_char_p),
     "dp_table_info_make": ([_D, _D, _D, _D, _D, _INFO], ctypes.c_int),
@@ -96,11 +107,16 @@ _SIGS = {
     "dp_profile_begin": ([_P, ctypes.c_int], ctypes.c_int),
     "dp_profile_end": ([], ctypes.c_int),
     "dp_profile_name": ([ctypes.c_int], ctypes.c_char_p),
+    "dp_tc_wait_timeouts": ([ctypes.POINTER(ctypes.c_uint)], ctypes.c_int),
     "dp_tabulate_tc_work_bytes": ([_INFO, _I64, ctypes.c_int, ctypes.c_int, ctypes.c_int], ctypes.c_size_t),
-    "dp_tabulate_fusion_fwd_tc_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+    "dp_tabulate_tc_plan_bytes": ([_INFO, ctypes.c_int, ctypes.c_int, ctypes.c_int], ctypes.c_size_t),
+    "dp_tabulate_tc_plan_f64": ([_P, _INFO, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, ctypes.c_size_t, _PLAN,
+                                 _P], ctypes.c_int),
+    "dp_tabulate_fusion_fwd_tc_f64": ([_PLAN, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                        ctypes.c_int, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
-    "dp_tabulate_fusion_grad_tc_f64": ([_P, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
-                                        ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
+    "dp_tabulate_fusion_grad_tc_f64": ([_PLAN, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                        ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t, ctypes.c_int, _P],
+                                       ctypes.c_int),
     "dp_env_mat_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_env_mat_f32": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_f64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
@@ -234,10 +250,7 @@ def _sel_arr(sel):
     return (ctypes.c_int32 * len(sel))(*sel), len(sel), sum(sel)
 
 
-def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
-    df = isinstance(table, torch.Tensor) and is_df64_table(table)
-    table = _dev(table, "table", None)
-    dtype = torch.float64 if df else table.dtype
+def _fusion_arrays(dtype, s, Rt, nvalid, atype, sel):
     s = _dev(s, "s", dtype)
     nloc, nnei = (int(x) for x in s.shape)
     Rt = _dev(Rt, "Rt", dtype, (nloc, nnei, 4))
@@ -248,6 +261,14 @@ def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
         nvalid = _dev(nvalid, "nvalid", torch.int32, (nloc, ntypes))
     if atype is not None:
         atype = _dev(atype, "atype", torch.int32, (nloc,))
+    return s, Rt, nvalid, atype, selc, ntypes, nloc, nnei
+
+
+def _fusion_inputs(table, s, Rt, nvalid, atype, sel):
+    df = isinstance(table, torch.Tensor) and is_df64_table(table)
+    table = _dev(table, "table", None)
+    dtype = torch.float64 if df else table.dtype
+    s, Rt, nvalid, atype, selc, ntypes, nloc, nnei = _fusion_arrays(dtype, s, Rt, nvalid, atype, sel)
     if table.dim() != 5 or table.shape[-3] != 3 or table.shape[-1] != (4 if df else 2):
         raise ValueError("table must be [npair][nint][3][M1][2] (or [..][4] for df64) from dp_table_build")
     M1 = int(table.shape[-2])
@@ -355,6 +376,13 @@ def dp_profile_end():
     return [_lib.dp_profile_name(i).decode() for i in range(n)]
 
 
+def dp_tc_wait_timeouts() -> int:
+    """Tensor-core GEMM waits that gave up since the last call (synchronises the device); 0 normally."""
+    n = ctypes.c_uint(0)
+    _check(_lib.dp_tc_wait_timeouts(ctypes.byref(n)))
+    return int(n.value)
+
+
 def dp_tabulate_tc_work_bytes(info: dp_table_info, nloc, nnei, ntypes, M1) -> int:
     """Bytes of device scratch dp_tabulate_fusion_{fwd,grad}_tc_f64 need (one size for both)."""
     n = int(_lib.dp_tabulate_tc_work_bytes(ctypes.byref(info), int(nloc), int(nnei), int(ntypes), int(M1)))
@@ -372,33 +400,84 @@ def _tab_tc_work(work, info, nloc, nnei, ntypes, M1, device):
     return work
 
 
-def _tc_inputs(table, s, Rt, nvalid, atype, sel):
-    r = _fusion_inputs(table, s, Rt, nvalid, atype, sel)
-    if r[-1] != torch.float64:
-        raise TypeError("the tensor-core calls take an f64 table and f64 arrays")
-    return r
+class TcPlan:
+    """A tensor-core tabulation plan: the device buffer dp_tabulate_tc_plan_f64 filled (kept alive here)
+    and its host record."""
+
+    def __init__(self, buf: torch.Tensor, rec: dp_tc_plan):
+        self.buf, self.rec = buf, rec
+
+    @property
+    def info(self) -> dp_table_info:
+        return self.rec.info
 
 
-def dp_tabulate_fusion_fwd_tc_f64(table, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None, work=None):
+def dp_tabulate_tc_plan_bytes(info: dp_table_info, nnei, ntypes, M1) -> int:
+    """Bytes of the device buffer of a tensor-core tabulation plan."""
+    n = int(_lib.dp_tabulate_tc_plan_bytes(ctypes.byref(info), int(nnei), int(ntypes), int(M1)))
+    if n == 0:
+        raise ValueError(_lib.dp_last_error().decode())
+    return n
+
+
+def dp_tabulate_tc_plan_f64(table, info: dp_table_info, nnei, ntypes=None, buf=None) -> TcPlan:
+    """The plan of an f64 table [ntypes^2][nint][3][M1][2] for rows of nnei neighbours (setup, once per
+    table): its scaled coefficients and their digit planes; buf: a uint8 CUDA tensor or None."""
+    table = _dev(table, "table", torch.float64)
+    if table.dim() != 5:
+        raise ValueError("table must be [ntypes^2][nint][3][M1][2]")
+    npair, M1 = int(table.shape[0]), int(table.shape[3])
+    ntypes = int(round(npair ** 0.5)) if ntypes is None else int(ntypes)
+    if ntypes * ntypes != npair:
+        raise ValueError("table must hold ntypes^2 pair tables")
+    need = dp_tabulate_tc_plan_bytes(info, nnei, ntypes, M1)
+    if buf is None:
+        buf = torch.empty((need,), dtype=torch.uint8, device=table.device)
+    elif not buf.is_cuda or buf.dtype != torch.uint8 or not buf.is_contiguous() or buf.numel() < need:
+        raise ValueError(f"buf must be a contiguous CUDA uint8 tensor of at least {need} bytes")
+    rec = dp_tc_plan()
+    _check(_lib.dp_tabulate_tc_plan_f64(_ptr(table), ctypes.byref(info), int(nnei), ntypes, M1, _ptr(buf),
+                                        buf.numel(), ctypes.byref(rec), _stream(table)))
+    return TcPlan(buf, rec)
+
+
+def _tc_inputs(plan, info, s, Rt, nvalid, atype, sel):
+    """The call's checked arrays and its plan: a TcPlan as given, or one made now from an f64 table."""
+    if isinstance(plan, TcPlan):
+        s, Rt, nvalid, atype, selc, ntypes, nloc, nnei = _fusion_arrays(torch.float64, s, Rt, nvalid, atype, sel)
+        M1 = int(plan.rec.M1)
+    else:
+        dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, arith = _fusion_inputs(plan, s, Rt, nvalid,
+                                                                                                 atype, sel)
+        if arith != torch.float64:
+            raise TypeError("the tensor-core calls take an f64 table and f64 arrays")
+        plan = dp_tabulate_tc_plan_f64(table, info, nnei, ntypes)
+    return plan, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, torch.float64
+
+
+def dp_tabulate_fusion_fwd_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None, work=None):
     """T of dp_tabulate_fusion_fwd in f64 with the per-interval contraction on the tensor cores (interval
-    moments times the scaled table, an exact digit-split GEMM); work: a uint8 CUDA tensor of
+    moments times the scaled table, an exact digit-split GEMM).  plan: a TcPlan (dp_tabulate_tc_plan_f64)
+    or the f64 table itself, planned for this call; work: a uint8 CUDA tensor of
     dp_tabulate_tc_work_bytes(...) bytes, or None to allocate one."""
-    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, _ = _tc_inputs(table, s, Rt, nvalid, atype, sel)
+    plan, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, dtype = _tc_inputs(plan, info, s, Rt, nvalid, atype, sel)
     shape = (nloc, 4, M1)
     T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
     if nloc == 0:
         return T
     work = _tab_tc_work(work, info, nloc, nnei, ntypes, M1, s.device)
-    _check(_lib.dp_tabulate_fusion_fwd_tc_f64(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid),
-                                              _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(T), _ptr(work),
-                                              work.numel(), _stream(s)))
+    _check(_lib.dp_tabulate_fusion_fwd_tc_f64(ctypes.byref(plan.rec), ctypes.byref(info), _ptr(s), _ptr(Rt),
+                                              _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(T),
+                                              _ptr(work), work.numel(), _stream(s)))
     return T
 
 
-def dp_tabulate_fusion_grad_tc_f64(table, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None, work=None):
+def dp_tabulate_fusion_grad_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None, work=None,
+                                   flags=0):
     """(ds, dRt) of dp_tabulate_fusion_grad in f64 with the per-interval contraction on the tensor cores;
-    work as dp_tabulate_fusion_fwd_tc_f64."""
-    dtype, table, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, _ = _tc_inputs(table, s, Rt, nvalid, atype, sel)
+    plan and work as dp_tabulate_fusion_fwd_tc_f64; flags=DP_TC_REUSE_RUNS takes the interval runs the
+    forward left in `work` for the same inputs (see include/dp_compress.h)."""
+    plan, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, dtype = _tc_inputs(plan, info, s, Rt, nvalid, atype, sel)
     dT = _dev(dT, "dT", dtype, (nloc, 4, M1))
     if out is None:
         ds = torch.empty((nloc, nnei), dtype=dtype, device=s.device)
@@ -408,10 +487,13 @@ def dp_tabulate_fusion_grad_tc_f64(table, info: dp_table_info, s, Rt, nvalid, at
         dRt = _dev(out[1], "dRt", dtype, (nloc, nnei, 4))
     if nloc == 0:
         return ds, dRt
+    if flags and work is None:
+        raise ValueError("DP_TC_REUSE_RUNS needs the forward's work buffer")
     work = _tab_tc_work(work, info, nloc, nnei, ntypes, M1, s.device)
-    _check(_lib.dp_tabulate_fusion_grad_tc_f64(_ptr(table), ctypes.byref(info), _ptr(s), _ptr(Rt), _ptr(nvalid),
-                                               _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(dT), _ptr(ds),
-                                               _ptr(dRt), _ptr(work), work.numel(), _stream(s)))
+    _check(_lib.dp_tabulate_fusion_grad_tc_f64(ctypes.byref(plan.rec), ctypes.byref(info), _ptr(s), _ptr(Rt),
+                                               _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(dT),
+                                               _ptr(ds), _ptr(dRt), _ptr(work), work.numel(), int(flags),
+                                               _stream(s)))
     return ds, dRt
 
 

@@ -19,6 +19,8 @@ int set_error(int code, const char *fmt, ...);  // stores the message, returns c
 void clear_error();
 int launch_status(const char *what);  // DP_ERR_CUDA if the last launch failed
 void prof_mark(const char *name, cudaStream_t st);  // kernel timing hook (dp_profile_begin)
+int take_wait_timeouts_tabulate(unsigned int *count);  // GEMM wait timeouts per unit (dp_tc_wait_timeouts)
+int take_wait_timeouts_fitting(unsigned int *count);
 
 // --------------------------------------------------------- table geometry
 // dp_table_info with its derived sizes and reciprocal steps.

@@ -143,6 +143,15 @@ int dp_profile_end(void) {
 
 const char *dp_profile_name(int i) { return i >= 0 && i < dpc::g_prof.n ? dpc::g_prof.name[i] : ""; }
 
+int dp_tc_wait_timeouts(unsigned int *count) {
+  dpc::clear_error();
+  if (!count) return dpc::set_error(DP_ERR_NULL, "dp_tc_wait_timeouts: count is NULL");
+  *count = 0;
+  int rc = dpc::take_wait_timeouts_tabulate(count);
+  if (!rc) rc = dpc::take_wait_timeouts_fitting(count);
+  return rc;
+}
+
 int dp_table_info_make(double s_min, double s_max, double stride0, double stride1, double ext, dp_table_info *out) {
   dpc::clear_error();
   if (!out) return dpc::set_error(DP_ERR_NULL, "out is NULL");

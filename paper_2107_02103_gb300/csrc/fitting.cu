@@ -718,6 +718,10 @@ int fitting_grad_noalloc(const double *params, const int32_t *widths, int nlayer
 }
 
 }  // namespace
+
+// This unit's GEMM wait timeouts (see tc_gemm.cuh), for dp_tc_wait_timeouts.
+int take_wait_timeouts_fitting(unsigned int *count) { return tc::take_wait_timeouts(count); }
+
 }  // namespace dpc
 
 extern "C" {

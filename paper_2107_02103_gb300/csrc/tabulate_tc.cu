@@ -26,16 +26,18 @@
 // interval an atom uses, found through a per-atom map), and the GEMMs skip the
 // slices (forward) or output tiles (backward) that no atom of a tile uses.
 //
+// C'_alpha and its digit planes are made once per table by dp_tabulate_tc_plan_f64 (the plan).
 // Per chunk of at most kChunkAtoms atoms and per centre type alpha:
-//   forward:  runs_kernel<true> (map, W, column exponents, slice flags),
+//   forward:  runs_kernel<true> (slot keys, W, column exponents, slice flags),
 //             split_mom_kernel (W -> B digit planes, used slices only),
 //             gemm_kernel (A = C'_alpha^T: channels x K, B = W^T: K x (atom, k); a tile whose
 //             used slices fit one share writes its atoms' T directly),
 //             fwd_epilogue_kernel (T of the tiles with several shares, or none);
-//   backward: runs_kernel<false> (map, tile flags), split of dT (B), gemm_kernel
-//             (A = C'_alpha: K x channels, B = dT^T) scattering each used
-//             (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
-// C'_alpha and its digit planes are made per call from the table.
+//   backward: runs_kernel<false> (slot keys, slice flags; skipped when the forward's are reused),
+//             split of dT (B), gemm_kernel (A = C'_alpha: K x channels, B = dT^T) scattering
+//             each used (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
+// The slot keys, their counts and the slice flags of every atom stay in the work buffer after
+// the forward, so that a backward on the same inputs can skip its own key pass.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -58,7 +60,7 @@ constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' res
 constexpr int kMaxKeys = 4096;  // ntypes x nint: each warp's key map (int16) lives in shared memory
 static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
 
-// Sizes shared by the kernels and the work-buffer layout.
+// Sizes shared by the kernels, the plan and the work-buffer layout.
 struct Shape {
   int ntypes, nint, nkeys, M1, cap;
   int Kp;    // round_up(6 nkeys, 16): K of the forward GEMM, rows of the backward A
@@ -66,27 +68,48 @@ struct Shape {
   int Mpf;   // round_up(M1, 128): rows of the forward A
   int Kpm;   // round_up(M1, 16): K of the backward GEMM
   int Mpb;   // round_up(Kp, 128): rows of the backward A
+  int64_t nloc, tiles_all;    // atoms of the call and their 12-atom tiles
   int64_t chunk, Np, ntiles;  // atoms per chunk, its columns round_up(4 chunk, 48), Np / 48
   int zmax;                   // forward shares per tile at most
 };
 
-struct Layout {
-  size_t cp, afwd, efwd, abwd, ebwd, map, keys, nslots, occ, fexp, bplanes, w, part, total;
+// The plan: C' of every centre type and the digit planes of both GEMMs' A operands.
+struct PlanLayout {
+  size_t nodes, cp, afwd, efwd, abwd, ebwd, total;
 };
 
-Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1) {
+// The work buffer: the slot keys, their counts and the slice flags of every atom of the call
+// (kept from the forward for the backward), then one chunk's scratch.
+struct Layout {
+  size_t keys, nslots, occ, map, fexp, bplanes, w, part, total;
+};
+
+size_t take(size_t &off, size_t bytes) {
+  const size_t at = off;
+  off += (size_t)round_up((int64_t)bytes, 256);
+  return at;
+}
+
+Shape table_shape(const TableGeom &g, int ntypes, int M1) {
   Shape s{};
   s.ntypes = ntypes;
   s.nint = g.nint;
   s.nkeys = ntypes * g.nint;
   s.M1 = M1;
-  s.cap = std::min(nnei, s.nkeys);
   s.Kp = (int)round_up((int64_t)s.nkeys * kQ, kTK);
   s.nsl = s.Kp / kTK;
   s.Mpf = (int)round_up(M1, kTM);
   s.Kpm = (int)round_up(M1, kTK);
   s.Mpb = (int)round_up(s.Kp, kTM);
   s.zmax = (s.nsl + kShareSlices - 1) / kShareSlices;
+  return s;
+}
+
+Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1) {
+  Shape s = table_shape(g, ntypes, M1);
+  s.cap = std::min(nnei, s.nkeys);
+  s.nloc = nloc;
+  s.tiles_all = (nloc + kTileAtoms - 1) / kTileAtoms;
   int64_t chunk = std::min<int64_t>(round_up(std::max<int64_t>(nloc, 1), kTileAtoms), kChunkAtoms);
   while (chunk > kTileAtoms &&
          (size_t)s.zmax * s.Mpf * round_up(kCols * chunk, kTN) * sizeof(float4) > kPartBudget)
@@ -97,28 +120,31 @@ Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1)
   return s;
 }
 
+PlanLayout plan_layout(const Shape &s) {
+  PlanLayout L{};
+  size_t off = 0;
+  const size_t nt = (size_t)s.ntypes;
+  L.nodes = take(off, (size_t)(s.nint + 1) * sizeof(double));
+  L.cp = take(off, nt * s.Kp * s.M1 * sizeof(double));
+  L.afwd = take(off, nt * kS * (size_t)s.Mpf * s.Kp * 2);
+  L.efwd = take(off, nt * s.Mpf * sizeof(int));
+  L.abwd = take(off, nt * kS * (size_t)s.Mpb * s.Kpm * 2);
+  L.ebwd = take(off, nt * s.Mpb * sizeof(int));
+  L.total = off;
+  return L;
+}
+
 Layout make_layout(const Shape &s) {
   Layout L{};
   size_t off = 0;
-  auto take = [&](size_t bytes) {
-    const size_t at = off;
-    off += (size_t)round_up((int64_t)bytes, 256);
-    return at;
-  };
-  const size_t nt = (size_t)s.ntypes;
-  L.cp = take(nt * s.Kp * s.M1 * sizeof(double));
-  L.afwd = take(nt * kS * (size_t)s.Mpf * s.Kp * 2);
-  L.efwd = take(nt * s.Mpf * sizeof(int));
-  L.abwd = take(nt * kS * (size_t)s.Mpb * s.Kpm * 2);
-  L.ebwd = take(nt * s.Mpb * sizeof(int));
-  L.map = take((size_t)s.chunk * s.nkeys * sizeof(int));
-  L.keys = take((size_t)s.chunk * s.cap * sizeof(int));
-  L.nslots = take((size_t)s.chunk * sizeof(int));
-  L.occ = take(nt * s.ntiles * std::max(s.nsl, s.Mpb / kTM));
-  L.fexp = take((size_t)s.Np * sizeof(int));
-  L.bplanes = take((size_t)s.ntiles * std::max(s.nsl, s.Kpm / kTK) * kS * kPlaneB);
-  L.w = take((size_t)s.chunk * s.cap * 24 * sizeof(float4));  // backward float4 slots; forward doubles fit
-  L.part = take((size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
+  L.keys = take(off, (size_t)std::max<int64_t>(s.nloc, 1) * s.cap * sizeof(short));
+  L.nslots = take(off, (size_t)std::max<int64_t>(s.nloc, 1) * sizeof(int));
+  L.occ = take(off, (size_t)s.ntypes * std::max<int64_t>(s.tiles_all, 1) * s.nsl);
+  L.map = take(off, (size_t)s.chunk * s.nkeys * sizeof(int));
+  L.fexp = take(off, (size_t)s.Np * sizeof(int));
+  L.bplanes = take(off, (size_t)s.ntiles * std::max(s.nsl, s.Kpm / kTK) * kS * kPlaneB);
+  L.w = take(off, (size_t)s.chunk * s.cap * 24 * sizeof(float4));  // backward float4 slots; forward doubles fit
+  L.part = take(off, (size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
   L.total = off;
   return L;
 }
@@ -149,21 +175,69 @@ __global__ void __launch_bounds__(256) coef_kernel(const double *__restrict__ ta
   }
 }
 
+// The grid's nodes x_0 .. x_nint as the interval search forms them (node_x), for the per-row kernels.
+__global__ void nodes_kernel(TableGeom g, double *__restrict__ nodes) {
+  for (int l = blockIdx.x * blockDim.x + threadIdx.x; l <= g.nint; l += gridDim.x * blockDim.x) nodes[l] = node_x(g, l);
+}
+
+// An f32 value within 2^-23 (relative) of s, formed from the fields of s by integer operations (no
+// FP64 instruction); ok is false where that fails: |s| outside [2^-100, 2^100), zero, inf, NaN.
+__device__ __forceinline__ float approx_f32(double s, bool &ok) {
+  const unsigned hi = (unsigned)__double2hiint(s), lo = (unsigned)__double2loint(s);
+  const int e = (int)((hi >> 20) & 0x7ff) - 1023;
+  ok = e > -100 && e < 100;
+  return __uint_as_float((hi & 0x80000000u) | ((unsigned)(e + 127) << 23) | ((hi & 0xfffffu) << 3) | (lo >> 29));
+}
+
+// floor(x) clamped into [0, n], for x below 2^22, on the FP32 pipe: 2^23 added with rounding down.
+__device__ __forceinline__ int floor_clamped(float x, int n) {
+  return __float_as_int(__fadd_rd(fminf(fmaxf(x, 0.0f), (float)n), 8388608.0f)) - 0x4B000000;
+}
+
+// The interval search of the tensor-core path's per-row kernels.  The segment and the index come from
+// the f32 approximation of s; t = s - x_l is one f64 subtraction from the node table.  The f32 index can
+// differ from floor((s - x_0) / Delta) by one where s lies within ~1e-4 steps of a node; either interval
+// is correct there (the table is C2, so both polynomials agree to the rounding at the node, and t then
+// lies a hair outside [0, Delta]).  Inputs within 2^-18 (relative) of lower, upper or upper_ext, where
+// the f32 comparison could take the wrong side, and inputs outside the f32 range take the f64 search,
+// whose clamping they follow exactly.  Deterministic: the forward and the backward find the same l.
+__device__ __forceinline__ int locate_fast(const TableGeom &g, const TableGeomF &f, const double *__restrict__ nodes,
+                                           double s, double &t, bool &clamped) {
+  bool ok;
+  const float sf = approx_f32(s, ok);
+  const float tol = 0x1p-18f * fabsf(sf);
+  if (!ok || fabsf(sf - f.lower) <= tol || fabsf(sf - f.upper) <= tol || fabsf(sf - f.upper_ext) <= tol)
+    return locate(g, s, t, clamped);
+  clamped = sf < f.lower || sf >= f.upper_ext;
+  if (sf < f.lower) {
+    t = 0.0;
+    return 0;
+  }
+  if (sf >= f.upper_ext) {
+    t = g.n1 > 0 ? g.stride1 : g.stride0;
+    return g.nint - 1;
+  }
+  const int l = sf < f.upper ? floor_clamped((sf - f.lower) * f.inv0, g.n0 - 1)
+                             : g.n0 + floor_clamped((sf - f.upper) * f.inv1, g.n1 - 1);
+  t = s - __ldg(nodes + l);
+  return l;
+}
+
 struct RunsParams {
   const double *s, *Rt;
   const int32_t *nvalid, *atype;
   TableGeom g;
-  int64_t atom0, natoms, ntiles;
-  int nnei, ntypes, nkeys, cap;
+  TableGeomF gf;
+  const double *nodes;  // [nint + 1] (the plan's)
+  int64_t atom0, natoms, tiles_all;  // the chunk's first atom (a multiple of 12) and size; all tiles
+  int nnei, ntypes, nkeys, cap, nsl;
   int sel[DP_MAX_TYPES];
-  int *map;            // [natoms][nkeys]: run slot of the key, or -1
-  int *keys;           // [natoms][cap]: key of each slot
-  int *nslots;         // [natoms]: slots in use
+  short *keys;         // [nloc][cap]: key of each slot (every atom of the call)
+  int *nslots;         // [nloc]: slots in use
+  unsigned char *occ;  // [ntypes][tiles_all][nsl]: the K slices some atom of the tile uses
+  int *map;            // forward: [natoms][nkeys] run slot of the key, or -1 (this chunk)
   double *W;           // forward: [natoms][cap][24] moments W[k][q] at 6 k + q
   int *fexp;           // forward: [Np] exponents of the columns 4 a + k
-  unsigned char *occ;  // [ntypes][ntiles][occ_cols]
-  int occ_cols;        // forward: K slices; backward: 128-row tiles of the backward A
-  int unit;            // K entries (rows) per flag: 16 (a slice) or 128 (a tile)
 };
 
 struct alignas(16) RunsStage {
@@ -207,9 +281,9 @@ __device__ __forceinline__ int valid_row(int v, const int *nvb, const int *sel, 
 
 // One warp per atom: the runs of rows sharing an interval (consecutive rows with one key; rows
 // sorted by distance give one run per interval, and a key met again adds to its slot), each
-// interval's slot (a shared-memory map of the keys, copied out at the end with each slot's key and
-// the slot count) and its flag for the atom's tile; forward also its moments W and the atom's four
-// column exponents (over every value written, which bounds the final ones).
+// interval's slot (a shared-memory map of the keys; each slot's key and the slot count are written
+// out) and the flags of its K slices for the atom's tile; forward also the map, its moments W and
+// the atom's four column exponents (over every value written, which bounds the final ones).
 // Warps (one atom each) per block of the runs and rows kernels: a few per block, so that launching
 // thousands of tiny blocks does not set the pace of a short kernel.
 constexpr int kRunsWarps = 4, kRowsWarps = 2;
@@ -227,8 +301,8 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
   for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
   const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the reset)
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
-  unsigned char *occ = P.occ + ((size_t)alpha * P.ntiles + (size_t)(a / kTileAtoms)) * P.occ_cols;
-  int *keys = P.keys + a * P.cap;
+  unsigned char *occ = P.occ + ((size_t)alpha * P.tiles_all + (size_t)(i / kTileAtoms)) * P.nsl;
+  short *keys = P.keys + i * P.cap;
   double *Wa = kMom ? P.W + (size_t)a * P.cap * 24 : nullptr;
   int nslot = 0;
   int cur = -1;       // key of the open run (uniform)
@@ -242,9 +316,9 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
       slot = nslot++;
       if (lane == 0) {
         smap[cur] = (short)slot;
-        keys[slot] = cur;
-        occ[kQ * cur / P.unit] = 1;  // the key's entries 6 key .. 6 key + 5, in one or two units
-        occ[(kQ * cur + kQ - 1) / P.unit] = 1;
+        keys[slot] = (short)cur;
+        occ[kQ * cur / kTK] = 1;  // the key's entries 6 key .. 6 key + 5, in one or two slices
+        occ[(kQ * cur + kQ - 1) / kTK] = 1;
       }
     }
     if (kMom && lane < 24) {
@@ -264,7 +338,7 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
       const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
       double t;
       bool clamped;
-      const int l = locate(P.g, __ldg(srow + row), t, clamped);
+      const int l = locate_fast(P.g, P.gf, P.nodes, __ldg(srow + row), t, clamped);
       st.key[lane] = b * P.g.nint + l;
       if constexpr (kMom) {
         const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
@@ -305,10 +379,10 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
     __syncwarp();
   }
   if (cur >= 0) flush();
-  int *map = P.map + a * P.nkeys;
-  for (int k = lane; k < P.nkeys; k += 32) map[k] = smap[k];
-  if (lane == 0) P.nslots[a] = nslot;
+  if (lane == 0) P.nslots[i] = nslot;
   if constexpr (kMom) {
+    int *map = P.map + a * P.nkeys;
+    for (int k = lane; k < P.nkeys; k += 32) map[k] = smap[k];
     int m = eb;  // per k: the largest over its six lanes
 #pragma unroll
     for (int q = 1; q < 6; ++q) m = max(m, __shfl_sync(0xffffffffu, eb, min(lane + q, 31)));
@@ -322,8 +396,9 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
 __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict__ W, const int *__restrict__ map,
                                                         const int *__restrict__ fexp,
                                                         const unsigned char *__restrict__ occ, int ntypes,
-                                                        int64_t ntiles, int64_t natoms, int nkeys, int cap,
-                                                        int64_t rows_p, int Kp, unsigned char *__restrict__ planes) {
+                                                        int64_t tiles_all, int64_t tile0, int64_t natoms, int nkeys,
+                                                        int cap, int64_t rows_p, int Kp,
+                                                        unsigned char *__restrict__ planes) {
   const int lane = threadIdx.x & 31, ri8 = lane >> 2, kp = lane & 3;
   const int kchunks = (Kp + kSplitK - 1) / kSplitK;
   const int nsl = Kp / kTK;
@@ -342,7 +417,7 @@ __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict
   for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
     const int sl = k0 / kTK;
     bool used = false;
-    for (int t = 0; t < ntypes; ++t) used |= occ[((size_t)t * ntiles + tile) * nsl + sl] != 0;
+    for (int t = 0; t < ntypes; ++t) used |= occ[((size_t)t * tiles_all + tile0 + tile) * nsl + sl] != 0;
     if (!used) continue;  // uniform
     const int kk = k0 + 2 * kp;  // this lane's two entries, of one key (6 is even)
     const int key = kk / kQ, q0 = kk - kQ * key;
@@ -411,12 +486,15 @@ struct RowsParams {
   const double *s, *Rt;
   const int32_t *nvalid, *atype;
   TableGeom g;
+  TableGeomF gf;
+  const double *nodes;  // [nint + 1] (the plan's)
   int64_t atom0;
   int nnei, ntypes, nkeys, cap;
   int sel[DP_MAX_TYPES];
-  const int *map, *keys, *nslots;
+  const short *keys;   // [nloc][cap]: key of each slot
+  const int *nslots;   // [nloc]
   float4 *dW;          // [natoms][cap][24]: the backward GEMM's result per slot (four floats), then in place
-                       // (dW, q dW / Delta) as two doubles
+                       // dW as a double in the first half of each entry
   const int *eexp;     // [ntypes][Mpb]: exponents of the backward A's rows 6 key + q
   int Mpb;
   const int *fexp;     // [Np]: exponents of dT's rows 4 a + k
@@ -426,17 +504,15 @@ struct RowsParams {
 
 struct alignas(16) RowsStage {
   double r[32][4];
-  double u[32];
-  double dw[32][24];   // per run of the batch: dW[k][q] at 6 k + q
-  double dwq[32][24];  // q dW[k][q] / Delta_l
-  int slot[32], run[32], clamped[32], row[32], rslot[32];
+  double u[32], dinv[32];  // u and 1 / Delta_l of each staged row
+  double dw[32][24];       // per run of the batch: dW[k][q] at 6 k + q
+  int run[32], clamped[32], row[32], rslot[32];
   int nvb[DP_MAX_TYPES];
-  double qinv[2][kQ];  // q / Delta on the fine and the coarse grid
 };
 
 // One warp per atom: every slot's dW finished from the GEMM's four floats (all lanes, in place),
 // then per 32-row batch the batch's runs copied to shared memory and each valid row's dE/dR~ and
-// dE/ds by Horner's rule in u (a lane per row); padded rows get zeros.
+// dE/ds by Horner's rule in u with its derivative (a lane per row); padded rows get zeros.
 __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams P) {
   __shared__ RowsStage stw[kRowsWarps];
   extern __shared__ short smapw[];  // [kRowsWarps][nkeys]
@@ -446,25 +522,20 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
   RowsStage &st = stw[warp];
   short *smap = smapw + (size_t)warp * P.nkeys;
   const int64_t i = P.atom0 + a;
-  const int *gmap = P.map + a * P.nkeys;
-  for (int k = lane; k < P.nkeys; k += 32) smap[k] = (short)gmap[k];
-  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);
+  const short *keys = P.keys + i * P.cap;
+  const int nslot = P.nslots[i];
+  for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
+  __syncwarp();
+  for (int x = lane; x < nslot; x += 32) smap[keys[x]] = (short)x;  // the map of the atom's keys
+  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the map)
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   const int *eexp = P.eexp + (size_t)alpha * P.Mpb;
-  const int *keys = P.keys + a * P.cap;
   float4 *dWa = P.dW + (size_t)a * P.cap * 24;
-  double2 *dWd = reinterpret_cast<double2 *>(dWa);
-  const int nslot = P.nslots[a];
-  if (lane < 2 * kQ) st.qinv[lane / kQ][lane % kQ] = (double)(lane % kQ) * (lane < kQ ? P.g.inv0 : P.g.inv1);
-  __syncwarp();
-  for (int x = lane; x < nslot * 24; x += 32) {
+  for (int x = lane; x < nslot * 24; x += 32) {  // each lane rewrites only the entry it read
     const int sl = x / 24, j = x - 24 * sl, k = j / 6, q = j - 6 * k;
-    const int key = keys[sl];
-    const int l = key % P.g.nint;
     Sum3 acc;
     acc.add(dWa[x]);
-    const double d = acc.value(eexp[key * kQ + q], P.fexp[kCols * a + k]);
-    dWd[x] = make_double2(d, d * st.qinv[l < P.g.n0 ? 0 : 1][q]);
+    *reinterpret_cast<double *>(dWa + x) = acc.value(eexp[keys[sl] * kQ + q], P.fexp[kCols * a + k]);
   }
   __syncwarp();
   const double *srow = P.s + i * P.nnei;
@@ -479,13 +550,15 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
       const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
       double t;
       bool clamped;
-      const int l = locate(P.g, __ldg(srow + row), t, clamped);
+      const int l = locate_fast(P.g, P.gf, P.nodes, __ldg(srow + row), t, clamped);
       const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
       st.r[lane][0] = rr.x;
       st.r[lane][1] = rr.y;
       st.r[lane][2] = rr.z;
       st.r[lane][3] = rr.w;
-      st.u[lane] = t * (l < P.g.n0 ? P.g.inv0 : P.g.inv1);
+      const double dinv = l < P.g.n0 ? P.g.inv0 : P.g.inv1;
+      st.u[lane] = t * dinv;
+      st.dinv[lane] = dinv;
       mykey = b * P.g.nint + l;
       st.clamped[lane] = clamped;
       st.row[lane] = row;
@@ -501,31 +574,29 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
     __syncwarp();
     for (int x = lane; x < nrun * 24; x += 32) {
       const int r = x / 24, j = x - 24 * r;
-      const double2 w = dWd[(size_t)st.rslot[r] * 24 + j];
-      st.dw[r][j] = w.x;
-      st.dwq[r][j] = w.y;
+      st.dw[r][j] = *reinterpret_cast<const double *>(dWa + (size_t)st.rslot[r] * 24 + j);
     }
     __syncwarp();
     if (lane < cnt) {
-      const double *dw = st.dw[st.run[lane]], *dq = st.dwq[st.run[lane]];
+      const double *dw = st.dw[st.run[lane]];
       const double u = st.u[lane];
       double d4[4], ds = 0.0;
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const double *c = dw + 6 * k, *cq = dq + 6 * k;
-        double h = fma(c[5], u, c[4]);
-        h = fma(h, u, c[3]);
-        h = fma(h, u, c[2]);
-        h = fma(h, u, c[1]);
-        d4[k] = fma(h, u, c[0]);
-        double gq = fma(cq[5], u, cq[4]);
-        gq = fma(gq, u, cq[3]);
-        gq = fma(gq, u, cq[2]);
-        gq = fma(gq, u, cq[1]);
-        ds = fma(st.r[lane][k], gq, ds);
+      for (int k = 0; k < 4; ++k) {  // P_k(u) = sum_q dW[k][q] u^q and P_k'(u): 5 + 4 FMA
+        const double *c = dw + 6 * k;
+        double p = fma(c[5], u, c[4]), dp = c[5];
+        dp = fma(dp, u, p);
+        p = fma(p, u, c[3]);
+        dp = fma(dp, u, p);
+        p = fma(p, u, c[2]);
+        dp = fma(dp, u, p);
+        p = fma(p, u, c[1]);
+        dp = fma(dp, u, p);
+        d4[k] = fma(p, u, c[0]);
+        ds = fma(st.r[lane][k], dp, ds);
       }
       const int row = st.row[lane];
-      dsrow[row] = st.clamped[lane] ? 0.0 : ds;
+      dsrow[row] = st.clamped[lane] ? 0.0 : ds * st.dinv[lane];
       st4(drow + (size_t)row * 4, d4[0], d4[1], d4[2], d4[3]);
     }
     __syncwarp();
@@ -548,95 +619,155 @@ int check_work(const Layout &L, const void *work, size_t nbytes, const char *who
   return DP_OK;
 }
 
+// Sizes of a plan for this geometry; DP_OK or an error (message set).
+int plan_shape(const dp_table_info *info, int nnei, int ntypes, int M1, TableGeom *g, Shape *S, const char *who) {
+  int rc = make_geom(info, g);
+  if (rc) return rc;
+  if (nnei < 1 || ntypes < 1 || ntypes > DP_MAX_TYPES || M1 < 1 || M1 > DP_MAX_M1)
+    return set_error(DP_ERR_SHAPE, "%s: nnei %d, ntypes %d, M1 %d out of range", who, nnei, ntypes, M1);
+  if ((int64_t)ntypes * g->nint > kMaxKeys)
+    return set_error(DP_ERR_UNSUPPORTED, "%s: ntypes x nint = %lld intervals per centre type, at most %d", who,
+                     (long long)ntypes * g->nint, kMaxKeys);
+  *S = table_shape(*g, ntypes, M1);
+  return DP_OK;
+}
+
+// The plan of a call: present, large enough and made for the call's geometry (checked on the host).
+int check_plan(const dp_tc_plan *plan, const dp_table_info *info, int nnei, int ntypes, int M1, const Shape &S,
+               const char *who) {
+  if (!plan || !plan->data) return set_error(DP_ERR_NULL, "%s: plan is NULL", who);
+  const dp_table_info &a = plan->info;
+  if (a.lower != info->lower || a.upper != info->upper || a.upper_ext != info->upper_ext ||
+      a.stride0 != info->stride0 || a.stride1 != info->stride1 || plan->nnei != nnei || plan->ntypes != ntypes ||
+      plan->M1 != M1)
+    return set_error(DP_ERR_SHAPE, "%s: the plan was made for another table info, nnei, ntypes or M1", who);
+  if (plan->bytes < plan_layout(S).total) return set_error(DP_ERR_SHAPE, "%s: plan buffer too short", who);
+  return DP_OK;
+}
+
 // C' of every centre type from the table, then its digit planes: forward A = C'^T (rows: the
 // channels, K: 6 key + q), backward A = C' (rows: 6 key + q, K: the channels).
-int prep(const double *table, const TableGeom &g, const Shape &s, const Layout &L, unsigned char *wk, bool fwd,
-         int nnei, cudaStream_t st, const char *who) {
-  double *Cp = reinterpret_cast<double *>(wk + L.cp);
+int make_plan(const double *table, const dp_table_info *info, int nnei, int ntypes, int M1, void *buf,
+              size_t bytes, dp_tc_plan *out, void *stream) {
+  clear_error();
+  static const char *who = "dp_tabulate_tc_plan_f64";
+  TableGeom g;
+  Shape s{};
+  int rc = plan_shape(info, nnei, ntypes, M1, &g, &s, who);
+  if (rc) return rc;
+  if (!table || !buf || !out) return set_error(DP_ERR_NULL, "%s: table, plan buffer or plan is NULL", who);
+  const PlanLayout P = plan_layout(s);
+  if (bytes < P.total) return set_error(DP_ERR_SHAPE, "%s: plan buffer holds %zu bytes, needs %zu", who, bytes, P.total);
+  if (reinterpret_cast<uintptr_t>(buf) % 256) return set_error(DP_ERR_SHAPE, "%s: plan buffer is not 256-byte aligned", who);
+  const cudaStream_t st = (cudaStream_t)stream;
+  unsigned char *wk = static_cast<unsigned char *>(buf);
+  nodes_kernel<<<(unsigned)((g.nint + 256) / 256), 256, 0, st>>>(g, reinterpret_cast<double *>(wk + P.nodes));
+  if ((rc = launch_status(who))) return rc;
+  double *Cp = reinterpret_cast<double *>(wk + P.cp);
   const int64_t total = (int64_t)s.ntypes * s.Kp * s.M1;
-  coef_kernel<<<(unsigned)std::min<int64_t>((total + 255) / 256, 152 * 16), 256, 0, st>>>(table, g, s.ntypes, s.M1,
-                                                                                          s.Kp, 1.0 / (double)nnei, Cp);
-  int rc = launch_status(who);
+  coef_kernel<<<(unsigned)std::min<int64_t>((total + 255) / 256, 1 << 16), 256, 0, st>>>(table, g, s.ntypes, s.M1, s.Kp,
+                                                                                        1.0 / (double)nnei, Cp);
+  rc = launch_status(who);
   for (int t = 0; t < s.ntypes && !rc; ++t) {
     const double *Ct = Cp + (size_t)t * s.Kp * s.M1;
-    rc = fwd ? split_rows(Ct, 1, s.M1, s.M1, s.Kp, s.Mpf, s.Kp, kTM, wk + L.afwd + (size_t)t * kS * s.Mpf * s.Kp * 2,
-                          wk + L.efwd + (size_t)t * s.Mpf * sizeof(int), st, who)
-             : split_rows(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM, wk + L.abwd + (size_t)t * kS * s.Mpb * s.Kpm * 2,
-                          wk + L.ebwd + (size_t)t * s.Mpb * sizeof(int), st, who);
+    rc = split_rows(Ct, 1, s.M1, s.M1, s.Kp, s.Mpf, s.Kp, kTM, wk + P.afwd + (size_t)t * kS * s.Mpf * s.Kp * 2,
+                    wk + P.efwd + (size_t)t * s.Mpf * sizeof(int), st, who);
+    if (!rc)
+      rc = split_rows(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM, wk + P.abwd + (size_t)t * kS * s.Mpb * s.Kpm * 2,
+                      wk + P.ebwd + (size_t)t * s.Mpb * sizeof(int), st, who);
   }
-  return rc;
+  if (rc) return rc;
+  out->data = buf;
+  out->bytes = bytes;
+  out->info = *info;
+  out->nnei = nnei;
+  out->ntypes = ntypes;
+  out->M1 = M1;
+  return DP_OK;
 }
 
 RunsParams runs_params(const double *s, const double *Rt, const int32_t *nvalid, const int32_t *atype,
                        const TableGeom &g, const Segments &seg, const Shape &S, const Layout &L, unsigned char *wk,
-                       int nnei) {
+                       int nnei, const double *nodes) {
   RunsParams R{};
   R.s = s;
   R.Rt = Rt;
   R.nvalid = nvalid;
   R.atype = atype;
   R.g = g;
+  R.gf = to_f32(g);
   R.nnei = nnei;
   R.ntypes = S.ntypes;
   R.nkeys = S.nkeys;
   R.cap = S.cap;
+  R.nsl = S.nsl;
+  R.tiles_all = S.tiles_all;
   for (int b = 0; b < DP_MAX_TYPES; ++b) R.sel[b] = seg.sel[b];
-  R.map = reinterpret_cast<int *>(wk + L.map);
-  R.keys = reinterpret_cast<int *>(wk + L.keys);
+  R.keys = reinterpret_cast<short *>(wk + L.keys);
   R.nslots = reinterpret_cast<int *>(wk + L.nslots);
   R.occ = wk + L.occ;
+  R.map = reinterpret_cast<int *>(wk + L.map);
   R.fexp = reinterpret_cast<int *>(wk + L.fexp);
+  R.nodes = nodes;
   return R;
 }
 
-int fwd(const double *table, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
+// Validation shared by the forward and the backward; fills g, seg, S, L.
+int tc_args(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, int64_t nloc,
+            int nnei, int ntypes, const int32_t *sel, int M1, const void *out0, const void *out1, void *work,
+            size_t work_bytes, TableGeom *g, Segments *seg, Shape *S, Layout *L, const char *who) {
+  int rc = check_fusion_args(plan ? plan->data : nullptr, info, s, Rt, nloc, nnei, ntypes, sel, M1, out0, out1, g, seg);
+  if (rc || nloc == 0) return rc;
+  Shape T{};
+  if ((rc = plan_shape(info, nnei, ntypes, M1, g, &T, who))) return rc;
+  if ((rc = check_plan(plan, info, nnei, ntypes, M1, T, who))) return rc;
+  *S = make_shape(*g, nloc, nnei, ntypes, M1);
+  *L = make_layout(*S);
+  if ((rc = check_work(*L, work, work_bytes, who))) return rc;
+  return set_smem(who);
+}
+
+int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
         const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *work,
         size_t work_bytes, void *stream) {
   clear_error();
   static const char *who = "dp_tabulate_fusion_fwd_tc_f64";
   TableGeom g;
   Segments seg;
-  int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, T, &g, &seg);
-  if (rc) return rc;
-  if (nloc == 0) return DP_OK;
-  if ((int64_t)ntypes * g.nint > kMaxKeys)
-    return set_error(DP_ERR_UNSUPPORTED, "%s: ntypes x nint = %lld intervals per centre type, at most %d", who,
-                     (long long)ntypes * g.nint, kMaxKeys);
-  const Shape S = make_shape(g, nloc, nnei, ntypes, M1);
-  const Layout L = make_layout(S);
-  if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
+  Shape S{};
+  Layout L{};
+  int rc = tc_args(plan, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, T, work, work_bytes, &g, &seg, &S, &L, who);
+  if (rc || nloc == 0) return rc;
+  const PlanLayout PL = plan_layout(S);
+  const unsigned char *pk = static_cast<const unsigned char *>(plan->data);
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
   prof_mark("tc_fwd", st);
-  if ((rc = prep(table, g, S, L, wk, true, nnei, st, who))) return rc;
-  prof_mark("tc_coef_split", st);
-  RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
+  if (cudaMemsetAsync(wk + L.occ, 0, (size_t)ntypes * S.tiles_all * S.nsl, st) != cudaSuccess)
+    return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+  RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei,
+                             reinterpret_cast<const double *>(pk + PL.nodes));
   R.W = reinterpret_cast<double *>(wk + L.w);
-  R.occ_cols = S.nsl;
-  R.unit = kTK;
   float4 *part = reinterpret_cast<float4 *>(wk + L.part);
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
     const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
-    const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN;
-    const size_t occ_per_type = (size_t)ntiles * S.nsl;
-    if (cudaMemsetAsync(wk + L.occ, 0, (size_t)ntypes * occ_per_type, st) != cudaSuccess)
-      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+    const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN, tile0 = c0 / kTileAtoms;
     R.atom0 = c0;
     R.natoms = n;
-    R.ntiles = ntiles;
     runs_kernel<true><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
                         kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_runs_moments", st);
     const int64_t warps = Np / 8 * ((S.Kp + kSplitK - 1) / kSplitK);
-    split_mom_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(R.W, R.map, R.fexp, wk + L.occ, ntypes, ntiles, n,
-                                                                   S.nkeys, S.cap, Np, S.Kp, wk + L.bplanes);
+    split_mom_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(R.W, R.map, R.fexp, wk + L.occ, ntypes, S.tiles_all,
+                                                                   tile0, n, S.nkeys, S.cap, Np, S.Kp,
+                                                                   wk + L.bplanes);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_split_moments", st);
     for (int t = 0; t < ntypes; ++t) {
       TcGemm G{};
-      G.aplanes = wk + L.afwd + (size_t)t * kS * S.Mpf * S.Kp * 2;
-      G.Eexp = reinterpret_cast<const int *>(wk + L.efwd) + (size_t)t * S.Mpf;
+      G.aplanes = pk + PL.afwd + (size_t)t * kS * S.Mpf * S.Kp * 2;
+      G.Eexp = reinterpret_cast<const int *>(pk + PL.efwd) + (size_t)t * S.Mpf;
       G.Mp = S.Mpf;
       G.planes = wk + L.bplanes;
       G.Fexp = R.fexp;
@@ -644,7 +775,7 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
       G.Kp = S.Kp;
       G.part = part;
       G.slices_per_split = kShareSlices;
-      G.kocc = wk + L.occ + (size_t)t * occ_per_type;
+      G.kocc = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
       G.tout = T;  // tiles with one share write T themselves
       G.ldt = M1;
       G.natoms = n;
@@ -665,32 +796,30 @@ int fwd(const double *table, const dp_table_info *info, const double *s, const d
   return DP_OK;
 }
 
-int grad(const double *table, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
+int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
          const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, const double *dT,
-         double *ds, double *dRt, void *work, size_t work_bytes, void *stream) {
+         double *ds, double *dRt, void *work, size_t work_bytes, int flags, void *stream) {
   clear_error();
   static const char *who = "dp_tabulate_fusion_grad_tc_f64";
+  if (flags & ~DP_TC_REUSE_RUNS) return set_error(DP_ERR_SHAPE, "%s: unknown flags %#x", who, flags);
   TableGeom g;
   Segments seg;
-  int rc = check_fusion_args(table, info, s, Rt, nloc, nnei, ntypes, sel, M1, ds, dRt, &g, &seg);
-  if (rc) return rc;
-  if (nloc > 0 && !dT) return set_error(DP_ERR_NULL, "%s: dT is NULL", who);
-  if (nloc == 0) return DP_OK;
-  if ((int64_t)ntypes * g.nint > kMaxKeys)
-    return set_error(DP_ERR_UNSUPPORTED, "%s: ntypes x nint = %lld intervals per centre type, at most %d", who,
-                     (long long)ntypes * g.nint, kMaxKeys);
-  const Shape S = make_shape(g, nloc, nnei, ntypes, M1);
-  const Layout L = make_layout(S);
-  if ((rc = check_work(L, work, work_bytes, who)) || (rc = set_smem(who))) return rc;
+  Shape S{};
+  Layout L{};
+  int rc = tc_args(plan, info, s, Rt, nloc, nnei, ntypes, sel, M1, ds, dRt, work, work_bytes, &g, &seg, &S, &L, who);
+  if (rc || nloc == 0) return rc;
+  if (!dT) return set_error(DP_ERR_NULL, "%s: dT is NULL", who);
+  const PlanLayout PL = plan_layout(S);
+  const unsigned char *pk = static_cast<const unsigned char *>(plan->data);
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
+  const bool reuse = (flags & DP_TC_REUSE_RUNS) != 0;
   prof_mark("tc_grad", st);
-  if ((rc = prep(table, g, S, L, wk, false, nnei, st, who))) return rc;
-  prof_mark("tc_coef_split", st);
-  RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei);
+  if (!reuse && cudaMemsetAsync(wk + L.occ, 0, (size_t)ntypes * S.tiles_all * S.nsl, st) != cudaSuccess)
+    return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+  RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei,
+                             reinterpret_cast<const double *>(pk + PL.nodes));
   const int mtiles = S.Mpb / kTM;
-  R.occ_cols = mtiles;
-  R.unit = kTM;
   float4 *dW = reinterpret_cast<float4 *>(wk + L.w);
   RowsParams Q{};
   Q.s = s;
@@ -698,33 +827,32 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
   Q.nvalid = nvalid;
   Q.atype = atype;
   Q.g = g;
+  Q.gf = R.gf;
+  Q.nodes = R.nodes;
   Q.nnei = nnei;
   Q.ntypes = ntypes;
   Q.nkeys = S.nkeys;
   Q.cap = S.cap;
   for (int b = 0; b < DP_MAX_TYPES; ++b) Q.sel[b] = seg.sel[b];
-  Q.map = R.map;
   Q.keys = R.keys;
   Q.nslots = R.nslots;
   Q.dW = dW;
-  Q.eexp = reinterpret_cast<const int *>(wk + L.ebwd);
+  Q.eexp = reinterpret_cast<const int *>(pk + PL.ebwd);
   Q.Mpb = S.Mpb;
   Q.fexp = R.fexp;
   Q.ds = ds;
   Q.dRt = dRt;
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
     const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
-    const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN;
-    const size_t occ_per_type = (size_t)ntiles * mtiles;
-    if (cudaMemsetAsync(wk + L.occ, 0, (size_t)ntypes * occ_per_type, st) != cudaSuccess)
-      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+    const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN, tile0 = c0 / kTileAtoms;
     R.atom0 = c0;
     R.natoms = n;
-    R.ntiles = ntiles;
-    runs_kernel<false><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
-                         kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
-    if ((rc = launch_status(who))) return rc;
-    prof_mark("tc_runs", st);
+    if (!reuse) {
+      runs_kernel<false><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
+                           kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
+      if ((rc = launch_status(who))) return rc;
+      prof_mark("tc_runs", st);
+    }
     // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
     if ((rc = split_rows(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, Np, S.Kpm, kTN, wk + L.bplanes, wk + L.fexp, st,
                          who)))
@@ -732,7 +860,7 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
     prof_mark("tc_split_dT", st);
     for (int t = 0; t < ntypes; ++t) {
       TcGemm G{};
-      G.aplanes = wk + L.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
+      G.aplanes = pk + PL.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
       G.Eexp = Q.eexp + (size_t)t * S.Mpb;
       G.Mp = S.Mpb;
       G.planes = wk + L.bplanes;
@@ -740,9 +868,11 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
       G.Np = (int)Np;
       G.Kp = S.Kpm;
       G.slices_per_split = S.Kpm / kTK;
-      G.tocc = wk + L.occ + (size_t)t * occ_per_type;
+      G.sflags = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
+      G.nsf = S.nsl;
       G.scat = dW;
-      G.map = R.map;
+      G.keys = R.keys;
+      G.nslots = R.nslots;
       G.atype = atype;
       G.natoms = n;
       G.atom0 = c0;
@@ -769,18 +899,29 @@ int grad(const double *table, const dp_table_info *info, const double *s, const 
 size_t work_bytes_api(const dp_table_info *info, int64_t nloc, int nnei, int ntypes, int M1) {
   clear_error();
   TableGeom g;
-  if (make_geom(info, &g)) return 0;
-  if (nloc < 0 || nnei < 1 || ntypes < 1 || ntypes > DP_MAX_TYPES || M1 < 1 || M1 > DP_MAX_M1 ||
-      (int64_t)ntypes * g.nint > kMaxKeys) {
-    set_error(DP_ERR_SHAPE, "dp_tabulate_tc_work_bytes: nloc %lld, nnei %d, ntypes %d, M1 %d (%d intervals) out of range",
-              (long long)nloc, nnei, ntypes, M1, g.nint);
+  Shape S{};
+  if (nloc < 0) {
+    set_error(DP_ERR_SHAPE, "dp_tabulate_tc_work_bytes: nloc %lld < 0", (long long)nloc);
     return 0;
   }
+  if (plan_shape(info, nnei, ntypes, M1, &g, &S, "dp_tabulate_tc_work_bytes")) return 0;
   return make_layout(make_shape(g, nloc, nnei, ntypes, M1)).total;
+}
+
+size_t plan_bytes_api(const dp_table_info *info, int nnei, int ntypes, int M1) {
+  clear_error();
+  TableGeom g;
+  Shape S{};
+  if (plan_shape(info, nnei, ntypes, M1, &g, &S, "dp_tabulate_tc_plan_bytes")) return 0;
+  return plan_layout(S).total;
 }
 
 }  // namespace tt
 }  // namespace
+
+// This unit's GEMM wait timeouts (see tc_gemm.cuh), for dp_tc_wait_timeouts.
+int take_wait_timeouts_tabulate(unsigned int *count) { return tc::take_wait_timeouts(count); }
+
 }  // namespace dpc
 
 extern "C" {
@@ -789,19 +930,28 @@ size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nn
   return dpc::tt::work_bytes_api(info, nloc, nnei, ntypes, M1);
 }
 
-int dp_tabulate_fusion_fwd_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+size_t dp_tabulate_tc_plan_bytes(const dp_table_info *info, int nnei, int ntypes, int M1) {
+  return dpc::tt::plan_bytes_api(info, nnei, ntypes, M1);
+}
+
+int dp_tabulate_tc_plan_f64(const double *table, const dp_table_info *info, int nnei, int ntypes, int M1, void *buf,
+                            size_t bytes, dp_tc_plan *plan, void *stream) {
+  return dpc::tt::make_plan(table, info, nnei, ntypes, M1, buf, bytes, plan, stream);
+}
+
+int dp_tabulate_fusion_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
                                   const int32_t *sel, int M1, double *T, void *work, size_t work_bytes,
                                   void *stream) {
-  return dpc::tt::fwd(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, work, work_bytes, stream);
+  return dpc::tt::fwd(plan, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, work, work_bytes, stream);
 }
 
-int dp_tabulate_fusion_grad_tc_f64(const double *table, const dp_table_info *info, const double *s, const double *Rt,
+int dp_tabulate_fusion_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
                                    const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
                                    const int32_t *sel, int M1, const double *dT, double *ds, double *dRt, void *work,
-                                   size_t work_bytes, void *stream) {
-  return dpc::tt::grad(table, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, work, work_bytes,
-                       stream);
+                                   size_t work_bytes, int flags, void *stream) {
+  return dpc::tt::grad(plan, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, dT, ds, dRt, work, work_bytes,
+                       flags, stream);
 }
 
 }  // extern "C"

@@ -52,10 +52,11 @@ namespace {
 // operands (the tabulated embedding's interval moments): a per-tile list of the
 // K slices in use (the others are zero and are skipped; the shares then cut the
 // used slices, and a tile whose used slices fit one share can write its f64
-// outputs itself), and a per-tile flag that skips unwanted output tiles, whose
-// wanted outputs are scattered to per-run slots instead of a dense array.
+// outputs itself), and per-tile slice flags that skip unwanted output tiles,
+// whose wanted outputs are scattered to per-run slots instead of a dense array.
 // Every wait on an mbarrier is bounded; a wait that gives up makes the tile's
-// outputs NaN.
+// outputs NaN (the accumulators are not read) and counts one timeout in
+// g_wait_timeouts, which the host reads through dp_tc_wait_timeouts.
 namespace tc {
 constexpr int kS = 9;      // digits per operand element
 constexpr int kBits = 6;   // bits per digit
@@ -226,12 +227,16 @@ struct TcGemm {
   const unsigned char *kocc;  // [Np / kTN][Kp / kTK]: nonzero where the B tile has a nonzero entry in the
                               // slice; share z of a tile then takes its used slices z S .. z S + S - 1
                               // (S = slices_per_split), and a share past its last used slice writes nothing
-  const unsigned char *tocc;  // [Np / kTN][Mp / kTM]: nonzero where the output tile is wanted
-  // scatter (with tocc): output (row kq key + q, column 4 a + k), q < 6 <= kq, key < nkeys, a < natoms,
-  // goes to scat[(a cap + slot) 24 + 6 k + q] when slot = map[a nkeys + key] >= 0 and atom atom0 + a
-  // has type alpha (atype clamped into [0, ntypes)); nothing is written to part
+  const unsigned char *sflags;  // [Np / kTN][nsf]: flags of the K slices the atoms of a B tile use; output
+                                // tile (x, y) is wanted when one of slices 8 y .. 8 y + 7 is flagged
+  int nsf;
+  // scatter (with sflags): output (row kq key + q, column 4 a + k), q < 6 <= kq, key < nkeys, a < natoms,
+  // goes to scat[(a cap + slot) 24 + 6 k + q] when atom atom0 + a has type alpha (atype clamped into
+  // [0, ntypes)) and key is keys[(atom0 + a) cap + slot] for a slot < nslots[atom0 + a]; nothing is
+  // written to part
   float4 *scat;
-  const int *map;
+  const short *keys;
+  const int *nslots;
   const int32_t *atype;
   int64_t natoms, atom0;
   int nkeys, cap, alpha, ntypes, kq;
@@ -271,6 +276,20 @@ constexpr uint32_t kIdescNoN = (1u << 4) | ((uint32_t)(kTM >> 4) << 24);  // N >
 constexpr int kMaxPlanesPerMma = 256 / kTN;  // N <= 256 for M = 128
 static_assert(kTN % 16 == 0 && kMaxPlanesPerMma >= 1, "MMA N: multiples of 16 up to 256");
 
+// Bounded mbarrier waits that gave up, one count per CTA (this translation unit's kernels).
+__device__ unsigned int g_wait_timeouts;
+
+// The count, read after a device synchronisation, then cleared.
+int take_wait_timeouts(unsigned int *count) {
+  unsigned int v = 0, zero = 0;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaMemcpyFromSymbol(&v, g_wait_timeouts, sizeof v);
+  if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_wait_timeouts, &zero, sizeof zero);
+  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "dp_tc_wait_timeouts: %s", cudaGetErrorString(e));
+  *count += v;
+  return DP_OK;
+}
+
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   uint32_t done = 0;
   for (int it = 0; it < (1 << 24) && !done; ++it)
@@ -295,16 +314,30 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   const int n0 = blockIdx.x * kTN;
   const int nslices = P.Kp / kTK;
   const int i0 = blockIdx.z * P.slices_per_split;
-  if (P.tocc && !P.tocc[(size_t)blockIdx.x * gridDim.y + blockIdx.y]) return;  // unwanted tile (uniform)
-  if (P.scat)  // the tile's slots, loaded once and in parallel
-    for (int x = tid; x < kScatKeys * kScatAtoms; x += kThreads) {
-      const int key = (int)(m0 / P.kq) + x / kScatAtoms;
-      const int64_t a = (int64_t)(n0 / 4) + x % kScatAtoms;
-      int slot = -1;
-      if (key < P.nkeys && a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha))
-        slot = P.map[a * P.nkeys + key];
-      stab[x] = slot;
+  if (P.sflags) {  // an output tile no atom of the B tile uses is skipped (uniform)
+    const unsigned char *f = P.sflags + (size_t)blockIdx.x * P.nsf;
+    const int lo = (int)(m0 / kTK), hi = min(P.nsf, (int)((m0 + kTM) / kTK));
+    bool any = false;
+    for (int x = lo; x < hi; ++x) any |= f[x] != 0;
+    if (!any) return;
+  }
+  if (P.scat) {  // the tile's slots: (key of the tile, atom) -> slot, or -1
+    int *nsa = slist;  // the slot count of each atom of the tile (0: not of type alpha); slist is free here
+    for (int x = tid; x < kScatKeys * kScatAtoms; x += kThreads) stab[x] = -1;
+    if (tid < kScatAtoms) {
+      const int64_t a = (int64_t)(n0 / 4) + tid, i = P.atom0 + a;
+      nsa[tid] = a < P.natoms && (!P.atype || clampi(P.atype[i], 0, P.ntypes - 1) == P.alpha) ? P.nslots[i] : 0;
     }
+    __syncthreads();
+    const int key0 = (int)(m0 / P.kq);
+    for (int al = warp; al < kScatAtoms; al += kThreads / 32) {  // a warp per atom, its lanes over the slots
+      const short *keys = P.keys + (P.atom0 + n0 / 4 + al) * P.cap;
+      for (int slot = lane; slot < nsa[al]; slot += 32) {
+        const int key = keys[slot];
+        if (key >= key0 && key < key0 + kScatKeys) stab[(key - key0) * kScatAtoms + al] = slot;
+      }
+    }
+  }
   if (P.tout)
     for (int x = tid; x < kScatAtoms; x += kThreads) {
       const int64_t a = (int64_t)(n0 / 4) + x;
@@ -419,6 +452,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   __syncthreads();
   ok = flags[0] && flags[1];
   ok = mbar_wait(smem_u32(done), 0) && ok;
+  ok = __syncthreads_and(ok) != 0;  // one verdict for the CTA: its accumulators are read only if every wait ended
+  if (!ok && tid == 0) atomicAdd(&g_wait_timeouts, 1u);
   asm volatile("tcgen05.fence::after_thread_sync;");
 
   // combine the diagonals of row 32 (warp % 4) + lane (the warp's TMEM lane quadrant), the warp's
@@ -435,13 +470,20 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
 #pragma unroll 1
   for (int c0 = (warp >> 2) * kColsPerWarp; c0 < (warp >> 2) * kColsPerWarp + kColsPerWarp; c0 += 8) {
     float v[kS][8];
+    if (ok) {  // uniform over the CTA
 #pragma unroll
-    for (int d = 0; d < kS; ++d)
-      asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                   : "=f"(v[d][0]), "=f"(v[d][1]), "=f"(v[d][2]), "=f"(v[d][3]), "=f"(v[d][4]), "=f"(v[d][5]),
-                     "=f"(v[d][6]), "=f"(v[d][7])
-                   : "r"(trow + (uint32_t)(d * kTN + c0)));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+      for (int d = 0; d < kS; ++d)
+        asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                     : "=f"(v[d][0]), "=f"(v[d][1]), "=f"(v[d][2]), "=f"(v[d][3]), "=f"(v[d][4]), "=f"(v[d][5]),
+                       "=f"(v[d][6]), "=f"(v[d][7])
+                     : "r"(trow + (uint32_t)(d * kTN + c0)));
+      asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+    } else {
+#pragma unroll
+      for (int d = 0; d < kS; ++d)
+#pragma unroll
+        for (int c = 0; c < 8; ++c) v[d][c] = 0.0f;
+    }
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
       // sum_d v_d 64^-(d+2) as four floats on the FP32 pipe: diagonals 2 and 3 (d = 0, 1) as an exact

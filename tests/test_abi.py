@@ -135,3 +135,45 @@ def test_binding_rejects_cpu_tensors(dpc):
         dpc.dp_tabulate_fusion_fwd(torch.zeros(1, 10, 4, 6, dtype=torch.float64), info,
                                    torch.zeros(2, 3, dtype=torch.float64), torch.zeros(2, 3, 4, dtype=torch.float64),
                                    None, None, [3])
+
+
+def test_tc_plan_and_work_validation_without_gpu(dpc):
+    """The tensor-core calls refuse, on the host and before any CUDA call, a missing plan, a plan made for
+    another geometry or too short, a missing, short or misaligned work buffer, and unknown flags; the
+    plan builder refuses a missing, short or misaligned buffer.  The fake pointers are never dereferenced."""
+    lib = dpc._lib
+    info = dpc.dp_table_info_make(0.0, 1.05)
+    fake = ctypes.c_void_p(0x1000)
+    sel = (ctypes.c_int32 * 1)(8)
+    need = dpc.dp_tabulate_tc_plan_bytes(info, 8, 1, 16)
+    wb = dpc.dp_tabulate_tc_work_bytes(info, 5, 8, 1, 16)
+
+    def plan(**kw):
+        d = dict(data=0x1000, bytes=need, info=info, nnei=8, ntypes=1, M1=16)
+        d.update(kw)
+        return dpc.dp_tc_plan(**d)
+
+    def fwd(rec, work=fake, nbytes=wb):
+        return lib.dp_tabulate_fusion_fwd_tc_f64(None if rec is None else ctypes.byref(rec), ctypes.byref(info), fake,
+                                                 fake, None, None, 5, 8, 1, sel, 16, fake, work, nbytes, None)
+
+    def grad(rec, flags=0, work=fake, nbytes=wb):
+        return lib.dp_tabulate_fusion_grad_tc_f64(None if rec is None else ctypes.byref(rec), ctypes.byref(info),
+                                                  fake, fake, None, None, 5, 8, 1, sel, 16, fake, fake, fake, work,
+                                                  nbytes, flags, None)
+
+    assert fwd(None) == dpc.DP_ERR_NULL and grad(None) == dpc.DP_ERR_NULL
+    assert fwd(plan(data=None)) == dpc.DP_ERR_NULL
+    other = dpc.dp_table_info_make(0.0, 1.25)
+    for bad in (plan(nnei=9), plan(M1=32), plan(bytes=need - 1), plan(info=other)):
+        assert fwd(bad) == dpc.DP_ERR_SHAPE and grad(bad) == dpc.DP_ERR_SHAPE
+    assert fwd(plan(), work=None) == dpc.DP_ERR_NULL
+    assert fwd(plan(), nbytes=wb - 1) == dpc.DP_ERR_SHAPE
+    assert fwd(plan(), work=ctypes.c_void_p(0x1010)) == dpc.DP_ERR_SHAPE
+    assert grad(plan(), flags=2) == dpc.DP_ERR_SHAPE and "flags" in dpc.dp_last_error()
+    rec = dpc.dp_tc_plan()
+    build = lambda buf, n: lib.dp_tabulate_tc_plan_f64(fake, ctypes.byref(info), 8, 1, 16, buf, n,  # noqa: E731
+                                                       ctypes.byref(rec), None)
+    assert build(None, need) == dpc.DP_ERR_NULL
+    assert build(fake, need - 1) == dpc.DP_ERR_SHAPE
+    assert build(ctypes.c_void_p(0x1010), need) == dpc.DP_ERR_SHAPE

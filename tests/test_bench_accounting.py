@@ -119,3 +119,14 @@ def test_report_takes_the_roofline_on_the_dominant_tc_kernel():
             assert r["peak"] == round(bench.tensor_peak()[0], 1)
         assert "tensor_frac" in out["kernels"]["tc_gemm_fwd"] and "frac" in out["kernels"]["tc_rows"]
         assert out["gpu_launches"] == 3 * 2 + 16 * 2 - 2 * 2
+        # the step against the bound of the algorithm it runs: FP64 per-row work and D, digit products, bytes
+        st = r["step"]
+        rows = w.evals / w.M1
+        fp64_ms = 2 * (64 * rows + 4 * w.M1 * w.M2 * w.nloc) / (bench.peak_tflops("f64") * 1e12) * 1e3
+        tensor_ms = 45 * 2 * 2 * 24 * w.M1 * len(runs) / (bench.tensor_peak()[0] * 1e12) * 1e3
+        nbytes = 8 * (2 * 5 * rows + 3 * 4 * w.M1 * w.nloc + w.M1 * w.M2 * w.nloc + 5 * w.nloc * w.nnei)
+        hbm_ms = nbytes / (bench.hbm_peak()[0] * 1e9) * 1e3
+        assert abs(st["fp64_ms"] - fp64_ms) < 1e-4 and abs(st["tensor_ms"] - tensor_ms) < 1e-4
+        assert abs(st["hbm_ms"] - hbm_ms) < 1e-4
+        assert st["t_roof_ms"] == max(st["fp64_ms"], st["tensor_ms"], st["hbm_ms"])
+        assert abs(st["frac"] - st["t_roof_ms"] / 1.0) < 1e-4

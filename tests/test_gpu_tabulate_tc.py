@@ -22,16 +22,23 @@ def _gpu():
     need_gpu()
 
 
-def _tc(w, model=None, x=None, nvalid="w", atype="w", work=None, out=None, grad_out=None):
+def _tc(w, model=None, x=None, nvalid="w", atype="w", work=None, out=None, grad_out=None, reuse=False, plan=None):
+    """Forward then backward on the tensor-core path; reuse: the backward takes the forward's interval runs
+    from the shared work buffer (the benchmark's configuration); plan: a TcPlan, else the table is planned
+    per call."""
     dpc = lib()
     model = model or product_model(w, F64)
     x = x or to_dev(w, F64)
     nv = x["nvalid"] if isinstance(nvalid, str) else nvalid
     at = x["atype"] if isinstance(atype, str) else atype
-    T = dpc.dp_tabulate_fusion_fwd_tc_f64(model.table, model.info, x["s"], x["Rt"], nv, at, w.sel, out=out,
-                                          work=work)
-    ds, dRt = dpc.dp_tabulate_fusion_grad_tc_f64(model.table, model.info, x["s"], x["Rt"], nv, at, w.sel, x["dT"],
-                                                 out=grad_out, work=work)
+    tab = plan if plan is not None else model.table
+    if reuse and work is None:
+        need = dpc.dp_tabulate_tc_work_bytes(model.info, w.nloc, w.nnei, w.ntypes, w.M1)
+        work = torch.empty((need,), dtype=torch.uint8, device="cuda")
+    T = dpc.dp_tabulate_fusion_fwd_tc_f64(tab, model.info, x["s"], x["Rt"], nv, at, w.sel, out=out, work=work)
+    ds, dRt = dpc.dp_tabulate_fusion_grad_tc_f64(tab, model.info, x["s"], x["Rt"], nv, at, w.sel, x["dT"],
+                                                 out=grad_out, work=work,
+                                                 flags=dpc.DP_TC_REUSE_RUNS if reuse else 0)
     torch.cuda.synchronize()
     return dict(T=T.cpu().numpy(), ds=ds.cpu().numpy(), dRt=dRt.cpu().numpy())
 
@@ -57,12 +64,17 @@ CHUNK = 4104  # atoms per chunk of the tensor-core calls (their work buffer hold
 
 @pytest.mark.parametrize("name,kw,nsample", CASES, ids=[f"{c[0]}-{c[1]}" for c in CASES])
 def test_tc_against_oracle_and_fp64_path(name, kw, nsample):
-    """T, ds and dR~ against the oracle (sampled atoms at the largest sizes) and against the FP64-pipe
-    moment kernels on every atom."""
+    """T, ds and dR~ in the benchmark's configuration (a plan made once, the backward reusing the forward's
+    interval runs) against the oracle (sampled atoms at the largest sizes) and against the FP64-pipe moment
+    kernels on every atom; bit-identical to a backward that finds the runs itself."""
     w = workload(name, **kw)
     model = product_model(w, F64)
     x = to_dev(w, F64)
-    got = _tc(w, model, x)
+    plan = lib().dp_tabulate_tc_plan_f64(model.table, model.info, w.nnei)
+    got = _tc(w, model, x, reuse=True, plan=plan)
+    fresh = _tc(w, model, x)  # the backward finding the runs itself, the table planned per call
+    for k in got:
+        assert np.array_equal(got[k], fresh[k]), k
     atoms = None
     if nsample:
         atoms = np.sort(np.random.default_rng(5).choice(w.nloc, nsample, replace=False))
@@ -101,6 +113,28 @@ def test_tc_channel_counts_clamped_and_nan(M1, widths):
         assert rel(g, r) <= TOL[F64], (k, rel(g, r))
 
 
+def test_tc_rows_at_nodes_and_range_boundaries():
+    """s on every node of the grid, one ulp and 1e-9 either side of it, and on the three range boundaries
+    (lower, the fine/coarse junction upper, upper_ext) and just either side of them, in random order: the
+    per-row kernels take the interval from an f32 view of s, which may pick either interval at a node, and
+    the f64 search near the range boundaries; T, ds and dR~ match the oracle, with the backward reusing the
+    forward's runs."""
+    w = W.tiny(seed=61, nloc=24, nreal=30, sel=32, widths=(1, 8, 16, 32), M2=4)
+    info = oracle.default().table_info(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    nodes = [info.lower + l * info.stride0 for l in range(info.n0)]
+    nodes += [info.upper + k * info.stride1 for k in range(info.n1 + 1)]
+    vals = []
+    for x in nodes + [info.lower, info.upper, info.upper_ext]:
+        vals += [x, np.nextafter(x, -np.inf), np.nextafter(x, np.inf), x - 1e-9, x + 1e-9]
+    rng = np.random.default_rng(3)
+    s = w.s.copy()
+    nv = w.nvalid.sum(axis=1)
+    for i in range(w.nloc):
+        s[i, :nv[i]] = rng.choice(np.array(vals), nv[i])
+    w2 = W.Workload(**{**w.__dict__, "s": s})
+    assert_parity(_tc(w2, atype=None, reuse=True), run_oracle(w2, F64), F64, keys=("T", "ds", "dRt"))
+
+
 def test_tc_unsorted_rows_many_types_unsorted_centres():
     """ntypes = 8, centre types in random order (several GEMMs share tiles), rows of each segment in
     random order (an interval's rows in several runs add into one slot), some segments empty."""
@@ -127,7 +161,9 @@ def test_tc_unsorted_rows_many_types_unsorted_centres():
                    nvalid=nvalid, atype=rng.integers(0, nt, nloc).astype(np.int32),
                    params=W.net_params(78, [1, 4, 8, 16], nt * nt), dT=base.dT, s_min=float(s[s > 0].min()),
                    s_max=float(s.max()))
-    assert_parity(_tc(w), run_oracle(w, F64), F64, keys=("T", "ds", "dRt"))
+    ref = run_oracle(w, F64)
+    assert_parity(_tc(w), ref, F64, keys=("T", "ds", "dRt"))
+    assert_parity(_tc(w, reuse=True), ref, F64, keys=("T", "ds", "dRt"))
 
 
 def test_tc_empty_counts_and_overwrite():
@@ -155,11 +191,15 @@ def test_tc_empty_counts_and_overwrite():
 
 def test_tc_chunks_of_atoms():
     """More atoms than one chunk (4,104), with a ragged last chunk, against the FP64-pipe path, and the
-    oracle on atoms at the chunk edges."""
+    oracle on atoms at the chunk edges; the backward reusing the forward's runs of every chunk gives the
+    same bits as one that finds them itself."""
     w = workload("water", nmol=1500)  # 4,500 atoms
     model = product_model(w, F64)
     x = to_dev(w, F64)
-    got = _tc(w, model, x)
+    got = _tc(w, model, x, reuse=True)
+    fresh = _tc(w, model, x)
+    for k in got:
+        assert np.array_equal(got[k], fresh[k]), k
     pipe = _pipe(w, model, x)
     for k in ("T", "ds", "dRt"):
         assert rel(got[k], pipe[k]) <= CLOSE, k
@@ -169,7 +209,8 @@ def test_tc_chunks_of_atoms():
 
 def test_tc_work_buffer_rules_and_reuse():
     """The size query (one size for both directions), a short or misaligned buffer refused on the host,
-    and repeated calls on one dirty buffer giving bit-identical results."""
+    a plan made for another geometry refused, and repeated calls on one dirty buffer giving bit-identical
+    results, with and without the backward reusing the forward's runs."""
     dpc = lib()
     w = workload("water", nmol=256)
     model = product_model(w, F64)
@@ -178,10 +219,15 @@ def test_tc_work_buffer_rules_and_reuse():
     assert need > 0 and need % 256 == 0
     work = torch.empty((need + 256,), dtype=torch.uint8, device="cuda")
     a = _tc(w, model, x, work=work[:need])
-    work.fill_(0xff)
-    b = _tc(w, model, x, work=work[:need])
-    for k in a:
-        assert np.array_equal(a[k], b[k]), k
+    for reuse in (False, True):
+        work.fill_(0xff)
+        b = _tc(w, model, x, work=work[:need], reuse=reuse)
+        for k in a:
+            assert np.array_equal(a[k], b[k]), (k, reuse)
+    other = dpc.dp_tabulate_tc_plan_f64(model.table, model.info, w.nnei + 1)
+    with pytest.raises(dpc.DPError):
+        dpc.dp_tabulate_fusion_fwd_tc_f64(other, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel,
+                                          work=work[:need])
     args = (model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
     with pytest.raises(ValueError):
         dpc.dp_tabulate_fusion_fwd_tc_f64(*args, work=work[:need - 1])
@@ -189,12 +235,13 @@ def test_tc_work_buffer_rules_and_reuse():
         dpc.dp_tabulate_fusion_fwd_tc_f64(*args, work=work[16:need + 16])
     with pytest.raises(ValueError):
         dpc.dp_tabulate_tc_work_bytes(model.info, w.nloc, 0, w.ntypes, w.M1)
+    assert dpc.dp_tc_wait_timeouts() == 0  # no bounded wait of the GEMM kernels gave up
 
 
 def test_tc_water_large_chunk_edges():
     """The default f64 path at its largest size: 1,048,576 atoms in 256 chunks, in the benchmark's launch
-    configuration.  The oracle on 256 atoms gathered on the device: the first and last atom of 24
-    chunks spread over the run (edges from the 1st chunk to the 256th, byte offsets into R~ and dR~ past
+    configuration (one plan, one work buffer, the backward reusing the forward's interval runs).  The
+    oracle on 256 atoms gathered on the device: the first and last atom of 24 chunks spread over the run (edges from the 1st chunk to the 256th, byte offsets into R~ and dR~ past
     2^32) and random atoms; the FP64-pipe moment path on every atom, compared on the device; and
     the identity <dR~, R~> = <dT, T> over every atom, which holds at any size."""
     dpc = lib()
@@ -204,8 +251,12 @@ def test_tc_water_large_chunk_edges():
     model = product_model(w, F64)
     x = to_dev(w, F64)
     args = (model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
-    T = dpc.dp_tabulate_fusion_fwd_tc_f64(*args)
-    ds, dRt = dpc.dp_tabulate_fusion_grad_tc_f64(*args, x["dT"])
+    plan = dpc.dp_tabulate_tc_plan_f64(model.table, model.info, w.nnei)
+    pargs = (plan,) + args[1:]
+    work = torch.empty((dpc.dp_tabulate_tc_work_bytes(model.info, w.nloc, w.nnei, w.ntypes, w.M1),),
+                       dtype=torch.uint8, device="cuda")
+    T = dpc.dp_tabulate_fusion_fwd_tc_f64(*pargs, work=work)
+    ds, dRt = dpc.dp_tabulate_fusion_grad_tc_f64(*pargs, x["dT"], work=work, flags=dpc.DP_TC_REUSE_RUNS)
     torch.cuda.synchronize()
     edges = []
     for c in np.unique(np.r_[1, 2, 3, np.linspace(4, nchunks - 1, 21).astype(int)]):
@@ -226,5 +277,6 @@ def test_tc_water_large_chunk_edges():
     for k, a, b in (("ds", ds, dsp), ("dRt", dRt, dRtp)):
         d = float((a - b).abs().max() / b.abs().max())
         assert d <= CLOSE, (k, d)
-    del T, ds, dRt, dsp, dRtp, x, model
+    assert dpc.dp_tc_wait_timeouts() == 0
+    del T, ds, dRt, dsp, dRtp, x, model, work, plan
     torch.cuda.empty_cache()
