@@ -159,8 +159,8 @@ TC_CHUNK_ATOMS = 4104  # atoms per chunk of the tc calls
 
 def tc_profile_events(w) -> int:
     """Events one step of the tc calls records (an upper bound): a start per call, then per chunk forward
-    runs, split, and per centre type GEMM and epilogue; backward runs (unless the forward's are reused),
-    dT split, per type GEMM, rows."""
+    runs, split, slice lists, and per centre type GEMM and epilogue; backward runs (unless the forward's
+    are reused), dT split, per type GEMM, rows."""
     chunks = -(-w.nloc // TC_CHUNK_ATOMS)
     return min(4096, 4 + chunks * (2 + 2 * w.ntypes + 3 + w.ntypes) + 8)
 

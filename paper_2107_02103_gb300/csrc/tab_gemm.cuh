@@ -1,0 +1,336 @@
+// Persistent exact-f64 GEMM for the tensor-core tabulation (tabulate_tc.cu): the per-interval
+// contraction of every 12-atom tile, forward (T = W C' over the used K slices) and backward
+// (dW = dT C'^T over the used 128-row output tiles), on the digit-split operands of tc_gemm.cuh.
+//
+// One CTA per SM walks its units -- (atom tile, 128-row tile of A, share of K) forward, (atom tile,
+// 128-row output tile) backward, from a list of the units with work -- round-robin over the grid.  The TMEM accumulators (nine
+// diagonals x 48 columns), the mbarriers and the stage ring are set up once per CTA, and the roles
+// run ahead of each other: warp 0 moves each slice's A and B blocks into a ring of four stages (bulk
+// copies counted on the stage's "full" barrier), lane 0 of warp 1 issues the slice's 13 MMAs and
+// frees the stage ("empty") when they complete, and eight epilogue warps (two per TMEM lane quadrant,
+// 24 columns each) read the unit's accumulators once its last MMA has completed ("acc_full"),
+// recombine each output's diagonals exactly as an integer and round it once to f64 (or, for a tile with
+// several shares, store four floats), write the outputs, then release the accumulators ("tmem_free")
+// for the next unit's MMAs.  The copies of the next unit overlap the epilogue of this one.
+// Every wait is bounded; a wait that gives up stops the CTA's copies and MMAs, its remaining
+// outputs are NaN and one timeout is counted (dp_tc_wait_timeouts).
+#pragma once
+
+#include "tc_gemm.cuh"
+
+namespace dpc {
+namespace {
+namespace tg {
+using namespace tc;
+
+constexpr int kEpiWarps = 8;                   // two per TMEM lane quadrant
+constexpr int kThreadsP = 32 * (2 + kEpiWarps);  // producer warp, MMA warp, epilogue warps
+constexpr int kEpiCols = kTN / 2;              // columns per epilogue warp
+constexpr int kMaxUnitSlices = kMaxShareSlices;
+
+struct Params {
+  bool fwd;
+  // A: blocks [Mp / 128][ka] of kS x kPlaneA bytes; E: [Mp] row exponents
+  const unsigned char *aplanes;
+  const int *Eexp;
+  int ka;   // K slices per row of blocks (forward: every K slice of the table; backward: M1 / 16)
+  int nmt;  // 128-row tiles of A
+  // B: blocks [ntiles][ka] of kS x kPlaneB bytes; F: [Np] column exponents
+  const unsigned char *bplanes;
+  const int *Fexp;
+  int64_t ntiles, Np, Mp;
+  // forward: the tile's used slices, in order ([ntiles][ka] and [ntiles]), in shares of 28
+  const short *slist;
+  const int *scount;
+  int zmax;
+  float4 *part;  // [zmax][Mp][Np]: results of tiles with several shares (four floats, see diag_combine)
+  double *tout;  // T, written by tiles with one share: [(atom0 + a) 4 + k][ldt]
+  int ldt;
+  // backward: output tile (tile, mt) wanted when one of K slices 8 mt .. 8 mt + 7 is flagged
+  const unsigned char *sflags;  // [ntiles][nsf]
+  int nsf;
+  double *scat;  // [natoms][cap][24]: the wanted outputs, per run slot, finished to f64
+  const short *keys;
+  const int *nslots;
+  int cap, nkeys, kq;
+  // both
+  const int32_t *atype;
+  int64_t natoms, atom0;
+  int alpha, ntypes;
+  const int *units;   // the launch's units, packed (unit_code), in any order
+  const int *nunits;  // their count (device)
+};
+
+// A unit packed into an int: tile (< 2^16), 128-row tile of A (< 2^8), share (< 2^8).
+__host__ __device__ constexpr int unit_code(int tile, int mt, int z) { return tile | (mt << 16) | (z << 24); }
+
+struct Unit {
+  int64_t tile;
+  int mt, z, nsl;  // nsl = 0: nothing to do
+};
+
+// Unit i of the launch's list (every role walks the same list).
+__device__ __forceinline__ Unit unit_of(const Params &P, int i) {
+  const int c = P.units[i];
+  Unit U;
+  U.tile = c & 0xffff;
+  U.mt = (c >> 16) & 0xff;
+  U.z = (c >> 24) & 0xff;
+  U.nsl = P.fwd ? min(P.scount[U.tile] - U.z * kMaxUnitSlices, kMaxUnitSlices) : P.ka;
+  return U;
+}
+
+// A wait on an mbarrier phase, bounded in time (2 s on the global timer), that also gives up once another
+// role has.  The waiting thread is suspended between polls (try_wait's time hint), so that a waiting
+// thread takes no issue slots or shared-memory bandwidth from the copies and the MMAs.
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+__device__ __forceinline__ bool wait_or_abort(uint32_t bar, uint32_t parity, volatile int *abortf) {
+  const uint64_t t0 = global_ns();
+  for (;;) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(done)
+        : "r"(bar), "r"(parity), "r"(20000u)
+        : "memory");
+    if (done) return true;
+    if (*abortf) return false;
+    if (global_ns() - t0 > 2000000000ull) {
+      *abortf = 1;
+      return false;
+    }
+  }
+}
+
+constexpr size_t kBarOff = (size_t)kStages * kStageBytes;  // full[4], empty[4], acc_full, tmem_free
+constexpr size_t kMiscOff = kBarOff + (2 * kStages + 2) * 8;  // tmem address, abort flag
+constexpr size_t kListOff = kMiscOff + 16;                     // producer's slice list
+constexpr size_t kStabOff = kListOff + kMaxUnitSlices * 4;     // epilogue: slot table, slot counts, flags
+constexpr size_t kSmemP = kStabOff + (kScatKeys * kScatAtoms + 2 * kScatAtoms + 4 + kTN) * 4;
+static_assert(kSmemP <= 227 * 1024, "shared memory per block");
+
+__global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
+  extern __shared__ __align__(1024) unsigned char smem[];
+  uint64_t *full = reinterpret_cast<uint64_t *>(smem + kBarOff);
+  uint64_t *empty = full + kStages;
+  uint64_t *acc_full = empty + kStages;
+  uint64_t *tmem_free = acc_full + 1;
+  uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(smem + kMiscOff);
+  volatile int *abortf = reinterpret_cast<volatile int *>(smem + kMiscOff + 4);
+  int *plist = reinterpret_cast<int *>(smem + kListOff);
+  int *stab = reinterpret_cast<int *>(smem + kStabOff);  // (key of the tile, atom) -> slot
+  int *nsa = stab + kScatKeys * kScatAtoms;                // per atom: slot count (backward) or wanted (forward)
+  int *uflag = nsa + 2 * kScatAtoms;  // [0]: the unit writes T directly; [1]: its accumulators are ready
+  int *fexp_s = uflag + 4;             // the unit's 48 column exponents
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nunits = *P.nunits;
+
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(full + s)));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(empty + s)));
+    }
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(acc_full)));
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(tmem_free)), "r"(kEpiWarps));
+    asm volatile("fence.mbarrier_init.release.cluster;");
+    *abortf = 0;
+  }
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_holder)),
+                 "r"(kTmemCols));
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+  }
+  asm volatile("tcgen05.fence::before_thread_sync;");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;");
+  const uint32_t tmem = *tmem_holder;
+  const uint32_t sbase = smem_u32(smem);
+
+  if (warp == 0) {
+    // ---- producer: each slice's A and B blocks into the next stage of the ring
+    int g = 0;  // slices loaded so far by this CTA
+    for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+      if (__shfl_sync(0xffffffffu, (int)*abortf, 0)) break;  // uniform over the warp
+      const Unit U = unit_of(P, u);
+      if (P.fwd && lane < U.nsl) plist[lane] = P.slist[(size_t)U.tile * P.ka + U.z * kMaxUnitSlices + lane];
+      __syncwarp();
+      if (lane == 0) {
+        for (int j = 0; j < U.nsl; ++j, ++g) {
+          const int sl = P.fwd ? plist[j] : j;
+          const int st = g % kStages;
+          if (g >= kStages && !wait_or_abort(smem_u32(empty + st), (uint32_t)((g / kStages - 1) & 1), abortf)) break;
+          const unsigned char *asrc = P.aplanes + ((size_t)U.mt * P.ka + sl) * (kS * kPlaneA);
+          const unsigned char *bsrc = P.bplanes + ((size_t)U.tile * P.ka + sl) * (kS * kPlaneB);
+          const uint32_t bar = smem_u32(full + st), dst = sbase + st * kStageBytes;
+          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"((uint32_t)kStageBytes)
+                       : "memory");
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+              "l"(asrc), "r"((uint32_t)(kS * kPlaneA)), "r"(bar)
+              : "memory");
+          asm volatile(
+              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                  dst + kS * kPlaneA),
+              "l"(bsrc), "r"((uint32_t)(kS * kPlaneB)), "r"(bar)
+              : "memory");
+        }
+      }
+      g = __shfl_sync(0xffffffffu, g, 0);
+      __syncwarp();  // the list is reused by the next unit
+    }
+  } else if (warp == 1) {
+    // ---- MMA issuer: per slice the 45 digit products as 13 MMAs (see gemm_kernel), per unit a commit
+    // on acc_full once they have all completed
+    if (lane == 0) {
+      int g = 0, li = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x) {
+        const Unit U = unit_of(P, u);
+        if (li > 0 && !(ok = wait_or_abort(smem_u32(tmem_free), (uint32_t)((li - 1) & 1), abortf))) break;
+        asm volatile("tcgen05.fence::after_thread_sync;");
+        for (int j = 0; j < U.nsl; ++j, ++g) {
+          const int st = g % kStages;
+          if (!(ok = wait_or_abort(smem_u32(full + st), (uint32_t)((g / kStages) & 1), abortf))) break;
+          asm volatile("tcgen05.fence::after_thread_sync;");
+          const uint64_t a0 = smem_desc(sbase + st * kStageBytes), b0 = smem_desc(sbase + st * kStageBytes + kS * kPlaneA);
+#pragma unroll
+          for (int s = 0; s < kS; ++s) {
+            const uint64_t ad = a0 + (uint64_t)((s * kPlaneA) >> 4);
+#pragma unroll
+            for (int t0 = 0; t0 < kS - s; t0 += kMaxPlanesPerMma) {
+              const int np = min(kMaxPlanesPerMma, kS - s - t0);
+              const uint64_t bd = b0 + (uint64_t)((t0 * kPlaneB) >> 4);
+              const uint32_t idesc = kIdescNoN | ((uint32_t)((np * kTN) >> 3) << 17);
+              const uint32_t acc = (j > 0 || s > 0) ? 1u : 0u;  // a unit's first digit product writes every diagonal
+              asm volatile(
+                  "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+                  " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem + (uint32_t)((s + t0) * kTN)),
+                  "l"(ad), "l"(bd), "r"(idesc), "r"(acc));
+            }
+          }
+          asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+              smem_u32(empty + st)));
+        }
+        // completes when every MMA issued so far has (also after a wait that gave up)
+        asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            smem_u32(acc_full)));
+        ++li;
+      }
+    }
+    __syncwarp();
+  } else {
+    // ---- epilogue: warps 2 .. 9, TMEM lane quadrant warp % 4, columns 24 ((warp - 2) / 4) .. + 23
+    const int et = tid - 64;
+    const int q = warp & 3, c_lo = ((warp - 2) / 4) * kEpiCols;
+    const int rl = 32 * q + lane;
+    const uint32_t trow = tmem + ((uint32_t)(32 * q) << 16);
+    int li = 0;
+    for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+      const Unit U = unit_of(P, u);
+      const int64_t m0 = (int64_t)U.mt * kTM;
+      const int n0 = (int)(U.tile * kTN);
+      asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps));  // the previous unit's tables are free
+      if (et < kTN) fexp_s[et] = P.Fexp[n0 + et];
+      if (P.fwd) {
+        if (et < kScatAtoms) {
+          const int64_t a = (int64_t)(n0 / 4) + et;
+          nsa[et] = a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha);
+        }
+        if (et == 0) uflag[0] = P.tout && P.scount[U.tile] <= kMaxUnitSlices;
+      } else {
+        for (int x = et; x < kScatKeys * kScatAtoms; x += 32 * kEpiWarps) stab[x] = -1;
+        if (et < kScatAtoms) {
+          const int64_t a = (int64_t)(n0 / 4) + et, i = P.atom0 + a;
+          nsa[et] = a < P.natoms && (!P.atype || clampi(P.atype[i], 0, P.ntypes - 1) == P.alpha) ? P.nslots[i] : 0;
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps));
+        const int key0 = (int)(m0 / P.kq);
+        for (int al = et >> 5; al < kScatAtoms; al += kEpiWarps) {  // a warp per atom, its lanes over the slots
+          const short *keys = P.keys + (P.atom0 + n0 / 4 + al) * P.cap;
+          for (int slot = lane; slot < nsa[al]; slot += 32) {
+            const int key = keys[slot];
+            if (key >= key0 && key < key0 + kScatKeys) stab[(key - key0) * kScatAtoms + al] = slot;
+          }
+        }
+      }
+      if (et == 0) uflag[1] = !*abortf && wait_or_abort(smem_u32(acc_full), (uint32_t)(li & 1), abortf);
+      asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps));  // the tables are built and the MMAs done
+      const bool ok = uflag[1] != 0;
+      asm volatile("tcgen05.fence::after_thread_sync;");
+      const bool direct = P.fwd && uflag[0];
+      const int Erow = (direct && m0 + rl < P.ldt) || (!P.fwd && m0 + rl < P.Mp) ? P.Eexp[m0 + rl] : 0;
+      const int key = P.fwd ? 0 : (int)((m0 + rl) / P.kq), qq = P.fwd ? 0 : (int)(m0 + rl - (int64_t)key * P.kq);
+      const int key_l = P.fwd ? 0 : key - (int)(m0 / P.kq);
+      const bool row_wanted = !P.fwd && qq < 6 && key < P.nkeys;
+      float4 *outp = P.fwd && !direct ? P.part + ((size_t)U.z * P.Mp + m0 + rl) * P.Np + n0 : nullptr;
+      // the warp's 24 columns of accumulators, four at a time: each output's nine diagonals recombined
+      // exactly as an integer (diag_int, no FP64 instruction: measured the cheapest here) and rounded
+      // once to f64, or kept as four floats for a tile with several shares
+#pragma unroll 1
+      for (int c0 = 0; c0 < kEpiCols; c0 += 4) {
+        float v[kS][4];
+        if (ok) {  // uniform over the CTA
+#pragma unroll
+          for (int d = 0; d < kS; ++d)
+            asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0,%1,%2,%3}, [%4];"
+                         : "=f"(v[d][0]), "=f"(v[d][1]), "=f"(v[d][2]), "=f"(v[d][3])
+                         : "r"(trow + (uint32_t)(d * kTN + c_lo + c0)));
+          asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int col = c_lo + c0 + c;
+          const int al = col >> 2, k = col & 3;
+          if (outp) {
+            outp[col] = ok ? diag_combine4(v, c) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
+            continue;
+          }
+          const double val = ok ? output_value(diag_int(v, c), Erow, fexp_s[col]) : __longlong_as_double(0x7ff8000000000000ll);
+          if (direct) {
+            if (m0 + rl < P.ldt && nsa[al])
+              P.tout[((P.atom0 + (int64_t)(n0 >> 2) + al) * 4 + k) * P.ldt + m0 + rl] = val;
+          } else if (row_wanted) {
+            const int slot = stab[key_l * kScatAtoms + al];
+            if (slot >= 0) P.scat[((size_t)((n0 >> 2) + al) * P.cap + slot) * 24 + 6 * k + qq] = val;
+          }
+        }
+      }
+      asm volatile("tcgen05.fence::before_thread_sync;");
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(tmem_free)) : "memory");
+      ++li;
+    }
+  }
+
+  asm volatile("tcgen05.fence::before_thread_sync;");
+  __syncthreads();
+  asm volatile("tcgen05.fence::after_thread_sync;");
+  if (tid == 0 && *abortf) atomicAdd(&g_wait_timeouts, 1u);
+  if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
+}
+
+int set_smem(const char *who) {
+  static std::atomic<bool> done{false};
+  if (done.load(std::memory_order_acquire)) return DP_OK;
+  const cudaError_t e = cudaFuncSetAttribute(tgemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemP);
+  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+  done.store(true, std::memory_order_release);
+  return DP_OK;
+}
+
+// One launch over the units of P's list: one CTA per SM.
+int launch(const Params &P, cudaStream_t st, const char *who) {
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(cudaGetLastError()));
+  tgemm_kernel<<<(unsigned)std::max(nsm, 1), kThreadsP, kSmemP, st>>>(P);
+  return launch_status(who);
+}
+
+}  // namespace tg
+}  // namespace
+}  // namespace dpc

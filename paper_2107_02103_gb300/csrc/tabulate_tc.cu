@@ -29,12 +29,12 @@
 // C'_alpha and its digit planes are made once per table by dp_tabulate_tc_plan_f64 (the plan).
 // Per chunk of at most kChunkAtoms atoms and per centre type alpha:
 //   forward:  runs_kernel<true> (slot keys, W, column exponents, slice flags),
-//             split_mom_kernel (W -> B digit planes, used slices only),
-//             gemm_kernel (A = C'_alpha^T: channels x K, B = W^T: K x (atom, k); a tile whose
-//             used slices fit one share writes its atoms' T directly),
+//             split_mom_kernel (W -> B digit planes, used slices only), slice_list_kernel,
+//             tgemm_kernel (tab_gemm.cuh; A = C'_alpha^T: channels x K, B = W^T: K x (atom, k); a
+//             tile whose used slices fit one share writes its atoms' T directly),
 //             fwd_epilogue_kernel (T of the tiles with several shares, or none);
 //   backward: runs_kernel<false> (slot keys, slice flags; skipped when the forward's are reused),
-//             split of dT (B), gemm_kernel (A = C'_alpha: K x channels, B = dT^T) scattering
+//             split of dT (B), tgemm_kernel (A = C'_alpha: K x channels, B = dT^T) scattering
 //             each used (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
 // The slot keys, their counts and the slice flags of every atom stay in the work buffer after
 // the forward, so that a backward on the same inputs can skip its own key pass.
@@ -44,6 +44,7 @@
 #include <cstdint>
 
 #include "dp_common.cuh"
+#include "tab_gemm.cuh"
 #include "tc_gemm.cuh"
 
 namespace dpc {
@@ -71,6 +72,7 @@ struct Shape {
   int64_t nloc, tiles_all;    // atoms of the call and their 12-atom tiles
   int64_t chunk, Np, ntiles;  // atoms per chunk, its columns round_up(4 chunk, 48), Np / 48
   int zmax;                   // forward shares per tile at most
+  int64_t maxunits;           // GEMM units per chunk and centre type at most
 };
 
 // The plan: C' of every centre type and the digit planes of both GEMMs' A operands.
@@ -81,7 +83,7 @@ struct PlanLayout {
 // The work buffer: the slot keys, their counts and the slice flags of every atom of the call
 // (kept from the forward for the backward), then one chunk's scratch.
 struct Layout {
-  size_t keys, nslots, occ, map, fexp, bplanes, w, part, total;
+  size_t keys, nslots, occ, map, slist, scount, units, nunits, fexp, bplanes, w, part, total;
 };
 
 size_t take(size_t &off, size_t bytes) {
@@ -117,6 +119,7 @@ Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1)
   s.chunk = chunk;
   s.Np = round_up(kCols * chunk, kTN);
   s.ntiles = s.Np / kTN;
+  s.maxunits = s.ntiles * std::max<int64_t>((int64_t)(s.Mpf / kTM) * s.zmax, s.Mpb / kTM);
   return s;
 }
 
@@ -141,9 +144,13 @@ Layout make_layout(const Shape &s) {
   L.nslots = take(off, (size_t)std::max<int64_t>(s.nloc, 1) * sizeof(int));
   L.occ = take(off, (size_t)s.ntypes * std::max<int64_t>(s.tiles_all, 1) * s.nsl);
   L.map = take(off, (size_t)s.chunk * s.nkeys * sizeof(int));
+  L.slist = take(off, (size_t)s.ntypes * s.ntiles * s.nsl * sizeof(short));
+  L.scount = take(off, (size_t)s.ntypes * s.ntiles * sizeof(int));
+  L.units = take(off, (size_t)s.ntypes * s.maxunits * sizeof(int));
+  L.nunits = take(off, (size_t)s.ntypes * sizeof(int));
   L.fexp = take(off, (size_t)s.Np * sizeof(int));
   L.bplanes = take(off, (size_t)s.ntiles * std::max(s.nsl, s.Kpm / kTK) * kS * kPlaneB);
-  L.w = take(off, (size_t)s.chunk * s.cap * 24 * sizeof(float4));  // backward float4 slots; forward doubles fit
+  L.w = take(off, (size_t)s.chunk * s.cap * 24 * sizeof(double));  // moments (forward) or their gradients
   L.part = take(off, (size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
   L.total = off;
   return L;
@@ -433,10 +440,62 @@ __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict
   }
 }
 
+// The used K slices of each tile of the chunk, in order, and their count, per centre type (one warp per
+// (type, tile)), and the forward GEMM's units (tile, 128-row tile of A, share of 28 slices) of the tiles
+// with used slices, appended to the type's unit list.
+__global__ void __launch_bounds__(128) slice_list_kernel(const unsigned char *__restrict__ occ, int64_t tiles_all,
+                                                         int64_t tile0, int64_t ntiles, int ntypes, int nsl, int nmt,
+                                                         int64_t maxunits, short *__restrict__ list,
+                                                         int *__restrict__ count, int *__restrict__ units,
+                                                         int *__restrict__ nunits) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (w >= (int64_t)ntypes * ntiles) return;  // warp-uniform
+  const int t = (int)(w / ntiles);
+  const int64_t tile = w - (int64_t)t * ntiles;
+  const unsigned char *f = occ + ((size_t)t * tiles_all + tile0 + tile) * nsl;
+  short *out = list + ((size_t)t * ntiles + tile) * nsl;
+  int rank = 0;
+  for (int b = 0; b < nsl; b += 32) {  // uniform
+    const bool used = b + lane < nsl && f[b + lane] != 0;
+    const unsigned m = __ballot_sync(0xffffffffu, used);
+    if (used) out[rank + __popc(m & ((1u << lane) - 1u))] = (short)(b + lane);
+    rank += __popc(m);
+  }
+  const int nz = (rank + kShareSlices - 1) / kShareSlices;
+  if (lane == 0) {
+    count[(size_t)t * ntiles + tile] = rank;
+    if (nz > 0) {
+      int at = atomicAdd(nunits + t, nz * nmt);
+      for (int z = 0; z < nz; ++z)
+        for (int mt = 0; mt < nmt; ++mt) units[(size_t)t * maxunits + at++] = tg::unit_code((int)tile, mt, z);
+    }
+  }
+}
+
+// The backward GEMM's units: the (tile, 128-row output tile) pairs whose K slices some atom of the tile
+// uses, per centre type (one thread per (type, tile)).
+__global__ void __launch_bounds__(128) bwd_units_kernel(const unsigned char *__restrict__ occ, int64_t tiles_all,
+                                                        int64_t tile0, int64_t ntiles, int ntypes, int nsl, int nmt,
+                                                        int64_t maxunits, int *__restrict__ units,
+                                                        int *__restrict__ nunits) {
+  const int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (x >= (int64_t)ntypes * ntiles) return;
+  const int t = (int)(x / ntiles);
+  const int64_t tile = x - (int64_t)t * ntiles;
+  const unsigned char *f = occ + ((size_t)t * tiles_all + tile0 + tile) * nsl;
+  constexpr int kPer = kTM / kTK;  // K slices per 128-row output tile
+  for (int mt = 0; mt < nmt; ++mt) {
+    bool any = false;
+    for (int q = mt * kPer; q < min(nsl, mt * kPer + kPer); ++q) any |= f[q] != 0;
+    if (any) units[(size_t)t * maxunits + atomicAdd(nunits + t, 1)] = tg::unit_code((int)tile, mt, 0);
+  }
+}
+
 // T for the atoms of type alpha of one 12-atom tile (one block) whose used slices take several shares
-// (one per kShareSlices; a single share's GEMM writes T itself) or none (T = 0): the shares summed and
-// scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at a time: read with the columns fastest
-// (the shares' rows), written with the channels fastest (T's).
+// (one per kShareSlices; a single share's GEMM writes T itself) or none (T = 0): the shares summed in
+// a three-float sum and scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at a time: read with
+// the columns fastest (the shares' rows), written with the channels fastest (T's).
 __global__ void __launch_bounds__(256) fwd_epilogue_kernel(const float4 *__restrict__ part, int Mp, int64_t Np,
                                                            const int *__restrict__ eexp,
                                                            const int *__restrict__ fexp,
@@ -493,11 +552,7 @@ struct RowsParams {
   int sel[DP_MAX_TYPES];
   const short *keys;   // [nloc][cap]: key of each slot
   const int *nslots;   // [nloc]
-  float4 *dW;          // [natoms][cap][24]: the backward GEMM's result per slot (four floats), then in place
-                       // dW as a double in the first half of each entry
-  const int *eexp;     // [ntypes][Mpb]: exponents of the backward A's rows 6 key + q
-  int Mpb;
-  const int *fexp;     // [Np]: exponents of dT's rows 4 a + k
+  const double *dW;    // [natoms][cap][24]: the backward GEMM's result per slot, dW[k][q] at 6 k + q
   double *ds, *dRt;
   int64_t natoms;
 };
@@ -510,9 +565,8 @@ struct alignas(16) RowsStage {
   int nvb[DP_MAX_TYPES];
 };
 
-// One warp per atom: every slot's dW finished from the GEMM's four floats (all lanes, in place),
-// then per 32-row batch the batch's runs copied to shared memory and each valid row's dE/dR~ and
-// dE/ds by Horner's rule in u with its derivative (a lane per row); padded rows get zeros.
+// One warp per atom: per 32-row batch the batch's runs copied to shared memory and each valid row's
+// dE/dR~ and dE/ds by Horner's rule in u with its derivative (a lane per row); padded rows get zeros.
 __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams P) {
   __shared__ RowsStage stw[kRowsWarps];
   extern __shared__ short smapw[];  // [kRowsWarps][nkeys]
@@ -528,16 +582,7 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
   __syncwarp();
   for (int x = lane; x < nslot; x += 32) smap[keys[x]] = (short)x;  // the map of the atom's keys
   const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the map)
-  const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
-  const int *eexp = P.eexp + (size_t)alpha * P.Mpb;
-  float4 *dWa = P.dW + (size_t)a * P.cap * 24;
-  for (int x = lane; x < nslot * 24; x += 32) {  // each lane rewrites only the entry it read
-    const int sl = x / 24, j = x - 24 * sl, k = j / 6, q = j - 6 * k;
-    Sum3 acc;
-    acc.add(dWa[x]);
-    *reinterpret_cast<double *>(dWa + x) = acc.value(eexp[keys[sl] * kQ + q], P.fexp[kCols * a + k]);
-  }
-  __syncwarp();
+  const double *dWa = P.dW + (size_t)a * P.cap * 24;
   const double *srow = P.s + i * P.nnei;
   const double *Rrow = P.Rt + i * P.nnei * 4;
   double *dsrow = P.ds + i * P.nnei;
@@ -574,7 +619,7 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
     __syncwarp();
     for (int x = lane; x < nrun * 24; x += 32) {
       const int r = x / 24, j = x - 24 * r;
-      st.dw[r][j] = *reinterpret_cast<const double *>(dWa + (size_t)st.rslot[r] * 24 + j);
+      st.dw[r][j] = dWa[(size_t)st.rslot[r] * 24 + j];
     }
     __syncwarp();
     if (lane < cnt) {
@@ -724,7 +769,7 @@ int tc_args(const dp_tc_plan *plan, const dp_table_info *info, const double *s, 
   *S = make_shape(*g, nloc, nnei, ntypes, M1);
   *L = make_layout(*S);
   if ((rc = check_work(*L, work, work_bytes, who))) return rc;
-  return set_smem(who);
+  return tg::set_smem(who);
 }
 
 int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
@@ -764,30 +809,44 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
                                                                    wk + L.bplanes);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_split_moments", st);
+    const int64_t nlist = (int64_t)ntypes * ntiles;
+    if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
+      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+    slice_list_kernel<<<(unsigned)((nlist + 3) / 4), 128, 0, st>>>(
+        wk + L.occ, S.tiles_all, tile0, ntiles, ntypes, S.nsl, S.Mpf / kTM, S.maxunits,
+        reinterpret_cast<short *>(wk + L.slist), reinterpret_cast<int *>(wk + L.scount),
+        reinterpret_cast<int *>(wk + L.units), reinterpret_cast<int *>(wk + L.nunits));
+    if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_slice_lists", st);
     for (int t = 0; t < ntypes; ++t) {
-      TcGemm G{};
+      tg::Params G{};
+      G.fwd = true;
       G.aplanes = pk + PL.afwd + (size_t)t * kS * S.Mpf * S.Kp * 2;
       G.Eexp = reinterpret_cast<const int *>(pk + PL.efwd) + (size_t)t * S.Mpf;
-      G.Mp = S.Mpf;
-      G.planes = wk + L.bplanes;
+      G.ka = S.nsl;
+      G.nmt = S.Mpf / kTM;
+      G.bplanes = wk + L.bplanes;
       G.Fexp = R.fexp;
-      G.Np = (int)Np;
-      G.Kp = S.Kp;
+      G.ntiles = ntiles;
+      G.Np = Np;
+      G.Mp = S.Mpf;
+      G.slist = reinterpret_cast<const short *>(wk + L.slist) + (size_t)t * ntiles * S.nsl;
+      G.scount = reinterpret_cast<const int *>(wk + L.scount) + (size_t)t * ntiles;
+      G.zmax = S.zmax;
       G.part = part;
-      G.slices_per_split = kShareSlices;
-      G.kocc = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
       G.tout = T;  // tiles with one share write T themselves
+      G.units = reinterpret_cast<const int *>(wk + L.units) + (size_t)t * S.maxunits;
+      G.nunits = reinterpret_cast<const int *>(wk + L.nunits) + t;
       G.ldt = M1;
+      G.atype = atype;
       G.natoms = n;
       G.atom0 = c0;
-      G.atype = atype;
       G.alpha = t;
       G.ntypes = ntypes;
-      const dim3 grid((unsigned)ntiles, (unsigned)(S.Mpf / kTM), (unsigned)S.zmax);
-      gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
-      if ((rc = launch_status(who))) return rc;
+      if ((rc = tg::launch(G, st, who))) return rc;
       prof_mark("tc_gemm_fwd", st);
-      fwd_epilogue_kernel<<<(unsigned)ntiles, 256, 0, st>>>(part, S.Mpf, Np, G.Eexp, R.fexp, G.kocc, S.nsl, n, c0,
+      const unsigned char *kocc = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
+      fwd_epilogue_kernel<<<(unsigned)ntiles, 256, 0, st>>>(part, S.Mpf, Np, G.Eexp, R.fexp, kocc, S.nsl, n, c0,
                                                             atype, ntypes, t, M1, T);
       if ((rc = launch_status(who))) return rc;
       prof_mark("tc_epilogue_fwd", st);
@@ -820,7 +879,7 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei,
                              reinterpret_cast<const double *>(pk + PL.nodes));
   const int mtiles = S.Mpb / kTM;
-  float4 *dW = reinterpret_cast<float4 *>(wk + L.w);
+  double *dW = reinterpret_cast<double *>(wk + L.w);
   RowsParams Q{};
   Q.s = s;
   Q.Rt = Rt;
@@ -837,9 +896,6 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
   Q.keys = R.keys;
   Q.nslots = R.nslots;
   Q.dW = dW;
-  Q.eexp = reinterpret_cast<const int *>(pk + PL.ebwd);
-  Q.Mpb = S.Mpb;
-  Q.fexp = R.fexp;
   Q.ds = ds;
   Q.dRt = dRt;
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
@@ -858,32 +914,43 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
                          who)))
       return rc;
     prof_mark("tc_split_dT", st);
+    if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
+      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+    const int64_t nlist = (int64_t)ntypes * ntiles;
+    bwd_units_kernel<<<(unsigned)((nlist + 127) / 128), 128, 0, st>>>(wk + L.occ, S.tiles_all, tile0, ntiles, ntypes,
+                                                                      S.nsl, mtiles, S.maxunits,
+                                                                      reinterpret_cast<int *>(wk + L.units),
+                                                                      reinterpret_cast<int *>(wk + L.nunits));
+    if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_units", st);
     for (int t = 0; t < ntypes; ++t) {
-      TcGemm G{};
+      tg::Params G{};
+      G.fwd = false;
       G.aplanes = pk + PL.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
-      G.Eexp = Q.eexp + (size_t)t * S.Mpb;
-      G.Mp = S.Mpb;
-      G.planes = wk + L.bplanes;
+      G.Eexp = reinterpret_cast<const int *>(pk + PL.ebwd) + (size_t)t * S.Mpb;
+      G.ka = S.Kpm / kTK;
+      G.nmt = mtiles;
+      G.bplanes = wk + L.bplanes;
       G.Fexp = R.fexp;
-      G.Np = (int)Np;
-      G.Kp = S.Kpm;
-      G.slices_per_split = S.Kpm / kTK;
+      G.ntiles = ntiles;
+      G.Np = Np;
+      G.Mp = S.Mpb;
       G.sflags = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
       G.nsf = S.nsl;
       G.scat = dW;
       G.keys = R.keys;
       G.nslots = R.nslots;
+      G.cap = S.cap;
+      G.nkeys = S.nkeys;
+      G.kq = kQ;
       G.atype = atype;
       G.natoms = n;
       G.atom0 = c0;
-      G.nkeys = S.nkeys;
-      G.cap = S.cap;
       G.alpha = t;
       G.ntypes = ntypes;
-      G.kq = kQ;
-      const dim3 grid((unsigned)ntiles, (unsigned)mtiles, 1);
-      gemm_kernel<<<grid, kThreads, kSmemTotal, st>>>(G);
-      if ((rc = launch_status(who))) return rc;
+      G.units = reinterpret_cast<const int *>(wk + L.units) + (size_t)t * S.maxunits;
+      G.nunits = reinterpret_cast<const int *>(wk + L.nunits) + t;
+      if ((rc = tg::launch(G, st, who))) return rc;
       prof_mark("tc_gemm_grad", st);
     }
     Q.atom0 = c0;

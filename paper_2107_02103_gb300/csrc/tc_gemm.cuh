@@ -300,6 +300,75 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
   return done != 0;
 }
 
+// sum_d v[d][c] 64^-(d+2) (the diagonal sums of one output, read from TMEM) as four floats on the FP32
+// pipe: diagonals 2 and 3 (d = 0, 1) as an exact two-sum, 4 .. 10 in float-float, smallest first (its
+// rounding lies ~2^-60 below the sum).
+template <int W>
+__device__ __forceinline__ float4 diag_combine_w(const float (&v)[kS][W], int c) {
+  dfl::df64 lo(0.0f);
+#pragma unroll
+  for (int d = kS - 1; d >= 2; --d) {
+    const float x = v[d][c] * __uint_as_float((uint32_t)(127 - kBits * (d + 2)) << 23);  // exact: 64^-(d+2)
+    lo = lo + dfl::df64(x);
+  }
+  const float a = v[0][c] * 0x1p-12f, b = v[1][c] * 0x1p-18f;  // exact
+  const float s = __fadd_rn(a, b), bb = __fsub_rn(s, a);
+  const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  return make_float4(s, e, lo.hi, lo.lo);
+}
+__device__ __forceinline__ float4 diag_combine(const float (&v)[kS][8], int c) { return diag_combine_w<8>(v, c); }
+__device__ __forceinline__ float4 diag_combine4(const float (&v)[kS][4], int c) { return diag_combine_w<4>(v, c); }
+
+// A float that holds an integer below 2^24 in magnitude (a diagonal sum) as an int: exact.
+__device__ __forceinline__ int exact_int(float f) { return __float2int_rz(f); }
+
+// The nine diagonal sums of one output (exact integers below 2^24; diagonal d weighs 64^-(d+2)) as one
+// exact integer in units of 2^-60, S = sum_d v[d][c] 2^(6 (8 - d)), |S| < 2^74: integer adds, no rounding.
+template <int W>
+__device__ __forceinline__ __int128 diag_int(const float (&v)[kS][W], int c) {
+  static_assert(kS == 9 && kBits == 6, "the integer recombination assumes nine 6-bit digits");
+  long long lo = 0;  // diagonals 4 .. 10: below 2^24 2^36 64/63 < 2^61
+#pragma unroll
+  for (int d = 2; d < kS; ++d) lo += (long long)exact_int(v[d][c]) << (kBits * (kS - 1 - d));
+  const long long hi = (long long)exact_int(v[0][c]) * 64 + exact_int(v[1][c]);  // diagonals 2, 3 over 2^42
+  return ((__int128)hi << 42) + lo;
+}
+
+// S 2^e2 rounded once to the nearest f64 (ties to even), from its bits: integer operations only, except
+// where the result falls outside the normal range (never for these sums in practice).
+__device__ __forceinline__ double i128_to_double(__int128 S, int e2) {
+  if (S == 0) return 0.0;
+  const bool neg = S < 0;
+  const unsigned __int128 U = neg ? (unsigned __int128)(-S) : (unsigned __int128)S;
+  const unsigned long long uh = (unsigned long long)(U >> 64), ul = (unsigned long long)U;
+  const int n = uh ? 128 - __clzll((long long)uh) : 64 - __clzll((long long)ul);  // bit length of |S|
+  int ex = n - 1 + e2;  // exponent of the leading bit
+  unsigned long long m;
+  if (n <= 53) {
+    m = ul << (53 - n);
+  } else {
+    const int sh = n - 53;
+    m = (unsigned long long)(U >> sh);
+    const unsigned long long rem = ul & ((1ull << sh) - 1ull), half = 1ull << (sh - 1);
+    if (rem > half || (rem == half && (m & 1ull))) {
+      ++m;
+      if (m == (1ull << 53)) {
+        m >>= 1;
+        ++ex;
+      }
+    }
+  }
+  if (ex < -1022 || ex > 1023) return (neg ? -1.0 : 1.0) * scalbn((double)m, ex - 52);
+  return __longlong_as_double((long long)(((unsigned long long)neg << 63) | ((unsigned long long)(ex + 1023) << 52) |
+                                          (m & ((1ull << 52) - 1ull))));
+}
+
+// An output from its exact integer: NaN for a row or column with an inf or NaN.
+__device__ __forceinline__ double output_value(__int128 S, int E, int F) {
+  if (E >= kNonFinite || F >= kNonFinite) return __longlong_as_double(0x7ff8000000000000ll);
+  return i128_to_double(S, E + F - kFrac - kBits);
+}
+
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);  // stage loaded
@@ -486,20 +555,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
     }
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
-      // sum_d v_d 64^-(d+2) as four floats on the FP32 pipe: diagonals 2 and 3 (d = 0, 1) as an exact
-      // two-sum, 4 .. 10 in float-float, smallest first (its rounding lies ~2^-60 below the sum).
       // The scaling by 2^(E+F), and all f64 arithmetic, is left to the epilogue (or, for a direct
       // output, to the two f64 adds below).
-      dfl::df64 lo(0.0f);
-#pragma unroll
-      for (int d = kS - 1; d >= 2; --d) {
-        const float x = v[d][c] * __uint_as_float((uint32_t)(127 - kBits * (d + 2)) << 23);  // exact: 64^-(d+2)
-        lo = lo + dfl::df64(x);
-      }
-      const float a = v[0][c] * 0x1p-12f, b = v[1][c] * 0x1p-18f;  // exact
-      const float s = __fadd_rn(a, b), bb = __fsub_rn(s, a);
-      const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
-      const float4 val = ok ? make_float4(s, e, lo.hi, lo.lo) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
+      const float4 val = ok ? diag_combine(v, c) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
       if (direct) {
         if (m0 + rl < P.ldt && stab[(c0 + c) >> 2]) {
           Sum3 acc;
