@@ -250,10 +250,10 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  * takes dRt[i][j][k] = sum_q dW[k][(b, l, q)] u_j^q and ds[i][j] =
  * sum_k R~[i][j][k] sum_{q>=1} q dW[k][(b, l, q)] u_j^(q-1) / Delta_l (0
  * where s was clamped).  Both GEMMs run exactly as in dp_fitting_*_tc_f64:
- * nine 6-bit digits per element, scaled by the row's or column's power of
- * two, fp16 MMAs with exact fp32 sums (at most 448 of K per partial sum),
- * one rounding to f64; per output the error is below about
- * K 2^-50 max|row| max|column| (K: the used intervals x 6, or M1).  Only
+ * nine balanced 6-bit digits per element (in [-32, 32]), scaled by the row's
+ * or column's power of two, fp16 MMAs with exact fp32 sums (at most 1792 of
+ * K per partial sum), one rounding to f64; per output the error is below
+ * about K 2^-49 max|row| max|column| (K: the used intervals x 6, or M1).  Only
  * the intervals some atom of a 12-atom tile uses enter its GEMM.  Rows need
  * not be sorted, though sorted rows (one run per interval) do the least
  * FP64 work.  NaN s gives NaN in that atom's T (forward) and in that row's
@@ -560,12 +560,12 @@ int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer
  * The f64 fitting net with its hidden-layer GEMMs on the tensor cores
  * (tcgen05).  Same inputs, outputs and results as dp_fitting_fwd_f64 /
  * dp_fitting_grad_f64 (Sec. II: E_i from D_i, and dE_i/dD_i), to f64
- * accuracy: every GEMM operand element is split exactly into nine 6-bit
- * digits scaled by its row's (A) or column's (B) power of two, the 45 digit
+ * accuracy: every GEMM operand element is split exactly into nine balanced
+ * 6-bit digits scaled by its row's (A) or column's (B) power of two, the 45 digit
  * products that matter run as fp16 MMAs whose fp32 sums are exact integers
- * (at most 448 of K per partial sum), and those sums are recombined exactly
+ * (at most 1792 of K per partial sum), and those sums are recombined exactly
  * before one rounding to f64.  Per output the error is below about
- * K 2^-50 max_k |a_ik| max_k |b_kj| (an f64 dot product: K 2^-53 sum_k
+ * K 2^-49 max_k |a_ik| max_k |b_kj| (an f64 dot product: K 2^-53 sum_k
  * |a_ik b_kj|).  A row or column holding inf or NaN gives NaN outputs.  The
  * paper computes the net in double; this is that computation on hardware
  * whose FP64 rate is ~1000 times below its fp16 tensor rate.

@@ -156,7 +156,8 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
     for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
       if (__shfl_sync(0xffffffffu, (int)*abortf, 0)) break;  // uniform over the warp
       const Unit U = unit_of(P, u);
-      if (P.fwd && lane < U.nsl) plist[lane] = P.slist[(size_t)U.tile * P.ka + U.z * kMaxUnitSlices + lane];
+      if (P.fwd)
+        for (int j = lane; j < U.nsl; j += 32) plist[j] = P.slist[(size_t)U.tile * P.ka + U.z * kMaxUnitSlices + j];
       __syncwarp();
       if (lane == 0) {
         for (int j = 0; j < U.nsl; ++j, ++g) {

@@ -56,7 +56,7 @@ constexpr int kQ = 6;                 // K entries per interval: u^0 .. u^5
 constexpr int kCols = 4;              // GEMM columns per atom: k = 0 .. 3
 constexpr int kTileAtoms = kTN / kCols;  // 12 atoms per 48-column tile
 constexpr int64_t kChunkAtoms = 4104;    // a multiple of 12 (16,416 columns)
-constexpr int kShareSlices = kMaxShareSlices;  // used K slices per forward share (28, the exactness bound)
+constexpr int kShareSlices = kMaxShareSlices;  // used K slices per forward share (112, the exactness bound)
 constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' results per chunk
 constexpr int kMaxKeys = 4096;  // ntypes x nint: each warp's key map (int16) lives in shared memory
 static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
@@ -433,7 +433,7 @@ __global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict
     const double x0 = slot >= 0 ? wp[q0] : 0.0;
     const double x1 = slot >= 0 ? wp[q0 + 1] : 0.0;
     uint32_t h[kS];
-    digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
+    digit_pairs(biased_fixed(x0, E), biased_fixed(x1, E), h);
     unsigned char *dst = rowbase + (size_t)sl * block + ((k0 % kTK) >> 3) * kLBO;
 #pragma unroll
     for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];

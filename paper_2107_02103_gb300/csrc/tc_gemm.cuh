@@ -16,20 +16,23 @@ namespace {
 // GB300 retires FP64 at 2 lanes per clock per SM but fp16 products on its
 // tcgen05 tensor cores at ~1000 times that rate.  An f64 GEMM C = A B is
 // recovered from fp16 products by splitting every operand element into base-64
-// digits (the error-free splitting of Ozaki et al.):
-//   a_ik = 2^E_i sum_{s=1..9} A_s[i][k] 64^-s + r_ik,  A_s integers in [-63, 63],  |r_ik| < 2^(E_i - 54),
-// with max_k |a_ik| < 2^E_i, and likewise b_kj with a column exponent F_j, so that
-//   C_ij = 2^(E_i + F_j) sum_{d=2..10} 64^-d sum_{s+t=d} (A_s B_t)_ij + (terms with s + t > 10 and the r).
-// Every (A_s B_t)_ij is a sum of integer products |A_s B_t| <= 3969; a diagonal
+// digits (the error-free splitting of Ozaki et al., here with balanced digits):
+//   a_ik = 2^(E_i + 1) sum_{s=1..9} A_s[i][k] 64^-s + r_ik,  A_s integers in [-32, 32],  |r_ik| < 2^(E_i - 53),
+// with max_k |a_ik| < 2^E_i: the row's 53-bit fixed point a 2^(53 - E) is truncated toward zero and
+// biased by 32 (64^7 + ... + 1); its eight low 6-bit fields less 32 are digits 2 .. 9, and what lies
+// above them (an arithmetic shift) is digit 1.  Likewise b_kj with a column exponent F_j, so that
+//   C_ij = 2^(E_i + F_j + 2) sum_{d=2..10} 64^-d sum_{s+t=d} (A_s B_t)_ij + (terms with s + t > 10 and the r).
+// Every (A_s B_t)_ij is a sum of integer products |A_s B_t| <= 1024; a diagonal
 // d has at most 9 of them, so its fp32 sum on the tensor cores is exact while
-// a block's share of K is at most kMaxShareK = 448 (9 x 448 x 3969 < 2^24).
+// a block's share of K is at most kMaxShareK = 1792 (9 x 1792 x 1024 < 2^24).
 // The 9 diagonal sums of an output are combined on the FP32 pipe into four
 // floats (the two largest by an exact two-sum, the rest in float-float, whose
 // rounding lies ~2^-60 below the result); the caller's epilogue (Sum3 below)
 // adds the shares' floats into a three-float sum by exact two-sums and
-// converts it to f64 once.
-// What rounds is that conversion, the 54-bit truncation of the operands and
-// the dropped terms: |error| <~ K 2^-50 max_k|a_ik| max_k|b_kj|, against
+// converts it to f64 once -- or recombines the diagonals exactly as one
+// integer and rounds that once (diag_int, i128_to_double).
+// What rounds is that conversion, the 53-bit truncation of the operands and
+// the dropped terms: |error| <~ K 2^-49 max_k|a_ik| max_k|b_kj|, against
 // K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column with an
 // inf or NaN gives NaN outputs.
 //
@@ -60,11 +63,15 @@ namespace {
 namespace tc {
 constexpr int kS = 9;      // digits per operand element
 constexpr int kBits = 6;   // bits per digit
-constexpr int kFrac = kS * kBits;  // 54 fractional bits
+constexpr int kFrac = kS * kBits - 1;  // 53 fractional bits; the ninth digit's spare bit keeps the balanced top digit in range
+constexpr int kPad = kS * kBits - kFrac;  // a digit vector stands for 2^(E + kPad) sum_s d_s 64^-s
+// 32 (64^7 + ... + 1): added to a fixed point f in (-2^53, 2^53), it makes each of the eight low 6-bit
+// fields a digit plus 32 and leaves floor((f + bias) / 64^8) in [-32, 32] as the top digit
+constexpr int64_t kDigitBias = 32ll * ((1ll << 48) - 1ll) / 63ll;
 constexpr int kTM = 128, kTN = 48, kTK = 16;  // CTA tile; K per stage (one MMA)
 constexpr int kStages = 4;
 constexpr int kThreads = 128;  // one warp per TMEM lane quadrant; lane 0 of warps 0 and 1: producer and MMA issuer
-constexpr int kMaxShareK = 448;
+constexpr int kMaxShareK = 1792;
 constexpr int kNonFinite = 1 << 20;  // exponent of a row or column holding inf or NaN
 constexpr uint32_t kLBO = 128, kSBO = 256;  // core matrices: next along K at +128 B, next 8 rows at +256 B
 constexpr int kPlaneA = kTM * kTK * 2, kPlaneB = kTN * kTK * 2;  // bytes of one digit plane in a stage
@@ -74,7 +81,8 @@ constexpr int kMaxShareSlices = kMaxShareK / kTK;
 constexpr size_t kSmemTail = (size_t)kStages * kStageBytes + (2 * kStages + 1) * 8 + 16;  // used-slice list
 constexpr int kScatKeys = kTM / 4 + 1, kScatAtoms = kTN / 4;  // scatter: keys (kq >= 4) and atoms of a tile
 constexpr size_t kSmemTotal = kSmemTail + (kMaxShareSlices + 2) * 4 + kScatKeys * kScatAtoms * 4;
-static_assert((size_t)kS * kMaxShareK * 63 * 63 < (1u << 24), "fp32 diagonal sums must stay exact");
+static_assert((size_t)kS * kMaxShareK * 32 * 32 < (1u << 24), "fp32 diagonal sums must stay exact");
+static_assert(kDigitBias < (1ll << 48) && kFrac == 53 && kS == 9, "top digit floor((f + bias) / 2^48) within [-32, 32]");
 static_assert(kMaxShareK % kTK == 0 && kS * kTN <= (int)kTmemCols, "shares and TMEM");
 static_assert(kSmemTotal <= 227 * 1024, "shared memory per block");
 
@@ -84,34 +92,29 @@ __device__ __forceinline__ int exp_bits(double x) { return (int)(((uint64_t)__do
 // E with max |x| < 2^E from the largest biased exponent (normal x: |x| < 2^(eb - 1022))
 __device__ __forceinline__ int exp_of_max(int ebmax) { return ebmax == 0x7ff ? kNonFinite : max(ebmax, 1) - 1022; }
 
-// |x| 2^-E as an integer with kFrac fractional bits, truncated; below 2^kFrac since |x| < 2^E
-__device__ __forceinline__ uint64_t fixed_point(double x, int E) {
+// x 2^(kFrac - E) truncated toward zero (|x| < 2^E, so |.| < 2^kFrac), plus kDigitBias (see digit_pairs)
+__device__ __forceinline__ int64_t biased_fixed(double x, int E) {
   const uint64_t b = (uint64_t)__double_as_longlong(x);
   const int eb = (int)((b >> 52) & 0x7ff);
   const uint64_t mant = b & 0xfffffffffffffull;
   const uint64_t m = eb ? (mant | (1ull << 52)) : mant;
-  const int sh = (eb ? eb - 1075 : -1074) - E + kFrac;  // |x| 2^(kFrac - E) = m 2^sh, sh <= 1 for finite x
-  if (sh >= 0) return m << min(sh, 10);
-  return sh > -64 ? m >> -sh : 0ull;
+  const int sh = (eb ? eb - 1075 : -1074) - E + kFrac;  // |x| 2^(kFrac - E) = m 2^sh, sh <= 0 for finite x
+  const int64_t mag = (int64_t)(sh >= 0 ? m << min(sh, 10) : (sh > -64 ? m >> -sh : 0ull));
+  return (b >> 63 ? -mag : mag) + kDigitBias;
 }
 
-// The kS digits of two fixed-point values, digit s of both packed as an fp16 pair (element 0 in the
-// low half), each with its element's sign: 0x6400 | d is the fp16 1024 + d, and 1024 comes off exactly.
-__device__ __forceinline__ void digit_pairs(uint64_t f0, uint64_t f1, uint32_t sign2, uint32_t (&h)[kS]) {
+// The kS balanced digits of two elements from their biased fixed points g, digit s of both packed as an
+// fp16 pair (element 0 in the low half): field u in [0, 64] (digit + 32) is encoded as 0x6400 | u, the
+// fp16 1024 + u, and 1056 comes off exactly.  Digits 2 .. 9 are the eight low fields; digit 1 is g >> 48.
+__device__ __forceinline__ void digit_pairs(int64_t g0, int64_t g1, uint32_t (&h)[kS]) {
   constexpr uint32_t kMask = (1u << kBits) - 1;
 #pragma unroll
   for (int s = 1; s <= kS; ++s) {
-    const uint32_t d0 = (uint32_t)(f0 >> (kFrac - kBits * s)) & kMask;
-    const uint32_t d1 = (uint32_t)(f1 >> (kFrac - kBits * s)) & kMask;
-    uint32_t v;
-    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(v) : "r"(0x64006400u | d0 | (d1 << 16)), "r"(0x64006400u));
-    h[s - 1] = v ^ sign2;
+    const int sh = kBits * (kS - s);
+    const uint32_t d0 = s == 1 ? (uint32_t)((g0 >> sh) + 32) : (uint32_t)(g0 >> sh) & kMask;
+    const uint32_t d1 = s == 1 ? (uint32_t)((g1 >> sh) + 32) : (uint32_t)(g1 >> sh) & kMask;
+    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(h[s - 1]) : "r"(0x64006400u | d0 | (d1 << 16)), "r"(0x64206420u));
   }
-}
-
-__device__ __forceinline__ uint32_t sign_pair(double x0, double x1) {
-  return (uint32_t)((uint64_t)__double_as_longlong(x0) >> 63) << 15 | (uint32_t)((uint64_t)__double_as_longlong(x1) >> 63)
-                                                                          << 31;
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -161,7 +164,7 @@ __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restric
     const int k = k0 + 2 * kp;
     const double x0 = x(k), x1 = x(k + 1);
     uint32_t h[kS];
-    digit_pairs(fixed_point(x0, E), fixed_point(x1, E), sign_pair(x0, x1), h);
+    digit_pairs(biased_fixed(x0, E), biased_fixed(x1, E), h);
     unsigned char *dst = rowbase + (size_t)(k0 / kTK) * block + ((k0 % kTK) >> 3) * kLBO;
 #pragma unroll
     for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
@@ -200,9 +203,10 @@ struct Sum3 {
   // the sum times 2^(E + F); NaN for a row or column with an inf or NaN, or a NaN share
   __device__ __forceinline__ double value(int E, int F) const {
     if (E >= kNonFinite || F >= kNonFinite || s0 != s0) return __longlong_as_double(0x7ff8000000000000ll);
-    if (E + F > -900 && E + F < 900)  // the scaling moves exponent fields only (sums stay normal)
-      return __dadd_rn(__dadd_rn(widen_pow2(s0, E + F), widen_pow2(s1, E + F)), widen_pow2(s2, E + F));
-    return scalbn(__dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2)), E + F);
+    const int e = E + F + 2 * kPad;
+    if (e > -900 && e < 900)  // the scaling moves exponent fields only (sums stay normal)
+      return __dadd_rn(__dadd_rn(widen_pow2(s0, e), widen_pow2(s1, e)), widen_pow2(s2, e));
+    return scalbn(__dadd_rn(__dadd_rn(dfl::widen(s0), dfl::widen(s1)), dfl::widen(s2)), e);
   }
 };
 
@@ -366,7 +370,7 @@ __device__ __forceinline__ double i128_to_double(__int128 S, int e2) {
 // An output from its exact integer: NaN for a row or column with an inf or NaN.
 __device__ __forceinline__ double output_value(__int128 S, int E, int F) {
   if (E >= kNonFinite || F >= kNonFinite) return __longlong_as_double(0x7ff8000000000000ll);
-  return i128_to_double(S, E + F - kFrac - kBits);
+  return i128_to_double(S, E + F + 2 * kPad - 2 * kBits - kBits * (kS - 1));
 }
 
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
@@ -555,7 +559,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
     }
 #pragma unroll
     for (int c = 0; c < 8; ++c) {
-      // The scaling by 2^(E+F), and all f64 arithmetic, is left to the epilogue (or, for a direct
+      // The scaling by 2^(E+F+2 kPad), and all f64 arithmetic, is left to the epilogue (or, for a direct
       // output, to the two f64 adds below).
       const float4 val = ok ? diag_combine(v, c) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
       if (direct) {

@@ -1,10 +1,11 @@
 """The arithmetic behind dp_fitting_*_tc_f64 (the f64 fitting-net GEMMs on the tensor cores),
-emulated exactly on the CPU: each operand element is cut into nine 6-bit digits against its row's
-(A) or column's (B) power of two, the 45 digit products with s + t <= 10 are summed per diagonal
-as integers, and the result is rebuilt.  The checks are the ones the kernels rely on: every
-diagonal sum over a share of K <= 448 stays below 2^24 (so fp32 sums of it are exact), digits fit
-fp16 exactly, and the result lies within K 2^-50 max|a_i| max|b_j| of the exact dot product (an
-f64 dot product's bound is K 2^-53 sum|a b|).  Plus the host-side work-size query.  CPU only."""
+emulated exactly on the CPU: each operand element is cut into nine balanced 6-bit digits (in
+[-32, 32]) against its row's (A) or column's (B) power of two, the 45 digit products with s + t <= 10
+are summed per diagonal as integers, and the result is rebuilt.  The checks are the ones the kernels
+rely on: the digits rebuild the 53-bit fixed point exactly, every diagonal sum over a share of
+K <= 1792 stays below 2^24 (so fp32 sums of it are exact), digits fit fp16 exactly, and the result
+lies within K 2^-49 max|a_i| max|b_j| of the exact dot product (an f64 dot product's bound is
+K 2^-53 sum|a b|).  Plus the host-side work-size query.  CPU only."""
 import math
 from fractions import Fraction
 
@@ -12,8 +13,10 @@ import numpy as np
 import pytest
 
 S, BITS = 9, 6
-FRAC = S * BITS          # fractional bits kept
-MAX_SHARE_K = 448
+FRAC = S * BITS - 1      # fractional bits kept (53)
+PAD = S * BITS - FRAC    # the digits stand for 2^(E + PAD) sum_s d_s 64^-s
+BIAS = sum(32 * 64 ** k for k in range(S - 1))  # makes the eight low fields digit + 32
+MAX_SHARE_K = 1792
 
 
 def row_exponent(v):
@@ -26,12 +29,16 @@ def row_exponent(v):
 
 
 def digits(x, E):
-    """The S base-2^BITS digits of |x| 2^-E truncated to FRAC bits, each with the sign of x."""
-    f = Fraction(abs(x)) / Fraction(2) ** E
-    assert f < 1
-    fixed = math.floor(f * 2 ** FRAC)
-    sgn = -1 if x < 0 else 1
-    return [sgn * ((fixed >> (FRAC - BITS * s)) & (2 ** BITS - 1)) for s in range(1, S + 1)]
+    """The S balanced base-2^BITS digits of x 2^(FRAC - E) truncated toward zero: the eight low fields of
+    the fixed point plus BIAS, less 32 each, and the top digit floor((fixed + BIAS) / 2^48)."""
+    f = Fraction(x) / Fraction(2) ** E
+    assert abs(f) < 1
+    fixed = math.trunc(f * 2 ** FRAC)
+    g = fixed + BIAS
+    low = [((g >> (BITS * (S - s))) & (2 ** BITS - 1)) - 32 for s in range(2, S + 1)]
+    d = [g >> (BITS * (S - 1))] + low
+    assert sum(dd * 64 ** (S - s) for s, dd in enumerate(d, 1)) == fixed
+    return d
 
 
 def product(A, B):
@@ -55,17 +62,21 @@ def product(A, B):
                             diag[s + t] += Ad[i, k][s] * Bd[k, j][t]
                 peak = max(peak, max(abs(d) for d in diag))
                 total += sum(Fraction(d, 2 ** (BITS * (dd + 2))) for dd, d in enumerate(diag))
-            C[i, j] = float(total * Fraction(2) ** (E[i] + F[j]))
+            C[i, j] = float(total * Fraction(2) ** (E[i] + F[j] + 2 * PAD))
     return C, peak
 
 
 def test_exactness_bounds_of_the_fp32_diagonal_sums():
-    assert S * MAX_SHARE_K * (2 ** BITS - 1) ** 2 < 2 ** 24      # a diagonal's sum over a share
-    assert 2 ** BITS - 1 <= 2 ** 11                              # a digit is an exact fp16 integer
-    assert S * BITS >= 53 + 1                                   # 54 bits: every f64 significand
+    assert S * MAX_SHARE_K * 32 * 32 < 2 ** 24                   # a diagonal's sum over a share
+    assert 1024 + 64 <= 2 ** 11                                  # a digit + 32 + 1024 is an exact fp16 integer
+    assert FRAC >= 53                                            # every f64 significand
+    assert BIAS < 2 ** 48                                        # the top digit stays in [-32, 32]
+    for f in (2 ** FRAC - 1, -(2 ** FRAC - 1)):
+        top = (f + BIAS) >> 48
+        assert -32 <= top <= 32
 
 
-@pytest.mark.parametrize("K,scaled", [(70, False), (500, False), (40, True)])
+@pytest.mark.parametrize("K,scaled", [(70, False), (500, False), (40, True), (1900, False)])
 def test_digit_product_within_its_bound(K, scaled):
     rng = np.random.default_rng(K)
     A = rng.standard_normal((3, K))
@@ -80,7 +91,7 @@ def test_digit_product_within_its_bound(K, scaled):
     for i in range(A.shape[0]):
         for j in range(B.shape[1]):
             exact = sum(Fraction(A[i, k]) * Fraction(B[k, j]) for k in range(K))
-            bound = K * 2.0 ** -50 * np.abs(A[i]).max() * np.abs(B[:, j]).max()
+            bound = K * 2.0 ** -49 * np.abs(A[i]).max() * np.abs(B[:, j]).max()
             assert abs(Fraction(C[i, j]) - exact) <= Fraction(bound) + Fraction(abs(float(exact))) * 2 ** -52
 
 
