@@ -270,7 +270,9 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
       float4 *outp = P.fwd && !direct ? P.part + ((size_t)U.z * P.Mp + m0 + rl) * P.Np + n0 : nullptr;
       // the warp's 24 columns of accumulators, four at a time: each output's nine diagonals recombined
       // exactly as an integer (diag_int, no FP64 instruction: measured the cheapest here) and rounded
-      // once to f64, or kept as four floats for a tile with several shares
+      // once to f64, or kept as four floats for a tile with several shares.  A unit of at most 28 slices
+      // has diagonal sums below 2^22 (9 x 1024 x 448), which convert to int on the FP32 pipe.
+      const bool small = U.nsl * kTK * 9 * 1024 < (1 << 22);
 #pragma unroll 1
       for (int c0 = 0; c0 < kEpiCols; c0 += 4) {
         float v[kS][4];
@@ -290,13 +292,19 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
             outp[col] = ok ? diag_combine4(v, c) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
             continue;
           }
-          const double val = ok ? output_value(diag_int(v, c), Erow, fexp_s[col]) : __longlong_as_double(0x7ff8000000000000ll);
+          // only the wanted outputs are recombined (a scattered tile keeps about a third of them)
+          int64_t at = -1;
           if (direct) {
-            if (m0 + rl < P.ldt && nsa[al])
-              P.tout[((P.atom0 + (int64_t)(n0 >> 2) + al) * 4 + k) * P.ldt + m0 + rl] = val;
+            if (m0 + rl < P.ldt && nsa[al]) at = ((P.atom0 + (int64_t)(n0 >> 2) + al) * 4 + k) * P.ldt + m0 + rl;
           } else if (row_wanted) {
             const int slot = stab[key_l * kScatAtoms + al];
-            if (slot >= 0) P.scat[((size_t)((n0 >> 2) + al) * P.cap + slot) * 24 + 6 * k + qq] = val;
+            if (slot >= 0) at = ((int64_t)((n0 >> 2) + al) * P.cap + slot) * 24 + 6 * k + qq;
+          }
+          if (at >= 0) {
+            const double val = !ok ? __longlong_as_double(0x7ff8000000000000ll)
+                               : small ? output_value(diag_int_small(v, c), Erow, fexp_s[col])
+                                       : output_value(diag_int(v, c), Erow, fexp_s[col]);
+            (direct ? P.tout : P.scat)[at] = val;
           }
         }
       }

@@ -338,6 +338,18 @@ __device__ __forceinline__ __int128 diag_int(const float (&v)[kS][W], int c) {
   return ((__int128)hi << 42) + lo;
 }
 
+// diag_int for diagonal sums below 2^22 in magnitude: each converts to int by one FP32 add of
+// 1.5 2^23 (the sum's integer lands in the low significand bits exactly) and one integer subtract.
+template <int W>
+__device__ __forceinline__ __int128 diag_int_small(const float (&v)[kS][W], int c) {
+  auto to_int = [](float f) { return __float_as_int(__fadd_rn(f, 12582912.0f)) - 0x4B400000; };
+  long long lo = 0;
+#pragma unroll
+  for (int d = 2; d < kS; ++d) lo += (long long)to_int(v[d][c]) << (kBits * (kS - 1 - d));
+  const long long hi = (long long)to_int(v[0][c]) * 64 + to_int(v[1][c]);
+  return ((__int128)hi << 42) + lo;
+}
+
 // S 2^e2 rounded once to the nearest f64 (ties to even), from its bits: integer operations only, except
 // where the result falls outside the normal range (never for these sums in practice).
 __device__ __forceinline__ double i128_to_double(__int128 S, int e2) {
