@@ -6,7 +6,9 @@
 // 128-row output tile) backward, from a list of the units with work -- round-robin over the grid.  The TMEM accumulators (nine
 // diagonals x 48 columns), the mbarriers and the stage ring are set up once per CTA, and the roles
 // run ahead of each other: warp 0 moves each slice's A and B blocks into a ring of four stages (bulk
-// copies counted on the stage's "full" barrier), lane 0 of warp 1 issues the slice's 13 MMAs and
+// copies counted on the stage's "full" barrier; in the forward a split warp per stage writes the B
+// block from the moments instead, as digit planes, and arrives on the same barrier), lane 0 of warp 1
+// issues the slice's 13 MMAs and
 // frees the stage ("empty") when they complete, and eight epilogue warps (two per TMEM lane quadrant,
 // 24 columns each) read the unit's accumulators once its last MMA has completed ("acc_full"),
 // recombine each output's diagonals exactly as an integer and round it once to f64 (or, for a tile with
@@ -23,10 +25,12 @@ namespace {
 namespace tg {
 using namespace tc;
 
-constexpr int kEpiWarps = 8;                   // two per TMEM lane quadrant
-constexpr int kThreadsP = 32 * (2 + kEpiWarps);  // producer warp, MMA warp, epilogue warps
+constexpr int kEpiWarps = 8;    // two per TMEM lane quadrant
+constexpr int kSplitWarps = 4;  // forward: the B digit planes of each slice, made in shared memory
+constexpr int kThreadsP = 32 * (2 + kEpiWarps + kSplitWarps);  // producer, MMA issuer, epilogue, split warps
 constexpr int kEpiCols = kTN / 2;              // columns per epilogue warp
 constexpr int kMaxUnitSlices = kMaxShareSlices;
+constexpr int kTileAtomsP = kTN / 4;  // atoms per tile (four columns each)
 
 struct Params {
   bool fwd;
@@ -35,8 +39,11 @@ struct Params {
   const int *Eexp;
   int ka;   // K slices per row of blocks (forward: every K slice of the table; backward: M1 / 16)
   int nmt;  // 128-row tiles of A
-  // B: blocks [ntiles][ka] of kS x kPlaneB bytes; F: [Np] column exponents
+  // B: blocks [ntiles][ka] of kS x kPlaneB bytes, or (W != NULL) made by the split warps from the
+  // moments W[natoms][cap][24] and the run map [natoms][nkeys]; F: [Np] column exponents
   const unsigned char *bplanes;
+  const double *W;
+  const int *map;
   const int *Fexp;
   int64_t ntiles, Np, Mp;
   // forward: the tile's used slices, in order ([ntiles][ka] and [ntiles]), in shares of 28
@@ -129,9 +136,10 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nunits = *P.nunits;
 
+  const bool fused = P.W != nullptr;  // B made in shared memory by the split warps
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
-      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(full + s)));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(full + s)), "r"(fused ? 2 : 1));
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(empty + s)));
     }
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(acc_full)));
@@ -167,17 +175,18 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
           const unsigned char *asrc = P.aplanes + ((size_t)U.mt * P.ka + sl) * (kS * kPlaneA);
           const unsigned char *bsrc = P.bplanes + ((size_t)U.tile * P.ka + sl) * (kS * kPlaneB);
           const uint32_t bar = smem_u32(full + st), dst = sbase + st * kStageBytes;
-          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"((uint32_t)kStageBytes)
-                       : "memory");
+          const uint32_t bytes = fused ? kS * kPlaneA : kStageBytes;
+          asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
           asm volatile(
               "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
               "l"(asrc), "r"((uint32_t)(kS * kPlaneA)), "r"(bar)
               : "memory");
-          asm volatile(
-              "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                  dst + kS * kPlaneA),
-              "l"(bsrc), "r"((uint32_t)(kS * kPlaneB)), "r"(bar)
-              : "memory");
+          if (!fused)
+            asm volatile(
+                "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                    dst + kS * kPlaneA),
+                "l"(bsrc), "r"((uint32_t)(kS * kPlaneB)), "r"(bar)
+                : "memory");
         }
       }
       g = __shfl_sync(0xffffffffu, g, 0);
@@ -223,6 +232,67 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
       }
     }
     __syncwarp();
+  } else if (warp >= 2 + kEpiWarps) {
+    // ---- split warps (forward): each slice's B block -- B[6 key + q][4 a + k] = W_a[k][(key, q)], the
+    // moments of the atom's run slot of that interval -- as balanced digit planes in the stage, in the
+    // tcgen05 K-major core-matrix layout.  Warp w owns stage w (the slices g with g % 4 == w), so four
+    // slices are made at once; a lane makes 12 pairs of K entries (never across a key, 6 being even),
+    // their slot and moment loads issued together, then a fence makes the writes visible to the tensor
+    // core and the warp arrives on the stage's "full" barrier.
+    static_assert(kSplitWarps == kStages, "a split warp per stage");
+    if (fused) {
+      const int w = warp - (2 + kEpiWarps);
+      constexpr int kPairs = kTN * kTK / 2 / 32;  // per lane and slice
+      int g = 0;
+      for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+        if (__shfl_sync(0xffffffffu, (int)*abortf, 0)) break;  // uniform over the warp
+        const Unit U = unit_of(P, u);
+        const int64_t a_base = (int64_t)U.tile * kTileAtomsP;
+        bool ok = true;
+        for (int j = 0; j < U.nsl; ++j, ++g) {
+          if (g % kStages != w) continue;  // another warp's stage
+          if (g >= kStages) {
+            int wv = 1;
+            if (lane == 0) wv = wait_or_abort(smem_u32(empty + w), (uint32_t)((g / kStages - 1) & 1), abortf);
+            ok = __shfl_sync(0xffffffffu, wv, 0) != 0;
+            if (!ok) break;
+          }
+          const int sl = P.slist[(size_t)U.tile * P.ka + U.z * kMaxUnitSlices + j];
+          int slot[kPairs];
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i) {  // the slots of the lane's pairs, loaded together
+            const int p = lane + 32 * i, r = p >> 3, kp = p & 7;
+            const int64_t a = a_base + (r >> 2);
+            const int key = (sl * kTK + 2 * kp) / 6;
+            slot[i] = (a < P.natoms && key < P.nkeys) ? P.map[a * P.nkeys + key] : -1;
+          }
+          double2 xv[kPairs];
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i) {  // then their moments
+            const int p = lane + 32 * i, r = p >> 3, kp = p & 7;
+            const int64_t a = a_base + (r >> 2);
+            const int k = r & 3, kk = sl * kTK + 2 * kp, q0 = kk - 6 * (kk / 6);
+            xv[i] = slot[i] >= 0 ? *reinterpret_cast<const double2 *>(P.W + ((size_t)a * P.cap + slot[i]) * 24 + 6 * k + q0)
+                                 : make_double2(0.0, 0.0);
+          }
+          unsigned char *bstage = smem + w * kStageBytes + kS * kPlaneA;
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i) {
+            const int p = lane + 32 * i, r = p >> 3, kp = p & 7;
+            const int E = P.Fexp[U.tile * kTN + r];
+            uint32_t h[kS];
+            digit_pairs(biased_fixed(xv[i].x, E), biased_fixed(xv[i].y, E), h);
+            unsigned char *dst = bstage + (r >> 3) * kSBO + (r & 7) * 16 + (kp >> 2) * kLBO + (kp & 3) * 4;
+#pragma unroll
+            for (int d = 0; d < kS; ++d) *reinterpret_cast<uint32_t *>(dst + d * kPlaneB) = h[d];
+          }
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          __syncwarp();
+          if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(full + w)) : "memory");
+        }
+        if (!ok) break;
+      }
+    }
   } else {
     // ---- epilogue: warps 2 .. 9, TMEM lane quadrant warp % 4, columns 24 ((warp - 2) / 4) .. + 23
     const int et = tid - 64;

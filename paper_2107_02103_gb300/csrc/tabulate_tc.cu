@@ -28,10 +28,10 @@
 //
 // C'_alpha and its digit planes are made once per table by dp_tabulate_tc_plan_f64 (the plan).
 // Per chunk of at most kChunkAtoms atoms and per centre type alpha:
-//   forward:  runs_kernel<true> (slot keys, W, column exponents, slice flags),
-//             split_mom_kernel (W -> B digit planes, used slices only), slice_list_kernel,
-//             tgemm_kernel (tab_gemm.cuh; A = C'_alpha^T: channels x K, B = W^T: K x (atom, k); a
-//             tile whose used slices fit one share writes its atoms' T directly),
+//   forward:  runs_kernel<true> (slot keys, W, column exponents, slice flags), slice_list_kernel,
+//             tgemm_kernel (tab_gemm.cuh; A = C'_alpha^T: channels x K, B = W^T: K x (atom, k), its
+//             digit planes made in shared memory from W; a tile whose used slices fit one share
+//             writes its atoms' T directly),
 //             fwd_epilogue_kernel (T of the tiles with several shares, or none);
 //   backward: runs_kernel<false> (slot keys, slice flags; skipped when the forward's are reused),
 //             split of dT (B), tgemm_kernel (A = C'_alpha: K x channels, B = dT^T) scattering
@@ -394,49 +394,6 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
 #pragma unroll
     for (int q = 1; q < 6; ++q) m = max(m, __shfl_sync(0xffffffffu, eb, min(lane + q, 31)));
     if (lane < 24 && lane % 6 == 0) P.fexp[kCols * a + lane / 6] = exp_of_max(m);
-  }
-}
-
-// The forward's B operand: B[6 key + q][4 a + k] = W_a[k][(key, q)] as digit planes with the column
-// exponents, in split_rows_kernel's block layout (RT = 48), for the slices some atom of the tile
-// uses (any centre type); the other blocks are never read.  One warp per (8 columns, 64 of K).
-__global__ void __launch_bounds__(128) split_mom_kernel(const double *__restrict__ W, const int *__restrict__ map,
-                                                        const int *__restrict__ fexp,
-                                                        const unsigned char *__restrict__ occ, int ntypes,
-                                                        int64_t tiles_all, int64_t tile0, int64_t natoms, int nkeys,
-                                                        int cap, int64_t rows_p, int Kp,
-                                                        unsigned char *__restrict__ planes) {
-  const int lane = threadIdx.x & 31, ri8 = lane >> 2, kp = lane & 3;
-  const int kchunks = (Kp + kSplitK - 1) / kSplitK;
-  const int nsl = Kp / kTK;
-  const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
-  const int64_t g8 = w / kchunks;
-  if (g8 * 8 >= rows_p) return;  // warp-uniform
-  const int kc = (int)(w - g8 * kchunks);
-  const int64_t r = g8 * 8 + ri8;  // column 4 a + k of the GEMM
-  const int64_t a = r >> 2;
-  const int k = (int)(r & 3);
-  const int64_t tile = r / kTN;   // the same for the warp's 8 columns
-  const int E = fexp[r];
-  constexpr size_t plane = (size_t)kTN * kTK * 2, block = kS * plane;
-  const int ri = (int)(r % kTN);
-  unsigned char *rowbase = planes + (size_t)tile * nsl * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
-  for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
-    const int sl = k0 / kTK;
-    bool used = false;
-    for (int t = 0; t < ntypes; ++t) used |= occ[((size_t)t * tiles_all + tile0 + tile) * nsl + sl] != 0;
-    if (!used) continue;  // uniform
-    const int kk = k0 + 2 * kp;  // this lane's two entries, of one key (6 is even)
-    const int key = kk / kQ, q0 = kk - kQ * key;
-    const int slot = (a < natoms && key < nkeys) ? map[a * nkeys + key] : -1;
-    const double *wp = W + ((size_t)a * cap + (slot >= 0 ? slot : 0)) * 24 + 6 * k;
-    const double x0 = slot >= 0 ? wp[q0] : 0.0;
-    const double x1 = slot >= 0 ? wp[q0 + 1] : 0.0;
-    uint32_t h[kS];
-    digit_pairs(biased_fixed(x0, E), biased_fixed(x1, E), h);
-    unsigned char *dst = rowbase + (size_t)sl * block + ((k0 % kTK) >> 3) * kLBO;
-#pragma unroll
-    for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
   }
 }
 
@@ -803,12 +760,6 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
                         kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_runs_moments", st);
-    const int64_t warps = Np / 8 * ((S.Kp + kSplitK - 1) / kSplitK);
-    split_mom_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(R.W, R.map, R.fexp, wk + L.occ, ntypes, S.tiles_all,
-                                                                   tile0, n, S.nkeys, S.cap, Np, S.Kp,
-                                                                   wk + L.bplanes);
-    if ((rc = launch_status(who))) return rc;
-    prof_mark("tc_split_moments", st);
     const int64_t nlist = (int64_t)ntypes * ntiles;
     if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
       return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
@@ -825,7 +776,10 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
       G.Eexp = reinterpret_cast<const int *>(pk + PL.efwd) + (size_t)t * S.Mpf;
       G.ka = S.nsl;
       G.nmt = S.Mpf / kTM;
-      G.bplanes = wk + L.bplanes;
+      G.W = R.W;  // B made from the moments inside the GEMM
+      G.map = R.map;
+      G.nkeys = S.nkeys;
+      G.cap = S.cap;
       G.Fexp = R.fexp;
       G.ntiles = ntiles;
       G.Np = Np;
