@@ -180,7 +180,8 @@ def moment_fmas(runs, M1: int) -> dict:
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
 # `ncu --set full` capture of its current version; absent means no capture of the current kernel
 # exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640}
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,
+                       ("cu85", "f64", "tc_rows", "tc"): 104700160 + 32997632}
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ, nsm: int = NSM) -> float:
