@@ -149,7 +149,7 @@ Layout make_layout(const Shape &s) {
   L.units = take(off, (size_t)s.ntypes * s.maxunits * sizeof(int));
   L.nunits = take(off, (size_t)s.ntypes * sizeof(int));
   L.fexp = take(off, (size_t)s.Np * sizeof(int));
-  L.bplanes = take(off, (size_t)s.ntiles * std::max(s.nsl, s.Kpm / kTK) * kS * kPlaneB);
+  L.bplanes = take(off, (size_t)s.ntiles * (s.Kpm / kTK) * kS * kPlaneB);  // the backward's dT planes
   L.w = take(off, (size_t)s.chunk * s.cap * 24 * sizeof(double));  // moments (forward) or their gradients
   L.part = take(off, (size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
   L.total = off;

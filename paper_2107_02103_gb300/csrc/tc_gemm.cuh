@@ -537,7 +537,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   __syncthreads();
   ok = flags[0] && flags[1];
   ok = mbar_wait(smem_u32(done), 0) && ok;
-  ok = __syncthreads_and(ok) != 0;  // one verdict for the CTA: its accumulators are read only if every wait ended
+  ok = __syncthreads_and(ok) != 0;  // one answer for the CTA: its accumulators are read only if every wait ended
   if (!ok && tid == 0) atomicAdd(&g_wait_timeouts, 1u);
   asm volatile("tcgen05.fence::after_thread_sync;");
 
