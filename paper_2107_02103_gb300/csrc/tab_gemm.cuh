@@ -338,11 +338,11 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
       const int key_l = P.fwd ? 0 : key - (int)(m0 / P.kq);
       const bool row_wanted = !P.fwd && qq < 6 && key < P.nkeys;
       float4 *outp = P.fwd && !direct ? P.part + ((size_t)U.z * P.Mp + m0 + rl) * P.Np + n0 : nullptr;
-      // the warp's 24 columns of accumulators, four at a time: each output's nine diagonals recombined
-      // exactly as an integer (diag_int, no FP64 instruction: measured the cheapest here) and rounded
-      // once to f64, or kept as four floats for a tile with several shares.  A unit of at most 28 slices
-      // has diagonal sums below 2^22 (9 x 1024 x 448), which convert to int on the FP32 pipe.
-      const bool small = U.nsl * kTK * 9 * 1024 < (1 << 22);
+      // the warp's 24 columns of accumulators, four (one atom) at a time: each output's nine diagonals
+      // recombined exactly as an integer and rounded once to f64 (diag_to_f64: integer operations, no
+      // branch, the four outputs interleaved), or kept as four floats for a tile with several shares.
+      // One copy of the loop body, so that it stays in the instruction cache (measured: two copies of
+      // it, or two conversion variants, made the epilogue several times slower).
 #pragma unroll 1
       for (int c0 = 0; c0 < kEpiCols; c0 += 4) {
         float v[kS][4];
@@ -353,29 +353,39 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
                          : "=f"(v[d][0]), "=f"(v[d][1]), "=f"(v[d][2]), "=f"(v[d][3])
                          : "r"(trow + (uint32_t)(d * kTN + c_lo + c0)));
           asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-        }
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const int col = c_lo + c0 + c;
-          const int al = col >> 2, k = col & 3;
-          if (outp) {
-            outp[col] = ok ? diag_combine4(v, c) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
-            continue;
-          }
-          // only the wanted outputs are recombined (a scattered tile keeps about a third of them)
-          int64_t at = -1;
-          if (direct) {
-            if (m0 + rl < P.ldt && nsa[al]) at = ((P.atom0 + (int64_t)(n0 >> 2) + al) * 4 + k) * P.ldt + m0 + rl;
-          } else if (row_wanted) {
-            const int slot = stab[key_l * kScatAtoms + al];
-            if (slot >= 0) at = ((int64_t)((n0 >> 2) + al) * P.cap + slot) * 24 + 6 * k + qq;
-          }
-          if (at >= 0) {
-            const double val = !ok ? __longlong_as_double(0x7ff8000000000000ll)
-                               : small ? output_value(diag_int_small(v, c), Erow, fexp_s[col])
-                                       : output_value(diag_int(v, c), Erow, fexp_s[col]);
-            (direct ? P.tout : P.scat)[at] = val;
-          }
+          for (int d = 0; d < kS; ++d) asm volatile("" : "+f"(v[d][0]), "+f"(v[d][1]), "+f"(v[d][2]), "+f"(v[d][3]));
+        }
+        const int al = (c_lo + c0) >> 2;  // the group's atom; column c0 + k is its component k
+        if (outp) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            outp[c_lo + c0 + k] = ok ? diag_combine4(v, k) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
+          continue;
+        }
+        // only the wanted outputs are stored; a warp skips a group none of its rows wants
+        int64_t at = -1, ldk = 0;
+        if (direct) {
+          if (m0 + rl < P.ldt && nsa[al]) at = (P.atom0 + (int64_t)(n0 >> 2) + al) * 4 * P.ldt + m0 + rl, ldk = P.ldt;
+        } else if (row_wanted) {
+          const int slot = stab[key_l * kScatAtoms + al];
+          if (slot >= 0) at = ((int64_t)((n0 >> 2) + al) * P.cap + slot) * 24 + qq, ldk = 6;
+        }
+        if (!__any_sync(0xffffffffu, at >= 0)) continue;
+        double val[4];
+        int F[4];
+        bool rare = false;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) F[k] = fexp_s[c_lo + c0 + k];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) val[k] = diag_to_f64(v, k, Erow, F[k], rare);
+        if (__any_sync(0xffffffffu, rare))  // warp-uniform, and never taken with these operands
+#pragma unroll
+          for (int k = 0; k < 4; ++k) val[k] = output_value(diag_int(v, k), Erow, F[k]);
+        if (at >= 0) {
+          double *dst = (direct ? P.tout : P.scat) + at;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) dst[k * ldk] = ok ? val[k] : __longlong_as_double(0x7ff8000000000000ll);
         }
       }
       asm volatile("tcgen05.fence::before_thread_sync;");

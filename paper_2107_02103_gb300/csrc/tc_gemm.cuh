@@ -385,6 +385,50 @@ __device__ __forceinline__ double output_value(__int128 S, int E, int F) {
   return i128_to_double(S, E + F + 2 * kPad - 2 * kBits - kBits * (kS - 1));
 }
 
+// The exponent offset of output_value: an output is S 2^(E + F + kOutExp).
+constexpr int kOutExp = 2 * kPad - 2 * kBits - kBits * (kS - 1);
+
+// output_value without branches, for the wide epilogues: the nine diagonal sums become
+// S = T 2^36 + M 2^18 + L (T, M, L each three diagonals, |.| < 2^36.03) as a 128-bit two's complement
+// pair, |S| is normalised by its leading-zero count, and the top 53 bits are rounded to nearest even from
+// the round bit and the sticky bits; the exponent is added into the bit pattern, so a rounding carry
+// moves into it.  Equal to output_value(diag_int(v, c), E, F) except where the result falls outside the
+// normal range (never with these operands), which sets `rare`: the caller then takes output_value for
+// the group, after all of its outputs, so that no call or branch sits between their independent
+// instruction chains (measured: a call site inside each conversion made it 3.5 times slower).
+template <int W>
+__device__ __forceinline__ double diag_to_f64(const float (&v)[kS][W], int c, int E, int F, bool &rare) {
+  static_assert(kS == 9 && kBits == 6, "three groups of three 6-bit diagonals");
+  int x[kS];
+#pragma unroll
+  for (int d = 0; d < kS; ++d) x[d] = exact_int(v[d][c]);
+  const long long T = (long long)x[0] * 4096 + (long long)x[1] * 64 + x[2];
+  const long long M = (long long)x[3] * 4096 + (long long)x[4] * 64 + x[5];
+  const long long L = (long long)x[6] * 4096 + (long long)x[7] * 64 + x[8];
+  const long long A = M * 262144 + L;  // |A| < 2^55
+  const unsigned long long tl = (unsigned long long)T << 36;
+  const unsigned long long lo = tl + (unsigned long long)A;
+  const long long hi = (T >> 28) + (A >> 63) + (lo < tl ? 1 : 0);
+  const unsigned long long sg = (unsigned long long)(hi >> 63);  // all ones when S < 0
+  const unsigned long long ml = (lo ^ sg) - sg;                   // |S|, low word
+  const unsigned long long mh = ((unsigned long long)hi ^ sg) + (sg & (ml == 0 ? 1ull : 0ull));
+  const bool top = mh != 0;
+  const int lz = top ? __clzll((long long)mh) : 64 + __clzll((long long)ml);
+  const unsigned long long hN = top ? mh : ml, lN = top ? ml : 0ull;
+  const int s1 = lz & 63;
+  const unsigned long long N = (hN << s1) | ((lN >> 1) >> (63 - s1));  // the leading 64 bits
+  const unsigned long long rest = lN << s1;
+  const unsigned long long mant = N >> 11;
+  const unsigned long long inc = ((N >> 10) & 1ull) & ((((N & 0x3ffull) | rest) != 0 ? 1ull : 0ull) | (mant & 1ull));
+  const int ex = 127 - lz + E + F + kOutExp;  // exponent of the leading bit
+  unsigned long long bits = (((unsigned long long)(ex + 1022) << 52) + mant + inc) | (sg << 63);
+  const bool nonfinite = E >= kNonFinite || F >= kNonFinite, zero = lz == 128;
+  rare |= !nonfinite && !zero && (unsigned)(ex + 1022) > 2045u;
+  bits = zero ? 0ull : bits;
+  bits = nonfinite ? 0x7ff8000000000000ull : bits;
+  return __longlong_as_double((long long)bits);
+}
+
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);  // stage loaded
