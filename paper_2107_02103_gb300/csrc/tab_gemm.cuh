@@ -236,52 +236,73 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
     // ---- split warps (forward): each slice's B block -- B[6 key + q][4 a + k] = W_a[k][(key, q)], the
     // moments of the atom's run slot of that interval -- as balanced digit planes in the stage, in the
     // tcgen05 K-major core-matrix layout.  Warp w owns stage w (the slices g with g % 4 == w), so four
-    // slices are made at once; a lane makes 12 pairs of K entries (never across a key, 6 being even),
-    // their slot and moment loads issued together, then a fence makes the writes visible to the tensor
-    // core and the warp arrives on the stage's "full" barrier.
+    // slices are made at once.  Lane (k = lane / 8, kp = lane % 8) makes the K entries 2 kp, 2 kp + 1 of
+    // column 4 i + k for the tile's atoms i = 0 .. 11 (one key per lane and slice, 6 being even): the
+    // column exponents and the unit's slice list are read once per unit, the run slots of the warp's
+    // next slice are loaded while this slice's moments are, and the stage is waited for only before
+    // the stores; then a fence makes the writes visible to the tensor core and the warp arrives on the
+    // stage's "full" barrier.  (Measured: with a global load chain per slice the tensor core waited
+    // ~0.6 us per slice for its B block.)
     static_assert(kSplitWarps == kStages, "a split warp per stage");
     if (fused) {
       const int w = warp - (2 + kEpiWarps);
-      constexpr int kPairs = kTN * kTK / 2 / 32;  // per lane and slice
-      int g = 0;
+      constexpr int kPairs = kTileAtomsP;  // per lane and slice: one pair of K entries per atom
+      static_assert(kTN * kTK / 2 == 32 * kPairs, "a pair per lane and atom");
+      const int k = lane >> 3, kp = lane & 7;
+      int g0 = 0;  // slices of this CTA before the unit
       for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
         if (__shfl_sync(0xffffffffu, (int)*abortf, 0)) break;  // uniform over the warp
         const Unit U = unit_of(P, u);
         const int64_t a_base = (int64_t)U.tile * kTileAtomsP;
+        const short *ulist = P.slist + (size_t)U.tile * P.ka + U.z * kMaxUnitSlices;
+        int E[kPairs];
+        bool av[kPairs];
+#pragma unroll
+        for (int i = 0; i < kPairs; ++i) {
+          E[i] = P.Fexp[U.tile * kTN + 4 * i + k];
+          av[i] = a_base + i < P.natoms;
+        }
+
+        auto load_slots = [&](int sl, int (&slot)[kPairs]) {
+          const int key = (sl * kTK + 2 * kp) / 6;
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i)
+            slot[i] = (av[i] && key < P.nkeys) ? P.map[(a_base + i) * P.nkeys + key] : -1;
+        };
+        int j = ((w - g0) % kStages + kStages) % kStages;  // the warp's first slice of the unit
+        // the warp's slices of the unit (at most 112 / 4 = 28): lane l holds entry j + 4 l of the list
+        static_assert(kMaxUnitSlices / kStages <= 32, "a lane per slice of the warp");
+        const int slr = j + kStages * lane < U.nsl ? ulist[j + kStages * lane] : 0;
+        const int j_first = j;
+        auto slice_at = [&](int jj) { return __shfl_sync(0xffffffffu, slr, ((jj - j_first) / kStages) & 31); };
+        int sl = j < U.nsl ? __shfl_sync(0xffffffffu, slr, 0) : 0;
+        int slot[kPairs], slotn[kPairs];
+        if (j < U.nsl) load_slots(sl, slot);
         bool ok = true;
-        for (int j = 0; j < U.nsl; ++j, ++g) {
-          if (g % kStages != w) continue;  // another warp's stage
+        for (; j < U.nsl; j += kStages) {
+          const int g = g0 + j;
+          const int jn = j + kStages;
+          const int sln = jn < U.nsl ? slice_at(jn) : 0;
+          if (jn < U.nsl) load_slots(sln, slotn);  // the next slice's slots, in flight with these moments
+          const int kk = sl * kTK + 2 * kp, q0 = kk - 6 * (kk / 6);
+          double2 xv[kPairs];
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i)
+            xv[i] = slot[i] >= 0
+                        ? *reinterpret_cast<const double2 *>(P.W + ((size_t)(a_base + i) * P.cap + slot[i]) * 24 + 6 * k + q0)
+                        : make_double2(0.0, 0.0);
           if (g >= kStages) {
             int wv = 1;
             if (lane == 0) wv = wait_or_abort(smem_u32(empty + w), (uint32_t)((g / kStages - 1) & 1), abortf);
             ok = __shfl_sync(0xffffffffu, wv, 0) != 0;
             if (!ok) break;
           }
-          const int sl = P.slist[(size_t)U.tile * P.ka + U.z * kMaxUnitSlices + j];
-          int slot[kPairs];
-#pragma unroll
-          for (int i = 0; i < kPairs; ++i) {  // the slots of the lane's pairs, loaded together
-            const int p = lane + 32 * i, r = p >> 3, kp = p & 7;
-            const int64_t a = a_base + (r >> 2);
-            const int key = (sl * kTK + 2 * kp) / 6;
-            slot[i] = (a < P.natoms && key < P.nkeys) ? P.map[a * P.nkeys + key] : -1;
-          }
-          double2 xv[kPairs];
-#pragma unroll
-          for (int i = 0; i < kPairs; ++i) {  // then their moments
-            const int p = lane + 32 * i, r = p >> 3, kp = p & 7;
-            const int64_t a = a_base + (r >> 2);
-            const int k = r & 3, kk = sl * kTK + 2 * kp, q0 = kk - 6 * (kk / 6);
-            xv[i] = slot[i] >= 0 ? *reinterpret_cast<const double2 *>(P.W + ((size_t)a * P.cap + slot[i]) * 24 + 6 * k + q0)
-                                 : make_double2(0.0, 0.0);
-          }
           unsigned char *bstage = smem + w * kStageBytes + kS * kPlaneA;
 #pragma unroll
           for (int i = 0; i < kPairs; ++i) {
-            const int p = lane + 32 * i, r = p >> 3, kp = p & 7;
-            const int E = P.Fexp[U.tile * kTN + r];
+            const int r = 4 * i + k;
             uint32_t h[kS];
-            digit_pairs(biased_fixed(xv[i].x, E), biased_fixed(xv[i].y, E), h);
+            digit_pairs(biased_fixed(xv[i].x, E[i]), biased_fixed(xv[i].y, E[i]), h);
             unsigned char *dst = bstage + (r >> 3) * kSBO + (r & 7) * 16 + (kp >> 2) * kLBO + (kp & 3) * 4;
 #pragma unroll
             for (int d = 0; d < kS; ++d) *reinterpret_cast<uint32_t *>(dst + d * kPlaneB) = h[d];
@@ -289,8 +310,12 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           __syncwarp();
           if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(full + w)) : "memory");
+          sl = sln;
+#pragma unroll
+          for (int i = 0; i < kPairs; ++i) slot[i] = slotn[i];
         }
         if (!ok) break;
+        g0 += U.nsl;
       }
     }
   } else {

@@ -45,6 +45,7 @@
 
 #include "dp_common.cuh"
 #include "tab_gemm.cuh"
+#include "tab_gemm_b8.cuh"
 #include "tc_gemm.cuh"
 
 namespace dpc {
@@ -73,6 +74,9 @@ struct Shape {
   int64_t chunk, Np, ntiles;  // atoms per chunk, its columns round_up(4 chunk, 48), Np / 48
   int zmax;                   // forward shares per tile at most
   int64_t maxunits;           // GEMM units per chunk and centre type at most
+  bool b8;                    // the backward GEMM uses the 7 x 8-bit digits on 8-atom tiles (Kpm <= 144)
+  int64_t Np8, ntiles8;       // its columns round_up(4 chunk, 32) and tiles Np8 / 32
+  int64_t maxunits8;          // its units per chunk and centre type at most
 };
 
 // The plan: C' of every centre type and the digit planes of both GEMMs' A operands.
@@ -104,6 +108,7 @@ Shape table_shape(const TableGeom &g, int ntypes, int M1) {
   s.Kpm = (int)round_up(M1, kTK);
   s.Mpb = (int)round_up(s.Kp, kTM);
   s.zmax = (s.nsl + kShareSlices - 1) / kShareSlices;
+  s.b8 = s.Kpm <= tb::kMaxKB;
   return s;
 }
 
@@ -120,6 +125,9 @@ Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1)
   s.Np = round_up(kCols * chunk, kTN);
   s.ntiles = s.Np / kTN;
   s.maxunits = s.ntiles * std::max<int64_t>((int64_t)(s.Mpf / kTM) * s.zmax, s.Mpb / kTM);
+  s.Np8 = round_up(kCols * chunk, tb::kTNB);
+  s.ntiles8 = s.Np8 / tb::kTNB;
+  s.maxunits8 = s.ntiles8 * (s.Mpb / kTM);
   return s;
 }
 
@@ -131,7 +139,7 @@ PlanLayout plan_layout(const Shape &s) {
   L.cp = take(off, nt * s.Kp * s.M1 * sizeof(double));
   L.afwd = take(off, nt * kS * (size_t)s.Mpf * s.Kp * 2);
   L.efwd = take(off, nt * s.Mpf * sizeof(int));
-  L.abwd = take(off, nt * kS * (size_t)s.Mpb * s.Kpm * 2);
+  L.abwd = take(off, nt * (s.b8 ? tb::kSB : kS) * (size_t)s.Mpb * s.Kpm * 2);
   L.ebwd = take(off, nt * s.Mpb * sizeof(int));
   L.total = off;
   return L;
@@ -146,10 +154,11 @@ Layout make_layout(const Shape &s) {
   L.map = take(off, (size_t)s.chunk * s.nkeys * sizeof(int));
   L.slist = take(off, (size_t)s.ntypes * s.ntiles * s.nsl * sizeof(short));
   L.scount = take(off, (size_t)s.ntypes * s.ntiles * sizeof(int));
-  L.units = take(off, (size_t)s.ntypes * s.maxunits * sizeof(int));
+  L.units = take(off, (size_t)s.ntypes * std::max(s.maxunits, s.maxunits8) * sizeof(int));
   L.nunits = take(off, (size_t)s.ntypes * sizeof(int));
-  L.fexp = take(off, (size_t)s.Np * sizeof(int));
-  L.bplanes = take(off, (size_t)s.ntiles * (s.Kpm / kTK) * kS * kPlaneB);  // the backward's dT planes
+  L.fexp = take(off, (size_t)std::max(s.Np, s.Np8) * sizeof(int));
+  L.bplanes = take(off, s.b8 ? (size_t)s.ntiles8 * (s.Kpm / kTK) * tb::kSB * tb::kPlaneBB  // the backward's dT planes
+                             : (size_t)s.ntiles * (s.Kpm / kTK) * kS * kPlaneB);
   L.w = take(off, (size_t)s.chunk * s.cap * 24 * sizeof(double));  // moments (forward) or their gradients
   L.part = take(off, (size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
   L.total = off;
@@ -449,6 +458,51 @@ __global__ void __launch_bounds__(128) bwd_units_kernel(const unsigned char *__r
   }
 }
 
+// The 7 x 8-bit backward GEMM's units: the (8-atom tile, 128-row output tile) pairs that hold the slot
+// of some atom of the tile of type t, from the atoms' slot keys (a key's rows are 6 key .. 6 key + 5),
+// per centre type; one warp per (type, tile), the row tiles marked in a shared-memory bit set.
+constexpr int kMaxRowTiles = 256;
+static_assert((int64_t)kMaxKeys * kQ <= (int64_t)kMaxRowTiles * kTM, "row tiles of the backward A fit the bit set");
+__global__ void __launch_bounds__(128) bwd_units8_kernel(const short *__restrict__ keys, const int *__restrict__ nslots,
+                                                         const int32_t *__restrict__ atype, int ntypes, int cap,
+                                                         int64_t atom0, int64_t natoms, int64_t ntiles8,
+                                                         int64_t maxunits8, int *__restrict__ units,
+                                                         int *__restrict__ nunits) {
+  __shared__ unsigned bits[4][kMaxRowTiles / 32];
+  const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
+  const int64_t w = (int64_t)blockIdx.x * 4 + wl;
+  if (w >= (int64_t)ntypes * ntiles8) return;  // warp-uniform
+  const int t = (int)(w / ntiles8);
+  const int64_t tile = w - (int64_t)t * ntiles8;
+  if (lane < kMaxRowTiles / 32) bits[wl][lane] = 0u;
+  __syncwarp();
+  for (int al = 0; al < tb::kAtomsB; ++al) {
+    const int64_t a = tile * tb::kAtomsB + al, i = atom0 + a;
+    if (a >= natoms || (atype && clampi(atype[i], 0, ntypes - 1) != t)) continue;  // warp-uniform
+    const int ns = nslots[i];
+    for (int slot = lane; slot < ns; slot += 32) {
+      const int r0 = kQ * (int)keys[i * cap + slot], m_lo = r0 / kTM, m_hi = (r0 + kQ - 1) / kTM;
+      atomicOr(&bits[wl][m_lo >> 5], 1u << (m_lo & 31));
+      atomicOr(&bits[wl][m_hi >> 5], 1u << (m_hi & 31));
+    }
+  }
+  __syncwarp();
+  const unsigned word = lane < kMaxRowTiles / 32 ? bits[wl][lane] : 0u;
+  const int cnt = __popc(word);
+  int before = cnt;  // inclusive prefix over the lanes
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, before, o);
+    if (lane >= o) before += y;
+  }
+  const int total = __shfl_sync(0xffffffffu, before, 31);
+  int base = 0;
+  if (lane == 0 && total) base = atomicAdd(nunits + t, total);
+  base = __shfl_sync(0xffffffffu, base, 0) + before - cnt;
+  for (unsigned m = word; m; m &= m - 1u)
+    units[(size_t)t * maxunits8 + base++] = tb::unit_code((int)tile, 32 * lane + __ffs((int)m) - 1);
+}
+
 // T for the atoms of type alpha of one 12-atom tile (one block) whose used slices take several shares
 // (one per kShareSlices; a single share's GEMM writes T itself) or none (T = 0): the shares summed in
 // a three-float sum and scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at a time: read with
@@ -674,9 +728,13 @@ int make_plan(const double *table, const dp_table_info *info, int nnei, int ntyp
     const double *Ct = Cp + (size_t)t * s.Kp * s.M1;
     rc = split_rows(Ct, 1, s.M1, s.M1, s.Kp, s.Mpf, s.Kp, kTM, wk + P.afwd + (size_t)t * kS * s.Mpf * s.Kp * 2,
                     wk + P.efwd + (size_t)t * s.Mpf * sizeof(int), st, who);
-    if (!rc)
-      rc = split_rows(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM, wk + P.abwd + (size_t)t * kS * s.Mpb * s.Kpm * 2,
-                      wk + P.ebwd + (size_t)t * s.Mpb * sizeof(int), st, who);
+    unsigned char *eb = wk + P.ebwd + (size_t)t * s.Mpb * sizeof(int);
+    if (!rc && s.b8)
+      rc = split_rows<Digits7x8>(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM,
+                                 wk + P.abwd + (size_t)t * tb::kSB * s.Mpb * s.Kpm * 2, eb, st, who);
+    else if (!rc)
+      rc = split_rows(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM, wk + P.abwd + (size_t)t * kS * s.Mpb * s.Kpm * 2, eb,
+                      st, who);
   }
   if (rc) return rc;
   out->data = buf;
@@ -863,49 +921,89 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
       if ((rc = launch_status(who))) return rc;
       prof_mark("tc_runs", st);
     }
-    // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
-    if ((rc = split_rows(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, Np, S.Kpm, kTN, wk + L.bplanes, wk + L.fexp, st,
-                         who)))
-      return rc;
-    prof_mark("tc_split_dT", st);
-    if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
-      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
-    const int64_t nlist = (int64_t)ntypes * ntiles;
-    bwd_units_kernel<<<(unsigned)((nlist + 127) / 128), 128, 0, st>>>(wk + L.occ, S.tiles_all, tile0, ntiles, ntypes,
-                                                                      S.nsl, mtiles, S.maxunits,
-                                                                      reinterpret_cast<int *>(wk + L.units),
-                                                                      reinterpret_cast<int *>(wk + L.nunits));
-    if ((rc = launch_status(who))) return rc;
-    prof_mark("tc_units", st);
-    for (int t = 0; t < ntypes; ++t) {
-      tg::Params G{};
-      G.fwd = false;
-      G.aplanes = pk + PL.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
-      G.Eexp = reinterpret_cast<const int *>(pk + PL.ebwd) + (size_t)t * S.Mpb;
-      G.ka = S.Kpm / kTK;
-      G.nmt = mtiles;
-      G.bplanes = wk + L.bplanes;
-      G.Fexp = R.fexp;
-      G.ntiles = ntiles;
-      G.Np = Np;
-      G.Mp = S.Mpb;
-      G.sflags = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
-      G.nsf = S.nsl;
-      G.scat = dW;
-      G.keys = R.keys;
-      G.nslots = R.nslots;
-      G.cap = S.cap;
-      G.nkeys = S.nkeys;
-      G.kq = kQ;
-      G.atype = atype;
-      G.natoms = n;
-      G.atom0 = c0;
-      G.alpha = t;
-      G.ntypes = ntypes;
-      G.units = reinterpret_cast<const int *>(wk + L.units) + (size_t)t * S.maxunits;
-      G.nunits = reinterpret_cast<const int *>(wk + L.nunits) + t;
-      if ((rc = tg::launch(G, st, who))) return rc;
-      prof_mark("tc_gemm_grad", st);
+    if (S.b8) {
+      // B = dT^T on 8-atom tiles in the 7 x 8-bit digits: the columns 4 a + k are the rows of this chunk's dT
+      if ((rc = split_rows<Digits7x8>(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, round_up(kCols * n, tb::kTNB),
+                                      S.Kpm, tb::kTNB, wk + L.bplanes, wk + L.fexp, st, who)))
+        return rc;
+      prof_mark("tc_split_dT", st);
+      if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
+        return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+      const int64_t ntiles8 = (n + tb::kAtomsB - 1) / tb::kAtomsB, nlist = (int64_t)ntypes * ntiles8;
+      bwd_units8_kernel<<<(unsigned)((nlist + 3) / 4), 128, 0, st>>>(
+          R.keys, R.nslots, atype, ntypes, S.cap, c0, n, ntiles8, S.maxunits8, reinterpret_cast<int *>(wk + L.units),
+          reinterpret_cast<int *>(wk + L.nunits));
+      if ((rc = launch_status(who))) return rc;
+      prof_mark("tc_units", st);
+      for (int t = 0; t < ntypes; ++t) {
+        tb::Params G{};
+        G.aplanes = pk + PL.abwd + (size_t)t * tb::kSB * S.Mpb * S.Kpm * 2;
+        G.Eexp = reinterpret_cast<const int *>(pk + PL.ebwd) + (size_t)t * S.Mpb;
+        G.ka = S.Kpm / kTK;
+        G.bplanes = wk + L.bplanes;
+        G.Fexp = R.fexp;
+        G.Mp = S.Mpb;
+        G.scat = dW;
+        G.keys = R.keys;
+        G.nslots = R.nslots;
+        G.cap = S.cap;
+        G.nkeys = S.nkeys;
+        G.kq = kQ;
+        G.atype = atype;
+        G.natoms = n;
+        G.atom0 = c0;
+        G.alpha = t;
+        G.ntypes = ntypes;
+        G.units = reinterpret_cast<const int *>(wk + L.units) + (size_t)t * S.maxunits8;
+        G.nunits = reinterpret_cast<const int *>(wk + L.nunits) + t;
+        if ((rc = tb::launch(G, st, who))) return rc;
+        prof_mark("tc_gemm_grad", st);
+      }
+    } else {
+      // B = dT^T: the columns 4 a + k are the rows of this chunk's dT
+      if ((rc = split_rows(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, Np, S.Kpm, kTN, wk + L.bplanes, wk + L.fexp, st,
+                           who)))
+        return rc;
+      prof_mark("tc_split_dT", st);
+      if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
+        return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
+      const int64_t nlist = (int64_t)ntypes * ntiles;
+      bwd_units_kernel<<<(unsigned)((nlist + 127) / 128), 128, 0, st>>>(wk + L.occ, S.tiles_all, tile0, ntiles, ntypes,
+                                                                        S.nsl, mtiles, S.maxunits,
+                                                                        reinterpret_cast<int *>(wk + L.units),
+                                                                        reinterpret_cast<int *>(wk + L.nunits));
+      if ((rc = launch_status(who))) return rc;
+      prof_mark("tc_units", st);
+      for (int t = 0; t < ntypes; ++t) {
+        tg::Params G{};
+        G.fwd = false;
+        G.aplanes = pk + PL.abwd + (size_t)t * kS * S.Mpb * S.Kpm * 2;
+        G.Eexp = reinterpret_cast<const int *>(pk + PL.ebwd) + (size_t)t * S.Mpb;
+        G.ka = S.Kpm / kTK;
+        G.nmt = mtiles;
+        G.bplanes = wk + L.bplanes;
+        G.Fexp = R.fexp;
+        G.ntiles = ntiles;
+        G.Np = Np;
+        G.Mp = S.Mpb;
+        G.sflags = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
+        G.nsf = S.nsl;
+        G.scat = dW;
+        G.keys = R.keys;
+        G.nslots = R.nslots;
+        G.cap = S.cap;
+        G.nkeys = S.nkeys;
+        G.kq = kQ;
+        G.atype = atype;
+        G.natoms = n;
+        G.atom0 = c0;
+        G.alpha = t;
+        G.ntypes = ntypes;
+        G.units = reinterpret_cast<const int *>(wk + L.units) + (size_t)t * S.maxunits;
+        G.nunits = reinterpret_cast<const int *>(wk + L.nunits) + t;
+        if ((rc = tg::launch(G, st, who))) return rc;
+        prof_mark("tc_gemm_grad", st);
+      }
     }
     Q.atom0 = c0;
     Q.natoms = n;

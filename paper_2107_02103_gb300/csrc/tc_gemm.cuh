@@ -92,28 +92,52 @@ __device__ __forceinline__ int exp_bits(double x) { return (int)(((uint64_t)__do
 // E with max |x| < 2^E from the largest biased exponent (normal x: |x| < 2^(eb - 1022))
 __device__ __forceinline__ int exp_of_max(int ebmax) { return ebmax == 0x7ff ? kNonFinite : max(ebmax, 1) - 1022; }
 
-// x 2^(kFrac - E) truncated toward zero (|x| < 2^E, so |.| < 2^kFrac), plus kDigitBias (see digit_pairs)
+// A digit scheme: NS balanced digits of NB bits (digit 1 in [-2^(NB-1), 2^(NB-1)], the others in
+// [-2^(NB-1), 2^(NB-1) - 1]) for an element's NS NB - 1 fractional bits.  The tensor-core GEMMs use 9 x 6
+// bits (kS, kBits: a share of K up to kMaxShareK = 1792) or, where K <= 144, 7 x 8 bits (products up to
+// 2^14, seven of them on a diagonal: 7 x 2^14 x 144 < 2^24), which needs 28 digit products instead of 45.
+template <int NS, int NB>
+struct Digits {
+  static constexpr int kNS = NS, kNB = NB;
+  static constexpr int kFrac = NS * NB - 1;
+  static constexpr int kPad = NS * NB - kFrac;  // a digit vector stands for 2^(E + kPad) sum_s d_s 2^(-NB s)
+  static constexpr int64_t kBias = (1ll << (NB - 1)) * ((1ll << (NB * (NS - 1))) - 1ll) / ((1ll << NB) - 1ll);
+  static constexpr uint32_t kHalf = 1u << (NB - 1);
+  // the fp16 pair 1024 + kHalf: field u in [0, 2^NB] is encoded as 0x6400 | u (1024 + u) and this comes off
+  static constexpr uint32_t kOffPair = (0x6400u + kHalf) * 0x10001u;
+  static_assert(kBias < (1ll << (NB * (NS - 1))) && NB * (NS - 1) <= 56 && NB <= 9, "balanced top digit in range");
+};
+using Digits9x6 = Digits<9, 6>;
+using Digits7x8 = Digits<7, 8>;
+static_assert(Digits9x6::kBias == kDigitBias && Digits9x6::kFrac == kFrac && Digits9x6::kPad == kPad, "the 9 x 6 scheme");
+static_assert(Digits7x8::kFrac == 55 && Digits7x8::kPad == 1 && Digits7x8::kBias < (1ll << 48), "the 7 x 8 scheme");
+
+// x 2^(kFrac - E) truncated toward zero (|x| < 2^E, so |.| < 2^kFrac), plus the scheme's bias (see digit_pairs)
+template <class D = Digits9x6>
 __device__ __forceinline__ int64_t biased_fixed(double x, int E) {
   const uint64_t b = (uint64_t)__double_as_longlong(x);
   const int eb = (int)((b >> 52) & 0x7ff);
   const uint64_t mant = b & 0xfffffffffffffull;
   const uint64_t m = eb ? (mant | (1ull << 52)) : mant;
-  const int sh = (eb ? eb - 1075 : -1074) - E + kFrac;  // |x| 2^(kFrac - E) = m 2^sh, sh <= 0 for finite x
+  const int sh = (eb ? eb - 1075 : -1074) - E + D::kFrac;  // |x| 2^(kFrac - E) = m 2^sh, sh <= kFrac - 53 for finite x
   const int64_t mag = (int64_t)(sh >= 0 ? m << min(sh, 10) : (sh > -64 ? m >> -sh : 0ull));
-  return (b >> 63 ? -mag : mag) + kDigitBias;
+  return (b >> 63 ? -mag : mag) + D::kBias;
 }
 
-// The kS balanced digits of two elements from their biased fixed points g, digit s of both packed as an
-// fp16 pair (element 0 in the low half): field u in [0, 64] (digit + 32) is encoded as 0x6400 | u, the
-// fp16 1024 + u, and 1056 comes off exactly.  Digits 2 .. 9 are the eight low fields; digit 1 is g >> 48.
-__device__ __forceinline__ void digit_pairs(int64_t g0, int64_t g1, uint32_t (&h)[kS]) {
-  constexpr uint32_t kMask = (1u << kBits) - 1;
+// The NS balanced digits of two elements from their biased fixed points g, digit s of both packed as an
+// fp16 pair (element 0 in the low half): field u in [0, 2^NB] (digit + 2^(NB-1)) is encoded as 0x6400 | u,
+// the fp16 1024 + u, and 1024 + 2^(NB-1) comes off exactly.  Digits 2 .. NS are the low NB-bit fields;
+// digit 1 is g shifted right by NB (NS - 1).
+template <class D = Digits9x6>
+__device__ __forceinline__ void digit_pairs(int64_t g0, int64_t g1, uint32_t (&h)[D::kNS]) {
+  constexpr int NS = D::kNS, NB = D::kNB;
+  constexpr uint32_t kMask = (1u << NB) - 1;
 #pragma unroll
-  for (int s = 1; s <= kS; ++s) {
-    const int sh = kBits * (kS - s);
-    const uint32_t d0 = s == 1 ? (uint32_t)((g0 >> sh) + 32) : (uint32_t)(g0 >> sh) & kMask;
-    const uint32_t d1 = s == 1 ? (uint32_t)((g1 >> sh) + 32) : (uint32_t)(g1 >> sh) & kMask;
-    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(h[s - 1]) : "r"(0x64006400u | d0 | (d1 << 16)), "r"(0x64206420u));
+  for (int s = 1; s <= NS; ++s) {
+    const int sh = NB * (NS - s);
+    const uint32_t d0 = s == 1 ? (uint32_t)((g0 >> sh) + D::kHalf) : (uint32_t)(g0 >> sh) & kMask;
+    const uint32_t d1 = s == 1 ? (uint32_t)((g1 >> sh) + D::kHalf) : (uint32_t)(g1 >> sh) & kMask;
+    asm("sub.rn.f16x2 %0, %1, %2;" : "=r"(h[s - 1]) : "r"(0x64006400u | d0 | (d1 << 16)), "r"(D::kOffPair));
   }
 }
 
@@ -141,6 +165,7 @@ __global__ void __launch_bounds__(128) row_exps_kernel(const double *__restrict_
 }
 
 constexpr int kSplitK = 64;  // K per warp of split_rows_kernel
+template <class D>
 __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
                                                          int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
                                                          unsigned char *__restrict__ planes,
@@ -157,17 +182,18 @@ __global__ void __launch_bounds__(128) split_rows_kernel(const double *__restric
   const double *__restrict__ xr = X + (r < nrows ? r : 0) * ld_r;
   auto x = [&](int k) { return (r < nrows && k < K) ? __ldg(xr + k * ld_k) : 0.0; };
   const int E = exps[r];
-  const size_t plane = (size_t)RT * kTK * 2, block = kS * plane;
+  constexpr int NS = D::kNS;
+  const size_t plane = (size_t)RT * kTK * 2, block = NS * plane;
   const int ri = (int)(r % RT);
   unsigned char *rowbase = planes + (size_t)(r / RT) * (Kp / kTK) * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
   for (int k0 = kc * kSplitK; k0 < min(Kp, kc * kSplitK + kSplitK); k0 += 8) {
     const int k = k0 + 2 * kp;
     const double x0 = x(k), x1 = x(k + 1);
-    uint32_t h[kS];
-    digit_pairs(biased_fixed(x0, E), biased_fixed(x1, E), h);
+    uint32_t h[NS];
+    digit_pairs<D>(biased_fixed<D>(x0, E), biased_fixed<D>(x1, E), h);
     unsigned char *dst = rowbase + (size_t)(k0 / kTK) * block + ((k0 % kTK) >> 3) * kLBO;
 #pragma unroll
-    for (int s = 0; s < kS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
+    for (int s = 0; s < NS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
   }
 }
 
@@ -388,14 +414,39 @@ __device__ __forceinline__ double output_value(__int128 S, int E, int F) {
 // The exponent offset of output_value: an output is S 2^(E + F + kOutExp).
 constexpr int kOutExp = 2 * kPad - 2 * kBits - kBits * (kS - 1);
 
+// S 2^(E + F + X) rounded once to the nearest double (ties to even), S the two's complement pair (hi, lo)
+// with |S| < 2^126, without branches: |S| is normalised by its leading-zero count, the top 53 bits are
+// rounded from the round bit and the sticky bits, and the exponent is added into the bit pattern, so a
+// rounding carry moves into it.  Sets `rare` where the result falls outside the normal range (never with
+// these operands; the caller then takes output_value), NaN for a row or column with an inf or NaN.
+template <int X>
+__device__ __forceinline__ double s128_to_f64(long long hi, unsigned long long lo, int E, int F, bool &rare) {
+  const unsigned long long sg = (unsigned long long)(hi >> 63);  // all ones when S < 0
+  const unsigned long long ml = (lo ^ sg) - sg;                   // |S|, low word
+  const unsigned long long mh = ((unsigned long long)hi ^ sg) + (sg & (ml == 0 ? 1ull : 0ull));
+  const bool top = mh != 0;
+  const int lz = top ? __clzll((long long)mh) : 64 + __clzll((long long)ml);
+  const unsigned long long hN = top ? mh : ml, lN = top ? ml : 0ull;
+  const int s1 = lz & 63;
+  const unsigned long long N = (hN << s1) | ((lN >> 1) >> (63 - s1));  // the leading 64 bits
+  const unsigned long long rest = lN << s1;
+  const unsigned long long mant = N >> 11;
+  const unsigned long long inc = ((N >> 10) & 1ull) & ((((N & 0x3ffull) | rest) != 0 ? 1ull : 0ull) | (mant & 1ull));
+  const int ex = 127 - lz + E + F + X;  // exponent of the leading bit
+  unsigned long long bits = (((unsigned long long)(ex + 1022) << 52) + mant + inc) | (sg << 63);
+  const bool nonfinite = E >= kNonFinite || F >= kNonFinite, zero = lz == 128;
+  rare |= !nonfinite && !zero && (unsigned)(ex + 1022) > 2045u;
+  bits = zero ? 0ull : bits;
+  bits = nonfinite ? 0x7ff8000000000000ull : bits;
+  return __longlong_as_double((long long)bits);
+}
+
 // output_value without branches, for the wide epilogues: the nine diagonal sums become
 // S = T 2^36 + M 2^18 + L (T, M, L each three diagonals, |.| < 2^36.03) as a 128-bit two's complement
-// pair, |S| is normalised by its leading-zero count, and the top 53 bits are rounded to nearest even from
-// the round bit and the sticky bits; the exponent is added into the bit pattern, so a rounding carry
-// moves into it.  Equal to output_value(diag_int(v, c), E, F) except where the result falls outside the
-// normal range (never with these operands), which sets `rare`: the caller then takes output_value for
-// the group, after all of its outputs, so that no call or branch sits between their independent
-// instruction chains (measured: a call site inside each conversion made it 3.5 times slower).
+// pair, rounded by s128_to_f64.  Equal to output_value(diag_int(v, c), E, F) except where `rare` is set:
+// the caller then takes output_value for the group, after all of its outputs, so that no call or branch
+// sits between their independent instruction chains (measured: a call site inside each conversion made
+// it 3.5 times slower).
 template <int W>
 __device__ __forceinline__ double diag_to_f64(const float (&v)[kS][W], int c, int E, int F, bool &rare) {
   static_assert(kS == 9 && kBits == 6, "three groups of three 6-bit diagonals");
@@ -409,24 +460,35 @@ __device__ __forceinline__ double diag_to_f64(const float (&v)[kS][W], int c, in
   const unsigned long long tl = (unsigned long long)T << 36;
   const unsigned long long lo = tl + (unsigned long long)A;
   const long long hi = (T >> 28) + (A >> 63) + (lo < tl ? 1 : 0);
-  const unsigned long long sg = (unsigned long long)(hi >> 63);  // all ones when S < 0
-  const unsigned long long ml = (lo ^ sg) - sg;                   // |S|, low word
-  const unsigned long long mh = ((unsigned long long)hi ^ sg) + (sg & (ml == 0 ? 1ull : 0ull));
-  const bool top = mh != 0;
-  const int lz = top ? __clzll((long long)mh) : 64 + __clzll((long long)ml);
-  const unsigned long long hN = top ? mh : ml, lN = top ? ml : 0ull;
-  const int s1 = lz & 63;
-  const unsigned long long N = (hN << s1) | ((lN >> 1) >> (63 - s1));  // the leading 64 bits
-  const unsigned long long rest = lN << s1;
-  const unsigned long long mant = N >> 11;
-  const unsigned long long inc = ((N >> 10) & 1ull) & ((((N & 0x3ffull) | rest) != 0 ? 1ull : 0ull) | (mant & 1ull));
-  const int ex = 127 - lz + E + F + kOutExp;  // exponent of the leading bit
-  unsigned long long bits = (((unsigned long long)(ex + 1022) << 52) + mant + inc) | (sg << 63);
-  const bool nonfinite = E >= kNonFinite || F >= kNonFinite, zero = lz == 128;
-  rare |= !nonfinite && !zero && (unsigned)(ex + 1022) > 2045u;
-  bits = zero ? 0ull : bits;
-  bits = nonfinite ? 0x7ff8000000000000ull : bits;
-  return __longlong_as_double((long long)bits);
+  return s128_to_f64<kOutExp>(hi, lo, E, F, rare);
+}
+
+// The 7 x 8-bit scheme (Digits7x8): seven diagonal sums, diagonal d weighing 256^-(d+2), as one exact
+// integer S = sum_d v[d][c] 2^(8 (6 - d)), |S| < 2^72.01; an output is S 2^(E + F + kOutExp7x8).
+constexpr int kOutExp7x8 = 2 * Digits7x8::kPad - 2 * 8 - 8 * 6;
+template <int W>
+__device__ __forceinline__ __int128 diag7_int(const float (&v)[7][W], int c) {
+  long long A = 0;  // diagonals 3 .. 6: below 2^24 2^24 256/255 < 2^49
+#pragma unroll
+  for (int d = 3; d < 7; ++d) A += (long long)exact_int(v[d][c]) << (8 * (6 - d));
+  const long long T = (long long)exact_int(v[0][c]) * 65536 + (long long)exact_int(v[1][c]) * 256 + exact_int(v[2][c]);
+  return ((__int128)T << 32) + A;
+}
+template <int W>
+__device__ __forceinline__ double diag7_to_f64(const float (&v)[7][W], int c, int E, int F, bool &rare) {
+  int x[7];
+#pragma unroll
+  for (int d = 0; d < 7; ++d) x[d] = exact_int(v[d][c]);
+  const long long T = (long long)x[0] * 65536 + (long long)x[1] * 256 + x[2];  // |T| < 2^40.01
+  const long long A = (long long)x[3] * 16777216 + (long long)x[4] * 65536 + (long long)x[5] * 256 + x[6];  // < 2^48.01
+  const unsigned long long tl = (unsigned long long)T << 32;
+  const unsigned long long lo = tl + (unsigned long long)A;
+  const long long hi = (T >> 32) + (A >> 63) + (lo < tl ? 1 : 0);
+  return s128_to_f64<kOutExp7x8>(hi, lo, E, F, rare);
+}
+__device__ __forceinline__ double output_value7(__int128 S, int E, int F) {
+  if (E >= kNonFinite || F >= kNonFinite) return __longlong_as_double(0x7ff8000000000000ll);
+  return i128_to_double(S, E + F + kOutExp7x8);
 }
 
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {
@@ -650,6 +712,7 @@ int set_smem(const char *who) {
   return DP_OK;
 }
 
+template <class D = Digits9x6>
 int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
                unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
   row_exps_kernel<<<(unsigned)((rows_p + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p,
@@ -657,7 +720,7 @@ int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K
   int rc = launch_status(who);
   if (rc) return rc;
   const int64_t warps = rows_p / 8 * ((Kp + kSplitK - 1) / kSplitK);
-  split_rows_kernel<<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT, planes,
+  split_rows_kernel<D><<<(unsigned)((warps + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT, planes,
                                                                  reinterpret_cast<const int *>(exps));
   return launch_status(who);
 }
