@@ -279,9 +279,9 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  *                     slot keys (int16, one per interval an atom uses), their
  *                     counts and the used-slice flags of every atom (kept
  *                     from the forward for the backward), and for one chunk
- *                     of at most 4104 atoms the moments or their gradients
- *                     per (atom, interval), the B digit planes and partial
- *                     results.  Calls sharing a work buffer must not overlap
+ *                     of at most 16416 atoms the moments or their gradients
+ *                     per (atom, interval), the backward's B digit planes,
+ *                     the forward's schedule and its partial results.  Calls sharing a work buffer must not overlap
  *                     on the GPU.
  *   flags (backward)  0, or DP_TC_REUSE_RUNS: the forward call on the same
  *                     plan, s, nvalid, atype, nloc and work buffer ran before

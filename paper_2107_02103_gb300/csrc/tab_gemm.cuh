@@ -26,6 +26,7 @@ namespace tg {
 using namespace tc;
 
 constexpr int kEpiWarps = 8;    // two per TMEM lane quadrant
+constexpr long long kPartNaN = 1ll << 62;  // high word of a piece's output whose accumulators were not read
 constexpr int kSplitWarps = 4;  // forward: the B digit planes of each slice, made in shared memory
 constexpr int kThreadsP = 32 * (2 + kEpiWarps + kSplitWarps);  // producer, MMA issuer, epilogue, split warps
 constexpr int kEpiCols = kTN / 2;              // columns per epilogue warp
@@ -50,7 +51,7 @@ struct Params {
   const short *slist;
   const int *scount;
   int zmax;
-  float4 *part;  // [zmax][Mp][Np]: results of tiles with several shares (four floats, see diag_combine)
+  longlong2 *part;  // [slot][48][Mp]: exact integers (lo, hi) of the pieces of cut items (see diag_s128)
   double *tout;  // T, written by tiles with one share: [(atom0 + a) 4 + k][ldt]
   int ldt;
   // backward: output tile (tile, mt) wanted when one of K slices 8 mt .. 8 mt + 7 is flagged
@@ -60,11 +61,19 @@ struct Params {
   const short *keys;
   const int *nslots;
   int cap, nkeys, kq;
+  // forward, every centre type in one launch: the pieces of work (int4: tile; type | mt << 4 | slices << 8;
+  // first slice in the tile's list; part slot, or -1 for a tile whose T the piece writes itself), CTA b
+  // taking pieces cta_start[b] .. cta_start[b + 1] - 1 in order; per type, the A planes lie astride
+  // bytes apart, the row exponents estride apart, the slice lists and counts ntiles ka and ntiles apart
+  const int4 *pieces;
+  const int *cta_start;
+  size_t astride;
+  int estride;
   // both
   const int32_t *atype;
   int64_t natoms, atom0;
-  int alpha, ntypes;
-  const int *units;   // the launch's units, packed (unit_code), in any order
+  int alpha, ntypes;  // backward: the launch's centre type
+  const int *units;   // backward: the launch's units, packed (unit_code), in any order
   const int *nunits;  // their count (device)
 };
 
@@ -73,18 +82,41 @@ __host__ __device__ constexpr int unit_code(int tile, int mt, int z) { return ti
 
 struct Unit {
   int64_t tile;
-  int mt, z, nsl;  // nsl = 0: nothing to do
+  int alpha, mt, s0, nsl, slot;  // centre type, 128-row tile of A, first slice and slice count, part slot
 };
 
-// Unit i of the launch's list (every role walks the same list).
+// Unit i of the CTA's walk (every role walks the same units).
+template <bool kFwd>
 __device__ __forceinline__ Unit unit_of(const Params &P, int i) {
-  const int c = P.units[i];
   Unit U;
-  U.tile = c & 0xffff;
-  U.mt = (c >> 16) & 0xff;
-  U.z = (c >> 24) & 0xff;
-  U.nsl = P.fwd ? min(P.scount[U.tile] - U.z * kMaxUnitSlices, kMaxUnitSlices) : P.ka;
+  if (kFwd) {
+    const int4 c = P.pieces[i];
+    U.tile = c.x;
+    U.alpha = c.y & 15;
+    U.mt = (c.y >> 4) & 15;
+    U.nsl = c.y >> 8;
+    U.s0 = c.z;
+    U.slot = c.w;
+  } else {
+    const int c = P.units[i];
+    U.tile = c & 0xffff;
+    U.alpha = P.alpha;
+    U.mt = (c >> 16) & 0xff;
+    U.nsl = P.ka;
+    U.s0 = 0;
+    U.slot = -1;
+  }
   return U;
+}
+
+// The CTA's units: forward its pieces in order, backward the launch's list round-robin.
+struct Walk {
+  int begin, end, step;
+};
+template <bool kFwd>
+__device__ __forceinline__ Walk walk_of(const Params &P) {
+  if (kFwd) return Walk{P.cta_start[blockIdx.x], P.cta_start[blockIdx.x + 1], 1};
+  return Walk{(int)blockIdx.x, *P.nunits, (int)gridDim.x};
 }
 
 // A wait on an mbarrier phase, bounded in time (2 s on the global timer), that also gives up once another
@@ -120,6 +152,10 @@ constexpr size_t kStabOff = kListOff + kMaxUnitSlices * 4;     // epilogue: slot
 constexpr size_t kSmemP = kStabOff + (kScatKeys * kScatAtoms + 2 * kScatAtoms + 4 + kTN) * 4;
 static_assert(kSmemP <= 227 * 1024, "shared memory per block");
 
+// kFwd: the forward (B made from the moments by the split warps, pieces in order); else the backward
+// (B copied from its digit planes, units round-robin).  Two instantiations, each carrying only its own
+// code (measured: one kernel with both directions stalled on instruction fetch).
+template <bool kFwd>
 __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
   extern __shared__ __align__(1024) unsigned char smem[];
   uint64_t *full = reinterpret_cast<uint64_t *>(smem + kBarOff);
@@ -134,9 +170,9 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
   int *uflag = nsa + 2 * kScatAtoms;  // [0]: the unit writes T directly; [1]: its accumulators are ready
   int *fexp_s = uflag + 4;             // the unit's 48 column exponents
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nunits = *P.nunits;
+  const Walk wk = walk_of<kFwd>(P);
 
-  const bool fused = P.W != nullptr;  // B made in shared memory by the split warps
+  constexpr bool fused = kFwd;  // B made in shared memory by the split warps
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(full + s)), "r"(fused ? 2 : 1));
@@ -161,18 +197,19 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
   if (warp == 0) {
     // ---- producer: each slice's A and B blocks into the next stage of the ring
     int g = 0;  // slices loaded so far by this CTA
-    for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+    for (int u = wk.begin; u < wk.end; u += wk.step) {
       if (__shfl_sync(0xffffffffu, (int)*abortf, 0)) break;  // uniform over the warp
-      const Unit U = unit_of(P, u);
-      if (P.fwd)
-        for (int j = lane; j < U.nsl; j += 32) plist[j] = P.slist[(size_t)U.tile * P.ka + U.z * kMaxUnitSlices + j];
+      const Unit U = unit_of<kFwd>(P, u);
+      if (kFwd)
+        for (int j = lane; j < U.nsl; j += 32)
+          plist[j] = P.slist[((size_t)U.alpha * P.ntiles + U.tile) * P.ka + U.s0 + j];
       __syncwarp();
       if (lane == 0) {
         for (int j = 0; j < U.nsl; ++j, ++g) {
-          const int sl = P.fwd ? plist[j] : j;
+          const int sl = kFwd ? plist[j] : j;
           const int st = g % kStages;
           if (g >= kStages && !wait_or_abort(smem_u32(empty + st), (uint32_t)((g / kStages - 1) & 1), abortf)) break;
-          const unsigned char *asrc = P.aplanes + ((size_t)U.mt * P.ka + sl) * (kS * kPlaneA);
+          const unsigned char *asrc = P.aplanes + U.alpha * P.astride + ((size_t)U.mt * P.ka + sl) * (kS * kPlaneA);
           const unsigned char *bsrc = P.bplanes + ((size_t)U.tile * P.ka + sl) * (kS * kPlaneB);
           const uint32_t bar = smem_u32(full + st), dst = sbase + st * kStageBytes;
           const uint32_t bytes = fused ? kS * kPlaneA : kStageBytes;
@@ -198,8 +235,8 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
     if (lane == 0) {
       int g = 0, li = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x) {
-        const Unit U = unit_of(P, u);
+      for (int u = wk.begin; u < wk.end && ok; u += wk.step) {
+        const Unit U = unit_of<kFwd>(P, u);
         if (li > 0 && !(ok = wait_or_abort(smem_u32(tmem_free), (uint32_t)((li - 1) & 1), abortf))) break;
         asm volatile("tcgen05.fence::after_thread_sync;");
         for (int j = 0; j < U.nsl; ++j, ++g) {
@@ -250,11 +287,11 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
       static_assert(kTN * kTK / 2 == 32 * kPairs, "a pair per lane and atom");
       const int k = lane >> 3, kp = lane & 7;
       int g0 = 0;  // slices of this CTA before the unit
-      for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+      for (int u = wk.begin; u < wk.end; u += wk.step) {
         if (__shfl_sync(0xffffffffu, (int)*abortf, 0)) break;  // uniform over the warp
-        const Unit U = unit_of(P, u);
+        const Unit U = unit_of<kFwd>(P, u);
         const int64_t a_base = (int64_t)U.tile * kTileAtomsP;
-        const short *ulist = P.slist + (size_t)U.tile * P.ka + U.z * kMaxUnitSlices;
+        const short *ulist = P.slist + ((size_t)U.alpha * P.ntiles + U.tile) * P.ka + U.s0;
         int E[kPairs];
         bool av[kPairs];
 #pragma unroll
@@ -325,18 +362,18 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
     const int rl = 32 * q + lane;
     const uint32_t trow = tmem + ((uint32_t)(32 * q) << 16);
     int li = 0;
-    for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
-      const Unit U = unit_of(P, u);
+    for (int u = wk.begin; u < wk.end; u += wk.step) {
+      const Unit U = unit_of<kFwd>(P, u);
       const int64_t m0 = (int64_t)U.mt * kTM;
       const int n0 = (int)(U.tile * kTN);
       asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps));  // the previous unit's tables are free
       if (et < kTN) fexp_s[et] = P.Fexp[n0 + et];
-      if (P.fwd) {
+      if (kFwd) {
         if (et < kScatAtoms) {
           const int64_t a = (int64_t)(n0 / 4) + et;
-          nsa[et] = a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == P.alpha);
+          nsa[et] = a < P.natoms && (!P.atype || clampi(P.atype[P.atom0 + a], 0, P.ntypes - 1) == U.alpha);
         }
-        if (et == 0) uflag[0] = P.tout && P.scount[U.tile] <= kMaxUnitSlices;
+        if (et == 0) uflag[0] = P.tout && U.slot < 0;
       } else {
         for (int x = et; x < kScatKeys * kScatAtoms; x += 32 * kEpiWarps) stab[x] = -1;
         if (et < kScatAtoms) {
@@ -357,12 +394,12 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
       asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarps));  // the tables are built and the MMAs done
       const bool ok = uflag[1] != 0;
       asm volatile("tcgen05.fence::after_thread_sync;");
-      const bool direct = P.fwd && uflag[0];
-      const int Erow = (direct && m0 + rl < P.ldt) || (!P.fwd && m0 + rl < P.Mp) ? P.Eexp[m0 + rl] : 0;
-      const int key = P.fwd ? 0 : (int)((m0 + rl) / P.kq), qq = P.fwd ? 0 : (int)(m0 + rl - (int64_t)key * P.kq);
-      const int key_l = P.fwd ? 0 : key - (int)(m0 / P.kq);
-      const bool row_wanted = !P.fwd && qq < 6 && key < P.nkeys;
-      float4 *outp = P.fwd && !direct ? P.part + ((size_t)U.z * P.Mp + m0 + rl) * P.Np + n0 : nullptr;
+      const bool direct = kFwd && uflag[0];
+      const int Erow = (direct && m0 + rl < P.ldt) || (!kFwd && m0 + rl < P.Mp) ? P.Eexp[U.alpha * P.estride + m0 + rl] : 0;
+      const int key = kFwd ? 0 : (int)((m0 + rl) / P.kq), qq = kFwd ? 0 : (int)(m0 + rl - (int64_t)key * P.kq);
+      const int key_l = kFwd ? 0 : key - (int)(m0 / P.kq);
+      const bool row_wanted = !kFwd && qq < 6 && key < P.nkeys;
+      longlong2 *outp = kFwd && !direct ? P.part + (size_t)U.slot * kTN * P.Mp + m0 + rl : nullptr;
       // the warp's 24 columns of accumulators, four (one atom) at a time: each output's nine diagonals
       // recombined exactly as an integer and rounded once to f64 (diag_to_f64: integer operations, no
       // branch, the four outputs interleaved), or kept as four floats for a tile with several shares.
@@ -382,10 +419,14 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
           for (int d = 0; d < kS; ++d) asm volatile("" : "+f"(v[d][0]), "+f"(v[d][1]), "+f"(v[d][2]), "+f"(v[d][3]));
         }
         const int al = (c_lo + c0) >> 2;  // the group's atom; column c0 + k is its component k
-        if (outp) {
+        if (outp) {  // a piece of a cut item: its outputs' exact integers, summed by fwd_epilogue_kernel
 #pragma unroll
-          for (int k = 0; k < 4; ++k)
-            outp[c_lo + c0 + k] = ok ? diag_combine4(v, k) : make_float4(__int_as_float(0x7fc00000), 0.f, 0.f, 0.f);
+          for (int k = 0; k < 4; ++k) {
+            long long hi;
+            unsigned long long lo;
+            diag_s128(v, k, hi, lo);
+            outp[(size_t)(c_lo + c0 + k) * P.Mp] = ok ? make_longlong2((long long)lo, hi) : make_longlong2(0, kPartNaN);
+          }
           continue;
         }
         // only the wanted outputs are stored; a warp skips a group none of its rows wants
@@ -406,7 +447,9 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
         for (int k = 0; k < 4; ++k) val[k] = diag_to_f64(v, k, Erow, F[k], rare);
         if (__any_sync(0xffffffffu, rare))  // warp-uniform, and never taken with these operands
 #pragma unroll
-          for (int k = 0; k < 4; ++k) val[k] = output_value(diag_int(v, k), Erow, F[k]);
+          for (int k = 0; k < 4; ++k)
+            val[k] = output_value_rare(v[0][k], v[1][k], v[2][k], v[3][k], v[4][k], v[5][k], v[6][k], v[7][k], v[8][k],
+                                       Erow, F[k], false);
         if (at >= 0) {
           double *dst = (direct ? P.tout : P.scat) + at;
 #pragma unroll
@@ -427,21 +470,29 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
   if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols));
 }
 
+// The kernels' shared-memory size, set once per device (bit d of set_on: done on device d).
 int set_smem(const char *who) {
-  static std::atomic<bool> done{false};
-  if (done.load(std::memory_order_acquire)) return DP_OK;
-  const cudaError_t e = cudaFuncSetAttribute(tgemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemP);
-  if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
-  done.store(true, std::memory_order_release);
+  static std::atomic<unsigned long long> set_on{0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(cudaGetLastError()));
+  if (dev < 64 && (set_on.load(std::memory_order_acquire) >> dev & 1ull)) return DP_OK;
+  for (const void *k : {(const void *)tgemm_kernel<true>, (const void *)tgemm_kernel<false>}) {
+    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemP);
+    if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+  }
+  if (dev < 64) set_on.fetch_or(1ull << dev, std::memory_order_acq_rel);
   return DP_OK;
 }
 
-// One launch over the units of P's list: one CTA per SM.
-int launch(const Params &P, cudaStream_t st, const char *who) {
+// One launch: grid CTAs (forward: the schedule's CTA count), or one per SM (backward, grid 0).
+int launch(const Params &P, cudaStream_t st, const char *who, int grid = 0) {
   int dev = 0, nsm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(cudaGetLastError()));
-  tgemm_kernel<<<(unsigned)std::max(nsm, 1), kThreadsP, kSmemP, st>>>(P);
+  if (P.fwd)
+    tgemm_kernel<true><<<(unsigned)std::max(grid > 0 ? grid : nsm, 1), kThreadsP, kSmemP, st>>>(P);
+  else
+    tgemm_kernel<false><<<(unsigned)std::max(grid > 0 ? grid : nsm, 1), kThreadsP, kSmemP, st>>>(P);
   return launch_status(who);
 }
 

@@ -239,7 +239,9 @@ __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
         for (int k = 0; k < 4; ++k) val[k] = diag7_to_f64(v, k, Erow, F[k], rare);
         if (__any_sync(0xffffffffu, rare))  // warp-uniform, and never taken with these operands
 #pragma unroll
-          for (int k = 0; k < 4; ++k) val[k] = output_value7(diag7_int(v, k), Erow, F[k]);
+          for (int k = 0; k < 4; ++k)
+            val[k] = output_value_rare(v[0][k], v[1][k], v[2][k], v[3][k], v[4][k], v[5][k], v[6][k], 0.f, 0.f, Erow,
+                                       F[k], true);
         if (at >= 0)
 #pragma unroll
           for (int k = 0; k < 4; ++k) P.scat[at + 6 * k] = ok ? val[k] : __longlong_as_double(0x7ff8000000000000ll);

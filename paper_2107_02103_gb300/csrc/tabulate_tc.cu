@@ -56,11 +56,14 @@ using namespace tc;
 constexpr int kQ = 6;                 // K entries per interval: u^0 .. u^5
 constexpr int kCols = 4;              // GEMM columns per atom: k = 0 .. 3
 constexpr int kTileAtoms = kTN / kCols;  // 12 atoms per 48-column tile
-constexpr int64_t kChunkAtoms = 4104;    // a multiple of 12 (16,416 columns)
+constexpr int64_t kChunkAtoms = 16416;   // a multiple of 24 (12- and 8-atom tiles; 65,664 columns)
 constexpr int kShareSlices = kMaxShareSlices;  // used K slices per forward share (112, the exactness bound)
-constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of forward shares' results per chunk
+constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of the forward's partial results per chunk at most
+constexpr int kMaxCtasF = 160;  // CTAs of the forward GEMM at most (its part slots are sized for them)
+constexpr int kEpiCost = 6;     // a forward unit's epilogue, in slices' time, for the forward schedule
+constexpr int kEpiBlocks = 8;   // fwd_epilogue_kernel's blocks per (type, tile)
 constexpr int kMaxKeys = 4096;  // ntypes x nint: each warp's key map (int16) lives in shared memory
-static_assert(kChunkAtoms % kTileAtoms == 0, "whole tiles per chunk");
+static_assert(kChunkAtoms % kTileAtoms == 0 && kChunkAtoms % 8 == 0, "whole tiles per chunk");
 
 // Sizes shared by the kernels, the plan and the work-buffer layout.
 struct Shape {
@@ -73,7 +76,9 @@ struct Shape {
   int64_t nloc, tiles_all;    // atoms of the call and their 12-atom tiles
   int64_t chunk, Np, ntiles;  // atoms per chunk, its columns round_up(4 chunk, 48), Np / 48
   int zmax;                   // forward shares per tile at most
-  int64_t maxunits;           // GEMM units per chunk and centre type at most
+  int64_t maxunits;           // backward GEMM units (9 x 6 digits) per chunk and centre type at most
+  int64_t nitems;             // forward items per chunk: (type, 12-atom tile, 128-row tile of A)
+  int64_t maxpieces, maxslots;  // forward pieces and part slots per chunk at most
   bool b8;                    // the backward GEMM uses the 7 x 8-bit digits on 8-atom tiles (Kpm <= 144)
   int64_t Np8, ntiles8;       // its columns round_up(4 chunk, 32) and tiles Np8 / 32
   int64_t maxunits8;          // its units per chunk and centre type at most
@@ -87,7 +92,8 @@ struct PlanLayout {
 // The work buffer: the slot keys, their counts and the slice flags of every atom of the call
 // (kept from the forward for the backward), then one chunk's scratch.
 struct Layout {
-  size_t keys, nslots, occ, map, slist, scount, units, nunits, fexp, bplanes, w, part, total;
+  size_t keys, nslots, occ, map, slist, scount, units, nunits, pieces, pcta, cta_start, npieces, pfirst, fexp, bplanes,
+      w, part, total;
 };
 
 size_t take(size_t &off, size_t bytes) {
@@ -118,13 +124,20 @@ Shape make_shape(const TableGeom &g, int64_t nloc, int nnei, int ntypes, int M1)
   s.nloc = nloc;
   s.tiles_all = (nloc + kTileAtoms - 1) / kTileAtoms;
   int64_t chunk = std::min<int64_t>(round_up(std::max<int64_t>(nloc, 1), kTileAtoms), kChunkAtoms);
-  while (chunk > kTileAtoms &&
-         (size_t)s.zmax * s.Mpf * round_up(kCols * chunk, kTN) * sizeof(float4) > kPartBudget)
+  // part slots: two per CTA boundary, and every piece of an item whose used slices exceed one share
+  auto slots_for = [&](int64_t c) {
+    const int64_t items = (int64_t)s.ntypes * (round_up(kCols * c, kTN) / kTN) * (s.Mpf / kTM);
+    return 2 * kMaxCtasF + (s.zmax > 1 ? items * s.zmax : 0);
+  };
+  while (chunk > kTileAtoms && (size_t)slots_for(chunk) * s.Mpf * kTN * sizeof(float4) > kPartBudget)
     chunk = round_up(chunk / 2, kTileAtoms);
   s.chunk = chunk;
   s.Np = round_up(kCols * chunk, kTN);
   s.ntiles = s.Np / kTN;
-  s.maxunits = s.ntiles * std::max<int64_t>((int64_t)(s.Mpf / kTM) * s.zmax, s.Mpb / kTM);
+  s.maxunits = s.ntiles * (s.Mpb / kTM);
+  s.nitems = (int64_t)s.ntypes * s.ntiles * (s.Mpf / kTM);
+  s.maxpieces = s.nitems * s.zmax + kMaxCtasF;
+  s.maxslots = slots_for(chunk);
   s.Np8 = round_up(kCols * chunk, tb::kTNB);
   s.ntiles8 = s.Np8 / tb::kTNB;
   s.maxunits8 = s.ntiles8 * (s.Mpb / kTM);
@@ -156,11 +169,16 @@ Layout make_layout(const Shape &s) {
   L.scount = take(off, (size_t)s.ntypes * s.ntiles * sizeof(int));
   L.units = take(off, (size_t)s.ntypes * std::max(s.maxunits, s.maxunits8) * sizeof(int));
   L.nunits = take(off, (size_t)s.ntypes * sizeof(int));
+  L.pieces = take(off, (size_t)s.maxpieces * sizeof(int4));
+  L.pcta = take(off, (size_t)s.maxpieces * sizeof(int));
+  L.cta_start = take(off, (size_t)(kMaxCtasF + 1) * sizeof(int));
+  L.npieces = take(off, (size_t)s.nitems * sizeof(int));
+  L.pfirst = take(off, (size_t)s.nitems * sizeof(int));
   L.fexp = take(off, (size_t)std::max(s.Np, s.Np8) * sizeof(int));
   L.bplanes = take(off, s.b8 ? (size_t)s.ntiles8 * (s.Kpm / kTK) * tb::kSB * tb::kPlaneBB  // the backward's dT planes
                              : (size_t)s.ntiles * (s.Kpm / kTK) * kS * kPlaneB);
   L.w = take(off, (size_t)s.chunk * s.cap * 24 * sizeof(double));  // moments (forward) or their gradients
-  L.part = take(off, (size_t)s.zmax * s.Mpf * s.Np * sizeof(float4));
+  L.part = take(off, (size_t)s.maxslots * s.Mpf * kTN * sizeof(longlong2));
   L.total = off;
   return L;
 }
@@ -407,13 +425,10 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
 }
 
 // The used K slices of each tile of the chunk, in order, and their count, per centre type (one warp per
-// (type, tile)), and the forward GEMM's units (tile, 128-row tile of A, share of 28 slices) of the tiles
-// with used slices, appended to the type's unit list.
+// (type, tile)).
 __global__ void __launch_bounds__(128) slice_list_kernel(const unsigned char *__restrict__ occ, int64_t tiles_all,
-                                                         int64_t tile0, int64_t ntiles, int ntypes, int nsl, int nmt,
-                                                         int64_t maxunits, short *__restrict__ list,
-                                                         int *__restrict__ count, int *__restrict__ units,
-                                                         int *__restrict__ nunits) {
+                                                         int64_t tile0, int64_t ntiles, int ntypes, int nsl,
+                                                         short *__restrict__ list, int *__restrict__ count) {
   const int lane = threadIdx.x & 31;
   const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
   if (w >= (int64_t)ntypes * ntiles) return;  // warp-uniform
@@ -428,14 +443,107 @@ __global__ void __launch_bounds__(128) slice_list_kernel(const unsigned char *__
     if (used) out[rank + __popc(m & ((1u << lane) - 1u))] = (short)(b + lane);
     rank += __popc(m);
   }
-  const int nz = (rank + kShareSlices - 1) / kShareSlices;
-  if (lane == 0) {
-    count[(size_t)t * ntiles + tile] = rank;
-    if (nz > 0) {
-      int at = atomicAdd(nunits + t, nz * nmt);
-      for (int z = 0; z < nz; ++z)
-        for (int mt = 0; mt < nmt; ++mt) units[(size_t)t * maxunits + at++] = tg::unit_code((int)tile, mt, z);
+  if (lane == 0) count[(size_t)t * ntiles + tile] = rank;
+}
+
+// Exclusive prefix sum over a block of 1024 threads of one value per thread; the block's total in *total.
+__device__ long long block_scan_1024(long long v, long long *red, long long *total) {
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  long long x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) red[wid] = x;
+  __syncthreads();
+  if (wid == 0) {
+    long long z = red[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(0xffffffffu, z, o);
+      if (lane >= o) z += y;
     }
+    red[lane] = z;  // inclusive over the warps
+  }
+  __syncthreads();
+  const long long before = (wid ? red[wid - 1] : 0ll) + x - v;
+  *total = red[31];
+  __syncthreads();  // red is reused by the next scan
+  return before;
+}
+
+// The forward GEMM's schedule over one chunk: every item (type, tile, 128-row tile of A) with used slices
+// costs its slice count plus kEpiCost; CTA b takes the cost range [b R, (b + 1) R) of the items' running
+// sum, R = ceil(total / ncta), so that every CTA gets the same work.  An item is cut where a CTA's range
+// begins and every 112 slices (the exactness bound of a share); the pieces of a cut item write their
+// partial results to consecutive part slots, which fwd_epilogue_kernel sums.  One block of 1024 threads,
+// each over a run of consecutive items.
+__global__ void __launch_bounds__(1024) fwd_schedule_kernel(const int *__restrict__ scount, int64_t nitems,
+                                                            int64_t ntiles, int nmt, int ncta, int4 *__restrict__ pieces,
+                                                            int *__restrict__ pcta, int *__restrict__ cta_start,
+                                                            int *__restrict__ npieces, int *__restrict__ pfirst) {
+  __shared__ long long red[32];
+  __shared__ long long s_R;
+  const int64_t per = (nitems + 1023) / 1024;
+  const int64_t i0 = min(nitems, (int64_t)threadIdx.x * per), i1 = min(nitems, i0 + per);
+  auto ns_of = [&](int64_t it) { return scount[it / nmt]; };  // item (t ntiles + tile) nmt + mt
+  long long c = 0;
+  for (int64_t it = i0; it < i1; ++it) {
+    const int ns = ns_of(it);
+    c += ns > 0 ? ns + kEpiCost : 0;
+  }
+  long long total;
+  const long long P0 = block_scan_1024(c, red, &total);
+  if (threadIdx.x == 0) s_R = max(1ll, (total + ncta - 1) / ncta);
+  __syncthreads();
+  const long long R = s_R;
+  // the pieces of an item: cut where P + x reaches a multiple of R and where x reaches a multiple of 112
+  auto for_pieces = [&](long long P, int ns, auto &&f) {
+    for (int x = 0; x < ns;) {
+      const long long nr = ((P + x) / R + 1) * R - P;
+      const int e = (int)min((long long)ns, min(nr, (long long)((x / kShareSlices + 1) * kShareSlices)));
+      f(x, e - x, (int)min((P + x) / R, (long long)ncta - 1));
+      x = e;
+    }
+  };
+  long long np = 0, nslot = 0, P = P0;
+  for (int64_t it = i0; it < i1; ++it) {
+    const int ns = ns_of(it);
+    int n = 0;
+    for_pieces(P, ns, [&](int, int, int) { ++n; });
+    np += n;
+    nslot += n > 1 ? n : 0;
+    P += ns > 0 ? ns + kEpiCost : 0;
+  }
+  long long np_total, nslot_total;
+  long long pbase = block_scan_1024(np, red, &np_total);
+  long long sbase = block_scan_1024(nslot, red, &nslot_total);
+  P = P0;
+  for (int64_t it = i0; it < i1; ++it) {
+    const int ns = ns_of(it);
+    int n = 0;
+    for_pieces(P, ns, [&](int, int, int) { ++n; });
+    npieces[it] = n;
+    pfirst[it] = n > 1 ? (int)sbase : -1;
+    const int64_t tt = it / nmt;
+    const int mt = (int)(it - tt * nmt), t = (int)(tt / ntiles), tile = (int)(tt - (int64_t)t * ntiles);
+    for_pieces(P, ns, [&](int x, int len, int cta) {
+      // tile, (type | mt << 4 | slices << 8), first slice in the tile's list, part slot
+      pieces[pbase] = make_int4(tile, t | mt << 4 | len << 8, x, n > 1 ? (int)sbase++ : -1);
+      pcta[pbase++] = cta;
+    });
+    P += ns > 0 ? ns + kEpiCost : 0;
+  }
+  __syncthreads();
+  // CTA b's pieces start at the first piece of a CTA >= b (pieces come in CTA order)
+  for (long long i = threadIdx.x; i < np_total; i += blockDim.x) {
+    const int cb = pcta[i], ca = i > 0 ? pcta[i - 1] : -1;
+    for (int b = ca + 1; b <= cb; ++b) cta_start[b] = (int)i;
+  }
+  if (threadIdx.x == 0) {
+    const int last = np_total > 0 ? pcta[np_total - 1] : -1;
+    for (int b = last + 1; b <= ncta; ++b) cta_start[b] = (int)np_total;
   }
 }
 
@@ -503,52 +611,56 @@ __global__ void __launch_bounds__(128) bwd_units8_kernel(const short *__restrict
     units[(size_t)t * maxunits8 + base++] = tb::unit_code((int)tile, 32 * lane + __ffs((int)m) - 1);
 }
 
-// T for the atoms of type alpha of one 12-atom tile (one block) whose used slices take several shares
-// (one per kShareSlices; a single share's GEMM writes T itself) or none (T = 0): the shares summed in
-// a three-float sum and scaled by 2^(E_m + F_(a,k)) (1/N_c is in C'), 32 channels at a time: read with
-// the columns fastest (the shares' rows), written with the channels fastest (T's).
-__global__ void __launch_bounds__(256) fwd_epilogue_kernel(const float4 *__restrict__ part, int Mp, int64_t Np,
+// T for the atoms of type t of one 12-atom tile whose items were cut into several pieces, or have no
+// used slices (T = 0): each output's pieces' exact integers added as 128-bit integers and rounded once to
+// f64 (s128_to_f64: no FP64 instruction), read and written with the channels fastest.  kEpiBlocks blocks
+// per (type, tile), each over a share of its 48 columns; a tile whose items each came in one piece was
+// written by the GEMM.
+__global__ void __launch_bounds__(128) fwd_epilogue_kernel(const longlong2 *__restrict__ part, int Mp,
                                                            const int *__restrict__ eexp,
                                                            const int *__restrict__ fexp,
-                                                           const unsigned char *__restrict__ occ, int nsl,
+                                                           const int *__restrict__ npieces,
+                                                           const int *__restrict__ pfirst, int64_t ntiles, int nmt,
                                                            int64_t natoms, int64_t atom0,
-                                                           const int32_t *__restrict__ atype, int ntypes, int alpha,
-                                                           int M1, double *__restrict__ T) {
-  __shared__ int nused;
-  __shared__ double tile_out[kTN][33];
+                                                           const int32_t *__restrict__ atype, int ntypes, int M1,
+                                                           double *__restrict__ T) {
   __shared__ bool wanted[kTileAtoms];
-  const int64_t tile = blockIdx.x;
-  if (threadIdx.x == 0) nused = 0;
+  const int64_t tt = blockIdx.x / kEpiBlocks;
+  const int part_of = (int)(blockIdx.x - tt * kEpiBlocks);
+  const int t = (int)(tt / ntiles);
+  const int64_t tile = tt - (int64_t)t * ntiles;
+  const int64_t item0 = tt * nmt;
+  bool direct = true;
+  for (int mt = 0; mt < nmt; ++mt) direct = direct && npieces[item0 + mt] == 1;
+  if (direct) return;  // uniform
   if (threadIdx.x < kTileAtoms) {
     const int64_t a = tile * kTileAtoms + threadIdx.x;
-    wanted[threadIdx.x] = a < natoms && (!atype || clampi(atype[atom0 + a], 0, ntypes - 1) == alpha);
+    wanted[threadIdx.x] = a < natoms && (!atype || clampi(atype[atom0 + a], 0, ntypes - 1) == t);
   }
   __syncthreads();
-  int c = 0;
-  for (int x = threadIdx.x; x < nsl; x += blockDim.x) c += occ[tile * nsl + x] != 0;
-  if (c) atomicAdd(&nused, c);
-  __syncthreads();
-  const int nz = (nused + kShareSlices - 1) / kShareSlices;
-  if (nz == 1) return;  // uniform: the GEMM wrote this tile's T itself
-  for (int m0 = 0; m0 < M1; m0 += 32) {
-    for (int e = threadIdx.x; e < kTN * 32; e += blockDim.x) {
-      const int col = e % kTN, m = m0 + e / kTN;
-      const int64_t n = tile * kTN + col;
-      double v = 0.0;  // an atom of a tile without used slices has no valid rows
-      if (m < M1 && wanted[col >> 2] && nz > 0) {
-        Sum3 acc;
-        for (int z = 0; z < nz; ++z) acc.add(part[((size_t)z * Mp + m) * Np + n]);
-        v = acc.value(eexp[m], fexp[n]);
-      }
-      tile_out[col][e / kTN] = v;
+  constexpr int kColsPer = kTN / kEpiBlocks;
+  static_assert(kTN % kEpiBlocks == 0, "whole columns per block");
+  for (int e = threadIdx.x; e < kColsPer * M1; e += blockDim.x) {
+    const int col = part_of * kColsPer + e / M1, m = e - (e / M1) * M1;
+    if (!wanted[col >> 2]) continue;
+    const int np = npieces[item0 + m / kTM], first = pfirst[item0 + m / kTM];
+    if (np == 1) continue;  // these channels were written by the GEMM
+    long long hi = 0;
+    unsigned long long lo = 0;
+    bool nan = false;
+    for (int z = 0; z < np; ++z) {  // an atom of a tile without used slices has no valid rows: T = 0
+      const longlong2 x = part[((size_t)(first + z) * kTN + col) * Mp + m];
+      const unsigned long long l = lo + (unsigned long long)x.x;
+      hi += x.y + (l < lo ? 1 : 0);
+      lo = l;
+      nan = nan || x.y == tg::kPartNaN;
     }
-    __syncthreads();
-    for (int e = threadIdx.x; e < kTN * 32; e += blockDim.x) {
-      const int col = e >> 5, m = m0 + (e & 31);
-      const int64_t a = tile * kTileAtoms + (col >> 2);
-      if (m < M1 && wanted[col >> 2]) T[((atom0 + a) * kCols + (col & 3)) * M1 + m] = tile_out[col][e & 31];
-    }
-    __syncthreads();
+    bool rare = false;
+    const int E = eexp[(size_t)t * Mp + m], F = fexp[tile * kTN + col];
+    double v = s128_to_f64<kOutExp>(hi, lo, E, F, rare);
+    if (rare) v = output_value((__int128)(((unsigned __int128)(unsigned long long)hi << 64) | lo), E, F);
+    const int64_t a = tile * kTileAtoms + (col >> 2);
+    T[((atom0 + a) * kCols + (col & 3)) * M1 + m] = nan ? __longlong_as_double(0x7ff8000000000000ll) : v;
   }
 }
 
@@ -808,7 +920,11 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei,
                              reinterpret_cast<const double *>(pk + PL.nodes));
   R.W = reinterpret_cast<double *>(wk + L.w);
-  float4 *part = reinterpret_cast<float4 *>(wk + L.part);
+  longlong2 *part = reinterpret_cast<longlong2 *>(wk + L.part);
+  int dev = 0, nsm = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(cudaGetLastError()));
+  const int ncta = std::max(1, std::min(nsm, kMaxCtasF));
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
     const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
     const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN, tile0 = c0 / kTileAtoms;
@@ -819,50 +935,54 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_runs_moments", st);
     const int64_t nlist = (int64_t)ntypes * ntiles;
-    if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
-      return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
-    slice_list_kernel<<<(unsigned)((nlist + 3) / 4), 128, 0, st>>>(
-        wk + L.occ, S.tiles_all, tile0, ntiles, ntypes, S.nsl, S.Mpf / kTM, S.maxunits,
-        reinterpret_cast<short *>(wk + L.slist), reinterpret_cast<int *>(wk + L.scount),
-        reinterpret_cast<int *>(wk + L.units), reinterpret_cast<int *>(wk + L.nunits));
+    slice_list_kernel<<<(unsigned)((nlist + 3) / 4), 128, 0, st>>>(wk + L.occ, S.tiles_all, tile0, ntiles, ntypes,
+                                                                    S.nsl, reinterpret_cast<short *>(wk + L.slist),
+                                                                    reinterpret_cast<int *>(wk + L.scount));
+    if ((rc = launch_status(who))) return rc;
+    const int nmt = S.Mpf / kTM;
+    fwd_schedule_kernel<<<1, 1024, 0, st>>>(reinterpret_cast<const int *>(wk + L.scount), nlist * nmt, ntiles, nmt, ncta,
+                                            reinterpret_cast<int4 *>(wk + L.pieces), reinterpret_cast<int *>(wk + L.pcta),
+                                            reinterpret_cast<int *>(wk + L.cta_start),
+                                            reinterpret_cast<int *>(wk + L.npieces),
+                                            reinterpret_cast<int *>(wk + L.pfirst));
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_slice_lists", st);
-    for (int t = 0; t < ntypes; ++t) {
-      tg::Params G{};
-      G.fwd = true;
-      G.aplanes = pk + PL.afwd + (size_t)t * kS * S.Mpf * S.Kp * 2;
-      G.Eexp = reinterpret_cast<const int *>(pk + PL.efwd) + (size_t)t * S.Mpf;
-      G.ka = S.nsl;
-      G.nmt = S.Mpf / kTM;
-      G.W = R.W;  // B made from the moments inside the GEMM
-      G.map = R.map;
-      G.nkeys = S.nkeys;
-      G.cap = S.cap;
-      G.Fexp = R.fexp;
-      G.ntiles = ntiles;
-      G.Np = Np;
-      G.Mp = S.Mpf;
-      G.slist = reinterpret_cast<const short *>(wk + L.slist) + (size_t)t * ntiles * S.nsl;
-      G.scount = reinterpret_cast<const int *>(wk + L.scount) + (size_t)t * ntiles;
-      G.zmax = S.zmax;
-      G.part = part;
-      G.tout = T;  // tiles with one share write T themselves
-      G.units = reinterpret_cast<const int *>(wk + L.units) + (size_t)t * S.maxunits;
-      G.nunits = reinterpret_cast<const int *>(wk + L.nunits) + t;
-      G.ldt = M1;
-      G.atype = atype;
-      G.natoms = n;
-      G.atom0 = c0;
-      G.alpha = t;
-      G.ntypes = ntypes;
-      if ((rc = tg::launch(G, st, who))) return rc;
-      prof_mark("tc_gemm_fwd", st);
-      const unsigned char *kocc = wk + L.occ + ((size_t)t * S.tiles_all + tile0) * S.nsl;
-      fwd_epilogue_kernel<<<(unsigned)ntiles, 256, 0, st>>>(part, S.Mpf, Np, G.Eexp, R.fexp, kocc, S.nsl, n, c0,
-                                                            atype, ntypes, t, M1, T);
-      if ((rc = launch_status(who))) return rc;
-      prof_mark("tc_epilogue_fwd", st);
-    }
+    tg::Params G{};
+    G.fwd = true;
+    G.aplanes = pk + PL.afwd;
+    G.astride = (size_t)kS * S.Mpf * S.Kp * 2;
+    G.Eexp = reinterpret_cast<const int *>(pk + PL.efwd);
+    G.estride = S.Mpf;
+    G.ka = S.nsl;
+    G.nmt = nmt;
+    G.W = R.W;  // B made from the moments inside the GEMM
+    G.map = R.map;
+    G.nkeys = S.nkeys;
+    G.cap = S.cap;
+    G.Fexp = R.fexp;
+    G.ntiles = ntiles;
+    G.Np = Np;
+    G.Mp = S.Mpf;
+    G.slist = reinterpret_cast<const short *>(wk + L.slist);
+    G.scount = reinterpret_cast<const int *>(wk + L.scount);
+    G.zmax = S.zmax;
+    G.part = part;
+    G.tout = T;  // items in one piece write T themselves
+    G.pieces = reinterpret_cast<const int4 *>(wk + L.pieces);
+    G.cta_start = reinterpret_cast<const int *>(wk + L.cta_start);
+    G.ldt = M1;
+    G.atype = atype;
+    G.natoms = n;
+    G.atom0 = c0;
+    G.ntypes = ntypes;
+    if ((rc = tg::launch(G, st, who, ncta))) return rc;
+    prof_mark("tc_gemm_fwd", st);
+    fwd_epilogue_kernel<<<(unsigned)(nlist * kEpiBlocks), 128, 0, st>>>(part, S.Mpf, G.Eexp, R.fexp,
+                                                         reinterpret_cast<const int *>(wk + L.npieces),
+                                                         reinterpret_cast<const int *>(wk + L.pfirst), ntiles, nmt, n, c0,
+                                                         atype, ntypes, M1, T);
+    if ((rc = launch_status(who))) return rc;
+    prof_mark("tc_epilogue_fwd", st);
   }
   return DP_OK;
 }

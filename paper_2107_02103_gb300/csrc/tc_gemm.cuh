@@ -448,7 +448,7 @@ __device__ __forceinline__ double s128_to_f64(long long hi, unsigned long long l
 // sits between their independent instruction chains (measured: a call site inside each conversion made
 // it 3.5 times slower).
 template <int W>
-__device__ __forceinline__ double diag_to_f64(const float (&v)[kS][W], int c, int E, int F, bool &rare) {
+__device__ __forceinline__ void diag_s128(const float (&v)[kS][W], int c, long long &hi, unsigned long long &lo) {
   static_assert(kS == 9 && kBits == 6, "three groups of three 6-bit diagonals");
   int x[kS];
 #pragma unroll
@@ -458,8 +458,14 @@ __device__ __forceinline__ double diag_to_f64(const float (&v)[kS][W], int c, in
   const long long L = (long long)x[6] * 4096 + (long long)x[7] * 64 + x[8];
   const long long A = M * 262144 + L;  // |A| < 2^55
   const unsigned long long tl = (unsigned long long)T << 36;
-  const unsigned long long lo = tl + (unsigned long long)A;
-  const long long hi = (T >> 28) + (A >> 63) + (lo < tl ? 1 : 0);
+  lo = tl + (unsigned long long)A;
+  hi = (T >> 28) + (A >> 63) + (lo < tl ? 1 : 0);
+}
+template <int W>
+__device__ __forceinline__ double diag_to_f64(const float (&v)[kS][W], int c, int E, int F, bool &rare) {
+  long long hi;
+  unsigned long long lo;
+  diag_s128(v, c, hi, lo);
   return s128_to_f64<kOutExp>(hi, lo, E, F, rare);
 }
 
@@ -489,6 +495,19 @@ __device__ __forceinline__ double diag7_to_f64(const float (&v)[7][W], int c, in
 __device__ __forceinline__ double output_value7(__int128 S, int E, int F) {
   if (E >= kNonFinite || F >= kNonFinite) return __longlong_as_double(0x7ff8000000000000ll);
   return i128_to_double(S, E + F + kOutExp7x8);
+}
+
+// The rare case of diag_to_f64 / diag7_to_f64 (a result outside the normal range), out of line so that
+// the epilogue loops stay small: one output from its diagonal sums (the seventh to ninth unused by the
+// 7 x 8 scheme).
+__device__ __noinline__ double output_value_rare(float v0, float v1, float v2, float v3, float v4, float v5, float v6,
+                                                 float v7, float v8, int E, int F, bool seven) {
+  if (seven) {
+    const float v[7][1] = {{v0}, {v1}, {v2}, {v3}, {v4}, {v5}, {v6}};
+    return output_value7(diag7_int(v, 0), E, F);
+  }
+  const float v[kS][1] = {{v0}, {v1}, {v2}, {v3}, {v4}, {v5}, {v6}, {v7}, {v8}};
+  return output_value(diag_int(v, 0), E, F);
 }
 
 __global__ void __launch_bounds__(kThreads, 1) gemm_kernel(const TcGemm P) {

@@ -59,7 +59,7 @@ CASES = [
     ("cugeo", {}, 512), ("alcumg", dict(pad=0.1), 384), ("alcumg", dict(pad=0.3), 384),
     ("alcumg", dict(pad=0.6), 384),
 ]
-CHUNK = 4104  # atoms per chunk of the tensor-core calls (their work buffer holds one chunk)
+CHUNK = 16416  # atoms per chunk of the tensor-core calls (their work buffer holds one chunk)
 
 
 @pytest.mark.parametrize("name,kw,nsample", CASES, ids=[f"{c[0]}-{c[1]}" for c in CASES])
@@ -190,10 +190,10 @@ def test_tc_empty_counts_and_overwrite():
 
 
 def test_tc_chunks_of_atoms():
-    """More atoms than one chunk (4,104), with a ragged last chunk, against the FP64-pipe path, and the
+    """More atoms than one chunk (16,416), with a ragged last chunk, against the FP64-pipe path, and the
     oracle on atoms at the chunk edges; the backward reusing the forward's runs of every chunk gives the
     same bits as one that finds them itself."""
-    w = workload("water", nmol=1500)  # 4,500 atoms
+    w = workload("water", nmol=6000)  # 18,000 atoms
     model = product_model(w, F64)
     x = to_dev(w, F64)
     got = _tc(w, model, x, reuse=True)

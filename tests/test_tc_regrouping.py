@@ -102,19 +102,19 @@ def test_regrouping_slips_are_caught(mistake):
 def test_tc_work_and_plan_size_queries():
     """dp_tabulate_tc_work_bytes and dp_tabulate_tc_plan_bytes on the host: one work size for both
     directions, 256-byte multiples; the work grows with the atoms by the chunk's scratch until the
-    chunk (4,104 atoms) caps it, and past that only by what every atom keeps (its int16 slot keys,
+    chunk (16,416 atoms) caps it, and past that only by what every atom keeps (its int16 slot keys,
     their count and its tile's slice flags); the plan does not depend on the atoms; refusals for bad
     sizes and for more intervals per centre type than the shared-memory key map holds."""
     import __graft_entry__
     __graft_entry__._load_builder().build()
     import paper_2107_02103_gb300 as dpc
     info = dpc.dp_table_info_make(0.0, 0.5, 0.01, 0.1, 5.0)   # 50 fine + 20 coarse intervals
-    sizes = [dpc.dp_tabulate_tc_work_bytes(info, n, 512, 1, 100) for n in (1, 100, 4104, 20000)]
+    sizes = [dpc.dp_tabulate_tc_work_bytes(info, n, 512, 1, 100) for n in (1, 100, 16416, 40000)]
     assert all(b > 0 and b % 256 == 0 for b in sizes)
     assert sizes[0] <= sizes[1] <= sizes[2] < sizes[3]
     cap, nsl = 70, -(-6 * 70 // 16)                            # slots per atom, K slices
     per_atom = 2 * cap + 4 + nsl / 12                          # keys, count, flags of its tile
-    assert abs(sizes[3] - sizes[2] - (20000 - 4104) * per_atom) <= 4 * 256
+    assert abs(sizes[3] - sizes[2] - (40000 - 16416) * per_atom) <= 4 * 256
     assert dpc.dp_tabulate_tc_work_bytes(info, 100, 512, 3, 100) > sizes[1]   # K grows with the types
     for bad in ((info, -1, 512, 1, 100), (info, 10, 0, 1, 100), (info, 10, 512, 9, 100), (info, 10, 512, 1, 0)):
         with pytest.raises(ValueError):
