@@ -320,7 +320,7 @@ __device__ __forceinline__ int valid_row(int v, const int *nvb, const int *sel, 
 // the atom's four column exponents (over every value written, which bounds the final ones).
 // Warps (one atom each) per block of the runs and rows kernels: a few per block, so that launching
 // thousands of tiny blocks does not set the pace of a short kernel.
-constexpr int kRunsWarps = 4, kRowsWarps = 2;
+constexpr int kRunsWarps = 4, kRowsWarps = 4;
 
 template <bool kMom>
 __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams P) {
@@ -568,34 +568,34 @@ __global__ void __launch_bounds__(128) bwd_units_kernel(const unsigned char *__r
 
 // The 7 x 8-bit backward GEMM's units: the (8-atom tile, 128-row output tile) pairs that hold the slot
 // of some atom of the tile of type t, from the atoms' slot keys (a key's rows are 6 key .. 6 key + 5),
-// per centre type; one warp per (type, tile), the row tiles marked in a shared-memory bit set.
+// per centre type; one block per (type, tile), a warp per atom, the row tiles marked in a shared-memory
+// bit set.
 constexpr int kMaxRowTiles = 256;
 static_assert((int64_t)kMaxKeys * kQ <= (int64_t)kMaxRowTiles * kTM, "row tiles of the backward A fit the bit set");
-__global__ void __launch_bounds__(128) bwd_units8_kernel(const short *__restrict__ keys, const int *__restrict__ nslots,
-                                                         const int32_t *__restrict__ atype, int ntypes, int cap,
-                                                         int64_t atom0, int64_t natoms, int64_t ntiles8,
-                                                         int64_t maxunits8, int *__restrict__ units,
-                                                         int *__restrict__ nunits) {
-  __shared__ unsigned bits[4][kMaxRowTiles / 32];
-  const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5;
-  const int64_t w = (int64_t)blockIdx.x * 4 + wl;
-  if (w >= (int64_t)ntypes * ntiles8) return;  // warp-uniform
-  const int t = (int)(w / ntiles8);
-  const int64_t tile = w - (int64_t)t * ntiles8;
-  if (lane < kMaxRowTiles / 32) bits[wl][lane] = 0u;
-  __syncwarp();
-  for (int al = 0; al < tb::kAtomsB; ++al) {
-    const int64_t a = tile * tb::kAtomsB + al, i = atom0 + a;
-    if (a >= natoms || (atype && clampi(atype[i], 0, ntypes - 1) != t)) continue;  // warp-uniform
+__global__ void __launch_bounds__(32 * tb::kAtomsB) bwd_units8_kernel(const short *__restrict__ keys,
+                                                                    const int *__restrict__ nslots,
+                                                                    const int32_t *__restrict__ atype, int ntypes,
+                                                                    int cap, int64_t atom0, int64_t natoms,
+                                                                    int64_t ntiles8, int64_t maxunits8,
+                                                                    int *__restrict__ units, int *__restrict__ nunits) {
+  __shared__ unsigned bits[kMaxRowTiles / 32];
+  const int lane = threadIdx.x & 31, al = threadIdx.x >> 5;
+  const int t = (int)(blockIdx.x / ntiles8);
+  const int64_t tile = blockIdx.x - (int64_t)t * ntiles8;
+  if (threadIdx.x < kMaxRowTiles / 32) bits[threadIdx.x] = 0u;
+  __syncthreads();
+  const int64_t a = tile * tb::kAtomsB + al, i = atom0 + a;
+  if (a < natoms && (!atype || clampi(atype[i], 0, ntypes - 1) == t)) {  // warp-uniform
     const int ns = nslots[i];
     for (int slot = lane; slot < ns; slot += 32) {
       const int r0 = kQ * (int)keys[i * cap + slot], m_lo = r0 / kTM, m_hi = (r0 + kQ - 1) / kTM;
-      atomicOr(&bits[wl][m_lo >> 5], 1u << (m_lo & 31));
-      atomicOr(&bits[wl][m_hi >> 5], 1u << (m_hi & 31));
+      atomicOr(&bits[m_lo >> 5], 1u << (m_lo & 31));
+      atomicOr(&bits[m_hi >> 5], 1u << (m_hi & 31));
     }
   }
-  __syncwarp();
-  const unsigned word = lane < kMaxRowTiles / 32 ? bits[wl][lane] : 0u;
+  __syncthreads();
+  if (al != 0) return;
+  const unsigned word = lane < kMaxRowTiles / 32 ? bits[lane] : 0u;
   const int cnt = __popc(word);
   int before = cnt;  // inclusive prefix over the lanes
 #pragma unroll
@@ -680,23 +680,16 @@ struct RowsParams {
   int64_t natoms;
 };
 
-struct alignas(16) RowsStage {
-  double r[32][4];
-  double u[32], dinv[32];  // u and 1 / Delta_l of each staged row
-  double dw[32][24];       // per run of the batch: dW[k][q] at 6 k + q
-  int run[32], clamped[32], row[32], rslot[32];
-  int nvb[DP_MAX_TYPES];
-};
-
-// One warp per atom: per 32-row batch the batch's runs copied to shared memory and each valid row's
-// dE/dR~ and dE/ds by Horner's rule in u with its derivative (a lane per row); padded rows get zeros.
+// One warp per atom, a lane per valid row: the row's interval from s, its run slot from the atom's key map
+// (shared memory), the slot's gradient coefficients dW[k][q] read through L1 (the rows of a run share
+// them), and dE/dR~ and dE/ds by Horner's rule in u with its derivative; padded rows get zeros.
 __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams P) {
-  __shared__ RowsStage stw[kRowsWarps];
+  __shared__ int nvbw[kRowsWarps][DP_MAX_TYPES];
   extern __shared__ short smapw[];  // [kRowsWarps][nkeys]
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t a = (int64_t)blockIdx.x * kRowsWarps + warp;
   if (a >= P.natoms) return;  // warp-uniform
-  RowsStage &st = stw[warp];
+  int *nvb = nvbw[warp];
   short *smap = smapw + (size_t)warp * P.nkeys;
   const int64_t i = P.atom0 + a;
   const short *keys = P.keys + i * P.cap;
@@ -704,75 +697,45 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
   for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
   __syncwarp();
   for (int x = lane; x < nslot; x += 32) smap[keys[x]] = (short)x;  // the map of the atom's keys
-  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the map)
+  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, nvb);  // (its __syncwarp orders the map)
   const double *dWa = P.dW + (size_t)a * P.cap * 24;
   const double *srow = P.s + i * P.nnei;
   const double *Rrow = P.Rt + i * P.nnei * 4;
   double *dsrow = P.ds + i * P.nnei;
   double *drow = P.dRt + i * P.nnei * 4;
-  for (int base = 0; base < nv; base += 32) {
-    const int v = base + lane;
-    int mykey = -1;
-    if (v < nv) {
-      int b;
-      const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
-      double t;
-      bool clamped;
-      const int l = locate_fast(P.g, P.gf, P.nodes, __ldg(srow + row), t, clamped);
-      const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
-      st.r[lane][0] = rr.x;
-      st.r[lane][1] = rr.y;
-      st.r[lane][2] = rr.z;
-      st.r[lane][3] = rr.w;
-      const double dinv = l < P.g.n0 ? P.g.inv0 : P.g.inv1;
-      st.u[lane] = t * dinv;
-      st.dinv[lane] = dinv;
-      mykey = b * P.g.nint + l;
-      st.clamped[lane] = clamped;
-      st.row[lane] = row;
-    }
-    const int cnt = min(32, nv - base);
-    const int prev = __shfl_up_sync(0xffffffffu, mykey, 1);
-    const bool start = lane < cnt && (lane == 0 || mykey != prev);
-    const unsigned starts = __ballot_sync(0xffffffffu, start);
-    const int nrun = __popc(starts);
-    const int myrun = __popc(starts & (0xffffffffu >> (31 - lane))) - 1;  // runs starting at lanes <= this one
-    if (lane < cnt) st.run[lane] = myrun;
-    if (start) st.rslot[myrun] = smap[mykey];
-    __syncwarp();
-    for (int x = lane; x < nrun * 24; x += 32) {
-      const int r = x / 24, j = x - 24 * r;
-      st.dw[r][j] = dWa[(size_t)st.rslot[r] * 24 + j];
-    }
-    __syncwarp();
-    if (lane < cnt) {
-      const double *dw = st.dw[st.run[lane]];
-      const double u = st.u[lane];
-      double d4[4], ds = 0.0;
+  for (int v = lane; v < nv; v += 32) {
+    int b;
+    const int row = valid_row(v, nvb, P.sel, P.ntypes, b);
+    double t;
+    bool clamped;
+    const int l = locate_fast(P.g, P.gf, P.nodes, __ldg(srow + row), t, clamped);
+    const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
+    const double dinv = l < P.g.n0 ? P.g.inv0 : P.g.inv1;
+    const double u = t * dinv;
+    const double2 *dw = reinterpret_cast<const double2 *>(dWa + (size_t)smap[b * P.g.nint + l] * 24);
+    const double r4[4] = {rr.x, rr.y, rr.z, rr.w};
+    double d4[4], ds = 0.0;
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {  // P_k(u) = sum_q dW[k][q] u^q and P_k'(u): 5 + 4 FMA
-        const double *c = dw + 6 * k;
-        double p = fma(c[5], u, c[4]), dp = c[5];
-        dp = fma(dp, u, p);
-        p = fma(p, u, c[3]);
-        dp = fma(dp, u, p);
-        p = fma(p, u, c[2]);
-        dp = fma(dp, u, p);
-        p = fma(p, u, c[1]);
-        dp = fma(dp, u, p);
-        d4[k] = fma(p, u, c[0]);
-        ds = fma(st.r[lane][k], dp, ds);
-      }
-      const int row = st.row[lane];
-      dsrow[row] = st.clamped[lane] ? 0.0 : ds * st.dinv[lane];
-      st4(drow + (size_t)row * 4, d4[0], d4[1], d4[2], d4[3]);
+    for (int k = 0; k < 4; ++k) {  // P_k(u) = sum_q dW[k][q] u^q and P_k'(u): 5 + 4 FMA
+      const double2 c01 = __ldg(dw + 3 * k), c23 = __ldg(dw + 3 * k + 1), c45 = __ldg(dw + 3 * k + 2);
+      double p = fma(c45.y, u, c45.x), dp = c45.y;
+      dp = fma(dp, u, p);
+      p = fma(p, u, c23.y);
+      dp = fma(dp, u, p);
+      p = fma(p, u, c23.x);
+      dp = fma(dp, u, p);
+      p = fma(p, u, c01.y);
+      dp = fma(dp, u, p);
+      d4[k] = fma(p, u, c01.x);
+      ds = fma(r4[k], dp, ds);
     }
-    __syncwarp();
+    dsrow[row] = clamped ? 0.0 : ds * dinv;
+    st4(drow + (size_t)row * 4, d4[0], d4[1], d4[2], d4[3]);
   }
   // padded rows of each segment
   int off = 0;
   for (int b = 0; b < P.ntypes; ++b) {  // uniform
-    for (int j = st.nvb[b] + lane; j < P.sel[b]; j += 32) {
+    for (int j = nvb[b] + lane; j < P.sel[b]; j += 32) {
       dsrow[off + j] = 0.0;
       st4(drow + (size_t)(off + j) * 4, 0.0, 0.0, 0.0, 0.0);
     }
@@ -1043,14 +1006,14 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
     }
     if (S.b8) {
       // B = dT^T on 8-atom tiles in the 7 x 8-bit digits: the columns 4 a + k are the rows of this chunk's dT
-      if ((rc = split_rows<Digits7x8>(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, round_up(kCols * n, tb::kTNB),
-                                      S.Kpm, tb::kTNB, wk + L.bplanes, wk + L.fexp, st, who)))
+      if ((rc = split_rows_1k<Digits7x8>(dT + c0 * kCols * M1, M1, 1, kCols * n, M1, round_up(kCols * n, tb::kTNB),
+                                         S.Kpm, tb::kTNB, wk + L.bplanes, wk + L.fexp, st, who)))
         return rc;
       prof_mark("tc_split_dT", st);
       if (cudaMemsetAsync(wk + L.nunits, 0, (size_t)ntypes * sizeof(int), st) != cudaSuccess)
         return set_error(DP_ERR_CUDA, "%s: cudaMemsetAsync: %s", who, cudaGetErrorString(cudaGetLastError()));
       const int64_t ntiles8 = (n + tb::kAtomsB - 1) / tb::kAtomsB, nlist = (int64_t)ntypes * ntiles8;
-      bwd_units8_kernel<<<(unsigned)((nlist + 3) / 4), 128, 0, st>>>(
+      bwd_units8_kernel<<<(unsigned)nlist, 32 * tb::kAtomsB, 0, st>>>(
           R.keys, R.nslots, atype, ntypes, S.cap, c0, n, ntiles8, S.maxunits8, reinterpret_cast<int *>(wk + L.units),
           reinterpret_cast<int *>(wk + L.nunits));
       if ((rc = launch_status(who))) return rc;

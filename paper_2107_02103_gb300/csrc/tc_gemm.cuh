@@ -731,6 +731,48 @@ int set_smem(const char *who) {
   return DP_OK;
 }
 
+// split_rows_kernel with the row exponents found in the same kernel: one warp per group of 8 rows and
+// all of K (lane = (row ri8 = lane / 4, pair of k kp = lane % 4)), a first pass over the rows for their
+// largest exponents (reduced over the row's four lanes), a second for the digits.  For short rows
+// (the tabulation's dT^T, K = M1), where a launch per pass costs more than the passes.
+template <class D>
+__global__ void __launch_bounds__(128) split_rows_1k_kernel(const double *__restrict__ X, int64_t ld_r, int64_t ld_k,
+                                                            int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
+                                                            unsigned char *__restrict__ planes, int *__restrict__ exps) {
+  constexpr int NS = D::kNS;
+  const int lane = threadIdx.x & 31, ri8 = lane >> 2, kp = lane & 3;
+  const int64_t g = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);  // 8-row group
+  if (g * 8 >= rows_p) return;                                      // warp-uniform
+  const int64_t r = g * 8 + ri8;
+  const double *__restrict__ xr = X + (r < nrows ? r : 0) * ld_r;
+  auto x = [&](int k) { return (r < nrows && k < K) ? __ldg(xr + k * ld_k) : 0.0; };
+  int eb = 0;
+  for (int k0 = 0; k0 < Kp; k0 += 8) eb = max(eb, max(exp_bits(x(k0 + 2 * kp)), exp_bits(x(k0 + 2 * kp + 1))));
+  eb = max(eb, __shfl_xor_sync(0xffffffffu, eb, 1));
+  eb = max(eb, __shfl_xor_sync(0xffffffffu, eb, 2));
+  const int E = exp_of_max(eb);
+  if (kp == 0) exps[r] = E;
+  const size_t plane = (size_t)RT * kTK * 2, block = NS * plane;
+  const int ri = (int)(r % RT);
+  unsigned char *rowbase = planes + (size_t)(r / RT) * (Kp / kTK) * block + (ri >> 3) * kSBO + (ri & 7) * 16 + kp * 4;
+  for (int k0 = 0; k0 < Kp; k0 += 8) {
+    const int k = k0 + 2 * kp;
+    uint32_t h[NS];
+    digit_pairs<D>(biased_fixed<D>(x(k), E), biased_fixed<D>(x(k + 1), E), h);
+    unsigned char *dst = rowbase + (size_t)(k0 / kTK) * block + ((k0 % kTK) >> 3) * kLBO;
+#pragma unroll
+    for (int s = 0; s < NS; ++s) *reinterpret_cast<uint32_t *>(dst + s * plane) = h[s];
+  }
+}
+
+template <class D>
+int split_rows_1k(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
+                  unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
+  split_rows_1k_kernel<D><<<(unsigned)((rows_p / 8 + 3) / 4), 128, 0, st>>>(X, ld_r, ld_k, nrows, K, rows_p, Kp, RT,
+                                                                            planes, reinterpret_cast<int *>(exps));
+  return launch_status(who);
+}
+
 template <class D = Digits9x6>
 int split_rows(const double *X, int64_t ld_r, int64_t ld_k, int64_t nrows, int K, int64_t rows_p, int Kp, int RT,
                unsigned char *planes, unsigned char *exps, cudaStream_t st, const char *who) {
