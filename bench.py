@@ -178,10 +178,10 @@ def moment_fmas(runs, M1: int) -> dict:
 
 
 # DRAM bytes per launch (dram__bytes_read.sum + dram__bytes_write.sum) of a kernel, from the one
-# `ncu --set full` capture of its current version; absent means no capture of the current kernel
-# exists and `traffic` is reported as null.
-PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,
-                       ("cu85", "f64", "tc_rows", "tc"): 104700160 + 32997632}
+# `ncu --set full` capture of its current version (the commit the capture was taken at beside each);
+# absent means no capture of the current kernel exists and `traffic` is reported as null.
+PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,   # commit 7987c32
+                       ("cu85", "f64", "tc_rows", "tc"): 104687872 + 32025856}    # commit 640c6cd
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ, nsm: int = NSM) -> float:
