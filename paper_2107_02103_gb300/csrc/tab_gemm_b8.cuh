@@ -10,8 +10,11 @@
 // the tensor core waiting for every epilogue.  Roles: warp 0 moves each slice's A and B blocks into a
 // ring of five stages (bulk copies counted on the stage's "full" barrier), lane 0 of warp 1 issues the
 // MMAs into accumulator buffer (unit & 1) once the epilogue has released it ("tmem_free") and commits
-// "acc_full" for that buffer, and eight epilogue warps (two per TMEM lane quadrant, 16 columns each)
-// finish the outputs.  Every wait is bounded; a wait that gives up stops the CTA's copies and MMAs,
+// "acc_full" for that buffer, warp 10 builds each unit's slot table (the run slot of every (interval,
+// atom) of the unit, from the atoms' slot keys) and column exponents into table buffer (unit & 1)
+// ahead of the epilogue ("tbl_full", released by "tbl_empty"), and eight epilogue warps (two per TMEM
+// lane quadrant, 16 columns each) finish the outputs.  (Measured: with the epilogue warps building the
+// tables themselves, the tensor core waited for the epilogue about 40 % of the time.)  Every wait is bounded; a wait that gives up stops the CTA's copies and MMAs,
 // its remaining outputs are NaN and one timeout is counted (dp_tc_wait_timeouts).
 #pragma once
 
@@ -33,7 +36,8 @@ constexpr int kPlaneBB = kTNB * kTK * 2; // of a 32-row B block: 1 KB
 constexpr int kStageBytesB = kSB * (kPlaneAB + kPlaneBB);
 constexpr int kMaxKB = 144;              // K (channels, padded to 16) of one exact share
 constexpr int kEpiWarpsB = 8;
-constexpr int kThreadsB = 32 * (2 + kEpiWarpsB);
+constexpr int kThreadsB = 32 * (3 + kEpiWarpsB);  // producer, MMA issuer, epilogue, table warp
+constexpr int kTableWarp = 2 + kEpiWarpsB;
 constexpr int kEpiColsB = kTNB / 2;      // columns per epilogue warp
 constexpr uint32_t kBufColsB = 256;      // TMEM columns per accumulator buffer (7 x 32 used)
 constexpr int kScatKeysB = kTM / 4 + 1;  // keys a 128-row tile touches (kq >= 4)
@@ -61,10 +65,12 @@ struct Params {
 
 __host__ __device__ constexpr int unit_code(int tile, int mt) { return tile | (mt << 16); }
 
-constexpr size_t kBarOffB = (size_t)kStagesB * kStageBytesB;    // full[5], empty[5], acc_full[2], tmem_free[2]
-constexpr size_t kMiscOffB = kBarOffB + (2 * kStagesB + 4) * 8;   // tmem address, abort flag
-constexpr size_t kStabOffB = kMiscOffB + 16;                      // slot table, slot counts, flag, exponents
-constexpr size_t kSmemB = kStabOffB + (kScatKeysB * kAtomsB + kAtomsB + 4 + kTNB) * 4;
+// full[5], empty[5], acc_full[2], tmem_free[2], tbl_full[2], tbl_empty[2]
+constexpr size_t kBarOffB = (size_t)kStagesB * kStageBytesB;
+constexpr size_t kMiscOffB = kBarOffB + (2 * kStagesB + 8) * 8;   // tmem address, abort flag
+constexpr size_t kStabOffB = kMiscOffB + 16;                      // two tables: slots, exponents; flags
+constexpr int kTableInts = kScatKeysB * kAtomsB + kTNB;          // one table buffer
+constexpr size_t kSmemB = kStabOffB + (2 * kTableInts + 4) * 4;
 static_assert(kSmemB <= 227 * 1024, "shared memory per block");
 
 __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
@@ -73,12 +79,13 @@ __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
   uint64_t *empty = full + kStagesB;
   uint64_t *acc_full = empty + kStagesB;
   uint64_t *tmem_free = acc_full + 2;
+  uint64_t *tbl_full = tmem_free + 2;
+  uint64_t *tbl_empty = tbl_full + 2;
   uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(smem + kMiscOffB);
   volatile int *abortf = reinterpret_cast<volatile int *>(smem + kMiscOffB + 4);
-  int *stab = reinterpret_cast<int *>(smem + kStabOffB);  // (key of the unit, atom) -> slot, or -1
-  int *nsa = stab + kScatKeysB * kAtomsB;                   // per atom: slot count (0: not of type alpha)
-  int *uflag = nsa + kAtomsB;                               // [0]: the unit's accumulators are ready
-  int *fexp_s = uflag + 4;                                  // the unit's 32 column exponents
+  // table buffer b: (key of the unit, atom) -> slot or -1, then the unit's 32 column exponents
+  int *tables = reinterpret_cast<int *>(smem + kStabOffB);
+  int *uflag = tables + 2 * kTableInts;  // [0]: the unit's accumulators and table are ready
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nunits = *P.nunits;
 
@@ -90,6 +97,8 @@ __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
     for (int b = 0; b < 2; ++b) {
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(acc_full + b)));
       asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(tmem_free + b)), "r"(kEpiWarpsB));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(tbl_full + b)));
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(tbl_empty + b)), "r"(kEpiWarpsB));
     }
     asm volatile("fence.mbarrier_init.release.cluster;");
     *abortf = 0;
@@ -170,6 +179,48 @@ __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
       }
     }
     __syncwarp();
+  } else if (warp == kTableWarp) {
+    // ---- table warp: each unit's slot table and column exponents into table buffer (unit & 1)
+    int li = 0;
+    for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+      const int c = P.units[u], tile = c & 0xffff, mt = c >> 16;
+      const int b = li & 1;
+      if (li >= 2) {
+        int wv = 1;
+        if (lane == 0) wv = wait_or_abort(smem_u32(tbl_empty + b), (uint32_t)(((li >> 1) - 1) & 1), abortf);
+        if (!__shfl_sync(0xffffffffu, wv, 0)) break;
+      }
+      int *stab = tables + b * kTableInts, *fexp_s = stab + kScatKeysB * kAtomsB;
+      const int64_t a_first = (int64_t)tile * kAtomsB;
+      const int key0 = (int)((int64_t)mt * kTM / P.kq);
+      for (int x = lane; x < kScatKeysB * kAtomsB; x += 32) stab[x] = -1;
+      fexp_s[lane] = P.Fexp[(int64_t)tile * kTNB + lane];
+      __syncwarp();
+      // the slot counts of the unit's atoms (0: past the chunk or not of type alpha), lane al < 8
+      int nsl = 0;
+      if (lane < kAtomsB) {
+        const int64_t a = a_first + lane, i = P.atom0 + a;
+        nsl = a < P.natoms && (!P.atype || clampi(P.atype[i], 0, P.ntypes - 1) == P.alpha) ? P.nslots[i] : 0;
+      }
+      int nmax = nsl;
+#pragma unroll
+      for (int o = 1; o < kAtomsB; o <<= 1) nmax = max(nmax, __shfl_xor_sync(0xffffffffu, nmax, o));
+      nmax = __shfl_sync(0xffffffffu, nmax, 0);  // lanes 0 .. 7 hold the maximum; the loop below is uniform
+      // (atom, slot) pairs over the lanes, four slots of an atom per pass so that the key loads overlap
+      const short *keys = P.keys + (P.atom0 + a_first) * P.cap;
+      for (int s0 = 0; s0 < nmax; s0 += 16) {  // uniform
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+          const int al = lane >> 2, slot = s0 + 4 * h + (lane & 3);
+          const int ns = __shfl_sync(0xffffffffu, nsl, al);
+          const int key = slot < ns ? keys[(size_t)al * P.cap + slot] : -1;
+          if (key >= key0 && key < key0 + kScatKeysB) stab[(key - key0) * kAtomsB + al] = slot;
+        }
+      }
+      __syncwarp();
+      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(tbl_full + b)) : "memory");
+      ++li;
+    }
   } else {
     // ---- epilogue: warps 2 .. 9, TMEM lane quadrant warp % 4, columns 16 ((warp - 2) / 4) .. + 15
     const int et = tid - 64;
@@ -181,25 +232,12 @@ __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
       const int b = li & 1;
       const int64_t m0 = (int64_t)mt * kTM;
       const int64_t a_first = (int64_t)tile * kAtomsB;  // the unit's first atom in the chunk
-      asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarpsB));  // the previous unit's tables are free
-      if (et < kTNB) fexp_s[et] = P.Fexp[(int64_t)tile * kTNB + et];
-      for (int x = et; x < kScatKeysB * kAtomsB; x += 32 * kEpiWarpsB) stab[x] = -1;
-      if (et < kAtomsB) {
-        const int64_t a = a_first + et, i = P.atom0 + a;
-        nsa[et] = a < P.natoms && (!P.atype || clampi(P.atype[i], 0, P.ntypes - 1) == P.alpha) ? P.nslots[i] : 0;
-      }
-      asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarpsB));
+      const int *stab = tables + b * kTableInts, *fexp_s = stab + kScatKeysB * kAtomsB;
       const int key0 = (int)(m0 / P.kq);
-      {  // a warp per atom, its lanes over the slots
-        const int al = et >> 5;
-        const short *keys = P.keys + (P.atom0 + a_first + al) * P.cap;
-        for (int slot = lane; slot < nsa[al]; slot += 32) {
-          const int key = keys[slot];
-          if (key >= key0 && key < key0 + kScatKeysB) stab[(key - key0) * kAtomsB + al] = slot;
-        }
-      }
-      if (et == 0) uflag[0] = !*abortf && wait_or_abort(smem_u32(acc_full + b), (uint32_t)((li >> 1) & 1), abortf);
-      asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarpsB));  // the tables are built and the MMAs done
+      if (et == 0)
+        uflag[0] = !*abortf && wait_or_abort(smem_u32(tbl_full + b), (uint32_t)((li >> 1) & 1), abortf) &&
+                   wait_or_abort(smem_u32(acc_full + b), (uint32_t)((li >> 1) & 1), abortf);
+      asm volatile("bar.sync 1, %0;" ::"r"(32 * kEpiWarpsB));  // the table is built and the MMAs done
       const bool ok = uflag[0] != 0;
       asm volatile("tcgen05.fence::after_thread_sync;");
       const int Erow = m0 + rl < P.Mp ? P.Eexp[m0 + rl] : 0;
@@ -248,7 +286,10 @@ __global__ void __launch_bounds__(kThreadsB, 1) bgemm_kernel(const Params P) {
       }
       asm volatile("tcgen05.fence::before_thread_sync;");
       __syncwarp();
-      if (lane == 0) asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(tmem_free + b)) : "memory");
+      if (lane == 0) {
+        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(tmem_free + b)) : "memory");
+        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(tbl_empty + b)) : "memory");
+      }
       ++li;
     }
   }
