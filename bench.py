@@ -68,7 +68,13 @@ def footprint(w, esize: int, hbm_bytes: float = 280e9) -> dict:
 # f64 fitting GEMMs on the tensor cores: every operand element is split into 9 digits and the 45 digit
 # products with s + t <= 10 run as fp16 MMAs, so a GEMM of 2 n K N FP64 flop issues 45 times as many
 # fp16 MMA flop; their roofline is the dense 16-bit tensor rate (fp16 and bf16 run at the same rate).
-TC_DIGIT_PRODUCTS = 45
+TC_DIGIT_PRODUCTS = 45  # fp16 digit products per FP64-equivalent FMA: nine 6-bit digits (s + t <= 10)
+
+
+def tc_products(kernel: str, M1: int) -> int:
+    """Digit products per FP64-equivalent FMA of a tensor-core tabulation GEMM: the backward uses seven
+    8-bit digits (28 products) while its K, M1 padded to 16, is at most 144; else nine 6-bit (45)."""
+    return 28 if kernel == "tc_gemm_grad" and -(-M1 // 16) * 16 <= 144 else TC_DIGIT_PRODUCTS
 
 
 def tensor_peak() -> tuple:
@@ -152,9 +158,9 @@ TC_FMA = {"tc_runs_moments": ("row", 24), "tc_rows": ("row", 40), "tc_gemm_fwd":
           "tc_gemm_grad": ("run", 24)}
 TC_KERNEL = {"tc_runs_moments": "runs_kernel<moments> (dp_tabulate_fusion_fwd_tc_f64)",
              "tc_rows": "rows_kernel (dp_tabulate_fusion_grad_tc_f64)",
-             "tc_gemm_fwd": "gemm_kernel (dp_tabulate_fusion_fwd_tc_f64)",
-             "tc_gemm_grad": "gemm_kernel (dp_tabulate_fusion_grad_tc_f64)"}
-TC_CHUNK_ATOMS = 4104  # atoms per chunk of the tc calls
+             "tc_gemm_fwd": "tgemm_kernel (dp_tabulate_fusion_fwd_tc_f64)",
+             "tc_gemm_grad": "bgemm_kernel (dp_tabulate_fusion_grad_tc_f64)"}
+TC_CHUNK_ATOMS = 16416  # atoms per chunk of the tc calls
 
 
 def tc_profile_events(w) -> int:
@@ -222,11 +228,12 @@ def step_bytes(w, esize: int) -> dict:
 def tc_step_bound(w, nruns: float, nsm: int, ms_step: float) -> dict:
     """The roofline of the step the tensor-core path runs: the slowest of its FP64-pipe work (the per-row
     moments, 24 FMA, and derivatives, 40 FMA, per valid row, and the descriptor's 4 M1 M2 per atom) at the
-    FP64 peak, its digit-product MMAs (24 M1 FMA per run and direction, 45 fp16 products each) at the
-    measured dense 16-bit tensor peak, and its algorithmic bytes at the measured HBM bandwidth."""
+    FP64 peak, its digit-product MMAs (24 M1 FMA per run and direction, 45 fp16 products each forward and
+    28 backward) at the measured dense 16-bit tensor peak, and its algorithmic bytes at the measured HBM
+    bandwidth."""
     rows = float(w.evals) / w.M1
     fp64_fma = (24 + 40) * rows + DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc
-    tensor_flop = 2.0 * TC_DIGIT_PRODUCTS * 2 * 24 * w.M1 * float(nruns)
+    tensor_flop = 2.0 * (tc_products("tc_gemm_fwd", w.M1) + tc_products("tc_gemm_grad", w.M1)) * 24 * w.M1 * float(nruns)
     hbm, hbasis = hbm_peak()
     tpk, tbasis = tensor_peak()
     t = {"fp64": 2.0 * fp64_fma / (peak_tflops("f64", nsm=nsm) * 1e12) * 1e3,
@@ -735,7 +742,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
             if k in tcf:
                 e["tflops"] = round(2.0 * tcf[k] / (ms * 1e-3) / 1e12, 4)  # FP64 (equivalent) flop
                 if k.startswith("tc_gemm"):
-                    e["tensor_tflops"] = round(TC_DIGIT_PRODUCTS * e["tflops"], 2)
+                    e["tensor_tflops"] = round(tc_products(k, w.M1) * e["tflops"], 2)
                     e["tensor_frac"] = round(e["tensor_tflops"] / tpk, 4)
                 else:
                     e["frac"] = round(e["tflops"] / pk, 4)
@@ -750,7 +757,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                         "frac": e["tensor_frac"] if gemm else e["frac"],
                         "traffic": PROFILED_DRAM_BYTES.get((w.name, args.dtype, dom, args.algo)),
                         "kernel": TC_KERNEL[dom],
-                        "peak_basis": (f"{tbasis}; achieved counts all {TC_DIGIT_PRODUCTS} fp16 digit products"
+                        "peak_basis": (f"{tbasis}; achieved counts all {tc_products(dom, w.M1)} fp16 digit products"
                                        if gemm else peak_basis(args.dtype, nsm)),
                         "fwd_grad_frac_fp64_equivalent": round(path_tflops / pk, 4)}
         if not args.chain:  # the whole step against the bound of the algorithm it runs

@@ -1,19 +1,22 @@
 // Persistent exact-f64 GEMM for the tensor-core tabulation (tabulate_tc.cu): the per-interval
-// contraction of every 12-atom tile, forward (T = W C' over the used K slices) and backward
-// (dW = dT C'^T over the used 128-row output tiles), on the digit-split operands of tc_gemm.cuh.
+// contraction of every 12-atom tile in the forward (T = W C' over the used K slices), on the 9 x 6-bit
+// digit-split operands of tc_gemm.cuh; also the backward (dW = dT C'^T over the used 128-row output
+// tiles) where M1 > 144 (else tab_gemm_b8.cuh's 7 x 8-bit kernel runs it).
 //
-// One CTA per SM walks its units -- (atom tile, 128-row tile of A, share of K) forward, (atom tile,
-// 128-row output tile) backward, from a list of the units with work -- round-robin over the grid.  The TMEM accumulators (nine
-// diagonals x 48 columns), the mbarriers and the stage ring are set up once per CTA, and the roles
-// run ahead of each other: warp 0 moves each slice's A and B blocks into a ring of four stages (bulk
-// copies counted on the stage's "full" barrier; in the forward a split warp per stage writes the B
-// block from the moments instead, as digit planes, and arrives on the same barrier), lane 0 of warp 1
-// issues the slice's 13 MMAs and
-// frees the stage ("empty") when they complete, and eight epilogue warps (two per TMEM lane quadrant,
-// 24 columns each) read the unit's accumulators once its last MMA has completed ("acc_full"),
-// recombine each output's diagonals exactly as an integer and round it once to f64 (or, for a tile with
-// several shares, store four floats), write the outputs, then release the accumulators ("tmem_free")
-// for the next unit's MMAs.  The copies of the next unit overlap the epilogue of this one.
+// One CTA per SM walks its units: forward, the pieces the schedule gave it, in order -- (centre type,
+// atom tile, 128-row tile of A, a run of at most 112 of the tile's used slices), every centre type in
+// one launch; backward, a list of the (atom tile, 128-row output tile) pairs with work, round-robin
+// over the grid.  The TMEM accumulators (nine diagonals x 48 columns), the mbarriers and the stage ring
+// are set up once per CTA, and the roles run ahead of each other: warp 0 moves each slice's A block
+// (and in the backward its B block) into a ring of four stages (bulk copies counted on the stage's
+// "full" barrier); in the forward a split warp per stage writes the B block from the moments, as digit
+// planes, and arrives on the same barrier; lane 0 of warp 1 issues the slice's 13 MMAs and frees the
+// stage ("empty") when they complete; eight epilogue warps (two per TMEM lane quadrant, 24 columns
+// each) read the unit's accumulators once its last MMA has completed ("acc_full"), recombine each
+// output's diagonals exactly as an integer and round it once to f64 (diag_to_f64) -- or, for a piece
+// of a cut item, store the integer for fwd_epilogue_kernel to sum -- write the outputs, then release
+// the accumulators ("tmem_free") for the next unit's MMAs.  The copies of the next unit overlap the
+// epilogue of this one.  The two directions are separate instantiations of the kernel.
 // Every wait is bounded; a wait that gives up stops the CTA's copies and MMAs, its remaining
 // outputs are NaN and one timeout is counted (dp_tc_wait_timeouts).
 #pragma once

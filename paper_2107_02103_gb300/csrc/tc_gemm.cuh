@@ -29,8 +29,10 @@ namespace {
 // floats (the two largest by an exact two-sum, the rest in float-float, whose
 // rounding lies ~2^-60 below the result); the caller's epilogue (Sum3 below)
 // adds the shares' floats into a three-float sum by exact two-sums and
-// converts it to f64 once -- or recombines the diagonals exactly as one
-// integer and rounds that once (diag_int, i128_to_double).
+// converts it to f64 once -- or, in the tabulation's GEMMs, recombines the
+// diagonals exactly as one 128-bit integer and rounds that once (diag_s128,
+// s128_to_f64).  The tabulation's backward, whose K is M1 <= 144, splits into
+// seven 8-bit digits instead (Digits7x8; 28 products, diag7_to_f64).
 // What rounds is that conversion, the 53-bit truncation of the operands and
 // the dropped terms: |error| <~ K 2^-49 max_k|a_ik| max_k|b_kj|, against
 // K 2^-53 sum_k |a_ik b_kj| for an f64 dot product.  A row or column with an

@@ -239,9 +239,9 @@ def test_tc_work_buffer_rules_and_reuse():
 
 
 def test_tc_water_large_chunk_edges():
-    """The default f64 path at its largest size: 1,048,576 atoms in 256 chunks, in the benchmark's launch
+    """The default f64 path at its largest size: 1,048,576 atoms in 64 chunks, in the benchmark's launch
     configuration (one plan, one work buffer, the backward reusing the forward's interval runs).  The
-    oracle on 256 atoms gathered on the device: the first and last atom of 24 chunks spread over the run (edges from the 1st chunk to the 256th, byte offsets into R~ and dR~ past
+    oracle on 256 atoms gathered on the device: the first and last atom of 24 chunks spread over the run (edges from the 1st chunk to the 64th, byte offsets into R~ and dR~ past
     2^32) and random atoms; the FP64-pipe moment path on every atom, compared on the device; and
     the identity <dR~, R~> = <dT, T> over every atom, which holds at any size."""
     dpc = lib()
