@@ -155,8 +155,9 @@ def interval_runs(w, info, n0: int, n1: int):
 #   tc_gemm_fwd      T += W C' per run                    24 M1 per run
 #   tc_gemm_grad     dW = dT C'^T per run                 24 M1 per run
 TC_FMA = {"tc_runs_moments": ("row", 24), "tc_rows": ("row", 40), "tc_gemm_fwd": ("run", 24),
-          "tc_gemm_grad": ("run", 24)}
+          "tc_gemm_grad": ("run", 24), "tc_finish_fwd": ("atom", 0)}  # the finish: D's 4 M1 M2 per atom
 TC_KERNEL = {"tc_runs_moments": "runs_kernel<moments> (dp_tabulate_fusion_fwd_tc_f64)",
+             "tc_finish_fwd": "fwd_finish_kernel: T of cut items and D (dp_tabulate_fusion_fwd_tc_f64)",
              "tc_rows": "rows_kernel (dp_tabulate_fusion_grad_tc_f64)",
              "tc_gemm_fwd": "tgemm_kernel (dp_tabulate_fusion_fwd_tc_f64)",
              "tc_gemm_grad": "bgemm_kernel (dp_tabulate_fusion_grad_tc_f64)"}
@@ -173,7 +174,8 @@ def tc_profile_events(w) -> int:
 
 def tc_fmas(w, runs) -> dict:
     rows = float(w.evals) / w.M1
-    return {k: (n * rows if per == "row" else n * w.M1 * float(len(runs))) for k, (per, n) in TC_FMA.items()}
+    return {k: (n * rows if per == "row" else DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc if per == "atom"
+                else n * w.M1 * float(len(runs))) for k, (per, n) in TC_FMA.items()}
 
 
 def moment_fmas(runs, M1: int) -> dict:
@@ -360,12 +362,13 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
                           device=dev)
         plan = dpc.dp_tabulate_tc_plan_f64(model.table, info, w.nnei)  # setup, once per table (like the build)
 
-        def fwd(table, *a, out=None):
-            return dpc.dp_tabulate_fusion_fwd_tc_f64(plan, *a, out=out, work=tcw)
+        def fwd(table, *a, out=None, D=None):  # with D: the descriptor written by the same call
+            return dpc.dp_tabulate_fusion_fwd_tc_f64(plan, *a, out=out, work=tcw, M2=None if D is None else w.M2, D=D)
 
         def grad(table, *a, out=None):  # on the forward's inputs: it takes the forward's interval runs
             return dpc.dp_tabulate_fusion_grad_tc_f64(plan, *a, out=out, work=tcw, flags=dpc.DP_TC_REUSE_RUNS)
     arith = dpc.DF64 if args.dtype == "df64" else None  # the table picks the fusion kernels' arithmetic
+    fused_d = args.algo == "tc"  # D from the tensor-core forward itself (no descriptor_kernel launch)
     T = torch.empty((w.nloc, 4, w.M1), dtype=dtype, device=dev)
     D = torch.empty((w.nloc, w.M1, w.M2), dtype=dtype, device=dev)
     ds = torch.empty((w.nloc, w.nnei), dtype=dtype, device=dev)
@@ -375,16 +378,19 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
                 "nvalid": w.nvalid, "atype": w.atype, "dT": np.ascontiguousarray(w.dT.astype(npdt))}
         d = {k: torch.from_numpy(v).to(dev) for k, v in host.items()}
         outs = dict(T=T, D=D, ds=ds, dRt=dRt)
-        names = ["fwd", "descriptor", "grad"]
+        names = ["fwd", "grad"] if fused_d else ["fwd", "descriptor", "grad"]
 
         def step(rec, x, o):
-            rec(0)
-            fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
-            rec(1)
-            dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"], arith=arith)
-            rec(2)
+            rec(k := 0)
+            if fused_d:  # the tensor-core forward writes D as well
+                fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"], D=o["D"])
+            else:
+                fwd(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, out=o["T"])
+                rec(k := k + 1)
+                dpc.dp_descriptor_contract(o["T"], w.M2, out=o["D"], arith=arith)
+            rec(k := k + 1)
             grad(model.table, info, x["s"], x["Rt"], x["nvalid"], x["atype"], sel, x["dT"], out=(o["ds"], o["dRt"]))
-            rec(3)
+            rec(k := k + 1)
         return host, d, outs, names, step
 
     coord, nlist, _ = W.ghost_system(w)
@@ -406,6 +412,8 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     outs = dict(D=D, F=torch.empty((coord.shape[0], 3), dtype=dtype, device=dev),
                 virial=torch.empty((3, 3), dtype=dtype, device=dev))
     names = ["env_mat", "fwd", "descriptor", "descriptor_grad", "grad", "force_virial"]
+    if fused_d:
+        names.remove("descriptor")
     if args.fitting:
         H = sum(fwidths[1:-1])
         outs["E"] = torch.empty((w.nloc,), dtype=dtype, device=dev)
@@ -417,15 +425,20 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
                                          device=dev)
         names = ["env_mat", "fwd", "descriptor", "fitting_fwd", "fitting_grad", "descriptor_grad", "grad",
                  "force_virial"]
+        if fused_d:
+            names.remove("descriptor")
 
     def step(rec, x, o):
         k = 0
         rec(k)
         dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]), arith=arith)
         rec(k := k + 1)
-        fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
-        rec(k := k + 1)
-        dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"], arith=arith)
+        if fused_d:
+            fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"], D=o["D"])
+        else:
+            fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
+            rec(k := k + 1)
+            dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"], arith=arith)
         rec(k := k + 1)
         if args.fitting and args.fitting_tc:
             dpc.dp_fitting_fwd_tc_f64(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), work=work["fit_tc"])
@@ -538,7 +551,8 @@ def run_native(args, rank, world, local_rank):
         fmas = moment_fmas(interval_runs(w, info, *dpc.dp_table_info_sizes(info)), w.M1)
     nall = int(host["coord"].shape[0]) if "coord" in host else w.nloc
     tcf = tc_fmas(w, interval_runs(w, info, *dpc.dp_table_info_sizes(info))) if tc_ms else None
-    per_mark = {"tc_split_dT": 2, "tc_fwd": 0, "tc_grad": 0}  # kernels per mark
+    per_mark = {"tc_split_dT": 1 if -(-w.M1 // 16) * 16 <= 144 else 2, "tc_slice_lists": 2, "tc_fwd": 0,
+                "tc_grad": 0}  # kernels per mark
     out = report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas, nall, tc_ms, tcf,
                  [sum(per_mark.get(x, 1) for x in nm) for nm in pnames])
     if graph is not None:
@@ -702,6 +716,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     flops = {"fwd": 2.0 * fmas["fwd"], "grad": 2.0 * fmas["grad"],
              "descriptor": 2.0 * DESC_FMA_PER_ATOM(w.M1, w.M2) * w.nloc,
              "descriptor_grad": 2.0 * DESC_GRAD_FMA_PER_ATOM(w.M1, w.M2) * w.nloc}
+    if "descriptor" not in k_ms:  # the forward wrote D as well (tensor-core path)
+        flops["fwd"] += flops["descriptor"]
     if getattr(args, "fitting", False):
         flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w)[0]).items()})
     nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
@@ -772,7 +788,8 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
                    "step": (("env_mat + fwd + descriptor + fitting_fwd + fitting_grad + descriptor_grad + grad + "
                              "force_virial (energy and forces of the whole model)") if args.fitting else
                             "env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain
-                            else "fwd + descriptor + grad"), "algo": args.algo,
+                            else "fwd + descriptor + grad" if "descriptor" in k_ms
+                            else "fwd (writing D) + grad"), "algo": args.algo,
                    "fma_basis": ("interval moments: per run min(9 M1 L, 24 M1 + 24 L) fwd, "
                                  "min(18 M1 L, 24 M1 + 40 L) grad" if args.algo in ("moments", "tc")
                                  else "per row: 9 M1 fwd, 18 M1 grad"),

@@ -249,15 +249,24 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  * (1/nnei) sum_m dT[i][k][m] c'_q(..., l, m), from which every valid row
  * takes dRt[i][j][k] = sum_q dW[k][(b, l, q)] u_j^q and ds[i][j] =
  * sum_k R~[i][j][k] sum_{q>=1} q dW[k][(b, l, q)] u_j^(q-1) / Delta_l (0
- * where s was clamped).  Both GEMMs run exactly as in dp_fitting_*_tc_f64:
- * nine balanced 6-bit digits per element (in [-32, 32]), scaled by the row's
- * or column's power of two, fp16 MMAs with exact fp32 sums (at most 1792 of
- * K per partial sum), one rounding to f64; per output the error is below
- * about K 2^-49 max|row| max|column| (K: the used intervals x 6, or M1).  Only
- * the intervals some atom of a 12-atom tile uses enter its GEMM.  Rows need
+ * where s was clamped).  Both GEMMs run on digit-split operands with fp16
+ * MMAs and exact fp32 sums, and round each output once to f64: the forward
+ * as in dp_fitting_*_tc_f64 (nine balanced 6-bit digits per element, in
+ * [-32, 32], scaled by the row's or column's power of two; at most 1792 of K
+ * per partial sum; error below about K 2^-49 max|row| max|column|, K the
+ * used intervals x 6), the backward, whose K is M1, in seven balanced 8-bit
+ * digits (in [-128, 128]; error below K 2^-50 max|row| max|column|) while
+ * M1 <= 144, else as the forward.  Only the intervals some atom of a 12-atom
+ * (forward) or 8-atom (backward) tile uses enter its GEMM.  Rows need
  * not be sorted, though sorted rows (one run per interval) do the least
  * FP64 work.  NaN s gives NaN in that atom's T (forward) and in that row's
  * ds and dRt (backward); inf or NaN in dT gives NaN in the atom's rows.
+ *
+ * The forward also writes the descriptor when D is not NULL: D[i][m][n] =
+ * sum_k T[i][k][m] T[i][k][n] for n < M2 (dp_descriptor_contract_f64,
+ * computed from T in the same kernel that finishes T, with the same bits as
+ * that call), D [nloc][M1][M2] on the device, 1 <= M2 <= M1 (else
+ * DP_ERR_SHAPE).  With D NULL, M2 is ignored.
  *
  * The plan holds the scaled coefficients c'_q / nnei of every centre type
  * and their digit planes for both GEMMs; it depends only on the table, its
@@ -281,8 +290,9 @@ int dp_tabulate_fusion_grad_moments_f32(const float *table, const dp_table_info 
  *                     from the forward for the backward), and for one chunk
  *                     of at most 16416 atoms the moments or their gradients
  *                     per (atom, interval), the backward's B digit planes,
- *                     the forward's schedule and its partial results.  Calls sharing a work buffer must not overlap
- *                     on the GPU.
+ *                     the forward's schedule and its partial results.
+ *                     Calls sharing a work buffer must not overlap on the
+ *                     GPU.
  *   flags (backward)  0, or DP_TC_REUSE_RUNS: the forward call on the same
  *                     plan, s, nvalid, atype, nloc and work buffer ran before
  *                     this call on the stream, and nothing has written the
@@ -310,7 +320,8 @@ size_t dp_tabulate_tc_work_bytes(const dp_table_info *info, int64_t nloc, int nn
                                  int M1); /* 0 on bad sizes or table info */
 int dp_tabulate_fusion_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
-                                  const int32_t *sel, int M1, double *T, void *work, size_t work_bytes, void *stream);
+                                  const int32_t *sel, int M1, double *T, int M2, double *D, void *work,
+                                  size_t work_bytes, void *stream);
 int dp_tabulate_fusion_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
                                    const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
                                    const int32_t *sel, int M1, const double *dT, double *ds, double *dRt, void *work,

@@ -113,7 +113,7 @@ _SIGS = {
     "dp_tabulate_tc_plan_f64": ([_P, _INFO, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, ctypes.c_size_t, _PLAN,
                                  _P], ctypes.c_int),
     "dp_tabulate_fusion_fwd_tc_f64": ([_PLAN, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
-                                       ctypes.c_int, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
+                                       ctypes.c_int, _P, ctypes.c_int, _P, _P, ctypes.c_size_t, _P], ctypes.c_int),
     "dp_tabulate_fusion_grad_tc_f64": ([_PLAN, _INFO, _P, _P, _P, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
                                         ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t, ctypes.c_int, _P],
                                        ctypes.c_int),
@@ -455,21 +455,28 @@ def _tc_inputs(plan, info, s, Rt, nvalid, atype, sel):
     return plan, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, torch.float64
 
 
-def dp_tabulate_fusion_fwd_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None, work=None):
+def dp_tabulate_fusion_fwd_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, atype, sel, out=None, work=None,
+                                  M2=None, D=None):
     """T of dp_tabulate_fusion_fwd in f64 with the per-interval contraction on the tensor cores (interval
     moments times the scaled table, an exact digit-split GEMM).  plan: a TcPlan (dp_tabulate_tc_plan_f64)
     or the f64 table itself, planned for this call; work: a uint8 CUDA tensor of
-    dp_tabulate_tc_work_bytes(...) bytes, or None to allocate one."""
+    dp_tabulate_tc_work_bytes(...) bytes, or None to allocate one.  With M2 given, the same call also
+    writes the descriptor (dp_descriptor_contract of T) into D [nloc][M1][M2] (allocated when None) and
+    returns (T, D)."""
     plan, s, Rt, nvalid, atype, selc, ntypes, nloc, nnei, M1, dtype = _tc_inputs(plan, info, s, Rt, nvalid, atype, sel)
     shape = (nloc, 4, M1)
     T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
+    if M2 is not None:
+        dshape = (nloc, M1, int(M2))
+        D = torch.empty(dshape, dtype=dtype, device=s.device) if D is None else _dev(D, "D", dtype, dshape)
     if nloc == 0:
-        return T
+        return T if M2 is None else (T, D)
     work = _tab_tc_work(work, info, nloc, nnei, ntypes, M1, s.device)
     _check(_lib.dp_tabulate_fusion_fwd_tc_f64(ctypes.byref(plan.rec), ctypes.byref(info), _ptr(s), _ptr(Rt),
                                               _ptr(nvalid), _ptr(atype), nloc, nnei, ntypes, selc, M1, _ptr(T),
+                                              0 if M2 is None else int(M2), None if M2 is None else _ptr(D),
                                               _ptr(work), work.numel(), _stream(s)))
-    return T
+    return T if M2 is None else (T, D)
 
 
 def dp_tabulate_fusion_grad_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, atype, sel, dT, out=None, work=None,

@@ -14,7 +14,7 @@
 // stage ("empty") when they complete; eight epilogue warps (two per TMEM lane quadrant, 24 columns
 // each) read the unit's accumulators once its last MMA has completed ("acc_full"), recombine each
 // output's diagonals exactly as an integer and round it once to f64 (diag_to_f64) -- or, for a piece
-// of a cut item, store the integer for fwd_epilogue_kernel to sum -- write the outputs, then release
+// of a cut item, store the integer for fwd_finish_kernel to sum -- write the outputs, then release
 // the accumulators ("tmem_free") for the next unit's MMAs.  The copies of the next unit overlap the
 // epilogue of this one.  The two directions are separate instantiations of the kernel.
 // Every wait is bounded; a wait that gives up stops the CTA's copies and MMAs, its remaining
@@ -422,7 +422,7 @@ __global__ void __launch_bounds__(kThreadsP, 1) tgemm_kernel(const Params P) {
           for (int d = 0; d < kS; ++d) asm volatile("" : "+f"(v[d][0]), "+f"(v[d][1]), "+f"(v[d][2]), "+f"(v[d][3]));
         }
         const int al = (c_lo + c0) >> 2;  // the group's atom; column c0 + k is its component k
-        if (outp) {  // a piece of a cut item: its outputs' exact integers, summed by fwd_epilogue_kernel
+        if (outp) {  // a piece of a cut item: its outputs' exact integers, summed by fwd_finish_kernel
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
             long long hi;

@@ -32,7 +32,7 @@
 //             tgemm_kernel (tab_gemm.cuh; A = C'_alpha^T: channels x K, B = W^T: K x (atom, k), its
 //             digit planes made in shared memory from W; a tile whose used slices fit one share
 //             writes its atoms' T directly),
-//             fwd_epilogue_kernel (T of the tiles with several shares, or none);
+//             fwd_finish_kernel (T of the atoms whose items were cut into pieces, or have none; D);
 //   backward: runs_kernel<false> (slot keys, slice flags; skipped when the forward's are reused),
 //             split of dT (B), tgemm_kernel (A = C'_alpha: K x channels, B = dT^T) scattering
 //             each used (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
@@ -61,7 +61,6 @@ constexpr int kShareSlices = kMaxShareSlices;  // used K slices per forward shar
 constexpr size_t kPartBudget = (size_t)1 << 30;  // bytes of the forward's partial results per chunk at most
 constexpr int kMaxCtasF = 160;  // CTAs of the forward GEMM at most (its part slots are sized for them)
 constexpr int kEpiCost = 6;     // a forward unit's epilogue, in slices' time, for the forward schedule
-constexpr int kEpiBlocks = 8;   // fwd_epilogue_kernel's blocks per (type, tile)
 constexpr int kMaxKeys = 4096;  // ntypes x nint: each warp's key map (int16) lives in shared memory
 static_assert(kChunkAtoms % kTileAtoms == 0 && kChunkAtoms % 8 == 0, "whole tiles per chunk");
 
@@ -477,7 +476,7 @@ __device__ long long block_scan_1024(long long v, long long *red, long long *tot
 // costs its slice count plus kEpiCost; CTA b takes the cost range [b R, (b + 1) R) of the items' running
 // sum, R = ceil(total / ncta), so that every CTA gets the same work.  An item is cut where a CTA's range
 // begins and every 112 slices (the exactness bound of a share); the pieces of a cut item write their
-// partial results to consecutive part slots, which fwd_epilogue_kernel sums.  One block of 1024 threads,
+// partial results to consecutive part slots, which fwd_finish_kernel sums.  One block of 1024 threads,
 // each over a run of consecutive items.
 __global__ void __launch_bounds__(1024) fwd_schedule_kernel(const int *__restrict__ scount, int64_t nitems,
                                                             int64_t ntiles, int nmt, int ncta, int4 *__restrict__ pieces,
@@ -611,56 +610,66 @@ __global__ void __launch_bounds__(32 * tb::kAtomsB) bwd_units8_kernel(const shor
     units[(size_t)t * maxunits8 + base++] = tb::unit_code((int)tile, 32 * lane + __ffs((int)m) - 1);
 }
 
-// T for the atoms of type t of one 12-atom tile whose items were cut into several pieces, or have no
-// used slices (T = 0): each output's pieces' exact integers added as 128-bit integers and rounded once to
-// f64 (s128_to_f64: no FP64 instruction), read and written with the channels fastest.  kEpiBlocks blocks
-// per (type, tile), each over a share of its 48 columns; a tile whose items each came in one piece was
-// written by the GEMM.
-__global__ void __launch_bounds__(128) fwd_epilogue_kernel(const longlong2 *__restrict__ part, int Mp,
-                                                           const int *__restrict__ eexp,
-                                                           const int *__restrict__ fexp,
-                                                           const int *__restrict__ npieces,
-                                                           const int *__restrict__ pfirst, int64_t ntiles, int nmt,
-                                                           int64_t natoms, int64_t atom0,
-                                                           const int32_t *__restrict__ atype, int ntypes, int M1,
-                                                           double *__restrict__ T) {
-  __shared__ bool wanted[kTileAtoms];
-  const int64_t tt = blockIdx.x / kEpiBlocks;
-  const int part_of = (int)(blockIdx.x - tt * kEpiBlocks);
-  const int t = (int)(tt / ntiles);
-  const int64_t tile = tt - (int64_t)t * ntiles;
-  const int64_t item0 = tt * nmt;
+// The forward's finish, one block per atom of the chunk: T of an atom whose item (its centre type, its
+// tile, a 128-row tile of A) was cut into several pieces -- the pieces' exact integers added as 128-bit
+// integers and rounded once to f64 (s128_to_f64: no FP64 instruction) -- or has no used slices (T = 0);
+// the other atoms' T the GEMM wrote.  Then, when D is wanted, the atom's descriptor D[m][n] =
+// sum_k T[k][m] T[k][n] (n < M2) from its T staged in shared memory, in descriptor_kernel's order of
+// operations, so that the two give the same bits.
+__global__ void __launch_bounds__(128) fwd_finish_kernel(const longlong2 *__restrict__ part, int Mp,
+                                                         const int *__restrict__ eexp, const int *__restrict__ fexp,
+                                                         const int *__restrict__ npieces,
+                                                         const int *__restrict__ pfirst, int64_t ntiles, int nmt,
+                                                         int64_t atom0, const int32_t *__restrict__ atype,
+                                                         int ntypes, int M1, double *__restrict__ T, int M2,
+                                                         double *__restrict__ D) {
+  extern __shared__ double Ts[];  // [4][M1], when D is wanted
+  const int64_t a = blockIdx.x;
+  const int64_t tile = a / kTileAtoms;
+  const int al = (int)(a - tile * kTileAtoms);
+  const int t = atype ? clampi(atype[atom0 + a], 0, ntypes - 1) : 0;
+  const int64_t item0 = ((int64_t)t * ntiles + tile) * nmt;
   bool direct = true;
   for (int mt = 0; mt < nmt; ++mt) direct = direct && npieces[item0 + mt] == 1;
-  if (direct) return;  // uniform
-  if (threadIdx.x < kTileAtoms) {
-    const int64_t a = tile * kTileAtoms + threadIdx.x;
-    wanted[threadIdx.x] = a < natoms && (!atype || clampi(atype[atom0 + a], 0, ntypes - 1) == t);
-  }
-  __syncthreads();
-  constexpr int kColsPer = kTN / kEpiBlocks;
-  static_assert(kTN % kEpiBlocks == 0, "whole columns per block");
-  for (int e = threadIdx.x; e < kColsPer * M1; e += blockDim.x) {
-    const int col = part_of * kColsPer + e / M1, m = e - (e / M1) * M1;
-    if (!wanted[col >> 2]) continue;
-    const int np = npieces[item0 + m / kTM], first = pfirst[item0 + m / kTM];
-    if (np == 1) continue;  // these channels were written by the GEMM
-    long long hi = 0;
-    unsigned long long lo = 0;
-    bool nan = false;
-    for (int z = 0; z < np; ++z) {  // an atom of a tile without used slices has no valid rows: T = 0
-      const longlong2 x = part[((size_t)(first + z) * kTN + col) * Mp + m];
-      const unsigned long long l = lo + (unsigned long long)x.x;
-      hi += x.y + (l < lo ? 1 : 0);
-      lo = l;
-      nan = nan || x.y == tg::kPartNaN;
+  if (direct && !D) return;  // uniform
+  double *Ta = T + (atom0 + a) * kCols * M1;
+  for (int e = threadIdx.x; e < kCols * M1; e += blockDim.x) {
+    const int k = e / M1, m = e - k * M1, col = al * kCols + k;
+    const int np = npieces[item0 + m / kTM];
+    double v;
+    if (np == 1) {
+      v = Ta[e];  // written by the GEMM (read only for D)
+    } else {
+      const int first = pfirst[item0 + m / kTM];
+      long long hi = 0;
+      unsigned long long lo = 0;
+      bool nan = false;
+      for (int z = 0; z < np; ++z) {  // np == 0: a tile without used slices, whose atoms have no valid rows
+        const longlong2 x = part[((size_t)(first + z) * kTN + col) * Mp + m];
+        const unsigned long long l = lo + (unsigned long long)x.x;
+        hi += x.y + (l < lo ? 1 : 0);
+        lo = l;
+        nan = nan || x.y == tg::kPartNaN;
+      }
+      bool rare = false;
+      const int E = eexp[(size_t)t * Mp + m], F = fexp[tile * kTN + col];
+      v = s128_to_f64<kOutExp>(hi, lo, E, F, rare);
+      if (rare) v = output_value((__int128)(((unsigned __int128)(unsigned long long)hi << 64) | lo), E, F);
+      if (nan) v = __longlong_as_double(0x7ff8000000000000ll);
+      Ta[e] = v;
     }
-    bool rare = false;
-    const int E = eexp[(size_t)t * Mp + m], F = fexp[tile * kTN + col];
-    double v = s128_to_f64<kOutExp>(hi, lo, E, F, rare);
-    if (rare) v = output_value((__int128)(((unsigned __int128)(unsigned long long)hi << 64) | lo), E, F);
-    const int64_t a = tile * kTileAtoms + (col >> 2);
-    T[((atom0 + a) * kCols + (col & 3)) * M1 + m] = nan ? __longlong_as_double(0x7ff8000000000000ll) : v;
+    if (D) Ts[e] = v;
+  }
+  if (!D) return;  // uniform
+  __syncthreads();
+  double *Da = D + (atom0 + a) * (int64_t)M1 * M2;
+  for (int e = threadIdx.x; e < M1 * M2; e += blockDim.x) {
+    const int m = e / M2, n = e - m * M2;
+    double v = Ts[m] * Ts[n];
+    v = fma(Ts[M1 + m], Ts[M1 + n], v);
+    v = fma(Ts[2 * M1 + m], Ts[2 * M1 + n], v);
+    v = fma(Ts[3 * M1 + m], Ts[3 * M1 + n], v);
+    Da[e] = v;
   }
 }
 
@@ -863,14 +872,15 @@ int tc_args(const dp_tc_plan *plan, const dp_table_info *info, const double *s, 
 }
 
 int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
-        const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, double *T, void *work,
-        size_t work_bytes, void *stream) {
+        const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, double *T, int M2,
+        double *D, void *work, size_t work_bytes, void *stream) {
   clear_error();
   static const char *who = "dp_tabulate_fusion_fwd_tc_f64";
   TableGeom g;
   Segments seg;
   Shape S{};
   Layout L{};
+  if (D && (M2 < 1 || M2 > M1)) return set_error(DP_ERR_SHAPE, "%s: M2 %d not in 1 .. M1 = %d", who, M2, M1);
   int rc = tc_args(plan, info, s, Rt, nloc, nnei, ntypes, sel, M1, T, T, work, work_bytes, &g, &seg, &S, &L, who);
   if (rc || nloc == 0) return rc;
   const PlanLayout PL = plan_layout(S);
@@ -940,12 +950,11 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
     G.ntypes = ntypes;
     if ((rc = tg::launch(G, st, who, ncta))) return rc;
     prof_mark("tc_gemm_fwd", st);
-    fwd_epilogue_kernel<<<(unsigned)(nlist * kEpiBlocks), 128, 0, st>>>(part, S.Mpf, G.Eexp, R.fexp,
-                                                         reinterpret_cast<const int *>(wk + L.npieces),
-                                                         reinterpret_cast<const int *>(wk + L.pfirst), ntiles, nmt, n, c0,
-                                                         atype, ntypes, M1, T);
+    fwd_finish_kernel<<<(unsigned)n, 128, D ? (size_t)kCols * M1 * sizeof(double) : 0, st>>>(
+        part, S.Mpf, G.Eexp, R.fexp, reinterpret_cast<const int *>(wk + L.npieces),
+        reinterpret_cast<const int *>(wk + L.pfirst), ntiles, nmt, c0, atype, ntypes, M1, T, M2, D);
     if ((rc = launch_status(who))) return rc;
-    prof_mark("tc_epilogue_fwd", st);
+    prof_mark("tc_finish_fwd", st);
   }
   return DP_OK;
 }
@@ -1143,9 +1152,10 @@ int dp_tabulate_tc_plan_f64(const double *table, const dp_table_info *info, int 
 
 int dp_tabulate_fusion_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
                                   const int32_t *nvalid, const int32_t *atype, int64_t nloc, int nnei, int ntypes,
-                                  const int32_t *sel, int M1, double *T, void *work, size_t work_bytes,
-                                  void *stream) {
-  return dpc::tt::fwd(plan, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, work, work_bytes, stream);
+                                  const int32_t *sel, int M1, double *T, int M2, double *D, void *work,
+                                  size_t work_bytes, void *stream) {
+  return dpc::tt::fwd(plan, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, M2, D, work, work_bytes,
+                      stream);
 }
 
 int dp_tabulate_fusion_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,

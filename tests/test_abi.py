@@ -153,9 +153,9 @@ def test_tc_plan_and_work_validation_without_gpu(dpc):
         d.update(kw)
         return dpc.dp_tc_plan(**d)
 
-    def fwd(rec, work=fake, nbytes=wb):
+    def fwd(rec, work=fake, nbytes=wb, M2=0, D=None):
         return lib.dp_tabulate_fusion_fwd_tc_f64(None if rec is None else ctypes.byref(rec), ctypes.byref(info), fake,
-                                                 fake, None, None, 5, 8, 1, sel, 16, fake, work, nbytes, None)
+                                                 fake, None, None, 5, 8, 1, sel, 16, fake, M2, D, work, nbytes, None)
 
     def grad(rec, flags=0, work=fake, nbytes=wb):
         return lib.dp_tabulate_fusion_grad_tc_f64(None if rec is None else ctypes.byref(rec), ctypes.byref(info),
@@ -171,6 +171,8 @@ def test_tc_plan_and_work_validation_without_gpu(dpc):
     assert fwd(plan(), nbytes=wb - 1) == dpc.DP_ERR_SHAPE
     assert fwd(plan(), work=ctypes.c_void_p(0x1010)) == dpc.DP_ERR_SHAPE
     assert grad(plan(), flags=2) == dpc.DP_ERR_SHAPE and "flags" in dpc.dp_last_error()
+    for bad_m2 in (0, 17):  # the descriptor's M2 outside 1 .. M1 (16), refused on the host
+        assert fwd(plan(), M2=bad_m2, D=fake) == dpc.DP_ERR_SHAPE and "M2" in dpc.dp_last_error()
     rec = dpc.dp_tc_plan()
     build = lambda buf, n: lib.dp_tabulate_tc_plan_f64(fake, ctypes.byref(info), 8, 1, 16, buf, n,  # noqa: E731
                                                        ctypes.byref(rec), None)

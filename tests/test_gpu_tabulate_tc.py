@@ -23,9 +23,9 @@ def _gpu():
 
 
 def _tc(w, model=None, x=None, nvalid="w", atype="w", work=None, out=None, grad_out=None, reuse=False, plan=None):
-    """Forward then backward on the tensor-core path; reuse: the backward takes the forward's interval runs
-    from the shared work buffer (the benchmark's configuration); plan: a TcPlan, else the table is planned
-    per call."""
+    """Forward (writing D as well) then backward on the tensor-core path; reuse: the backward takes the
+    forward's interval runs from the shared work buffer (the benchmark's configuration); plan: a TcPlan,
+    else the table is planned per call."""
     dpc = lib()
     model = model or product_model(w, F64)
     x = x or to_dev(w, F64)
@@ -35,12 +35,15 @@ def _tc(w, model=None, x=None, nvalid="w", atype="w", work=None, out=None, grad_
     if reuse and work is None:
         need = dpc.dp_tabulate_tc_work_bytes(model.info, w.nloc, w.nnei, w.ntypes, w.M1)
         work = torch.empty((need,), dtype=torch.uint8, device="cuda")
-    T = dpc.dp_tabulate_fusion_fwd_tc_f64(tab, model.info, x["s"], x["Rt"], nv, at, w.sel, out=out, work=work)
+    T, D = dpc.dp_tabulate_fusion_fwd_tc_f64(tab, model.info, x["s"], x["Rt"], nv, at, w.sel, out=out, work=work,
+                                             M2=w.M2)
     ds, dRt = dpc.dp_tabulate_fusion_grad_tc_f64(tab, model.info, x["s"], x["Rt"], nv, at, w.sel, x["dT"],
                                                  out=grad_out, work=work,
                                                  flags=dpc.DP_TC_REUSE_RUNS if reuse else 0)
+    Dc = dpc.dp_descriptor_contract(T, w.M2)  # the same T contracted by the separate call
     torch.cuda.synchronize()
-    return dict(T=T.cpu().numpy(), ds=ds.cpu().numpy(), dRt=dRt.cpu().numpy())
+    assert torch.equal(D.view(torch.int64), Dc.view(torch.int64)), "the forward's D differs from dp_descriptor_contract"
+    return dict(T=T.cpu().numpy(), D=D.cpu().numpy(), ds=ds.cpu().numpy(), dRt=dRt.cpu().numpy())
 
 
 def _pipe(w, model, x):
@@ -64,9 +67,10 @@ CHUNK = 16416  # atoms per chunk of the tensor-core calls (their work buffer hol
 
 @pytest.mark.parametrize("name,kw,nsample", CASES, ids=[f"{c[0]}-{c[1]}" for c in CASES])
 def test_tc_against_oracle_and_fp64_path(name, kw, nsample):
-    """T, ds and dR~ in the benchmark's configuration (a plan made once, the backward reusing the forward's
-    interval runs) against the oracle (sampled atoms at the largest sizes) and against the FP64-pipe moment
-    kernels on every atom; bit-identical to a backward that finds the runs itself."""
+    """T, D (written by the forward), ds and dR~ in the benchmark's configuration (a plan made once, the
+    backward reusing the forward's interval runs) against the oracle (sampled atoms at the largest sizes)
+    and against the FP64-pipe moment kernels on every atom; bit-identical to a backward that finds the runs
+    itself, and D to dp_descriptor_contract of the same T."""
     w = workload(name, **kw)
     model = product_model(w, F64)
     x = to_dev(w, F64)
@@ -80,7 +84,7 @@ def test_tc_against_oracle_and_fp64_path(name, kw, nsample):
         atoms = np.sort(np.random.default_rng(5).choice(w.nloc, nsample, replace=False))
         atoms[0], atoms[-1] = 0, w.nloc - 1
     ref = run_oracle(w, F64, atoms=atoms)
-    assert_parity(got, ref, F64, atoms=atoms, keys=("T", "ds", "dRt"))
+    assert_parity(got, ref, F64, atoms=atoms, keys=("T", "D", "ds", "dRt"))
     pipe = _pipe(w, model, x)
     for k in ("T", "ds", "dRt"):
         assert rel(got[k], pipe[k]) <= CLOSE, (k, rel(got[k], pipe[k]))
