@@ -412,8 +412,11 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     outs = dict(D=D, F=torch.empty((coord.shape[0], 3), dtype=dtype, device=dev),
                 virial=torch.empty((3, 3), dtype=dtype, device=dev))
     names = ["env_mat", "fwd", "descriptor", "descriptor_grad", "grad", "force_virial"]
+    fused_env = fused_d and not args.unfused  # rows formed and forces added inside the tensor-core calls
     if fused_d:
         names.remove("descriptor")
+    if fused_env:
+        names = [n for n in names if n not in ("env_mat", "force_virial")]
     if args.fitting:
         H = sum(fwidths[1:-1])
         outs["E"] = torch.empty((w.nloc,), dtype=dtype, device=dev)
@@ -427,13 +430,21 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
                  "force_virial"]
         if fused_d:
             names.remove("descriptor")
+        if fused_env:
+            names = [n for n in names if n not in ("env_mat", "force_virial")]
 
     def step(rec, x, o):
         k = 0
         rec(k)
-        dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]), arith=arith)
-        rec(k := k + 1)
-        if fused_d:
+        if fused_env:  # coordinates -> T, D (and the valid-row counts) in one call
+            dpc.dp_tabulate_fusion_env_fwd_tc_f64(plan, info, x["coord"], x["nlist"], sel, env, x["atype"],
+                                                  out=work["T"], work=tcw, M2=w.M2, D=o["D"], nvalid=work["nvalid"])
+        else:
+            dpc.dp_env_mat(x["coord"], x["nlist"], sel, env, out=(work["s"], work["Rt"], work["nvalid"]), arith=arith)
+            rec(k := k + 1)
+        if fused_env:
+            pass
+        elif fused_d:
             fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"], D=o["D"])
         else:
             fwd(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, out=work["T"])
@@ -457,6 +468,11 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
             dD_in = x["dD"]
         dpc.dp_descriptor_contract_grad(work["T"], dD_in, out=work["dT"], arith=arith)
         rec(k := k + 1)
+        if fused_env:  # dE/dT -> forces and virial in one call, on the forward's interval runs
+            dpc.dp_tabulate_fusion_env_grad_tc_f64(plan, info, x["coord"], x["nlist"], sel, env, x["atype"], work["dT"],
+                                                   out=(o["F"], o["virial"]), work=tcw, flags=dpc.DP_TC_REUSE_RUNS)
+            rec(k := k + 1)
+            return
         grad(model.table, info, work["s"], work["Rt"], work["nvalid"], x["atype"], sel, work["dT"],
              out=(work["ds"], work["dRt"]))
         rec(k := k + 1)
@@ -937,6 +953,9 @@ def main():
     ap.add_argument("--no-graph", action="store_true", help="with --chain: skip the CUDA-graph replay timing")
     ap.add_argument("--no-variants", action="store_true",
                     help="skip the per-row and df64 timings added to the default f64 line")
+    ap.add_argument("--unfused", action="store_true",
+                    help="with --chain --algo tc: the front and back end as separate kernels (dp_env_mat, "
+                         "dp_force_virial) instead of fused into the tensor-core calls")
     ap.add_argument("--chain", action="store_true",
                     help="time the whole chain from coordinates to forces (env_mat ... force_virial)")
     ap.add_argument("--fitting", action="store_true",

@@ -328,6 +328,38 @@ int dp_tabulate_fusion_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *
                                    size_t work_bytes, int flags, void *stream);
 
 /*
+ * The same two calls with the environment matrix's front end and the force
+ * back end fused in (Sec. II: s(r), the rows R~ and their normalisation;
+ * the forces and virial by the chain rule), so that s, R~, ds and dR~ never
+ * reach memory.  The rows are formed from coord [nall][3] and the neighbour
+ * list nlist [nloc][nnei] (each type segment's neighbours first, -1 after)
+ * exactly as dp_env_mat_f64 forms them, with the same env; the forward then
+ * writes T (and D when D is not NULL, as dp_tabulate_fusion_fwd_tc_f64) and,
+ * when nvalid is not NULL, the counts of rows with a neighbour [nloc][ntypes]
+ * as dp_env_mat_f64 does.  The backward takes dT and adds what
+ * dp_force_virial_f64 would add from the ds and dR~ that
+ * dp_tabulate_fusion_grad_tc_f64 would write: F [nall][3] and virial [9],
+ * both zeroed first (F holds the forces on the local atoms and the
+ * reactions on the neighbours, ghosts included), up to the order of the
+ * floating-point additions.  plan, work and flags as for the unfused calls
+ * (DP_TC_REUSE_RUNS: the fused forward ran on the same plan, coord, nlist,
+ * env, atype, nloc and work buffer).  Extra errors: DP_ERR_NULL for a missing
+ * env, coord, nlist, F or virial; DP_ERR_TABLE_INFO for env out of range
+ * (as dp_env_mat_f64); DP_ERR_SHAPE for nall < nloc.
+ */
+struct dp_env_info; /* defined with dp_env_mat_f64 below */
+int dp_tabulate_fusion_env_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *coord,
+                                      const int32_t *nlist, const struct dp_env_info *env, const int32_t *atype,
+                                      int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1,
+                                      int32_t *nvalid, double *T, int M2, double *D, void *work, size_t work_bytes,
+                                      void *stream);
+int dp_tabulate_fusion_env_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *coord,
+                                       const int32_t *nlist, const struct dp_env_info *env, const int32_t *atype,
+                                       int64_t nloc, int64_t nall, int nnei, int ntypes, const int32_t *sel, int M1,
+                                       const double *dT, double *F, double *virial, void *work, size_t work_bytes,
+                                       int flags, void *stream);
+
+/*
  * Kernel timing hook, for profiling (off by default; not thread-safe: one
  * profiling session per process).  dp_profile_begin hands the library n
  * caller-created cudaEvent_t handles (as void*, created with timing enabled,

@@ -118,6 +118,12 @@ _SIGS = {
                                         ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t, ctypes.c_int, _P],
                                        ctypes.c_int),
     "dp_env_mat_f64": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
+    "dp_tabulate_fusion_env_fwd_tc_f64": ([_PLAN, _INFO, _P, _P, _ENV, _P, _I64, ctypes.c_int, ctypes.c_int, _P,
+                                           ctypes.c_int, _P, _P, ctypes.c_int, _P, _P, ctypes.c_size_t, _P],
+                                          ctypes.c_int),
+    "dp_tabulate_fusion_env_grad_tc_f64": ([_PLAN, _INFO, _P, _P, _ENV, _P, _I64, _I64, ctypes.c_int, ctypes.c_int,
+                                            _P, ctypes.c_int, _P, _P, _P, _P, ctypes.c_size_t, ctypes.c_int, _P],
+                                           ctypes.c_int),
     "dp_env_mat_f32": ([_P, _P, _I64, ctypes.c_int, ctypes.c_int, _P, _ENV, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_f64": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_force_virial_f32": ([_P, _P, _I64, _I64, ctypes.c_int, _ENV, _P, _P, _P, _P, _P], ctypes.c_int),
@@ -502,6 +508,70 @@ def dp_tabulate_fusion_grad_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, aty
                                                _ptr(ds), _ptr(dRt), _ptr(work), work.numel(), int(flags),
                                                _stream(s)))
     return ds, dRt
+
+
+def _env_tc_inputs(plan, info, coord, nlist, sel, atype):
+    """The fused calls' checked arrays and plan (a TcPlan, or one made now from an f64 table)."""
+    coord = _dev(coord, "coord", torch.float64)
+    if coord.dim() != 2 or coord.shape[1] != 3:
+        raise ValueError("coord must be [nall][3]")
+    nlist = _dev(nlist, "nlist", torch.int32)
+    nloc, nnei = (int(x) for x in nlist.shape)
+    selc, ntypes, nsum = _sel_arr(sel)
+    if nsum != nnei:
+        raise ValueError(f"sum(sel) = {nsum} != nnei = {nnei}")
+    atype = None if atype is None else _dev(atype, "atype", torch.int32, (nloc,))
+    if not isinstance(plan, TcPlan):
+        plan = dp_tabulate_tc_plan_f64(_dev(plan, "table", torch.float64), info, nnei, ntypes)
+    return plan, coord, nlist, atype, selc, ntypes, nloc, nnei, int(plan.rec.M1)
+
+
+def dp_tabulate_fusion_env_fwd_tc_f64(plan, info: dp_table_info, coord, nlist, sel, env: dp_env_info, atype=None,
+                                      out=None, work=None, M2=None, D=None, nvalid=None):
+    """(T, D, nvalid) of dp_env_mat followed by dp_tabulate_fusion_fwd_tc_f64, in one pass that forms the rows
+    from coord [nall][3] and nlist [nloc][nnei] itself (s and R~ never reach memory); D is None unless M2 is
+    given.  plan and work as dp_tabulate_fusion_fwd_tc_f64."""
+    plan, coord, nlist, atype, selc, ntypes, nloc, nnei, M1 = _env_tc_inputs(plan, info, coord, nlist, sel, atype)
+    T = torch.empty((nloc, 4, M1), dtype=torch.float64, device=coord.device) if out is None else \
+        _dev(out, "out", torch.float64, (nloc, 4, M1))
+    if M2 is not None:
+        dshape = (nloc, M1, int(M2))
+        D = torch.empty(dshape, dtype=torch.float64, device=coord.device) if D is None else \
+            _dev(D, "D", torch.float64, dshape)
+    nvalid = torch.empty((nloc, ntypes), dtype=torch.int32, device=coord.device) if nvalid is None else \
+        _dev(nvalid, "nvalid", torch.int32, (nloc, ntypes))
+    if nloc == 0:
+        return T, D, nvalid
+    work = _tab_tc_work(work, info, nloc, nnei, ntypes, M1, coord.device)
+    _check(_lib.dp_tabulate_fusion_env_fwd_tc_f64(ctypes.byref(plan.rec), ctypes.byref(info), _ptr(coord), _ptr(nlist),
+                                                  ctypes.byref(env), _ptr(atype), nloc, nnei, ntypes, selc, M1,
+                                                  _ptr(nvalid), _ptr(T), 0 if M2 is None else int(M2),
+                                                  None if M2 is None else _ptr(D), _ptr(work), work.numel(),
+                                                  _stream(coord)))
+    return T, D, nvalid
+
+
+def dp_tabulate_fusion_env_grad_tc_f64(plan, info: dp_table_info, coord, nlist, sel, env: dp_env_info, atype, dT,
+                                       out=None, work=None, flags=0):
+    """(F [nall][3], virial [3][3]) of dp_tabulate_fusion_grad_tc_f64 followed by dp_force_virial, in one pass
+    from coordinates (s, R~, ds and dR~ never reach memory).  plan, work and flags as
+    dp_tabulate_fusion_grad_tc_f64 (DP_TC_REUSE_RUNS after dp_tabulate_fusion_env_fwd_tc_f64 on the same
+    inputs and work buffer)."""
+    plan, coord, nlist, atype, selc, ntypes, nloc, nnei, M1 = _env_tc_inputs(plan, info, coord, nlist, sel, atype)
+    nall = int(coord.shape[0])
+    dT = _dev(dT, "dT", torch.float64, (nloc, 4, M1))
+    if out is None:
+        F = torch.empty((nall, 3), dtype=torch.float64, device=coord.device)
+        W = torch.empty((3, 3), dtype=torch.float64, device=coord.device)
+    else:
+        F = _dev(out[0], "F", torch.float64, (nall, 3))
+        W = _dev(out[1], "virial", torch.float64, (3, 3))
+    work = _tab_tc_work(work, info, max(nloc, 1), nnei, ntypes, M1, coord.device)
+    _check(_lib.dp_tabulate_fusion_env_grad_tc_f64(ctypes.byref(plan.rec), ctypes.byref(info), _ptr(coord),
+                                                   _ptr(nlist), ctypes.byref(env), _ptr(atype), nloc, nall, nnei,
+                                                   ntypes, selc, M1, _ptr(dT), _ptr(F), _ptr(W), _ptr(work),
+                                                   work.numel(), int(flags), _stream(coord)))
+    return F, W
 
 
 def dp_env_mat(coord, nlist, sel, env: dp_env_info, out=None, arith=None):

@@ -44,6 +44,7 @@
 #include <cstdint>
 
 #include "dp_common.cuh"
+#include "env_row.cuh"
 #include "tab_gemm.cuh"
 #include "tab_gemm_b8.cuh"
 #include "tc_gemm.cuh"
@@ -256,8 +257,73 @@ __device__ __forceinline__ int locate_fast(const TableGeom &g, const TableGeomF 
   return l;
 }
 
+// The environment matrix's inputs, where the tensor-core path forms its rows from coordinates itself
+// (dp_tabulate_fusion_env_*_tc_f64: s and R~ never reach HBM, nor ds and dR~ in the backward).
+struct EnvRow {
+  const double *coord;   // [nall][3]
+  const int32_t *nlist;  // [nloc][nnei]: the neighbour's index into coord, or -1 (each segment's first)
+  double rcs, rc, inv_width, mean, inv_std, inv_std_all;
+  int kind;
+};
+
+// Row (i, j) as dp_env_mat forms it, by the same operations: d = x_j - x_i, r, 1/r, s(r) and ds/dr, the
+// table input and R~[0] sh = (s - mean)/std, and R~[1 .. 3] = s d / (r std_all).
+struct EnvVals {
+  double d[3], inv_r, sv, dsv, r4[4];
+};
+__device__ __forceinline__ EnvVals env_vals(const EnvRow &E, int64_t i, int j) {
+  EnvVals v;
+  const double xi = E.coord[3 * i], yi = E.coord[3 * i + 1], zi = E.coord[3 * i + 2];
+  v.d[0] = E.coord[3 * (int64_t)j] - xi;
+  v.d[1] = E.coord[3 * (int64_t)j + 1] - yi;
+  v.d[2] = E.coord[3 * (int64_t)j + 2] - zi;
+  const double r2 = fma(v.d[0], v.d[0], fma(v.d[1], v.d[1], v.d[2] * v.d[2]));
+  const double r = sqrt(r2);
+  v.inv_r = recip(r);
+  weight(E, r, v.inv_r, v.sv, v.dsv);
+  const double a = v.sv * v.inv_r * E.inv_std_all;
+  v.r4[0] = (v.sv - E.mean) * E.inv_std;
+  v.r4[1] = a * v.d[0];
+  v.r4[2] = a * v.d[1];
+  v.r4[3] = a * v.d[2];
+  return v;
+}
+
+// Valid rows per type segment of atom i from its neighbour list (the rows with a neighbour, each
+// segment's first, as dp_env_mat counts them) into nvb, and into nvalid_out when given; their total.
+__device__ __forceinline__ int env_valid_rows(const EnvRow &E, int nnei, const int *sel, int ntypes, int64_t i,
+                                              int lane, int *nvb, int32_t *nvalid_out) {
+  int count = 0;  // lane b < ntypes: segment b's rows with a neighbour
+  for (int q0 = 0; q0 < nnei; q0 += 32) {  // uniform
+    const int q = q0 + lane;
+    const int j = q < nnei ? __ldg(E.nlist + i * nnei + q) : -1;
+    int b = 0, lim = sel[0];
+#pragma unroll
+    for (int c = 1; c < DP_MAX_TYPES; ++c)
+      if (c < ntypes && q >= lim) {
+        b = c;
+        lim += sel[c];
+      }
+#pragma unroll
+    for (int c = 0; c < DP_MAX_TYPES; ++c) {
+      if (c >= ntypes) break;  // uniform
+      const int n = __popc(__ballot_sync(0xffffffffu, j >= 0 && b == c));
+      if (lane == c) count += n;
+    }
+  }
+  if (lane < DP_MAX_TYPES) nvb[lane] = lane < ntypes ? count : 0;
+  if (nvalid_out && lane < ntypes) nvalid_out[i * ntypes + lane] = count;
+  __syncwarp();
+  int nv = 0;
+#pragma unroll
+  for (int q = 0; q < DP_MAX_TYPES; ++q) nv += nvb[q];
+  return nv;
+}
+
 struct RunsParams {
   const double *s, *Rt;
+  EnvRow env;           // kEnv: rows from coordinates (s and Rt unused)
+  int32_t *nvalid_out;  // kEnv forward: the counts of valid rows it finds
   const int32_t *nvalid, *atype;
   TableGeom g;
   TableGeomF gf;
@@ -321,7 +387,7 @@ __device__ __forceinline__ int valid_row(int v, const int *nvb, const int *sel, 
 // thousands of tiny blocks does not set the pace of a short kernel.
 constexpr int kRunsWarps = 4, kRowsWarps = 4;
 
-template <bool kMom>
+template <bool kMom, bool kEnv = false>
 __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams P) {
   __shared__ RunsStage stw[kRunsWarps];
   extern __shared__ short smapw[];  // [kRunsWarps][nkeys]
@@ -332,7 +398,8 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
   short *smap = smapw + (size_t)warp * P.nkeys;
   const int64_t i = P.atom0 + a;
   for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
-  const int nv = valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (its __syncwarp orders the reset)
+  const int nv = kEnv ? env_valid_rows(P.env, P.nnei, P.sel, P.ntypes, i, lane, st.nvb, P.nvalid_out)
+                      : valid_rows(P.nvalid, P.sel, P.ntypes, i, lane, st.nvb);  // (their __syncwarp orders the reset)
   const int alpha = P.atype ? clampi(__ldg(P.atype + i), 0, P.ntypes - 1) : 0;
   unsigned char *occ = P.occ + ((size_t)alpha * P.tiles_all + (size_t)(i / kTileAtoms)) * P.nsl;
   short *keys = P.keys + i * P.cap;
@@ -369,12 +436,24 @@ __global__ void __launch_bounds__(32 * kRunsWarps) runs_kernel(const RunsParams 
     if (v < nv) {
       int b;
       const int row = valid_row(v, st.nvb, P.sel, P.ntypes, b);
-      double t;
+      double t, sv, r4[4];
+      if constexpr (kEnv) {
+        const EnvVals ev = env_vals(P.env, i, __ldg(P.env.nlist + i * P.nnei + row));
+        sv = ev.r4[0];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) r4[k] = ev.r4[k];
+      } else {
+        sv = __ldg(srow + row);
+      }
       bool clamped;
-      const int l = locate_fast(P.g, P.gf, P.nodes, __ldg(srow + row), t, clamped);
+      const int l = locate_fast(P.g, P.gf, P.nodes, sv, t, clamped);
       st.key[lane] = b * P.g.nint + l;
       if constexpr (kMom) {
-        const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
+        Vec4<double> rr;
+        if constexpr (kEnv)
+          rr = Vec4<double>{r4[0], r4[1], r4[2], r4[3]};
+        else
+          rr = ld4(Rrow + (size_t)row * 4);
         st.r[lane][0] = rr.x;
         st.r[lane][1] = rr.y;
         st.r[lane][2] = rr.z;
@@ -687,6 +766,8 @@ struct RowsParams {
   const double *dW;    // [natoms][cap][24]: the backward GEMM's result per slot, dW[k][q] at 6 k + q
   double *ds, *dRt;
   int64_t natoms;
+  EnvRow env;             // rows_force_kernel: rows from coordinates,
+  double *F, *virial;     // and the forces [nall][3] and virial [9] they add to
 };
 
 // One warp per atom, a lane per valid row: the row's interval from s, its run slot from the atom's key map
@@ -749,6 +830,92 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
       st4(drow + (size_t)(off + j) * 4, 0.0, 0.0, 0.0, 0.0);
     }
     off += P.sel[b];
+  }
+}
+
+// rows_kernel fused with the environment and the force back end (dp_tabulate_fusion_env_grad_tc_f64): a
+// lane per valid row forms the row from coordinates (env_vals, as dp_env_mat), its dE/ds and dE/dR~ as
+// rows_kernel does, and from them, in registers, the row's force contribution g = dE/d(x_j - x_i) by
+// dp_force_virial's arithmetic: F_i += g, F_j -= g (atomics), virial -= d (x) g; s, R~, ds and dR~ never
+// reach memory.  The per-atom sums are reduced over the warp and added once.
+__global__ void __launch_bounds__(32 * kRowsWarps) rows_force_kernel(const RowsParams P) {
+  __shared__ int nvbw[kRowsWarps][DP_MAX_TYPES];
+  extern __shared__ short smapw[];  // [kRowsWarps][nkeys]
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int64_t a = (int64_t)blockIdx.x * kRowsWarps + warp;
+  if (a >= P.natoms) return;  // warp-uniform
+  int *nvb = nvbw[warp];
+  short *smap = smapw + (size_t)warp * P.nkeys;
+  const int64_t i = P.atom0 + a;
+  const short *keys = P.keys + i * P.cap;
+  const int nslot = P.nslots[i];
+  for (int k = lane; k < P.nkeys; k += 32) smap[k] = -1;
+  __syncwarp();
+  for (int x = lane; x < nslot; x += 32) smap[keys[x]] = (short)x;  // the map of the atom's keys
+  const int nv = env_valid_rows(P.env, P.nnei, P.sel, P.ntypes, i, lane, nvb, nullptr);  // (orders the map)
+  const double *dWa = P.dW + (size_t)a * P.cap * 24;
+  double f[3] = {0.0, 0.0, 0.0}, w[9];
+#pragma unroll
+  for (int x = 0; x < 9; ++x) w[x] = 0.0;
+  for (int v = lane; v < nv; v += 32) {
+    int b;
+    const int row = valid_row(v, nvb, P.sel, P.ntypes, b);
+    const int j = __ldg(P.env.nlist + i * P.nnei + row);
+    const EnvVals ev = env_vals(P.env, i, j);
+    double t;
+    bool clamped;
+    const int l = locate_fast(P.g, P.gf, P.nodes, ev.r4[0], t, clamped);
+    const double dinv = l < P.g.n0 ? P.g.inv0 : P.g.inv1;
+    const double u = t * dinv;
+    const double2 *dw = reinterpret_cast<const double2 *>(dWa + (size_t)smap[b * P.g.nint + l] * 24);
+    double d4[4], ds = 0.0;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {  // as rows_kernel
+      const double2 c01 = __ldg(dw + 3 * k), c23 = __ldg(dw + 3 * k + 1), c45 = __ldg(dw + 3 * k + 2);
+      double p = fma(c45.y, u, c45.x), dp = c45.y;
+      dp = fma(dp, u, p);
+      p = fma(p, u, c23.y);
+      dp = fma(dp, u, p);
+      p = fma(p, u, c23.x);
+      dp = fma(dp, u, p);
+      p = fma(p, u, c01.y);
+      dp = fma(dp, u, p);
+      d4[k] = fma(p, u, c01.x);
+      ds = fma(ev.r4[k], dp, ds);
+    }
+    ds = clamped ? 0.0 : ds * dinv;
+    // as dp_force_virial: the s column feeds both the table input and R~[0]
+    const double g0 = ds + d4[0];
+    const double p = fma(d4[1], ev.d[0], fma(d4[2], ev.d[1], d4[3] * ev.d[2]));
+    const double cd = fma(g0 * ev.dsv, ev.inv_r * P.env.inv_std,
+                          (ev.dsv - ev.sv * ev.inv_r) * ev.inv_r * ev.inv_r * p * P.env.inv_std_all);
+    const double ce = ev.sv * ev.inv_r * P.env.inv_std_all;
+    const double g[3] = {fma(cd, ev.d[0], ce * d4[1]), fma(cd, ev.d[1], ce * d4[2]), fma(cd, ev.d[2], ce * d4[3])};
+#pragma unroll
+    for (int c = 0; c < 3; ++c) {
+      f[c] += g[c];
+      atomicAdd(P.F + 3 * (int64_t)j + c, -g[c]);
+    }
+#pragma unroll
+    for (int x = 0; x < 3; ++x)
+#pragma unroll
+      for (int y = 0; y < 3; ++y) w[3 * x + y] = fma(-ev.d[x], g[y], w[3 * x + y]);
+  }
+#pragma unroll
+  for (int c = 0; c < 3; ++c)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) f[c] += __shfl_xor_sync(0xffffffffu, f[c], o);
+#pragma unroll
+  for (int x = 0; x < 9; ++x)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) w[x] += __shfl_xor_sync(0xffffffffu, w[x], o);
+  if (lane < 3) atomicAdd(P.F + 3 * i + lane, lane == 0 ? f[0] : lane == 1 ? f[1] : f[2]);
+  if (lane < 9) {
+    double vv = w[0];
+#pragma unroll
+    for (int x = 1; x < 9; ++x)
+      if (lane == x) vv = w[x];
+    atomicAdd(P.virial + lane, vv);
   }
 }
 
@@ -871,11 +1038,13 @@ int tc_args(const dp_tc_plan *plan, const dp_table_info *info, const double *s, 
   return tg::set_smem(who);
 }
 
+// env: the rows come from coordinates (dp_tabulate_fusion_env_fwd_tc_f64; s, Rt and nvalid unused, the
+// counts of valid rows written to nvalid_out when given).
 int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
         const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, double *T, int M2,
-        double *D, void *work, size_t work_bytes, void *stream) {
+        double *D, void *work, size_t work_bytes, void *stream, const EnvRow *env = nullptr,
+        int32_t *nvalid_out = nullptr, const char *who = "dp_tabulate_fusion_fwd_tc_f64") {
   clear_error();
-  static const char *who = "dp_tabulate_fusion_fwd_tc_f64";
   TableGeom g;
   Segments seg;
   Shape S{};
@@ -893,6 +1062,10 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
   RunsParams R = runs_params(s, Rt, nvalid, atype, g, seg, S, L, wk, nnei,
                              reinterpret_cast<const double *>(pk + PL.nodes));
   R.W = reinterpret_cast<double *>(wk + L.w);
+  if (env) {
+    R.env = *env;
+    R.nvalid_out = nvalid_out;
+  }
   longlong2 *part = reinterpret_cast<longlong2 *>(wk + L.part);
   int dev = 0, nsm = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
@@ -903,8 +1076,11 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
     const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN, tile0 = c0 / kTileAtoms;
     R.atom0 = c0;
     R.natoms = n;
-    runs_kernel<true><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
-                        kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
+    const dim3 rgrid((unsigned)((n + kRunsWarps - 1) / kRunsWarps));
+    if (env)
+      runs_kernel<true, true><<<rgrid, 32 * kRunsWarps, kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
+    else
+      runs_kernel<true><<<rgrid, 32 * kRunsWarps, kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_runs_moments", st);
     const int64_t nlist = (int64_t)ntypes * ntiles;
@@ -959,18 +1135,29 @@ int fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *s, cons
   return DP_OK;
 }
 
+// env: the rows come from coordinates and the rows kernel adds the forces and virial instead of writing
+// ds and dRt (dp_tabulate_fusion_env_grad_tc_f64; s, Rt, nvalid, ds and dRt unused; F [nall][3] and
+// virial [9] are zeroed first).
 int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt, const int32_t *nvalid,
          const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel, int M1, const double *dT,
-         double *ds, double *dRt, void *work, size_t work_bytes, int flags, void *stream) {
+         double *ds, double *dRt, void *work, size_t work_bytes, int flags, void *stream, const EnvRow *env = nullptr,
+         double *F = nullptr, double *virial = nullptr, int64_t nall = 0,
+         const char *who = "dp_tabulate_fusion_grad_tc_f64") {
   clear_error();
-  static const char *who = "dp_tabulate_fusion_grad_tc_f64";
   if (flags & ~DP_TC_REUSE_RUNS) return set_error(DP_ERR_SHAPE, "%s: unknown flags %#x", who, flags);
   TableGeom g;
   Segments seg;
   Shape S{};
   Layout L{};
-  int rc = tc_args(plan, info, s, Rt, nloc, nnei, ntypes, sel, M1, ds, dRt, work, work_bytes, &g, &seg, &S, &L, who);
-  if (rc || nloc == 0) return rc;
+  int rc = tc_args(plan, info, s, Rt, nloc, nnei, ntypes, sel, M1, env ? (void *)F : ds, env ? (void *)virial : dRt,
+                   work, work_bytes, &g, &seg, &S, &L, who);
+  if (rc) return rc;
+  if (env) {  // the forces and virial are sums: zeroed first, also for nloc = 0
+    cudaError_t e = cudaMemsetAsync(virial, 0, 9 * sizeof(double), (cudaStream_t)stream);
+    if (e == cudaSuccess && nall > 0) e = cudaMemsetAsync(F, 0, (size_t)nall * 3 * sizeof(double), (cudaStream_t)stream);
+    if (e != cudaSuccess) return set_error(DP_ERR_CUDA, "%s: %s", who, cudaGetErrorString(e));
+  }
+  if (nloc == 0) return DP_OK;
   if (!dT) return set_error(DP_ERR_NULL, "%s: dT is NULL", who);
   const PlanLayout PL = plan_layout(S);
   const unsigned char *pk = static_cast<const unsigned char *>(plan->data);
@@ -1002,14 +1189,23 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
   Q.dW = dW;
   Q.ds = ds;
   Q.dRt = dRt;
+  if (env) {
+    R.env = *env;
+    Q.env = *env;
+    Q.F = F;
+    Q.virial = virial;
+  }
   for (int64_t c0 = 0; c0 < nloc; c0 += S.chunk) {
     const int64_t n = std::min<int64_t>(S.chunk, nloc - c0);
     const int64_t Np = round_up(kCols * n, kTN), ntiles = Np / kTN, tile0 = c0 / kTileAtoms;
     R.atom0 = c0;
     R.natoms = n;
     if (!reuse) {
-      runs_kernel<false><<<(unsigned)((n + kRunsWarps - 1) / kRunsWarps), 32 * kRunsWarps,
-                           kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
+      const dim3 rgrid((unsigned)((n + kRunsWarps - 1) / kRunsWarps));
+      if (env)
+        runs_kernel<false, true><<<rgrid, 32 * kRunsWarps, kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
+      else
+        runs_kernel<false><<<rgrid, 32 * kRunsWarps, kRunsWarps * S.nkeys * sizeof(short), st>>>(R);
       if ((rc = launch_status(who))) return rc;
       prof_mark("tc_runs", st);
     }
@@ -1099,12 +1295,55 @@ int grad(const dp_tc_plan *plan, const dp_table_info *info, const double *s, con
     }
     Q.atom0 = c0;
     Q.natoms = n;
-    rows_kernel<<<(unsigned)((n + kRowsWarps - 1) / kRowsWarps), 32 * kRowsWarps, kRowsWarps * S.nkeys * sizeof(short),
-                  st>>>(Q);
+    const dim3 qgrid((unsigned)((n + kRowsWarps - 1) / kRowsWarps));
+    if (env)
+      rows_force_kernel<<<qgrid, 32 * kRowsWarps, kRowsWarps * S.nkeys * sizeof(short), st>>>(Q);
+    else
+      rows_kernel<<<qgrid, 32 * kRowsWarps, kRowsWarps * S.nkeys * sizeof(short), st>>>(Q);
     if ((rc = launch_status(who))) return rc;
     prof_mark("tc_rows", st);
   }
   return DP_OK;
+}
+
+EnvRow env_row(const dp_env_info *e, const double *coord, const int32_t *nlist) {
+  EnvRow E{};
+  E.coord = coord;
+  E.nlist = nlist;
+  E.rcs = e->rcs;
+  E.rc = e->rc;
+  E.inv_width = 1.0 / (e->rc - e->rcs);
+  E.mean = e->mean;
+  E.inv_std = 1.0 / e->std;
+  E.inv_std_all = 1.0 / e->std_all;
+  E.kind = e->kind;
+  return E;
+}
+
+int env_fwd(const dp_tc_plan *plan, const dp_table_info *info, const double *coord, const int32_t *nlist,
+            const dp_env_info *env, const int32_t *atype, int64_t nloc, int nnei, int ntypes, const int32_t *sel,
+            int M1, int32_t *nvalid, double *T, int M2, double *D, void *work, size_t work_bytes, void *stream) {
+  clear_error();
+  static const char *who = "dp_tabulate_fusion_env_fwd_tc_f64";
+  if (int rc = check_env(env)) return rc;
+  const EnvRow E = env_row(env, coord, nlist);
+  // coord and nlist stand where the plain call's s and Rt are checked for NULL
+  return fwd(plan, info, coord, reinterpret_cast<const double *>(nlist), nullptr, atype, nloc, nnei, ntypes, sel, M1,
+             T, M2, D, work, work_bytes, stream, &E, nvalid, who);
+}
+
+int env_grad(const dp_tc_plan *plan, const dp_table_info *info, const double *coord, const int32_t *nlist,
+             const dp_env_info *env, const int32_t *atype, int64_t nloc, int64_t nall, int nnei, int ntypes,
+             const int32_t *sel, int M1, const double *dT, double *F, double *virial, void *work, size_t work_bytes,
+             int flags, void *stream) {
+  clear_error();
+  static const char *who = "dp_tabulate_fusion_env_grad_tc_f64";
+  if (int rc = check_env(env)) return rc;
+  if (nall < nloc) return set_error(DP_ERR_SHAPE, "%s: nall = %lld < nloc = %lld", who, (long long)nall, (long long)nloc);
+  if (!virial || (nall > 0 && !F)) return set_error(DP_ERR_NULL, "%s: NULL output", who);
+  const EnvRow E = env_row(env, coord, nlist);
+  return grad(plan, info, coord, reinterpret_cast<const double *>(nlist), nullptr, atype, nloc, nnei, ntypes, sel, M1,
+              dT, nullptr, nullptr, work, work_bytes, flags, stream, &E, F, virial, nall, who);
 }
 
 size_t work_bytes_api(const dp_table_info *info, int64_t nloc, int nnei, int ntypes, int M1) {
@@ -1156,6 +1395,23 @@ int dp_tabulate_fusion_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *i
                                   size_t work_bytes, void *stream) {
   return dpc::tt::fwd(plan, info, s, Rt, nvalid, atype, nloc, nnei, ntypes, sel, M1, T, M2, D, work, work_bytes,
                       stream);
+}
+
+int dp_tabulate_fusion_env_fwd_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *coord,
+                                      const int32_t *nlist, const dp_env_info *env, const int32_t *atype, int64_t nloc,
+                                      int nnei, int ntypes, const int32_t *sel, int M1, int32_t *nvalid, double *T,
+                                      int M2, double *D, void *work, size_t work_bytes, void *stream) {
+  return dpc::tt::env_fwd(plan, info, coord, nlist, env, atype, nloc, nnei, ntypes, sel, M1, nvalid, T, M2, D, work,
+                          work_bytes, stream);
+}
+
+int dp_tabulate_fusion_env_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *coord,
+                                       const int32_t *nlist, const dp_env_info *env, const int32_t *atype,
+                                       int64_t nloc, int64_t nall, int nnei, int ntypes, const int32_t *sel, int M1,
+                                       const double *dT, double *F, double *virial, void *work, size_t work_bytes,
+                                       int flags, void *stream) {
+  return dpc::tt::env_grad(plan, info, coord, nlist, env, atype, nloc, nall, nnei, ntypes, sel, M1, dT, F, virial,
+                           work, work_bytes, flags, stream);
 }
 
 int dp_tabulate_fusion_grad_tc_f64(const dp_tc_plan *plan, const dp_table_info *info, const double *s, const double *Rt,
