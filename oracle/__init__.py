@@ -93,6 +93,12 @@ def load(path: str | None = None):
     lib.or_descriptor_grad.restype = None
     lib.or_fitting.argtypes = [P, i64, P, ctypes.c_int, P, P, i64, P, P, P, ctypes.c_int]
     lib.or_fitting.restype = ctypes.c_int
+    for f in ("or_vector_head", "or_tensor_head"):
+        getattr(lib, f).argtypes = [P, P, i64, ctypes.c_int, P]
+        getattr(lib, f).restype = None
+    for f in ("or_vector_head_grad", "or_tensor_head_grad"):
+        getattr(lib, f).argtypes = [P, P, P, i64, ctypes.c_int, P, P]
+        getattr(lib, f).restype = None
     lib.or_embed_rows.argtypes = [P, ctypes.POINTER(Info), P, P, ctypes.c_int, ctypes.c_int, P, ctypes.c_int, P,
                                   i64, P, P]
     lib.or_embed_rows.restype = None
@@ -253,20 +259,58 @@ class Oracle:
         return dT
 
     def fitting(self, params, widths, D, atype=None, g=None, grad=True, nthreads=0):
-        """Atomic energies E [n] of the fitting net and, with grad, dE_i/dD_i [n][widths[0]] (scaled by g)."""
+        """Outputs of the fitting net, E [n] (widths[-1] == 1: the atomic energies) or [n][widths[-1]],
+        and, with grad, sum_c g_c dE_c/dD_i [n][widths[0]] (g shaped like E; None: all ones)."""
         params = _c(np.atleast_2d(params), np.float64)
         w = _c(widths, np.int32)
         D = _c(D.reshape(D.shape[0], -1), np.float64)
         n = D.shape[0]
         assert D.shape[1] == w[0]
+        nout = int(w[-1])
         at = None if atype is None else _c(atype, np.int32)
-        gg = None if g is None else _c(g, np.float64)
-        E = np.empty(n)
+        gg = None if g is None else _c(np.reshape(g, (n, nout)), np.float64)
+        E = np.empty((n, nout))
         dD = np.empty((n, int(w[0]))) if grad else None
         if self.lib.or_fitting(_p(params), params.shape[1], _p(w), len(w) - 1, _p(D), _p(at), n, _p(gg), _p(E),
                                _p(dD), nthreads):
             raise ValueError("or_fitting failed")
+        E = E[:, 0] if nout == 1 else E
         return (E, dD) if grad else E
+
+    # -- vector and tensor heads ------------------------------------------------
+    def vector_head(self, T, a):
+        """v [n][3] = sum_m a[m] T[1:4, m] per atom."""
+        T, a = _c(T, np.float64), _c(a, np.float64)
+        n, four, M = T.shape
+        assert a.shape == (n, M)
+        v = np.empty((n, 3))
+        self.lib.or_vector_head(_p(T), _p(a), n, M, _p(v))
+        return v
+
+    def vector_head_grad(self, T, a, dv):
+        """(dT [n][4][M], da [n][M]) from dE/dv [n][3]."""
+        T, a, dv = _c(T, np.float64), _c(a, np.float64), _c(dv, np.float64)
+        n, four, M = T.shape
+        dT, da = np.empty_like(T), np.empty((n, M))
+        self.lib.or_vector_head_grad(_p(T), _p(a), _p(dv), n, M, _p(dT), _p(da))
+        return dT, da
+
+    def tensor_head(self, T, a):
+        """A [n][3][3] = sum_m a[m] T[1:4, m] T[1:4, m]^T per atom."""
+        T, a = _c(T, np.float64), _c(a, np.float64)
+        n, four, M = T.shape
+        assert a.shape == (n, M)
+        A = np.empty((n, 3, 3))
+        self.lib.or_tensor_head(_p(T), _p(a), n, M, _p(A))
+        return A
+
+    def tensor_head_grad(self, T, a, dA):
+        """(dT [n][4][M], da [n][M]) from dE/dA [n][3][3]."""
+        T, a, dA = _c(T, np.float64), _c(a, np.float64), _c(dA, np.float64)
+        n, four, M = T.shape
+        dT, da = np.empty_like(T), np.empty((n, M))
+        self.lib.or_tensor_head_grad(_p(T), _p(a), _p(dA), n, M, _p(dT), _p(da))
+        return dT, da
 
     def embed_rows(self, table, info, s, atype, sel, atoms=None, deriv=False):
         table, s = (_c(a, np.float64) for a in (table, s))

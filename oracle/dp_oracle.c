@@ -628,18 +628,21 @@ void or_force_virial(int64_t nloc, int64_t nall, const double *coord, const int3
  * Fitting net (Sec. II: the descriptor D_i is passed to a fully connected
  * network that outputs the atomic energy E_i; the total energy is
  * E = sum_i E_i).  For centre type t the net has nlayer layers with widths
- * widths[0..nlayer], widths[0] = the length of D_i, widths[nlayer] = 1:
+ * widths[0..nlayer], widths[0] = the length of D_i, widths[nlayer] = nout
+ * (1 for the energy; M1 for the vector and tensor heads below, the models the
+ * conclusion of the paper says compression carries over to):
  *   hidden layer l (l < nlayer - 1):  v_l = tanh(v_{l-1} W_l + b_l) (+ v_{l-1} when the widths agree)
- *   output layer:                     E_i = v_{nlayer-1} W_nlayer + b_nlayer
+ *   output layer:                     E_i = v_{nlayer-1} W_nlayer + b_nlayer   (nout values)
  * params [ntypes][P], layer by layer W_l [a][b] row-major then b_l [b].
- * E [n]; when dD is not NULL also dE_i/dD_i [n][widths[0]] by the chain rule
- * backwards through the layers (d tanh(z)/dz = 1 - tanh(z)^2), scaled by
- * g[i] (NULL: 1).  Returns -1 for a width above OR_FITW or bad sizes.
+ * E [n][nout]; when dD is not NULL also sum_c g[i][c] dE_ic/dD_i [n][widths[0]]
+ * by the chain rule backwards through the layers (d tanh(z)/dz = 1 - tanh(z)^2),
+ * g [n][nout] (NULL: all 1).  Returns -1 for a width above OR_FITW or bad sizes.
  */
 #define OR_FITW 4096
 int or_fitting(const double *params, int64_t P, const int32_t *widths, int nlayer, const double *D,
                const int32_t *atype, int64_t n, const double *g, double *E, double *dD, int nthreads) {
-  if (nlayer < 1 || widths[nlayer] != 1) return -1;
+  if (nlayer < 1) return -1;
+  const int nout = widths[nlayer];
   int hid = 0;  // sum of the hidden widths
   for (int l = 0; l <= nlayer; ++l)
     if (widths[l] < 1 || widths[l] > OR_FITW) return -1;
@@ -681,15 +684,20 @@ int or_fitting(const double *params, int64_t P, const int32_t *widths, int nlaye
       off_t += b;
     }
     const int a = widths[nlayer - 1];
-    const double *Wo = p, *bo = p + a;
-    double e = bo[0];
-    for (int k = 0; k < a; ++k) e += act[off_in + k] * Wo[k];
-    E[i] = e;
+    const double *Wo = p, *bo = p + (size_t)a * nout;
+    for (int c = 0; c < nout; ++c) {
+      double e = bo[c];
+      for (int k = 0; k < a; ++k) e += act[off_in + k] * Wo[(size_t)k * nout + c];
+      E[(size_t)i * nout + c] = e;
+    }
     if (dD) {
-      // backward: gv holds dE_i/dv_l for the current layer
-      const double gi = g ? g[i] : 1.0;
+      // backward: gv holds dE_i/dv_l for the current layer (E_i weighted by g)
       double *cur = gv, *nxt = gv + OR_FITW;
-      for (int k = 0; k < a; ++k) cur[k] = gi * Wo[k];
+      for (int k = 0; k < a; ++k) {
+        double v = 0.0;
+        for (int c = 0; c < nout; ++c) v += (g ? g[(size_t)i * nout + c] : 1.0) * Wo[(size_t)k * nout + c];
+        cur[k] = v;
+      }
       // walk the hidden layers from the last to the first; their parameters precede Wo
       const double *pl = Wo;
       int toff = off_t;
@@ -717,4 +725,73 @@ int or_fitting(const double *params, int64_t P, const int32_t *widths, int nlaye
     free(gv);
   }
   return err ? -1 : 0;
+}
+
+/* --------------------------------------------- vector and tensor heads */
+
+/*
+ * Vector and tensor DP models (the paper's conclusion: compression carries
+ * over to models of vectors, such as dipoles, and of tensors, such as
+ * polarizabilities).  The compressed path is the same up to T_i; the head
+ * contracts the rotation-covariant rows k = 1..3 of T_i (the x, y, z columns
+ * of R~, Sec. II) with the fitting net's M outputs a_i, which are invariant:
+ *   vector:  v_i[c]    = sum_m a_i[m] T_i[1+c][m]
+ *   tensor:  A_i[c][d] = sum_m a_i[m] (T_i[1+c][m] T_i[1+d][m])   (symmetric to the bit)
+ * T [n][4][M], a [n][M], v [n][3], A [n][3][3].
+ * Backward, from dE/dv or dE/dA: dE/dT (row 0 zero) and dE/da:
+ *   vector:  dT_i[1+c][m] = a_i[m] dv_i[c];  da_i[m] = sum_c dv_i[c] T_i[1+c][m]
+ *   tensor:  dT_i[1+c][m] = a_i[m] sum_d (dA_i[c][d] + dA_i[d][c]) T_i[1+d][m];
+ *            da_i[m] = sum_{c,d} dA_i[c][d] T_i[1+c][m] T_i[1+d][m]
+ */
+void or_vector_head(const double *T, const double *a, int64_t n, int M, double *v) {
+  for (int64_t i = 0; i < n; ++i)
+    for (int c = 0; c < 3; ++c) {
+      double s = 0.0;
+      for (int m = 0; m < M; ++m) s += a[i * M + m] * T[(i * 4 + 1 + c) * M + m];
+      v[i * 3 + c] = s;
+    }
+}
+
+void or_vector_head_grad(const double *T, const double *a, const double *dv, int64_t n, int M, double *dT,
+                         double *da) {
+  for (int64_t i = 0; i < n; ++i)
+    for (int m = 0; m < M; ++m) {
+      dT[(i * 4 + 0) * M + m] = 0.0;
+      double s = 0.0;
+      for (int c = 0; c < 3; ++c) {
+        dT[(i * 4 + 1 + c) * M + m] = a[i * M + m] * dv[i * 3 + c];
+        s += dv[i * 3 + c] * T[(i * 4 + 1 + c) * M + m];
+      }
+      da[i * M + m] = s;
+    }
+}
+
+void or_tensor_head(const double *T, const double *a, int64_t n, int M, double *A) {
+  for (int64_t i = 0; i < n; ++i)
+    for (int c = 0; c < 3; ++c)
+      for (int d = 0; d < 3; ++d) {
+        double s = 0.0;
+        for (int m = 0; m < M; ++m) s += a[i * M + m] * (T[(i * 4 + 1 + c) * M + m] * T[(i * 4 + 1 + d) * M + m]);
+        A[(i * 3 + c) * 3 + d] = s;
+      }
+}
+
+void or_tensor_head_grad(const double *T, const double *a, const double *dA, int64_t n, int M, double *dT,
+                         double *da) {
+  for (int64_t i = 0; i < n; ++i)
+    for (int m = 0; m < M; ++m) {
+      const double *G = dA + i * 9;
+      dT[(i * 4 + 0) * M + m] = 0.0;
+      double s = 0.0;
+      for (int c = 0; c < 3; ++c) {
+        double u = 0.0;
+        for (int d = 0; d < 3; ++d) {
+          const double td = T[(i * 4 + 1 + d) * M + m];
+          u += (G[3 * c + d] + G[3 * d + c]) * td;
+          s += G[3 * c + d] * T[(i * 4 + 1 + c) * M + m] * td;
+        }
+        dT[(i * 4 + 1 + c) * M + m] = a[i * M + m] * u;
+      }
+      da[i * M + m] = s;
+    }
 }

@@ -649,9 +649,116 @@ def pin_fitting_types(o):
         assert _rel(E[sel], Et) < 1e-15 and _rel(dD[sel], dDt) < 1e-15
 
 
+def pin_fitting_multi_output(o):
+    """A net with several outputs is several scalar nets sharing the hidden layers: output c equals the
+    one-output net whose output layer is column c of W_out and b_out[c] (a net pinned above by hand and
+    by differences), and the backward weighted by g [n][nout] is sum_c g_c times that net's dE/dD."""
+    widths = [12, 8, 8, 5]
+    params = W.net_params(65, widths, 2)
+    D = W.normal(66, (7, 12))
+    at = np.array([0, 1, 1, 0, 1, 0, 0], dtype=np.int32)
+    g = W.normal(67, (7, 5))
+    E, dD = o.fitting(params, widths, D, at, g=g)
+    a = widths[-2]
+    nh = params.shape[1] - (a + 1) * widths[-1]  # the hidden layers' parameters
+    ref_dD = np.zeros_like(dD)
+    for c in range(widths[-1]):
+        Wo = params[:, nh:nh + a * widths[-1]].reshape(2, a, widths[-1])[:, :, c]
+        bo = params[:, nh + a * widths[-1] + c]
+        pc = np.concatenate([params[:, :nh], Wo, bo[:, None]], axis=1)
+        Ec, dDc = o.fitting(pc, widths[:-1] + [1], D, at)
+        assert _rel(E[:, c], Ec) < 1e-15, c
+        ref_dD += g[:, c:c + 1] * dDc
+    assert _rel(dD, ref_dD) < 1e-13
+
+
+# ------------------------------------------------------------ vector and tensor heads
+
+def _rotation():
+    c, sn = math.cos(0.7), math.sin(0.7)
+    Rz = np.array([[c, -sn, 0], [sn, c, 0], [0, 0, 1.0]])
+    c2, s2 = math.cos(-1.1), math.sin(-1.1)
+    Rx = np.array([[1.0, 0, 0], [0, c2, -s2], [0, s2, c2]])
+    return Rz @ Rx
+
+
+def _head_chain(o, x, t, nlist, nvalid, sel, env, tabs, info, fparams, fwidths, M2):
+    """Coordinates -> R~ -> T -> D -> the fitting net's M outputs a (invariant) and T."""
+    s, Rt = o.env_mat(x, nlist, env[0], env[1], env[2], env[3])
+    T = o.fwd(tabs, info, s, Rt, nvalid, t, sel)
+    a = o.fitting(fparams, fwidths, o.descriptor(T, M2).reshape(x.shape[0], -1), t, grad=False)
+    return T, a
+
+
+def _head_fd(o, head, grad, T, a, dout, h=1e-6):
+    """dT and da of L = <dout, head(T, a)> against central differences in a sample of entries."""
+    dT, da = grad(T, a, dout)
+    L = lambda T_, a_: float(np.sum(dout * head(T_, a_)))
+    for i, k, m in ((0, 0, 0), (1, 1, 2), (2, 2, 5), (3, 3, 7), (1, 3, 0)):
+        Tp, Tm = T.copy(), T.copy()
+        Tp[i, k, m] += h
+        Tm[i, k, m] -= h
+        fd = (L(Tp, a) - L(Tm, a)) / (2 * h)
+        assert abs(fd - dT[i, k, m]) <= 1e-8 * max(1.0, np.abs(dT).max()), (i, k, m, fd, dT[i, k, m])
+    for i, m in ((0, 0), (2, 3), (3, 7)):
+        ap, am = a.copy(), a.copy()
+        ap[i, m] += h
+        am[i, m] -= h
+        fd = (L(T, ap) - L(T, am)) / (2 * h)
+        assert abs(fd - da[i, m]) <= 1e-8 * max(1.0, np.abs(da).max()), (i, m, fd, da[i, m])
+
+
+def pin_vector_head(o):
+    """v = sum_m a_m T[1:4, m]: a one-hot a picks a column of T's last three rows; a numpy matmul on
+    random inputs; the backward against differences; and on the whole vector model from coordinates
+    (R~ -> T -> D -> fitting net with M outputs -> v) rotating the coordinates rotates v while a, a
+    function of the invariant D, stays (the rotation covariance the head exists for)."""
+    T = W.normal(71, (4, 4, 8))
+    a = W.normal(72, (4, 8))
+    for m in (0, 5):
+        e = np.zeros((4, 8))
+        e[:, m] = 1.0
+        assert np.array_equal(o.vector_head(T, e), T[:, 1:4, m])
+    assert _rel(o.vector_head(T, a), np.einsum("ikm,im->ik", T[:, 1:4, :], a)) < 1e-15
+    _head_fd(o, o.vector_head, o.vector_head_grad, T, a, W.normal(73, (4, 3)))
+    x, t, nlist, nvalid, sel, env, tabs, info, _ = _cluster_model(o, 74, 0, None)
+    fwidths = [8 * 3, 10, 10, 8]
+    fparams = W.net_params(75, fwidths, 2)
+    T, a = _head_chain(o, x, t, nlist, nvalid, sel, env, tabs, info, fparams, fwidths, 3)
+    R = _rotation()
+    T2, a2 = _head_chain(o, x @ R.T, t, nlist, nvalid, sel, env, tabs, info, fparams, fwidths, 3)
+    assert _rel(a2, a) < 1e-12
+    assert _rel(o.vector_head(T2, a2), o.vector_head(T, a) @ R.T) < 1e-11
+
+
+def pin_tensor_head(o):
+    """A = sum_m a_m t_m t_m^T (t_m = T[1:4, m]): symmetric; a one-hot a gives the outer product
+    t_m t_m^T; its trace is sum_m a_m |t_m|^2; a numpy einsum on random inputs; the backward against
+    differences with a non-symmetric dE/dA; and A -> R A R^T when the coordinates of the whole tensor
+    model rotate."""
+    T = W.normal(81, (4, 4, 8))
+    a = W.normal(82, (4, 8))
+    A = o.tensor_head(T, a)
+    assert np.array_equal(A, np.transpose(A, (0, 2, 1)))
+    e = np.zeros((4, 8))
+    e[:, 3] = 1.0
+    assert _rel(o.tensor_head(T, e), np.einsum("ic,id->icd", T[:, 1:4, 3], T[:, 1:4, 3])) < 1e-15
+    assert _rel(np.trace(A, axis1=1, axis2=2), np.einsum("im,ikm,ikm->i", a, T[:, 1:4], T[:, 1:4])) < 1e-14
+    assert _rel(A, np.einsum("im,icm,idm->icd", a, T[:, 1:4], T[:, 1:4])) < 1e-14
+    _head_fd(o, o.tensor_head, o.tensor_head_grad, T, a, W.normal(83, (4, 3, 3)))
+    x, t, nlist, nvalid, sel, env, tabs, info, _ = _cluster_model(o, 84, 1, (0.2, 0.3, 0.25))
+    fwidths = [8 * 3, 10, 8]
+    fparams = W.net_params(85, fwidths, 2)
+    T, a = _head_chain(o, x, t, nlist, nvalid, sel, env, tabs, info, fparams, fwidths, 3)
+    R = _rotation()
+    T2, a2 = _head_chain(o, x @ R.T, t, nlist, nvalid, sel, env, tabs, info, fparams, fwidths, 3)
+    assert _rel(o.tensor_head(T2, a2), R @ o.tensor_head(T, a) @ R.T) < 1e-11
+
+
 ALL_PINS = [pin_net_skip_wiring, pin_net_single_neuron, pin_net_derivatives_fd, pin_table_info, pin_locate,
             pin_table_nodes, pin_table_quintic_exact, pin_table_sin_bound, pin_compressed_vs_net,
             pin_fwd_brute_force, pin_fwd_constant_G, pin_fwd_vs_explicit_G, pin_fwd_padding, pin_fwd_symmetries,
             pin_grad_fd, pin_grad_identities, pin_grad_brute_force, pin_descriptor, pin_descriptor_grad,
             pin_switch, pin_env_mat_hand, pin_env_mat_matches_generator, pin_force_fd, pin_force_invariants,
-            pin_fitting_hand, pin_fitting_fd, pin_fitting_types]
+            pin_fitting_hand, pin_fitting_fd, pin_fitting_types, pin_fitting_multi_output, pin_vector_head,
+            pin_tensor_head]

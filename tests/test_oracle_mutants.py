@@ -64,6 +64,22 @@ MUTANTS = [
     ("fitting: transposed weights", "for (int k = 0; k < a; ++k) z += act[off_in + k] * W[(size_t)k * b + o];",
      "for (int k = 0; k < a; ++k) z += act[off_in + k] * W[(size_t)o * a + k];"),
     ("fitting: centre type ignored", "const double *pp = params + (size_t)(atype ? atype[i] : 0) * P;", "const double *pp = params;"),
+    ("fitting: output weights read transposed", "for (int k = 0; k < a; ++k) e += act[off_in + k] * Wo[(size_t)k * nout + c];",
+     "for (int k = 0; k < a; ++k) e += act[off_in + k] * Wo[(size_t)c * a + k];"),
+    ("fitting: upstream weights of output 0 only",
+     "v += (g ? g[(size_t)i * nout + c] : 1.0) * Wo[(size_t)k * nout + c];",
+     "v += (g ? g[(size_t)i * nout] : 1.0) * Wo[(size_t)k * nout + c];"),
+    ("vector head: row 0 of T included", "s += a[i * M + m] * T[(i * 4 + 1 + c) * M + m];",
+     "s += a[i * M + m] * T[(i * 4 + c) * M + m];"),
+    ("vector head grad: one component of dv", "dT[(i * 4 + 1 + c) * M + m] = a[i * M + m] * dv[i * 3 + c];",
+     "dT[(i * 4 + 1 + c) * M + m] = a[i * M + m] * dv[i * 3];"),
+    ("tensor head: diagonal rows only",
+     "s += a[i * M + m] * (T[(i * 4 + 1 + c) * M + m] * T[(i * 4 + 1 + d) * M + m]);",
+     "s += a[i * M + m] * (T[(i * 4 + 1 + c) * M + m] * T[(i * 4 + 1 + c) * M + m]);"),
+    ("tensor head grad: transposed dA term dropped", "u += (G[3 * c + d] + G[3 * d + c]) * td;",
+     "u += (G[3 * c + d] + G[3 * c + d]) * td;"),
+    ("tensor head grad: da without the a-free product", "s += G[3 * c + d] * T[(i * 4 + 1 + c) * M + m] * td;",
+     "s += G[3 * c + d] * td;"),
 ]
 
 
