@@ -528,10 +528,12 @@ int dp_force_virial_f32(const float *coord, const int32_t *nlist, int64_t nloc, 
  * network that outputs the atomic energy E_i; the total energy is
  * E = sum_i E_i).  Each centre type t has its own net of nlayer layers with
  * widths widths[0..nlayer] (host), widths[0] = the length of D_i (M1 * M2),
- * widths[nlayer] = 1:
+ * widths[nlayer] = nout, the outputs per atom: 1 for the energy, M1 for the
+ * weights a_i of the vector and tensor heads (dp_vector_head_*,
+ * dp_tensor_head_*; the tensor-core variants below take nout = 1 only):
  *   v_0 = D_i
  *   v_l = tanh(v_{l-1} W_l + b_l) (+ v_{l-1} when widths[l] == widths[l-1]),  0 < l < nlayer
- *   E_i = v_{nlayer-1} W_nlayer + b_nlayer
+ *   E_i = v_{nlayer-1} W_nlayer + b_nlayer   (nout values)
  *   params      [ntypes][P]: per type, layer by layer, W_l [widths[l-1]][widths[l]]
  *               row-major then b_l [widths[l]]; P = sum_l (widths[l-1] + 1) widths[l].
  *   type_start  [ntypes + 1] HOST int64: the atoms of centre type t are rows
@@ -539,10 +541,10 @@ int dp_force_virial_f32(const float *coord, const int32_t *nlist, int64_t nloc, 
  *               type, as in every workload here); type_start[0] = 0 and
  *               nloc = type_start[ntypes].
  *   D    [nloc][widths[0]] input (the descriptor, flattened)
- *   E    [nloc] output
+ *   E    [nloc][nout] output
  *   act  [nloc][H] output, H = the sum of the hidden widths: tanh(v_{l-1} W_l + b_l)
  *        of every hidden layer, in layer order -- what the backward needs.
- * Errors: DP_ERR_NULL, DP_ERR_SHAPE (widths[nlayer] != 1, type_start not
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (a width outside [1, 2^20], type_start not
  * increasing or not starting at 0, more than 4,194,240 atoms of one type),
  * DP_ERR_UNSUPPORTED (nlayer or ntypes above DP_MAX_LAYERS / DP_MAX_TYPES),
  * DP_ERR_CUDA.  nloc == 0 reads no device pointer.
@@ -553,15 +555,17 @@ int dp_fitting_fwd_f32(const float *params, const int32_t *widths, int nlayer, i
                        const float *D, float *E, float *act, void *stream);
 
 /*
- * Backward of the fitting net: dD[i] = g_i dE_i/dD_i, the chain rule through
- * the layers in reverse (d tanh(z)/dz = 1 - tanh(z)^2; an identity skip
- * passes dE/dv_l on to v_{l-1}).
+ * Backward of the fitting net: dD[i] = sum_c g_ic dE_ic/dD_i, the chain rule
+ * through the layers in reverse (d tanh(z)/dz = 1 - tanh(z)^2; an identity
+ * skip passes dE/dv_l on to v_{l-1}).
  *   act   [nloc][H] from dp_fitting_fwd_* on the same D
- *   g     [nloc] upstream dE/dE_i, or NULL for all ones (E = sum_i E_i)
+ *   g     [nloc][nout] upstream dE/dE_i, or NULL for all ones (nout = 1 only:
+ *         E = sum_i E_i)
  *   dD    [nloc][widths[0]] output (feed it to dp_descriptor_contract_grad_*)
  *   work  [2][nloc][max hidden width] scratch, caller-owned, overwritten
- *         (NULL allowed when the net has a single hidden layer).
- * Errors as dp_fitting_fwd_*; a net without hidden layers is DP_ERR_UNSUPPORTED.
+ *         (NULL allowed when the net has a single hidden layer and nout = 1).
+ * Errors as dp_fitting_fwd_*; a net without hidden layers is DP_ERR_UNSUPPORTED;
+ * g NULL with nout > 1 is DP_ERR_NULL.
  */
 int dp_fitting_grad_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
                         const int64_t *type_start, const double *act, const double *g, double *dD, double *work,
@@ -619,7 +623,7 @@ int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer
  *                     width] buffers between layers.  Calls sharing a work
  *                     buffer must not overlap on the GPU.
  * Errors as the f64 calls, plus DP_ERR_NULL / DP_ERR_SHAPE for a missing,
- * short or misaligned work buffer.
+ * short or misaligned work buffer; widths[nlayer] must be 1 (DP_ERR_SHAPE).
  */
 size_t dp_fitting_tc_work_bytes(const int32_t *widths, int nlayer, int64_t nloc); /* 0 on bad widths */
 int dp_fitting_fwd_tc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
@@ -628,6 +632,45 @@ int dp_fitting_fwd_tc_f64(const double *params, const int32_t *widths, int nlaye
 int dp_fitting_grad_tc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,
                            const int64_t *type_start, const double *act, const double *g, double *dD, void *work,
                            size_t work_bytes, void *stream);
+
+/* ------------------------------------------------------------------------
+ * Vector and tensor heads.  The paper's conclusion states that compression
+ * carries over to DP models of vectors (dipoles) and tensors
+ * (polarizabilities): their compressed path is the same up to T_i; the head
+ * contracts the rotation-covariant rows k = 1..3 of T_i (the x, y, z columns
+ * of R~, Sec. II) with M1 rotation-invariant weights a_i that a fitting net
+ * with nout = M1 makes from D_i:
+ *   vector:  v_i[c]    = sum_m a_i[m] T_i[1+c][m]
+ *   tensor:  A_i[c][d] = sum_m a_i[m] (T_i[1+c][m] T_i[1+d][m])   (symmetric)
+ * so v rotates as a vector and A as a rank-2 tensor when the coordinates do.
+ *   T   [nloc][4][M1] input (dp_tabulate_fusion_fwd_*)
+ *   a   [nloc][M1] input (dp_fitting_fwd_* with widths[nlayer] = M1)
+ *   v   [nloc][3] output; A [nloc][3][3] output
+ * Backward, from dE/dv [nloc][3] or dE/dA [nloc][3][3] (any, not only
+ * symmetric):
+ *   vector:  dT_i[1+c][m] = a_i[m] dv_i[c];  da_i[m] = sum_c dv_i[c] T_i[1+c][m]
+ *   tensor:  dT_i[1+c][m] = a_i[m] sum_d (dA_i[c][d] + dA_i[d][c]) T_i[1+d][m];
+ *            da_i[m] = sum_{c,d} dA_i[c][d] T_i[1+c][m] T_i[1+d][m]
+ *   dT  [nloc][4][M1] output: overwritten (row k = 0 set to zero) when
+ *       accumulate is 0; otherwise the head's dT is added to what dT holds
+ *       (dE/dT of the descriptor, dp_descriptor_contract_grad_*), row 0 kept
+ *   da  [nloc][M1] output (the upstream g of dp_fitting_grad_*)
+ * All arrays device, row-major, caller-owned; nothing is allocated.
+ * Errors: DP_ERR_NULL, DP_ERR_SHAPE (nloc < 0, M1 outside [1, 4096]),
+ * DP_ERR_CUDA.  nloc == 0 reads no device pointer.
+ */
+int dp_vector_head_f64(const double *T, const double *a, int64_t nloc, int M1, double *v, void *stream);
+int dp_vector_head_f32(const float *T, const float *a, int64_t nloc, int M1, float *v, void *stream);
+int dp_vector_head_grad_f64(const double *T, const double *a, const double *dv, int64_t nloc, int M1, double *dT,
+                            double *da, int accumulate, void *stream);
+int dp_vector_head_grad_f32(const float *T, const float *a, const float *dv, int64_t nloc, int M1, float *dT,
+                            float *da, int accumulate, void *stream);
+int dp_tensor_head_f64(const double *T, const double *a, int64_t nloc, int M1, double *A, void *stream);
+int dp_tensor_head_f32(const float *T, const float *a, int64_t nloc, int M1, float *A, void *stream);
+int dp_tensor_head_grad_f64(const double *T, const double *a, const double *dA, int64_t nloc, int M1, double *dT,
+                            double *da, int accumulate, void *stream);
+int dp_tensor_head_grad_f32(const float *T, const float *a, const float *dA, int64_t nloc, int M1, float *dT,
+                            float *da, int accumulate, void *stream);
 
 #ifdef __cplusplus
 }

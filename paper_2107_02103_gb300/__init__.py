@@ -146,6 +146,10 @@ _SIGS = {
     "dp_fitting_grad_df64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_fitting_grad_noalloc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P], ctypes.c_int),
     "dp_fitting_tc_work_bytes": ([_P, ctypes.c_int, _I64], ctypes.c_size_t),
+    **{f"dp_{h}_head_{x}": ([_P, _P, _I64, ctypes.c_int, _P, _P], ctypes.c_int)
+       for h in ("vector", "tensor") for x in ("f64", "f32")},
+    **{f"dp_{h}_head_grad_{x}": ([_P, _P, _P, _I64, ctypes.c_int, _P, _P, ctypes.c_int, _P], ctypes.c_int)
+       for h in ("vector", "tensor") for x in ("f64", "f32")},
     "dp_fitting_fwd_tc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P],
                               ctypes.c_int),
     "dp_fitting_grad_tc_f64": ([_P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P],
@@ -697,9 +701,16 @@ def _fit_shape(params, widths, type_start):
             widths, H)
 
 
+def _out_shape(nloc, widths):
+    """Shape of the fitting net's outputs (and of g): [nloc] for one output, else [nloc][nout]."""
+    return (nloc,) if widths[-1] == 1 else (nloc, widths[-1])
+
+
 def dp_fitting_fwd(params, widths, type_start, D, out=None, arith=None):
-    """(E [nloc], act [nloc][H]) of the fitting net; D [nloc][widths[0]] (a [nloc][M1][M2] descriptor is
-    flattened), atoms sorted by centre type with type_start [ntypes+1] (host); arith="df64" as elsewhere."""
+    """(E, act [nloc][H]) of the fitting net, E [nloc] (widths[-1] == 1: the atomic energies) or
+    [nloc][widths[-1]] (e.g. the M1 weights of dp_vector_head / dp_tensor_head); D [nloc][widths[0]]
+    (a [nloc][M1][M2] descriptor is flattened), atoms sorted by centre type with type_start [ntypes+1]
+    (host); arith="df64" as elsewhere."""
     params = _dev(params, "params", None)
     dtype = params.dtype
     w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
@@ -707,10 +718,10 @@ def dp_fitting_fwd(params, widths, type_start, D, out=None, arith=None):
     if D.shape[0] != nloc or D.numel() != nloc * widths[0]:
         raise ValueError(f"D must hold [{nloc}][{widths[0]}]")
     if out is None:
-        E = torch.empty((nloc,), dtype=dtype, device=params.device)
+        E = torch.empty(_out_shape(nloc, widths), dtype=dtype, device=params.device)
         act = torch.empty((nloc, max(H, 1)), dtype=dtype, device=params.device)
     else:
-        E = _dev(out[0], "E", dtype, (nloc,))
+        E = _dev(out[0], "E", dtype, _out_shape(nloc, widths))
         act = _dev(out[1], "act", dtype, (nloc, max(H, 1)))
     fn = getattr(_lib, f"dp_fitting_fwd_{_suffix(arith or dtype)}")
     _check(fn(_ptr(params), w, nlayer, ntypes, ts, _ptr(D), _ptr(E), _ptr(act), _stream(params)))
@@ -718,13 +729,14 @@ def dp_fitting_fwd(params, widths, type_start, D, out=None, arith=None):
 
 
 def dp_fitting_grad(params, widths, type_start, act, g=None, out=None, work=None, arith=None):
-    """dD [nloc][widths[0]] = g_i dE_i/dD_i from the forward's act; g [nloc] or None (all ones)."""
+    """dD [nloc][widths[0]] = sum_c g_ic dE_ic/dD_i from the forward's act; g shaped like the forward's
+    E, or None (all ones; one output only)."""
     params = _dev(params, "params", None)
     dtype = params.dtype
     w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
     act = _dev(act, "act", dtype, (nloc, max(H, 1)))
     if g is not None:
-        g = _dev(g, "g", dtype, (nloc,))
+        g = _dev(g, "g", dtype, _out_shape(nloc, widths))
     dD = torch.empty((nloc, widths[0]), dtype=dtype, device=params.device) if out is None else \
         _dev(out, "out", dtype, (nloc, widths[0]))
     maxh = max(widths[1:-1]) if len(widths) > 2 else 1
@@ -744,7 +756,7 @@ def dp_fitting_grad_noalloc_f64(params, widths, type_start, act, g=None, out=Non
     w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
     act = _dev(act, "act", torch.float64, (nloc, max(H, 1)))
     if g is not None:
-        g = _dev(g, "g", torch.float64, (nloc,))
+        g = _dev(g, "g", torch.float64, _out_shape(nloc, widths))
     dD = torch.empty((nloc, widths[0]), dtype=torch.float64, device=params.device) if out is None else \
         _dev(out, "out", torch.float64, (nloc, widths[0]))
     _check(_lib.dp_fitting_grad_noalloc_f64(_ptr(params), w, nlayer, ntypes, ts, _ptr(act), _ptr(g), _ptr(dD),
@@ -832,3 +844,54 @@ def table_rows(table: torch.Tensor) -> torch.Tensor:
 
 
 EXPORTS = tuple(_SIGS)
+
+
+def _head_inputs(T, a):
+    T = _dev(T, "T", None)
+    if T.dtype not in (torch.float64, torch.float32) or T.dim() != 3 or T.shape[1] != 4:
+        raise ValueError("T must be an f64 or f32 [nloc][4][M1] tensor")
+    nloc, M1 = int(T.shape[0]), int(T.shape[2])
+    a = _dev(a, "a", T.dtype, (nloc, M1))
+    return T, a, nloc, M1
+
+
+def dp_vector_head(T, a, out=None):
+    """v [nloc][3] = sum_m a[m] T[1:4, m] per atom (a vector DP model's head on the compressed T)."""
+    T, a, nloc, M1 = _head_inputs(T, a)
+    v = torch.empty((nloc, 3), dtype=T.dtype, device=T.device) if out is None else _dev(out, "v", T.dtype, (nloc, 3))
+    _check(getattr(_lib, f"dp_vector_head_{_suffix(T.dtype)}")(_ptr(T), _ptr(a), nloc, M1, _ptr(v), _stream(T)))
+    return v
+
+
+def dp_tensor_head(T, a, out=None):
+    """A [nloc][3][3] = sum_m a[m] t_m t_m^T, t_m = T[1:4, m] (a tensor DP model's head)."""
+    T, a, nloc, M1 = _head_inputs(T, a)
+    A = torch.empty((nloc, 3, 3), dtype=T.dtype, device=T.device) if out is None else \
+        _dev(out, "A", T.dtype, (nloc, 3, 3))
+    _check(getattr(_lib, f"dp_tensor_head_{_suffix(T.dtype)}")(_ptr(T), _ptr(a), nloc, M1, _ptr(A), _stream(T)))
+    return A
+
+
+def _head_grad(kind, T, a, dout, shape, dT, da, accumulate):
+    T, a, nloc, M1 = _head_inputs(T, a)
+    dout = _dev(dout, "dout", T.dtype, (nloc,) + shape)
+    if dT is None:
+        if accumulate:
+            raise ValueError("accumulate needs the dT to add to")
+        dT = torch.empty((nloc, 4, M1), dtype=T.dtype, device=T.device)
+    else:
+        dT = _dev(dT, "dT", T.dtype, (nloc, 4, M1))
+    da = torch.empty((nloc, M1), dtype=T.dtype, device=T.device) if da is None else _dev(da, "da", T.dtype, (nloc, M1))
+    fn = getattr(_lib, f"dp_{kind}_head_grad_{_suffix(T.dtype)}")
+    _check(fn(_ptr(T), _ptr(a), _ptr(dout), nloc, M1, _ptr(dT), _ptr(da), int(bool(accumulate)), _stream(T)))
+    return dT, da
+
+
+def dp_vector_head_grad(T, a, dv, dT=None, da=None, accumulate=False):
+    """(dT [nloc][4][M1], da [nloc][M1]) from dE/dv [nloc][3]; accumulate adds the head's dT to dT."""
+    return _head_grad("vector", T, a, dv, (3,), dT, da, accumulate)
+
+
+def dp_tensor_head_grad(T, a, dA, dT=None, da=None, accumulate=False):
+    """(dT [nloc][4][M1], da [nloc][M1]) from dE/dA [nloc][3][3]; accumulate adds the head's dT to dT."""
+    return _head_grad("tensor", T, a, dA, (3, 3), dT, da, accumulate)

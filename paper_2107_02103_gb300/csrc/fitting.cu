@@ -86,8 +86,10 @@ struct FitGemm {
   const io_t<real> *wo;  // output-layer weights [K]
   const io_t<real> *T;
   int64_t ldT;
-  const io_t<real> *W;     // forward: W [K][N]; backward: W [N][K] read as its transpose
-  const io_t<real> *bias;  // forward: [N]
+  const io_t<real> *W;     // forward: W [K][N] (wt: W [N][K] read as its transpose); backward: W [N][K] transposed
+  const io_t<real> *bias;  // forward: [N], NULL (lin only) for none
+  bool lin;                // forward: out = acc + bias, no tanh (an output layer of several outputs, or g W^T)
+  bool wt;                 // forward: read W as [N][K]
   bool skip;               // backward: add S(i, n) (the layer had an identity skip)
   io_t<real> *out;
   int64_t ldo;
@@ -113,7 +115,7 @@ __device__ __forceinline__ real load_a(const FitGemm<real> &P, int64_t row, int 
 template <typename real, bool kFwd>
 __device__ __forceinline__ real load_b(const FitGemm<real> &P, int k, int nn) {
   if constexpr (kFwd)
-    return from_io<real>(P.W[(size_t)k * P.N + nn]);
+    return from_io<real>(P.wt ? P.W[(size_t)nn * P.K + k] : P.W[(size_t)k * P.N + nn]);
   else
     return from_io<real>(P.W[(size_t)nn * P.K + k]);
 }
@@ -171,7 +173,10 @@ __global__ void __launch_bounds__(kFitThreads) fit_gemm_kernel(const FitGemm<rea
       if (nn >= P.N) continue;
       real v = acc[p][q];
       if constexpr (kFwd) {
-        v = tanh_r(v + from_io<real>(P.bias[nn]));
+        if (P.lin)
+          v = P.bias ? v + from_io<real>(P.bias[nn]) : v;
+        else
+          v = tanh_r(v + from_io<real>(P.bias[nn]));
       } else if (P.skip) {
         const int64_t r = P.r0 + row;
         v += P.S ? from_io<real>(P.S[r * P.ldS + nn])
@@ -197,7 +202,7 @@ __global__ void __launch_bounds__(128) fit_out_kernel(const FitGemm<real> P, con
 }
 
 struct FitShape {
-  int nlayer, ntypes;
+  int nlayer, ntypes, nout;  // nout = widths[nlayer], the outputs per atom
   int w[DP_MAX_LAYERS + 1];
   int64_t P;       // parameters per type
   int64_t H;       // sum of hidden widths (row length of act)
@@ -207,13 +212,18 @@ struct FitShape {
   int64_t start[DP_MAX_TYPES + 1];
 };
 
-int fit_shape(const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start, FitShape *s) {
+// multi: whether the output layer may have several outputs (the FMA-pipe kernels); the tensor-core
+// net has one (the energy).
+int fit_shape(const int32_t *widths, int nlayer, int ntypes, const int64_t *type_start, FitShape *s,
+              bool multi = false) {
   if (!widths || !type_start) return set_error(DP_ERR_NULL, "widths or type_start is NULL");
   if (nlayer < 1 || nlayer > DP_MAX_LAYERS)
     return set_error(DP_ERR_UNSUPPORTED, "nlayer = %d outside [1, %d]", nlayer, DP_MAX_LAYERS);
   if (ntypes < 1 || ntypes > DP_MAX_TYPES)
     return set_error(DP_ERR_UNSUPPORTED, "ntypes = %d outside [1, %d]", ntypes, DP_MAX_TYPES);
-  if (widths[nlayer] != 1) return set_error(DP_ERR_SHAPE, "the output layer has width %d, not 1", widths[nlayer]);
+  if (!multi && widths[nlayer] != 1)
+    return set_error(DP_ERR_SHAPE, "the output layer has width %d, not 1", widths[nlayer]);
+  s->nout = widths[nlayer];
   s->nlayer = nlayer;
   s->ntypes = ntypes;
   s->P = 0;
@@ -273,7 +283,7 @@ int fitting_fwd(const io_t<real> *params, const int32_t *widths, int nlayer, int
                 const io_t<real> *D, io_t<real> *E, io_t<real> *act, void *stream) {
   clear_error();
   FitShape s{};
-  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
+  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s, true);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
   if (nloc == 0) return DP_OK;
@@ -298,11 +308,21 @@ int fitting_fwd(const io_t<real> *params, const int32_t *widths, int nlayer, int
       if (rc) return rc;
     }
     G.K = s.w[nlayer - 1];
-    G.N = 1;
     chain_sources<real>(s, nlayer, D, act, G);
-    G.wo = pt + s.woff[nlayer];
-    fit_out_kernel<real><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(G, G.wo + G.K, E);
-    rc = launch_status("dp_fitting_fwd");
+    if (s.nout == 1) {  // E_i = v . wo + bo: a dot product per atom
+      G.N = 1;
+      G.wo = pt + s.woff[nlayer];
+      fit_out_kernel<real><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(G, G.wo + G.K, E);
+      rc = launch_status("dp_fitting_fwd");
+    } else {  // E_i = v W_out + b_out: a GEMM without tanh
+      G.N = s.nout;
+      G.W = pt + s.woff[nlayer];
+      G.bias = G.W + (size_t)G.K * G.N;
+      G.lin = true;
+      G.out = E;
+      G.ldo = s.nout;
+      rc = launch_gemm<real, true>(G, st, "dp_fitting_fwd");
+    }
     if (rc) return rc;
   }
   return DP_OK;
@@ -313,12 +333,13 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
                  const io_t<real> *act, const io_t<real> *g, io_t<real> *dD, io_t<real> *work, void *stream) {
   clear_error();
   FitShape s{};
-  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
+  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s, true);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
   if (nloc == 0) return DP_OK;
-  if (!params || !dD || (s.H > 0 && !act) || (nlayer > 2 && !work))
+  if (!params || !dD || (s.H > 0 && !act) || ((nlayer > 2 || s.nout > 1) && !work))
     return set_error(DP_ERR_NULL, "dp_fitting_grad: NULL array");
+  if (s.nout > 1 && !g) return set_error(DP_ERR_NULL, "dp_fitting_grad: g is NULL for a net of %d outputs", s.nout);
   const cudaStream_t st = (cudaStream_t)stream;
   io_t<real> *buf[2] = {work, work ? work + (size_t)nloc * s.maxh : nullptr};
   for (int t = 0; t < ntypes; ++t) {
@@ -334,6 +355,25 @@ int fitting_grad(const io_t<real> *params, const int32_t *widths, int nlayer, in
     const io_t<real> *S = nullptr;  // dE/dv of the layer being walked; NULL: g wo (the last hidden layer)
     int64_t ldS = 0;
     int cur = 0;
+    if (s.nout > 1) {  // dE/dv_{nlayer-1} = g W_out^T, [n][nout] x [nout][widths[nlayer-1]], first
+      FitGemm<real> Z{};
+      Z.r0 = G.r0;
+      Z.n = n;
+      Z.K = s.nout;
+      Z.N = s.w[nlayer - 1];
+      Z.src[0] = g;
+      Z.lds[0] = s.nout;
+      Z.nsrc = 1;
+      Z.W = pt + s.woff[nlayer];  // W_out [widths[nlayer-1]][nout], read transposed
+      Z.wt = true;
+      Z.lin = true;
+      Z.out = buf[0];
+      Z.ldo = s.maxh;
+      if ((rc = launch_gemm<real, true>(Z, st, "dp_fitting_grad"))) return rc;
+      S = buf[0];
+      ldS = s.maxh;
+      cur = 1;
+    }
     for (int l = nlayer - 1; l >= 1; --l) {
       G.K = s.w[l];      // contraction over the layer's outputs
       G.N = s.w[l - 1];  // producing dE/dv_{l-1}
@@ -700,10 +740,10 @@ int fitting_grad_noalloc(const double *params, const int32_t *widths, int nlayer
                          const int64_t *type_start, const double *act, const double *g, double *dD, void *stream) {
   clear_error();
   FitShape s{};
-  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
+  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s, true);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
-  const size_t need = nlayer > 2 ? (size_t)2 * (size_t)nloc * (size_t)s.maxh : 0;
+  const size_t need = (nlayer > 2 || s.nout > 1) ? (size_t)2 * (size_t)nloc * (size_t)s.maxh : 0;
   if (need > kStaticScratchDoubles)
     return set_error(DP_ERR_UNSUPPORTED,
                      "dp_fitting_grad_noalloc: needs 2 x %lld atoms x %d = %zu doubles of scratch, the static array "

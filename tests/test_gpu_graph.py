@@ -70,3 +70,43 @@ def test_whole_model_replays_as_a_cuda_graph():
     assert torch.equal(buf["dD"], eager["dD"])
     for k in ("F", "virial"):                        # forces and virial add with atomics
         assert rel(buf[k].cpu().numpy(), eager[k].cpu().numpy()) <= 1e-13, k
+
+
+def test_tc_calls_replay_as_a_cuda_graph():
+    """The tensor-core forward (writing D) and backward (reusing the forward's runs) captured as a graph
+    at a size of several backward GEMM units per CTA: the replays give the eager bits."""
+    dpc = lib()
+    w = W.make("water", seed=67, nmol=1536)  # 4,608 atoms
+    info = dpc.dp_table_info_make(w.s_min, w.s_max, w.stride0, w.stride1, w.ext)
+    model = dpc.Model.compress(torch.from_numpy(w.params).cuda(), w.widths, info, torch.float64)
+    plan = dpc.dp_tabulate_tc_plan_f64(model.table, info, w.nnei)
+    x = {k: torch.from_numpy(getattr(w, k)).cuda() for k in ("s", "Rt", "dT", "nvalid", "atype")}
+    f64 = dict(dtype=torch.float64, device="cuda")
+    buf = dict(T=torch.empty((w.nloc, 4, w.M1), **f64), D=torch.empty((w.nloc, w.M1, w.M2), **f64),
+               ds=torch.empty((w.nloc, w.nnei), **f64), dRt=torch.empty((w.nloc, w.nnei, 4), **f64),
+               work=torch.empty((dpc.dp_tabulate_tc_work_bytes(info, w.nloc, w.nnei, w.ntypes, w.M1),),
+                                dtype=torch.uint8, device="cuda"))
+    args = (plan, info, x["s"], x["Rt"], x["nvalid"], x["atype"], [int(v) for v in w.sel])
+
+    def step():
+        dpc.dp_tabulate_fusion_fwd_tc_f64(*args, out=buf["T"], work=buf["work"], M2=w.M2, D=buf["D"])
+        dpc.dp_tabulate_fusion_grad_tc_f64(*args, x["dT"], out=(buf["ds"], buf["dRt"]), work=buf["work"],
+                                           flags=dpc.DP_TC_REUSE_RUNS)
+
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()  # eager, on the capture stream: the one-time setup of the calls
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    eager = {k: buf[k].clone() for k in ("T", "D", "ds", "dRt")}
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+        step()
+    for k in eager:
+        buf[k].fill_(float("nan"))  # the replays must rewrite every output
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    for k in eager:
+        assert torch.equal(buf[k], eager[k]), k
