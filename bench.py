@@ -93,11 +93,16 @@ KERNEL_API = {"fwd": "dp_tabulate_fusion_fwd", "grad": "dp_tabulate_fusion_grad"
               "fitting_grad": "dp_fitting_grad", "env_mat": "dp_env_mat", "force_virial": "dp_force_virial"}
 
 
-def fitting_model(w):
+def fitting_model(w, head=None):
     """The fitting net of the --fitting chain: the paper's (240, 240, 240) hidden layers per centre type
-    on the flattened descriptor, random-init (seeded) weights."""
+    on the flattened descriptor, random-init (seeded) weights; one output (the energy), or M1 (the
+    weights of a vector or tensor head)."""
     import workloads as W
-    return W.fitting_net(W._sub_seed(w.seed, 606), w.M1 * w.M2, (240, 240, 240), w.ntypes)
+    widths, params = W.fitting_net(W._sub_seed(w.seed, 606), w.M1 * w.M2, (240, 240, 240), w.ntypes)
+    if head:
+        widths = widths[:-1] + [w.M1]
+        params = W.net_params(W._sub_seed(w.seed, 607), widths, w.ntypes)
+    return widths, params
 
 
 def fitting_fmas(w, widths) -> dict:
@@ -398,7 +403,7 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
     env = dpc.env_info(w.env["rcs"], w.env["rc"], w.env["kind"], nv)
     host = {"coord": np.ascontiguousarray(coord.astype(npdt)), "nlist": nlist, "atype": w.atype}
     if args.fitting:  # the energy of the whole model: dE/dD comes from the fitting net
-        fwidths, fparams = fitting_model(w)
+        fwidths, fparams = fitting_model(w, args.head)
         fpar = torch.from_numpy(np.ascontiguousarray(fparams.astype(npdt))).to(dev)  # parameters stay resident
         ts = [0] + [int(x) for x in np.cumsum(w.ncentre())]
     else:
@@ -417,9 +422,17 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
         names.remove("descriptor")
     if fused_env:
         names = [n for n in names if n not in ("env_mat", "force_virial")]
+    if args.head:  # dE/dv or dE/dA of the vector or tensor model: a resident synthetic input
+        hshape = (w.nloc, 3) if args.head == "vector" else (w.nloc, 3, 3)
+        host["dhead"] = np.ascontiguousarray(W.normal(W._sub_seed(w.seed, 405), hshape).astype(npdt))
+        d["dhead"] = torch.from_numpy(host["dhead"]).to(dev)
+        outs["head"] = torch.empty(hshape, dtype=dtype, device=dev)
+        work["da"] = torch.empty((w.nloc, w.M1), dtype=dtype, device=dev)
+        head_fwd = dpc.dp_vector_head if args.head == "vector" else dpc.dp_tensor_head
+        head_grad = dpc.dp_vector_head_grad if args.head == "vector" else dpc.dp_tensor_head_grad
     if args.fitting:
         H = sum(fwidths[1:-1])
-        outs["E"] = torch.empty((w.nloc,), dtype=dtype, device=dev)
+        outs["E"] = torch.empty((w.nloc, fwidths[-1]) if args.head else (w.nloc,), dtype=dtype, device=dev)
         work["act"] = torch.empty((w.nloc, H), dtype=dtype, device=dev)
         work["dD"] = torch.empty((w.nloc, w.M1 * w.M2), dtype=dtype, device=dev)
         work["fit_scratch"] = torch.empty((2, w.nloc, max(fwidths[1:-1])), dtype=dtype, device=dev)
@@ -428,6 +441,9 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
                                          device=dev)
         names = ["env_mat", "fwd", "descriptor", "fitting_fwd", "fitting_grad", "descriptor_grad", "grad",
                  "force_virial"]
+        if args.head:
+            names = ["env_mat", "fwd", "descriptor", "fitting_fwd", "head", "head_grad_da", "fitting_grad",
+                     "descriptor_grad", "head_grad_dT", "grad", "force_virial"]
         if fused_d:
             names.remove("descriptor")
         if fused_env:
@@ -460,14 +476,22 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
         elif args.fitting:
             dpc.dp_fitting_fwd(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), arith=arith)
             rec(k := k + 1)
-            dpc.dp_fitting_grad(fpar, fwidths, ts, work["act"], out=work["dD"], work=work["fit_scratch"],
-                                arith=arith)
+            if args.head:  # v or A from T and the net's M1 outputs; dE/da for the net's backward
+                head_fwd(work["T"], o["E"], out=o["head"])
+                rec(k := k + 1)
+                head_grad(work["T"], o["E"], x["dhead"], da=work["da"], want=("da",))
+                rec(k := k + 1)
+            dpc.dp_fitting_grad(fpar, fwidths, ts, work["act"], g=work["da"] if args.head else None,
+                                out=work["dD"], work=work["fit_scratch"], arith=arith)
             rec(k := k + 1)
             dD_in = work["dD"].view(w.nloc, w.M1, w.M2)
         else:
             dD_in = x["dD"]
         dpc.dp_descriptor_contract_grad(work["T"], dD_in, out=work["dT"], arith=arith)
         rec(k := k + 1)
+        if args.head:  # the head's own dE/dT added to the descriptor's
+            head_grad(work["T"], o["E"], x["dhead"], dT=work["dT"], accumulate=True, want=("dT",))
+            rec(k := k + 1)
         if fused_env:  # dE/dT -> forces and virial in one call, on the forward's interval runs
             dpc.dp_tabulate_fusion_env_grad_tc_f64(plan, info, x["coord"], x["nlist"], sel, env, x["atype"], work["dT"],
                                                    out=(o["F"], o["virial"]), work=tcw, flags=dpc.DP_TC_REUSE_RUNS)
@@ -735,7 +759,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     if "descriptor" not in k_ms:  # the forward wrote D as well (tensor-core path)
         flops["fwd"] += flops["descriptor"]
     if getattr(args, "fitting", False):
-        flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w)[0]).items()})
+        flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w, args.head)[0]).items()})
     nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
     nsm = getattr(args, "nsm", NSM)
     pk = peak_tflops(args.dtype, nsm=nsm)
@@ -801,7 +825,11 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         "config": {"workload": workload_label(w),
                    "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
                                    else f"atoms split over {world} ranks"),
-                   "step": (("env_mat + fwd + descriptor + fitting_fwd + fitting_grad + descriptor_grad + grad + "
+                   "step": ((f"env_mat + fwd + descriptor + fitting_fwd (M1 outputs) + {args.head}_head + its "
+                             "backward + fitting_grad + descriptor_grad + grad + force_virial (the "
+                             f"{args.head} model and the forces of <dE/d{args.head}, {args.head}>)")
+                            if args.head else
+                            ("env_mat + fwd + descriptor + fitting_fwd + fitting_grad + descriptor_grad + grad + "
                              "force_virial (energy and forces of the whole model)") if args.fitting else
                             "env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain
                             else "fwd + descriptor + grad" if "descriptor" in k_ms
@@ -960,6 +988,9 @@ def main():
                     help="time the whole chain from coordinates to forces (env_mat ... force_virial)")
     ap.add_argument("--fitting", action="store_true",
                     help="with --chain: add the fitting net, so the step yields the model's energy and forces")
+    ap.add_argument("--head", choices=["vector", "tensor"], default=None,
+                    help="with --fitting (FMA-pipe net): a vector or tensor model, the net's M1 outputs weighting "
+                         "T's rotation-covariant rows; the backward is that of <dE/dv, v> (dE/dv synthetic)")
     ap.add_argument("--fitting-tc", action="store_true",
                     help="with --fitting and double arrays (f64, df64): the fitting net's f64 GEMMs on the tensor "
                          "cores (exact splitting)")
@@ -976,6 +1007,8 @@ def main():
         ap.error("--fitting extends the --chain step")
     if args.fitting_tc and (not args.fitting or args.dtype not in ("f64", "df64")):
         ap.error("--fitting-tc needs --fitting and double arrays (--dtype f64 or df64)")
+    if args.head and (not args.fitting or args.fitting_tc or args.dtype == "df64"):
+        ap.error("--head needs --fitting with the FMA-pipe net (not --fitting-tc) in f64 or f32")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -655,6 +655,9 @@ int dp_fitting_grad_tc_f64(const double *params, const int32_t *widths, int nlay
  *       accumulate is 0; otherwise the head's dT is added to what dT holds
  *       (dE/dT of the descriptor, dp_descriptor_contract_grad_*), row 0 kept
  *   da  [nloc][M1] output (the upstream g of dp_fitting_grad_*)
+ * Either output of the backward may be NULL (not computed), not both: a
+ * model's backward takes da first (for the fitting net's backward, which
+ * leads to the descriptor's dT) and then adds the head's dT to that.
  * All arrays device, row-major, caller-owned; nothing is allocated.
  * Errors: DP_ERR_NULL, DP_ERR_SHAPE (nloc < 0, M1 outside [1, 4096]),
  * DP_ERR_CUDA.  nloc == 0 reads no device pointer.

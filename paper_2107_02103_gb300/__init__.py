@@ -872,26 +872,36 @@ def dp_tensor_head(T, a, out=None):
     return A
 
 
-def _head_grad(kind, T, a, dout, shape, dT, da, accumulate):
+def _head_grad(kind, T, a, dout, shape, dT, da, accumulate, want):
     T, a, nloc, M1 = _head_inputs(T, a)
     dout = _dev(dout, "dout", T.dtype, (nloc,) + shape)
-    if dT is None:
+    if not want or set(want) - {"dT", "da"}:
+        raise ValueError("want names dT, da or both")
+    if "dT" not in want:
+        dT = None
+    elif dT is None:
         if accumulate:
             raise ValueError("accumulate needs the dT to add to")
         dT = torch.empty((nloc, 4, M1), dtype=T.dtype, device=T.device)
     else:
         dT = _dev(dT, "dT", T.dtype, (nloc, 4, M1))
-    da = torch.empty((nloc, M1), dtype=T.dtype, device=T.device) if da is None else _dev(da, "da", T.dtype, (nloc, M1))
+    if "da" not in want:
+        da = None
+    else:
+        da = torch.empty((nloc, M1), dtype=T.dtype, device=T.device) if da is None else \
+            _dev(da, "da", T.dtype, (nloc, M1))
     fn = getattr(_lib, f"dp_{kind}_head_grad_{_suffix(T.dtype)}")
     _check(fn(_ptr(T), _ptr(a), _ptr(dout), nloc, M1, _ptr(dT), _ptr(da), int(bool(accumulate)), _stream(T)))
     return dT, da
 
 
-def dp_vector_head_grad(T, a, dv, dT=None, da=None, accumulate=False):
-    """(dT [nloc][4][M1], da [nloc][M1]) from dE/dv [nloc][3]; accumulate adds the head's dT to dT."""
-    return _head_grad("vector", T, a, dv, (3,), dT, da, accumulate)
+def dp_vector_head_grad(T, a, dv, dT=None, da=None, accumulate=False, want=("dT", "da")):
+    """(dT [nloc][4][M1], da [nloc][M1]) from dE/dv [nloc][3]; accumulate adds the head's dT to dT;
+    want: the outputs to compute (the other is returned as None)."""
+    return _head_grad("vector", T, a, dv, (3,), dT, da, accumulate, want)
 
 
-def dp_tensor_head_grad(T, a, dA, dT=None, da=None, accumulate=False):
-    """(dT [nloc][4][M1], da [nloc][M1]) from dE/dA [nloc][3][3]; accumulate adds the head's dT to dT."""
-    return _head_grad("tensor", T, a, dA, (3, 3), dT, da, accumulate)
+def dp_tensor_head_grad(T, a, dA, dT=None, da=None, accumulate=False, want=("dT", "da")):
+    """(dT [nloc][4][M1], da [nloc][M1]) from dE/dA [nloc][3][3]; accumulate adds the head's dT to dT;
+    want: the outputs to compute (the other is returned as None)."""
+    return _head_grad("tensor", T, a, dA, (3, 3), dT, da, accumulate, want)

@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(kHeadThreads)
   const real *Ti = T + i * 4 * M1;
   const real t[3] = {__ldg(Ti + M1 + m), __ldg(Ti + 2 * M1 + m), __ldg(Ti + 3 * M1 + m)};
   const real am = __ldg(a + e);
-  real *dTi = dT + i * 4 * M1;
+  real *dTi = dT ? dT + i * 4 * M1 : nullptr;
   real g[3], dam = real(0);
   if constexpr (kTensor) {
     const real *G = dout + i * 9;
@@ -101,7 +101,8 @@ __global__ void __launch_bounds__(kHeadThreads)
       dam = fma(dv, t[c], dam);
     }
   }
-  if (accumulate) {
+  if (!dT) {  // launch-uniform: only da wanted
+  } else if (accumulate) {
 #pragma unroll
     for (int c = 0; c < 3; ++c) dTi[(1 + c) * M1 + m] += g[c];
   } else {
@@ -109,7 +110,7 @@ __global__ void __launch_bounds__(kHeadThreads)
 #pragma unroll
     for (int c = 0; c < 3; ++c) dTi[(1 + c) * M1 + m] = g[c];
   }
-  da[e] = dam;
+  if (da) da[e] = dam;
 }
 
 int head_check(const void *T, const void *a, const void *x, const void *y, int64_t nloc, int M1, const char *who) {
@@ -134,9 +135,8 @@ template <typename real, bool kTensor>
 int head_grad(const real *T, const real *a, const real *dout, int64_t nloc, int M1, real *dT, real *da,
               int accumulate, void *stream, const char *who) {
   clear_error();
-  int rc = head_check(T, a, dout, dT, nloc, M1, who);
+  int rc = head_check(T, a, dout, dT ? (const void *)dT : (const void *)da, nloc, M1, who);
   if (rc || nloc == 0) return rc;
-  if (!da) return set_error(DP_ERR_NULL, "%s: NULL array", who);
   const int64_t blocks = (nloc * M1 + kHeadThreads - 1) / kHeadThreads;
   if (blocks > 0x7fffffffLL) return set_error(DP_ERR_SHAPE, "%s: nloc = %lld too large", who, (long long)nloc);
   head_grad_kernel<real, kTensor><<<(unsigned)blocks, kHeadThreads, 0, (cudaStream_t)stream>>>(

@@ -48,6 +48,10 @@ def test_heads_against_oracle(dtype, nloc, M1):
     dTA, daA = dpc.dp_tensor_head_grad(Tg, ag, _cast(dA, dtype))
     acc = _cast(base, dtype)
     dpc.dp_tensor_head_grad(Tg, ag, _cast(dA, dtype), dT=acc, accumulate=True)
+    none_dT, da_only = dpc.dp_vector_head_grad(Tg, ag, _cast(dv, dtype), want=("da",))
+    acc_v = _cast(base, dtype)
+    _, none_da = dpc.dp_vector_head_grad(Tg, ag, _cast(dv, dtype), dT=acc_v, accumulate=True, want=("dT",))
+    assert none_dT is None and none_da is None
     torch.cuda.synchronize()
     if nloc == 0:
         assert v.shape == (0, 3) and A.shape == (0, 3, 3)
@@ -63,10 +67,11 @@ def test_heads_against_oracle(dtype, nloc, M1):
         assert rel(dTg.double().cpu().numpy(), dTo) <= tol
         assert not dTg[:, 0].any()
         assert rel(dag.double().cpu().numpy(), dao) <= tol
-    dTo = o.tensor_head_grad(T, a, dA)[0]
-    got = acc.double().cpu().numpy()
-    assert np.array_equal(got[:, 0], base[:, 0].astype(NP[dtype]).astype(np.float64))
-    assert rel(got, base + dTo) <= tol
+    assert torch.equal(da_only, dav)  # one output alone: the same bits
+    for accg, (dTo, _) in ((acc, o.tensor_head_grad(T, a, dA)), (acc_v, o.vector_head_grad(T, a, dv))):
+        got = accg.double().cpu().numpy()
+        assert np.array_equal(got[:, 0], base[:, 0].astype(NP[dtype]).astype(np.float64))
+        assert rel(got, base + dTo) <= tol
 
 
 def test_head_refusals():
