@@ -316,6 +316,7 @@ MOMENT_CASES = [
     ("cu85", dict(cells=(6, 6, 6)), torch.float64, None), ("cu85", dict(cells=(6, 6, 6)), torch.float32, None),
     ("alcumg", dict(pad=0.1, cells=(6, 6, 6)), torch.float64, None),
     ("cu85", {}, torch.float64, None), ("alcumg", dict(pad=0.3), torch.float64, 384),
+    ("cu85", {}, torch.float32, None), ("water", {}, torch.float32, 512),
 ]
 
 
@@ -404,15 +405,20 @@ def test_moments_grad_shapes(M1, widths):
         assert_parity(got, ref, dtype, keys=("ds", "dRt"))
 
 
-def test_moments_grad_no_valid_rows():
-    """Atoms without real neighbours: every row is padding and gets zeros over stale outputs."""
+@pytest.mark.parametrize("dtype", [torch.float64, torch.float32])
+def test_moments_grad_no_valid_rows(dtype):
+    """Atoms without real neighbours: every row is padding and gets zeros over stale outputs, and T is
+    zero, in f64 and f32."""
     dpc = lib()
-    w = W.tiny(seed=7, nloc=3, nreal=5, sel=8)
-    model = product_model(w, torch.float64)
-    x = to_dev(w, torch.float64)
-    stale = (torch.ones((w.nloc, w.nnei), dtype=torch.float64, device="cuda"),
-             torch.ones((w.nloc, w.nnei, 4), dtype=torch.float64, device="cuda"))
-    ds, dRt = dpc.dp_tabulate_fusion_grad_moments(model.table, model.info, x["s"], x["Rt"],
-                                                  torch.zeros_like(x["nvalid"]), x["atype"], w.sel, x["dT"], out=stale)
+    w = W.tiny(seed=7, nloc=3, nreal=5, sel=80)
+    model = product_model(w, dtype)
+    x = to_dev(w, dtype)
+    stale = (torch.ones((w.nloc, w.nnei), dtype=dtype, device="cuda"),
+             torch.ones((w.nloc, w.nnei, 4), dtype=dtype, device="cuda"))
+    nv0 = torch.zeros_like(x["nvalid"])
+    ds, dRt = dpc.dp_tabulate_fusion_grad_moments(model.table, model.info, x["s"], x["Rt"], nv0, x["atype"], w.sel,
+                                                  x["dT"], out=stale)
+    T = dpc.dp_tabulate_fusion_fwd_moments(model.table, model.info, x["s"], x["Rt"], nv0, x["atype"], w.sel,
+                                           out=torch.ones((w.nloc, 4, w.M1), dtype=dtype, device="cuda"))
     torch.cuda.synchronize()
-    assert not ds.abs().max().item() and not dRt.abs().max().item()
+    assert not ds.abs().max().item() and not dRt.abs().max().item() and not T.abs().max().item()
