@@ -748,6 +748,7 @@ def measure_e2e(args, host, d, outs, step, stream, dev, world, barrier, evals_al
 
 def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, fmas=None, nall=0, tc_ms=None,
            tcf=None, tc_launches=None):
+    head = getattr(args, "head", None)  # a vector or tensor model
     value = evals_all * args.steps / total_s
     # ---- roofline of the dominant kernel (FMA pipe of the path's dtype), on the FMAs of the
     # algorithm the kernels run: per-row evaluation, or interval moments (fmas, from the run lengths)
@@ -759,7 +760,7 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
     if "descriptor" not in k_ms:  # the forward wrote D as well (tensor-core path)
         flops["fwd"] += flops["descriptor"]
     if getattr(args, "fitting", False):
-        flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w, args.head)[0]).items()})
+        flops.update({k: 2.0 * v for k, v in fitting_fmas(w, fitting_model(w, getattr(args, "head", None))[0]).items()})
     nbytes = chain_bytes(w, 4 if args.dtype == "f32" else 8, nall) if args.chain else {}
     nsm = getattr(args, "nsm", NSM)
     pk = peak_tflops(args.dtype, nsm=nsm)
@@ -825,10 +826,10 @@ def report(args, w, world, step_ms, k_ms, total_s, evals_all, e2e, clk, t_wall, 
         "config": {"workload": workload_label(w),
                    "parallelism": (f"replicas x{world} (independent seeded instances)" if args.scaling == "weak"
                                    else f"atoms split over {world} ranks"),
-                   "step": ((f"env_mat + fwd + descriptor + fitting_fwd (M1 outputs) + {args.head}_head + its "
+                   "step": ((f"env_mat + fwd + descriptor + fitting_fwd (M1 outputs) + {head}_head + its "
                              "backward + fitting_grad + descriptor_grad + grad + force_virial (the "
-                             f"{args.head} model and the forces of <dE/d{args.head}, {args.head}>)")
-                            if args.head else
+                             f"{head} model and the forces of <dE/d{head}, {head}>)")
+                            if head else
                             ("env_mat + fwd + descriptor + fitting_fwd + fitting_grad + descriptor_grad + grad + "
                              "force_virial (energy and forces of the whole model)") if args.fitting else
                             "env_mat + fwd + descriptor + descriptor_grad + grad + force_virial" if args.chain

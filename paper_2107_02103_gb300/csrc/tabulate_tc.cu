@@ -27,15 +27,21 @@
 // slices (forward) or output tiles (backward) that no atom of a tile uses.
 //
 // C'_alpha and its digit planes are made once per table by dp_tabulate_tc_plan_f64 (the plan).
-// Per chunk of at most kChunkAtoms atoms and per centre type alpha:
-//   forward:  runs_kernel<true> (slot keys, W, column exponents, slice flags), slice_list_kernel,
-//             tgemm_kernel (tab_gemm.cuh; A = C'_alpha^T: channels x K, B = W^T: K x (atom, k), its
-//             digit planes made in shared memory from W; a tile whose used slices fit one share
-//             writes its atoms' T directly),
-//             fwd_finish_kernel (T of the atoms whose items were cut into pieces, or have none; D);
+// Per chunk of at most kChunkAtoms atoms:
+//   forward:  runs_kernel<true> (slot keys, W, column exponents, slice flags), slice_list_kernel (each
+//             tile's used slices), fwd_schedule_kernel (every centre type's items cut into pieces of
+//             equal cost per CTA), tgemm_kernel<true> (tab_gemm.cuh, one launch; A = C'_alpha^T:
+//             channels x K, B = W^T: K x (atom, k), its digit planes made in shared memory from W; an
+//             uncut item writes its atoms' T, a piece its exact 128-bit partial sums),
+//             fwd_finish_kernel (T of the cut items, and D_i = T_i^T T_i[:, :M2] when asked for);
 //   backward: runs_kernel<false> (slot keys, slice flags; skipped when the forward's are reused),
-//             split of dT (B), tgemm_kernel (A = C'_alpha: K x channels, B = dT^T) scattering
-//             each used (atom, interval) block to its run slot, rows_kernel (dE/ds, dE/dR~).
+//             the split of dT (B), the GEMM units, and per centre type the GEMM (A = C'_alpha: K x
+//             channels, B = dT^T) scattering each used (atom, interval) block to its run slot --
+//             bgemm_kernel (tab_gemm_b8.cuh: 8-atom tiles, seven 8-bit digits) when M1 rounds up to
+//             at most 144, else tgemm_kernel<false> (12-atom tiles, nine 6-bit digits) -- and
+//             rows_kernel (dE/ds, dE/dR~).
+// The environment-fused calls (dp_tabulate_fusion_env_*_tc_f64) form each row from coordinates in
+// runs_kernel<.., true> and add each row's force and virial in rows_force_kernel instead.
 // The slot keys, their counts and the slice flags of every atom stay in the work buffer after
 // the forward, so that a backward on the same inputs can skip its own key pass.
 #include <cuda_runtime.h>

@@ -130,3 +130,22 @@ def test_report_takes_the_roofline_on_the_dominant_tc_kernel():
         assert abs(st["hbm_ms"] - hbm_ms) < 1e-4
         assert st["t_roof_ms"] == max(st["fp64_ms"], st["tensor_ms"], st["hbm_ms"])
         assert abs(st["frac"] - st["t_roof_ms"] / 1.0) < 1e-4
+
+
+def test_head_options_and_their_fitting_net(monkeypatch):
+    """--head needs the FMA-pipe fitting net of the chain (refused before any device work otherwise),
+    and its net ends in M1 outputs, the head's weights, where the energy model's ends in one."""
+    import pytest
+    for argv in (["--head", "vector"], ["--chain", "--head", "tensor"],
+                 ["--chain", "--fitting", "--fitting-tc", "--head", "vector"],
+                 ["--chain", "--fitting", "--dtype", "df64", "--head", "vector"]):
+        monkeypatch.setattr("sys.argv", ["bench.py", *argv])
+        with pytest.raises(SystemExit) as e:
+            bench.main()
+        assert e.value.code == 2, argv
+    w = W.tiny()
+    we, pe = bench.fitting_model(w)
+    wv, pv = bench.fitting_model(w, "vector")
+    assert we[-1] == 1 and wv[-1] == w.M1 and we[:-1] == wv[:-1]
+    P = sum((wv[l - 1] + 1) * wv[l] for l in range(1, len(wv)))
+    assert pv.shape == (w.ntypes, P)
