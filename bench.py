@@ -467,22 +467,24 @@ def build_step(args, w, dpc, model, info, sel, dtype, npdt, dev):
             rec(k := k + 1)
             dpc.dp_descriptor_contract(work["T"], w.M2, out=o["D"], arith=arith)
         rec(k := k + 1)
-        if args.fitting and args.fitting_tc:
-            dpc.dp_fitting_fwd_tc_f64(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), work=work["fit_tc"])
-            rec(k := k + 1)
-            dpc.dp_fitting_grad_tc_f64(fpar, fwidths, ts, work["act"], out=work["dD"], work=work["fit_tc"])
-            rec(k := k + 1)
-            dD_in = work["dD"].view(w.nloc, w.M1, w.M2)
-        elif args.fitting:
-            dpc.dp_fitting_fwd(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), arith=arith)
+        if args.fitting:
+            if args.fitting_tc:
+                dpc.dp_fitting_fwd_tc_f64(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), work=work["fit_tc"])
+            else:
+                dpc.dp_fitting_fwd(fpar, fwidths, ts, o["D"], out=(o["E"], work["act"]), arith=arith)
             rec(k := k + 1)
             if args.head:  # v or A from T and the net's M1 outputs; dE/da for the net's backward
                 head_fwd(work["T"], o["E"], out=o["head"])
                 rec(k := k + 1)
                 head_grad(work["T"], o["E"], x["dhead"], da=work["da"], want=("da",))
                 rec(k := k + 1)
-            dpc.dp_fitting_grad(fpar, fwidths, ts, work["act"], g=work["da"] if args.head else None,
-                                out=work["dD"], work=work["fit_scratch"], arith=arith)
+            g_fit = work["da"] if args.head else None
+            if args.fitting_tc:
+                dpc.dp_fitting_grad_tc_f64(fpar, fwidths, ts, work["act"], g=g_fit, out=work["dD"],
+                                           work=work["fit_tc"])
+            else:
+                dpc.dp_fitting_grad(fpar, fwidths, ts, work["act"], g=g_fit, out=work["dD"],
+                                    work=work["fit_scratch"], arith=arith)
             rec(k := k + 1)
             dD_in = work["dD"].view(w.nloc, w.M1, w.M2)
         else:
@@ -990,8 +992,8 @@ def main():
     ap.add_argument("--fitting", action="store_true",
                     help="with --chain: add the fitting net, so the step yields the model's energy and forces")
     ap.add_argument("--head", choices=["vector", "tensor"], default=None,
-                    help="with --fitting (FMA-pipe net): a vector or tensor model, the net's M1 outputs weighting "
-                         "T's rotation-covariant rows; the backward is that of <dE/dv, v> (dE/dv synthetic)")
+                    help="with --fitting: a vector or tensor model, the net's M1 outputs weighting T's "
+                         "rotation-covariant rows; the backward is that of <dE/dv, v> (dE/dv synthetic)")
     ap.add_argument("--fitting-tc", action="store_true",
                     help="with --fitting and double arrays (f64, df64): the fitting net's f64 GEMMs on the tensor "
                          "cores (exact splitting)")
@@ -1008,8 +1010,8 @@ def main():
         ap.error("--fitting extends the --chain step")
     if args.fitting_tc and (not args.fitting or args.dtype not in ("f64", "df64")):
         ap.error("--fitting-tc needs --fitting and double arrays (--dtype f64 or df64)")
-    if args.head and (not args.fitting or args.fitting_tc or args.dtype == "df64"):
-        ap.error("--head needs --fitting with the FMA-pipe net (not --fitting-tc) in f64 or f32")
+    if args.head and (not args.fitting or args.dtype == "df64"):
+        ap.error("--head needs --fitting in f64 or f32")
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

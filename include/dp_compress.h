@@ -530,7 +530,7 @@ int dp_force_virial_f32(const float *coord, const int32_t *nlist, int64_t nloc, 
  * widths widths[0..nlayer] (host), widths[0] = the length of D_i (M1 * M2),
  * widths[nlayer] = nout, the outputs per atom: 1 for the energy, M1 for the
  * weights a_i of the vector and tensor heads (dp_vector_head_*,
- * dp_tensor_head_*; the tensor-core variants below take nout = 1 only):
+ * dp_tensor_head_*):
  *   v_0 = D_i
  *   v_l = tanh(v_{l-1} W_l + b_l) (+ v_{l-1} when widths[l] == widths[l-1]),  0 < l < nlayer
  *   E_i = v_{nlayer-1} W_nlayer + b_nlayer   (nout values)
@@ -622,8 +622,10 @@ int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer
  *                     every call), partial results, and the [nloc][max hidden
  *                     width] buffers between layers.  Calls sharing a work
  *                     buffer must not overlap on the GPU.
- * Errors as the f64 calls, plus DP_ERR_NULL / DP_ERR_SHAPE for a missing,
- * short or misaligned work buffer; widths[nlayer] must be 1 (DP_ERR_SHAPE).
+ * The output layer (a dot product per atom, or with several outputs a GEMM
+ * without tanh) and, with several outputs, the backward's g W_out^T run on
+ * the FP64 pipe.  Errors as the f64 calls, plus DP_ERR_NULL / DP_ERR_SHAPE
+ * for a missing, short or misaligned work buffer.
  */
 size_t dp_fitting_tc_work_bytes(const int32_t *widths, int nlayer, int64_t nloc); /* 0 on bad widths */
 int dp_fitting_fwd_tc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,

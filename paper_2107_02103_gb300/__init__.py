@@ -792,10 +792,10 @@ def dp_fitting_fwd_tc_f64(params, widths, type_start, D, out=None, work=None):
     if D.shape[0] != nloc or D.numel() != nloc * widths[0]:
         raise ValueError(f"D must hold [{nloc}][{widths[0]}]")
     if out is None:
-        E = torch.empty((nloc,), dtype=torch.float64, device=params.device)
+        E = torch.empty(_out_shape(nloc, widths), dtype=torch.float64, device=params.device)
         act = torch.empty((nloc, max(H, 1)), dtype=torch.float64, device=params.device)
     else:
-        E = _dev(out[0], "E", torch.float64, (nloc,))
+        E = _dev(out[0], "E", torch.float64, _out_shape(nloc, widths))
         act = _dev(out[1], "act", torch.float64, (nloc, max(H, 1)))
     work = _tc_work(work, widths, nloc, params.device)
     _check(_lib.dp_fitting_fwd_tc_f64(_ptr(params), w, nlayer, ntypes, ts, _ptr(D), _ptr(E), _ptr(act), _ptr(work),
@@ -809,7 +809,7 @@ def dp_fitting_grad_tc_f64(params, widths, type_start, act, g=None, out=None, wo
     w, nlayer, ntypes, ts, nloc, widths, H = _fit_shape(params, widths, type_start)
     act = _dev(act, "act", torch.float64, (nloc, max(H, 1)))
     if g is not None:
-        g = _dev(g, "g", torch.float64, (nloc,))
+        g = _dev(g, "g", torch.float64, _out_shape(nloc, widths))
     dD = torch.empty((nloc, widths[0]), dtype=torch.float64, device=params.device) if out is None else \
         _dev(out, "out", torch.float64, (nloc, widths[0]))
     work = _tc_work(work, widths, nloc, params.device)

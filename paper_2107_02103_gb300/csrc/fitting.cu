@@ -438,15 +438,18 @@ __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int kspli
   }
 }
 
-// dz of the last hidden layer: Z[row][k] = g_row wo_k (1 - t_k^2), t its tanh outputs
+// dz of the last hidden layer: Z[row][k] = s (1 - t_k^2), t its tanh outputs and s = dE/dv of that layer:
+// g_row wo_k (one output) or S[row][k] (several: g W_out^T, made first)
 __global__ void __launch_bounds__(256) last_dz_kernel(int64_t r0, int64_t n, int K, const double *__restrict__ g,
-                                                      const double *__restrict__ wo, const double *__restrict__ T,
-                                                      int64_t ldT, double *__restrict__ Z, int64_t ldz) {
+                                                      const double *__restrict__ wo, const double *__restrict__ S,
+                                                      int64_t ldS, const double *__restrict__ T, int64_t ldT,
+                                                      double *__restrict__ Z, int64_t ldz) {
   for (int64_t rr = blockIdx.x; rr < n; rr += gridDim.x)
   for (int k = threadIdx.x; k < K; k += blockDim.x) {
     const int64_t row = r0 + rr;
     const double t = T[row * ldT + k];
-    Z[row * ldz + k] = (g ? g[row] : 1.0) * wo[k] * fma(-t, t, 1.0);
+    const double sv = S ? S[row * ldS + k] : (g ? g[row] : 1.0) * wo[k];
+    Z[row * ldz + k] = sv * fma(-t, t, 1.0);
   }
 }
 
@@ -580,7 +583,7 @@ int fwd(const double *params, const int32_t *widths, int nlayer, int ntypes, con
   clear_error();
   static const char *who = "dp_fitting_fwd_tc_f64";
   FitShape s{};
-  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
+  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s, true);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
   if (nloc == 0) return DP_OK;
@@ -619,17 +622,28 @@ int fwd(const double *params, const int32_t *widths, int nlayer, int ntypes, con
       in = G.V;
       ldin = G.ldv;
     }
-    FitGemm<double> O{};  // output layer: E_i = v_{L-1} . wo + bo
+    FitGemm<double> O{};  // output layer: E_i = v_{L-1} W_out + b_out, on the FP64 pipe
     O.r0 = s.start[t];
     O.n = n;
     O.K = s.w[nlayer - 1];
-    O.N = 1;
     O.src[0] = in;
     O.lds[0] = ldin;
     O.nsrc = 1;
-    O.wo = pt + s.woff[nlayer];
-    fit_out_kernel<double><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(O, O.wo + O.K, E);
-    if ((rc = launch_status(who))) return rc;
+    if (s.nout == 1) {  // a dot product per atom
+      O.N = 1;
+      O.wo = pt + s.woff[nlayer];
+      fit_out_kernel<double><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(O, O.wo + O.K, E);
+      rc = launch_status(who);
+    } else {  // several outputs: a GEMM without tanh
+      O.N = s.nout;
+      O.W = pt + s.woff[nlayer];
+      O.bias = O.W + (size_t)O.K * O.N;
+      O.lin = true;
+      O.out = E;
+      O.ldo = s.nout;
+      rc = launch_gemm<double, true>(O, st, who);
+    }
+    if (rc) return rc;
   }
   return DP_OK;
 }
@@ -639,12 +653,13 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
   clear_error();
   static const char *who = "dp_fitting_grad_tc_f64";
   FitShape s{};
-  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s);
+  int rc = fit_shape(widths, nlayer, ntypes, type_start, &s, true);
   if (rc) return rc;
   const int64_t nloc = s.start[ntypes];
   if (nloc == 0) return DP_OK;
   if (nlayer == 1) return set_error(DP_ERR_UNSUPPORTED, "a fitting net without hidden layers has dD = wo");
   if (!params || !dD || (s.H > 0 && !act)) return set_error(DP_ERR_NULL, "%s: NULL array", who);
+  if (s.nout > 1 && !g) return set_error(DP_ERR_NULL, "%s: g is NULL for a net of %d outputs", who, s.nout);
   if ((rc = check_work(s, nloc, work, work_nbytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
@@ -661,14 +676,32 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
     for (int q = 0; q + 1 < nlayer; ++q)
       if ((rc = split_b(pt + s.woff[nlayer - 1 - q], L[q], false, wk, st, who))) return rc;
     const double *wo = pt + s.woff[nlayer];
+    const double *S = nullptr;  // dE/dv of the layer being walked; NULL: g wo (the last hidden layer)
+    if (s.nout > 1) {  // dE/dv_{nlayer-1} = g W_out^T ([n][nout] x [nout][widths[nlayer-1]], FP64 pipe), into
+                       // Sb[1], which the walk below first writes after its first GEMM has read it
+      FitGemm<double> O{};
+      O.r0 = s.start[t];
+      O.n = n;
+      O.K = s.nout;
+      O.N = s.w[nlayer - 1];
+      O.src[0] = g;
+      O.lds[0] = s.nout;
+      O.nsrc = 1;
+      O.W = wo;  // W_out [widths[nlayer-1]][nout], read transposed
+      O.wt = true;
+      O.lin = true;
+      O.out = Sb[1];
+      O.ldo = s.maxh;
+      if ((rc = launch_gemm<double, true>(O, st, who))) return rc;
+      S = Sb[1];
+    }
     {  // dz of the last hidden layer
       const int K = s.w[nlayer - 1];
-      last_dz_kernel<<<(unsigned)std::min<int64_t>(n, 152 * 32), 256, 0, st>>>(s.start[t], n, K, g, wo,
+      last_dz_kernel<<<(unsigned)std::min<int64_t>(n, 152 * 32), 256, 0, st>>>(s.start[t], n, K, g, wo, S, s.maxh,
                                                                              act + s.aoff[nlayer - 1], s.H, Z[0],
                                                                              s.maxh);
       if ((rc = launch_status(who))) return rc;
     }
-    const double *S = nullptr;  // dE/dv of the layer being walked; NULL: g wo (the last hidden layer)
     int cur = 0;
     for (int l = nlayer - 1; l >= 1; --l) {
       TcGemm G{};
@@ -706,7 +739,7 @@ size_t work_bytes_api(const int32_t *widths, int nlayer, int64_t nloc) {
   if (nloc < 0) return 0;
   const int64_t ts[2] = {0, nloc};
   FitShape s{};
-  if (fit_shape(widths, nlayer, 1, ts, &s)) return 0;
+  if (fit_shape(widths, nlayer, 1, ts, &s, true)) return 0;
   return work_bytes(s, nloc);
 }
 }  // namespace tc

@@ -133,11 +133,10 @@ def test_report_takes_the_roofline_on_the_dominant_tc_kernel():
 
 
 def test_head_options_and_their_fitting_net(monkeypatch):
-    """--head needs the FMA-pipe fitting net of the chain (refused before any device work otherwise),
-    and its net ends in M1 outputs, the head's weights, where the energy model's ends in one."""
+    """--head needs the fitting net of the chain, in f64 or f32 (refused before any device work
+    otherwise), and its net ends in M1 outputs, the head's weights, where the energy model's in one."""
     import pytest
     for argv in (["--head", "vector"], ["--chain", "--head", "tensor"],
-                 ["--chain", "--fitting", "--fitting-tc", "--head", "vector"],
                  ["--chain", "--fitting", "--dtype", "df64", "--head", "vector"]):
         monkeypatch.setattr("sys.argv", ["bench.py", *argv])
         with pytest.raises(SystemExit) as e:

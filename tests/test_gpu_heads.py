@@ -120,17 +120,23 @@ def test_fitting_with_several_outputs(name, dtype, hidden, nout, nat):
     assert rel(dD.double().cpu().numpy(), dDo) <= tol
     with pytest.raises(dpc.DPError):  # several outputs need g
         dpc.dp_fitting_grad(p, widths, ts, act, arith=arith)
-    if name == "f64":  # the tensor-core net has one output
-        with pytest.raises((ValueError, dpc.DPError)):
-            dpc.dp_fitting_fwd_tc_f64(p, widths, ts, _cast(D, dtype))
+    if name == "f64":  # the net with its hidden layers on the tensor cores
+        Et, actt = dpc.dp_fitting_fwd_tc_f64(p, widths, ts, _cast(D, dtype))
+        dDt = dpc.dp_fitting_grad_tc_f64(p, widths, ts, actt, g=_cast(g, dtype))
+        torch.cuda.synchronize()
+        assert rel(Et.cpu().numpy(), Eo) <= tol and rel(dDt.cpu().numpy(), dDo) <= tol
+        with pytest.raises(dpc.DPError):
+            dpc.dp_fitting_grad_tc_f64(p, widths, ts, actt)
 
 
-@pytest.mark.parametrize("head", ["vector", "tensor"])
-def test_vector_and_tensor_models_from_coordinates(head):
+@pytest.mark.parametrize("head,tc_net", [("vector", False), ("tensor", False), ("vector", True)],
+                         ids=["vector", "tensor", "vector-tc-net"])
+def test_vector_and_tensor_models_from_coordinates(head, tc_net):
     """Coordinates -> s, R~ -> T, D (the tensor-core forward, D written by it) -> a = fitting net with
     M1 outputs -> v or A, and back for L = <dE/dv, v> or <dE/dA, A>: the head's dT added to the
     descriptor's (dE/da -> fitting backward -> dD -> dT), the tensor-core backward, forces and virial;
-    every step on the GPU, against the oracle's chain; the folded forces sum to zero."""
+    every step on the GPU, against the oracle's chain; the folded forces sum to zero.  tc_net: the
+    fitting net's hidden layers on the tensor cores."""
     dpc = lib()
     from test_gpu_env_force import _system
     w, coord, nlist, owner, env = _system("water", dict(seed=321, nmol=160), 0, None)
@@ -147,12 +153,14 @@ def test_vector_and_tensor_models_from_coordinates(head):
     s, Rt, nvalid = dpc.dp_env_mat(cg, ng, w.sel, ei)
     T, D = dpc.dp_tabulate_fusion_fwd_tc_f64(plan, info, s, Rt, nvalid, at, w.sel, M2=w.M2)
     fp = torch.from_numpy(fparams).cuda()
-    a, act = dpc.dp_fitting_fwd(fp, widths, ts, D)
+    fit_fwd = dpc.dp_fitting_fwd_tc_f64 if tc_net else dpc.dp_fitting_fwd
+    fit_grad = dpc.dp_fitting_grad_tc_f64 if tc_net else dpc.dp_fitting_grad
+    a, act = fit_fwd(fp, widths, ts, D)
     fwd_head = dpc.dp_vector_head if head == "vector" else dpc.dp_tensor_head
     grad_head = dpc.dp_vector_head_grad if head == "vector" else dpc.dp_tensor_head_grad
     out = fwd_head(T, a)
     dT0, da = grad_head(T, a, torch.from_numpy(dout).cuda())
-    dD = dpc.dp_fitting_grad(fp, widths, ts, act, g=da)
+    dD = fit_grad(fp, widths, ts, act, g=da)
     dT = dpc.dp_descriptor_contract_grad(T, dD.reshape(D.shape))
     dT_desc = dT.clone()
     grad_head(T, a, torch.from_numpy(dout).cuda(), dT=dT, accumulate=True)
