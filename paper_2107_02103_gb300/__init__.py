@@ -477,6 +477,8 @@ def dp_tabulate_fusion_fwd_tc_f64(plan, info: dp_table_info, s, Rt, nvalid, atyp
     shape = (nloc, 4, M1)
     T = torch.empty(shape, dtype=dtype, device=s.device) if out is None else _dev(out, "out", dtype, shape)
     if M2 is not None:
+        if not 1 <= int(M2) <= M1:
+            raise ValueError(f"M2 = {M2} not in 1 .. M1 = {M1}")
         dshape = (nloc, M1, int(M2))
         D = torch.empty(dshape, dtype=dtype, device=s.device) if D is None else _dev(D, "D", dtype, dshape)
     if nloc == 0:

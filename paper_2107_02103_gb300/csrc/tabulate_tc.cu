@@ -10,10 +10,12 @@
 //   W_i[k][(l, q)] = sum_{j in l} R~_j[k] u_j^q,     T_i[k][m] = (1/N_c) sum_{(l, q)} W_i[k][(l, q)] c'_q^{l,m},
 // a GEMM whose K index is (neighbour type, interval, power): the same sum as
 // the per-row evaluation, associated per interval.  The backward is the
-// transposed GEMM,
-//   dW_i[k][(l, q)] = (1/N_c) sum_m dT_i[k][m] c'_q^{l,m},
-//   dE/dR~_j[k] = sum_q dW_i[k][(l, q)] u_j^q,
-//   dE/ds_j     = sum_k R~_j[k] sum_{q >= 1} q dW_i[k][(l, q)] u_j^(q-1) / Delta_l   (0 where s_j was clamped).
+// transposed GEMM, on the unscaled coefficients (its A rows 6 key + q each
+// carry their own exponent, so no scale is needed there), and the rows'
+// polynomials in t itself:
+//   dW_i[k][(l, q)] = (1/N_c) sum_m dT_i[k][m] c_q^{l,m},
+//   dE/dR~_j[k] = sum_q dW_i[k][(l, q)] t_j^q,
+//   dE/ds_j     = sum_k R~_j[k] sum_{q >= 1} q dW_i[k][(l, q)] t_j^(q-1)   (0 where s_j was clamped).
 // The FP64 pipe keeps the per-row work (24 FMAs per row for W, 40 for the
 // derivatives); the per-interval work (24 M1 FMAs per interval and atom in
 // each direction), which is most of it, runs as exact digit-split GEMMs on
@@ -192,8 +194,9 @@ Layout make_layout(const Shape &s) {
 // C'[alpha][6 key + q][m] = c_q Delta_l^q / N_c (key = beta nint + l; rows past the keys: 0).
 // The interval's block of the table is pair-planar [3][M1][2] holding (a, b, c, d, e, f), the
 // coefficients of t^5 .. t^0.
+// kU: the coefficients of u^q, c_q Delta^q (the forward's); else of t^q, c_q (the backward's)
 __global__ void __launch_bounds__(256) coef_kernel(const double *__restrict__ table, TableGeom g, int ntypes, int M1,
-                                                   int Kp, double scale, double *__restrict__ Cp) {
+                                                   int Kp, double scale, bool kU, double *__restrict__ Cp) {
   const int64_t total = (int64_t)ntypes * Kp * M1;
   for (int64_t x = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; x < total; x += (int64_t)gridDim.x * blockDim.x) {
     const int m = (int)(x % M1);
@@ -208,7 +211,8 @@ __global__ void __launch_bounds__(256) coef_kernel(const double *__restrict__ ta
       const double c = blk[(size_t)(j >> 1) * 2 * M1 + 2 * m + (j & 1)];
       const double delta = l < g.n0 ? g.stride0 : g.stride1;
       double p = 1.0;
-      for (int e = 0; e < q; ++e) p *= delta;
+      if (kU)
+        for (int e = 0; e < q; ++e) p *= delta;
       v = c * p * scale;
     }
     Cp[x] = v;
@@ -806,26 +810,24 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_kernel(const RowsParams 
     bool clamped;
     const int l = locate_fast(P.g, P.gf, P.nodes, __ldg(srow + row), t, clamped);
     const Vec4<double> rr = ld4(Rrow + (size_t)row * 4);
-    const double dinv = l < P.g.n0 ? P.g.inv0 : P.g.inv1;
-    const double u = t * dinv;
     const double2 *dw = reinterpret_cast<const double2 *>(dWa + (size_t)smap[b * P.g.nint + l] * 24);
     const double r4[4] = {rr.x, rr.y, rr.z, rr.w};
     double d4[4], ds = 0.0;
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {  // P_k(u) = sum_q dW[k][q] u^q and P_k'(u): 5 + 4 FMA
+    for (int k = 0; k < 4; ++k) {  // P_k(t) = sum_q dW[k][q] t^q and P_k'(t): 5 + 4 FMA
       const double2 c01 = __ldg(dw + 3 * k), c23 = __ldg(dw + 3 * k + 1), c45 = __ldg(dw + 3 * k + 2);
-      double p = fma(c45.y, u, c45.x), dp = c45.y;
-      dp = fma(dp, u, p);
-      p = fma(p, u, c23.y);
-      dp = fma(dp, u, p);
-      p = fma(p, u, c23.x);
-      dp = fma(dp, u, p);
-      p = fma(p, u, c01.y);
-      dp = fma(dp, u, p);
-      d4[k] = fma(p, u, c01.x);
+      double p = fma(c45.y, t, c45.x), dp = c45.y;
+      dp = fma(dp, t, p);
+      p = fma(p, t, c23.y);
+      dp = fma(dp, t, p);
+      p = fma(p, t, c23.x);
+      dp = fma(dp, t, p);
+      p = fma(p, t, c01.y);
+      dp = fma(dp, t, p);
+      d4[k] = fma(p, t, c01.x);
       ds = fma(r4[k], dp, ds);
     }
-    dsrow[row] = clamped ? 0.0 : ds * dinv;
+    dsrow[row] = clamped ? 0.0 : ds;
     st4(drow + (size_t)row * 4, d4[0], d4[1], d4[2], d4[3]);
   }
   // padded rows of each segment
@@ -871,25 +873,23 @@ __global__ void __launch_bounds__(32 * kRowsWarps) rows_force_kernel(const RowsP
     double t;
     bool clamped;
     const int l = locate_fast(P.g, P.gf, P.nodes, ev.r4[0], t, clamped);
-    const double dinv = l < P.g.n0 ? P.g.inv0 : P.g.inv1;
-    const double u = t * dinv;
     const double2 *dw = reinterpret_cast<const double2 *>(dWa + (size_t)smap[b * P.g.nint + l] * 24);
     double d4[4], ds = 0.0;
 #pragma unroll
     for (int k = 0; k < 4; ++k) {  // as rows_kernel
       const double2 c01 = __ldg(dw + 3 * k), c23 = __ldg(dw + 3 * k + 1), c45 = __ldg(dw + 3 * k + 2);
-      double p = fma(c45.y, u, c45.x), dp = c45.y;
-      dp = fma(dp, u, p);
-      p = fma(p, u, c23.y);
-      dp = fma(dp, u, p);
-      p = fma(p, u, c23.x);
-      dp = fma(dp, u, p);
-      p = fma(p, u, c01.y);
-      dp = fma(dp, u, p);
-      d4[k] = fma(p, u, c01.x);
+      double p = fma(c45.y, t, c45.x), dp = c45.y;
+      dp = fma(dp, t, p);
+      p = fma(p, t, c23.y);
+      dp = fma(dp, t, p);
+      p = fma(p, t, c23.x);
+      dp = fma(dp, t, p);
+      p = fma(p, t, c01.y);
+      dp = fma(dp, t, p);
+      d4[k] = fma(p, t, c01.x);
       ds = fma(ev.r4[k], dp, ds);
     }
-    ds = clamped ? 0.0 : ds * dinv;
+    ds = clamped ? 0.0 : ds;
     // as dp_force_virial: the s column feeds both the table input and R~[0]
     const double g0 = ds + d4[0];
     const double p = fma(d4[1], ev.d[0], fma(d4[2], ev.d[1], d4[3] * ev.d[2]));
@@ -978,13 +978,23 @@ int make_plan(const double *table, const dp_table_info *info, int nnei, int ntyp
   if ((rc = launch_status(who))) return rc;
   double *Cp = reinterpret_cast<double *>(wk + P.cp);
   const int64_t total = (int64_t)s.ntypes * s.Kp * s.M1;
-  coef_kernel<<<(unsigned)std::min<int64_t>((total + 255) / 256, 1 << 16), 256, 0, st>>>(table, g, s.ntypes, s.M1, s.Kp,
-                                                                                        1.0 / (double)nnei, Cp);
+  const unsigned cblocks = (unsigned)std::min<int64_t>((total + 255) / 256, 1 << 16);
+  // forward: the u^q coefficients (the moments are in u, all K entries of a column of one scale)
+  coef_kernel<<<cblocks, 256, 0, st>>>(table, g, s.ntypes, s.M1, s.Kp, 1.0 / (double)nnei, true, Cp);
   rc = launch_status(who);
   for (int t = 0; t < s.ntypes && !rc; ++t) {
     const double *Ct = Cp + (size_t)t * s.Kp * s.M1;
     rc = split_rows(Ct, 1, s.M1, s.M1, s.Kp, s.Mpf, s.Kp, kTM, wk + P.afwd + (size_t)t * kS * s.Mpf * s.Kp * 2,
                     wk + P.efwd + (size_t)t * s.Mpf * sizeof(int), st, who);
+  }
+  // backward: the t^q coefficients (each row 6 key + q of A has its own exponent), so that the rows
+  // kernel evaluates its polynomials in t itself, with no 1/Delta on the way in or out
+  if (!rc) {
+    coef_kernel<<<cblocks, 256, 0, st>>>(table, g, s.ntypes, s.M1, s.Kp, 1.0 / (double)nnei, false, Cp);
+    rc = launch_status(who);
+  }
+  for (int t = 0; t < s.ntypes && !rc; ++t) {
+    const double *Ct = Cp + (size_t)t * s.Kp * s.M1;
     unsigned char *eb = wk + P.ebwd + (size_t)t * s.Mpb * sizeof(int);
     if (!rc && s.b8)
       rc = split_rows<Digits7x8>(Ct, s.M1, 1, s.Kp, s.M1, s.Mpb, s.Kpm, kTM,

@@ -284,3 +284,24 @@ def test_tc_water_large_chunk_edges():
     assert dpc.dp_tc_wait_timeouts() == 0
     del T, ds, dRt, dsp, dRtp, x, model, work, plan
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("M2", [1, 7, 32])
+def test_tc_descriptor_widths(M2):
+    """D written by the tensor-core forward at M2 = 1, an odd width and M2 = M1: bit for bit
+    dp_descriptor_contract of the same T, and the oracle's D; M2 = 0 or M2 > M1 refused."""
+    dpc = lib()
+    w = W.water(seed=33, nmol=64, widths=(1, 8, 16, 32), M2=4, sel=(24, 48), rc=5.0)
+    model = product_model(w, F64)
+    x = to_dev(w, F64)
+    args = (model.table, model.info, x["s"], x["Rt"], x["nvalid"], x["atype"], w.sel)
+    T, D = dpc.dp_tabulate_fusion_fwd_tc_f64(*args, M2=M2)
+    Dc = dpc.dp_descriptor_contract(T, M2)
+    torch.cuda.synchronize()
+    assert D.shape == (w.nloc, w.M1, M2)
+    assert torch.equal(D.view(torch.int64), Dc.view(torch.int64))
+    Do = oracle.default().descriptor(T.cpu().numpy(), M2)
+    assert rel(D.cpu().numpy(), Do) <= 1e-14
+    for bad in (0, w.M1 + 1):
+        with pytest.raises(ValueError):
+            dpc.dp_tabulate_fusion_fwd_tc_f64(*args, M2=bad)

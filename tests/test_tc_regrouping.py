@@ -1,11 +1,11 @@
 """The arithmetic of the tensor-core tabulation, restated in numpy on the CPU and held against the
 oracle (Sec. II: T_i = R~_i^T G_i / N_c and its backward): per interval l of an atom's rows, the
 moments W[k][q] = sum_j R~_jk u_j^q with u = t / Delta_l, the scaled coefficients
-c'_q = c_q Delta_l^q, T[k][m] = (1/N_c) sum_(l,q) W[k][q] c'_q[m]; backward
-dW[k][q] = (1/N_c) sum_m dT[k][m] c'_q[m], dE/dR~_jk = sum_q dW[k][q] u_j^q and
-dE/ds_j = sum_k R~_jk sum_q q dW[k][q] u_j^(q-1) / Delta_l (0 for clamped s).  These are the sums
-the GPU GEMMs compute (in exact digit-split form); a dropped power of Delta, a wrong factor q or a
-missing clamp fails here, before any GPU run.  CPU only."""
+c'_q = c_q Delta_l^q, T[k][m] = (1/N_c) sum_(l,q) W[k][q] c'_q[m]; backward on the unscaled
+coefficients, dW[k][q] = (1/N_c) sum_m dT[k][m] c_q[m], dE/dR~_jk = sum_q dW[k][q] t_j^q and
+dE/ds_j = sum_k R~_jk sum_q q dW[k][q] t_j^(q-1) (0 for clamped s).  These are the sums the GPU
+GEMMs compute (in exact digit-split form); a dropped power of Delta, the backward on the forward's
+scaled coefficients, a wrong factor q or a missing clamp fails here, before any GPU run.  CPU only."""
 import numpy as np
 import pytest
 
@@ -15,9 +15,10 @@ import workloads as W
 TOL = 1e-12
 
 
-def regrouped(o, tabs, info, w, dT, scale_delta=True, q_factor=True):
-    """T, ds, dR~ by interval moments and scaled coefficients (rows need not be sorted); the two
-    switches plant a slip (coefficients left unscaled, the derivative without its factor q)."""
+def regrouped(o, tabs, info, w, dT, scale_delta=True, q_factor=True, bwd_scaled=False):
+    """T, ds, dR~ by interval moments and scaled coefficients, the backward in t on the unscaled
+    ones (rows need not be sorted); the switches plant a slip (the forward's coefficients left
+    unscaled, the derivative without its factor q, the backward on the scaled coefficients)."""
     nloc, nnei = w.s.shape
     M1 = tabs.shape[-2]
     off = np.concatenate([[0], np.cumsum(w.sel)])
@@ -31,19 +32,20 @@ def regrouped(o, tabs, info, w, dT, scale_delta=True, q_factor=True):
             for j in range(off[b], off[b] + int(w.nvalid[i, b])):
                 l, t, clamped = o.locate(info, w.s[i, j])
                 delta = info.stride0 if l < info.n0 else info.stride1
-                rows.setdefault((b, l), []).append((j, t / delta, clamped))
+                rows.setdefault((b, l), []).append((j, t, t / delta, clamped))
         for (b, l), rr in rows.items():
             delta = info.stride0 if l < info.n0 else info.stride1
             c = tabs[alpha * w.ntypes + b, l]                          # [M1][6]: t^5 .. t^0
             cp = np.stack([c[:, 5 - q] * (delta ** q if scale_delta else 1.0) for q in range(6)])  # c'_q
+            ct = np.stack([c[:, 5 - q] for q in range(6)])             # c_q
             Wm = np.zeros((4, 6))
-            for j, u, _ in rr:
+            for j, _, u, _ in rr:
                 Wm += np.outer(w.Rt[i, j], u ** np.arange(6))
             T[i] += Wm @ cp / nnei
-            dW = dT[i] @ cp.T / nnei                                   # [4][6]
-            for j, u, clamped in rr:
-                dR[i, j] = dW @ (u ** np.arange(6))
-                dq = dW[:, 1:] @ ((np.arange(1, 6) if q_factor else 1.0) * u ** np.arange(5)) / delta
+            dW = dT[i] @ (cp if bwd_scaled else ct).T / nnei           # [4][6]
+            for j, t, _, clamped in rr:
+                dR[i, j] = dW @ (t ** np.arange(6))
+                dq = dW[:, 1:] @ ((np.arange(1, 6) if q_factor else 1.0) * t ** np.arange(5))
                 ds[i, j] = 0.0 if clamped else float(w.Rt[i, j] @ dq)
     return T, ds, dR
 
@@ -84,7 +86,7 @@ def test_regrouping_matches_oracle_two_types_unsorted_clamped():
     _check(w2)
 
 
-@pytest.mark.parametrize("mistake", ["unscaled_coefficients", "no_q_factor"])
+@pytest.mark.parametrize("mistake", ["unscaled_coefficients", "no_q_factor", "backward_scaled"])
 def test_regrouping_slips_are_caught(mistake):
     """The comparison above notices a plausible slip in the regrouping itself."""
     w = W.tiny(seed=4, nloc=6, nreal=16, sel=16, widths=(1, 4, 8), M2=4)
@@ -93,7 +95,8 @@ def test_regrouping_slips_are_caught(mistake):
     tabs = o.tables(w.params, w.widths, info)
     To = o.fwd(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel)
     dso, _ = o.grad(tabs, info, w.s, w.Rt, w.nvalid, w.atype, w.sel, w.dT)
-    kw = {"scale_delta": False} if mistake == "unscaled_coefficients" else {"q_factor": False}
+    kw = {"unscaled_coefficients": {"scale_delta": False}, "no_q_factor": {"q_factor": False},
+          "backward_scaled": {"bwd_scaled": True}}[mistake]
     T, ds, _ = regrouped(o, tabs, info, w, w.dT, **kw)
     rel = lambda a, b: np.max(np.abs(a - b)) / np.max(np.abs(b))  # noqa: E731
     assert max(rel(T, To), rel(ds, dso)) > 1e-3
