@@ -147,5 +147,6 @@ def test_work_size_query():
     assert all(b % 256 == 0 and b > 0 for b in sizes)
     assert sizes == sorted(sizes)
     assert sizes[-1] >= 4 * 20000 * 240 * 8                 # the buffers between layers
+    assert dpc.dp_fitting_tc_work_bytes([1600, 240, 100], 10) > 0   # several outputs (a head's weights)
     with pytest.raises(ValueError):
-        dpc.dp_fitting_tc_work_bytes([1600, 240, 2], 10)     # the output layer must have width 1
+        dpc.dp_fitting_tc_work_bytes([1600, 240, 0], 10)     # an empty output layer
