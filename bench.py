@@ -194,7 +194,7 @@ def moment_fmas(runs, M1: int) -> dict:
 # `ncu --set full` capture of its current version (the commit the capture was taken at beside each);
 # absent means no capture of the current kernel exists and `traffic` is reported as null.
 PROFILED_DRAM_BYTES = {("cu85", "f64", "grad", "moments"): 83838464 + 32080640,   # commit 7987c32
-                       }  # the tc rows kernel: recaptured after its change to t^q coefficients
+                       ("cu85", "f64", "tc_rows", "tc"): 104717312 + 32222720}    # commit a508952
 
 
 def peak_tflops(dtype: str, mhz: float = SM_MAX_MHZ, nsm: int = NSM) -> float:
