@@ -622,10 +622,10 @@ int dp_fitting_grad_df64(const double *params, const int32_t *widths, int nlayer
  *                     every call), partial results, and the [nloc][max hidden
  *                     width] buffers between layers.  Calls sharing a work
  *                     buffer must not overlap on the GPU.
- * The output layer (a dot product per atom, or with several outputs a GEMM
- * without tanh) and, with several outputs, the backward's g W_out^T run on
- * the FP64 pipe.  Errors as the f64 calls, plus DP_ERR_NULL / DP_ERR_SHAPE
- * for a missing, short or misaligned work buffer.
+ * One output: the output layer is a dot product per atom on the FP64 pipe.
+ * Several outputs: the output layer (without tanh) and the backward's
+ * g W_out^T are GEMMs on the tensor cores too.  Errors as the f64 calls, plus
+ * DP_ERR_NULL / DP_ERR_SHAPE for a missing, short or misaligned work buffer.
  */
 size_t dp_fitting_tc_work_bytes(const int32_t *widths, int nlayer, int64_t nloc); /* 0 on bad widths */
 int dp_fitting_fwd_tc_f64(const double *params, const int32_t *widths, int nlayer, int ntypes,

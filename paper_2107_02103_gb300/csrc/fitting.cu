@@ -422,9 +422,13 @@ __global__ void __launch_bounds__(256) epilogue_kernel(const TcGemm P, int kspli
     for (int z = 0; z < ksplit; ++z) acc.add(P.part[((size_t)z * P.Mp + rc) * P.Np + nn]);
     double v = acc.value(P.Eexp[rc], P.Fexp[nn]);
     if constexpr (kFwd) {
-      const double t = dfl::tanh_d(v + P.bias[nn]);
-      P.act[row * P.ldact + nn] = t;
-      P.V[row * P.ldv + nn] = P.skip ? t + P.A[row * P.lda + nn] : t;
+      if (P.lin) {
+        P.V[row * P.ldv + nn] = v + P.bias[nn];
+      } else {
+        const double t = dfl::tanh_d(v + P.bias[nn]);
+        P.act[row * P.ldact + nn] = t;
+        P.V[row * P.ldv + nn] = P.skip ? t + P.A[row * P.lda + nn] : t;
+      }
     } else {
       if (P.skip) v += P.S ? P.S[row * P.ldS + nn] : (P.g ? P.g[row] : 1.0) * P.wo[nn];
       if (P.T) {
@@ -453,10 +457,17 @@ __global__ void __launch_bounds__(256) last_dz_kernel(int64_t r0, int64_t n, int
   }
 }
 
-// Where the B planes and column exponents of each hidden-layer GEMM of one type sit in the work
-// buffer (forward: layers 1 .. L-1; backward: L-1 .. 1).  After them come the A planes and row
-// exponents of one chunk of at most kChunkRows atoms, and the [nloc][max hidden width] buffers
-// between layers (forward: 2, backward: 4).
+// The GEMMs on the tensor cores: the hidden layers, and with several outputs the output layer too
+// (forward: v W_out + b_out; backward: g W_out^T, first).  GEMM q of a direction works on layer
+// gemm_layer(s, fwd, q): forward 1 .. L-1 (then L), backward (L, then) L-1 .. 1.
+int gemm_count(const FitShape &s) { return s.nlayer - 1 + (s.nout > 1 ? 1 : 0); }
+int gemm_layer(const FitShape &s, bool fwd, int q) {
+  return fwd ? q + 1 : s.nlayer - q - (s.nout > 1 ? 0 : 1);
+}
+
+// Where the B planes and column exponents of each GEMM of one type sit in the work buffer.  After
+// them come the A planes and row exponents of one chunk of at most kChunkRows atoms, and the
+// [nloc][max hidden width] buffers between layers (forward: 2, backward: 4).
 constexpr int64_t kChunkRows = 16384;
 struct Layer {
   int K, N, Np, Kp;
@@ -464,8 +475,8 @@ struct Layer {
 };
 size_t layout(const FitShape &s, bool fwd, Layer *out) {
   size_t off = 0;
-  for (int q = 0; q + 1 < s.nlayer; ++q) {
-    const int l = fwd ? q + 1 : s.nlayer - 1 - q;
+  for (int q = 0; q < gemm_count(s); ++q) {
+    const int l = gemm_layer(s, fwd, q);
     Layer &L = out[q];
     L.K = fwd ? s.w[l - 1] : s.w[l];
     L.N = fwd ? s.w[l] : s.w[l - 1];
@@ -503,11 +514,11 @@ int ksplit_for(int64_t Mp, int Np, int Kp) {
 }
 
 WorkMap work_map(const FitShape &s, int64_t nloc) {
-  Layer L[DP_MAX_LAYERS];
+  Layer L[DP_MAX_LAYERS + 1];
   WorkMap m{};
   m.bplanes = std::max(layout(s, true, L), layout(s, false, L));
   int kmax = 1;
-  for (int l = 0; l < s.nlayer; ++l) kmax = std::max(kmax, s.w[l]);  // every GEMM's K is a layer width
+  for (int l = 0; l <= s.nlayer; ++l) kmax = std::max(kmax, s.w[l]);  // every GEMM's K is a layer width
   m.Kpmax = (int)round_up(kmax, kTK);
   int64_t maxn = 0;  // rows of the largest type
   for (int t = 0; t < s.ntypes; ++t) maxn = std::max<int64_t>(maxn, s.start[t + 1] - s.start[t]);
@@ -518,9 +529,9 @@ WorkMap work_map(const FitShape &s, int64_t nloc) {
   // shares x Mp x Np over the GEMMs: below kTargetCtas tiles plus the largest chunk's Mp x Np, or
   // the exactness bound's shares at the largest chunk (a smaller chunk stays under both)
   int Npmax = kTN;
-  for (int l = 0; l < s.nlayer; ++l) Npmax = std::max(Npmax, (int)round_up(s.w[l], kTN));
+  for (int l = 0; l <= s.nlayer; ++l) Npmax = std::max(Npmax, (int)round_up(s.w[l], kTN));
   int64_t part = kTargetCtas * kTM * kTN + m.Mp * Npmax;
-  for (int q = 0; q + 1 < s.nlayer; ++q)
+  for (int q = 0; q < gemm_count(s); ++q)
     for (int dir = 0; dir < 2; ++dir) {
       layout(s, dir == 0, L);
       part = std::max<int64_t>(part, (int64_t)ksplit_for(m.Mp, L[q].Np, L[q].Kp) * m.Mp * L[q].Np);
@@ -591,7 +602,7 @@ int fwd(const double *params, const int32_t *widths, int nlayer, int ntypes, con
   if ((rc = check_work(s, nloc, work, work_nbytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
-  Layer L[DP_MAX_LAYERS];
+  Layer L[DP_MAX_LAYERS + 1];
   layout(s, true, L);
   const WorkMap m = work_map(s, nloc);
   double *V[2] = {reinterpret_cast<double *>(wk + m.buffers), nullptr};
@@ -600,8 +611,8 @@ int fwd(const double *params, const int32_t *widths, int nlayer, int ntypes, con
     const int64_t n = s.start[t + 1] - s.start[t];
     if (n == 0) continue;
     const double *pt = params + (size_t)t * s.P;
-    for (int l = 1; l < nlayer; ++l)  // this type's weights as digit planes (the previous type's are done with)
-      if ((rc = split_b(pt + s.woff[l], L[l - 1], true, wk, st, who))) return rc;
+    for (int q = 0; q < gemm_count(s); ++q)  // this type's weights as digit planes (the previous type's are done with)
+      if ((rc = split_b(pt + s.woff[gemm_layer(s, true, q)], L[q], true, wk, st, who))) return rc;
     const double *in = D;  // v_{l-1}: D, then the layer outputs with their skips
     int64_t ldin = s.w[0];
     for (int l = 1; l < nlayer; ++l) {
@@ -622,26 +633,31 @@ int fwd(const double *params, const int32_t *widths, int nlayer, int ntypes, con
       in = G.V;
       ldin = G.ldv;
     }
-    FitGemm<double> O{};  // output layer: E_i = v_{L-1} W_out + b_out, on the FP64 pipe
-    O.r0 = s.start[t];
-    O.n = n;
-    O.K = s.w[nlayer - 1];
-    O.src[0] = in;
-    O.lds[0] = ldin;
-    O.nsrc = 1;
-    if (s.nout == 1) {  // a dot product per atom
+    if (s.nout == 1) {  // output layer: E_i = v_{L-1} . wo + bo, a dot product per atom (FP64 pipe)
+      FitGemm<double> O{};
+      O.r0 = s.start[t];
+      O.n = n;
+      O.K = s.w[nlayer - 1];
       O.N = 1;
+      O.src[0] = in;
+      O.lds[0] = ldin;
+      O.nsrc = 1;
       O.wo = pt + s.woff[nlayer];
       fit_out_kernel<double><<<(unsigned)((n + 3) / 4), 128, 0, st>>>(O, O.wo + O.K, E);
       rc = launch_status(who);
-    } else {  // several outputs: a GEMM without tanh
-      O.N = s.nout;
-      O.W = pt + s.woff[nlayer];
-      O.bias = O.W + (size_t)O.K * O.N;
-      O.lin = true;
-      O.out = E;
-      O.ldo = s.nout;
-      rc = launch_gemm<double, true>(O, st, who);
+    } else {  // several outputs: E_i = v_{L-1} W_out + b_out, a GEMM on the tensor cores without tanh
+      TcGemm G{};
+      G.r0 = s.start[t];
+      G.n = n;
+      G.K = s.w[nlayer - 1];
+      G.N = s.nout;
+      G.A = in;
+      G.lda = ldin;
+      G.lin = true;
+      G.bias = pt + s.woff[nlayer] + (size_t)G.K * G.N;
+      G.V = E;
+      G.ldv = s.nout;
+      rc = gemm<true>(G, L[nlayer - 1], wk, m, st, who);
     }
     if (rc) return rc;
   }
@@ -663,7 +679,7 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
   if ((rc = check_work(s, nloc, work, work_nbytes, who)) || (rc = set_smem(who))) return rc;
   const cudaStream_t st = (cudaStream_t)stream;
   unsigned char *wk = static_cast<unsigned char *>(work);
-  Layer L[DP_MAX_LAYERS];
+  Layer L[DP_MAX_LAYERS + 1];
   layout(s, false, L);
   const WorkMap m = work_map(s, nloc);
   double *buf = reinterpret_cast<double *>(wk + m.buffers);
@@ -673,26 +689,23 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
     const int64_t n = s.start[t + 1] - s.start[t];
     if (n == 0) continue;
     const double *pt = params + (size_t)t * s.P;
-    for (int q = 0; q + 1 < nlayer; ++q)
-      if ((rc = split_b(pt + s.woff[nlayer - 1 - q], L[q], false, wk, st, who))) return rc;
+    for (int q = 0; q < gemm_count(s); ++q)
+      if ((rc = split_b(pt + s.woff[gemm_layer(s, false, q)], L[q], false, wk, st, who))) return rc;
     const double *wo = pt + s.woff[nlayer];
     const double *S = nullptr;  // dE/dv of the layer being walked; NULL: g wo (the last hidden layer)
-    if (s.nout > 1) {  // dE/dv_{nlayer-1} = g W_out^T ([n][nout] x [nout][widths[nlayer-1]], FP64 pipe), into
-                       // Sb[1], which the walk below first writes after its first GEMM has read it
-      FitGemm<double> O{};
-      O.r0 = s.start[t];
-      O.n = n;
-      O.K = s.nout;
-      O.N = s.w[nlayer - 1];
-      O.src[0] = g;
-      O.lds[0] = s.nout;
-      O.nsrc = 1;
-      O.W = wo;  // W_out [widths[nlayer-1]][nout], read transposed
-      O.wt = true;
-      O.lin = true;
-      O.out = Sb[1];
-      O.ldo = s.maxh;
-      if ((rc = launch_gemm<double, true>(O, st, who))) return rc;
+    const int q0 = s.nout > 1 ? 1 : 0;  // the hidden layers' GEMMs come after g W_out^T
+    if (s.nout > 1) {  // dE/dv_{nlayer-1} = g W_out^T ([n][nout] x [nout][widths[nlayer-1]], tensor cores),
+                       // into Sb[1], which the walk below first writes after its first GEMM has read it
+      TcGemm G{};
+      G.r0 = s.start[t];
+      G.n = n;
+      G.K = s.nout;
+      G.N = s.w[nlayer - 1];
+      G.A = g;
+      G.lda = s.nout;
+      G.out = Sb[1];
+      G.ldo = s.maxh;
+      if ((rc = gemm<false>(G, L[0], wk, m, st, who))) return rc;
       S = Sb[1];
     }
     {  // dz of the last hidden layer
@@ -726,7 +739,7 @@ int grad(const double *params, const int32_t *widths, int nlayer, int ntypes, co
         G.out = dD;
         G.ldo = s.w[0];
       }
-      if ((rc = gemm<false>(G, L[nlayer - 1 - l], wk, m, st, who))) return rc;
+      if ((rc = gemm<false>(G, L[q0 + nlayer - 1 - l], wk, m, st, who))) return rc;
       S = G.Snext;
       cur ^= 1;
     }

@@ -279,6 +279,7 @@ struct TcGemm {
   int ldt;
   bool skip;
   // forward
+  bool lin;  // an output layer of several outputs: V[row][col] = acc + bias, no tanh, act unused
   const double *bias;
   double *act;
   int64_t ldact;
