@@ -190,3 +190,23 @@ def test_vector_and_tensor_models_from_coordinates(head, tc_net):
     folded = np.zeros((w.nloc, 3))
     np.add.at(folded, owner, F.cpu().numpy())
     assert np.abs(folded.sum(axis=0)).max() <= 1e-9 * np.abs(folded).max()
+
+
+def test_fitting_noalloc_with_several_outputs():
+    """dp_fitting_grad_noalloc_f64 on a net of several outputs (its scratch from the library's fixed
+    array) gives the bits of dp_fitting_grad_f64 with a work buffer; without g it is refused."""
+    dpc = lib()
+    widths = [40, 32, 32, 12]
+    params = W.net_params(331, widths, 2)
+    ts = np.array([0, 30, 75], dtype=np.int64)
+    D = W.normal(332, (75, 40))
+    g = W.normal(333, (75, 12))
+    p = torch.from_numpy(params).cuda()
+    E, act = dpc.dp_fitting_fwd(p, widths, ts, torch.from_numpy(D).cuda())
+    gd = torch.from_numpy(g).cuda()
+    a = dpc.dp_fitting_grad(p, widths, ts, act, g=gd)
+    b = dpc.dp_fitting_grad_noalloc_f64(p, widths, ts, act, g=gd)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+    with pytest.raises(dpc.DPError):
+        dpc.dp_fitting_grad_noalloc_f64(p, widths, ts, act)
